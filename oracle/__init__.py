@@ -1,0 +1,201 @@
+"""CPU oracle for the VestigeKV decode hot path (plain C, fp64).
+
+TEST INFRASTRUCTURE ONLY: the test suite, ``__graft_entry__.smoke()`` and the CPU-baseline leg of
+``bench.py`` are the only callers. The product (the CUDA library and its binding) never imports this
+package. The C source is ``vk_oracle.c``; ``build()`` compiles it with gcc.
+
+Every function takes a :class:`paper_2609_03949_gb300.datagen.Workload`-like set of host arrays, passes
+their raw storage (bf16 bits or fp32) to C, and returns numpy arrays in fp64.
+"""
+from __future__ import annotations
+
+import ctypes
+import math
+import os
+import subprocess
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_SRC = os.path.join(_HERE, "vk_oracle.c")
+_LIB_PATH = os.path.join(_HERE, "libvk_oracle.so")
+_lib = None
+
+D_LATENT, D_ROPE, PAGE = 512, 64, 64
+
+# Deliberate mistakes the "known-bad first" tests plant in the oracle (see vk_oracle.c).
+MUT_NONE, MUT_TIE_LARGER, MUT_DROP_WINDOW, MUT_SCALE_SQUARED = 0, 1, 2, 3
+MUT_ROT_TRANSPOSE, MUT_DROP_ROPE, MUT_TRIGGER_NO_Z = 4, 5, 6
+
+
+def build(force: bool = False) -> str:
+    """Compile vk_oracle.c into libvk_oracle.so (gcc, -O2, OpenMP over (batch, head))."""
+    if force or not os.path.exists(_LIB_PATH) or os.path.getmtime(_LIB_PATH) < os.path.getmtime(_SRC):
+        tmp = _LIB_PATH + f".tmp{os.getpid()}"
+        subprocess.run(["gcc", "-O2", "-fopenmp", "-fPIC", "-shared", "-std=c11", "-o", tmp, _SRC, "-lm"],
+                       check=True)
+        os.replace(tmp, _LIB_PATH)
+    return _LIB_PATH
+
+
+class _View(ctypes.Structure):
+    _fields_ = [("B", ctypes.c_int32), ("H", ctypes.c_int32), ("N", ctypes.c_int32), ("dtype", ctypes.c_int32),
+                ("latent", ctypes.c_void_p), ("latent_ld", ctypes.c_int64), ("latent_bstride", ctypes.c_int64),
+                ("rope", ctypes.c_void_p), ("rope_ld", ctypes.c_int64), ("rope_bstride", ctypes.c_int64),
+                ("q_latent", ctypes.c_void_p), ("q_rope", ctypes.c_void_p)]
+
+
+def lib():
+    global _lib
+    if _lib is None:
+        build()
+        L = ctypes.CDLL(_LIB_PATH)
+        P, I32, I64, D, F = ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64, ctypes.c_double, ctypes.c_float
+        VP = ctypes.POINTER(_View)
+        L.vko_keep_count.argtypes = [I32, D, I32, I32]
+        L.vko_keep_count.restype = I64
+        L.vko_bf16_rne.argtypes = [D]
+        L.vko_bf16_rne.restype = ctypes.c_uint16
+        L.vko_build_index.argtypes = [VP, I32, P, P, P, P, P]
+        L.vko_scores.argtypes = [VP, I32, P, P, P]
+        L.vko_select.argtypes = [I32, I32, I32, P, I64, I32, I32, I32, P, P, P]
+        L.vko_attention.argtypes = [VP, D, P, P, I32, P, P, P]
+        L.vko_trigger.argtypes = [VP, I32, P, D, D, I32, P, P, P, P, P, I32, P, I32, I32, I32, P, P]
+        L.vko_decode_step.argtypes = [VP, D, I32, I32, I32, D, I32, D, I32, P, P, I32, P, P, P, P, P, P]
+        L.vko_decode_step.restype = ctypes.c_int
+        L.vko_set_mutation.argtypes = [ctypes.c_int]
+        L.vko_num_threads.restype = ctypes.c_int
+        del F
+        _lib = L
+    return _lib
+
+
+def _ptr(a: np.ndarray) -> int:
+    return a.ctypes.data if a is not None else 0
+
+
+class HostInputs:
+    """Host copies of one workload in its storage format, kept alive while C reads them."""
+
+    def __init__(self, wl):
+        import torch
+        self.B, self.H, self.N, self.dtype = wl.B, wl.H, wl.N, wl.dtype
+        if wl.dtype == "bf16":
+            conv = lambda t: t.detach().cpu().contiguous().view(torch.int16).numpy().view(np.uint16)
+        else:
+            conv = lambda t: t.detach().cpu().contiguous().float().numpy()
+        self.cache = conv(wl.cache)
+        self.q_latent = conv(wl.q_latent)
+        self.q_rope = conv(wl.q_rope)
+        self.rot = wl.rot.detach().cpu().contiguous().float().numpy()
+        esz = self.cache.itemsize
+        row = self.cache.shape[-1]
+        self.view = _View(B=self.B, H=self.H, N=self.N, dtype=0 if self.dtype == "bf16" else 1,
+                          latent=self.cache.ctypes.data, latent_ld=row, latent_bstride=self.N * row,
+                          rope=self.cache.ctypes.data + D_LATENT * esz, rope_ld=row, rope_bstride=self.N * row,
+                          q_latent=self.q_latent.ctypes.data, q_rope=self.q_rope.ctypes.data)
+
+
+def set_mutation(m: int) -> None:
+    lib().vko_set_mutation(int(m))
+
+
+def num_threads() -> int:
+    return int(lib().vko_num_threads())
+
+
+def keep_count(N: int, rho: float, window: int, n_sink: int = 0) -> int:
+    """k = min(ceil(rho*N), |A|), A = [n_sink, N-W)."""
+    return int(lib().vko_keep_count(N, rho, window, n_sink))
+
+
+def bf16_rne(x: float) -> int:
+    return int(lib().vko_bf16_rne(float(x)))
+
+
+def build_index(hi: HostInputs, r: int):
+    """(digest fp64 [B,N,r] or None, digest bf16 bits [B,N,r] or None, eta [B,N], page_res [B,P])."""
+    B, N = hi.B, hi.N
+    P = (N + PAGE - 1) // PAGE
+    dig = np.zeros((B, N, r), np.float64) if r < D_ROPE else None
+    dig16 = np.zeros((B, N, r), np.uint16) if r < D_ROPE else None
+    eta = np.zeros((B, N), np.float64)
+    pres = np.zeros((B, P), np.float64)
+    lib().vko_build_index(ctypes.byref(hi.view), r, _ptr(hi.rot), _ptr(dig), _ptr(dig16), _ptr(eta), _ptr(pres))
+    return dig, dig16, eta, pres
+
+
+def scores(hi: HostInputs, r: int = 64, digest_bf16: np.ndarray | None = None) -> np.ndarray:
+    """a[b,h,u] (unscaled RoPE-branch or digest score), fp64 [B,H,N]."""
+    a = np.zeros((hi.B, hi.H, hi.N), np.float64)
+    dg = None if digest_bf16 is None else np.ascontiguousarray(digest_bf16, dtype=np.uint16)
+    if r < D_ROPE and dg is None:
+        raise ValueError("a width-r digest needs the stored bf16 digest")
+    lib().vko_scores(ctypes.byref(hi.view), r, _ptr(hi.rot), _ptr(dg), _ptr(a))
+    return a
+
+
+def select(a: np.ndarray, k: int, window: int, n_sink: int = 0, cap: int | None = None):
+    """(idx [B,H,cap] int32, count [B,H] int32, kth [B,H] fp64) — per-head top-k + window (+ sinks)."""
+    a = np.ascontiguousarray(a, dtype=np.float64)
+    B, H, N = a.shape
+    cap = cap if cap is not None else max(1, k + window + n_sink)
+    idx = np.full((B, H, cap), -1, np.int32)
+    count = np.zeros((B, H), np.int32)
+    kth = np.zeros((B, H), np.float64)
+    lib().vko_select(B, H, N, _ptr(a), k, window, n_sink, cap, _ptr(idx), _ptr(count), _ptr(kth))
+    return idx, count, kth
+
+
+def attention(hi: HostInputs, lam: float, idx: np.ndarray, count: np.ndarray):
+    """(out [B,H,512], lse [B,H], smax [B,H]) over the attended sets idx[b,h,:count]."""
+    idx = np.ascontiguousarray(idx, dtype=np.int32)
+    count = np.ascontiguousarray(count, dtype=np.int32)
+    cap = idx.shape[-1]
+    out = np.zeros((hi.B, hi.H, D_LATENT), np.float64)
+    lse = np.zeros((hi.B, hi.H), np.float64)
+    smax = np.zeros((hi.B, hi.H), np.float64)
+    lib().vko_attention(ctypes.byref(hi.view), float(lam), _ptr(idx), _ptr(count), cap, _ptr(out), _ptr(lse),
+                        _ptr(smax))
+    return out, lse, smax
+
+
+def trigger(hi: HostInputs, r: int, lam: float, z_eff: float, top_j: int, a: np.ndarray, eta: np.ndarray,
+            page_res: np.ndarray, idx: np.ndarray, count: np.ndarray, smax: np.ndarray, window: int,
+            n_sink: int = 0):
+    """(fired idx [B,H,N] int32, fired count [B,H]) of the row-level Cauchy-Schwarz trigger."""
+    a = np.ascontiguousarray(a, dtype=np.float64)
+    idx = np.ascontiguousarray(idx, dtype=np.int32)
+    count = np.ascontiguousarray(count, dtype=np.int32)
+    smax = np.ascontiguousarray(smax, dtype=np.float64)
+    eta = np.ascontiguousarray(eta, dtype=np.float64)
+    page_res = np.ascontiguousarray(page_res, dtype=np.float64)
+    capf = hi.N
+    fidx = np.full((hi.B, hi.H, capf), -1, np.int32)
+    fcount = np.zeros((hi.B, hi.H), np.int32)
+    lib().vko_trigger(ctypes.byref(hi.view), r, _ptr(hi.rot), float(lam), float(z_eff), int(top_j), _ptr(a),
+                      _ptr(eta), _ptr(page_res), _ptr(idx), _ptr(count), idx.shape[-1], _ptr(smax), window,
+                      n_sink, capf, _ptr(fidx), _ptr(fcount))
+    return fidx, fcount
+
+
+def decode_step(hi: HostInputs, *, rho: float, r: int = 64, window: int = 0, n_sink: int = 0,
+                sm_scale: float | None = None, trigger: int = 0, z_eff: float = 1.0, top_j: int = 0,
+                digest_bf16: np.ndarray | None = None, cap: int | None = None):
+    """Whole step. Returns dict(out, lse, smax, idx, count, kth, rc)."""
+    lam = (1.0 / math.sqrt(192.0)) if sm_scale is None else float(sm_scale)
+    if cap is None:
+        cap = hi.N if trigger else max(1, keep_count(hi.N, rho, window, n_sink) + window + n_sink)
+    out = np.zeros((hi.B, hi.H, D_LATENT), np.float64)
+    lse = np.zeros((hi.B, hi.H), np.float64)
+    smax = np.zeros((hi.B, hi.H), np.float64)
+    kth = np.zeros((hi.B, hi.H), np.float64)
+    idx = np.full((hi.B, hi.H, cap), -1, np.int32)
+    count = np.zeros((hi.B, hi.H), np.int32)
+    dg = None if digest_bf16 is None else np.ascontiguousarray(digest_bf16, dtype=np.uint16)
+    if r < D_ROPE and dg is None:
+        raise ValueError("a width-r digest needs the stored bf16 digest")
+    rc = lib().vko_decode_step(ctypes.byref(hi.view), float(rho), r, window, n_sink, lam, int(trigger),
+                               float(z_eff), int(top_j), _ptr(hi.rot), _ptr(dg), cap, _ptr(out), _ptr(lse),
+                               _ptr(smax), _ptr(idx), _ptr(count), _ptr(kth))
+    return dict(out=out, lse=lse, smax=smax, idx=idx, count=count, kth=kth, rc=int(rc))

@@ -1,0 +1,375 @@
+/*
+ * vk_oracle.c -- plain, slow, fp64 CPU restatement of the VestigeKV decode hot path.
+ *
+ * TEST INFRASTRUCTURE ONLY. The test suite, the smoke check and the benchmark's CPU-baseline leg are the
+ * only code that may load this library. The CUDA library never calls it, and the two share no code,
+ * headers, tables or helpers.
+ *
+ * Source: "VestigeKV: The NoPE-MLA KV Cache Carries Its Own Sparse-Attention Signal in a Vestigial
+ * Branch" (arXiv 2609.03949). Every stored input (bf16 or fp32) is decoded exactly to double and all
+ * arithmetic is double. Nothing is blocked, fused or reordered beyond what each definition states.
+ *
+ * Pinned by tests/test_oracle_pins.py (closed forms, hand cases with a known answer, library routines on
+ * special cases, brute force on tiny inputs, the paper's lemmas as invariants). No function here is
+ * "parity unpinned".
+ *
+ * Readings of the paper used here (each listed with its reason in the design notes):
+ *   - the cache holds rows 0..N-1; the query sits at position N; the recent window is [N-W, N);
+ *   - the archive is A = [n_sink, N-W); k = min(ceil(rho*N), |A|) rows are kept from it per head;
+ *   - ties in the top-k go to the smaller position;
+ *   - the trigger is row level: Eq. 5 with sketch rank 0 (the content summand is bounded by
+ *     Cauchy-Schwarz with eta_u = |L_u|), plus a page-level bound on the RoPE dims that the width-r
+ *     digest does not cover.
+ */
+#include <math.h>
+#include <stdint.h>
+#include <stdlib.h>
+#include <string.h>
+#ifdef _OPENMP
+#include <omp.h>
+#endif
+
+#define D_LAT 512
+#define D_ROPE 64
+#define PAGE 64
+
+/* Deliberate mistakes for the "known-bad input first" checks: a test sets one, shows that a pin fails,
+ * and clears it. 0 = the oracle as written. */
+enum {
+  MUT_NONE = 0,
+  MUT_TIE_LARGER = 1,     /* ties go to the larger position */
+  MUT_DROP_WINDOW = 2,    /* the recent window is not attended */
+  MUT_SCALE_SQUARED = 3,  /* logits use lambda^2 */
+  MUT_ROT_TRANSPOSE = 4,  /* the digest rotation is applied as O^T */
+  MUT_DROP_ROPE = 5,      /* attention logits drop the RoPE summand */
+  MUT_TRIGGER_NO_Z = 6,   /* trigger ignores the certificate term */
+};
+static int g_mutation = MUT_NONE;
+void vko_set_mutation(int m) { g_mutation = m; }
+
+typedef struct {
+  int32_t B, H, N;
+  int32_t dtype;                              /* 0 = bf16 storage, 1 = fp32 storage */
+  const void* latent; int64_t latent_ld, latent_bstride;   /* elements */
+  const void* rope;   int64_t rope_ld, rope_bstride;       /* elements */
+  const void* q_latent;                       /* [B,H,512] contiguous */
+  const void* q_rope;                         /* [B,H,64] contiguous */
+} vko_view;
+
+/* ---------------------------------------------------------------- exact decoding of the stored values */
+static double from_bf16(uint16_t h) {
+  uint32_t bits = (uint32_t)h << 16;
+  float f;
+  memcpy(&f, &bits, 4);
+  return (double)f;
+}
+static double load(const void* base, int dtype, int64_t i) {
+  if (dtype == 1) return (double)((const float*)base)[i];
+  return from_bf16(((const uint16_t*)base)[i]);
+}
+static double L(const vko_view* v, int b, int64_t u, int j) {
+  return load(v->latent, v->dtype, (int64_t)b * v->latent_bstride + u * v->latent_ld + j);
+}
+static double K(const vko_view* v, int b, int64_t u, int j) {
+  return load(v->rope, v->dtype, (int64_t)b * v->rope_bstride + u * v->rope_ld + j);
+}
+static double QC(const vko_view* v, int b, int h, int j) {
+  return load(v->q_latent, v->dtype, ((int64_t)b * v->H + h) * D_LAT + j);
+}
+static double QR(const vko_view* v, int b, int h, int j) {
+  return load(v->q_rope, v->dtype, ((int64_t)b * v->H + h) * D_ROPE + j);
+}
+
+/* bf16 round-to-nearest-even of a double, straight from the double (no detour through float). */
+uint16_t vko_bf16_rne(double x) {
+  if (x == 0.0 || !isfinite(x)) {
+    float f = (float)x;
+    uint32_t b;
+    memcpy(&b, &f, 4);
+    return (uint16_t)(b >> 16);
+  }
+  int e;
+  double m = frexp(x, &e);              /* x = m * 2^e, 0.5 <= |m| < 1 */
+  double scaled = ldexp(m, 8);          /* 8 significant bits -> an integer in [128, 256) */
+  double fl = floor(scaled), diff = scaled - fl, q;
+  if (diff > 0.5) q = fl + 1.0;
+  else if (diff < 0.5) q = fl;
+  else q = (fmod(fl, 2.0) == 0.0) ? fl : fl + 1.0;
+  float f = (float)ldexp(q, e - 8);     /* exact: 8 significant bits fit a float */
+  uint32_t b;
+  memcpy(&b, &f, 4);
+  return (uint16_t)(b >> 16);
+}
+
+/* ---------------------------------------------------------------- set sizes (Sec. 4.1, spec rho) */
+/* Archive A = [n_sink, N-W); keep k = min(ceil(rho*N), |A|) archived rows per head. */
+int64_t vko_keep_count(int32_t N, double rho, int32_t W, int32_t n_sink) {
+  int64_t A = (int64_t)N - W - n_sink;
+  if (A < 0) A = 0;
+  int64_t k = (int64_t)ceil(rho * (double)N);
+  return k < A ? k : A;
+}
+
+/* ---------------------------------------------------------------- rotated query (digest scoring) */
+/* qt = O * qr (row-major O; the digest keeps its first r coordinates). */
+static void rotate64(const float* rot, const double* x, double* y) {
+  for (int j = 0; j < D_ROPE; ++j) {
+    double acc = 0.0;
+    for (int i = 0; i < D_ROPE; ++i) {
+      double o = (g_mutation == MUT_ROT_TRANSPOSE) ? (double)rot[i * D_ROPE + j] : (double)rot[j * D_ROPE + i];
+      acc += o * x[i];
+    }
+    y[j] = acc;
+  }
+}
+
+/* ---------------------------------------------------------------- index build (Sec. 4.2 index entry) */
+/* For every row: digest = (O K_u)[0:r] (before rounding; r < 64 only), its bf16 RNE rounding,
+ * eta_u = |L_u|_2 (the certificate's row norm with sketch rank 0), and per 64-row page the largest
+ * norm of the uncovered RoPE coordinates (O K_u)[r:64] (0 when r = 64). */
+void vko_build_index(const vko_view* v, int32_t r, const float* rot, double* digest, uint16_t* digest_bf16,
+                     double* eta, double* page_res) {
+  const int64_t N = v->N, P = (N + PAGE - 1) / PAGE;
+#pragma omp parallel for schedule(static)
+  for (int b = 0; b < v->B; ++b) {
+    for (int64_t p = 0; p < P; ++p) page_res[(int64_t)b * P + p] = 0.0;
+    for (int64_t u = 0; u < N; ++u) {
+      double ss = 0.0;
+      for (int j = 0; j < D_LAT; ++j) ss += L(v, b, u, j) * L(v, b, u, j);
+      eta[(int64_t)b * N + u] = sqrt(ss);
+      if (r < D_ROPE) {
+        double k[D_ROPE], y[D_ROPE];
+        for (int j = 0; j < D_ROPE; ++j) k[j] = K(v, b, u, j);
+        rotate64(rot, k, y);
+        for (int j = 0; j < r; ++j) {
+          digest[((int64_t)b * N + u) * r + j] = y[j];
+          if (digest_bf16) digest_bf16[((int64_t)b * N + u) * r + j] = vko_bf16_rne(y[j]);
+        }
+        double res = 0.0;
+        for (int j = r; j < D_ROPE; ++j) res += y[j] * y[j];
+        res = sqrt(res);
+        double* pr = &page_res[(int64_t)b * P + u / PAGE];
+        if (res > *pr) *pr = res;
+      }
+    }
+  }
+}
+
+/* ---------------------------------------------------------------- scores (Eq. 5, exact summand) */
+/* a[b,h,u] = qr_h . K_u over the 64 RoPE columns (r = 64), or, for a width-r digest,
+ * a = (O qr_h)[0:r] . digest_u with the stored bf16 digest. The attention scale is applied later. */
+void vko_scores(const vko_view* v, int32_t r, const float* rot, const uint16_t* digest, double* a) {
+  const int64_t N = v->N;
+#pragma omp parallel for collapse(2) schedule(static)
+  for (int b = 0; b < v->B; ++b) {
+    for (int h = 0; h < v->H; ++h) {
+      double q[D_ROPE], qt[D_ROPE];
+      for (int j = 0; j < D_ROPE; ++j) q[j] = QR(v, b, h, j);
+      if (r < D_ROPE) rotate64(rot, q, qt);
+      double* out = &a[((int64_t)b * v->H + h) * N];
+      for (int64_t u = 0; u < N; ++u) {
+        double acc = 0.0;
+        if (r == D_ROPE) {
+          for (int j = 0; j < D_ROPE; ++j) acc += q[j] * K(v, b, u, j);
+        } else {
+          for (int j = 0; j < r; ++j) acc += qt[j] * from_bf16(digest[((int64_t)b * N + u) * r + j]);
+        }
+        out[u] = acc;
+      }
+    }
+  }
+}
+
+/* ---------------------------------------------------------------- selection (Sec. 4.1) */
+typedef struct { double key; int32_t u; } item;
+
+static int by_key_desc_pos_asc(const void* x, const void* y) {
+  const item* a = (const item*)x;
+  const item* b = (const item*)y;
+  if (a->key > b->key) return -1;
+  if (a->key < b->key) return 1;
+  if (g_mutation == MUT_TIE_LARGER) return (a->u > b->u) ? -1 : (a->u < b->u);
+  return (a->u < b->u) ? -1 : (a->u > b->u);
+}
+
+/* Per (b,h): sort the archive by (score desc, position asc), keep the first k; the attended set is that
+ * together with the sinks [0, n_sink) and the recent window [N-W, N), listed in ascending position.
+ * kth = the k-th largest archive score (+inf when k = 0). count = k + W + n_sink. */
+void vko_select(int32_t B, int32_t H, int32_t N, const double* a, int64_t k, int32_t W, int32_t n_sink,
+                int32_t cap, int32_t* idx, int32_t* count, double* kth) {
+#pragma omp parallel for collapse(2) schedule(dynamic)
+  for (int b = 0; b < B; ++b) {
+    for (int h = 0; h < H; ++h) {
+      const double* s = &a[((int64_t)b * H + h) * N];
+      int64_t lo = n_sink, hi = (int64_t)N - W;
+      int64_t na = hi > lo ? hi - lo : 0;
+      item* it = (item*)malloc(sizeof(item) * (size_t)(na > 0 ? na : 1));
+      for (int64_t i = 0; i < na; ++i) { it[i].key = s[lo + i]; it[i].u = (int32_t)(lo + i); }
+      qsort(it, (size_t)na, sizeof(item), by_key_desc_pos_asc);
+      char* mark = (char*)calloc((size_t)N + 1, 1);
+      for (int64_t i = 0; i < k && i < na; ++i) mark[it[i].u] = 1;
+      for (int64_t u = 0; u < n_sink && u < N; ++u) mark[u] = 1;
+      if (g_mutation != MUT_DROP_WINDOW)
+        for (int64_t u = hi > 0 ? hi : 0; u < N; ++u) mark[u] = 1;
+      int32_t c = 0;
+      int32_t* out = &idx[((int64_t)b * H + h) * cap];
+      for (int64_t u = 0; u < N; ++u)
+        if (mark[u]) { if (c < cap) out[c] = (int32_t)u; ++c; }
+      count[b * H + h] = c;
+      kth[b * H + h] = (k > 0 && na > 0) ? it[(k < na ? k : na) - 1].key : INFINITY;
+      free(mark);
+      free(it);
+    }
+  }
+}
+
+/* ---------------------------------------------------------------- attention (Eq. 1, Lemma 1) */
+/* Absorbed MLA over an attended set: s_u = lambda*(qc_h . L_u + qr_h . K_u); softmax over the set;
+ * the output is the 512-wide latent combination sum_u p_u L_u (the value up-projection W_UV is applied
+ * outside the cache read). lse = max + log(sum exp(s - max)); smax = the max logit s*.
+ * An empty set gives out = 0, lse = smax = -inf. */
+static double logit(const vko_view* v, int b, int h, int64_t u, double lam) {
+  double acc = 0.0;
+  for (int j = 0; j < D_LAT; ++j) acc += QC(v, b, h, j) * L(v, b, u, j);
+  if (g_mutation != MUT_DROP_ROPE)
+    for (int j = 0; j < D_ROPE; ++j) acc += QR(v, b, h, j) * K(v, b, u, j);
+  return (g_mutation == MUT_SCALE_SQUARED ? lam * lam : lam) * acc;
+}
+
+void vko_attention(const vko_view* v, double lam, const int32_t* idx, const int32_t* count, int32_t cap,
+                   double* out, double* lse, double* smax) {
+#pragma omp parallel for collapse(2) schedule(dynamic)
+  for (int b = 0; b < v->B; ++b) {
+    for (int h = 0; h < v->H; ++h) {
+      const int32_t* set = &idx[((int64_t)b * v->H + h) * cap];
+      int32_t n = count[b * v->H + h];
+      if (n > cap) n = cap;
+      double* o = &out[((int64_t)b * v->H + h) * D_LAT];
+      for (int j = 0; j < D_LAT; ++j) o[j] = 0.0;
+      if (n <= 0) { lse[b * v->H + h] = -INFINITY; smax[b * v->H + h] = -INFINITY; continue; }
+      double* s = (double*)malloc(sizeof(double) * (size_t)n);
+      double m = -INFINITY;
+      for (int32_t i = 0; i < n; ++i) { s[i] = logit(v, b, h, set[i], lam); if (s[i] > m) m = s[i]; }
+      double z = 0.0;
+      for (int32_t i = 0; i < n; ++i) z += exp(s[i] - m);
+      for (int32_t i = 0; i < n; ++i) {
+        double p = exp(s[i] - m) / z;
+        for (int j = 0; j < D_LAT; ++j) o[j] += p * L(v, b, set[i], j);
+      }
+      lse[b * v->H + h] = m + log(z);
+      smax[b * v->H + h] = m;
+      free(s);
+    }
+  }
+}
+
+/* ---------------------------------------------------------------- recall trigger (Eq. 5, Lemma 2) */
+/* With sketch rank 0 the content summand is bounded by Cauchy-Schwarz: |qc_h . L_u| <= |qc_h| eta_u.
+ * For a width-r digest the RoPE dims it leaves out are bounded the same way, page by page:
+ * |(O qr_h)[r:] . (O K_u)[r:]| <= |(O qr_h)[r:]| page_res[u/64]. The trigger score of an archived row
+ * not already attended is
+ *     T = lambda * (a[h,u] + |(O qr_h)[r:]| * page_res[page(u)] + z_eff * |qc_h| * eta_u)
+ * and the row fires when T > s*_h, the attended set's max logit. With top_j > 0 only the top_j fired
+ * rows by (T desc, position asc) are kept. Fired ids are listed in ascending position. */
+void vko_trigger(const vko_view* v, int32_t r, const float* rot, double lam, double z_eff, int32_t top_j,
+                 const double* a, const double* eta, const double* page_res, const int32_t* idx,
+                 const int32_t* count, int32_t cap, const double* smax, int32_t W, int32_t n_sink,
+                 int32_t capf, int32_t* fidx, int32_t* fcount) {
+  const int64_t N = v->N, P = (N + PAGE - 1) / PAGE;
+#pragma omp parallel for collapse(2) schedule(dynamic)
+  for (int b = 0; b < v->B; ++b) {
+    for (int h = 0; h < v->H; ++h) {
+      double q[D_ROPE], qt[D_ROPE], qres = 0.0, qcn = 0.0;
+      for (int j = 0; j < D_ROPE; ++j) q[j] = QR(v, b, h, j);
+      if (r < D_ROPE) {
+        rotate64(rot, q, qt);
+        for (int j = r; j < D_ROPE; ++j) qres += qt[j] * qt[j];
+        qres = sqrt(qres);
+      }
+      for (int j = 0; j < D_LAT; ++j) qcn += QC(v, b, h, j) * QC(v, b, h, j);
+      qcn = sqrt(qcn);
+      double zz = (g_mutation == MUT_TRIGGER_NO_Z) ? 0.0 : z_eff;
+
+      char* in_set = (char*)calloc((size_t)N + 1, 1);
+      const int32_t* set = &idx[((int64_t)b * v->H + h) * cap];
+      int32_t n = count[b * v->H + h];
+      if (n > cap) n = cap;
+      for (int32_t i = 0; i < n; ++i) in_set[set[i]] = 1;
+      double sstar = smax[b * v->H + h];
+      const double* s = &a[((int64_t)b * v->H + h) * N];
+
+      int64_t lo = n_sink, hi = N - W;
+      item* fired = (item*)malloc(sizeof(item) * (size_t)(hi > lo ? hi - lo : 1));
+      int64_t nf = 0;
+      for (int64_t u = lo; u < hi; ++u) {
+        if (in_set[u]) continue;
+        double t = lam * (s[u] + qres * page_res[(int64_t)b * P + u / PAGE] + zz * qcn * eta[(int64_t)b * N + u]);
+        if (t > sstar) { fired[nf].key = t; fired[nf].u = (int32_t)u; ++nf; }
+      }
+      if (top_j > 0 && nf > top_j) {
+        qsort(fired, (size_t)nf, sizeof(item), by_key_desc_pos_asc);
+        nf = top_j;
+      }
+      char* mark = (char*)calloc((size_t)N + 1, 1);
+      for (int64_t i = 0; i < nf; ++i) mark[fired[i].u] = 1;
+      int32_t c = 0;
+      int32_t* out = &fidx[((int64_t)b * v->H + h) * capf];
+      for (int64_t u = 0; u < N; ++u)
+        if (mark[u]) { if (c < capf) out[c] = (int32_t)u; ++c; }
+      fcount[b * v->H + h] = c;
+      free(mark);
+      free(fired);
+      free(in_set);
+    }
+  }
+}
+
+/* ---------------------------------------------------------------- one decode step */
+/* Score -> select -> attend; in two-tier mode also index -> trigger -> attend over S u F, which equals
+ * the LSE merge of the two partial softmaxes (Lemma 1). idx lists S_h (ascending) followed by F_h
+ * (ascending); count = |S_h| + |F_h|. Returns 0, or -4 when a list does not fit in cap. */
+int vko_decode_step(const vko_view* v, double rho, int32_t r, int32_t W, int32_t n_sink, double lam,
+                    int32_t trigger, double z_eff, int32_t top_j, const float* rot, const uint16_t* digest,
+                    int32_t cap, double* out, double* lse, double* smax, int32_t* idx, int32_t* count,
+                    double* kth) {
+  const int64_t BH = (int64_t)v->B * v->H, N = v->N, P = (N + PAGE - 1) / PAGE;
+  int rc = 0;
+  double* a = (double*)malloc(sizeof(double) * (size_t)(BH * N));
+  vko_scores(v, r, rot, digest, a);
+  int64_t k = vko_keep_count(v->N, rho, W, n_sink);
+  vko_select(v->B, v->H, v->N, a, k, W, n_sink, cap, idx, count, kth);
+  for (int64_t i = 0; i < BH; ++i) if (count[i] > cap) rc = -4;
+  vko_attention(v, lam, idx, count, cap, out, lse, smax);
+  if (trigger) {
+    double* eta = (double*)malloc(sizeof(double) * (size_t)(v->B * N));
+    double* pres = (double*)malloc(sizeof(double) * (size_t)(v->B * P));
+    double* dig = (r < D_ROPE) ? (double*)malloc(sizeof(double) * (size_t)(v->B * N * r)) : NULL;
+    vko_build_index(v, r, rot, dig, NULL, eta, pres);
+    int32_t capf = (int32_t)N;
+    int32_t* fidx = (int32_t*)malloc(sizeof(int32_t) * (size_t)(BH * capf));
+    int32_t* fcount = (int32_t*)malloc(sizeof(int32_t) * (size_t)BH);
+    vko_trigger(v, r, rot, lam, z_eff, top_j, a, eta, pres, idx, count, cap, smax, W, n_sink, capf, fidx, fcount);
+    for (int64_t i = 0; i < BH; ++i) {
+      int32_t* dst = &idx[i * cap];
+      int32_t c = count[i];
+      for (int32_t j = 0; j < fcount[i]; ++j, ++c)
+        if (c < cap) dst[c] = fidx[i * capf + j];
+      if (c > cap) rc = -4;
+      count[i] = c;
+    }
+    double* smax_s = (double*)malloc(sizeof(double) * (size_t)BH);
+    vko_attention(v, lam, idx, count, cap, out, lse, smax_s);
+    free(smax_s);
+    free(fidx); free(fcount); free(eta); free(pres); free(dig);
+  }
+  free(a);
+  return rc;
+}
+
+int vko_num_threads(void) {
+#ifdef _OPENMP
+  return omp_get_max_threads();
+#else
+  return 1;
+#endif
+}
