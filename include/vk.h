@@ -1,0 +1,165 @@
+/*
+ * vk.h -- C ABI of libvk.so: the decode hot path of VestigeKV (arXiv 2609.03949) on one GB300 (sm_103a).
+ *
+ * One decode step of one attention layer over B independent sequences, each with an MLA cache of N rows.
+ * Row u of sequence b is C_u = [L_u ; K_u]: the 512-wide compressed latent and the 64-wide decoupled RoPE key,
+ * stored already rotated at position u (Sec. 3, Eq. 1). The query of head h is absorbed: Qc_h (512 wide, the
+ * latent-side query W_UK^T q^c) and Qr_h (64 wide, rotated at position N). The step is
+ *
+ *   score   a[h,u] = Qr_h . K_u, or (O Qr_h)[0:r] . D_u on a width-r rotated digest D_u
+ *           (Eq. 5's exact summand; the digest is the branch-width reading of Sec. 5)
+ *   select  S_h = top-k of a[h, .] over the archive A = [n_sink, N-W) (ties -> smaller position),
+ *           k = min(ceil(rho*N), |A|), joined with the recent window [N-W, N) and the sinks [0, n_sink)
+ *           (Sec. 4.1: keep top-m plus sinks plus the recent window)
+ *   attend  s[h,u] = lambda (Qc_h . L_u + Qr_h . K_u) over u in S_h; out_h = sum softmax(s) L_u (512 wide),
+ *           lse_h, and s*_h = max s (Eq. 1, Lemma 1)
+ *   trigger (two-tier) F_h = { u in A \ S_h : lambda (a[h,u] + |(O Qr_h)[r:]| P_res[u/64]
+ *           + z_eff |Qc_h| eta_u) > s*_h }, optionally the top_j of them (Eq. 5 with sketch rank 0,
+ *           Lemma 2; the fetch of rows that beat the tier-1 max), attended too and merged by LSE.
+ *
+ * Conventions
+ *   - Every pointer in vk_view / vk_index and every output is DEVICE memory owned by the caller.
+ *     The library never allocates device memory; scratch comes from the caller's workspace.
+ *   - Every call is asynchronous on `stream` (a cudaStream_t, NULL = the legacy default stream) and
+ *     does not synchronise with the host, except vk_poll_status.
+ *   - Arguments are checked on the host before any launch; a bad argument returns VK_ERR_INVALID_ARG or
+ *     VK_ERR_UNSUPPORTED and launches nothing (it is never clamped). vk_last_error() describes it.
+ *   - Element strides (ld, bstride) are in elements of `dtype`. Device pointers must be 16-byte aligned
+ *     and ld * element size a multiple of 16 bytes.
+ *   - Errors found on the device (an id out of range, a full list, a bounded wait that gave up) are written
+ *     to a status word at the start of the workspace; vk_poll_status reads and clears it. The first error
+ *     since the last poll is kept. A new workspace is zeroed once with vk_workspace_init.
+ *   - Calls that share a workspace must be ordered (same stream, or synchronised): they reuse its scratch.
+ */
+#ifndef VK_H
+#define VK_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  VK_OK = 0,
+  VK_ERR_INVALID_ARG = -1,  /* a size, pointer, stride or parameter is out of its documented range */
+  VK_ERR_UNSUPPORTED = -2,  /* valid but not built (e.g. a dtype/shape combination without a kernel) */
+  VK_ERR_WORKSPACE = -3,    /* ws is NULL or smaller than vk_workspace_bytes() */
+  VK_ERR_CAPACITY = -4,     /* an output list was longer than cap (device status) */
+  VK_ERR_CUDA = -5,         /* a CUDA launch or runtime call failed */
+  VK_ERR_TIMEOUT = -6       /* a bounded device-side wait gave up (device status) */
+} vk_status;
+
+typedef enum { VK_BF16 = 0, VK_F32 = 1 } vk_dtype;
+
+typedef enum {
+  VK_TRIG_OFF = 0,  /* tier 1 only: the top-k plus window (plus sinks) */
+  VK_TRIG_CS = 1    /* two-tier: also fetch the archived rows whose Cauchy-Schwarz trigger score beats s* */
+} vk_trigger;
+
+/* The cache and the query of one decode step. */
+typedef struct {
+  int32_t B, H, N;          /* sequences, heads, cached rows per sequence (1 <= N <= 2^24 - 1) */
+  int32_t dtype;            /* vk_dtype of latent, rope, q_latent and q_rope */
+  const void* latent;       /* [B, N, 512]: row u of sequence b at latent + b*latent_bstride + u*latent_ld */
+  int64_t latent_ld, latent_bstride;
+  const void* rope;         /* [B, N, 64]; may alias latent + 512 with rope_ld = latent_ld = 576 */
+  int64_t rope_ld, rope_bstride;
+  const void* q_latent;     /* [B, H, 512] contiguous: the absorbed latent-side query */
+  const void* q_rope;       /* [B, H, 64] contiguous: the RoPE query, rotated at position N */
+} vk_view;
+
+/* Selection and trigger parameters. */
+typedef struct {
+  double rho;               /* keep ratio, 0 < rho <= 1 */
+  int32_t r;                /* score width: 64 (the RoPE columns) or a digest width in {4, 8, 16, 32} */
+  int32_t window;           /* recent window W, 0 <= W <= N */
+  int32_t n_sink;           /* leading sink rows, 0 <= n_sink <= N - W */
+  float sm_scale;           /* attention scale lambda > 0 (1/sqrt(192) for 128 + 64 qk head dims) */
+  int32_t trigger;          /* vk_trigger */
+  float z_eff;              /* trigger certificate multiplier z / sqrt(d_c - r_sk); 1 = the sound bound */
+  int32_t top_j;            /* keep only the top_j fired rows per head; 0 = uncapped */
+  uint32_t flags;           /* VK_FLAG_* below; 0 for normal use */
+} vk_params;
+
+/* Force the exact fallback of the fused selection on every head (for tests; results are unchanged). */
+#define VK_FLAG_FORCE_FALLBACK 0x1u
+/* Use the materialised-score selection path even where the fused path would run (for tests). */
+#define VK_FLAG_FORCE_DENSE 0x2u
+
+/* The per-cache index built once by vk_build_digest (Sec. 4.2 index entry with sketch rank 0). */
+typedef struct {
+  const void* digest;       /* [B, N, r] bf16 contiguous, (O K_u)[0:r] rounded to nearest even; NULL iff r = 64 */
+  const float* eta;         /* [B, N] |L_u|_2; needed only by the trigger */
+  const float* page_res;    /* [B, ceil(N/64)] max over the page of |(O K_u)[r:64]| (0 when r = 64); trigger only */
+  const float* rot;         /* [64, 64] row-major orthogonal O; NULL iff r = 64 */
+} vk_index;
+
+/* k = min(ceil(rho*N), N - W - n_sink): archived rows kept per head (-1 on bad arguments). */
+int64_t vk_keep_count(int32_t N, double rho, int32_t window, int32_t n_sink);
+
+/* Smallest cap that vk_select / vk_decode_step accept: k + W + n_sink (tier 1 only). */
+int32_t vk_min_cap(const vk_view* view, const vk_params* params);
+
+/* Workspace bytes that every call below needs for these shapes with this cap (the worst case; the same
+ * buffer may be reused by consecutive calls on one stream). 0 on bad arguments. */
+size_t vk_workspace_bytes(const vk_view* view, const vk_params* params, int32_t cap);
+
+/* Index build (the compression-time work of Sec. 4.2): for every row, digest = bf16((O K_u)[0:r]) when
+ * r < 64, eta_u = |L_u|_2, and per 64-row page the max of |(O K_u)[r:64]|. Any output may be NULL to skip
+ * it. rot64: [64,64] row-major fp32 orthogonal matrix (device); may be NULL when r = 64. */
+int vk_build_digest(const vk_view* view, const vk_params* params, const float* rot64, void* digest, float* eta,
+                    float* page_res, void* stream);
+
+/* Score every cached row: scores[b,h,u] = a[h,u] (unscaled) as fp32, [B, H, N] contiguous. The RoPE columns
+ * are read when r = 64, the index's digest otherwise. ws holds the rotated queries. */
+int vk_score(const vk_view* view, const vk_params* params, const vk_index* index, float* scores, void* ws,
+             size_t ws_bytes, void* stream);
+
+/* Per-head selection from materialised scores ([B,H,N] fp32, e.g. from vk_score): idx[b,h,0:count) lists
+ * S_h in ascending position, count[b,h] = k + W + n_sink, kth[b,h] = the k-th largest archive score
+ * (+inf when k = 0; kth may be NULL). cap >= vk_min_cap. */
+int vk_select(const vk_view* view, const vk_params* params, const float* scores, int32_t* idx, int32_t* count,
+              float* kth, int32_t cap, void* ws, size_t ws_bytes, void* stream);
+
+/* Absorbed-MLA attention over caller-given sets idx[b,h,0:count[b,h]) (distinct positions in [0,N); an
+ * id out of range is skipped and flags VK_ERR_INVALID_ARG in the device status). out [B,H,512] fp32,
+ * lse [B,H] and smax [B,H] (s*, the max logit) fp32; lse and smax may be NULL. An empty set gives
+ * out = 0 and lse = smax = -inf. */
+int vk_sparse_attn(const vk_view* view, const vk_params* params, const int32_t* idx, const int32_t* count,
+                   int32_t cap, float* out, float* lse, float* smax, void* ws, size_t ws_bytes, void* stream);
+
+/* The whole step: score, select, attend, and with params->trigger = VK_TRIG_CS also the trigger scan, the
+ * attention over the fired rows and the LSE merge. out [B,H,512], lse [B,H]; smax [B,H] (s* of the tier-1
+ * set; may be NULL). idx[b,h,:] lists S_h (ascending) followed by F_h (ascending) and count[b,h] is
+ * |S_h| + |F_h|; fired rows that do not fit in cap are still attended (out/lse stay exact) but are left
+ * out of the list, and VK_ERR_CAPACITY is raised in the device status. index may be NULL when r = 64
+ * and the trigger is off. Nothing synchronises with the host; the call can be captured in a CUDA graph. */
+int vk_decode_step(const vk_view* view, const vk_params* params, const vk_index* index, float* out, float* lse,
+                   float* smax, int32_t* idx, int32_t* count, int32_t cap, void* ws, size_t ws_bytes,
+                   void* stream);
+
+/* Zero the device status word of a new workspace (asynchronous on `stream`). Call once after allocating it. */
+int vk_workspace_init(void* ws, size_t ws_bytes, void* stream);
+
+/* Wait for `stream`, read the device status word at the start of ws (VK_OK or a device-side error of the
+ * calls since the last poll) and clear it. */
+int vk_poll_status(void* ws, void* stream);
+
+/* Profiling: record events[i] (cudaEvent_t handles) on the step's stream at the stage boundaries of every
+ * later vk_decode_step on this host thread: [0] start, then after [1] query prep, [2] scoring, [3] selection,
+ * [4] tier-1 attention, [5] trigger and fired attention (recorded right after [4] when the trigger is off),
+ * [6] the merge. n must be 0 (recording off) or 7. The events must outlive the calls that record them. */
+int vk_profile_set_events(void* const* events, int32_t n);
+
+/* Kernels launched through the library by this host thread since it started. */
+int64_t vk_profile_launches(void);
+
+/* Description of the last error returned on this host thread ("" if none). */
+const char* vk_last_error(void);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* VK_H */

@@ -1,0 +1,359 @@
+// vk_api.cu -- the extern "C" entry points of libvk.so: argument checks, workspace layout, launch order.
+//
+// Every entry point checks its arguments on the host before touching the GPU and refuses (never clamps) a
+// bad one. The launch sequence of a decode step has no host synchronisation and no allocation, so a CUDA
+// graph can capture it.
+#include <cmath>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <mutex>
+
+#include <algorithm>
+
+#include "vk_common.cuh"
+
+namespace vk {
+thread_local int64_t g_launches = 0;
+void count_launches(int n) { g_launches += n; }
+}  // namespace vk
+
+namespace {
+
+thread_local char g_err[512] = "";
+thread_local cudaEvent_t g_prof_events[7];
+thread_local int g_prof_n = 0;
+
+void prof(int i, cudaStream_t st) {
+  if (g_prof_n) cudaEventRecord(g_prof_events[i], st);
+}
+
+int fail(int code, const char* fmt, ...) {
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(g_err, sizeof(g_err), fmt, ap);
+  va_end(ap);
+  return code;
+}
+
+int cuda_fail(cudaError_t e, const char* where) {
+  return fail(VK_ERR_CUDA, "%s: %s", where, cudaGetErrorString(e));
+}
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+constexpr int64_t MAX_N = (1 << 24) - 1;
+constexpr int NUM_SMS_TARGET = 152;   // GB300: splits are sized for 2 CTAs per SM
+
+int check_view(const vk_view* v) {
+  if (!v) return fail(VK_ERR_INVALID_ARG, "view is NULL");
+  if (v->B < 1 || v->H < 1 || v->N < 1) return fail(VK_ERR_INVALID_ARG, "B, H, N must be >= 1 (got %d, %d, %d)", v->B, v->H, v->N);
+  if (v->N > MAX_N) return fail(VK_ERR_INVALID_ARG, "N = %d exceeds %lld", v->N, (long long)MAX_N);
+  if (v->H > vk::MAX_H) return fail(VK_ERR_UNSUPPORTED, "H = %d exceeds %d", v->H, vk::MAX_H);
+  if (v->dtype != VK_BF16 && v->dtype != VK_F32) return fail(VK_ERR_INVALID_ARG, "dtype %d is not VK_BF16/VK_F32", v->dtype);
+  if (!v->latent || !v->rope || !v->q_latent || !v->q_rope) return fail(VK_ERR_INVALID_ARG, "a view pointer is NULL");
+  if (!aligned16(v->latent) || !aligned16(v->rope) || !aligned16(v->q_latent) || !aligned16(v->q_rope))
+    return fail(VK_ERR_INVALID_ARG, "view pointers must be 16-byte aligned");
+  const int64_t esz = v->dtype == VK_BF16 ? 2 : 4;
+  if (v->latent_ld < vk::D_LAT || v->rope_ld < vk::D_ROPE)
+    return fail(VK_ERR_INVALID_ARG, "latent_ld >= 512 and rope_ld >= 64 required (got %lld, %lld)",
+                (long long)v->latent_ld, (long long)v->rope_ld);
+  if ((v->latent_ld * esz) % 16 || (v->rope_ld * esz) % 16 || (v->latent_bstride * esz) % 16 ||
+      (v->rope_bstride * esz) % 16)
+    return fail(VK_ERR_INVALID_ARG, "row and batch strides must be multiples of 16 bytes");
+  if (v->B > 1 && (v->latent_bstride < (int64_t)(v->N - 1) * v->latent_ld + vk::D_LAT ||
+                   v->rope_bstride < (int64_t)(v->N - 1) * v->rope_ld + vk::D_ROPE))
+    return fail(VK_ERR_INVALID_ARG, "batch strides overlap the previous sequence");
+  return VK_OK;
+}
+
+int64_t keep_count(int64_t N, double rho, int64_t W, int64_t s) {
+  int64_t A = N - W - s;
+  if (A < 0) A = 0;
+  int64_t k = (int64_t)std::ceil(rho * (double)N);
+  return k < A ? k : A;
+}
+
+int check_params(const vk_view* v, const vk_params* p) {
+  if (!p) return fail(VK_ERR_INVALID_ARG, "params is NULL");
+  if (!(p->rho > 0.0 && p->rho <= 1.0)) return fail(VK_ERR_INVALID_ARG, "rho = %g is outside (0, 1]", p->rho);
+  if (p->r != 4 && p->r != 8 && p->r != 16 && p->r != 32 && p->r != 64)
+    return fail(VK_ERR_INVALID_ARG, "r = %d is not in {4, 8, 16, 32, 64}", p->r);
+  if (p->window < 0 || p->window > v->N) return fail(VK_ERR_INVALID_ARG, "window = %d is outside [0, N]", p->window);
+  if (p->n_sink < 0 || p->n_sink > v->N - p->window)
+    return fail(VK_ERR_INVALID_ARG, "n_sink = %d is outside [0, N - window]", p->n_sink);
+  if (!(p->sm_scale > 0.f) || !std::isfinite(p->sm_scale)) return fail(VK_ERR_INVALID_ARG, "sm_scale must be finite and > 0");
+  if (p->trigger != VK_TRIG_OFF && p->trigger != VK_TRIG_CS) return fail(VK_ERR_INVALID_ARG, "trigger = %d is unknown", p->trigger);
+  if (!(p->z_eff >= 0.f) || !std::isfinite(p->z_eff)) return fail(VK_ERR_INVALID_ARG, "z_eff must be finite and >= 0");
+  if (p->top_j < 0) return fail(VK_ERR_INVALID_ARG, "top_j must be >= 0");
+  if (p->flags & ~(VK_FLAG_FORCE_FALLBACK | VK_FLAG_FORCE_DENSE)) return fail(VK_ERR_INVALID_ARG, "unknown flags 0x%x", p->flags);
+  return VK_OK;
+}
+
+int check_index(const vk_view* v, const vk_params* p, const vk_index* ix, bool need_trigger) {
+  if (p->r < vk::D_ROPE) {
+    if (!ix || !ix->digest || !ix->rot) return fail(VK_ERR_INVALID_ARG, "r < 64 needs index->digest and index->rot");
+    if (!aligned16(ix->digest) || !aligned16(ix->rot)) return fail(VK_ERR_INVALID_ARG, "index pointers must be 16-byte aligned");
+  }
+  if (need_trigger) {
+    if (!ix || !ix->eta || !ix->page_res) return fail(VK_ERR_INVALID_ARG, "the trigger needs index->eta and index->page_res");
+  }
+  (void)v;
+  return VK_OK;
+}
+
+size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+
+// Positions per attention split: enough CTAs to fill the GPU twice over, within the shared-memory budget.
+void choose_splits(const vk_view& v, int64_t* nsplit, int64_t* split_len) {
+  const int64_t n_hg = (v.H + vk::HG - 1) / vk::HG;
+  const int64_t esz = v.dtype == VK_BF16 ? 2 : 4;
+  const int64_t fixed = (std::min<int64_t>(v.H, vk::HG) + 32) * (vk::D_LAT + vk::D_ROPE) * esz + 1024;
+  int64_t max_len = (vk::SMEM_BUDGET - fixed) / 12 / 32 * 32;
+  max_len = std::max<int64_t>(32, std::min<int64_t>(max_len, vk::SPLIT_MAX));
+  const int64_t min_splits = (v.N + max_len - 1) / max_len;
+  const int64_t target = (2 * NUM_SMS_TARGET + v.B * n_hg - 1) / (v.B * n_hg);
+  const int64_t cap_by_len = (v.N + 255) / 256;
+  int64_t ns = std::max<int64_t>(min_splits, std::min<int64_t>(target, cap_by_len));
+  ns = std::max<int64_t>(1, ns);
+  int64_t len = ((v.N + ns - 1) / ns + 31) / 32 * 32;
+  *split_len = len;
+  *nsplit = (v.N + len - 1) / len;
+}
+
+VkLayout make_layout(const vk_view& v, const vk_params& p) {
+  VkLayout L{};
+  L.B = v.B; L.H = v.H; L.N = v.N;
+  L.nw = (v.N + 31) / 32;
+  L.n_hg = (v.H + vk::HG - 1) / vk::HG;
+  choose_splits(v, &L.nsplit, &L.split_len);
+  L.two_tier = p.trigger != VK_TRIG_OFF;
+  L.dense_scores = true;
+  const int64_t BH = (int64_t)v.B * v.H;
+  const int64_t nslot = L.nsplit * (L.two_tier ? 2 : 1);
+  size_t off = 0;
+  auto take = [&](size_t bytes) { size_t o = off; off = align_up(off + bytes, 256); return o; };
+  L.off_status = take(256);
+  L.off_qt = take(sizeof(float) * BH * vk::D_ROPE);
+  L.off_qcn = take(sizeof(float) * BH);
+  L.off_qrn = take(sizeof(float) * BH);
+  L.off_smax1 = take(sizeof(float) * BH);
+  L.off_nfired = take(sizeof(int64_t) * BH);
+  L.off_scores = take(L.dense_scores ? sizeof(float) * BH * v.N : 0);
+  L.off_selbm = take(sizeof(uint32_t) * BH * L.nw);
+  L.off_firebm = take(L.two_tier ? sizeof(uint32_t) * BH * L.nw : 0);
+  L.off_part_o = take(sizeof(float) * v.B * nslot * v.H * vk::D_LAT);
+  L.off_part_ml = take(sizeof(float) * v.B * nslot * v.H * 2);
+  L.total = off;
+  return L;
+}
+
+template <typename T>
+T* at(void* ws, size_t off) { return reinterpret_cast<T*>(static_cast<char*>(ws) + off); }
+
+int check_ws(const VkLayout& L, void* ws, size_t ws_bytes) {
+  if (!ws) return fail(VK_ERR_WORKSPACE, "workspace is NULL (%zu bytes needed)", L.total);
+  if ((reinterpret_cast<uintptr_t>(ws) & 255u) != 0) return fail(VK_ERR_WORKSPACE, "workspace must be 256-byte aligned");
+  if (ws_bytes < L.total) return fail(VK_ERR_WORKSPACE, "workspace has %zu bytes, %zu needed", ws_bytes, L.total);
+  return VK_OK;
+}
+
+#define VK_CUDA(call, where)                         \
+  do {                                               \
+    cudaError_t e_ = (call);                         \
+    if (e_ != cudaSuccess) return cuda_fail(e_, where); \
+  } while (0)
+
+}  // namespace
+
+extern "C" {
+
+const char* vk_last_error(void) { return g_err; }
+
+int vk_profile_set_events(void* const* events, int32_t n) {
+  g_err[0] = 0;
+  if (n != 0 && n != 7) return fail(VK_ERR_INVALID_ARG, "n must be 0 or 7 (got %d)", n);
+  if (n && !events) return fail(VK_ERR_INVALID_ARG, "events is NULL");
+  for (int i = 0; i < n; ++i) {
+    if (!events[i]) return fail(VK_ERR_INVALID_ARG, "events[%d] is NULL", i);
+    g_prof_events[i] = static_cast<cudaEvent_t>(events[i]);
+  }
+  g_prof_n = n;
+  return VK_OK;
+}
+
+int64_t vk_profile_launches(void) { return vk::g_launches; }
+
+int64_t vk_keep_count(int32_t N, double rho, int32_t window, int32_t n_sink) {
+  if (N < 1 || !(rho > 0.0 && rho <= 1.0) || window < 0 || window > N || n_sink < 0 || n_sink > N - window) return -1;
+  return keep_count(N, rho, window, n_sink);
+}
+
+int32_t vk_min_cap(const vk_view* view, const vk_params* params) {
+  if (check_view(view) != VK_OK || check_params(view, params) != VK_OK) return -1;
+  return (int32_t)(keep_count(view->N, params->rho, params->window, params->n_sink) + params->window + params->n_sink);
+}
+
+size_t vk_workspace_bytes(const vk_view* view, const vk_params* params, int32_t cap) {
+  if (check_view(view) != VK_OK || check_params(view, params) != VK_OK) return 0;
+  (void)cap;
+  return make_layout(*view, *params).total;
+}
+
+int vk_build_digest(const vk_view* view, const vk_params* params, const float* rot64, void* digest, float* eta,
+                    float* page_res, void* stream) {
+  g_err[0] = 0;
+  int rc;
+  if ((rc = check_view(view)) != VK_OK || (rc = check_params(view, params)) != VK_OK) return rc;
+  if (params->r < vk::D_ROPE && (digest || page_res) && !rot64)
+    return fail(VK_ERR_INVALID_ARG, "r < 64 needs rot64 for the digest and page_res");
+  if ((digest && !aligned16(digest)) || (eta && !aligned16(eta)) || (page_res && !aligned16(page_res)))
+    return fail(VK_ERR_INVALID_ARG, "outputs must be 16-byte aligned");
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  VK_CUDA(vk::launch_build_digest(*view, params->r, rot64, static_cast<__nv_bfloat16*>(digest), eta, page_res, st),
+          "build_digest");
+  return VK_OK;
+}
+
+int vk_workspace_init(void* ws, size_t ws_bytes, void* stream) {
+  g_err[0] = 0;
+  if (!ws || ws_bytes < 256) return fail(VK_ERR_WORKSPACE, "workspace is NULL or smaller than 256 bytes");
+  VK_CUDA(cudaMemsetAsync(ws, 0, 256, static_cast<cudaStream_t>(stream)), "workspace init");
+  return VK_OK;
+}
+
+int vk_score(const vk_view* view, const vk_params* params, const vk_index* index, float* scores, void* ws,
+             size_t ws_bytes, void* stream) {
+  g_err[0] = 0;
+  int rc;
+  if ((rc = check_view(view)) != VK_OK || (rc = check_params(view, params)) != VK_OK ||
+      (rc = check_index(view, params, index, false)) != VK_OK)
+    return rc;
+  if (!scores || !aligned16(scores)) return fail(VK_ERR_INVALID_ARG, "scores must be a 16-byte aligned pointer");
+  const VkLayout L = make_layout(*view, *params);
+  if ((rc = check_ws(L, ws, ws_bytes)) != VK_OK) return rc;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  float* qt = at<float>(ws, L.off_qt);
+  VK_CUDA(vk::launch_qprep(*view, params->r, index ? index->rot : nullptr, qt, at<float>(ws, L.off_qcn),
+                           at<float>(ws, L.off_qrn), st), "qprep");
+  VK_CUDA(vk::launch_score_simt(*view, params->r, qt,
+                                static_cast<const __nv_bfloat16*>(index ? index->digest : nullptr), scores, st),
+          "score");
+  return VK_OK;
+}
+
+int vk_select(const vk_view* view, const vk_params* params, const float* scores, int32_t* idx, int32_t* count,
+              float* kth, int32_t cap, void* ws, size_t ws_bytes, void* stream) {
+  g_err[0] = 0;
+  int rc;
+  if ((rc = check_view(view)) != VK_OK || (rc = check_params(view, params)) != VK_OK) return rc;
+  if (!scores || !idx || !count) return fail(VK_ERR_INVALID_ARG, "scores, idx and count must be non-NULL");
+  const int64_t k = keep_count(view->N, params->rho, params->window, params->n_sink);
+  if ((int64_t)cap < k + params->window + params->n_sink)
+    return fail(VK_ERR_INVALID_ARG, "cap = %d < k + W + n_sink = %lld", cap, (long long)(k + params->window + params->n_sink));
+  int* status = nullptr;
+  if (ws) {
+    if ((reinterpret_cast<uintptr_t>(ws) & 255u) != 0 || ws_bytes < 256) return fail(VK_ERR_WORKSPACE, "workspace too small or misaligned");
+    status = at<int>(ws, 0);
+  }
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  VK_CUDA(vk::launch_select_dense(view->B, view->H, view->N, scores, nullptr, k, params->window, params->n_sink, idx,
+                                  count, cap, 0, kth, nullptr, 0, status, st), "select");
+  return VK_OK;
+}
+
+int vk_sparse_attn(const vk_view* view, const vk_params* params, const int32_t* idx, const int32_t* count,
+                   int32_t cap, float* out, float* lse, float* smax, void* ws, size_t ws_bytes, void* stream) {
+  g_err[0] = 0;
+  int rc;
+  if ((rc = check_view(view)) != VK_OK || (rc = check_params(view, params)) != VK_OK) return rc;
+  if (!idx || !count || !out || cap < 0) return fail(VK_ERR_INVALID_ARG, "idx, count and out must be non-NULL, cap >= 0");
+  if (!aligned16(out)) return fail(VK_ERR_INVALID_ARG, "out must be 16-byte aligned");
+  const VkLayout L = make_layout(*view, *params);
+  if ((rc = check_ws(L, ws, ws_bytes)) != VK_OK) return rc;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  int* status = at<int>(ws, L.off_status);
+  uint32_t* bm = at<uint32_t>(ws, L.off_selbm);
+  float* po = at<float>(ws, L.off_part_o);
+  float* pml = at<float>(ws, L.off_part_ml);
+  VK_CUDA(vk::launch_list_to_bitmap(view->B, view->H, view->N, idx, count, cap, bm, L.nw, status, st), "list_to_bitmap");
+  VK_CUDA(vk::launch_attn(*view, params->sm_scale, bm, L.nw, (int)L.nsplit, (int)L.split_len, 0, (int)L.nsplit, po, pml, st),
+          "attention");
+  VK_CUDA(vk::launch_combine(view->B, view->H, (int)L.nsplit, (int)L.nsplit, po, pml, out, lse, smax, st), "combine");
+  return VK_OK;
+}
+
+int vk_decode_step(const vk_view* view, const vk_params* params, const vk_index* index, float* out, float* lse,
+                   float* smax, int32_t* idx, int32_t* count, int32_t cap, void* ws, size_t ws_bytes, void* stream) {
+  g_err[0] = 0;
+  int rc;
+  if ((rc = check_view(view)) != VK_OK || (rc = check_params(view, params)) != VK_OK) return rc;
+  const bool two_tier = params->trigger != VK_TRIG_OFF;
+  if ((rc = check_index(view, params, index, two_tier)) != VK_OK) return rc;
+  if (!out || !lse || !idx || !count) return fail(VK_ERR_INVALID_ARG, "out, lse, idx and count must be non-NULL");
+  if (!aligned16(out)) return fail(VK_ERR_INVALID_ARG, "out must be 16-byte aligned");
+  const int64_t k = keep_count(view->N, params->rho, params->window, params->n_sink);
+  if ((int64_t)cap < k + params->window + params->n_sink)
+    return fail(VK_ERR_INVALID_ARG, "cap = %d < k + W + n_sink = %lld", cap, (long long)(k + params->window + params->n_sink));
+  const VkLayout L = make_layout(*view, *params);
+  if ((rc = check_ws(L, ws, ws_bytes)) != VK_OK) return rc;
+
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  const vk_view& v = *view;
+  const int B = v.B, H = v.H, N = v.N, W = params->window, S = params->n_sink;
+  int* status = at<int>(ws, L.off_status);
+  float* qt = at<float>(ws, L.off_qt);
+  float* qcn = at<float>(ws, L.off_qcn);
+  float* qrn = at<float>(ws, L.off_qrn);
+  float* scores = at<float>(ws, L.off_scores);
+  uint32_t* selbm = at<uint32_t>(ws, L.off_selbm);
+  float* po = at<float>(ws, L.off_part_o);
+  float* pml = at<float>(ws, L.off_part_ml);
+  const int ns = (int)L.nsplit, nslot = two_tier ? 2 * ns : ns;
+
+  prof(0, st);
+  VK_CUDA(vk::launch_qprep(v, params->r, index ? index->rot : nullptr, qt, qcn, qrn, st), "qprep");
+  prof(1, st);
+  VK_CUDA(vk::launch_score_simt(v, params->r, qt, static_cast<const __nv_bfloat16*>(index ? index->digest : nullptr),
+                                scores, st), "score");
+  prof(2, st);
+  VK_CUDA(vk::launch_select_dense(B, H, N, scores, nullptr, k, W, S, idx, count, cap, 0, nullptr, selbm, L.nw, status, st),
+          "select");
+  prof(3, st);
+  VK_CUDA(vk::launch_attn(v, params->sm_scale, selbm, L.nw, ns, (int)L.split_len, 0, nslot, po, pml, st), "attention");
+  prof(4, st);
+  if (two_tier) {
+    float* smax1 = at<float>(ws, L.off_smax1);
+    int64_t* nfired = at<int64_t>(ws, L.off_nfired);
+    uint32_t* firebm = at<uint32_t>(ws, L.off_firebm);
+    VK_CUDA(vk::launch_smax_reduce(B, H, ns, nslot, pml, smax1, st), "smax");
+    VK_CUDA(vk::launch_trigger_dense(B, H, N, W, S, params->sm_scale, params->z_eff, params->top_j, scores, qcn, qrn,
+                                     index->eta, index->page_res, smax1, selbm, firebm, L.nw, nfired, st), "trigger");
+    if (params->top_j > 0) {
+      VK_CUDA(vk::launch_select_dense(B, H, N, scores, nfired, params->top_j, 0, 0, idx, count, cap, 1, nullptr, firebm,
+                                      L.nw, status, st), "top_j");
+    } else {
+      VK_CUDA(vk::launch_bitmap_to_list(B, H, N, firebm, L.nw, idx, count, cap, status, st), "fired list");
+    }
+    VK_CUDA(vk::launch_attn(v, params->sm_scale, firebm, L.nw, ns, (int)L.split_len, ns, nslot, po, pml, st),
+            "fired attention");
+  }
+  prof(5, st);
+  VK_CUDA(vk::launch_combine(B, H, nslot, ns, po, pml, out, lse, smax, st), "combine");
+  prof(6, st);
+  return VK_OK;
+}
+
+int vk_poll_status(void* ws, void* stream) {
+  g_err[0] = 0;
+  if (!ws) return fail(VK_ERR_WORKSPACE, "workspace is NULL");
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  int code = 0;
+  VK_CUDA(cudaStreamSynchronize(st), "poll: synchronize");
+  VK_CUDA(cudaMemcpy(&code, ws, sizeof(int), cudaMemcpyDeviceToHost), "poll: read");
+  VK_CUDA(cudaMemset(ws, 0, sizeof(int)), "poll: clear");
+  if (code != 0) return fail(code, "device status %d", code);
+  return VK_OK;
+}
+
+}  // extern "C"

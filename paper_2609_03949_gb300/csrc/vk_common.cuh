@@ -1,0 +1,115 @@
+// vk_common.cuh -- device helpers and launch declarations shared by the libvk.so translation units.
+#pragma once
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "../../include/vk.h"
+
+namespace vk {
+
+constexpr int D_LAT = 512;
+constexpr int D_ROPE = 64;
+constexpr int PAGE = 64;
+constexpr int MAX_H = 256;           // heads per call supported by the kernels
+constexpr int HG = 64;               // heads per attention CTA (one bit each in a 64-bit row mask)
+constexpr int SPLIT_MAX = 4096;      // positions per attention split (bounds the CTA's union list)
+constexpr int SMEM_OPTIN = 227 * 1024;  // opt-in shared memory per CTA on sm_103a (static + dynamic)
+constexpr int SMEM_BUDGET = 220 * 1024; // what the host plans dynamic shared memory against
+
+// ------------------------------------------------------------------------------------------ scalar helpers
+__device__ __forceinline__ float to_f(float x) { return x; }
+__device__ __forceinline__ float to_f(__nv_bfloat16 x) { return __bfloat162float(x); }
+__device__ __forceinline__ float bf_lo(uint32_t w) { return __uint_as_float(w << 16); }
+__device__ __forceinline__ float bf_hi(uint32_t w) { return __uint_as_float(w & 0xffff0000u); }
+
+// Order-preserving map float -> uint32 (a < b  <=>  key(a) < key(b)); -0 is folded onto +0 first.
+__device__ __forceinline__ uint32_t fkey(float f) {
+  if (f == 0.0f) f = 0.0f;
+  uint32_t b = __float_as_uint(f);
+  return (b & 0x80000000u) ? ~b : (b | 0x80000000u);
+}
+__device__ __forceinline__ float funkey(uint32_t k) {
+  uint32_t b = (k & 0x80000000u) ? (k & 0x7fffffffu) : ~k;
+  return __uint_as_float(b);
+}
+
+// First error wins; later ones are dropped until the host polls and clears the word.
+__device__ __forceinline__ void raise_status(int* status, int code) {
+  if (status) atomicCAS(status, 0, code);
+}
+
+// Block-wide exclusive scan of one int per thread (blockDim.x multiple of 32, <= 1024).
+// `scratch` needs 33 ints. Returns the exclusive prefix; *total receives the block sum.
+__device__ __forceinline__ int block_exclusive_scan(int v, int* scratch, int* total) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nwarps = blockDim.x >> 5;
+  int x = v;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    int y = __shfl_up_sync(0xffffffffu, x, o);
+    if (lane >= o) x += y;
+  }
+  if (lane == 31) scratch[warp] = x;
+  __syncthreads();
+  if (warp == 0) {
+    int w = lane < nwarps ? scratch[lane] : 0;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      int y = __shfl_up_sync(0xffffffffu, w, o);
+      if (lane >= o) w += y;
+    }
+    if (lane < nwarps) scratch[lane] = w;     // inclusive per-warp totals
+    if (lane == 31) scratch[32] = w;
+  }
+  __syncthreads();
+  int prefix = (warp ? scratch[warp - 1] : 0) + x - v;
+  *total = scratch[32];
+  __syncthreads();
+  return prefix;
+}
+
+}  // namespace vk
+
+// ------------------------------------------------------------------------------------------ workspace
+// Byte offsets of every scratch region inside the caller's workspace, for one set of shapes.
+struct VkLayout {
+  int64_t B, H, N, nw;          // nw = 32-bit words per head bitmap
+  int64_t nsplit;               // attention splits per sequence (per tier)
+  int64_t split_len;            // positions per split (multiple of 32)
+  int64_t n_hg;                 // head groups of 64
+  bool dense_scores;            // materialised [B,H,N] scores are part of the layout
+  bool two_tier;
+  size_t off_status, off_qt, off_qcn, off_qrn, off_smax1, off_nfired, off_scores, off_selbm, off_firebm,
+      off_part_o, off_part_ml, total;
+};
+
+// ------------------------------------------------------------------------------------------ launchers
+// Every launcher enqueues on `st`, counts its kernel launches and returns cudaGetLastError().
+namespace vk {
+void count_launches(int n);
+cudaError_t launch_qprep(const vk_view& v, int r, const float* rot, float* qt, float* qcn, float* qrn,
+                         cudaStream_t st);
+cudaError_t launch_score_simt(const vk_view& v, int r, const float* qt, const __nv_bfloat16* digest,
+                              float* scores, cudaStream_t st);
+cudaError_t launch_select_dense(int B, int H, int N, const float* scores, const int64_t* k_per_head,
+                                int64_t k, int W, int n_sink, int32_t* idx, int32_t* count, int cap,
+                                int append_from_count, float* kth, uint32_t* bitmap, int64_t nw, int* status,
+                                cudaStream_t st);
+cudaError_t launch_build_digest(const vk_view& v, int r, const float* rot, __nv_bfloat16* digest, float* eta,
+                                float* page_res, cudaStream_t st);
+cudaError_t launch_list_to_bitmap(int B, int H, int N, const int32_t* idx, const int32_t* count, int cap,
+                                  uint32_t* bitmap, int64_t nw, int* status, cudaStream_t st);
+size_t attn_smem_bytes(int dtype, int H, int split_len);
+cudaError_t launch_attn(const vk_view& v, float lam, const uint32_t* bitmap, int64_t nw, int nsplit,
+                        int split_len, int slot0, int nslot, float* part_o, float* part_ml, cudaStream_t st);
+cudaError_t launch_smax_reduce(int B, int H, int nsplit, int nslot, const float* part_ml, float* smax,
+                               cudaStream_t st);
+cudaError_t launch_combine(int B, int H, int nslot, int nslot_tier1, const float* part_o, const float* part_ml,
+                           float* out, float* lse, float* smax, cudaStream_t st);
+cudaError_t launch_trigger_dense(int B, int H, int N, int W, int n_sink, float lam, float z_eff, int top_j,
+                                 float* scores, const float* qcn, const float* qrn, const float* eta,
+                                 const float* page_res, const float* smax1, const uint32_t* selbm,
+                                 uint32_t* firebm, int64_t nw, int64_t* nfired, cudaStream_t st);
+cudaError_t launch_bitmap_to_list(int B, int H, int N, const uint32_t* bitmap, int64_t nw, int32_t* idx,
+                                  int32_t* count, int cap, int* status, cudaStream_t st);
+}  // namespace vk

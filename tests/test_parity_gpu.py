@@ -1,0 +1,276 @@
+"""GPU parity: the CUDA path through the C ABI against the CPU oracle on seeded synthetic workloads.
+
+Tolerances (from the specification of the path): selections exact except rows within 1e-3 relative of the
+k-th threshold; outputs within max relative error 2e-2 (bf16 inputs, fp32 accumulation); lse within 2e-2.
+Small and medium cases are checked on every sequence; the large throughput-sweep cases on sequences 0 and B-1.
+"""
+import math
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2609_03949_gb300 import datagen
+from paper_2609_03949_gb300 import vk
+
+from parity_util import GpuStep, check_fired, check_outputs, check_selection
+
+pytestmark = pytest.mark.gpu
+LAM = vk.DEFAULT_SM_SCALE
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _lib():
+    from paper_2609_03949_gb300 import _build
+    _build.build()
+    vk.lib()
+
+
+def run_case(wl, *, rho, r=64, window=0, n_sink=0, trigger=0, z_eff=1.0, top_j=0, flags=0, check_seqs=None,
+             cap=None):
+    """Run one step on the GPU and check it against the oracle on the sequences `check_seqs`."""
+    seqs = list(range(wl.B)) if check_seqs is None else check_seqs
+    sub = wl.slice_batch(seqs) if check_seqs is not None else wl
+    hi = oracle.HostInputs(sub)
+    dig16 = None
+    if r < 64:
+        hi_all = oracle.HostInputs(wl)
+        _, dig16, _, _ = oracle.build_index(hi_all, r)
+    g = GpuStep(wl, rho=rho, r=r, window=window, n_sink=n_sink, trigger=trigger, z_eff=z_eff, top_j=top_j,
+                flags=flags, digest_bf16=dig16, cap=cap).run()
+    for key in ("out", "lse", "smax", "idx", "count"):
+        g[key] = g[key][seqs]
+    a = oracle.scores(hi, r, None if dig16 is None else dig16[seqs])
+    k = oracle.keep_count(wl.N, rho, window, n_sink)
+    nS = k + window + n_sink
+    st = check_selection(a, g["idx"], g["count"], k, window, n_sink)
+    res = dict(gpu=g, a=a, k=k, sel=st, hi=hi, sub=sub)
+    if not trigger:
+        assert np.all(g["count"] == nS)
+        res["out"] = check_outputs(hi, LAM, g)
+        return res
+    # two-tier: s* of the GPU's tier-1 set, the fired rows, then the output over S u F
+    _, _, smax_ref = oracle.attention(hi, LAM, g["idx"][..., :nS], np.full_like(g["count"], nS))
+    np.testing.assert_allclose(g["smax"], smax_ref, rtol=1e-4, atol=1e-4)
+    _, _, eta, pres = oracle.build_index(hi, r)
+    gF = [[g["idx"][b, h, nS:g["count"][b, h]].tolist() for h in range(wl.H)] for b in range(len(seqs))]
+    res["swaps"] = check_fired(a, eta, pres, sub, LAM, z_eff, r, smax_ref, g["idx"], np.full_like(g["count"], nS), gF,
+                               window, n_sink, top_j)
+    res["out"] = check_outputs(hi, LAM, g)
+    res["fired"] = int((g["count"] - nS).sum())
+    return res
+
+
+# ------------------------------------------------------------------------------------------------ configs
+def test_config1_fp32():
+    wl = datagen.config_workload(1)
+    res = run_case(wl, rho=1 / 8, window=64)
+    for pos, h in zip(wl.planted_pos[0].tolist(), wl.planted_head.tolist()):
+        assert pos in res["gpu"]["idx"][0, h].tolist()
+    assert res["out"]["out_rel"] < 1e-4
+
+
+@pytest.mark.parametrize("r", [4, 8, 16, 32, 64])
+@pytest.mark.parametrize("rho", [1 / 8, 1 / 32, 1 / 128])
+def test_config2_rho_r(rho, r):
+    wl = datagen.config_workload(2, device="cuda")
+    res = run_case(wl, rho=rho, r=r, window=128)
+    assert res["out"]["out_rel"] < 1e-3
+
+
+@pytest.mark.parametrize("rho", [1 / 32, 1 / 128])
+def test_config3_lognormal(rho):
+    wl = datagen.config_workload(3, device="cuda")
+    run_case(wl, rho=rho, window=256)
+
+
+def test_config4_two_tier():
+    wl = datagen.config_workload(4, device="cuda")
+    res = run_case(wl, rho=1 / 32, window=256, trigger=1, z_eff=1.0, check_seqs=[0, wl.B - 1])
+    assert res["fired"] > 0
+
+
+@pytest.mark.parametrize("r,z,top_j", [(16, 1.0, 0), (64, 1.0, 16), (8, 0.5, 0)])
+def test_two_tier_variants(r, z, top_j):
+    wl = datagen.config_workload(4, device="cuda", B=2, N=8192)
+    res = run_case(wl, rho=1 / 32, r=r, window=256, trigger=1, z_eff=z, top_j=top_j)
+    assert res["fired"] > 0
+
+
+@pytest.mark.parametrize("N", [16384, 65536, 131072])
+@pytest.mark.parametrize("B", [1, 8, 32, 64])
+def test_config5_sweep(N, B):
+    wl = datagen.make_workload(B, 64, N, dtype="bf16", seed=1000 + 10 * B + N // 16384, n_planted=64,
+                               planted_hi=N - 256, device="cuda")
+    res = run_case(wl, rho=1 / 32, window=256, check_seqs=sorted({0, B - 1}))
+    sub = res["sub"]
+    for i in range(sub.B):
+        for pos, h in zip(sub.planted_pos[i].tolist(), sub.planted_head.tolist()):
+            assert pos in res["gpu"]["idx"][i, h].tolist()
+
+
+# ------------------------------------------------------------------------------------------------ edges
+EDGES = [
+    dict(B=1, H=4, N=1, rho=1.0, window=1),
+    dict(B=1, H=4, N=1, rho=1.0, window=0),
+    dict(B=2, H=8, N=7, rho=0.5, window=2),
+    dict(B=1, H=8, N=63, rho=1 / 8, window=16),
+    dict(B=1, H=8, N=64, rho=1 / 8, window=64),            # k = 0: window only
+    dict(B=1, H=8, N=65, rho=1 / 8, window=16),
+    dict(B=3, H=16, N=1000, rho=1 / 8, window=100, n_sink=4),
+    dict(B=1, H=100, N=4097, rho=1 / 32, window=128),      # two head groups, ragged tail
+    dict(B=1, H=1, N=5000, rho=1 / 16, window=0),
+    dict(B=2, H=64, N=2048, rho=1.0, window=0),            # dense
+    dict(B=2, H=64, N=3000, rho=1 / 8, window=64, dtype="f32"),
+    dict(B=1, H=256, N=2048, rho=1 / 8, window=64),
+]
+
+
+@pytest.mark.parametrize("case", EDGES, ids=lambda c: "-".join(f"{k}{v}" for k, v in c.items()))
+def test_edge_cases(case):
+    c = dict(case)
+    B, H, N = c.pop("B"), c.pop("H"), c.pop("N")
+    dtype = c.pop("dtype", "bf16")
+    wl = datagen.make_workload(B, H, N, dtype=dtype, seed=77 + N + H, n_planted=min(4, N),
+                               planted_hi=max(1, N - c["window"]), device="cuda")
+    res = run_case(wl, **c)
+    if c["rho"] == 1.0 and c.get("window", 0) == 0:
+        assert np.all(res["gpu"]["count"] == N)
+
+
+def test_two_tier_sinks_and_capacity():
+    wl = datagen.make_workload(2, 32, 6000, seed=5, n_planted=16, planted_hi=6000 - 128, device="cuda")
+    run_case(wl, rho=1 / 32, window=128, n_sink=4, trigger=1, z_eff=0.5)
+    # a list cap below |S| + |F|: the fired list is cut and the device status says so, outputs stay exact
+    k = oracle.keep_count(6000, 1 / 32, 128, 4)
+    step = GpuStep(wl, rho=1 / 32, window=128, n_sink=4, trigger=1, z_eff=1.0, cap=k + 128 + 4 + 3)
+    g = step.run()
+    assert g["status"] == vk.VK_ERR_CAPACITY
+    full = GpuStep(wl, rho=1 / 32, window=128, n_sink=4, trigger=1, z_eff=1.0).run()
+    np.testing.assert_array_equal(g["out"], full["out"])
+    np.testing.assert_array_equal(g["lse"], full["lse"])
+
+
+# ------------------------------------------------------------------------------------------------ entry points
+def test_vk_score_matches_oracle():
+    wl = datagen.config_workload(2, device="cuda", N=3000, H=32)
+    hi = oracle.HostInputs(wl)
+    for r in (64, 16):
+        _, dig16, _, _ = oracle.build_index(hi, r)
+        step = GpuStep(wl, rho=1 / 8, r=r, window=0, digest_bf16=dig16)
+        scores = torch.empty(wl.B, wl.H, wl.N, dtype=torch.float32, device="cuda")
+        vk.vk_score(step.view, step.params, step.index, scores, step.buf.ws)
+        got = scores.cpu().double().numpy()
+        ref = oracle.scores(hi, r, dig16)
+        np.testing.assert_allclose(got, ref, rtol=1e-5, atol=1e-4)
+
+
+def test_vk_select_exact_on_integer_ties():
+    # integer-valued scores are exact in fp32, so the selection must match the oracle bit for bit
+    rng = np.random.default_rng(3)
+    B, H, N = 2, 5, 3333
+    a = rng.integers(0, 7, size=(B, H, N)).astype(np.float64)
+    wl = datagen.make_workload(B, H, N, seed=1, device="cuda")
+    view = vk.make_view(wl.cache, wl.q_latent, wl.q_rope)
+    for rho, W, s in ((1 / 8, 100, 3), (1 / 3, 0, 0), (1.0, 50, 0)):
+        p = vk.make_params(rho, window=W, n_sink=s)
+        k = oracle.keep_count(N, rho, W, s)
+        cap = k + W + s
+        idx = torch.full((B, H, cap), -1, dtype=torch.int32, device="cuda")
+        cnt = torch.zeros(B, H, dtype=torch.int32, device="cuda")
+        kth = torch.zeros(B, H, dtype=torch.float32, device="cuda")
+        vk.vk_select(view, p, torch.from_numpy(a).float().cuda(), idx, cnt, kth)
+        ridx, rcnt, rkth = oracle.select(a, k, W, s, cap)
+        np.testing.assert_array_equal(cnt.cpu().numpy(), rcnt)
+        np.testing.assert_array_equal(idx.cpu().numpy(), ridx)
+        np.testing.assert_array_equal(kth.cpu().double().numpy(), rkth)
+
+
+def test_vk_sparse_attn_given_sets():
+    wl = datagen.make_workload(2, 64, 5000, seed=8, device="cuda")
+    hi = oracle.HostInputs(wl)
+    rng = np.random.default_rng(0)
+    cap = 700
+    idx = np.full((2, 64, cap), -1, np.int32)
+    cnt = rng.integers(0, cap + 1, size=(2, 64)).astype(np.int32)
+    cnt[0, 0] = 0
+    for b in range(2):
+        for h in range(64):
+            idx[b, h, :cnt[b, h]] = rng.choice(5000, size=cnt[b, h], replace=False)   # unsorted on purpose
+    view = vk.make_view(wl.cache, wl.q_latent, wl.q_rope)
+    p = vk.make_params(1 / 8)
+    ws = vk.alloc_workspace(view, p, cap)
+    out = torch.empty(2, 64, 512, device="cuda")
+    lse = torch.empty(2, 64, device="cuda")
+    smax = torch.empty(2, 64, device="cuda")
+    vk.vk_sparse_attn(view, p, torch.from_numpy(idx).cuda(), torch.from_numpy(cnt).cuda(), out, lse, smax, ws)
+    assert vk.vk_poll_status(ws) == vk.VK_OK
+    g = dict(out=out.cpu().double().numpy(), lse=lse.cpu().double().numpy())
+    r = check_outputs(hi, LAM, g, idx, cnt)
+    np.testing.assert_allclose(smax.cpu().double().numpy()[cnt > 0], r["smax"][cnt > 0], rtol=1e-4, atol=1e-4)
+    # an id out of range is skipped and reported in the device status
+    idx[1, 3, 0] = 5000
+    vk.vk_sparse_attn(view, p, torch.from_numpy(idx).cuda(), torch.from_numpy(cnt).cuda(), out, lse, smax, ws)
+    assert vk.vk_poll_status(ws) == vk.VK_ERR_INVALID_ARG
+    assert vk.vk_poll_status(ws) == vk.VK_OK
+
+
+def test_build_digest_matches_oracle():
+    wl = datagen.make_workload(2, 4, 1000, seed=12, device="cuda")
+    hi = oracle.HostInputs(wl)
+    view = vk.make_view(wl.cache, wl.q_latent, wl.q_rope)
+    for r in (4, 16, 32, 64):
+        p = vk.make_params(1 / 8, r=r)
+        dig = torch.empty(2, 1000, r, dtype=torch.bfloat16, device="cuda") if r < 64 else None
+        eta = torch.empty(2, 1000, device="cuda")
+        pres = torch.empty(2, 16, device="cuda")
+        vk.vk_build_digest(view, p, wl.rot.cuda(), dig, eta, pres)
+        d64, d16, reta, rpres = oracle.build_index(hi, r)
+        np.testing.assert_allclose(eta.cpu().double().numpy(), reta, rtol=1e-5)
+        np.testing.assert_allclose(pres.cpu().double().numpy(), rpres, rtol=1e-4, atol=1e-5)
+        if r < 64:
+            got = dig.float().cpu().double().numpy()
+            ulp = np.exp2(np.floor(np.log2(np.maximum(np.abs(d64), 1e-30))) - 7)
+            assert np.all(np.abs(got - d64) <= ulp * 1.0001)
+
+
+def test_deterministic_and_graph_capturable():
+    wl = datagen.config_workload(5, device="cuda", B=4, N=16384)
+    step = GpuStep(wl, rho=1 / 32, window=256)
+    a = step.run()
+    b = step.run()
+    for key in ("out", "lse", "idx", "count"):
+        np.testing.assert_array_equal(a[key], b[key])
+    s = torch.cuda.Stream()
+    s.wait_stream(torch.cuda.current_stream())
+    g = torch.cuda.CUDAGraph()
+    step.buf.out.zero_()
+    with torch.cuda.graph(g, stream=s):
+        vk.vk_decode_step(step.view, step.params, step.index, step.buf.out, step.buf.lse, step.buf.smax, step.buf.idx,
+                          step.buf.count, step.buf.ws, stream=s)
+    step.buf.out.zero_()
+    g.replay()
+    torch.cuda.synchronize()
+    np.testing.assert_array_equal(step.buf.out.cpu().double().numpy(), a["out"])
+    np.testing.assert_array_equal(step.buf.idx.cpu().numpy(), a["idx"])
+
+
+def test_permutation_invariance_gpu():
+    # Lemma 1 on the GPU: permuting the cache rows and remapping the ids leaves the attention output unchanged
+    wl = datagen.make_workload(1, 64, 3000, seed=4, device="cuda")
+    rng = np.random.default_rng(1)
+    cap = 300
+    idx = np.stack([np.sort(rng.choice(3000, cap, replace=False)) for _ in range(64)])[None].astype(np.int32)
+    cnt = np.full((1, 64), cap, np.int32)
+    perm = rng.permutation(3000)
+    inv = np.argsort(perm)
+    outs = []
+    for cache, ids in ((wl.cache, idx), (wl.cache[:, perm].contiguous(), inv[idx].astype(np.int32))):
+        view = vk.make_view(cache, wl.q_latent, wl.q_rope)
+        p = vk.make_params(1 / 8)
+        ws = vk.alloc_workspace(view, p, cap)
+        out = torch.empty(1, 64, 512, device="cuda")
+        vk.vk_sparse_attn(view, p, torch.from_numpy(ids).cuda(), torch.from_numpy(cnt).cuda(), out, None, None, ws)
+        outs.append(out.cpu().numpy())
+    np.testing.assert_allclose(outs[0], outs[1], rtol=1e-5, atol=1e-6)
