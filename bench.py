@@ -1,0 +1,364 @@
+"""Benchmark of the sparse MLA decode step (VestigeKV hot path) on GB300.
+
+Workload: a Kimi-K2-shaped layer (64 heads, 512 latent + 64 RoPE, bf16 cache), N = 65536 cached rows per
+sequence, rho = 1/32, r = 64, recent window 256, 64 planted rows per sequence, a batch of 64 independent
+decode sequences per GPU (weak scaling: every rank owns its own 64 sequences). Metric: decode query-tokens/s
+per layer (one query token per sequence per step).
+
+Prints one JSON line (rank 0). `python bench.py --impl reference` times the CPU oracle on the same workload
+instead (a bounded sample of sequences per step), on the host cores.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import numpy as np  # noqa: E402
+import torch  # noqa: E402
+
+H, N, RHO, WINDOW, R, N_PLANTED = 64, 65536, 1 / 32, 256, 64, 64
+B_PER_GPU = 64
+METRIC = "decode query-tokens/s per layer at N=64K, rho=1/32"
+UNIT = "query-tokens/s"
+STAGES = ["qprep", "score", "select", "attn", "trigger", "combine"]
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=50)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", default="native", choices=["native", "reference"])
+    ap.add_argument("--batch", type=int, default=B_PER_GPU)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    return ap.parse_args()
+
+
+def dist_env():
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return rank, world, local
+
+
+def workload_config(B, n_gpus):
+    return {"workload": f"sparse MLA decode step: H={H}, N={N}, rho=1/32, r={R}, window={WINDOW}, bf16 cache "
+                        f"[512 latent + 64 RoPE], {N_PLANTED} planted rows/seq, B={B} sequences per GPU",
+            "heads": H, "context": N, "rho": RHO, "r": R, "window": WINDOW, "batch_per_gpu": B,
+            "global_batch": B * n_gpus, "parallelism": f"independent sequences x{n_gpus} (no collective)",
+            "l2": "inputs larger than L2: each step streams a 4.8 GB cache per GPU (L2 is 129 MB)"}
+
+
+def peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        d = json.load(open(p))
+        return float(d["hbm_gbs"]), "measured"
+    return 6800.0, "fallback"
+
+
+# ------------------------------------------------------------------------------------------------ clocks
+class ClockSampler:
+    """nvidia-smi clocks and throttle reasons, sampled every 100 ms while the timed region runs."""
+
+    FIELDS = ("timestamp,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, device_index: int):
+        self.dev = device_index
+        self.proc = None
+        self.lines = []
+        self.t0 = self.t1 = None
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(["nvidia-smi", "-i", str(self.dev), f"--query-gpu={self.FIELDS}",
+                                          "--format=csv,noheader,nounits", "-lms", "100"],
+                                         stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.th = threading.Thread(target=self._read, daemon=True)
+            self.th.start()
+        except (FileNotFoundError, OSError):
+            self.proc = None
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append((time.time(), line.strip()))
+
+    def mark(self, begin: bool):
+        if begin:
+            self.t0 = time.time()
+        else:
+            self.t1 = time.time()
+
+    def stop(self) -> dict:
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        time.sleep(0.25)
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        rows = []
+        for t, line in self.lines:
+            parts = [x.strip() for x in line.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                rows.append((t, float(parts[1]), float(parts[2]), parts[4:]))
+            except ValueError:
+                continue
+        inside = [r for r in rows if self.t0 is not None and self.t0 - 0.05 <= r[0] <= self.t1 + 0.15]
+        use = inside or rows[-3:]
+        if not use:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"]}
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({n for r in use for n, v in zip(names, r[3][1:5]) if v.lower() == "active"})
+        return {"sm_mhz": float(np.median([r[1] for r in use])), "sm_max_mhz": max(r[2] for r in use),
+                "reasons": reasons, "samples": len(use), "in_timed_region": bool(inside)}
+
+
+# ------------------------------------------------------------------------------------------------ bytes
+def union_rows(idx: torch.Tensor, count: torch.Tensor, n: int) -> int:
+    """Distinct rows attended per sequence, summed over the batch (ids < 0 or past count are ignored)."""
+    B, Hh, cap = idx.shape
+    mask = torch.zeros(B, n + 1, dtype=torch.bool, device=idx.device)
+    valid = torch.arange(cap, device=idx.device)[None, None, :] < count[..., None]
+    ids = torch.where(valid, idx.long(), torch.full_like(idx, n, dtype=torch.long))
+    mask.scatter_(1, ids.reshape(B, -1), True)
+    return int(mask[:, :n].sum().item())
+
+
+def kernel_traffic(kernel: str):
+    """DRAM bytes per launch from the committed ncu summary, if the kernel's source is unchanged since."""
+    path = os.path.join(ROOT, "profiles", "traffic.json")
+    if not os.path.exists(path):
+        return None
+    d = json.load(open(path)).get(kernel)
+    if not d:
+        return None
+    src = os.path.join(ROOT, d["source"])
+    if not os.path.exists(src) or hashlib.sha256(open(src, "rb").read()).hexdigest()[:16] != d["source_sha"]:
+        return None
+    return float(d["bytes_per_launch"]) * d.get("scale_to_bench", 1.0)
+
+
+# ------------------------------------------------------------------------------------------------ CPU oracle
+def oracle_baseline(cache_dev, ql_dev, qr_dev, budget_s=12.0, max_seqs=1024):
+    """The CPU oracle, as it stands, on a bounded sample of this workload's sequences (host cores)."""
+    import oracle
+    from paper_2609_03949_gb300 import datagen
+    done, t_total = 0, 0.0
+    while done < max_seqs and (t_total < budget_s or done == 0):
+        b = done % cache_dev.shape[0]
+        wl = datagen.Workload(B=1, H=H, N=N, dtype="bf16", cache=cache_dev[b:b + 1].cpu(),
+                              q_latent=ql_dev[b:b + 1].cpu(), q_rope=qr_dev[b:b + 1].cpu(),
+                              rot=torch.eye(64), planted_pos=torch.zeros(1, 0, dtype=torch.int64),
+                              planted_head=torch.zeros(0, dtype=torch.int64), seed=0)
+        hi = oracle.HostInputs(wl)
+        t0 = time.perf_counter()
+        oracle.decode_step(hi, rho=RHO, window=WINDOW)
+        t_total += time.perf_counter() - t0
+        done += 1
+        if done == 1 and t_total * max_seqs > 4 * budget_s:
+            max_seqs = max(1, int(budget_s / t_total))
+    return {"value": done / t_total, "unit": UNIT, "cores": oracle.num_threads(), "kind": "oracle",
+            "sample": f"{done} sequence(s) of the bench workload (N={N}, H={H}) through the fp64 C oracle's "
+                      f"whole decode step, {t_total:.1f} s"}
+
+
+def run_reference(args):
+    rank, world, _ = dist_env()
+    if rank != 0:
+        return
+    import oracle
+    from paper_2609_03949_gb300 import datagen
+    wl = datagen.make_workload(2, H, N, seed=1000, n_planted=N_PLANTED, planted_hi=N - WINDOW, device="cpu")
+    his = [oracle.HostInputs(wl.slice_batch([b])) for b in range(wl.B)]
+    for i in range(args.warmup):
+        oracle.decode_step(his[i % 2], rho=RHO, window=WINDOW)
+    t0 = time.perf_counter()
+    for i in range(args.steps):
+        oracle.decode_step(his[i % 2], rho=RHO, window=WINDOW)
+    dt = time.perf_counter() - t0
+    value = args.steps / dt
+    line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": 1e3 * dt / args.steps, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic (seeded, bf16 storage)",
+            "impl": "reference", "config": workload_config(args.batch, args.gpus),
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": oracle.num_threads(), "kind": "oracle",
+                             "sample": f"each step: 1 sequence (N={N}, H={H}) through the fp64 C oracle"},
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+# ------------------------------------------------------------------------------------------------ native
+def run_native(args):
+    rank, world, local = dist_env()
+    if args.gpus != world and world > 1:
+        raise SystemExit(f"--gpus {args.gpus} but WORLD_SIZE {world}")
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    pg = None
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=dev)
+        pg = dist
+    from paper_2609_03949_gb300 import _build, datagen, vk
+    if rank == 0 or not os.path.exists(vk.LIB_PATH):
+        _build.build()
+    if pg:
+        pg.barrier()
+    vk.lib()
+    B = args.batch
+    wl = datagen.make_workload(B, H, N, seed=1000 + 7919 * rank, n_planted=N_PLANTED, planted_hi=N - WINDOW,
+                               device=dev)
+    view = vk.make_view(wl.cache, wl.q_latent, wl.q_rope)
+    params = vk.make_params(RHO, r=R, window=WINDOW)
+    buf = vk.DecodeBuffers(view, params, device=dev)
+    stream = torch.cuda.current_stream(dev)
+
+    # ---- device-timed region: inputs resident in HBM, per-stage CUDA events on the launching stream
+    for _ in range(max(3, args.warmup)):
+        buf.run(view, params)
+    torch.cuda.synchronize()
+    assert vk.vk_poll_status(buf.ws) == vk.VK_OK
+    step_events = [[torch.cuda.Event(enable_timing=True) for _ in range(7)] for _ in range(args.steps)]
+    for evs in step_events:          # create the underlying cudaEvent_t handles outside the timed region
+        for e in evs:
+            e.record(stream)
+    torch.cuda.synchronize()
+    clocks = ClockSampler(local)
+    clocks.start()
+    time.sleep(0.3)
+    t_start = torch.cuda.Event(enable_timing=True)
+    t_end = torch.cuda.Event(enable_timing=True)
+    if pg:
+        pg.barrier()
+    torch.cuda.synchronize()
+    launches0 = vk.vk_profile_launches()
+    clocks.mark(True)
+    t_start.record(stream)
+    for evs in step_events:
+        vk.vk_profile_set_events(evs)    # this step records its stage boundaries into its own events
+        buf.run(view, params)
+    t_end.record(stream)
+    torch.cuda.synchronize()
+    clocks.mark(False)
+    launches = vk.vk_profile_launches() - launches0
+    elapsed_ms = t_start.elapsed_time(t_end)
+    stage_ms = np.zeros(6)
+    total_ms_events = 0.0
+    for evs in step_events:
+        for i in range(6):
+            stage_ms[i] += evs[i].elapsed_time(evs[i + 1])
+        total_ms_events += evs[0].elapsed_time(evs[6])
+    if pg:
+        t = torch.tensor([elapsed_ms], device=dev)
+        pg.all_reduce(t, op=pg.ReduceOp.MAX)
+        elapsed_ms = float(t.item())
+    clk = clocks.stop()
+    vk.vk_profile_set_events([])
+    assert vk.vk_poll_status(buf.ws) == vk.VK_OK
+    # kernel-time per step: the events bracket only the library's launches (host gaps between steps excluded)
+    ms_step = elapsed_ms / args.steps
+    dev_ms_step = total_ms_events / args.steps
+    stage_ms /= args.steps
+
+    # ---- algorithmic bytes (union of the heads' selections, per sequence, summed)
+    from paper_2609_03949_gb300.bytes_model import step_bytes
+    U = union_rows(buf.idx, buf.count, N)
+    score_bytes = B * N * 2 * R
+    attn_bytes = U * 1152
+    step_b = step_bytes(N, B, R, "bf16", U)
+    hbm_peak, peak_kind = peaks()
+    stage_bytes = {"score": score_bytes, "attn": attn_bytes}
+    dom = max(("score", "attn"), key=lambda s: stage_ms[STAGES.index(s)])
+    dom_ms = stage_ms[STAGES.index(dom)]
+    kname = {"score": "score", "attn": "attn"}[dom]
+    achieved = stage_bytes[dom] / (dom_ms * 1e-3) / 1e9
+    roof = {"bound": "hbm", "kernel": kname, "achieved": achieved, "peak": hbm_peak, "unit": "GB/s",
+            "frac": achieved / hbm_peak, "peak_kind": f"{peak_kind} copy bandwidth",
+            "traffic": kernel_traffic(kname), "algorithmic_bytes_per_launch": stage_bytes[dom],
+            "ms_per_launch": dom_ms}
+
+    # ---- end to end through the public C entry point with host buffers (pinned)
+    qlh = wl.q_latent.cpu().pin_memory()
+    qrh = wl.q_rope.cpu().pin_memory()
+    outh = torch.empty_like(buf.out, device="cpu").pin_memory()
+    lseh = torch.empty_like(buf.lse, device="cpu").pin_memory()
+    h2d = qlh.numel() * qlh.element_size() + qrh.numel() * qrh.element_size()
+    d2h = outh.numel() * outh.element_size() + lseh.numel() * lseh.element_size()
+    for _ in range(3):
+        wl.q_latent.copy_(qlh, non_blocking=True)
+        wl.q_rope.copy_(qrh, non_blocking=True)
+        buf.run(view, params)
+        outh.copy_(buf.out, non_blocking=True)
+        lseh.copy_(buf.lse, non_blocking=True)
+    torch.cuda.synchronize()
+    if pg:
+        pg.barrier()
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(args.steps):
+        wl.q_latent.copy_(qlh, non_blocking=True)
+        wl.q_rope.copy_(qrh, non_blocking=True)
+        buf.run(view, params)
+        outh.copy_(buf.out, non_blocking=True)
+        lseh.copy_(buf.lse, non_blocking=True)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    e2e_ms = e0.elapsed_time(e1)
+    if pg:
+        t = torch.tensor([e2e_ms], device=dev)
+        pg.all_reduce(t, op=pg.ReduceOp.MAX)
+        e2e_ms = float(t.item())
+    assert torch.isfinite(lseh).all()
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        cpu = oracle_baseline(wl.cache, wl.q_latent, wl.q_rope)
+
+    total_seqs = B * world
+    line = {
+        "metric": METRIC, "value": total_seqs / (ms_step * 1e-3), "unit": UNIT, "n_gpus": world,
+        "steps": args.steps, "warmup": max(3, args.warmup), "ms_per_step": ms_step, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+        "data": "synthetic (seeded Gaussian MLA cache, bf16)", "config": workload_config(B, world),
+        "roofline": roof, "cpu_baseline": cpu,
+        "e2e": {"value": total_seqs / (e2e_ms / args.steps * 1e-3), "unit": UNIT, "h2d_bytes_per_step": h2d,
+                "d2h_bytes_per_step": d2h},
+        "gpu_launches": int(launches), "clocks": clk,
+        "step": {"device_ms_per_step": dev_ms_step, "algorithmic_bytes": step_b,
+                 "hbm_gbs": step_b / (ms_step * 1e-3) / 1e9, "frac_of_peak": step_b / (ms_step * 1e-3) / 1e9 / hbm_peak,
+                 "union_rows_per_seq": U / B, "union_frac": U / (B * N),
+                 "stage_ms": {s: float(stage_ms[i]) for i, s in enumerate(STAGES)}},
+    }
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if pg:
+        pg.barrier()
+        pg.destroy_process_group()
+
+
+def main():
+    args = parse()
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_native(args)
+
+
+if __name__ == "__main__":
+    main()

@@ -190,7 +190,8 @@ def vk_profile_set_events(events) -> None:
     (None or [] turns recording off)."""
     events = list(events or [])
     for e in events:
-        e.record()      # materialise the underlying cudaEvent_t
+        if e.cuda_event == 0:
+            e.record()  # materialise the underlying cudaEvent_t
     arr = (ctypes.c_void_p * max(1, len(events)))(*[e.cuda_event for e in events])
     _check(lib().vk_profile_set_events(arr, len(events)))
 
