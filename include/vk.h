@@ -7,14 +7,14 @@
  * latent-side query W_UK^T q^c) and Qr_h (64 wide, rotated at position N). The step is
  *
  *   score   a[h,u] = Qr_h . K_u, or (O Qr_h)[0:r] . D_u on a width-r rotated digest D_u
- *           (Eq. 5's exact summand; the digest is the branch-width reading of Sec. 5)
+ *           (Eq. 4's exact summand; the width-r digest follows the branch-width ablation of the appendix)
  *   select  S_h = top-k of a[h, .] over the archive A = [n_sink, N-W) (ties -> smaller position),
  *           k = min(ceil(rho*N), |A|), joined with the recent window [N-W, N) and the sinks [0, n_sink)
  *           (Sec. 4.1: keep top-m plus sinks plus the recent window)
  *   attend  s[h,u] = lambda (Qc_h . L_u + Qr_h . K_u) over u in S_h; out_h = sum softmax(s) L_u (512 wide),
  *           lse_h, and s*_h = max s (Eq. 1, Lemma 1)
  *   trigger (two-tier) F_h = { u in A \ S_h : lambda (a[h,u] + |(O Qr_h)[r:]| P_res[u/64]
- *           + z_eff |Qc_h| eta_u) > s*_h }, optionally the top_j of them (Eq. 5 with sketch rank 0,
+ *           + z_eff |Qc_h| eta_u) > s*_h }, optionally the top_j of them (Eq. 4 with sketch rank 0,
  *           Lemma 2; the fetch of rows that beat the tier-1 max), attended too and merged by LSE.
  *
  * Conventions

@@ -17,7 +17,7 @@
  *   - the cache holds rows 0..N-1; the query sits at position N; the recent window is [N-W, N);
  *   - the archive is A = [n_sink, N-W); k = min(ceil(rho*N), |A|) rows are kept from it per head;
  *   - ties in the top-k go to the smaller position;
- *   - the trigger is row level: Eq. 5 with sketch rank 0 (the content summand is bounded by
+ *   - the trigger is row level: Eq. 4 with sketch rank 0 (the content summand is bounded by
  *     Cauchy-Schwarz with eta_u = |L_u|), plus a page-level bound on the RoPE dims that the width-r
  *     digest does not cover.
  */
@@ -155,7 +155,7 @@ void vko_build_index(const vko_view* v, int32_t r, const float* rot, double* dig
   }
 }
 
-/* ---------------------------------------------------------------- scores (Eq. 5, exact summand) */
+/* ---------------------------------------------------------------- scores (Eq. 4, exact summand) */
 /* a[b,h,u] = qr_h . K_u over the 64 RoPE columns (r = 64), or, for a width-r digest,
  * a = (O qr_h)[0:r] . digest_u with the stored bf16 digest. The attention scale is applied later. */
 void vko_scores(const vko_view* v, int32_t r, const float* rot, const uint16_t* digest, double* a) {
@@ -263,7 +263,7 @@ void vko_attention(const vko_view* v, double lam, const int32_t* idx, const int3
   }
 }
 
-/* ---------------------------------------------------------------- recall trigger (Eq. 5, Lemma 2) */
+/* ---------------------------------------------------------------- recall trigger (Eq. 4, Lemma 2) */
 /* With sketch rank 0 the content summand is bounded by Cauchy-Schwarz: |qc_h . L_u| <= |qc_h| eta_u.
  * For a width-r digest the RoPE dims it leaves out are bounded the same way, page by page:
  * |(O qr_h)[r:] . (O K_u)[r:]| <= |(O qr_h)[r:]| page_res[u/64]. The trigger score of an archived row

@@ -2,7 +2,7 @@
 
 Two models:
 
-* :func:`paper_read_budget` -- the paper's three-term per-token read budget (Eq. 4):
+* :func:`paper_read_budget` -- the paper's three-term per-token read budget (Eq. 2):
   attended rows, the index scan and admitted rows, in bytes per cached token.
 * :func:`step_bytes` -- the algorithmic HBM bytes the decode step of this library must move, which the
   roofline is quoted against: the width-r score read of every cached row, plus every distinct attended row
@@ -17,7 +17,7 @@ ROW_DIMS = D_LATENT + D_ROPE
 
 
 def paper_read_budget(rho: float, r_sk: int, f: float, index_bytes: int = 2, row_bytes: int = 2) -> float:
-    """Eq. 4 in bytes/token: rho*576 attended dims + (1-rho)(64 + r_sk + 1) index dims + f*576 admitted dims.
+    """Eq. 2 in bytes/token: rho*576 attended dims + (1-rho)(64 + r_sk + 1) index dims + f*576 admitted dims.
 
     Attended and admitted dims are cache rows (``row_bytes`` per dim); index dims are ``index_bytes`` each.
     """

@@ -1,10 +1,10 @@
 // k_index.cu -- query preparation, the per-cache index build, SIMT scoring and the dense trigger scan.
 //
-// Query prep (Eq. 5 inputs): qt_h = O Qr_h (or Qr_h when r = 64), |Qc_h|, |(O Qr_h)[r:]|.
+// Query prep (Eq. 4 inputs): qt_h = O Qr_h (or Qr_h when r = 64), |Qc_h|, |(O Qr_h)[r:]|.
 // Index build (Sec. 4.2 index entry with sketch rank 0): digest = bf16((O K_u)[0:r]), eta_u = |L_u|,
 // page_res[page] = max_u |(O K_u)[r:64]|.
 // SIMT scoring: a[h,u] = qt_h[0:r] . key_u[0:r] (fp32) for fp32 caches, digests and small problems.
-// Dense trigger (Eq. 5, Lemma 2): T = lambda (a + |(O Qr)[r:]| page_res + z_eff |Qc| eta) > s*_h.
+// Dense trigger (Eq. 4, Lemma 2): T = lambda (a + |(O Qr)[r:]| page_res + z_eff |Qc| eta) > s*_h.
 #include "vk_common.cuh"
 
 namespace vk {
