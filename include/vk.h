@@ -143,6 +143,28 @@ int vk_decode_step(const vk_view* view, const vk_params* params, const vk_index*
 /* Zero the device status word of a new workspace (asynchronous on `stream`). Call once after allocating it. */
 int vk_workspace_init(void* ws, size_t ws_bytes, void* stream);
 
+/* Scratch size of vk_decode_step_noalloc: 16 MiB of device memory in a static array of this library. */
+#define VK_NOALLOC_SCRATCH_BYTES (16u << 20)
+
+/* The decode step of vk_decode_step for callers that cannot allocate device memory, so cannot pass a
+ * workspace: a plugin that may use only memory its host program gave it and has no allocator behind a C
+ * interface, or a serving loop that fixed its device-memory budget at start-up and forbids later cudaMalloc
+ * calls. The paper has no counterpart; this is a deployment convenience.
+ *   - Scratch comes from one static device array of VK_NOALLOC_SCRATCH_BYTES, which the CUDA runtime sets
+ *     aside on every GPU where this library's code is loaded and keeps until the process exits. The call
+ *     allocates nothing itself (no cudaMalloc, no allocating library routine).
+ *   - Problems whose vk_workspace_bytes() exceeds VK_NOALLOC_SCRATCH_BYTES are rejected with
+ *     VK_ERR_WORKSPACE; bad arguments are refused exactly as vk_decode_step refuses them.
+ *   - The first call on each device looks up the array's device address (cudaGetSymbolAddress) and caches
+ *     it; make that first call before any stream capture on that device.
+ *   - Every call on a device shares the one array and it keeps the last call's contents; the call clears
+ *     the status word it needs at zero. Calls that overlap on the GPU (other streams, other host threads,
+ *     without ordering between them) race on the array and corrupt each other's results.
+ *   - Device-side status (VK_ERR_CAPACITY, VK_ERR_TIMEOUT) is not reported: the status word is reset at
+ *     the start of every call. Outputs are the same as vk_decode_step's. */
+int vk_decode_step_noalloc(const vk_view* view, const vk_params* params, const vk_index* index, float* out,
+                           float* lse, float* smax, int32_t* idx, int32_t* count, int32_t cap, void* stream);
+
 /* Wait for `stream`, read the device status word at the start of ws (VK_OK or a device-side error of the
  * calls since the last poll) and clear it. */
 int vk_poll_status(void* ws, void* stream);

@@ -16,6 +16,7 @@
 namespace vk {
 thread_local int64_t g_launches = 0;
 void count_launches(int n) { g_launches += n; }
+int record_error(int code, const char* msg);
 }  // namespace vk
 
 namespace {
@@ -165,6 +166,9 @@ int check_ws(const VkLayout& L, void* ws, size_t ws_bytes) {
   } while (0)
 
 }  // namespace
+
+// Error reporting for entry points defined in other translation units.
+int vk::record_error(int code, const char* msg) { return fail(code, "%s", msg); }
 
 extern "C" {
 

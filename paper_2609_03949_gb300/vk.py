@@ -68,6 +68,7 @@ def lib():
             "vk_select": ([VP, PP, P, P, P, P, I32, P, SZ, P], ctypes.c_int),
             "vk_sparse_attn": ([VP, PP, P, P, I32, P, P, P, P, SZ, P], ctypes.c_int),
             "vk_decode_step": ([VP, PP, IP, P, P, P, P, P, I32, P, SZ, P], ctypes.c_int),
+            "vk_decode_step_noalloc": ([VP, PP, IP, P, P, P, P, P, I32, P], ctypes.c_int),
             "vk_workspace_init": ([P, SZ, P], ctypes.c_int),
             "vk_poll_status": ([P, P], ctypes.c_int),
             "vk_profile_set_events": ([ctypes.POINTER(ctypes.c_void_p), I32], ctypes.c_int),
@@ -85,7 +86,8 @@ def lib():
 def exported_symbols():
     """Names of the C entry points declared in include/vk.h."""
     return ["vk_keep_count", "vk_min_cap", "vk_workspace_bytes", "vk_build_digest", "vk_score", "vk_select",
-            "vk_sparse_attn", "vk_decode_step", "vk_workspace_init", "vk_poll_status", "vk_profile_set_events",
+            "vk_sparse_attn", "vk_decode_step", "vk_decode_step_noalloc", "vk_workspace_init", "vk_poll_status",
+            "vk_profile_set_events",
             "vk_profile_launches", "vk_last_error"]
 
 
@@ -198,6 +200,13 @@ def vk_profile_set_events(events) -> None:
 
 def vk_profile_launches() -> int:
     return int(lib().vk_profile_launches())
+
+
+def vk_decode_step_noalloc(view, params, index: vk_index | None, out, lse, smax, idx, count, stream=None) -> None:
+    """vk_decode_step with the library's static scratch instead of a workspace (see include/vk.h)."""
+    _check(lib().vk_decode_step_noalloc(ctypes.byref(view), ctypes.byref(params),
+                                        ctypes.byref(index) if index else None, _ptr(out), _ptr(lse), _ptr(smax),
+                                        _ptr(idx), _ptr(count), idx.shape[-1], _stream(stream)))
 
 
 def vk_poll_status(ws: torch.Tensor, stream=None) -> int:
