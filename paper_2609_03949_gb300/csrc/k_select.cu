@@ -11,27 +11,47 @@ namespace vk {
 
 constexpr int SEL_THREADS = 512;
 
-__global__ void __launch_bounds__(SEL_THREADS) k_select_dense(
-    int H, int N, const float* __restrict__ scores, const long long* __restrict__ k_per_head, long long k_all,
-    int W, int n_sink, int32_t* __restrict__ idx, int32_t* __restrict__ count, int cap, int append,
-    float* __restrict__ kth, uint32_t* __restrict__ bitmap, long long nw, int* status) {
+// Key sources for the ordered selection: scores stored in memory, or recomputed from the RoPE columns
+// (the exact fallback of the fused path: a[u] = qt . K_u in fp32, qt already in shared memory).
+struct StoredKeys {
+  const float* a;
+  __device__ __forceinline__ float operator()(int u) const { return a[u]; }
+};
+struct RecomputedKeys {
+  const __nv_bfloat16* rope;    // this sequence's RoPE rows
+  int64_t ld;
+  const float* qt;              // 64 floats in shared memory
+  __device__ __forceinline__ float operator()(int u) const {
+    const uint4* r = reinterpret_cast<const uint4*>(rope + (int64_t)u * ld);
+    float acc = 0.f;
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      const uint4 w = r[i];
+      acc = fmaf(qt[8 * i + 0], bf_lo(w.x), acc); acc = fmaf(qt[8 * i + 1], bf_hi(w.x), acc);
+      acc = fmaf(qt[8 * i + 2], bf_lo(w.y), acc); acc = fmaf(qt[8 * i + 3], bf_hi(w.y), acc);
+      acc = fmaf(qt[8 * i + 4], bf_lo(w.z), acc); acc = fmaf(qt[8 * i + 5], bf_hi(w.z), acc);
+      acc = fmaf(qt[8 * i + 6], bf_lo(w.w), acc); acc = fmaf(qt[8 * i + 7], bf_hi(w.w), acc);
+    }
+    return acc;
+  }
+};
+
+// Ordered per-head selection over positions [0, N) (one CTA): the k largest keys of the archive [lo, hi) by
+// (key desc, position asc), plus -- unless `append` -- every position outside the archive (sinks, window).
+// Writes the ascending id list (after count[bh] entries when appending), the bitmap words, count and kth.
+template <class Keys>
+__device__ void select_ordered(const Keys& key_of, int N, int lo, int hi, long long k, int32_t* out, int32_t* count_bh,
+                               int cap, int append, float* kth_bh, uint32_t* bitmap_bh, long long nw, int* status) {
   __shared__ unsigned int hist[256];
   __shared__ unsigned int s_prefix, s_need;
   __shared__ int scan_scratch[33];
-  const int64_t bh = blockIdx.x;
-  const float* a = scores + bh * (int64_t)N;
-  const int lo = n_sink, hi = N - W;
-  long long k = k_all;
-  if (k_per_head) k = min(k, k_per_head[bh]);
-  if (k > (long long)max(0, hi - lo)) k = max(0, hi - lo);
-
   unsigned int prefix = 0, mask = 0, need = (unsigned int)k;
   if (k > 0) {
     for (int shift = 24; shift >= 0; shift -= 8) {
       for (int i = threadIdx.x; i < 256; i += blockDim.x) hist[i] = 0;
       __syncthreads();
       for (int u = lo + threadIdx.x; u < hi; u += blockDim.x) {
-        const uint32_t key = fkey(a[u]);
+        const uint32_t key = fkey(key_of(u));
         if ((key & mask) == prefix) atomicAdd(&hist[(key >> shift) & 255u], 1u);
       }
       __syncthreads();
@@ -52,21 +72,19 @@ __global__ void __launch_bounds__(SEL_THREADS) k_select_dense(
       __syncthreads();
     }
   }
-  const uint32_t tau = prefix;   // the k-th largest key; `need` of the keys equal to it are kept
+  const uint32_t tau = prefix;   // the k-th largest key; `need` of the keys equal to it are kept (smallest u first)
 
-  int base = append ? count[bh] : 0;
-  const int start_base = base;
+  int base = append ? *count_bh : 0;
   int ties_seen = 0;
-  int32_t* out = idx + bh * (int64_t)cap;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   for (int c = 0; c < N; c += blockDim.x) {
     const int u = c + threadIdx.x;
     bool in = false, tie = false;
     if (u < N) {
       if (u < lo || u >= hi) {
-        in = !append;      // sinks and window are part of S_h, not of an appended list
+        in = !append;
       } else if (k > 0) {
-        const uint32_t key = fkey(a[u]);
+        const uint32_t key = fkey(key_of(u));
         if (key > tau) in = true;
         else if (key == tau) tie = true;
       }
@@ -78,18 +96,31 @@ __global__ void __launch_bounds__(SEL_THREADS) k_select_dense(
     const int pos = base + block_exclusive_scan(in ? 1 : 0, scan_scratch, &tot);
     if (in && pos < cap) out[pos] = u;
     base += tot;
-    if (bitmap) {
+    if (bitmap_bh) {
       const uint32_t word = __ballot_sync(0xffffffffu, in);
       const int w = (c >> 5) + warp;
-      if (lane == 0 && (long long)w < nw) bitmap[bh * nw + w] = word;
+      if (lane == 0 && (long long)w < nw) bitmap_bh[w] = word;
     }
   }
   if (threadIdx.x == 0) {
-    count[bh] = base;
-    if (kth && !append) kth[bh] = k > 0 ? funkey(tau) : INFINITY;
+    *count_bh = base;
+    if (kth_bh && !append) *kth_bh = k > 0 ? funkey(tau) : INFINITY;
     if (base > cap) raise_status(status, VK_ERR_CAPACITY);
-    (void)start_base;
   }
+}
+
+__global__ void __launch_bounds__(SEL_THREADS) k_select_dense(
+    int H, int N, const float* __restrict__ scores, const long long* __restrict__ k_per_head, long long k_all,
+    int W, int n_sink, int32_t* __restrict__ idx, int32_t* __restrict__ count, int cap, int append,
+    float* __restrict__ kth, uint32_t* __restrict__ bitmap, long long nw, int* status) {
+  const int64_t bh = blockIdx.x;
+  const int lo = n_sink, hi = N - W;
+  long long k = k_all;
+  if (k_per_head) k = min(k, k_per_head[bh]);
+  if (k > (long long)max(0, hi - lo)) k = max(0, hi - lo);
+  StoredKeys keys{scores + bh * (int64_t)N};
+  select_ordered(keys, N, lo, hi, k, idx + bh * (int64_t)cap, count + bh, cap, append, kth ? kth + bh : nullptr,
+                 bitmap ? bitmap + bh * nw : nullptr, nw, status);
 }
 
 cudaError_t launch_select_dense(int B, int H, int N, const float* scores, const int64_t* k_per_head, int64_t k,
@@ -98,6 +129,230 @@ cudaError_t launch_select_dense(int B, int H, int N, const float* scores, const 
   k_select_dense<<<B * H, SEL_THREADS, 0, st>>>(H, N, scores, reinterpret_cast<const long long*>(k_per_head),
                                                 (long long)k, W, n_sink, idx, count, cap, append, kth, bitmap,
                                                 (long long)nw, status);
+  count_launches(1);
+  return cudaGetLastError();
+}
+
+// ---------------------------------------------------------------------------------------------- fused path
+// Threshold from a strided sample of the archive: theta[b,h] = the j-th largest sampled score, so that about
+// j * stride archive rows score >= theta (chosen well above k). The candidate pass then emits only those rows.
+// sample[(b*H + h) * ns + i] is the score of position off + stride * i.
+__global__ void __launch_bounds__(SEL_THREADS) k_theta(int ns, int off, int stride, int lo, int hi, int j,
+                                                       const float* __restrict__ sample, float* __restrict__ theta) {
+  __shared__ unsigned int hist[256];
+  __shared__ unsigned int s_prefix, s_need;
+  const int64_t bh = blockIdx.x;
+  const float* a = sample + bh * (int64_t)ns;
+  auto in_archive = [&](int i) { const int u = off + stride * i; return u >= lo && u < hi; };
+  unsigned int prefix = 0, mask = 0, need = (unsigned int)j;
+  // number of sampled archive rows
+  __shared__ int n_arch;
+  if (threadIdx.x == 0) n_arch = 0;
+  __syncthreads();
+  int local = 0;
+  for (int i = threadIdx.x; i < ns; i += blockDim.x) local += in_archive(i);
+  atomicAdd(&n_arch, local);
+  __syncthreads();
+  if (j <= 0 || j > n_arch) {
+    if (threadIdx.x == 0) theta[bh] = -INFINITY;      // emit every archive row
+    return;
+  }
+  for (int shift = 24; shift >= 0; shift -= 8) {
+    for (int i = threadIdx.x; i < 256; i += blockDim.x) hist[i] = 0;
+    __syncthreads();
+    for (int i = threadIdx.x; i < ns; i += blockDim.x) {
+      if (!in_archive(i)) continue;
+      const uint32_t key = fkey(a[i]);
+      if ((key & mask) == prefix) atomicAdd(&hist[(key >> shift) & 255u], 1u);
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) {
+      unsigned int above = 0;
+      int d = 255;
+      for (; d > 0; --d) {
+        if (above + hist[d] >= need) break;
+        above += hist[d];
+      }
+      s_prefix = prefix | ((unsigned int)d << shift);
+      s_need = need - above;
+    }
+    __syncthreads();
+    prefix = s_prefix;
+    need = s_need;
+    mask |= 255u << shift;
+    __syncthreads();
+  }
+  if (threadIdx.x == 0) theta[bh] = funkey(prefix);
+}
+
+cudaError_t launch_theta(int B, int H, int ns, int off, int stride, int lo, int hi, int j, const float* sample,
+                         float* theta, cudaStream_t st) {
+  k_theta<<<B * H, SEL_THREADS, 0, st>>>(ns, off, stride, lo, hi, j, sample, theta);
+  count_launches(1);
+  return cudaGetLastError();
+}
+
+// Selection from a head's candidate list (every archive row with score >= theta, in arbitrary order). When the
+// list holds at least k and at most capc entries it contains the whole top-k, which is found by a radix select
+// (ties by smaller position, via a second select on the positions of the tied keys); the selected rows, the
+// sinks and the window become the head's bitmap and ascending id list. The list is staged in shared memory when
+// it has at most smem_cap entries and read from global memory otherwise. When the list is too short or too long
+// (theta landed too high or too low) or with VK_FLAG_FORCE_FALLBACK, the head takes the exact ordered selection
+// over scores recomputed from the RoPE columns. With `append` (the top_j of the fired rows, whose list can never
+// overflow) only candidates are selected, no sinks or window, and the ids are appended after count[b,h].
+__global__ void __launch_bounds__(SEL_THREADS) k_select_cand(
+    int H, int N, int lo, int hi, long long k_all, const long long* __restrict__ k_per_head,
+    const int* __restrict__ cand_cnt, const int2* __restrict__ cand, int capc, int smem_cap, int force_fallback,
+    const __nv_bfloat16* __restrict__ rope, int64_t rld, int64_t rbs, const float* __restrict__ qt,
+    int32_t* __restrict__ idx, int32_t* __restrict__ count, int cap, int append, float* __restrict__ kth,
+    uint32_t* __restrict__ bitmap, long long nw, int* status) {
+  extern __shared__ __align__(16) unsigned char smem[];
+  uint32_t* skey = reinterpret_cast<uint32_t*>(smem);          // [smem_cap]
+  int32_t* spos = reinterpret_cast<int32_t*>(skey + smem_cap); // [smem_cap]
+  __shared__ unsigned int hist[256];
+  __shared__ unsigned int s_prefix, s_need;
+  __shared__ float qts[D_ROPE];
+  __shared__ int scan_scratch[33];
+  const int64_t bh = blockIdx.x;
+  const int b = (int)(bh / H);
+  long long k = k_all;
+  if (k_per_head) k = min(k, k_per_head[bh]);
+  const int c = cand_cnt[bh];
+  if (append) k = min(k, (long long)c);
+  uint32_t* bm = bitmap + bh * nw;
+  int32_t* out = idx + bh * (int64_t)cap;
+
+  if (force_fallback || c < k || c > capc) {
+    if (append) {                       // cannot happen: the fired list has room for the whole archive
+      if (threadIdx.x == 0) raise_status(status, VK_ERR_CAPACITY);
+      return;
+    }
+    for (int i = threadIdx.x; i < D_ROPE; i += blockDim.x) qts[i] = qt[bh * D_ROPE + i];
+    __syncthreads();
+    RecomputedKeys keys{rope + (int64_t)b * rbs, rld, qts};
+    select_ordered(keys, N, lo, hi, k, out, count + bh, cap, 0, kth ? kth + bh : nullptr, bm, nw, status);
+    return;
+  }
+
+  const bool staged = c <= smem_cap;
+  const int2* g = cand + bh * (int64_t)capc;
+  if (staged) {
+    for (int i = threadIdx.x; i < c; i += blockDim.x) {
+      const int2 e = g[i];
+      spos[i] = e.x;
+      skey[i] = fkey(__int_as_float(e.y));
+    }
+    __syncthreads();
+  }
+  auto key_at = [&](int i) -> uint32_t { return staged ? skey[i] : fkey(__int_as_float(g[i].y)); };
+  auto pos_at = [&](int i) -> uint32_t { return staged ? (uint32_t)spos[i] : (uint32_t)g[i].x; };
+
+  // radix select of the k-th largest key among the c candidates
+  unsigned int prefix = 0, mask = 0, need = (unsigned int)k;
+  uint32_t pos_cut = 0u;
+  if (k > 0) {
+    for (int shift = 24; shift >= 0; shift -= 8) {
+      for (int i = threadIdx.x; i < 256; i += blockDim.x) hist[i] = 0;
+      __syncthreads();
+      for (int i = threadIdx.x; i < c; i += blockDim.x) {
+        const uint32_t key = key_at(i);
+        if ((key & mask) == prefix) atomicAdd(&hist[(key >> shift) & 255u], 1u);
+      }
+      __syncthreads();
+      if (threadIdx.x == 0) {
+        unsigned int above = 0;
+        int d = 255;
+        for (; d > 0; --d) {
+          if (above + hist[d] >= need) break;
+          above += hist[d];
+        }
+        s_prefix = prefix | ((unsigned int)d << shift);
+        s_need = need - above;
+      }
+      __syncthreads();
+      prefix = s_prefix;
+      need = s_need;
+      mask |= 255u << shift;
+      __syncthreads();
+    }
+    // among keys equal to tau keep the `need` smallest positions: find the need-th smallest of them
+    unsigned int pprefix = 0, pmask = 0, pneed = need;
+    for (int shift = 24; shift >= 0; shift -= 8) {
+      for (int i = threadIdx.x; i < 256; i += blockDim.x) hist[i] = 0;
+      __syncthreads();
+      for (int i = threadIdx.x; i < c; i += blockDim.x) {
+        const uint32_t p = pos_at(i);
+        if (key_at(i) == prefix && (p & pmask) == pprefix) atomicAdd(&hist[(p >> shift) & 255u], 1u);
+      }
+      __syncthreads();
+      if (threadIdx.x == 0) {
+        unsigned int below = 0;
+        int d = 0;
+        for (; d < 255; ++d) {
+          if (below + hist[d] >= pneed) break;
+          below += hist[d];
+        }
+        s_prefix = pprefix | ((unsigned int)d << shift);
+        s_need = pneed - below;
+      }
+      __syncthreads();
+      pprefix = s_prefix;
+      pneed = s_need;
+      pmask |= 255u << shift;
+      __syncthreads();
+    }
+    pos_cut = pprefix;
+  }
+  const uint32_t tau = prefix;
+  // bitmap: clear this head's words, then set sinks and window (tier 1) and the selected candidates
+  for (long long w = threadIdx.x; w < nw; w += blockDim.x) bm[w] = 0u;
+  __syncthreads();
+  if (!append) {
+    for (int u = threadIdx.x; u < lo; u += blockDim.x) atomicOr(&bm[u >> 5], 1u << (u & 31));
+    for (int u = hi + threadIdx.x; u < N; u += blockDim.x) atomicOr(&bm[u >> 5], 1u << (u & 31));
+  }
+  if (k > 0) {
+    for (int i = threadIdx.x; i < c; i += blockDim.x) {
+      const uint32_t key = key_at(i), p = pos_at(i);
+      if (key > tau || (key == tau && p <= pos_cut)) atomicOr(&bm[p >> 5], 1u << (p & 31));
+    }
+  }
+  __syncthreads();
+  // ascending ids from the bitmap
+  int base = append ? count[bh] : 0;
+  for (long long c0 = 0; c0 < nw; c0 += blockDim.x) {
+    const long long w = c0 + threadIdx.x;
+    const uint32_t word = (w < nw) ? bm[w] : 0u;
+    int tot;
+    int pos = base + block_exclusive_scan(__popc(word), scan_scratch, &tot);
+    uint32_t bits = word;
+    while (bits) {
+      const int i = __ffs(bits) - 1;
+      bits &= bits - 1;
+      if (pos < cap) out[pos] = (int32_t)(w * 32 + i);
+      ++pos;
+    }
+    base += tot;
+  }
+  if (threadIdx.x == 0) {
+    count[bh] = base;
+    if (kth && !append) kth[bh] = k > 0 ? funkey(tau) : INFINITY;
+    if (base > cap) raise_status(status, VK_ERR_CAPACITY);
+  }
+}
+
+cudaError_t launch_select_cand(int B, int H, int N, int lo, int hi, int64_t k, const int64_t* k_per_head,
+                               const int* cand_cnt, const int2* cand, int capc, int force_fallback, const vk_view& v,
+                               const float* qt, int32_t* idx, int32_t* count, int cap, int append, float* kth,
+                               uint32_t* bitmap, int64_t nw, int* status, cudaStream_t st) {
+  const int smem_cap = capc < 12288 ? capc : 12288;
+  const size_t smem = (size_t)smem_cap * 8;
+  cudaError_t e = cudaFuncSetAttribute(k_select_cand, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (e != cudaSuccess) return e;
+  k_select_cand<<<B * H, SEL_THREADS, smem, st>>>(
+      H, N, lo, hi, (long long)k, reinterpret_cast<const long long*>(k_per_head), cand_cnt, cand, capc, smem_cap,
+      force_fallback, static_cast<const __nv_bfloat16*>(v.rope), v.rope_ld, v.rope_bstride, qt, idx, count, cap,
+      append, kth, bitmap, (long long)nw, status);
   count_launches(1);
   return cudaGetLastError();
 }

@@ -12,6 +12,7 @@
 #include <algorithm>
 
 #include "vk_common.cuh"
+#include "vk_score_tc.h"
 
 namespace vk {
 thread_local int64_t g_launches = 0;
@@ -44,7 +45,7 @@ int cuda_fail(cudaError_t e, const char* where) {
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
 constexpr int64_t MAX_N = (1 << 24) - 1;
-constexpr int NUM_SMS_TARGET = 152;   // GB300: splits are sized for 2 CTAs per SM
+constexpr int NUM_SMS_TARGET = 152;   // GB300 SMs; attention splits are sized in whole waves
 
 int check_view(const vk_view* v) {
   if (!v) return fail(VK_ERR_INVALID_ARG, "view is NULL");
@@ -105,21 +106,44 @@ int check_index(const vk_view* v, const vk_params* p, const vk_index* ix, bool n
 
 size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
-// Positions per attention split: enough CTAs to fill the GPU twice over, within the shared-memory budget.
+// Positions per attention split. One attention CTA is resident per SM, so the split count is chosen to fill
+// the 152 SMs in whole waves: maximise (work) / (waves x 152 x positions per CTA), preferring longer splits
+// (fewer partials to merge) when two counts are equally good.
 void choose_splits(const vk_view& v, int64_t* nsplit, int64_t* split_len) {
-  const int64_t n_hg = (v.H + vk::HG - 1) / vk::HG;
-  const int64_t esz = v.dtype == VK_BF16 ? 2 : 4;
-  const int64_t fixed = (std::min<int64_t>(v.H, vk::HG) + 32) * (vk::D_LAT + vk::D_ROPE) * esz + 1024;
-  int64_t max_len = (vk::SMEM_BUDGET - fixed) / 12 / 32 * 32;
-  max_len = std::max<int64_t>(32, std::min<int64_t>(max_len, vk::SPLIT_MAX));
-  const int64_t min_splits = (v.N + max_len - 1) / max_len;
-  const int64_t target = (2 * NUM_SMS_TARGET + v.B * n_hg - 1) / (v.B * n_hg);
-  const int64_t cap_by_len = (v.N + 255) / 256;
-  int64_t ns = std::max<int64_t>(min_splits, std::min<int64_t>(target, cap_by_len));
-  ns = std::max<int64_t>(1, ns);
-  int64_t len = ((v.N + ns - 1) / ns + 31) / 32 * 32;
-  *split_len = len;
-  *nsplit = (v.N + len - 1) / len;
+  const int64_t per_pos = (int64_t)v.B * ((v.H + vk::HG - 1) / vk::HG);
+  const int64_t N = v.N;
+  const int64_t lo = std::max<int64_t>(1, (N + 16383) / 16384);
+  const int64_t hi = std::max<int64_t>(lo, std::min<int64_t>((N + 255) / 256, 2048));
+  double best = -1.0;
+  int64_t best_len = ((N + 31) / 32) * 32;
+  for (int64_t ns = lo; ns <= hi; ++ns) {
+    const int64_t len = ((N + ns - 1) / ns + 31) / 32 * 32;
+    const int64_t ns_eff = (N + len - 1) / len;
+    const int64_t ctas = per_pos * ns_eff;
+    const int64_t waves = (ctas + NUM_SMS_TARGET - 1) / NUM_SMS_TARGET;
+    const double eff = (double)(per_pos * N) / ((double)waves * NUM_SMS_TARGET * len);
+    if (eff > best + 1e-9) { best = eff; best_len = len; }
+  }
+  *split_len = best_len;
+  *nsplit = (N + best_len - 1) / best_len;
+}
+
+// Fused selection parameters: a strided sample of about 2048+ archive rows per head gives theta = its j-th
+// largest score, with j chosen so that ~1.5 k + 8 samples' worth of archive rows pass; the candidate list has
+// room for twice that (+2048) before the exact fallback takes over.
+void fused_params(int64_t N, int64_t lo, int64_t hi, int64_t k, VkLayout* L) {
+  const int64_t A = std::max<int64_t>(0, hi - lo);
+  L->ss = A >= 32768 ? 16 : std::max<int64_t>(1, A / 2048);
+  L->soff = L->ss / 2;
+  L->ns = N > L->soff ? (N - L->soff + L->ss - 1) / L->ss : 0;
+  int64_t n_arch = 0;                      // sampled rows inside the archive
+  for (int64_t i = 0; i < L->ns; ++i) {
+    const int64_t u = L->soff + L->ss * i;
+    n_arch += (u >= lo && u < hi);
+  }
+  L->j = n_arch ? (int64_t)std::ceil(1.5 * (double)k * (double)n_arch / (double)A) + 8 : 0;
+  const int64_t expect = n_arch ? (int64_t)std::ceil((double)std::min(L->j, n_arch) * (double)A / (double)n_arch) : 0;
+  L->capc = std::max<int64_t>(std::min<int64_t>(A, 2 * expect + 2048), std::max<int64_t>(k, 1));
 }
 
 VkLayout make_layout(const vk_view& v, const vk_params& p) {
@@ -129,7 +153,13 @@ VkLayout make_layout(const vk_view& v, const vk_params& p) {
   L.n_hg = (v.H + vk::HG - 1) / vk::HG;
   choose_splits(v, &L.nsplit, &L.split_len);
   L.two_tier = p.trigger != VK_TRIG_OFF;
-  L.dense_scores = true;
+  L.tc = vk::score_tc_supported(v, p.r);
+  L.fused = L.tc && !(p.flags & VK_FLAG_FORCE_DENSE);
+  L.dense_scores = !L.fused;
+  const int64_t lo = p.n_sink, hi = (int64_t)v.N - p.window;
+  const int64_t k = keep_count(v.N, p.rho, p.window, p.n_sink);
+  if (L.fused) fused_params(v.N, lo, hi, k, &L);
+  L.fcap = (L.fused && L.two_tier && p.top_j > 0) ? std::max<int64_t>(1, hi - lo) : 0;
   const int64_t BH = (int64_t)v.B * v.H;
   const int64_t nslot = L.nsplit * (L.two_tier ? 2 : 1);
   size_t off = 0;
@@ -145,6 +175,12 @@ VkLayout make_layout(const vk_view& v, const vk_params& p) {
   L.off_firebm = take(L.two_tier ? sizeof(uint32_t) * BH * L.nw : 0);
   L.off_part_o = take(sizeof(float) * v.B * nslot * v.H * vk::D_LAT);
   L.off_part_ml = take(sizeof(float) * v.B * nslot * v.H * 2);
+  L.off_sample = take(L.fused ? sizeof(float) * BH * L.ns : 0);
+  L.off_theta = take(L.fused ? sizeof(float) * BH : 0);
+  L.off_ccnt = take(L.fused ? sizeof(int) * BH : 0);
+  L.off_cand = take(L.fused ? sizeof(int2) * BH * L.capc : 0);
+  L.off_fcnt = take(L.fcap ? sizeof(int) * BH : 0);
+  L.off_fcand = take(L.fcap ? sizeof(int2) * BH * L.fcap : 0);
   L.total = off;
   return L;
 }
@@ -238,6 +274,15 @@ int vk_score(const vk_view* view, const vk_params* params, const vk_index* index
   if ((rc = check_ws(L, ws, ws_bytes)) != VK_OK) return rc;
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   float* qt = at<float>(ws, L.off_qt);
+  if (L.tc) {
+    vk::ScoreTcArgs a{};
+    a.mode = 0;
+    a.scores = scores;
+    a.scores_ld = view->N;
+    a.status = at<int>(ws, L.off_status);
+    VK_CUDA(vk::launch_score_tc(*view, 0, 1, view->N, a, st), "score (tcgen05)");
+    return VK_OK;
+  }
   VK_CUDA(vk::launch_qprep(*view, params->r, index ? index->rot : nullptr, qt, at<float>(ws, L.off_qcn),
                            at<float>(ws, L.off_qrn), st), "qprep");
   VK_CUDA(vk::launch_score_simt(*view, params->r, qt,
@@ -281,8 +326,8 @@ int vk_sparse_attn(const vk_view* view, const vk_params* params, const int32_t* 
   float* po = at<float>(ws, L.off_part_o);
   float* pml = at<float>(ws, L.off_part_ml);
   VK_CUDA(vk::launch_list_to_bitmap(view->B, view->H, view->N, idx, count, cap, bm, L.nw, status, st), "list_to_bitmap");
-  VK_CUDA(vk::launch_attn(*view, params->sm_scale, bm, L.nw, (int)L.nsplit, (int)L.split_len, 0, (int)L.nsplit, po, pml, st),
-          "attention");
+  VK_CUDA(vk::launch_attn(*view, params->sm_scale, bm, L.nw, (int)L.nsplit, (int)L.split_len, 0, (int)L.nsplit, po, pml,
+                          status, st), "attention");
   VK_CUDA(vk::launch_combine(view->B, view->H, (int)L.nsplit, (int)L.nsplit, po, pml, out, lse, smax, st), "combine");
   return VK_OK;
 }
@@ -315,31 +360,107 @@ int vk_decode_step(const vk_view* view, const vk_params* params, const vk_index*
   float* pml = at<float>(ws, L.off_part_ml);
   const int ns = (int)L.nsplit, nslot = two_tier ? 2 * ns : ns;
 
+  const int lo = S, hi = N - W;
   prof(0, st);
   VK_CUDA(vk::launch_qprep(v, params->r, index ? index->rot : nullptr, qt, qcn, qrn, st), "qprep");
   prof(1, st);
-  VK_CUDA(vk::launch_score_simt(v, params->r, qt, static_cast<const __nv_bfloat16*>(index ? index->digest : nullptr),
-                                scores, st), "score");
-  prof(2, st);
-  VK_CUDA(vk::launch_select_dense(B, H, N, scores, nullptr, k, W, S, idx, count, cap, 0, nullptr, selbm, L.nw, status, st),
-          "select");
+  if (L.fused) {
+    // threshold from a strided sample, then one scoring pass that keeps only the rows above it
+    float* sample = at<float>(ws, L.off_sample);
+    float* theta = at<float>(ws, L.off_theta);
+    int* ccnt = at<int>(ws, L.off_ccnt);
+    int2* cand = at<int2>(ws, L.off_cand);
+    VK_CUDA(cudaMemsetAsync(ccnt, 0, sizeof(int) * B * H, st), "candidate counts");
+    if (k > 0) {
+      vk::ScoreTcArgs a{};
+      a.mode = 0;
+      a.scores = sample;
+      a.scores_ld = L.ns;
+      a.status = status;
+      VK_CUDA(vk::launch_score_tc(v, (int)L.soff, (int)L.ss, (int)L.ns, a, st), "sample scores");
+      VK_CUDA(vk::launch_theta(B, H, (int)L.ns, (int)L.soff, (int)L.ss, lo, hi, (int)L.j, sample, theta, st), "theta");
+      vk::ScoreTcArgs c{};
+      c.mode = 1;
+      c.theta = theta;
+      c.arch_lo = lo;
+      c.arch_hi = hi;
+      c.cand_cnt = ccnt;
+      c.cand = cand;
+      c.capc = (int)L.capc;
+      c.status = status;
+      VK_CUDA(vk::launch_score_tc(v, 0, 1, N, c, st), "score (candidates)");
+    }
+    prof(2, st);
+    VK_CUDA(vk::launch_select_cand(B, H, N, lo, hi, k, nullptr, ccnt, cand, (int)L.capc,
+                                   (params->flags & VK_FLAG_FORCE_FALLBACK) ? 1 : 0, v, qt, idx, count, cap, 0, nullptr,
+                                   selbm, L.nw, status, st), "select (candidates)");
+  } else {
+    if (L.tc) {
+      vk::ScoreTcArgs a{};
+      a.mode = 0;
+      a.scores = scores;
+      a.scores_ld = N;
+      a.status = status;
+      VK_CUDA(vk::launch_score_tc(v, 0, 1, N, a, st), "score (tcgen05)");
+    } else {
+      VK_CUDA(vk::launch_score_simt(v, params->r, qt, static_cast<const __nv_bfloat16*>(index ? index->digest : nullptr),
+                                    scores, st), "score");
+    }
+    prof(2, st);
+    VK_CUDA(vk::launch_select_dense(B, H, N, scores, nullptr, k, W, S, idx, count, cap, 0, nullptr, selbm, L.nw, status, st),
+            "select");
+  }
   prof(3, st);
-  VK_CUDA(vk::launch_attn(v, params->sm_scale, selbm, L.nw, ns, (int)L.split_len, 0, nslot, po, pml, st), "attention");
+  VK_CUDA(vk::launch_attn(v, params->sm_scale, selbm, L.nw, ns, (int)L.split_len, 0, nslot, po, pml, status, st),
+          "attention");
   prof(4, st);
   if (two_tier) {
     float* smax1 = at<float>(ws, L.off_smax1);
     int64_t* nfired = at<int64_t>(ws, L.off_nfired);
     uint32_t* firebm = at<uint32_t>(ws, L.off_firebm);
     VK_CUDA(vk::launch_smax_reduce(B, H, ns, nslot, pml, smax1, st), "smax");
-    VK_CUDA(vk::launch_trigger_dense(B, H, N, W, S, params->sm_scale, params->z_eff, params->top_j, scores, qcn, qrn,
-                                     index->eta, index->page_res, smax1, selbm, firebm, L.nw, nfired, st), "trigger");
-    if (params->top_j > 0) {
-      VK_CUDA(vk::launch_select_dense(B, H, N, scores, nfired, params->top_j, 0, 0, idx, count, cap, 1, nullptr, firebm,
-                                      L.nw, status, st), "top_j");
+    if (L.fused) {
+      vk::ScoreTcArgs t{};
+      t.mode = 2;
+      t.arch_lo = lo;
+      t.arch_hi = hi;
+      t.qcn = qcn;
+      t.qrn = qrn;
+      t.eta = index->eta;
+      t.page_res = index->page_res;
+      t.smax1 = smax1;
+      t.lam = params->sm_scale;
+      t.z = params->z_eff;
+      t.selbm = selbm;
+      t.firebm = firebm;
+      t.nw = L.nw;
+      t.top_j = params->top_j;
+      t.status = status;
+      if (params->top_j > 0) {
+        int* fcnt = at<int>(ws, L.off_fcnt);
+        int2* fcand = at<int2>(ws, L.off_fcand);
+        VK_CUDA(cudaMemsetAsync(fcnt, 0, sizeof(int) * B * H, st), "fired counts");
+        t.cand_cnt = fcnt;
+        t.cand = fcand;
+        t.capc = (int)L.fcap;
+        VK_CUDA(vk::launch_score_tc(v, 0, 1, N, t, st), "trigger (candidates)");
+        VK_CUDA(vk::launch_select_cand(B, H, N, lo, hi, params->top_j, nullptr, fcnt, fcand, (int)L.fcap, 0, v, qt, idx,
+                                       count, cap, 1, nullptr, firebm, L.nw, status, st), "top_j");
+      } else {
+        VK_CUDA(vk::launch_score_tc(v, 0, 1, N, t, st), "trigger");
+        VK_CUDA(vk::launch_bitmap_to_list(B, H, N, firebm, L.nw, idx, count, cap, status, st), "fired list");
+      }
     } else {
-      VK_CUDA(vk::launch_bitmap_to_list(B, H, N, firebm, L.nw, idx, count, cap, status, st), "fired list");
+      VK_CUDA(vk::launch_trigger_dense(B, H, N, W, S, params->sm_scale, params->z_eff, params->top_j, scores, qcn, qrn,
+                                       index->eta, index->page_res, smax1, selbm, firebm, L.nw, nfired, st), "trigger");
+      if (params->top_j > 0) {
+        VK_CUDA(vk::launch_select_dense(B, H, N, scores, nfired, params->top_j, 0, 0, idx, count, cap, 1, nullptr, firebm,
+                                        L.nw, status, st), "top_j");
+      } else {
+        VK_CUDA(vk::launch_bitmap_to_list(B, H, N, firebm, L.nw, idx, count, cap, status, st), "fired list");
+      }
     }
-    VK_CUDA(vk::launch_attn(v, params->sm_scale, firebm, L.nw, ns, (int)L.split_len, ns, nslot, po, pml, st),
+    VK_CUDA(vk::launch_attn(v, params->sm_scale, firebm, L.nw, ns, (int)L.split_len, ns, nslot, po, pml, status, st),
             "fired attention");
   }
   prof(5, st);

