@@ -5,10 +5,12 @@
 // 128-row tiles:
 //   warp 0 (one thread)  TMA: the tile's 128 x 64 bf16 slice (128 B of every 1152-B row, 128-byte swizzle)
 //                        into an 8-stage ring, and the sequence's H x 64 query when the sequence changes;
-//   warp 1 (one thread)  tcgen05.mma M=128, N=H, K=16 (x4) into a double-buffered fp32 accumulator in tensor
-//                        memory (128 lanes = rows, H columns = heads); tcgen05.commit frees the ring slot and
-//                        hands the accumulator to the epilogue;
-//   warps 2..5           epilogue: tcgen05.ld of 32 heads at a time, one thread per row, then
+//   warp 1 (one thread)  tcgen05.mma M=128, N=H, K=16 (x4) into one of G fp32 accumulators in tensor memory
+//                        (128 lanes = rows, H columns = heads); tcgen05.commit frees the ring slot and hands the
+//                        accumulator to the epilogue group that owns it;
+//   G groups of 4 warps  epilogue, group g taking tiles i = g (mod G), so G tiles are in flight at once (the
+//                        candidate epilogue waits on global atomics): tcgen05.ld of 32 heads at a time, one
+//                        thread per row, then
 //                        mode 0  write fp32 scores [B][H][ld] (also used on a strided row sample),
 //                        mode 1  emit (u, a) for archive rows with a >= theta[b,h] into per-head candidate lists,
 //                        mode 2  trigger: T = lambda (a + |(O Qr)[r:]| page_res + z |Qc| eta) > s*_h for archive
@@ -27,9 +29,8 @@ namespace vk {
 
 constexpr int TC_M = 128;                    // rows per tile (MMA M)
 constexpr int TC_STAGES = 8;
-constexpr int TC_EPI = 4;                    // epilogue warps, one per TMEM lane quarter
-constexpr int TC_THREADS = (2 + TC_EPI) * 32;
 constexpr uint32_t TC_TILE_BYTES = TC_M * 128;   // 128 rows x 64 bf16
+constexpr int TC_MAX_G = 4;                  // epilogue groups (accumulator buffers)
 
 __device__ __forceinline__ void tma_load_3d(void* dst, const CUtensorMap* map, int x, int y, int z, uint64_t* bar) {
   asm volatile(
@@ -93,14 +94,15 @@ struct TcSmem {
     a = 0;                                              // TC_STAGES x 16 KB (1024-aligned)
     q = a + TC_STAGES * TC_TILE_BYTES;                  // 2 x H x 128 B
     bars = q + 2 * H * 128;                             // 8-byte barriers
-    params = bars + (2 * TC_STAGES + 6) * 8;            // 2 x 4 x H floats of per-sequence parameters
-    total = params + 2 * 4 * H * 4 + 1024;              // + slack to align the base to 1024
+    params = bars + (2 * TC_STAGES + 4 + 2 * TC_MAX_G) * 8;   // per group: 4 x H floats of per-sequence params
+    total = params + TC_MAX_G * 4 * H * 4 + 1024;       // + slack to align the base to 1024
   }
 };
 
-__global__ void __launch_bounds__(TC_THREADS, 1) k_score_tc(const __grid_constant__ CUtensorMap kmap,
-                                                            const __grid_constant__ CUtensorMap qmap,
-                                                            const ScoreTcArgs args) {
+template <int G>
+__global__ void __launch_bounds__((2 + 4 * G) * 32, 1) k_score_tc(const __grid_constant__ CUtensorMap kmap,
+                                                                const __grid_constant__ CUtensorMap qmap,
+                                                                const ScoreTcArgs args) {
   extern __shared__ __align__(1024) unsigned char smem_raw[];
   unsigned char* smem = reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   const int H = args.H;
@@ -112,9 +114,9 @@ __global__ void __launch_bounds__(TC_THREADS, 1) k_score_tc(const __grid_constan
   uint64_t* a_empty = bars + TC_STAGES;
   uint64_t* q_full = bars + 2 * TC_STAGES;              // [2]
   uint64_t* q_empty = q_full + 2;                        // [2]
-  uint64_t* d_full = q_empty + 2;                        // [2]
-  uint64_t* d_empty = d_full + 2;                        // [2]
-  float* sparams = reinterpret_cast<float*>(smem + Ls.params);   // [2 slots][4][H]
+  uint64_t* d_full = q_empty + 2;                        // [G]
+  uint64_t* d_empty = d_full + G;                        // [G]
+  float* sparams = reinterpret_cast<float*>(smem + Ls.params);   // [G groups][4][H]
   __shared__ uint32_t tmem_base;
   __shared__ int abort_flag;
 
@@ -130,10 +132,8 @@ __global__ void __launch_bounds__(TC_THREADS, 1) k_score_tc(const __grid_constan
   if (threadIdx.x == 0) {
     abort_flag = 0;
     for (int s = 0; s < TC_STAGES; ++s) { mbar_init(&a_full[s], 1); mbar_init(&a_empty[s], 1); }
-    for (int i = 0; i < 2; ++i) {
-      mbar_init(&q_full[i], 1); mbar_init(&q_empty[i], 1);
-      mbar_init(&d_full[i], 1); mbar_init(&d_empty[i], TC_EPI);
-    }
+    for (int i = 0; i < 2; ++i) { mbar_init(&q_full[i], 1); mbar_init(&q_empty[i], 1); }
+    for (int i = 0; i < G; ++i) { mbar_init(&d_full[i], 1); mbar_init(&d_empty[i], 4); }
     mbar_fence_init();
   }
   if (warp == 1) tmem_alloc(&tmem_base, args.tmem_cols);
@@ -175,7 +175,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1) k_score_tc(const __grid_constan
           prev_b = b;
         }
         const int s = i % TC_STAGES, use = i / TC_STAGES;
-        const int ds = i & 1, duse = i >> 1;
+        const int ds = i % G, duse = i / G;
         if (!mbar_wait(&a_full[s], use & 1, &abort_flag)) { abort_flag = 1; break; }
         if (duse > 0 && !mbar_wait(&d_empty[ds], (duse - 1) & 1, &abort_flag)) { abort_flag = 1; break; }
         tmem_fence_after();
@@ -191,18 +191,18 @@ __global__ void __launch_bounds__(TC_THREADS, 1) k_score_tc(const __grid_constan
     }
   } else {
     // ------------------------------------------------------------------ epilogue
-    const int quarter = warp & 3;
-    const int ew = warp - 2;                              // 0..TC_EPI-1
+    const int ew = warp - 2;                              // 0 .. 4G-1
+    const int g = ew >> 2;                                // group: tiles i = g (mod G), accumulator g
+    const int quarter = warp & 3;                         // TMEM lane quarter = the warp's 32 rows of the tile
+    float* prm = sparams + g * 4 * H;
     int prev_b = -1;
-    for (int i = 0; i < n; ++i) {
+    for (int i = g; i < n; i += G) {
       const int64_t t = t0 + i;
       const int b = (int)(t / tps), row0 = (int)(t % tps) * TC_M;
-      const int qi = (b - b_first) & 1;
-      float* prm = sparams + qi * 4 * H;
       if (b != prev_b) {
-        // per-sequence parameters -> shared memory (all epilogue threads, then a barrier among them)
-        named_barrier(2, TC_EPI * 32);
-        for (int h = ew * 32 + lane; h < H; h += TC_EPI * 32) {
+        // per-sequence parameters -> this group's shared-memory slot (the group's 4 warps, then a barrier)
+        named_barrier(2 + g, 128);
+        for (int h = (ew & 3) * 32 + lane; h < H; h += 128) {
           if (args.mode == 1) {
             prm[h] = args.theta[(int64_t)b * H + h];
           } else if (args.mode == 2) {
@@ -211,11 +211,11 @@ __global__ void __launch_bounds__(TC_THREADS, 1) k_score_tc(const __grid_constan
             prm[2 * H + h] = args.qrn[(int64_t)b * H + h];
           }
         }
-        named_barrier(2, TC_EPI * 32);
+        named_barrier(2 + g, 128);
         prev_b = b;
       }
-      const int ds = i & 1, duse = i >> 1;
-      if (!mbar_wait(&d_full[ds], duse & 1, &abort_flag)) {
+      const int duse = i / G;
+      if (!mbar_wait(&d_full[g], duse & 1, &abort_flag)) {
         if (lane == 0) { raise_status(args.status, VK_ERR_TIMEOUT); abort_flag = 1; }
         break;
       }
@@ -223,8 +223,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1) k_score_tc(const __grid_constan
       const int row = row0 + quarter * 32 + lane;          // row of the tensor map (position, or sample index)
       const bool in_rows = row < args.n_rows;
       const int64_t bh0 = (int64_t)b * H;
-      const uint32_t tbase = tmem_base + ((uint32_t)(quarter * 32) << 16) + ds * dcols;
-      // mode-specific per-row quantities
+      const uint32_t tbase = tmem_base + ((uint32_t)(quarter * 32) << 16) + g * dcols;
       bool arch = false;
       float row_add = 0.f, row_eta = 0.f;
       if (args.mode >= 1) arch = in_rows && row >= args.arch_lo && row < args.arch_hi;
@@ -234,51 +233,78 @@ __global__ void __launch_bounds__(TC_THREADS, 1) k_score_tc(const __grid_constan
       }
       const int64_t word = (row0 + quarter * 32) / 32;      // this warp's 32 rows = one bitmap word
       const bool word_ok = word < args.nw;
-      for (int c = 0; c < H; c += 32) {
-        float v[32];
+      const bool emit = args.mode == 1 || (args.mode == 2 && args.top_j > 0);
+      constexpr int NCH = G == 4 ? 4 : 8;                  // 32-head chunks (H <= 128 when G = 4)
+      uint32_t mine[NCH];                                  // ballot of head c + lane, per 32-head chunk
+      int base[NCH];
+#pragma unroll
+      for (int cc = 0; cc < NCH; ++cc) {
+        const int c = cc * 32;
+        if (c >= H) break;
         const int hn = min(32, H - c);                     // 32, or 16 for the last chunk when H % 32 == 16
-        if (hn == 32) tmem_ld32(tbase + c, v); else tmem_ld16(tbase + c, v);
-        tmem_wait_ld();
-        if (args.mode == 0) {
-          if (in_rows) {
+        uint32_t sel_word = 0;
+        if (args.mode == 2 && lane < hn && word_ok) sel_word = args.selbm[(bh0 + c + lane) * args.nw + word];
+        uint32_t m_lane = 0;
 #pragma unroll
-            for (int j = 0; j < 32; ++j)
-              if (j < hn) args.scores[(bh0 + c + j) * args.scores_ld + row] = v[j];
+        for (int half = 0; half < 2; ++half) {
+          if (16 * half >= hn) break;
+          float v[16];
+          tmem_ld16(tbase + c + 16 * half, v);
+          tmem_wait_ld();
+          if (args.mode == 0) {
+            if (in_rows) {
+#pragma unroll
+              for (int j = 0; j < 16; ++j) args.scores[(bh0 + c + 16 * half + j) * args.scores_ld + row] = v[j];
+            }
+            continue;
           }
-        } else {
-          // one 32-bit ballot per head: bit `lane` = this row passes the head's test
-          uint32_t sel_word = 0;
-          if (args.mode == 2 && lane < hn && word_ok) sel_word = args.selbm[(bh0 + c + lane) * args.nw + word];
-          uint32_t mine = 0;                               // ballot of head c + lane
 #pragma unroll
-          for (int j = 0; j < 32; ++j) {
+          for (int jj = 0; jj < 16; ++jj) {
+            const int j = 16 * half + jj;
             bool pass = false;
             if (args.mode == 1) {
-              pass = arch && v[j] >= prm[c + j];
+              pass = arch && v[jj] >= prm[c + j];
             } else {
               const uint32_t sw = __shfl_sync(0xffffffffu, sel_word, j);
-              const float T = args.lam * (v[j] + prm[2 * H + c + j] * row_add + prm[H + c + j] * row_eta);
-              v[j] = T;
+              const float T = args.lam * (v[jj] + prm[2 * H + c + j] * row_add + prm[H + c + j] * row_eta);
               pass = arch && !((sw >> lane) & 1u) && T > prm[c + j];
             }
-            const uint32_t m = __ballot_sync(0xffffffffu, pass && j < hn);
-            if (lane == j) mine = m;
+            const uint32_t m = __ballot_sync(0xffffffffu, pass);
+            if (lane == j) m_lane = m;
           }
-          if (args.mode == 2 && args.top_j == 0) {
-            if (lane < hn && word_ok) args.firebm[(bh0 + c + lane) * args.nw + word] = mine;
-          } else {
-            // reserve room in the heads' candidate lists, then scatter (u, score)
-            const int cnt = __popc(mine);
-            int base = 0;
-            if (cnt) base = atomicAdd(&args.cand_cnt[bh0 + c + lane], cnt);
+        }
+        mine[cc] = m_lane;
+        if (args.mode == 2 && !emit && lane < hn && word_ok) args.firebm[(bh0 + c + lane) * args.nw + word] = m_lane;
+      }
+      if (emit) {
+        // reserve room for every chunk first (the atomics overlap), then read the scores again and scatter
 #pragma unroll
-            for (int j = 0; j < 32; ++j) {
-              const uint32_t m = __shfl_sync(0xffffffffu, mine, j);
-              const int bj = __shfl_sync(0xffffffffu, base, j);
+        for (int cc = 0; cc < NCH; ++cc) {
+          if (cc * 32 >= H) break;
+          const int cnt = __popc(mine[cc]);
+          base[cc] = cnt ? atomicAdd(&args.cand_cnt[bh0 + cc * 32 + lane], cnt) : 0;
+        }
+#pragma unroll
+        for (int cc = 0; cc < NCH; ++cc) {
+          const int c = cc * 32;
+          if (c >= H) break;
+          const int hn = min(32, H - c);
+#pragma unroll
+          for (int half = 0; half < 2; ++half) {
+            if (16 * half >= hn) break;
+            float v[16];
+            tmem_ld16(tbase + c + 16 * half, v);
+            tmem_wait_ld();
+#pragma unroll
+            for (int jj = 0; jj < 16; ++jj) {
+              const int j = 16 * half + jj;
+              const uint32_t m = __shfl_sync(0xffffffffu, mine[cc], j);
+              const int bj = __shfl_sync(0xffffffffu, base[cc], j);
               if ((m >> lane) & 1u) {
                 const int pos = bj + __popc(m & ((1u << lane) - 1u));
-                if (pos < args.capc)
-                  args.cand[(bh0 + c + j) * args.capc + pos] = make_int2(row, __float_as_int(v[j]));
+                float val = v[jj];
+                if (args.mode == 2) val = args.lam * (v[jj] + prm[2 * H + c + j] * row_add + prm[H + c + j] * row_eta);
+                if (pos < args.capc) args.cand[(bh0 + c + j) * args.capc + pos] = make_int2(row, __float_as_int(val));
               }
             }
           }
@@ -286,7 +312,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1) k_score_tc(const __grid_constan
       }
       tmem_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive(&d_empty[ds]);
+      if (lane == 0) mbar_arrive(&d_empty[g]);
     }
   }
 
@@ -345,17 +371,23 @@ cudaError_t launch_score_tc(const vk_view& v, int row_offset, int row_stride, in
   args.tiles_per_seq = (n_rows + TC_M - 1) / TC_M;
   args.total_tiles = (int64_t)args.tiles_per_seq * v.B;
   args.n_pages = (v.N + PAGE - 1) / PAGE;
+  const int G = v.H <= 128 ? 4 : 2;                   // G accumulators of H columns fit in 512 TMEM columns
   uint32_t cols = 32;
-  while (cols < 2u * v.H) cols <<= 1;
+  while (cols < (uint32_t)(G * v.H)) cols <<= 1;
   args.tmem_cols = cols;
   const int grid = (int)std::min<int64_t>(args.total_tiles, 152);
   const size_t smem = TcSmem(v.H).total;
-  cudaError_t e = cudaFuncSetAttribute(k_score_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-  if (e != cudaSuccess) return e;
-  if (grid > 0) {
-    k_score_tc<<<grid, TC_THREADS, smem, st>>>(kmap, qmap, args);
-    count_launches(1);
+  cudaError_t e;
+  if (G == 4) {
+    e = cudaFuncSetAttribute(k_score_tc<4>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    if (grid > 0) k_score_tc<4><<<grid, (2 + 4 * 4) * 32, smem, st>>>(kmap, qmap, args);
+  } else {
+    e = cudaFuncSetAttribute(k_score_tc<2>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    if (grid > 0) k_score_tc<2><<<grid, (2 + 4 * 2) * 32, smem, st>>>(kmap, qmap, args);
   }
+  if (grid > 0) count_launches(1);
   return cudaGetLastError();
 }
 

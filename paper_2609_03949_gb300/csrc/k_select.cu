@@ -10,6 +10,72 @@
 namespace vk {
 
 constexpr int SEL_THREADS = 512;
+constexpr int CAND_THREADS = 256;
+
+// Radix-select step over a 256-bin histogram, run by one full warp: the largest digit d with
+// (count of bins above d) < need <= (count of bins at or above d). Lane l owns bins 255 - 8l .. 248 - 8l.
+// Writes d and the count above it to *d_out / *above_out (digit 0 if fewer than `need` keys remain).
+__device__ __forceinline__ void pick_digit_desc(const unsigned int* hist, unsigned int need, unsigned int* d_out,
+                                                unsigned int* above_out, unsigned int* count_out) {
+  const int lane = threadIdx.x & 31;
+  unsigned int v[8], sum = 0;
+#pragma unroll
+  for (int i = 0; i < 8; ++i) { v[i] = hist[255 - 8 * lane - i]; sum += v[i]; }
+  unsigned int incl = sum;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const unsigned int t = __shfl_up_sync(0xffffffffu, incl, o);
+    if (lane >= o) incl += t;
+  }
+  const unsigned int excl = incl - sum;
+  const unsigned int hit = __ballot_sync(0xffffffffu, excl < need && need <= incl);
+  const int src = hit ? __ffs(hit) - 1 : 31;
+  if (lane == src) {
+    unsigned int acc = excl, d = 255 - 8 * lane - 7, cnt = v[7];
+    if (hit) {
+#pragma unroll
+      for (int i = 0; i < 8; ++i) {
+        if (acc + v[i] >= need) { d = 255 - 8 * lane - i; cnt = v[i]; break; }
+        acc += v[i];
+      }
+    } else {
+      acc = incl - v[7];
+    }
+    *d_out = d;
+    *above_out = acc;
+    if (count_out) *count_out = cnt;
+  }
+}
+
+// Same, ascending: the smallest digit d with (count below d) < need <= (count at or below d).
+__device__ __forceinline__ void pick_digit_asc(const unsigned int* hist, unsigned int need, unsigned int* d_out,
+                                               unsigned int* below_out) {
+  const int lane = threadIdx.x & 31;
+  unsigned int v[8], sum = 0;
+#pragma unroll
+  for (int i = 0; i < 8; ++i) { v[i] = hist[8 * lane + i]; sum += v[i]; }
+  unsigned int incl = sum;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const unsigned int t = __shfl_up_sync(0xffffffffu, incl, o);
+    if (lane >= o) incl += t;
+  }
+  const unsigned int excl = incl - sum;
+  const unsigned int hit = __ballot_sync(0xffffffffu, excl < need && need <= incl);
+  const int src = hit ? __ffs(hit) - 1 : 0;
+  if (lane == src) {
+    unsigned int acc = excl, d = 8 * lane;
+    if (hit) {
+#pragma unroll
+      for (int i = 0; i < 8; ++i) {
+        if (acc + v[i] >= need) { d = 8 * lane + i; break; }
+        acc += v[i];
+      }
+    }
+    *d_out = d;
+    *below_out = acc;
+  }
+}
 
 // Key sources for the ordered selection: scores stored in memory, or recomputed from the RoPE columns
 // (the exact fallback of the fused path: a[u] = qt . K_u in fp32, qt already in shared memory).
@@ -43,7 +109,7 @@ template <class Keys>
 __device__ void select_ordered(const Keys& key_of, int N, int lo, int hi, long long k, int32_t* out, int32_t* count_bh,
                                int cap, int append, float* kth_bh, uint32_t* bitmap_bh, long long nw, int* status) {
   __shared__ unsigned int hist[256];
-  __shared__ unsigned int s_prefix, s_need;
+  __shared__ unsigned int s_prefix, s_need, s_digit, s_above, s_cnt;
   __shared__ int scan_scratch[33];
   unsigned int prefix = 0, mask = 0, need = (unsigned int)k;
   if (k > 0) {
@@ -55,15 +121,11 @@ __device__ void select_ordered(const Keys& key_of, int N, int lo, int hi, long l
         if ((key & mask) == prefix) atomicAdd(&hist[(key >> shift) & 255u], 1u);
       }
       __syncthreads();
+      if (threadIdx.x < 32) pick_digit_desc(hist, need, &s_digit, &s_above, nullptr);
+      __syncthreads();
       if (threadIdx.x == 0) {
-        unsigned int above = 0;
-        int d = 255;
-        for (; d > 0; --d) {
-          if (above + hist[d] >= need) break;
-          above += hist[d];
-        }
-        s_prefix = prefix | ((unsigned int)d << shift);
-        s_need = need - above;
+        s_prefix = prefix | (s_digit << shift);
+        s_need = need - s_above;
       }
       __syncthreads();
       prefix = s_prefix;
@@ -137,48 +199,39 @@ cudaError_t launch_select_dense(int B, int H, int N, const float* scores, const 
 // Threshold from a strided sample of the archive: theta[b,h] = the j-th largest sampled score, so that about
 // j * stride archive rows score >= theta (chosen well above k). The candidate pass then emits only those rows.
 // sample[(b*H + h) * ns + i] is the score of position off + stride * i.
-__global__ void __launch_bounds__(SEL_THREADS) k_theta(int ns, int off, int stride, int lo, int hi, int j,
-                                                       const float* __restrict__ sample, float* __restrict__ theta) {
+__global__ void __launch_bounds__(CAND_THREADS) k_theta(int ns, int off, int stride, int lo, int hi, int j,
+                                                        const float* __restrict__ sample, float* __restrict__ theta) {
+  extern __shared__ __align__(16) unsigned char smem[];
+  uint32_t* keys = reinterpret_cast<uint32_t*>(smem);         // the archive samples' keys, [n_arch]
   __shared__ unsigned int hist[256];
-  __shared__ unsigned int s_prefix, s_need;
+  __shared__ unsigned int s_digit, s_above;
+  __shared__ int n_arch;
   const int64_t bh = blockIdx.x;
   const float* a = sample + bh * (int64_t)ns;
-  auto in_archive = [&](int i) { const int u = off + stride * i; return u >= lo && u < hi; };
-  unsigned int prefix = 0, mask = 0, need = (unsigned int)j;
-  // number of sampled archive rows
-  __shared__ int n_arch;
-  if (threadIdx.x == 0) n_arch = 0;
+  // sampled positions off + stride * i inside [lo, hi) are a contiguous index range [i0, i1)
+  const int i0 = lo > off ? (lo - off + stride - 1) / stride : 0;
+  const int i1 = min(ns, hi > off ? (hi - off + stride - 1) / stride : 0);
+  const int na = max(0, i1 - i0);
+  for (int i = threadIdx.x; i < na; i += blockDim.x) keys[i] = fkey(a[i0 + i]);
+  if (threadIdx.x == 0) n_arch = na;
   __syncthreads();
-  int local = 0;
-  for (int i = threadIdx.x; i < ns; i += blockDim.x) local += in_archive(i);
-  atomicAdd(&n_arch, local);
-  __syncthreads();
-  if (j <= 0 || j > n_arch) {
+  if (j <= 0 || j > na) {
     if (threadIdx.x == 0) theta[bh] = -INFINITY;      // emit every archive row
     return;
   }
+  unsigned int prefix = 0, mask = 0, need = (unsigned int)j;
   for (int shift = 24; shift >= 0; shift -= 8) {
     for (int i = threadIdx.x; i < 256; i += blockDim.x) hist[i] = 0;
     __syncthreads();
-    for (int i = threadIdx.x; i < ns; i += blockDim.x) {
-      if (!in_archive(i)) continue;
-      const uint32_t key = fkey(a[i]);
+    for (int i = threadIdx.x; i < na; i += blockDim.x) {
+      const uint32_t key = keys[i];
       if ((key & mask) == prefix) atomicAdd(&hist[(key >> shift) & 255u], 1u);
     }
     __syncthreads();
-    if (threadIdx.x == 0) {
-      unsigned int above = 0;
-      int d = 255;
-      for (; d > 0; --d) {
-        if (above + hist[d] >= need) break;
-        above += hist[d];
-      }
-      s_prefix = prefix | ((unsigned int)d << shift);
-      s_need = need - above;
-    }
+    if (threadIdx.x < 32) pick_digit_desc(hist, need, &s_digit, &s_above, nullptr);
     __syncthreads();
-    prefix = s_prefix;
-    need = s_need;
+    prefix |= s_digit << shift;
+    need -= s_above;
     mask |= 255u << shift;
     __syncthreads();
   }
@@ -187,7 +240,10 @@ __global__ void __launch_bounds__(SEL_THREADS) k_theta(int ns, int off, int stri
 
 cudaError_t launch_theta(int B, int H, int ns, int off, int stride, int lo, int hi, int j, const float* sample,
                          float* theta, cudaStream_t st) {
-  k_theta<<<B * H, SEL_THREADS, 0, st>>>(ns, off, stride, lo, hi, j, sample, theta);
+  const size_t smem = (size_t)ns * 4;
+  cudaError_t e = cudaFuncSetAttribute(k_theta, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (e != cudaSuccess) return e;
+  k_theta<<<B * H, CAND_THREADS, smem, st>>>(ns, off, stride, lo, hi, j, sample, theta);
   count_launches(1);
   return cudaGetLastError();
 }
@@ -200,7 +256,7 @@ cudaError_t launch_theta(int B, int H, int ns, int off, int stride, int lo, int 
 // (theta landed too high or too low) or with VK_FLAG_FORCE_FALLBACK, the head takes the exact ordered selection
 // over scores recomputed from the RoPE columns. With `append` (the top_j of the fired rows, whose list can never
 // overflow) only candidates are selected, no sinks or window, and the ids are appended after count[b,h].
-__global__ void __launch_bounds__(SEL_THREADS) k_select_cand(
+__global__ void __launch_bounds__(CAND_THREADS) k_select_cand(
     int H, int N, int lo, int hi, long long k_all, const long long* __restrict__ k_per_head,
     const int* __restrict__ cand_cnt, const int2* __restrict__ cand, int capc, int smem_cap, int force_fallback,
     const __nv_bfloat16* __restrict__ rope, int64_t rld, int64_t rbs, const float* __restrict__ qt,
@@ -210,7 +266,7 @@ __global__ void __launch_bounds__(SEL_THREADS) k_select_cand(
   uint32_t* skey = reinterpret_cast<uint32_t*>(smem);          // [smem_cap]
   int32_t* spos = reinterpret_cast<int32_t*>(skey + smem_cap); // [smem_cap]
   __shared__ unsigned int hist[256];
-  __shared__ unsigned int s_prefix, s_need;
+  __shared__ unsigned int s_prefix, s_need, s_digit, s_above, s_cnt;
   __shared__ float qts[D_ROPE];
   __shared__ int scan_scratch[33];
   const int64_t bh = blockIdx.x;
@@ -248,8 +304,8 @@ __global__ void __launch_bounds__(SEL_THREADS) k_select_cand(
   auto pos_at = [&](int i) -> uint32_t { return staged ? (uint32_t)spos[i] : (uint32_t)g[i].x; };
 
   // radix select of the k-th largest key among the c candidates
-  unsigned int prefix = 0, mask = 0, need = (unsigned int)k;
-  uint32_t pos_cut = 0u;
+  unsigned int prefix = 0, mask = 0, need = (unsigned int)k, ties = 0;
+  uint32_t pos_cut = 0xffffffffu;
   if (k > 0) {
     for (int shift = 24; shift >= 0; shift -= 8) {
       for (int i = threadIdx.x; i < 256; i += blockDim.x) hist[i] = 0;
@@ -259,49 +315,34 @@ __global__ void __launch_bounds__(SEL_THREADS) k_select_cand(
         if ((key & mask) == prefix) atomicAdd(&hist[(key >> shift) & 255u], 1u);
       }
       __syncthreads();
-      if (threadIdx.x == 0) {
-        unsigned int above = 0;
-        int d = 255;
-        for (; d > 0; --d) {
-          if (above + hist[d] >= need) break;
-          above += hist[d];
-        }
-        s_prefix = prefix | ((unsigned int)d << shift);
-        s_need = need - above;
-      }
+      if (threadIdx.x < 32) pick_digit_desc(hist, need, &s_digit, &s_above, &s_cnt);
       __syncthreads();
-      prefix = s_prefix;
-      need = s_need;
+      prefix |= s_digit << shift;
+      need -= s_above;
+      ties = s_cnt;                                   // after the last pass: the keys equal to tau
       mask |= 255u << shift;
       __syncthreads();
     }
-    // among keys equal to tau keep the `need` smallest positions: find the need-th smallest of them
-    unsigned int pprefix = 0, pmask = 0, pneed = need;
-    for (int shift = 24; shift >= 0; shift -= 8) {
-      for (int i = threadIdx.x; i < 256; i += blockDim.x) hist[i] = 0;
-      __syncthreads();
-      for (int i = threadIdx.x; i < c; i += blockDim.x) {
-        const uint32_t p = pos_at(i);
-        if (key_at(i) == prefix && (p & pmask) == pprefix) atomicAdd(&hist[(p >> shift) & 255u], 1u);
-      }
-      __syncthreads();
-      if (threadIdx.x == 0) {
-        unsigned int below = 0;
-        int d = 0;
-        for (; d < 255; ++d) {
-          if (below + hist[d] >= pneed) break;
-          below += hist[d];
+    if (ties > need) {
+      // among keys equal to tau keep the `need` smallest positions: find the need-th smallest of them
+      unsigned int pprefix = 0, pmask = 0, pneed = need;
+      for (int shift = 24; shift >= 0; shift -= 8) {
+        for (int i = threadIdx.x; i < 256; i += blockDim.x) hist[i] = 0;
+        __syncthreads();
+        for (int i = threadIdx.x; i < c; i += blockDim.x) {
+          const uint32_t p = pos_at(i);
+          if (key_at(i) == prefix && (p & pmask) == pprefix) atomicAdd(&hist[(p >> shift) & 255u], 1u);
         }
-        s_prefix = pprefix | ((unsigned int)d << shift);
-        s_need = pneed - below;
+        __syncthreads();
+        if (threadIdx.x < 32) pick_digit_asc(hist, pneed, &s_digit, &s_above);
+        __syncthreads();
+        pprefix |= s_digit << shift;
+        pneed -= s_above;
+        pmask |= 255u << shift;
+        __syncthreads();
       }
-      __syncthreads();
-      pprefix = s_prefix;
-      pneed = s_need;
-      pmask |= 255u << shift;
-      __syncthreads();
+      pos_cut = pprefix;
     }
-    pos_cut = pprefix;
   }
   const uint32_t tau = prefix;
   // bitmap: clear this head's words, then set sinks and window (tier 1) and the selected candidates
@@ -349,7 +390,7 @@ cudaError_t launch_select_cand(int B, int H, int N, int lo, int hi, int64_t k, c
   const size_t smem = (size_t)smem_cap * 8;
   cudaError_t e = cudaFuncSetAttribute(k_select_cand, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
-  k_select_cand<<<B * H, SEL_THREADS, smem, st>>>(
+  k_select_cand<<<B * H, CAND_THREADS, smem, st>>>(
       H, N, lo, hi, (long long)k, reinterpret_cast<const long long*>(k_per_head), cand_cnt, cand, capc, smem_cap,
       force_fallback, static_cast<const __nv_bfloat16*>(v.rope), v.rope_ld, v.rope_bstride, qt, idx, count, cap,
       append, kth, bitmap, (long long)nw, status);
