@@ -149,6 +149,7 @@ __global__ void __launch_bounds__(AT_THREADS, 1) k_attn(
   const int p0 = split * split_len, p1 = min(N, p0 + split_len);
   const int nb = (p1 - p0 + AT_BLK - 1) / AT_BLK;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const bool contiguous = (rope == latent + D_LAT) && lld == ROWE && rld == ROWE && rbs == lbs;
 
   if (threadIdx.x == 0) {
     abort_flag = 0;
@@ -210,14 +211,36 @@ __global__ void __launch_bounds__(AT_THREADS, 1) k_attn(
         const uint32_t uni = __reduce_or_sync(0xffffffffu, ha | hb);
         if (lane == 0) hdr_union[s] = uni;
         __syncwarp();
-        if (lane == 0) mbar_arrive_expect_tx(&full[s], __popc(uni) * (uint32_t)(ROWE * ESZ));
-        __syncwarp();
-        if (lane < AT_BLK && ((uni >> lane) & 1u)) {
-          const int slot = __popc(uni & ((1u << lane) - 1u));
-          const int64_t u = pos0 + lane;
-          T* dst = rows + ((int64_t)s * AT_BLK + slot) * ROWE;
-          bulk_g2s(dst, latent + (int64_t)b * lbs + u * lld, D_LAT * ESZ, &full[s]);
-          bulk_g2s(dst + D_LAT, rope + (int64_t)b * rbs + u * rld, D_ROPE * ESZ, &full[s]);
+        // every union row goes to the stage slot of its position in the block; with the interleaved row layout
+        // (RoPE right after the latent, 576-wide rows) a run of consecutive union rows is one contiguous range
+        // and one bulk copy, otherwise each row takes two (latent, RoPE)
+        if (contiguous) {
+          if (lane == 0) {
+            uint32_t bytes = 0;
+            for (uint32_t m = uni; m; ) {
+              const int j0 = __ffs(m) - 1;
+              const int len = __ffs(~(m >> j0)) - 1;       // length of the run of set bits starting at j0
+              bytes += (uint32_t)len * (uint32_t)(ROWE * ESZ);
+              m &= ~(((len >= 32) ? 0xffffffffu : ((1u << len) - 1u)) << j0);
+            }
+            mbar_arrive_expect_tx(&full[s], bytes);
+          }
+          __syncwarp();
+          if (lane < AT_BLK && ((uni >> lane) & 1u) && (lane == 0 || !((uni >> (lane - 1)) & 1u))) {
+            const int len = __ffs(~(uni >> lane)) - 1;
+            const int64_t u = pos0 + lane;
+            bulk_g2s(rows + ((int64_t)s * AT_BLK + lane) * ROWE, latent + (int64_t)b * lbs + u * lld,
+                     (uint32_t)len * (uint32_t)(ROWE * ESZ), &full[s]);
+          }
+        } else {
+          if (lane == 0) mbar_arrive_expect_tx(&full[s], __popc(uni) * (uint32_t)(ROWE * ESZ));
+          __syncwarp();
+          if (lane < AT_BLK && ((uni >> lane) & 1u)) {
+            const int64_t u = pos0 + lane;
+            T* dst = rows + ((int64_t)s * AT_BLK + lane) * ROWE;
+            bulk_g2s(dst, latent + (int64_t)b * lbs + u * lld, D_LAT * ESZ, &full[s]);
+            bulk_g2s(dst + D_LAT, rope + (int64_t)b * rbs + u * rld, D_ROPE * ESZ, &full[s]);
+          }
         }
       }
 #pragma unroll
@@ -269,9 +292,8 @@ __global__ void __launch_bounds__(AT_THREADS, 1) k_attn(
       while (bits) {
         const int j = __ffs(bits) - 1;
         bits &= bits - 1;
-        const int slot = __popc(uni & ((1u << j) - 1u));
         Slice x;
-        x.load(stage + slot * ROWE, lane);
+        x.load(stage + j * ROWE, lane);                   // rows sit at their position's slot
         tmem_wait_st();
         tmem_ld16(tacc + 16 * i, o);                    // overlaps with the dot product below
         float d = slice_dot(q[i], x);
@@ -337,6 +359,9 @@ size_t attn_smem_bytes(int dtype, int H, int split_len) {
 
 cudaError_t launch_attn(const vk_view& v, float lam, const uint32_t* bitmap, int64_t nw, int nsplit, int split_len,
                         int slot0, int nslot, float* part_o, float* part_ml, int* status, cudaStream_t st) {
+  // bf16 caches: logits on the tensor cores (k_attn_tc.cu); fp32 caches: the SIMT kernel below
+  if (attn_tc_supported(v))
+    return launch_attn_tc(v, lam, bitmap, nw, nsplit, split_len, slot0, nslot, part_o, part_ml, status, st);
   dim3 grid(nsplit, (v.H + HG - 1) / HG, v.B);
   const int nst = attn_stages(v.dtype, v.H);
   const size_t smem = attn_smem_bytes(v.dtype, v.H, split_len);

@@ -105,6 +105,9 @@ cudaError_t launch_build_digest(const vk_view& v, int r, const float* rot, __nv_
 cudaError_t launch_list_to_bitmap(int B, int H, int N, const int32_t* idx, const int32_t* count, int cap,
                                   uint32_t* bitmap, int64_t nw, int* status, cudaStream_t st);
 size_t attn_smem_bytes(int dtype, int H, int split_len);
+bool attn_tc_supported(const vk_view& v);
+cudaError_t launch_attn_tc(const vk_view& v, float lam, const uint32_t* bitmap, int64_t nw, int nsplit, int split_len,
+                           int slot0, int nslot, float* part_o, float* part_ml, int* status, cudaStream_t st);
 cudaError_t launch_attn(const vk_view& v, float lam, const uint32_t* bitmap, int64_t nw, int nsplit,
                         int split_len, int slot0, int nslot, float* part_o, float* part_ml, int* status,
                         cudaStream_t st);
