@@ -99,7 +99,7 @@ struct TcSmem {
   }
 };
 
-template <int G>
+template <int G, int MODE>
 __global__ void __launch_bounds__((2 + 4 * G) * 32, 1) k_score_tc(const __grid_constant__ CUtensorMap kmap,
                                                                 const __grid_constant__ CUtensorMap qmap,
                                                                 const ScoreTcArgs args) {
@@ -203,9 +203,9 @@ __global__ void __launch_bounds__((2 + 4 * G) * 32, 1) k_score_tc(const __grid_c
         // per-sequence parameters -> this group's shared-memory slot (the group's 4 warps, then a barrier)
         named_barrier(2 + g, 128);
         for (int h = (ew & 3) * 32 + lane; h < H; h += 128) {
-          if (args.mode == 1) {
+          if (MODE == 1) {
             prm[h] = args.theta[(int64_t)b * H + h];
-          } else if (args.mode == 2) {
+          } else if (MODE == 2) {
             prm[h] = args.smax1[(int64_t)b * H + h];
             prm[H + h] = args.qcn[(int64_t)b * H + h] * args.z;
             prm[2 * H + h] = args.qrn[(int64_t)b * H + h];
@@ -226,14 +226,14 @@ __global__ void __launch_bounds__((2 + 4 * G) * 32, 1) k_score_tc(const __grid_c
       const uint32_t tbase = tmem_base + ((uint32_t)(quarter * 32) << 16) + g * dcols;
       bool arch = false;
       float row_add = 0.f, row_eta = 0.f;
-      if (args.mode >= 1) arch = in_rows && row >= args.arch_lo && row < args.arch_hi;
-      if (args.mode == 2 && in_rows) {
+      if (MODE >= 1) arch = in_rows && row >= args.arch_lo && row < args.arch_hi;
+      if (MODE == 2 && in_rows) {
         row_add = args.page_res[(int64_t)b * args.n_pages + row / PAGE];
         row_eta = args.eta[(int64_t)b * args.N + row];
       }
       const int64_t word = (row0 + quarter * 32) / 32;      // this warp's 32 rows = one bitmap word
       const bool word_ok = word < args.nw;
-      const bool emit = args.mode == 1 || (args.mode == 2 && args.top_j > 0);
+      const bool emit = MODE == 1 || (MODE == 2 && args.top_j > 0);
       constexpr int NCH = G == 4 ? 4 : 8;                  // 32-head chunks (H <= 128 when G = 4)
       uint32_t mine[NCH];                                  // ballot of head c + lane, per 32-head chunk
       int base[NCH];
@@ -243,7 +243,7 @@ __global__ void __launch_bounds__((2 + 4 * G) * 32, 1) k_score_tc(const __grid_c
         if (c >= H) break;
         const int hn = min(32, H - c);                     // 32, or 16 for the last chunk when H % 32 == 16
         uint32_t sel_word = 0;
-        if (args.mode == 2 && lane < hn && word_ok) sel_word = args.selbm[(bh0 + c + lane) * args.nw + word];
+        if (MODE == 2 && lane < hn && word_ok) sel_word = args.selbm[(bh0 + c + lane) * args.nw + word];
         uint32_t m_lane = 0;
 #pragma unroll
         for (int half = 0; half < 2; ++half) {
@@ -251,7 +251,7 @@ __global__ void __launch_bounds__((2 + 4 * G) * 32, 1) k_score_tc(const __grid_c
           float v[16];
           tmem_ld16(tbase + c + 16 * half, v);
           tmem_wait_ld();
-          if (args.mode == 0) {
+          if (MODE == 0) {
             if (in_rows) {
 #pragma unroll
               for (int j = 0; j < 16; ++j) args.scores[(bh0 + c + 16 * half + j) * args.scores_ld + row] = v[j];
@@ -262,7 +262,7 @@ __global__ void __launch_bounds__((2 + 4 * G) * 32, 1) k_score_tc(const __grid_c
           for (int jj = 0; jj < 16; ++jj) {
             const int j = 16 * half + jj;
             bool pass = false;
-            if (args.mode == 1) {
+            if (MODE == 1) {
               pass = arch && v[jj] >= prm[c + j];
             } else {
               const uint32_t sw = __shfl_sync(0xffffffffu, sel_word, j);
@@ -274,7 +274,7 @@ __global__ void __launch_bounds__((2 + 4 * G) * 32, 1) k_score_tc(const __grid_c
           }
         }
         mine[cc] = m_lane;
-        if (args.mode == 2 && !emit && lane < hn && word_ok) args.firebm[(bh0 + c + lane) * args.nw + word] = m_lane;
+        if (MODE == 2 && !emit && lane < hn && word_ok) args.firebm[(bh0 + c + lane) * args.nw + word] = m_lane;
       }
       if (emit) {
         // reserve room for every chunk first (the atomics overlap), then read the scores again and scatter
@@ -303,7 +303,7 @@ __global__ void __launch_bounds__((2 + 4 * G) * 32, 1) k_score_tc(const __grid_c
               if ((m >> lane) & 1u) {
                 const int pos = bj + __popc(m & ((1u << lane) - 1u));
                 float val = v[jj];
-                if (args.mode == 2) val = args.lam * (v[jj] + prm[2 * H + c + j] * row_add + prm[H + c + j] * row_eta);
+                if (MODE == 2) val = args.lam * (v[jj] + prm[2 * H + c + j] * row_add + prm[H + c + j] * row_eta);
                 if (pos < args.capc) args.cand[(bh0 + c + j) * args.capc + pos] = make_int2(row, __float_as_int(val));
               }
             }
@@ -352,8 +352,9 @@ cudaError_t launch_score_tc(const vk_view& v, int row_offset, int row_stride, in
   cuuint64_t kstr[2] = {(cuuint64_t)(v.rope_ld * row_stride * 2), (cuuint64_t)(v.rope_bstride * 2)};
   cuuint32_t kbox[3] = {D_ROPE, TC_M, 1};
   cuuint32_t es3[3] = {1, 1, 1};
+  // each row contributes one 128-byte segment 1152 bytes apart: no L2 promotion, so DRAM reads only those bytes
   if (encode(&kmap, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<__nv_bfloat16*>(rope), kdims, kstr, kbox, es3,
-             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_NONE,
              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
     return cudaErrorInvalidValue;
   cuuint64_t qdims[2] = {(cuuint64_t)D_ROPE, (cuuint64_t)v.B * v.H};
@@ -377,16 +378,17 @@ cudaError_t launch_score_tc(const vk_view& v, int row_offset, int row_stride, in
   args.tmem_cols = cols;
   const int grid = (int)std::min<int64_t>(args.total_tiles, 152);
   const size_t smem = TcSmem(v.H).total;
+  auto pick = [&](auto kernel, int g) -> cudaError_t {
+    cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    if (grid > 0) kernel<<<grid, (2 + 4 * g) * 32, smem, st>>>(kmap, qmap, args);
+    return cudaSuccess;
+  };
   cudaError_t e;
-  if (G == 4) {
-    e = cudaFuncSetAttribute(k_score_tc<4>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    if (e != cudaSuccess) return e;
-    if (grid > 0) k_score_tc<4><<<grid, (2 + 4 * 4) * 32, smem, st>>>(kmap, qmap, args);
-  } else {
-    e = cudaFuncSetAttribute(k_score_tc<2>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    if (e != cudaSuccess) return e;
-    if (grid > 0) k_score_tc<2><<<grid, (2 + 4 * 2) * 32, smem, st>>>(kmap, qmap, args);
-  }
+  const int m = args.mode;
+  if (G == 4) e = m == 0 ? pick(k_score_tc<4, 0>, 4) : m == 1 ? pick(k_score_tc<4, 1>, 4) : pick(k_score_tc<4, 2>, 4);
+  else e = m == 0 ? pick(k_score_tc<2, 0>, 2) : m == 1 ? pick(k_score_tc<2, 1>, 2) : pick(k_score_tc<2, 2>, 2);
+  if (e != cudaSuccess) return e;
   if (grid > 0) count_launches(1);
   return cudaGetLastError();
 }

@@ -11,6 +11,7 @@ namespace vk {
 
 constexpr int SEL_THREADS = 512;
 constexpr int CAND_THREADS = 256;
+constexpr long long SEL_SMEM_BITMAP_WORDS = 8192;   // positions up to 262,144: bitmap built in shared memory
 
 // Radix-select step over a 256-bin histogram, run by one full warp: the largest digit d with
 // (count of bins above d) < need <= (count of bins at or above d). Lane l owns bins 255 - 8l .. 248 - 8l.
@@ -345,25 +346,29 @@ __global__ void __launch_bounds__(CAND_THREADS) k_select_cand(
     }
   }
   const uint32_t tau = prefix;
-  // bitmap: clear this head's words, then set sinks and window (tier 1) and the selected candidates
-  for (long long w = threadIdx.x; w < nw; w += blockDim.x) bm[w] = 0u;
+  // bitmap (built in shared memory when it fits): clear, then set sinks and window (tier 1) and the selected
+  // candidates, then write it out
+  uint32_t* wbm = nw <= SEL_SMEM_BITMAP_WORDS ? reinterpret_cast<uint32_t*>(spos + smem_cap) : bm;
+  for (long long w = threadIdx.x; w < nw; w += blockDim.x) wbm[w] = 0u;
   __syncthreads();
   if (!append) {
-    for (int u = threadIdx.x; u < lo; u += blockDim.x) atomicOr(&bm[u >> 5], 1u << (u & 31));
-    for (int u = hi + threadIdx.x; u < N; u += blockDim.x) atomicOr(&bm[u >> 5], 1u << (u & 31));
+    for (int u = threadIdx.x; u < lo; u += blockDim.x) atomicOr(&wbm[u >> 5], 1u << (u & 31));
+    for (int u = hi + threadIdx.x; u < N; u += blockDim.x) atomicOr(&wbm[u >> 5], 1u << (u & 31));
   }
   if (k > 0) {
     for (int i = threadIdx.x; i < c; i += blockDim.x) {
       const uint32_t key = key_at(i), p = pos_at(i);
-      if (key > tau || (key == tau && p <= pos_cut)) atomicOr(&bm[p >> 5], 1u << (p & 31));
+      if (key > tau || (key == tau && p <= pos_cut)) atomicOr(&wbm[p >> 5], 1u << (p & 31));
     }
   }
   __syncthreads();
+  if (wbm != bm)
+    for (long long w = threadIdx.x; w < nw; w += blockDim.x) bm[w] = wbm[w];
   // ascending ids from the bitmap
   int base = append ? count[bh] : 0;
   for (long long c0 = 0; c0 < nw; c0 += blockDim.x) {
     const long long w = c0 + threadIdx.x;
-    const uint32_t word = (w < nw) ? bm[w] : 0u;
+    const uint32_t word = (w < nw) ? wbm[w] : 0u;
     int tot;
     int pos = base + block_exclusive_scan(__popc(word), scan_scratch, &tot);
     uint32_t bits = word;
@@ -387,7 +392,7 @@ cudaError_t launch_select_cand(int B, int H, int N, int lo, int hi, int64_t k, c
                                const float* qt, int32_t* idx, int32_t* count, int cap, int append, float* kth,
                                uint32_t* bitmap, int64_t nw, int* status, cudaStream_t st) {
   const int smem_cap = capc < 12288 ? capc : 12288;
-  const size_t smem = (size_t)smem_cap * 8;
+  const size_t smem = (size_t)smem_cap * 8 + (nw <= SEL_SMEM_BITMAP_WORDS ? (size_t)nw * 4 : 0);
   cudaError_t e = cudaFuncSetAttribute(k_select_cand, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
   k_select_cand<<<B * H, CAND_THREADS, smem, st>>>(
