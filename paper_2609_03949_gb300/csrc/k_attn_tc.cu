@@ -1,21 +1,28 @@
-// k_attn_tc.cu -- gather + absorbed-MLA attention with the logits on the tensor cores (bf16 caches).
+// k_attn_tc.cu -- gather + absorbed-MLA attention for bf16 caches, both contractions on the tensor cores.
 //
-// Per CTA: one sequence b, one range of positions, one group of <= 64 heads. Positions are walked in tiles of
-// 32 (one bitmap word per head). For each tile:
-//   warp 0 (producer)   stages the heads' 32-bit selection words and issues nine TMA loads (128-byte swizzle,
-//                       K-major) of the tile's 32 rows x 576 columns into a 4-slot ring (tiles without any
-//                       selected row are not loaded);
-//   warp 1 (MMA)        S = Q . X^T on tcgen05: M = 64 heads, N = 32 rows, K = 576 (36 x K=16) into tensor
-//                       memory; with M = 64 the logit of head 16g + t and row j sits in TMEM lane 32g + t,
-//                       column j of the tile's slot;
-//   warps 2..17         16 consumers, warp w owning heads 16 (w % 4) + 4 sub + i (sub = (w - 2) / 4, i < 4)
-//                       so that their logits are in the warp's own TMEM lane quarter. For every selected
-//                       (head, row) pair: read the logit (one tcgen05.ld), update the head's online softmax
-//                       and accumulate p * latent row (bf16 x bf16 -> fp32 mixed FMAs) into the head's
-//                       512-wide running sum, kept in registers (16 values per lane per head).
-// The dense S tile costs ~35% of the tensor time the HBM stream leaves; the sparse part (softmax and the
-// 512-wide axpy over ~4% of the (head, row) pairs) stays on the SIMT pipes. Partial (max, sum, out) per split
-// are merged by the same LSE combine as the SIMT kernel (Lemma 1). All mbarrier waits are bounded.
+// Per CTA: one sequence b, one range of positions (a multiple of 64 long), one group of <= 64 heads. Positions are
+// walked in tiles of 64 rows; a tile that no head of the group selects is neither loaded nor computed. Per tile:
+//   warp 0 (producer)  stages the heads' two 32-bit selection words of the tile, then TMA-loads its 64 rows x 576
+//                      columns (128-byte swizzle, one 8 KB block per 64 columns) as five groups -- the RoPE block
+//                      first, then four pairs of latent blocks, each as soon as the tile before it in that slot has
+//                      released it -- into one of two tile slots;
+//   warp 1 (MMA)       S = Q . X^T on tcgen05 (M = 64 heads, N = 64 rows, K = 576: 36 instructions) into one of two
+//                      S buffers in tensor memory; with M = 64 the logit of head 16 g + i and row j sits in TMEM lane
+//                      32 g + i, column j. Then, once the softmax warps have written P^T, O^T += X_lat^T . P^T
+//                      (M = 128 latent dims x 4 blocks, N = 64 heads, K = 64 rows: 16 instructions) into the O^T
+//                      accumulator, which stays in tensor memory for the whole range. X_lat^T is read straight from
+//                      the tile slot as an MN-major operand (the next 64 dims one 8 KB block away), so each latent
+//                      row is staged in shared memory once and feeds both contractions;
+//   warps 2..5         softmax: lane i < 16 of the warp on TMEM lane quarter g owns head 16 g + i. It reads its 64
+//                      logits, masks them with its selection words and writes P^T[h][row] = 2^(s lambda log2(e) - m_h)
+//                      (0 where the head did not select the row) in bf16 into shared memory (K-major, 128-byte
+//                      swizzle). m_h is a running max that only moves when a tile's max exceeds it by more than 8
+//                      (log2 units; the head's O^T column and sum are then rescaled in tensor memory), so rescaling
+//                      is rare and P stays <= 256. The exact max is tracked beside it, and at the end the head's sum
+//                      and output are re-based on it, so the partial carries the true max logit.
+// The partial (max, sum, out) of each range is merged by the LSE combine (Lemma 1). Rows inside a loaded tile that
+// no head selected still enter the O^T product with weight 0, so every row in [0, N) must hold finite values.
+// All waits are bounded: a wait that gives up raises VK_ERR_TIMEOUT and every role drains and leaves.
 #include <cuda.h>
 #include <cudaTypedefs.h>
 
@@ -26,28 +33,44 @@
 
 namespace vk {
 
-constexpr int AT2_T = 32;                              // positions (rows) per tile
-constexpr int AT2_NT = 4;                              // tile slots
-constexpr int AT2_CONS = 16;                           // consumer warps
-constexpr int AT2_THREADS = (2 + AT2_CONS) * 32;
-constexpr uint32_t AT2_KBLK_Q = 64 * 128;              // one 64-column block of Q: 64 heads x 128 B
-constexpr uint32_t AT2_KBLK_X = AT2_T * 128;           // one 64-column block of a tile: 32 rows x 128 B
-constexpr uint32_t AT2_Q_BYTES = 9 * AT2_KBLK_Q;       // 73,728
-constexpr uint32_t AT2_X_BYTES = 9 * AT2_KBLK_X;       // 36,864 per slot
-constexpr uint32_t AT2_TMEM_COLS = 128;                // 4 x 32 logit columns
-constexpr uint32_t AT2_S_COL0 = 0;
+constexpr int AT_T = 64;                               // rows per tile
+constexpr int AT_SMX = 4;                              // softmax warps (one per TMEM lane quarter)
+constexpr int AT_THREADS = (2 + AT_SMX) * 32;
+constexpr uint32_t AT_KBLK = 64 * 128;                 // one 64-column block of 64 rows (or 64 heads): 8 KB
+constexpr uint32_t AT_TILE = 9 * AT_KBLK;              // 73,728: one tile slot, and the queries
+constexpr uint32_t AT_P = 64 * 128;                    // P^T: 64 heads x 64 rows, bf16
+constexpr int AT_NG = 5;                               // load groups per tile: latent pairs 0..3, RoPE block 4
+constexpr float AT_TAU = 8.f;                          // log2 slack before a running max moves
+constexpr uint32_t AT_TMEM_COLS = 512;
+constexpr uint32_t AT_S_COL = 0;                       // S buffers: columns 0..63 and 64..127
+constexpr uint32_t AT_O_COL = 128;                     // O^T block j: columns 128 + 64 j .. + 63
 
-struct Attn2Smem {
-  uint32_t q, x, words, uni, logit, bars, total;
-  __host__ __device__ Attn2Smem() {
-    q = 0;
-    x = q + AT2_Q_BYTES;
-    words = x + AT2_NT * AT2_X_BYTES;                  // [NT][64] selection words
-    uni = words + AT2_NT * 64 * 4;                     // [NT] union words
-    logit = uni;
-    bars = (uni + AT2_NT * 4 + 7) & ~7u;               // x_full[NT], x_empty[NT], s_full[NT], q_full
-    total = bars + (3 * AT2_NT + 1) * 8 + 1024;        // + slack to align the base to 1024
-  }
+// Shared memory, from a 1024-byte aligned base. Barriers: xfull/xrel [2 slots][5 groups], sfull/sfree [2],
+// wfull/wfree [2], pfull, pfree, qfull, mdone, gbar [2], ebar.
+struct AtSmem {
+  static constexpr uint32_t q = 0;
+  static constexpr uint32_t x = q + AT_TILE;
+  static constexpr uint32_t p = x + 2 * AT_TILE;
+  static constexpr uint32_t words = p + AT_P;          // [2][64 heads][2] u32
+  static constexpr uint32_t uni = words + 2 * 64 * 2 * 4;
+  static constexpr uint32_t fac = uni + 2 * 4;         // [2][64] f32
+  static constexpr uint32_t anyw = fac + 2 * 64 * 4;   // [2][4] u32
+  static constexpr uint32_t misc = anyw + 2 * 4 * 4;   // TMEM base, abort flag
+  static constexpr uint32_t bars = (misc + 8 + 7) & ~7u;
+  static constexpr uint32_t nbars = 2 * AT_NG * 2 + 2 * 4 + 4 + 3;
+  static constexpr uint32_t total = bars + nbars * 8;
+};
+static_assert(AtSmem::total + 1024 <= 232448, "attention shared memory exceeds the 227 KB opt-in limit");
+
+struct AttnTcArgs {
+  int H, N;
+  int split_len, slot0, nslot;
+  int64_t nw;
+  float lam_log2e;
+  const uint32_t* bitmap;
+  float* part_o;
+  float* part_ml;
+  int* status;
 };
 
 __device__ __forceinline__ void tma_load_3d_(void* dst, const CUtensorMap* map, int x, int y, int z, uint64_t* bar) {
@@ -57,9 +80,11 @@ __device__ __forceinline__ void tma_load_3d_(void* dst, const CUtensorMap* map, 
       "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(z), "r"(smem_addr(bar))
       : "memory");
 }
-__device__ __forceinline__ uint64_t sw128_desc_(uint32_t saddr) {
-  return (uint64_t)((saddr >> 4) & 0x3FFFu) | ((uint64_t)1u << 16) | ((uint64_t)(1024u >> 4) << 32) |
-         ((uint64_t)1u << 46) | ((uint64_t)2u << 61);
+// Shared-memory matrix descriptor, 128-byte swizzle, 8-row groups 1024 B apart. `lbo` is the byte distance between
+// 64-element atoms along M/N for an MN-major operand (unused by K-major ones).
+__device__ __forceinline__ uint64_t sdesc_(uint32_t saddr, uint32_t lbo) {
+  return (uint64_t)((saddr >> 4) & 0x3FFFu) | ((uint64_t)((lbo >> 4) & 0x3FFFu) << 16) |
+         ((uint64_t)(1024u >> 4) << 32) | ((uint64_t)1u << 46) | ((uint64_t)2u << 61);
 }
 __device__ __forceinline__ void mma_bf16_(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc, uint32_t idesc,
                                           uint32_t accumulate) {
@@ -73,12 +98,14 @@ __device__ __forceinline__ void mma_commit_(uint64_t* bar) {
   asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];\n" ::"r"(smem_addr(bar))
                : "memory");
 }
-__device__ __forceinline__ float tmem_ld1(uint32_t taddr) {
+__device__ __forceinline__ float tmem_ld1_(uint32_t taddr) {
   uint32_t r;
   asm volatile("tcgen05.ld.sync.aligned.32x32b.x1.b32 {%0}, [%1];\n" : "=r"(r) : "r"(taddr) : "memory");
   return __uint_as_float(r);
 }
-
+__device__ __forceinline__ void tmem_st1_(uint32_t taddr, float v) {
+  asm volatile("tcgen05.st.sync.aligned.32x32b.x1.b32 [%0], {%1};\n" ::"r"(taddr), "r"(__float_as_uint(v)) : "memory");
+}
 __device__ __forceinline__ void tmem_ld32_(uint32_t taddr, float* v) {
   uint32_t* r = reinterpret_cast<uint32_t*>(v);
   asm volatile(
@@ -91,230 +118,375 @@ __device__ __forceinline__ void tmem_ld32_(uint32_t taddr, float* v) {
       : "r"(taddr)
       : "memory");
 }
+// Generic-proxy shared-memory writes become visible to the tensor core (async proxy).
+__device__ __forceinline__ void fence_async_smem_() { asm volatile("fence.proxy.async.shared::cta;\n" ::: "memory"); }
+// Warp-uniform bounded wait: lane 0 polls, the warp takes its verdict.
+__device__ __forceinline__ bool warp_wait_(uint64_t* bar, uint32_t parity, volatile int* abort_flag, int lane) {
+  bool w = true;
+  if (lane == 0) w = mbar_wait(bar, parity, abort_flag);
+  return __shfl_sync(0xffffffffu, w, 0);
+}
 
-__device__ __forceinline__ uint16_t lo16_(uint32_t w) { return static_cast<uint16_t>(w & 0xffffu); }
-__device__ __forceinline__ uint16_t hi16_(uint32_t w) { return static_cast<uint16_t>(w >> 16); }
-
-struct Attn2Args {
-  int H, N, nh_total;
-  int split_len, slot0, nslot;
-  int64_t nw;
-  float lam_log2e;
-  const uint32_t* bitmap;
-  float* part_o;
-  float* part_ml;
-  int* status;
-};
-
-__global__ void __launch_bounds__(AT2_THREADS, 1) k_attn_tc(const __grid_constant__ CUtensorMap lmap,
-                                                          const __grid_constant__ CUtensorMap rmap,
-                                                          const __grid_constant__ CUtensorMap qlmap,
-                                                          const __grid_constant__ CUtensorMap qrmap,
-                                                          const Attn2Args args) {
+__global__ void __launch_bounds__(AT_THREADS, 1) k_attn_tc(const __grid_constant__ CUtensorMap lmap,
+                                                         const __grid_constant__ CUtensorMap rmap,
+                                                         const __grid_constant__ CUtensorMap qlmap,
+                                                         const __grid_constant__ CUtensorMap qrmap,
+                                                         const AttnTcArgs args) {
   extern __shared__ __align__(1024) unsigned char smem_raw[];
   unsigned char* smem = reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  const Attn2Smem L;
-  unsigned char* sq = smem + L.q;
-  unsigned char* sx = smem + L.x;
-  uint32_t* words = reinterpret_cast<uint32_t*>(smem + L.words);
-  uint32_t* unis = reinterpret_cast<uint32_t*>(smem + L.uni);
-  uint64_t* x_full = reinterpret_cast<uint64_t*>(smem + L.bars);
-  uint64_t* x_empty = x_full + AT2_NT;
-  uint64_t* s_full = x_empty + AT2_NT;
-  uint64_t* q_full = s_full + AT2_NT;
-  __shared__ uint32_t tmem_base;
-  __shared__ int abort_flag;
+  unsigned char* sq = smem + AtSmem::q;
+  unsigned char* sx = smem + AtSmem::x;
+  unsigned char* sp = smem + AtSmem::p;
+  uint32_t* words = reinterpret_cast<uint32_t*>(smem + AtSmem::words);
+  uint32_t* unis = reinterpret_cast<uint32_t*>(smem + AtSmem::uni);
+  float* fac = reinterpret_cast<float*>(smem + AtSmem::fac);
+  uint32_t* anyw = reinterpret_cast<uint32_t*>(smem + AtSmem::anyw);
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + AtSmem::misc);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + AtSmem::misc + 4);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + AtSmem::bars);
+  uint64_t* xfull = bars;                     // [2][5]
+  uint64_t* xrel = bars + 2 * AT_NG;          // [2][5]
+  uint64_t* sfull = bars + 4 * AT_NG;         // [2]
+  uint64_t* sfree = sfull + 2;                // [2]
+  uint64_t* wfull = sfree + 2;                // [2]
+  uint64_t* wfree = wfull + 2;                // [2]
+  uint64_t* pfull = wfree + 2;
+  uint64_t* pfree = pfull + 1;
+  uint64_t* qfull = pfree + 1;
+  uint64_t* mdone = qfull + 1;
+  uint64_t* gbar = mdone + 1;                 // [2] softmax-group syncs, by tile parity
+  uint64_t* ebar = gbar + 2;                  // softmax-group sync before the epilogue
 
   const int split = blockIdx.x, hg = blockIdx.y, b = blockIdx.z;
   const int H = args.H;
   const int h0 = hg * 64, nh = min(64, H - h0);
   const int p0 = split * args.split_len, p1 = min(args.N, p0 + args.split_len);
-  const int ntile = (p1 - p0 + AT2_T - 1) / AT2_T;         // p0 is a multiple of 32
+  const int ntile = p1 > p0 ? (p1 - p0 + AT_T - 1) / AT_T : 0;    // p0 is a multiple of 64
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
   if (threadIdx.x == 0) {
-    abort_flag = 0;
-    for (int s = 0; s < AT2_NT; ++s) { mbar_init(&x_full[s], 1); mbar_init(&x_empty[s], AT2_CONS); mbar_init(&s_full[s], 1); }
-    mbar_init(q_full, 1);
+    *abort_flag = 0;
+    for (int i = 0; i < 2 * AT_NG; ++i) { mbar_init(&xfull[i], 1); mbar_init(&xrel[i], 1); }
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(&sfull[i], 1);
+      mbar_init(&sfree[i], AT_SMX);
+      mbar_init(&wfull[i], 1);
+      mbar_init(&wfree[i], AT_SMX + 1);
+      mbar_init(&gbar[i], AT_SMX);
+    }
+    mbar_init(pfull, AT_SMX);
+    mbar_init(pfree, 1);
+    mbar_init(qfull, 1);
+    mbar_init(mdone, 1);
+    mbar_init(ebar, AT_SMX);
     mbar_fence_init();
   }
-  if (warp == 1) tmem_alloc(&tmem_base, AT2_TMEM_COLS);
+  if (warp == 1) tmem_alloc(tmem_slot, AT_TMEM_COLS);
   tmem_fence_before();
   __syncthreads();
   tmem_fence_after();
+  const uint32_t tmem = *tmem_slot;
 
   if (warp == 0) {
     // ------------------------------------------------------------------ producer
     const uint32_t* bm = args.bitmap + ((int64_t)b * H + h0) * args.nw;
-    if (lane == 0) {
-      // the head group's queries: nine 64-column blocks of 64 rows (rows past nh read the next heads or zero fill;
-      // their logits are never used)
-      mbar_arrive_expect_tx(q_full, AT2_Q_BYTES);
-      const int qrow = b * H + h0;
-      for (int k = 0; k < 8; ++k) tma_load_3d_(sq + k * AT2_KBLK_Q, &qlmap, 64 * k, qrow, 0, q_full);
-      tma_load_3d_(sq + 8 * AT2_KBLK_Q, &qrmap, 0, qrow, 0, q_full);
+    int last_use[2 * AT_NG];                           // last load issued per (slot, group), for the drain
+#pragma unroll
+    for (int i = 0; i < 2 * AT_NG; ++i) last_use[i] = -1;
+    bool qissued = false;
+    if (lane == 0 && ntile > 0) {
+      mbar_arrive_expect_tx(qfull, AT_TILE);
+      const int qrow = b * H + h0;   // rows past the group's heads belong to other heads (or are zero-filled): unused
+      for (int k = 0; k < 8; ++k) tma_load_3d_(sq + k * AT_KBLK, &qlmap, 64 * k, qrow, 0, qfull);
+      tma_load_3d_(sq + 8 * AT_KBLK, &qrmap, 0, qrow, 0, qfull);
+      qissued = true;
     }
-    // the heads' selection words of tile t (lanes hold heads lane and lane + 32), fetched two tiles ahead
-    auto fetch = [&](int t, uint32_t& wa, uint32_t& wb) {
-      wa = wb = 0u;
+    // selection words of tile t: the lane holds heads lane and lane + 32, rows 0..31 and 32..63 of the tile
+    auto fetch = [&](int t, uint4& w) {
+      w = make_uint4(0u, 0u, 0u, 0u);
       if (t >= ntile) return;
-      const int pos0 = p0 + t * AT2_T;
-      const int64_t w = pos0 >> 5;
-      const int left = p1 - pos0;
-      const uint32_t vmask = left >= 32 ? 0xffffffffu : ((1u << left) - 1u);
-      if (lane < nh) wa = bm[(int64_t)lane * args.nw + w] & vmask;
-      if (lane + 32 < nh) wb = bm[(int64_t)(lane + 32) * args.nw + w] & vmask;
+      const int pos0 = p0 + t * AT_T;
+      const int64_t wi = pos0 >> 5;
+      const int left = p1 - pos0;                      // >= 1
+      const uint32_t m0 = left >= 32 ? 0xffffffffu : ((1u << left) - 1u);
+      const uint32_t m1 = left >= 64 ? 0xffffffffu : (left <= 32 ? 0u : ((1u << (left - 32)) - 1u));
+      if (lane < nh) {
+        const uint32_t* r = bm + (int64_t)lane * args.nw + wi;
+        w.x = r[0] & m0;
+        if (m1) w.y = r[1] & m1;
+      }
+      if (lane + 32 < nh) {
+        const uint32_t* r = bm + (int64_t)(lane + 32) * args.nw + wi;
+        w.z = r[0] & m0;
+        if (m1) w.w = r[1] & m1;
+      }
     };
-    uint32_t a0, b0, a1, b1, a2, b2;
-    fetch(0, a0, b0);
-    fetch(1, a1, b1);
+    uint4 cur, nxt;
+    fetch(0, cur);
+    int u = 0;                                         // tiles loaded so far
+    bool ok = true;
     for (int t = 0; t < ntile; ++t) {
-      fetch(t + 2, a2, b2);
-      const int s = t % AT2_NT, use = t / AT2_NT;
-      if (use > 0 && !mbar_wait(&x_empty[s], (use - 1) & 1, &abort_flag)) {
-        if (lane == 0) { raise_status(args.status, VK_ERR_TIMEOUT); abort_flag = 1; }
-        break;
-      }
-      if (abort_flag) break;
-      const int pos0 = p0 + t * AT2_T;
-      words[s * 64 + lane] = a0;
-      words[s * 64 + lane + 32] = b0;
-      const uint32_t uni = __reduce_or_sync(0xffffffffu, a0 | b0);
-      if (lane == 0) unis[s] = uni;
+      fetch(t + 1, nxt);
+      const int ws = t & 1;
+      if (t >= 2 && !warp_wait_(&wfree[ws], ((t >> 1) - 1) & 1, abort_flag, lane)) { ok = false; break; }
+      uint32_t* wd = words + ws * 128;
+      wd[lane * 2] = cur.x;
+      wd[lane * 2 + 1] = cur.y;
+      wd[(lane + 32) * 2] = cur.z;
+      wd[(lane + 32) * 2 + 1] = cur.w;
+      const uint32_t uni = __reduce_or_sync(0xffffffffu, cur.x | cur.y | cur.z | cur.w);
+      if (lane == 0) unis[ws] = uni;
       __syncwarp();
-      if (lane == 0) {
-        if (uni) {
-          mbar_arrive_expect_tx(&x_full[s], AT2_X_BYTES);
-          for (int k = 0; k < 8; ++k) tma_load_3d_(sx + s * AT2_X_BYTES + k * AT2_KBLK_X, &lmap, 64 * k, pos0, b, &x_full[s]);
-          tma_load_3d_(sx + s * AT2_X_BYTES + 8 * AT2_KBLK_X, &rmap, 0, pos0, b, &x_full[s]);
-        } else {
-          mbar_arrive(&x_full[s]);                      // nothing selected: no load, no work
+      if (lane == 0) mbar_arrive(&wfull[ws]);
+      if (uni) {
+        const int s = u & 1, use = u >> 1;
+        const int pos0 = p0 + t * AT_T;
+        unsigned char* xs = sx + s * AT_TILE;
+        bool lok = true;
+        if (lane == 0) {
+          for (int i = 0; i < AT_NG; ++i) {
+            const int g = i == 0 ? 4 : i - 1;          // RoPE block first: S can start on it
+            uint64_t* fb = &xfull[s * AT_NG + g];
+            if (use > 0 && !mbar_wait(&xrel[s * AT_NG + g], (use - 1) & 1, abort_flag)) { lok = false; break; }
+            if (g == 4) {
+              mbar_arrive_expect_tx(fb, AT_KBLK);
+              tma_load_3d_(xs + 8 * AT_KBLK, &rmap, 0, pos0, b, fb);
+            } else {
+              mbar_arrive_expect_tx(fb, 2 * AT_KBLK);
+              tma_load_3d_(xs + (2 * g) * AT_KBLK, &lmap, 128 * g, pos0, b, fb);
+              tma_load_3d_(xs + (2 * g + 1) * AT_KBLK, &lmap, 128 * g + 64, pos0, b, fb);
+            }
+            last_use[s * AT_NG + g] = use;
+          }
         }
+        if (!__shfl_sync(0xffffffffu, lok, 0)) { ok = false; break; }
+        ++u;
       }
-      a0 = a1; b0 = b1; a1 = a2; b1 = b2;
+      cur = nxt;
+    }
+    if (!ok && lane == 0) { raise_status(args.status, VK_ERR_TIMEOUT); *abort_flag = 1; }
+    // drain: every load issued must have landed before the CTA leaves (only matters after an abort)
+    if (lane == 0) {
+      if (qissued) mbar_wait(qfull, 0, nullptr);
+      for (int i = 0; i < 2 * AT_NG; ++i)
+        if (last_use[i] >= 0) mbar_wait(&xfull[i], last_use[i] & 1, nullptr);
     }
   } else if (warp == 1) {
     // ------------------------------------------------------------------ MMA issuer
-    if (lane == 0) {
-      const uint32_t idesc = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(AT2_T >> 3) << 17) | ((uint32_t)(64 >> 4) << 24);
-      bool ok = mbar_wait(q_full, 0, &abort_flag);
-      for (int t = 0; t < ntile && ok; ++t) {
-        const int s = t % AT2_NT, use = t / AT2_NT;
-        if (!mbar_wait(&x_full[s], use & 1, &abort_flag)) { ok = false; break; }
-        if (unis[s]) {
-          tmem_fence_after();
-          const uint32_t xa = smem_addr(sx + s * AT2_X_BYTES), qa = smem_addr(sq);
-          const uint32_t d = tmem_base + AT2_S_COL0 + s * AT2_T;
-#pragma unroll 1
-          for (int k = 0; k < 9; ++k)
+    if (lane == 0 && ntile > 0) {
+      // S: M = 64 heads, N = 64 rows, A = Q and B = X, both K-major
+      const uint32_t idesc_s =
+          (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(AT_T >> 3) << 17) | ((uint32_t)(64 >> 4) << 24);
+      // O^T: M = 128 dims, N = 64 heads, A = X_lat^T MN-major (bit 15), B = P^T K-major
+      const uint32_t idesc_o =
+          (1u << 4) | (1u << 7) | (1u << 10) | (1u << 15) | ((uint32_t)(64 >> 3) << 17) | ((uint32_t)(128 >> 4) << 24);
+      const uint64_t qd = sdesc_(smem_addr(sq), 16);
+      const uint64_t pd = sdesc_(smem_addr(sp), 16);
+      bool ok = mbar_wait(qfull, 0, abort_flag);
+      int u = 0;
+      auto issue_av = [&](int v) -> bool {
+        const int s = v & 1;
+        if (!mbar_wait(pfull, v & 1, abort_flag)) return false;
+        tmem_fence_after();
+        const uint64_t xd = sdesc_(smem_addr(sx + s * AT_TILE), AT_KBLK);
 #pragma unroll
-            for (int kk = 0; kk < 4; ++kk)
-              mma_bf16_(d, sw128_desc_(qa + k * AT2_KBLK_Q + 32 * kk), sw128_desc_(xa + k * AT2_KBLK_X + 32 * kk), idesc,
-                        (k | kk) != 0);
-          mma_commit_(&s_full[s]);
-        } else {
-          mbar_arrive(&s_full[s]);
+        for (int j = 0; j < 4; ++j) {
+#pragma unroll
+          for (int ks = 0; ks < 4; ++ks)
+            mma_bf16_(tmem + AT_O_COL + 64 * j, xd + (uint64_t)((2 * j * AT_KBLK + ks * 2048) >> 4),
+                      pd + (uint64_t)(ks * 2), idesc_o, (v > 0 || ks > 0) ? 1u : 0u);
+          mma_commit_(&xrel[s * AT_NG + j]);           // latent blocks 2j, 2j+1 of this slot are free again
         }
+        mma_commit_(pfree);                            // P^T free, O^T up to date
+        return true;
+      };
+      for (int t = 0; t < ntile && ok; ++t) {
+        const int ws = t & 1;
+        if (!mbar_wait(&wfull[ws], (t >> 1) & 1, abort_flag)) { ok = false; break; }
+        const uint32_t uni = unis[ws];
+        mbar_arrive(&wfree[ws]);
+        if (!uni) continue;
+        const int s = u & 1, use = u >> 1;
+        if (use > 0 && !mbar_wait(&sfree[s], (use - 1) & 1, abort_flag)) { ok = false; break; }
+        const uint32_t d = tmem + AT_S_COL + 64 * s;
+        const uint64_t xd = sdesc_(smem_addr(sx + s * AT_TILE), 16);
+        for (int i = 0; i < AT_NG; ++i) {
+          const int g = i == 0 ? 4 : i - 1;
+          if (!mbar_wait(&xfull[s * AT_NG + g], use & 1, abort_flag)) { ok = false; break; }
+          tmem_fence_after();
+          if (g == 4) {
+#pragma unroll
+            for (int kk = 0; kk < 4; ++kk) {
+              const uint64_t off = (uint64_t)((8 * AT_KBLK + 32 * kk) >> 4);
+              mma_bf16_(d, qd + off, xd + off, idesc_s, kk > 0 ? 1u : 0u);
+            }
+          } else {
+#pragma unroll
+            for (int kk = 0; kk < 8; ++kk) {
+              const uint64_t off = (uint64_t)(((2 * g + (kk >> 2)) * AT_KBLK + 32 * (kk & 3)) >> 4);
+              mma_bf16_(d, qd + off, xd + off, idesc_s, 1u);
+            }
+          }
+        }
+        if (!ok) break;
+        mma_commit_(&sfull[s]);
+        mma_commit_(&xrel[s * AT_NG + 4]);             // the RoPE block is read by S only
+        if (u > 0 && !issue_av(u - 1)) { ok = false; break; }
+        ++u;
       }
-      if (!ok) { raise_status(args.status, VK_ERR_TIMEOUT); abort_flag = 1; }
+      if (ok && u > 0) ok = issue_av(u - 1);
+      mma_commit_(mdone);
+      if (!ok) { raise_status(args.status, VK_ERR_TIMEOUT); *abort_flag = 1; }
+      mbar_wait(mdone, 0, nullptr);                    // nothing this thread issued may outlive the CTA
     }
   } else {
-    // ------------------------------------------------------------------ consumers
-    const int c = warp - 2;                              // 0..15
-    const int q = warp & 3;                              // TMEM lane quarter this warp may access
-    const int sub = c >> 2;                              // which 4 heads of the quarter's 16
-    const uint32_t lane_base = (uint32_t)(q * 32) << 16;
-    float o[4][16];                                      // the 4 heads' running sums: dims 8 lane + t, 256 + 8 lane + t
-    float m2[4], lsum[4];
-#pragma unroll
-    for (int i = 0; i < 4; ++i) {
-      m2[i] = -INFINITY;
-      lsum[i] = 0.f;
-#pragma unroll
-      for (int t = 0; t < 16; ++t) o[i][t] = 0.f;
-    }
-    const int hq0 = 16 * q + 4 * sub;                    // local heads hq0 .. hq0 + 3
-
+    // ------------------------------------------------------------------ softmax
+    const int q = warp & 3;                            // TMEM lane quarter of this warp
+    const bool own = lane < 16;
+    const int hl = 16 * q + lane;                      // this lane's head (lanes 0..15)
+    const uint32_t lrow = tmem + ((uint32_t)(32 * q) << 16);
+    float m = -INFINITY, mex = -INFINITY, lsum = 0.f;
+    int u = 0;
+    bool ok = true;
     for (int t = 0; t < ntile; ++t) {
-      const int s = t % AT2_NT, use = t / AT2_NT;
-      if (!mbar_wait(&s_full[s], use & 1, &abort_flag) || !mbar_wait(&x_full[s], use & 1, &abort_flag)) {
-        if (lane == 0) { raise_status(args.status, VK_ERR_TIMEOUT); abort_flag = 1; }
-        break;
-      }
+      const int ws = t & 1;
+      if (!warp_wait_(&wfull[ws], (t >> 1) & 1, abort_flag, lane)) { ok = false; break; }
+      const uint32_t uni = unis[ws];
+      uint32_t w0 = 0u, w1 = 0u;
+      if (own) { w0 = words[ws * 128 + hl * 2]; w1 = words[ws * 128 + hl * 2 + 1]; }
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&wfree[ws]);
+      if (!uni) continue;
+      const int s = u & 1, use = u >> 1, par = u & 1;
+      if (!warp_wait_(&sfull[s], use & 1, abort_flag, lane)) { ok = false; break; }
       tmem_fence_after();
-      const unsigned char* xs = sx + s * AT2_X_BYTES;
-      const uint32_t scol = tmem_base + lane_base + AT2_S_COL0 + s * AT2_T;
-#pragma unroll
-      for (int i = 0; i < 4; ++i) {
-        const int hl = hq0 + i;
-        if (hl >= nh) break;
-        uint32_t bits = words[s * 64 + hl];
-        while (bits) {
-          const int j = __ffs(bits) - 1;
-          bits &= bits - 1;
-          // logit of (head hl, row j): TMEM lane 32 q + (4 sub + i), column j of the slot
-          const float sv = tmem_ld1(scol + j);
-          // this lane's 16 latent values of row j: dims 8 lane .. + 7 and 256 + 8 lane .. + 7, un-swizzled
-          const int ch = (lane & 7) ^ (j & 7);
-          const uint4 xa = *reinterpret_cast<const uint4*>(xs + (lane >> 3) * AT2_KBLK_X + j * 128 + ch * 16);
-          const uint4 xb = *reinterpret_cast<const uint4*>(xs + (4 + (lane >> 3)) * AT2_KBLK_X + j * 128 + ch * 16);
-          tmem_wait_ld();
-          const float s2 = __shfl_sync(0xffffffffu, sv, 4 * sub + i) * args.lam_log2e;
-          if (s2 > m2[i]) {
-            const float sc = ex2(m2[i] - s2);
-            lsum[i] *= sc;
-#pragma unroll
-            for (int tt = 0; tt < 16; ++tt) o[i][tt] *= sc;
-            m2[i] = s2;
-          }
-          const __nv_bfloat16 pb = __float2bfloat16_rn(ex2(s2 - m2[i]));
-          const uint16_t p16 = __bfloat16_as_ushort(pb);
-          lsum[i] += __bfloat162float(pb);
-          const uint32_t wa[4] = {xa.x, xa.y, xa.z, xa.w}, wb[4] = {xb.x, xb.y, xb.z, xb.w};
-#pragma unroll
-          for (int k = 0; k < 4; ++k) {
-            o[i][2 * k] = fma_bf16(p16, lo16_(wa[k]), o[i][2 * k]);
-            o[i][2 * k + 1] = fma_bf16(p16, hi16_(wa[k]), o[i][2 * k + 1]);
-            o[i][8 + 2 * k] = fma_bf16(p16, lo16_(wb[k]), o[i][8 + 2 * k]);
-            o[i][8 + 2 * k + 1] = fma_bf16(p16, hi16_(wb[k]), o[i][8 + 2 * k + 1]);
-          }
-        }
-      }
+      float sv[64];
+      tmem_ld32_(lrow + AT_S_COL + 64 * s, sv);
+      tmem_ld32_(lrow + AT_S_COL + 64 * s + 32, sv + 32);
+      tmem_wait_ld();
       tmem_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive(&x_empty[s]);
-    }
-    // partials: part_o [B][nslot][H][512] (unnormalised), part_ml [B][nslot][H][2] = (max logit, sum)
-    const int slot = args.slot0 + split;
-    constexpr float LN2 = 0.6931471805599453f;
+      if (lane == 0) mbar_arrive(&sfree[s]);
+      // tile max over the selected rows, in log2 units
+      float mt = -INFINITY;
 #pragma unroll
-    for (int i = 0; i < 4; ++i) {
-      const int hl = hq0 + i;
-      if (hl >= nh) break;
-      const int64_t base = (((int64_t)b * args.nslot + slot) * H + h0 + hl);
-      float4* d0 = reinterpret_cast<float4*>(args.part_o + base * D_LAT + lane * 8);
-      float4* d1 = reinterpret_cast<float4*>(args.part_o + base * D_LAT + 256 + lane * 8);
-      d0[0] = make_float4(o[i][0], o[i][1], o[i][2], o[i][3]);
-      d0[1] = make_float4(o[i][4], o[i][5], o[i][6], o[i][7]);
-      d1[0] = make_float4(o[i][8], o[i][9], o[i][10], o[i][11]);
-      d1[1] = make_float4(o[i][12], o[i][13], o[i][14], o[i][15]);
-      if (lane == 0) { args.part_ml[base * 2] = m2[i] * LN2; args.part_ml[base * 2 + 1] = lsum[i]; }
+      for (int c = 0; c < 32; ++c) {
+        sv[c] *= args.lam_log2e;
+        sv[c + 32] *= args.lam_log2e;
+        if ((w0 >> c) & 1u) mt = fmaxf(mt, sv[c]);
+        if ((w1 >> c) & 1u) mt = fmaxf(mt, sv[c + 32]);
+      }
+      mex = fmaxf(mex, mt);
+      float f = 1.f;
+      if (mt > m + AT_TAU) {                           // includes the head's first selected row (m = -inf)
+        if (m != -INFINITY) f = ex2(m - mt);
+        m = mt;
+        lsum *= f;
+      }
+      uint32_t pk[32];
+#pragma unroll
+      for (int c = 0; c < 64; c += 2) {
+        const uint32_t wb = c < 32 ? w0 : w1;
+        const int cb = c & 31;
+        const float e0 = ((wb >> cb) & 1u) ? ex2(sv[c] - m) : 0.f;
+        const float e1 = ((wb >> (cb + 1)) & 1u) ? ex2(sv[c + 1] - m) : 0.f;
+        const __nv_bfloat162 pb = __floats2bfloat162_rn(e0, e1);
+        lsum += __low2float(pb) + __high2float(pb);
+        pk[c >> 1] = *reinterpret_cast<const uint32_t*>(&pb);
+      }
+      // publish this group's rescale factors (by tile parity: a warp that runs ahead writes the other buffer)
+      const uint32_t need = __ballot_sync(0xffffffffu, own && f != 1.f);
+      if (own) fac[par * 64 + hl] = f;
+      if (lane == 0) anyw[par * 4 + q] = need;
+      // the previous tile's O^T product must be complete: it reads P^T, and O^T may be rescaled now
+      if (u > 0 && !warp_wait_(pfree, (u - 1) & 1, abort_flag, lane)) { ok = false; break; }
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&gbar[par]);
+      if (!warp_wait_(&gbar[par], use & 1, abort_flag, lane)) { ok = false; break; }
+      if (anyw[par * 4] | anyw[par * 4 + 1] | anyw[par * 4 + 2] | anyw[par * 4 + 3]) {
+        tmem_fence_after();
+        for (int h = 0; h < 64; ++h) {
+          const float fh = fac[par * 64 + h];
+          if (fh != 1.f) {
+#pragma unroll
+            for (int j = 0; j < 4; ++j) {
+              const uint32_t a = lrow + AT_O_COL + 64 * j + h;
+              const float v = tmem_ld1_(a);
+              tmem_wait_ld();
+              tmem_st1_(a, v * fh);
+            }
+          }
+        }
+        tmem_wait_st();
+      }
+      if (own) {
+        unsigned char* row = sp + hl * 128;
+#pragma unroll
+        for (int c8 = 0; c8 < 8; ++c8)
+          *reinterpret_cast<uint4*>(row + ((c8 ^ (hl & 7)) * 16)) =
+              make_uint4(pk[4 * c8], pk[4 * c8 + 1], pk[4 * c8 + 2], pk[4 * c8 + 3]);
+      }
+      fence_async_smem_();
+      tmem_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(pfull);
+      ++u;
+    }
+    // the last O^T product
+    if (ok && u > 0) ok = warp_wait_(pfree, (u - 1) & 1, abort_flag, lane);
+    if (ok) {
+      // re-base each head on its exact max; the factors go through the parity buffer the last tile did not use
+      float ff = 1.f;
+      if (own && mex != -INFINITY && m != mex) ff = ex2(m - mex);
+      lsum *= ff;
+      float* facf = fac + (u & 1) * 64;
+      if (own) facf[hl] = ff;
+      __syncwarp();
+      if (lane == 0) mbar_arrive(ebar);
+      ok = warp_wait_(ebar, 0, abort_flag, lane);
+    }
+    if (ok) {
+      tmem_fence_after();
+      const float* facf = fac + (u & 1) * 64;
+      const int slot = args.slot0 + split;
+      const int64_t hbase = ((int64_t)b * args.nslot + slot) * H + h0;
+      constexpr float LN2 = 0.6931471805599453f;
+      if (own && hl < nh) {
+        args.part_ml[(hbase + hl) * 2] = mex * LN2;
+        args.part_ml[(hbase + hl) * 2 + 1] = lsum;
+      }
+      // O^T block j on this warp's lanes: dims 128 j + 32 q + lane; columns: heads
+#pragma unroll 1
+      for (int j = 0; j < 4; ++j) {
+        const int dim = 128 * j + 32 * q + lane;
+#pragma unroll 1
+        for (int c = 0; c < 64; c += 32) {
+          float v[32];
+          if (u > 0) {
+            tmem_ld32_(lrow + AT_O_COL + 64 * j + c, v);
+            tmem_wait_ld();
+          } else {
+#pragma unroll
+            for (int i = 0; i < 32; ++i) v[i] = 0.f;
+          }
+#pragma unroll
+          for (int i = 0; i < 32; ++i)
+            if (c + i < nh) args.part_o[(hbase + c + i) * D_LAT + dim] = v[i] * facf[c + i];
+        }
+      }
+    } else if (lane == 0) {
+      raise_status(args.status, VK_ERR_TIMEOUT);
+      *abort_flag = 1;
     }
   }
 
-  // wind down: nothing may still write this CTA's shared or tensor memory
+  // every role has finished its waits and its tensor-memory accesses: release tensor memory
   tmem_fence_before();
   __syncthreads();
-  if (warp == 0 && lane == 0) {
-    // drain tile loads that were issued but never consumed (only after an abort)
-    for (int s = 0; s < AT2_NT && s < ntile; ++s) {
-      const int last = (ntile - 1 - s) / AT2_NT;
-      mbar_wait(&x_full[s], last & 1, nullptr);
-    }
+  if (warp == 1) {
+    tmem_fence_after();
+    tmem_dealloc(tmem, AT_TMEM_COLS);
   }
-  __syncthreads();
-  tmem_fence_after();
-  if (warp == 1) tmem_dealloc(tmem_base, AT2_TMEM_COLS);
 }
 
 // ---------------------------------------------------------------------------------------------- host side
@@ -349,14 +521,15 @@ static bool make_map3(CUtensorMap* map, const void* base, uint64_t cols, uint64_
 cudaError_t launch_attn_tc(const vk_view& v, float lam, const uint32_t* bitmap, int64_t nw, int nsplit, int split_len,
                            int slot0, int nslot, float* part_o, float* part_ml, int* status, cudaStream_t st) {
   if (!encode2()) return cudaErrorNotSupported;
+  if (split_len % AT_T != 0) return cudaErrorInvalidValue;
   CUtensorMap lmap, rmap, qlmap, qrmap;
-  // cache rows: latent [B][N][512] and RoPE [B][N][64], 32-row boxes; queries: [B*H][512] and [B*H][64], 64-row boxes
-  if (!make_map3(&lmap, v.latent, D_LAT, v.N, v.B, v.latent_ld, v.latent_bstride, AT2_T) ||
-      !make_map3(&rmap, v.rope, D_ROPE, v.N, v.B, v.rope_ld, v.rope_bstride, AT2_T) ||
+  // cache rows: latent [B][N][512] and RoPE [B][N][64]; queries: [B*H][512] and [B*H][64]; 64-row boxes
+  if (!make_map3(&lmap, v.latent, D_LAT, v.N, v.B, v.latent_ld, v.latent_bstride, AT_T) ||
+      !make_map3(&rmap, v.rope, D_ROPE, v.N, v.B, v.rope_ld, v.rope_bstride, AT_T) ||
       !make_map3(&qlmap, v.q_latent, D_LAT, (uint64_t)v.B * v.H, 1, D_LAT, (int64_t)v.B * v.H * D_LAT, 64) ||
       !make_map3(&qrmap, v.q_rope, D_ROPE, (uint64_t)v.B * v.H, 1, D_ROPE, (int64_t)v.B * v.H * D_ROPE, 64))
     return cudaErrorInvalidValue;
-  Attn2Args a{};
+  AttnTcArgs a{};
   a.H = v.H;
   a.N = v.N;
   a.split_len = split_len;
@@ -368,11 +541,11 @@ cudaError_t launch_attn_tc(const vk_view& v, float lam, const uint32_t* bitmap, 
   a.part_o = part_o;
   a.part_ml = part_ml;
   a.status = status;
-  const size_t smem = Attn2Smem().total;
+  const size_t smem = AtSmem::total + 1024;
   cudaError_t e = cudaFuncSetAttribute(k_attn_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
   dim3 grid(nsplit, (v.H + 63) / 64, v.B);
-  k_attn_tc<<<grid, AT2_THREADS, smem, st>>>(lmap, rmap, qlmap, qrmap, a);
+  k_attn_tc<<<grid, AT_THREADS, smem, st>>>(lmap, rmap, qlmap, qrmap, a);
   count_launches(1);
   return cudaGetLastError();
 }

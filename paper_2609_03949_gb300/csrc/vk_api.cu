@@ -106,18 +106,18 @@ int check_index(const vk_view* v, const vk_params* p, const vk_index* ix, bool n
 
 size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
-// Positions per attention split. One attention CTA is resident per SM, so the split count is chosen to fill
-// the 152 SMs in whole waves: maximise (work) / (waves x 152 x positions per CTA), preferring longer splits
-// (fewer partials to merge) when two counts are equally good.
+// Positions per attention split, a multiple of 64 (the attention tile). One attention CTA is resident per SM,
+// so the split count is chosen to fill the 152 SMs in whole waves: maximise (work) / (waves x 152 x positions
+// per CTA), preferring longer splits (fewer partials to merge) when two counts are equally good.
 void choose_splits(const vk_view& v, int64_t* nsplit, int64_t* split_len) {
   const int64_t per_pos = (int64_t)v.B * ((v.H + vk::HG - 1) / vk::HG);
   const int64_t N = v.N;
   const int64_t lo = std::max<int64_t>(1, (N + 16383) / 16384);
   const int64_t hi = std::max<int64_t>(lo, std::min<int64_t>((N + 255) / 256, 2048));
   double best = -1.0;
-  int64_t best_len = ((N + 31) / 32) * 32;
+  int64_t best_len = ((N + 63) / 64) * 64;
   for (int64_t ns = lo; ns <= hi; ++ns) {
-    const int64_t len = ((N + ns - 1) / ns + 31) / 32 * 32;
+    const int64_t len = ((N + ns - 1) / ns + 63) / 64 * 64;
     const int64_t ns_eff = (N + len - 1) / len;
     const int64_t ctas = per_pos * ns_eff;
     const int64_t waves = (ctas + NUM_SMS_TARGET - 1) / NUM_SMS_TARGET;
