@@ -6,15 +6,18 @@
 //                      columns (128-byte swizzle, one 8 KB block per 64 columns) as five groups -- the RoPE block
 //                      first, then four pairs of latent blocks, each as soon as the tile before it in that slot has
 //                      released it -- into one of two tile slots;
-//   warp 1 (MMA)       S = Q . X^T on tcgen05 (M = 64 heads, N = 64 rows, K = 576: 36 instructions) into one of two
-//                      S buffers in tensor memory; with M = 64 the logit of head 16 g + i and row j sits in TMEM lane
-//                      32 g + i, column j. Then, once the softmax warps have written P^T, O^T += X_lat^T . P^T
-//                      (M = 128 latent dims x 4 blocks, N = 64 heads, K = 64 rows: 16 instructions) into the O^T
-//                      accumulator, which stays in tensor memory for the whole range. X_lat^T is read straight from
-//                      the tile slot as an MN-major operand (the next 64 dims one 8 KB block away), so each latent
-//                      row is staged in shared memory once and feeds both contractions;
-//   warps 2..5         softmax: lane i < 16 of the warp on TMEM lane quarter g owns head 16 g + i. It reads its 64
-//                      logits, masks them with its selection words and writes P^T[h][row] = 2^(s lambda log2(e) - m_h)
+//   warp 1 (S)         S = Q . X^T on tcgen05 (M = 64 heads, N = 64 rows, K = 576: 36 instructions, issued group by
+//                      group as the loads land) into one of two S buffers in tensor memory; with M = 64 the logit
+//                      of head 16 g + i and row j sits in TMEM lane 32 g + i, column j;
+//   warp 6 (O^T)       once the softmax warps have written P^T, O^T += X_lat^T . P^T (M = 128 latent dims x 4
+//                      blocks, N = 64 heads, K = 64 rows: 16 instructions) into the O^T accumulator, which stays in
+//                      tensor memory for the whole range. X_lat^T is read straight from the tile slot as an MN-major
+//                      operand (the next 64 dims one 8 KB block away), so each latent row is staged in shared memory
+//                      once and feeds both contractions. Two issuing threads, so neither contraction waits behind
+//                      the other's issue;
+//   warps 2..5         softmax: lanes i and 16 + i of the warp on TMEM lane quarter g own head 16 g + i, rows 0..31
+//                      and 32..63 of the tile. They read the head's logits, mask them with its selection words,
+//                      and write P^T[h][row] = 2^(s lambda log2(e) - m_h)
 //                      (0 where the head did not select the row) in bf16 into shared memory (K-major, 128-byte
 //                      swizzle). m_h is a running max that only moves when a tile's max exceeds it by more than 8
 //                      (log2 units; the head's O^T column and sum are then rescaled in tensor memory), so rescaling
@@ -35,7 +38,7 @@ namespace vk {
 
 constexpr int AT_T = 64;                               // rows per tile
 constexpr int AT_SMX = 4;                              // softmax warps (one per TMEM lane quarter)
-constexpr int AT_THREADS = (2 + AT_SMX) * 32;
+constexpr int AT_THREADS = (3 + AT_SMX) * 32;   // producer, S issuer, softmax x4, O^T issuer
 constexpr uint32_t AT_KBLK = 64 * 128;                 // one 64-column block of 64 rows (or 64 heads): 8 KB
 constexpr uint32_t AT_TILE = 9 * AT_KBLK;              // 73,728: one tile slot, and the queries
 constexpr uint32_t AT_P = 64 * 128;                    // P^T: 64 heads x 64 rows, bf16
@@ -46,7 +49,7 @@ constexpr uint32_t AT_S_COL = 0;                       // S buffers: columns 0..
 constexpr uint32_t AT_O_COL = 128;                     // O^T block j: columns 128 + 64 j .. + 63
 
 // Shared memory, from a 1024-byte aligned base. Barriers: xfull/xrel [2 slots][5 groups], sfull/sfree [2],
-// wfull/wfree [2], pfull, pfree, qfull, mdone, gbar [2], ebar.
+// wfull/wfree [2], pfull, pfree, qfull, mdone, gbar [2], ebar, adone.
 struct AtSmem {
   static constexpr uint32_t q = 0;
   static constexpr uint32_t x = q + AT_TILE;
@@ -57,7 +60,7 @@ struct AtSmem {
   static constexpr uint32_t anyw = fac + 2 * 64 * 4;   // [2][4] u32
   static constexpr uint32_t misc = anyw + 2 * 4 * 4;   // TMEM base, abort flag
   static constexpr uint32_t bars = (misc + 8 + 7) & ~7u;
-  static constexpr uint32_t nbars = 2 * AT_NG * 2 + 2 * 4 + 4 + 3;
+  static constexpr uint32_t nbars = 2 * AT_NG * 2 + 2 * 4 + 4 + 3 + 1;
   static constexpr uint32_t total = bars + nbars * 8;
 };
 static_assert(AtSmem::total + 1024 <= 232448, "attention shared memory exceeds the 227 KB opt-in limit");
@@ -156,6 +159,7 @@ __global__ void __launch_bounds__(AT_THREADS, 1) k_attn_tc(const __grid_constant
   uint64_t* mdone = qfull + 1;
   uint64_t* gbar = mdone + 1;                 // [2] softmax-group syncs, by tile parity
   uint64_t* ebar = gbar + 2;                  // softmax-group sync before the epilogue
+  uint64_t* adone = ebar + 1;                 // O^T issuer's final commit
 
   const int split = blockIdx.x, hg = blockIdx.y, b = blockIdx.z;
   const int H = args.H;
@@ -171,7 +175,7 @@ __global__ void __launch_bounds__(AT_THREADS, 1) k_attn_tc(const __grid_constant
       mbar_init(&sfull[i], 1);
       mbar_init(&sfree[i], AT_SMX);
       mbar_init(&wfull[i], 1);
-      mbar_init(&wfree[i], AT_SMX + 1);
+      mbar_init(&wfree[i], AT_SMX + 2);
       mbar_init(&gbar[i], AT_SMX);
     }
     mbar_init(pfull, AT_SMX);
@@ -179,6 +183,7 @@ __global__ void __launch_bounds__(AT_THREADS, 1) k_attn_tc(const __grid_constant
     mbar_init(qfull, 1);
     mbar_init(mdone, 1);
     mbar_init(ebar, AT_SMX);
+    mbar_init(adone, 1);
     mbar_fence_init();
   }
   if (warp == 1) tmem_alloc(tmem_slot, AT_TMEM_COLS);
@@ -272,48 +277,28 @@ __global__ void __launch_bounds__(AT_THREADS, 1) k_attn_tc(const __grid_constant
         if (last_use[i] >= 0) mbar_wait(&xfull[i], last_use[i] & 1, nullptr);
     }
   } else if (warp == 1) {
-    // ------------------------------------------------------------------ MMA issuer
+    // ------------------------------------------------------------------ S issuer
+    // Blocks on each load group in turn and issues its part of S = Q . X^T as soon as it lands.
     if (lane == 0 && ntile > 0) {
       // S: M = 64 heads, N = 64 rows, A = Q and B = X, both K-major
       const uint32_t idesc_s =
           (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(AT_T >> 3) << 17) | ((uint32_t)(64 >> 4) << 24);
-      // O^T: M = 128 dims, N = 64 heads, A = X_lat^T MN-major (bit 15), B = P^T K-major
-      const uint32_t idesc_o =
-          (1u << 4) | (1u << 7) | (1u << 10) | (1u << 15) | ((uint32_t)(64 >> 3) << 17) | ((uint32_t)(128 >> 4) << 24);
       const uint64_t qd = sdesc_(smem_addr(sq), 16);
-      const uint64_t pd = sdesc_(smem_addr(sp), 16);
       bool ok = mbar_wait(qfull, 0, abort_flag);
       int u = 0;
-      auto issue_av = [&](int v) -> bool {
-        const int s = v & 1;
-        if (!mbar_wait(pfull, v & 1, abort_flag)) return false;
-        tmem_fence_after();
-        const uint64_t xd = sdesc_(smem_addr(sx + s * AT_TILE), AT_KBLK);
-#pragma unroll
-        for (int j = 0; j < 4; ++j) {
-#pragma unroll
-          for (int ks = 0; ks < 4; ++ks)
-            mma_bf16_(tmem + AT_O_COL + 64 * j, xd + (uint64_t)((2 * j * AT_KBLK + ks * 2048) >> 4),
-                      pd + (uint64_t)(ks * 2), idesc_o, (v > 0 || ks > 0) ? 1u : 0u);
-          mma_commit_(&xrel[s * AT_NG + j]);           // latent blocks 2j, 2j+1 of this slot are free again
-        }
-        mma_commit_(pfree);                            // P^T free, O^T up to date
-        return true;
-      };
       for (int t = 0; t < ntile && ok; ++t) {
-        const int ws = t & 1;
-        if (!mbar_wait(&wfull[ws], (t >> 1) & 1, abort_flag)) { ok = false; break; }
-        const uint32_t uni = unis[ws];
-        mbar_arrive(&wfree[ws]);
+        if (!mbar_wait(&wfull[t & 1], (t >> 1) & 1, abort_flag)) { ok = false; break; }
+        const uint32_t uni = unis[t & 1];
+        mbar_arrive(&wfree[t & 1]);
         if (!uni) continue;
         const int s = u & 1, use = u >> 1;
         if (use > 0 && !mbar_wait(&sfree[s], (use - 1) & 1, abort_flag)) { ok = false; break; }
         const uint32_t d = tmem + AT_S_COL + 64 * s;
         const uint64_t xd = sdesc_(smem_addr(sx + s * AT_TILE), 16);
-        for (int i = 0; i < AT_NG; ++i) {
-          const int g = i == 0 ? 4 : i - 1;
+        // operands land by TMA and are observed through the mbarrier: no tensor-memory fence is needed
+        for (int i = 0; i < AT_NG && ok; ++i) {
+          const int g = i == 0 ? 4 : i - 1;            // RoPE block first
           if (!mbar_wait(&xfull[s * AT_NG + g], use & 1, abort_flag)) { ok = false; break; }
-          tmem_fence_after();
           if (g == 4) {
 #pragma unroll
             for (int kk = 0; kk < 4; ++kk) {
@@ -331,51 +316,99 @@ __global__ void __launch_bounds__(AT_THREADS, 1) k_attn_tc(const __grid_constant
         if (!ok) break;
         mma_commit_(&sfull[s]);
         mma_commit_(&xrel[s * AT_NG + 4]);             // the RoPE block is read by S only
-        if (u > 0 && !issue_av(u - 1)) { ok = false; break; }
         ++u;
       }
-      if (ok && u > 0) ok = issue_av(u - 1);
       mma_commit_(mdone);
       if (!ok) { raise_status(args.status, VK_ERR_TIMEOUT); *abort_flag = 1; }
       mbar_wait(mdone, 0, nullptr);                    // nothing this thread issued may outlive the CTA
     }
+  } else if (warp == 2 + AT_SMX) {
+    // ------------------------------------------------------------------ O^T issuer
+    // Issues each loaded tile's O^T += X_lat^T . P^T as soon as its P^T is written; its commits release the tile's
+    // latent blocks for the next load into the slot. (A commit tracks this thread's own MMAs; the tile's S, issued
+    // by the other thread, completed before its softmax could start.)
+    if (lane == 0 && ntile > 0) {
+      // O^T: M = 128 dims, N = 64 heads, A = X_lat^T MN-major (bit 15), B = P^T K-major
+      const uint32_t idesc_o =
+          (1u << 4) | (1u << 7) | (1u << 10) | (1u << 15) | ((uint32_t)(64 >> 3) << 17) | ((uint32_t)(128 >> 4) << 24);
+      const uint64_t pd = sdesc_(smem_addr(sp), 16);
+      bool ok = true;
+      int u = 0;
+      for (int t = 0; t < ntile; ++t) {
+        if (!mbar_wait(&wfull[t & 1], (t >> 1) & 1, abort_flag)) { ok = false; break; }
+        const uint32_t uni = unis[t & 1];
+        mbar_arrive(&wfree[t & 1]);
+        if (!uni) continue;
+        if (!mbar_wait(pfull, u & 1, abort_flag)) { ok = false; break; }
+        tmem_fence_after();                            // P^T and any O^T rescale come from the softmax warps
+        const int s = u & 1;
+        const uint64_t xd = sdesc_(smem_addr(sx + s * AT_TILE), AT_KBLK);
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+#pragma unroll
+          for (int ks = 0; ks < 4; ++ks)
+            mma_bf16_(tmem + AT_O_COL + 64 * j, xd + (uint64_t)((2 * j * AT_KBLK + ks * 2048) >> 4),
+                      pd + (uint64_t)(ks * 2), idesc_o, (u > 0 || ks > 0) ? 1u : 0u);
+          mma_commit_(&xrel[s * AT_NG + j]);           // latent blocks 2j, 2j+1 of this slot are free again
+        }
+        mma_commit_(pfree);                            // P^T free, O^T up to date
+        ++u;
+      }
+      mma_commit_(adone);
+      if (!ok) { raise_status(args.status, VK_ERR_TIMEOUT); *abort_flag = 1; }
+      mbar_wait(adone, 0, nullptr);
+    }
   } else {
     // ------------------------------------------------------------------ softmax
+    // Head hl = 16 q + (lane % 16); lanes 0..15 take rows 0..31 of the tile, lanes 16..31 rows 32..63 (one
+    // tcgen05.ld 16x32bx2 gives each half its 32 columns of the same 16 TMEM lanes).
     const int q = warp & 3;                            // TMEM lane quarter of this warp
-    const bool own = lane < 16;
-    const int hl = 16 * q + lane;                      // this lane's head (lanes 0..15)
+    const int hh = lane >> 4;                          // which half of the tile's rows
+    const int hl = 16 * q + (lane & 15);               // this lane's head
+    const bool own = hh == 0;                          // the lane that publishes per-head values
+    const float L = args.lam_log2e;
     const uint32_t lrow = tmem + ((uint32_t)(32 * q) << 16);
-    float m = -INFINITY, mex = -INFINITY, lsum = 0.f;
+    float m = -INFINITY, mex = -INFINITY, lsum = 0.f;  // lsum: this half's share of the head's sum
     int u = 0;
     bool ok = true;
     for (int t = 0; t < ntile; ++t) {
       const int ws = t & 1;
       if (!warp_wait_(&wfull[ws], (t >> 1) & 1, abort_flag, lane)) { ok = false; break; }
       const uint32_t uni = unis[ws];
-      uint32_t w0 = 0u, w1 = 0u;
-      if (own) { w0 = words[ws * 128 + hl * 2]; w1 = words[ws * 128 + hl * 2 + 1]; }
+      const uint32_t w = words[ws * 128 + hl * 2 + hh];
       __syncwarp();
       if (lane == 0) mbar_arrive(&wfree[ws]);
       if (!uni) continue;
       const int s = u & 1, use = u >> 1, par = u & 1;
       if (!warp_wait_(&sfull[s], use & 1, abort_flag, lane)) { ok = false; break; }
       tmem_fence_after();
-      float sv[64];
-      tmem_ld32_(lrow + AT_S_COL + 64 * s, sv);
-      tmem_ld32_(lrow + AT_S_COL + 64 * s + 32, sv + 32);
+      float sv[32];
+      {
+        uint32_t* r = reinterpret_cast<uint32_t*>(sv);
+        asm volatile(
+            "tcgen05.ld.sync.aligned.16x32bx2.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16,%17,"
+            "%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32], 32;\n"
+            : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+              "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]),
+              "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]),
+              "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+            : "r"(lrow + AT_S_COL + 64 * s)
+            : "memory");
+      }
       tmem_wait_ld();
       tmem_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(&sfree[s]);
-      // tile max over the selected rows, in log2 units
-      float mt = -INFINITY;
+      // the head's tile max over its selected rows (lambda log2(e) > 0 commutes with max)
+      float mr0 = -INFINITY, mr1 = -INFINITY;
 #pragma unroll
-      for (int c = 0; c < 32; ++c) {
-        sv[c] *= args.lam_log2e;
-        sv[c + 32] *= args.lam_log2e;
-        if ((w0 >> c) & 1u) mt = fmaxf(mt, sv[c]);
-        if ((w1 >> c) & 1u) mt = fmaxf(mt, sv[c + 32]);
+      for (int c = 0; c < 32; c += 2) {
+        if ((w >> c) & 1u) mr0 = fmaxf(mr0, sv[c]);
+        if ((w >> (c + 1)) & 1u) mr1 = fmaxf(mr1, sv[c + 1]);
       }
+      float mr = fmaxf(mr0, mr1);
+      mr = fmaxf(mr, __shfl_xor_sync(0xffffffffu, mr, 16));
+      const float mt = mr * L;
       mex = fmaxf(mex, mt);
       float f = 1.f;
       if (mt > m + AT_TAU) {                           // includes the head's first selected row (m = -inf)
@@ -383,17 +416,19 @@ __global__ void __launch_bounds__(AT_THREADS, 1) k_attn_tc(const __grid_constant
         m = mt;
         lsum *= f;
       }
-      uint32_t pk[32];
+      uint32_t pk[16];
+      float ls0 = 0.f, ls1 = 0.f;
 #pragma unroll
-      for (int c = 0; c < 64; c += 2) {
-        const uint32_t wb = c < 32 ? w0 : w1;
-        const int cb = c & 31;
-        const float e0 = ((wb >> cb) & 1u) ? ex2(sv[c] - m) : 0.f;
-        const float e1 = ((wb >> (cb + 1)) & 1u) ? ex2(sv[c + 1] - m) : 0.f;
+      for (int c = 0; c < 32; c += 2) {
+        const float e0 = ((w >> c) & 1u) ? ex2(fmaf(sv[c], L, -m)) : 0.f;
+        const float e1 = ((w >> (c + 1)) & 1u) ? ex2(fmaf(sv[c + 1], L, -m)) : 0.f;
         const __nv_bfloat162 pb = __floats2bfloat162_rn(e0, e1);
-        lsum += __low2float(pb) + __high2float(pb);
-        pk[c >> 1] = *reinterpret_cast<const uint32_t*>(&pb);
+        const uint32_t bits = *reinterpret_cast<const uint32_t*>(&pb);
+        ls0 += __uint_as_float(bits << 16);            // the rounded values: what the tensor core multiplies
+        ls1 += __uint_as_float(bits & 0xffff0000u);
+        pk[c >> 1] = bits;
       }
+      lsum += ls0 + ls1;
       // publish this group's rescale factors (by tile parity: a warp that runs ahead writes the other buffer)
       const uint32_t need = __ballot_sync(0xffffffffu, own && f != 1.f);
       if (own) fac[par * 64 + hl] = f;
@@ -419,12 +454,13 @@ __global__ void __launch_bounds__(AT_THREADS, 1) k_attn_tc(const __grid_constant
         }
         tmem_wait_st();
       }
-      if (own) {
+      {
+        // P^T row hl, rows 32 hh .. + 31 of the tile: four 16-byte chunks, 128-byte swizzle
         unsigned char* row = sp + hl * 128;
 #pragma unroll
-        for (int c8 = 0; c8 < 8; ++c8)
-          *reinterpret_cast<uint4*>(row + ((c8 ^ (hl & 7)) * 16)) =
-              make_uint4(pk[4 * c8], pk[4 * c8 + 1], pk[4 * c8 + 2], pk[4 * c8 + 3]);
+        for (int i = 0; i < 4; ++i)
+          *reinterpret_cast<uint4*>(row + (((4 * hh + i) ^ (hl & 7)) * 16)) =
+              make_uint4(pk[4 * i], pk[4 * i + 1], pk[4 * i + 2], pk[4 * i + 3]);
       }
       fence_async_smem_();
       tmem_fence_before();
@@ -434,10 +470,11 @@ __global__ void __launch_bounds__(AT_THREADS, 1) k_attn_tc(const __grid_constant
     }
     // the last O^T product
     if (ok && u > 0) ok = warp_wait_(pfree, (u - 1) & 1, abort_flag, lane);
+    lsum += __shfl_xor_sync(0xffffffffu, lsum, 16);    // both halves of the head
     if (ok) {
       // re-base each head on its exact max; the factors go through the parity buffer the last tile did not use
       float ff = 1.f;
-      if (own && mex != -INFINITY && m != mex) ff = ex2(m - mex);
+      if (mex != -INFINITY && m != mex) ff = ex2(m - mex);
       lsum *= ff;
       float* facf = fac + (u & 1) * 64;
       if (own) facf[hl] = ff;
@@ -479,7 +516,6 @@ __global__ void __launch_bounds__(AT_THREADS, 1) k_attn_tc(const __grid_constant
       *abort_flag = 1;
     }
   }
-
   // every role has finished its waits and its tensor-memory accesses: release tensor memory
   tmem_fence_before();
   __syncthreads();

@@ -1,13 +1,21 @@
 // vk_ptx.cuh -- inline-PTX wrappers for sm_103a: mbarriers, bulk (TMA) copies, bounded waits.
 //
-// Every wait on an mbarrier is bounded: it gives up after a fixed number of polls (a few seconds at most),
-// so a kernel that meets a copy that never lands reports VK_ERR_TIMEOUT instead of hanging the GPU.
+// Every wait on an mbarrier is bounded in time: it gives up after kWaitNs of the GPU's global timer (a poll of
+// mbarrier.try_wait may itself suspend for a system-defined while, so a count of polls is no time bound), and a
+// kernel that meets a copy that never lands reports VK_ERR_TIMEOUT instead of hanging the GPU.
 #pragma once
 #include <stdint.h>
 
 namespace vk {
 
-constexpr uint32_t kWaitPolls = 1u << 24;   // try_wait polls before a wait gives up
+constexpr uint64_t kWaitNs = 1000000000ull;  // a wait gives up after 1 s
+
+// Nanoseconds of the GPU's global timer.
+__device__ __forceinline__ uint64_t global_ns() {
+  uint64_t t;
+  asm volatile("mov.u64 %0, %%globaltimer;\n" : "=l"(t));
+  return t;
+}
 
 __device__ __forceinline__ uint32_t smem_addr(const void* p) {
   return static_cast<uint32_t>(__cvta_generic_to_shared(p));
@@ -43,14 +51,31 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
   return ok != 0;
 }
 
-// Wait until the phase with this parity has completed. Returns false if it gave up (after kWaitPolls polls,
-// or earlier once *abort is set by another warp that gave up).
+// Non-blocking test of the same condition (try_wait may suspend the thread for a while; an event loop that
+// polls several barriers must not).
+__device__ __forceinline__ bool mbar_test_wait(uint64_t* bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n .reg .pred p;\n mbarrier.test_wait.parity.acquire.cta.shared::cta.b64 p, [%1], %2;\n"
+      " selp.u32 %0, 1, 0, p;\n}\n"
+      : "=r"(ok)
+      : "r"(smem_addr(bar)), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+
+// Wait until the phase with this parity has completed. Returns false if it gave up (after kWaitNs, or earlier
+// once *abort is set by another warp that gave up).
 __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volatile int* abort) {
-  for (uint32_t it = 0; it < kWaitPolls; ++it) {
+  if (mbar_try_wait(bar, parity)) return true;
+  const uint64_t t0 = global_ns();
+  for (uint32_t it = 1;; ++it) {
     if (mbar_try_wait(bar, parity)) return true;
-    if ((it & 63u) == 63u && abort && *abort) return false;
+    if ((it & 15u) == 0u) {
+      if (abort && *abort) return false;
+      if (global_ns() - t0 > kWaitNs) return false;
+    }
   }
-  return false;
 }
 
 // Bulk copy global -> shared memory of this CTA, completing `bytes` of transaction on `bar`.
