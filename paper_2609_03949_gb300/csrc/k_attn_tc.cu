@@ -6,8 +6,8 @@
 //                      columns (128-byte swizzle, one 8 KB block per 64 columns) as five groups -- the RoPE block
 //                      first, then four pairs of latent blocks, each as soon as the tile before it in that slot has
 //                      released it -- into one of two tile slots;
-//   warp 1 (S)         S = Q . X^T on tcgen05 (M = 64 heads, N = 64 rows, K = 576: 36 instructions, issued group by
-//                      group as the loads land) into one of two S buffers in tensor memory; with M = 64 the logit
+//   warp 1 (S)         S = Q . X^T on tcgen05 (M = 64 heads, N = 64 rows, K = 576: 36 instructions, issued as one
+//                      burst once the tile has landed) into one of two S buffers in tensor memory; with M = 64 the logit
 //                      of head 16 g + i and row j sits in TMEM lane 32 g + i, column j;
 //   warp 6 (O^T)       once the softmax warps have written P^T, O^T += X_lat^T . P^T (M = 128 latent dims x 4
 //                      blocks, N = 64 heads, K = 64 rows: 16 instructions) into the O^T accumulator, which stays in
@@ -250,7 +250,7 @@ __global__ void __launch_bounds__(AT_THREADS, 1) k_attn_tc(const __grid_constant
         bool lok = true;
         if (lane == 0) {
           for (int i = 0; i < AT_NG; ++i) {
-            const int g = i == 0 ? 4 : i - 1;          // RoPE block first: S can start on it
+            const int g = i == 0 ? 4 : i - 1;          // RoPE block first (its slot part is released first)
             uint64_t* fb = &xfull[s * AT_NG + g];
             if (use > 0 && !mbar_wait(&xrel[s * AT_NG + g], (use - 1) & 1, abort_flag)) { lok = false; break; }
             if (g == 4) {
@@ -278,7 +278,6 @@ __global__ void __launch_bounds__(AT_THREADS, 1) k_attn_tc(const __grid_constant
     }
   } else if (warp == 1) {
     // ------------------------------------------------------------------ S issuer
-    // Blocks on each load group in turn and issues its part of S = Q . X^T as soon as it lands.
     if (lane == 0 && ntile > 0) {
       // S: M = 64 heads, N = 64 rows, A = Q and B = X, both K-major
       const uint32_t idesc_s =
@@ -295,22 +294,16 @@ __global__ void __launch_bounds__(AT_THREADS, 1) k_attn_tc(const __grid_constant
         if (use > 0 && !mbar_wait(&sfree[s], (use - 1) & 1, abort_flag)) { ok = false; break; }
         const uint32_t d = tmem + AT_S_COL + 64 * s;
         const uint64_t xd = sdesc_(smem_addr(sx + s * AT_TILE), 16);
-        // operands land by TMA and are observed through the mbarrier: no tensor-memory fence is needed
-        for (int i = 0; i < AT_NG && ok; ++i) {
-          const int g = i == 0 ? 4 : i - 1;            // RoPE block first
-          if (!mbar_wait(&xfull[s * AT_NG + g], use & 1, abort_flag)) { ok = false; break; }
-          if (g == 4) {
+        // the whole tile first, then its 36 instructions as one branch-free burst: control flow between
+        // tcgen05.mma issues costs the issuing thread far more than the instructions themselves
+        for (int g = 0; g < AT_NG && ok; ++g)
+          if (!mbar_wait(&xfull[s * AT_NG + g], use & 1, abort_flag)) ok = false;
+        if (ok) {
+          // operands land by TMA and are observed through the mbarrier: no tensor-memory fence is needed
 #pragma unroll
-            for (int kk = 0; kk < 4; ++kk) {
-              const uint64_t off = (uint64_t)((8 * AT_KBLK + 32 * kk) >> 4);
-              mma_bf16_(d, qd + off, xd + off, idesc_s, kk > 0 ? 1u : 0u);
-            }
-          } else {
-#pragma unroll
-            for (int kk = 0; kk < 8; ++kk) {
-              const uint64_t off = (uint64_t)(((2 * g + (kk >> 2)) * AT_KBLK + 32 * (kk & 3)) >> 4);
-              mma_bf16_(d, qd + off, xd + off, idesc_s, 1u);
-            }
+          for (int j = 0; j < 36; ++j) {
+            const uint64_t off = (uint64_t)(((j >> 2) * AT_KBLK + 32 * (j & 3)) >> 4);
+            mma_bf16_(d, qd + off, xd + off, idesc_s, j > 0 ? 1u : 0u);
           }
         }
         if (!ok) break;
