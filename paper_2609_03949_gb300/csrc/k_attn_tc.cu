@@ -6,9 +6,10 @@
 //                      columns (128-byte swizzle, one 8 KB block per 64 columns) as five groups -- the RoPE block
 //                      first, then four pairs of latent blocks, each as soon as the tile before it in that slot has
 //                      released it -- into one of two tile slots;
-//   warp 1 (S)         S = Q . X^T on tcgen05 (M = 64 heads, N = 64 rows, K = 576: 36 instructions, issued as one
-//                      burst once the tile has landed) into one of two S buffers in tensor memory; with M = 64 the logit
-//                      of head 16 g + i and row j sits in TMEM lane 32 g + i, column j;
+//   warps 1, 7 (S)     S = Q . X^T on tcgen05 (M = 64 heads, N = 64 rows, K = 576: 36 instructions) in two halves,
+//                      each issued by its own thread as one burst once its blocks have landed, into their own
+//                      accumulators (double-buffered); with M = 64 the logit of head 16 g + i and row j sits in TMEM
+//                      lane 32 g + i, column j, and the softmax adds the two halves;
 //   warp 6 (O^T)       once the softmax warps have written P^T, O^T += X_lat^T . P^T (M = 128 latent dims x 4
 //                      blocks, N = 64 heads, K = 64 rows: 16 instructions) into the O^T accumulator, which stays in
 //                      tensor memory for the whole range. X_lat^T is read straight from the tile slot as an MN-major
@@ -38,18 +39,19 @@ namespace vk {
 
 constexpr int AT_T = 64;                               // rows per tile
 constexpr int AT_SMX = 4;                              // softmax warps (one per TMEM lane quarter)
-constexpr int AT_THREADS = (3 + AT_SMX) * 32;   // producer, S issuer, softmax x4, O^T issuer
+constexpr int AT_THREADS = (4 + AT_SMX) * 32;   // producer, S issuer, softmax x4, O^T issuer, S issuer
 constexpr uint32_t AT_KBLK = 64 * 128;                 // one 64-column block of 64 rows (or 64 heads): 8 KB
 constexpr uint32_t AT_TILE = 9 * AT_KBLK;              // 73,728: one tile slot, and the queries
 constexpr uint32_t AT_P = 64 * 128;                    // P^T: 64 heads x 64 rows, bf16
 constexpr int AT_NG = 5;                               // load groups per tile: latent pairs 0..3, RoPE block 4
 constexpr float AT_TAU = 8.f;                          // log2 slack before a running max moves
 constexpr uint32_t AT_TMEM_COLS = 512;
-constexpr uint32_t AT_S_COL = 0;                       // S buffers: columns 0..63 and 64..127
+constexpr uint32_t AT_S_COL = 0;                       // S (RoPE + latent 0..255) buffers: columns 0..63, 64..127
+constexpr uint32_t AT_SB_COL = 384;                    // S (latent 256..511) buffers: columns 384..447, 448..511
 constexpr uint32_t AT_O_COL = 128;                     // O^T block j: columns 128 + 64 j .. + 63
 
 // Shared memory, from a 1024-byte aligned base. Barriers: xfull/xrel [2 slots][5 groups], sfull/sfree [2],
-// wfull/wfree [2], pfull, pfree, qfull, mdone, gbar [2], ebar, adone.
+// wfull/wfree [2], pfull, pfree, qfull, mdone, gbar [2], ebar, adone, bdone.
 struct AtSmem {
   static constexpr uint32_t q = 0;
   static constexpr uint32_t x = q + AT_TILE;
@@ -60,7 +62,7 @@ struct AtSmem {
   static constexpr uint32_t anyw = fac + 2 * 64 * 4;   // [2][4] u32
   static constexpr uint32_t misc = anyw + 2 * 4 * 4;   // TMEM base, abort flag
   static constexpr uint32_t bars = (misc + 8 + 7) & ~7u;
-  static constexpr uint32_t nbars = 2 * AT_NG * 2 + 2 * 4 + 4 + 3 + 1;
+  static constexpr uint32_t nbars = 2 * AT_NG * 2 + 2 * 4 + 4 + 3 + 2;
   static constexpr uint32_t total = bars + nbars * 8;
 };
 static_assert(AtSmem::total + 1024 <= 232448, "attention shared memory exceeds the 227 KB opt-in limit");
@@ -160,6 +162,7 @@ __global__ void __launch_bounds__(AT_THREADS, 1) k_attn_tc(const __grid_constant
   uint64_t* gbar = mdone + 1;                 // [2] softmax-group syncs, by tile parity
   uint64_t* ebar = gbar + 2;                  // softmax-group sync before the epilogue
   uint64_t* adone = ebar + 1;                 // O^T issuer's final commit
+  uint64_t* bdone = adone + 1;                // second S issuer's final commit
 
   const int split = blockIdx.x, hg = blockIdx.y, b = blockIdx.z;
   const int H = args.H;
@@ -172,10 +175,10 @@ __global__ void __launch_bounds__(AT_THREADS, 1) k_attn_tc(const __grid_constant
     *abort_flag = 0;
     for (int i = 0; i < 2 * AT_NG; ++i) { mbar_init(&xfull[i], 1); mbar_init(&xrel[i], 1); }
     for (int i = 0; i < 2; ++i) {
-      mbar_init(&sfull[i], 1);
+      mbar_init(&sfull[i], 2);                    // one commit from each S issuer
       mbar_init(&sfree[i], AT_SMX);
       mbar_init(&wfull[i], 1);
-      mbar_init(&wfree[i], AT_SMX + 2);
+      mbar_init(&wfree[i], AT_SMX + 3);
       mbar_init(&gbar[i], AT_SMX);
     }
     mbar_init(pfull, AT_SMX);
@@ -184,6 +187,7 @@ __global__ void __launch_bounds__(AT_THREADS, 1) k_attn_tc(const __grid_constant
     mbar_init(mdone, 1);
     mbar_init(ebar, AT_SMX);
     mbar_init(adone, 1);
+    mbar_init(bdone, 1);
     mbar_fence_init();
   }
   if (warp == 1) tmem_alloc(tmem_slot, AT_TMEM_COLS);
@@ -276,13 +280,17 @@ __global__ void __launch_bounds__(AT_THREADS, 1) k_attn_tc(const __grid_constant
       for (int i = 0; i < 2 * AT_NG; ++i)
         if (last_use[i] >= 0) mbar_wait(&xfull[i], last_use[i] & 1, nullptr);
     }
-  } else if (warp == 1) {
-    // ------------------------------------------------------------------ S issuer
+  } else if (warp == 1 || warp == 3 + AT_SMX) {
+    // ------------------------------------------------------------------ S issuers
+    // Two threads issue the two halves of the K = 576 contraction into their own accumulators (the softmax adds
+    // them): warp 1 the RoPE block and latent dims 0..255 (20 instructions), warp 7 latent dims 256..511 (16).
+    const int half = warp == 1 ? 0 : 1;
     if (lane == 0 && ntile > 0) {
       // S: M = 64 heads, N = 64 rows, A = Q and B = X, both K-major
       const uint32_t idesc_s =
           (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(AT_T >> 3) << 17) | ((uint32_t)(64 >> 4) << 24);
       const uint64_t qd = sdesc_(smem_addr(sq), 16);
+      uint64_t* done_bar = half == 0 ? mdone : bdone;
       bool ok = mbar_wait(qfull, 0, abort_flag);
       int u = 0;
       for (int t = 0; t < ntile && ok; ++t) {
@@ -292,28 +300,39 @@ __global__ void __launch_bounds__(AT_THREADS, 1) k_attn_tc(const __grid_constant
         if (!uni) continue;
         const int s = u & 1, use = u >> 1;
         if (use > 0 && !mbar_wait(&sfree[s], (use - 1) & 1, abort_flag)) { ok = false; break; }
-        const uint32_t d = tmem + AT_S_COL + 64 * s;
         const uint64_t xd = sdesc_(smem_addr(sx + s * AT_TILE), 16);
-        // the whole tile first, then its 36 instructions as one branch-free burst: control flow between
+        // this half's load groups first, then its instructions as one branch-free burst: control flow between
         // tcgen05.mma issues costs the issuing thread far more than the instructions themselves
-        for (int g = 0; g < AT_NG && ok; ++g)
-          if (!mbar_wait(&xfull[s * AT_NG + g], use & 1, abort_flag)) ok = false;
-        if (ok) {
+        if (half == 0) {
+          ok = mbar_wait(&xfull[s * AT_NG + 4], use & 1, abort_flag) && mbar_wait(&xfull[s * AT_NG + 0], use & 1, abort_flag) &&
+               mbar_wait(&xfull[s * AT_NG + 1], use & 1, abort_flag);
+          if (!ok) break;
           // operands land by TMA and are observed through the mbarrier: no tensor-memory fence is needed
+          const uint32_t d = tmem + AT_S_COL + 64 * s;
 #pragma unroll
-          for (int j = 0; j < 36; ++j) {
-            const uint64_t off = (uint64_t)(((j >> 2) * AT_KBLK + 32 * (j & 3)) >> 4);
+          for (int j = 0; j < 20; ++j) {
+            const int kb = j < 4 ? 8 : (j - 4) >> 2;
+            const uint64_t off = (uint64_t)((kb * AT_KBLK + 32 * (j & 3)) >> 4);
             mma_bf16_(d, qd + off, xd + off, idesc_s, j > 0 ? 1u : 0u);
           }
+          mma_commit_(&sfull[s]);
+          mma_commit_(&xrel[s * AT_NG + 4]);           // the RoPE block is read by S only
+        } else {
+          ok = mbar_wait(&xfull[s * AT_NG + 2], use & 1, abort_flag) && mbar_wait(&xfull[s * AT_NG + 3], use & 1, abort_flag);
+          if (!ok) break;
+          const uint32_t d = tmem + AT_SB_COL + 64 * s;
+#pragma unroll
+          for (int j = 0; j < 16; ++j) {
+            const uint64_t off = (uint64_t)(((4 + (j >> 2)) * AT_KBLK + 32 * (j & 3)) >> 4);
+            mma_bf16_(d, qd + off, xd + off, idesc_s, j > 0 ? 1u : 0u);
+          }
+          mma_commit_(&sfull[s]);
         }
-        if (!ok) break;
-        mma_commit_(&sfull[s]);
-        mma_commit_(&xrel[s * AT_NG + 4]);             // the RoPE block is read by S only
         ++u;
       }
-      mma_commit_(mdone);
+      mma_commit_(done_bar);
       if (!ok) { raise_status(args.status, VK_ERR_TIMEOUT); *abort_flag = 1; }
-      mbar_wait(mdone, 0, nullptr);                    // nothing this thread issued may outlive the CTA
+      mbar_wait(done_bar, 0, nullptr);                 // nothing this thread issued may outlive the CTA
     }
   } else if (warp == 2 + AT_SMX) {
     // ------------------------------------------------------------------ O^T issuer
@@ -387,8 +406,22 @@ __global__ void __launch_bounds__(AT_THREADS, 1) k_attn_tc(const __grid_constant
               "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
             : "r"(lrow + AT_S_COL + 64 * s)
             : "memory");
+        float sb[32];
+        uint32_t* rb = reinterpret_cast<uint32_t*>(sb);
+        asm volatile(
+            "tcgen05.ld.sync.aligned.16x32bx2.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16,%17,"
+            "%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32], 32;\n"
+            : "=r"(rb[0]), "=r"(rb[1]), "=r"(rb[2]), "=r"(rb[3]), "=r"(rb[4]), "=r"(rb[5]), "=r"(rb[6]), "=r"(rb[7]),
+              "=r"(rb[8]), "=r"(rb[9]), "=r"(rb[10]), "=r"(rb[11]), "=r"(rb[12]), "=r"(rb[13]), "=r"(rb[14]),
+              "=r"(rb[15]), "=r"(rb[16]), "=r"(rb[17]), "=r"(rb[18]), "=r"(rb[19]), "=r"(rb[20]), "=r"(rb[21]),
+              "=r"(rb[22]), "=r"(rb[23]), "=r"(rb[24]), "=r"(rb[25]), "=r"(rb[26]), "=r"(rb[27]), "=r"(rb[28]),
+              "=r"(rb[29]), "=r"(rb[30]), "=r"(rb[31])
+            : "r"(lrow + AT_SB_COL + 64 * s)
+            : "memory");
+        tmem_wait_ld();
+#pragma unroll
+        for (int c = 0; c < 32; ++c) sv[c] += sb[c];
       }
-      tmem_wait_ld();
       tmem_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(&sfree[s]);
