@@ -1,18 +1,20 @@
 // k_score_tc.cu -- RoPE-branch scoring on the 5th-generation tensor cores (tcgen05), bf16, r = 64.
 //
-// a[h,u] = Qr_h . K_u for every cached row (Eq. 4's exact summand): per sequence the [N x 64] RoPE slice times
-// the [64 x H] query, a dense contraction at H flop per byte. One CTA per SM walks a contiguous range of
+// a[h,u] = Qr_h . K_u for every cached row (Eq. 4's exact summand): per sequence the [H x 64] query times the
+// [64 x N] RoPE slice, a dense contraction at H flop per byte. One CTA per SM walks a contiguous range of
 // 128-row tiles:
-//   warp 0 (one thread)  TMA: the tile's 128 x 64 bf16 slice (128 B of every 1152-B row, 128-byte swizzle)
-//                        into an 8-stage ring, and the sequence's H x 64 query when the sequence changes;
-//   warp 1 (one thread)  tcgen05.mma M=128, N=H, K=16 (x4) into one of G fp32 accumulators in tensor memory
-//                        (128 lanes = rows, H columns = heads); tcgen05.commit frees the ring slot and hands the
-//                        accumulator to the epilogue group that owns it;
-//   G groups of 4 warps  epilogue, group g taking tiles i = g (mod G), so G tiles are in flight at once (the
-//                        candidate epilogue waits on global atomics): tcgen05.ld of 32 heads at a time, one
-//                        thread per row, then
+//   warp 0 (one thread)  TMA: the tile's 128 x 64 bf16 slice (128 B of every 1152-B row, 128-byte swizzle) into a
+//                        7-stage ring, and the sequence's H x 64 query when the sequence changes;
+//   warp 1 (one thread)  D = Q . K^T on tcgen05: M = 64 heads (H <= 64) or 128 per head group, N = 128 rows,
+//                        K = 16 (x4), issued as one burst into one of G accumulators in tensor memory (TMEM lane =
+//                        head, column = row); tcgen05.commit frees the ring slot and hands the accumulator on;
+//   G groups of 4 warps  epilogue, group g taking tiles i = g (mod G). The thread of head h reads its logits in
+//                        32-row chunks (tcgen05.ld 16x32bx2 for M = 64, 32x32b for M = 128), so a chunk's
+//                        threshold test is directly the head's 32-bit bitmap word of those rows:
 //                        mode 0  write fp32 scores [B][H][ld] (also used on a strided row sample),
-//                        mode 1  emit (u, a) for archive rows with a >= theta[b,h] into per-head candidate lists,
+//                        mode 1  emit (u, a) for archive rows with a >= theta[b,h] into per-head candidate lists:
+//                                one atomic per thread and tile reserves the room, then the chunk is staged in
+//                                shared memory and only its set bits are visited,
 //                        mode 2  trigger: T = lambda (a + |(O Qr)[r:]| page_res + z |Qc| eta) > s*_h for archive
 //                                rows outside S_h -> 32-row words of the fired bitmap (or candidates for top_j).
 // Every mbarrier wait is bounded; a wait that gives up raises VK_ERR_TIMEOUT and the CTA winds down.
@@ -27,10 +29,9 @@
 
 namespace vk {
 
-constexpr int TC_M = 128;                    // rows per tile (MMA M)
-constexpr int TC_STAGES = 8;
+constexpr int TC_M = 128;                        // rows per tile (MMA N)
+constexpr int TC_STAGES = 7;
 constexpr uint32_t TC_TILE_BYTES = TC_M * 128;   // 128 rows x 64 bf16
-constexpr int TC_MAX_G = 4;                  // epilogue groups (accumulator buffers)
 
 __device__ __forceinline__ void tma_load_3d(void* dst, const CUtensorMap* map, int x, int y, int z, uint64_t* bar) {
   asm volatile(
@@ -75,48 +76,74 @@ __device__ __forceinline__ void mma_commit(uint64_t* bar) {
                : "memory");
 }
 
-__device__ __forceinline__ void tmem_ld32(uint32_t taddr, float* v) {
+// One 32-row chunk of this thread's head: M = 128 (lane = head) reads 32 columns of its own lane; M = 64 (16 heads
+// per lane quarter) reads with 16x32bx2, lanes 0..15 columns [col, col + 32) and lanes 16..31 [col + 32, col + 64).
+template <int MH>
+__device__ __forceinline__ void tmem_ld_chunk(uint32_t taddr, float* v) {
   uint32_t* r = reinterpret_cast<uint32_t*>(v);
-  asm volatile(
-      "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16,%17,%18,%19,"
-      "%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];\n"
-      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]), "=r"(r[8]),
-        "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]), "=r"(r[16]),
-        "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]),
-        "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
-      : "r"(taddr)
-      : "memory");
+  if (MH == 128) {
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16,%17,%18,%19,"
+        "%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];\n"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]), "=r"(r[8]),
+          "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]), "=r"(r[16]),
+          "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]),
+          "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+        : "r"(taddr)
+        : "memory");
+  } else {
+    asm volatile(
+        "tcgen05.ld.sync.aligned.16x32bx2.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16,%17,"
+        "%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32], 32;\n"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]), "=r"(r[8]),
+          "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]), "=r"(r[16]),
+          "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]),
+          "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+        : "r"(taddr)
+        : "memory");
+  }
 }
 
+// Bits of the rows [lo, hi) within the 32 rows starting at r0.
+__device__ __forceinline__ uint32_t range_mask(int r0, int lo, int hi) {
+  const int a = max(lo - r0, 0), e = min(hi - r0, 32);
+  if (e <= a) return 0u;
+  const uint32_t upto = e >= 32 ? 0xffffffffu : ((1u << e) - 1u);
+  return upto & ~((1u << a) - 1u);
+}
+
+// Shared memory from a 1024-aligned base: the ring, two query buffers of NHG x MH rows, G x 128 staging rows of
+// 128 B (modes 1, 2), barriers.
+template <int MH, int NHG>
 struct TcSmem {
-  uint32_t a, q, bars, params, total;
-  __host__ __device__ TcSmem(int H) {
-    a = 0;                                              // TC_STAGES x 16 KB (1024-aligned)
-    q = a + TC_STAGES * TC_TILE_BYTES;                  // 2 x H x 128 B
-    bars = q + 2 * H * 128;                             // 8-byte barriers
-    params = bars + (2 * TC_STAGES + 4 + 2 * TC_MAX_G) * 8;   // per group: 4 x H floats of per-sequence params
-    total = params + TC_MAX_G * 4 * H * 4 + 1024;       // + slack to align the base to 1024
-  }
+  static constexpr int G = 4 / NHG;
+  static constexpr uint32_t a = 0;
+  static constexpr uint32_t q = a + TC_STAGES * TC_TILE_BYTES;
+  static constexpr uint32_t qbuf = NHG * MH * 128;
+  static constexpr uint32_t stg = q + 2 * qbuf;
+  static constexpr uint32_t bars = stg + G * 128 * 128;
+  static constexpr uint32_t total = bars + (2 * TC_STAGES + 4 + 2 * G) * 8 + 1024;
 };
 
-template <int G, int MODE>
-__global__ void __launch_bounds__((2 + 4 * G) * 32, 1) k_score_tc(const __grid_constant__ CUtensorMap kmap,
-                                                                const __grid_constant__ CUtensorMap qmap,
-                                                                const ScoreTcArgs args) {
+template <int MH, int NHG, int MODE>
+__global__ void __launch_bounds__((2 + 4 * (4 / NHG)) * 32, 1) k_score_tc(const __grid_constant__ CUtensorMap kmap,
+                                                                        const __grid_constant__ CUtensorMap qmap,
+                                                                        const ScoreTcArgs args) {
+  constexpr int G = 4 / NHG;
+  using L = TcSmem<MH, NHG>;
   extern __shared__ __align__(1024) unsigned char smem_raw[];
   unsigned char* smem = reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   const int H = args.H;
-  const TcSmem Ls(H);
-  unsigned char* sa = smem + Ls.a;
-  unsigned char* sq = smem + Ls.q;
-  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + Ls.bars);
+  unsigned char* sa = smem + L::a;
+  unsigned char* sq = smem + L::q;
+  float* stg = reinterpret_cast<float*>(smem + L::stg);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + L::bars);
   uint64_t* a_full = bars;
   uint64_t* a_empty = bars + TC_STAGES;
   uint64_t* q_full = bars + 2 * TC_STAGES;              // [2]
   uint64_t* q_empty = q_full + 2;                        // [2]
   uint64_t* d_full = q_empty + 2;                        // [G]
   uint64_t* d_empty = d_full + G;                        // [G]
-  float* sparams = reinterpret_cast<float*>(smem + Ls.params);   // [G groups][4][H]
   __shared__ uint32_t tmem_base;
   __shared__ int abort_flag;
 
@@ -126,8 +153,7 @@ __global__ void __launch_bounds__((2 + 4 * G) * 32, 1) k_score_tc(const __grid_c
   const int n = (int)(t1 - t0);
   const int tps = args.tiles_per_seq;
   const int b_first = (int)(t0 / tps);
-  const uint32_t dcols = (uint32_t)H;                   // columns per accumulator buffer
-  const uint32_t idesc = mma_idesc_bf16(TC_M, H);
+  constexpr uint32_t DCOLS = NHG * TC_M;                 // columns per accumulator
 
   if (threadIdx.x == 0) {
     abort_flag = 0;
@@ -136,7 +162,7 @@ __global__ void __launch_bounds__((2 + 4 * G) * 32, 1) k_score_tc(const __grid_c
     for (int i = 0; i < G; ++i) { mbar_init(&d_full[i], 1); mbar_init(&d_empty[i], 4); }
     mbar_fence_init();
   }
-  if (warp == 1) tmem_alloc(&tmem_base, args.tmem_cols);
+  if (warp == 1) tmem_alloc(&tmem_base, 512);
   tmem_fence_before();
   __syncthreads();
   tmem_fence_after();
@@ -152,7 +178,7 @@ __global__ void __launch_bounds__((2 + 4 * G) * 32, 1) k_score_tc(const __grid_c
           const int qi = (b - b_first) & 1, quse = (b - b_first) >> 1;
           if (quse > 0 && !mbar_wait(&q_empty[qi], (quse - 1) & 1, &abort_flag)) { abort_flag = 1; break; }
           mbar_arrive_expect_tx(&q_full[qi], (uint32_t)H * 128u);
-          tma_load_2d(sq + qi * H * 128, &qmap, 0, b * H, &q_full[qi]);
+          tma_load_2d(sq + qi * L::qbuf, &qmap, 0, b * H, &q_full[qi]);
           prev_b = b;
         }
         const int s = i % TC_STAGES, use = i / TC_STAGES;
@@ -165,6 +191,7 @@ __global__ void __launch_bounds__((2 + 4 * G) * 32, 1) k_score_tc(const __grid_c
   } else if (warp == 1) {
     // ------------------------------------------------------------------ MMA issuer
     if (lane == 0 && n > 0) {
+      constexpr uint32_t idesc = mma_idesc_bf16(MH, TC_M);
       int prev_b = -1;
       for (int i = 0; i < n; ++i) {
         const int64_t t = t0 + i;
@@ -178,11 +205,15 @@ __global__ void __launch_bounds__((2 + 4 * G) * 32, 1) k_score_tc(const __grid_c
         const int ds = i % G, duse = i / G;
         if (!mbar_wait(&a_full[s], use & 1, &abort_flag)) { abort_flag = 1; break; }
         if (duse > 0 && !mbar_wait(&d_empty[ds], (duse - 1) & 1, &abort_flag)) { abort_flag = 1; break; }
-        tmem_fence_after();
-        const uint32_t a0 = smem_addr(sa + s * TC_TILE_BYTES), b0 = smem_addr(sq + qi * H * 128);
+        tmem_fence_after();                              // the epilogue's reads of this accumulator came first
+        const uint64_t bd = sw128_desc(smem_addr(sa + s * TC_TILE_BYTES));
+        const uint64_t ad = sw128_desc(smem_addr(sq + qi * L::qbuf));
 #pragma unroll
-        for (int k = 0; k < 4; ++k)
-          mma_bf16(tmem_base + ds * dcols, sw128_desc(a0 + 32 * k), sw128_desc(b0 + 32 * k), idesc, k > 0);
+        for (int hg = 0; hg < NHG; ++hg)
+#pragma unroll
+          for (int k = 0; k < 4; ++k)
+            mma_bf16(tmem_base + ds * DCOLS + hg * TC_M, ad + (uint64_t)((hg * MH * 128 + 32 * k) >> 4),
+                     bd + (uint64_t)((32 * k) >> 4), idesc, k > 0 ? 1u : 0u);
         mma_commit(&a_empty[s]);
         mma_commit(&d_full[ds]);
         const bool last_of_seq = (i + 1 == n) || ((t + 1) / tps != b);
@@ -193,25 +224,29 @@ __global__ void __launch_bounds__((2 + 4 * G) * 32, 1) k_score_tc(const __grid_c
     // ------------------------------------------------------------------ epilogue
     const int ew = warp - 2;                              // 0 .. 4G-1
     const int g = ew >> 2;                                // group: tiles i = g (mod G), accumulator g
-    const int quarter = warp & 3;                         // TMEM lane quarter = the warp's 32 rows of the tile
-    float* prm = sparams + g * 4 * H;
+    const int quarter = warp & 3;                         // TMEM lane quarter this warp may read
+    constexpr int NC = MH == 128 ? 4 : 2;                 // 32-row chunks per thread and tile
+    float* my_stg = stg + (ew * 32 + lane) * 32;          // this thread's staging row (128 B, 16-byte swizzled)
     int prev_b = -1;
+    float th[NHG], p1[NHG], p2[NHG];                      // per head: theta, or (s*, |(O Qr)[r:]|, z |Qc|)
     for (int i = g; i < n; i += G) {
       const int64_t t = t0 + i;
       const int b = (int)(t / tps), row0 = (int)(t % tps) * TC_M;
       if (b != prev_b) {
-        // per-sequence parameters -> this group's shared-memory slot (the group's 4 warps, then a barrier)
-        named_barrier(2 + g, 128);
-        for (int h = (ew & 3) * 32 + lane; h < H; h += 128) {
-          if (MODE == 1) {
-            prm[h] = args.theta[(int64_t)b * H + h];
-          } else if (MODE == 2) {
-            prm[h] = args.smax1[(int64_t)b * H + h];
-            prm[H + h] = args.qcn[(int64_t)b * H + h] * args.z;
-            prm[2 * H + h] = args.qrn[(int64_t)b * H + h];
+#pragma unroll
+        for (int hg = 0; hg < NHG; ++hg) {
+          const int hh = hg * 128 + (MH == 128 ? 32 * quarter + lane : 16 * quarter + (lane & 15));
+          th[hg] = p1[hg] = p2[hg] = 0.f;
+          if (hh < H) {
+            const int64_t bh = (int64_t)b * H + hh;
+            if (MODE == 1) th[hg] = args.theta[bh];
+            if (MODE == 2) {
+              th[hg] = args.smax1[bh];
+              p1[hg] = args.qrn[bh];
+              p2[hg] = args.qcn[bh] * args.z;
+            }
           }
         }
-        named_barrier(2 + g, 128);
         prev_b = b;
       }
       const int duse = i / G;
@@ -220,91 +255,93 @@ __global__ void __launch_bounds__((2 + 4 * G) * 32, 1) k_score_tc(const __grid_c
         break;
       }
       tmem_fence_after();
-      const int row = row0 + quarter * 32 + lane;          // row of the tensor map (position, or sample index)
-      const bool in_rows = row < args.n_rows;
-      const int64_t bh0 = (int64_t)b * H;
-      const uint32_t tbase = tmem_base + ((uint32_t)(quarter * 32) << 16) + g * dcols;
-      bool arch = false;
-      float row_add = 0.f, row_eta = 0.f;
-      if (MODE >= 1) arch = in_rows && row >= args.arch_lo && row < args.arch_hi;
-      if (MODE == 2 && in_rows) {
-        row_add = args.page_res[(int64_t)b * args.n_pages + row / PAGE];
-        row_eta = args.eta[(int64_t)b * args.N + row];
-      }
-      const int64_t word = (row0 + quarter * 32) / 32;      // this warp's 32 rows = one bitmap word
-      const bool word_ok = word < args.nw;
-      const bool emit = MODE == 1 || (MODE == 2 && args.top_j > 0);
-      constexpr int NCH = G == 4 ? 4 : 8;                  // 32-head chunks (H <= 128 when G = 4)
-      uint32_t mine[NCH];                                  // ballot of head c + lane, per 32-head chunk
-      int base[NCH];
 #pragma unroll
-      for (int cc = 0; cc < NCH; ++cc) {
-        const int c = cc * 32;
-        if (c >= H) break;
-        const int hn = min(32, H - c);                     // 32, or 16 for the last chunk when H % 32 == 16
-        uint32_t sel_word = 0;
-        if (MODE == 2 && lane < hn && word_ok) sel_word = args.selbm[(bh0 + c + lane) * args.nw + word];
-        uint32_t m_lane = 0;
+      for (int hg = 0; hg < NHG; ++hg) {
+        const int hh = hg * 128 + (MH == 128 ? 32 * quarter + lane : 16 * quarter + (lane & 15));
+        const bool valid = hh < H;
+        const int64_t bh = (int64_t)b * H + hh;
+        const uint32_t taddr = tmem_base + ((uint32_t)(32 * quarter) << 16) + g * DCOLS + hg * TC_M;
+        const bool emit = MODE == 1 || (MODE == 2 && args.top_j > 0);
+        uint32_t msk[NC];
+        int cnt = 0;
 #pragma unroll
-        for (int half = 0; half < 2; ++half) {
-          if (16 * half >= hn) break;
-          float v[16];
-          tmem_ld16(tbase + c + 16 * half, v);
+        for (int c = 0; c < NC; ++c) {
+          float v[32];
+          tmem_ld_chunk<MH>(taddr + (MH == 128 ? 32 * c : 64 * c), v);
           tmem_wait_ld();
+          const int rc = row0 + (MH == 128 ? 32 * c : 64 * c + 32 * (lane >> 4));   // first row of the chunk
+          uint32_t m = 0u;
           if (MODE == 0) {
-            if (in_rows) {
+            if (valid) {
+              float* dst = args.scores + bh * args.scores_ld + rc;
+              if (rc + 32 <= args.n_rows && ((bh * args.scores_ld + rc) & 3) == 0) {
 #pragma unroll
-              for (int j = 0; j < 16; ++j) args.scores[(bh0 + c + 16 * half + j) * args.scores_ld + row] = v[j];
+                for (int k = 0; k < 8; ++k)
+                  reinterpret_cast<float4*>(dst)[k] = make_float4(v[4 * k], v[4 * k + 1], v[4 * k + 2], v[4 * k + 3]);
+              } else {
+#pragma unroll
+                for (int k = 0; k < 32; ++k)
+                  if (rc + k < args.n_rows) dst[k] = v[k];
+              }
             }
-            continue;
-          }
+          } else if (MODE == 1) {
 #pragma unroll
-          for (int jj = 0; jj < 16; ++jj) {
-            const int j = 16 * half + jj;
-            bool pass = false;
-            if (MODE == 1) {
-              pass = arch && v[jj] >= prm[c + j];
-            } else {
-              const uint32_t sw = __shfl_sync(0xffffffffu, sel_word, j);
-              const float T = args.lam * (v[jj] + prm[2 * H + c + j] * row_add + prm[H + c + j] * row_eta);
-              pass = arch && !((sw >> lane) & 1u) && T > prm[c + j];
+            for (int k = 0; k < 32; ++k) m |= (v[k] >= th[hg] ? 1u : 0u) << k;
+            m &= range_mask(rc, args.arch_lo, min(args.arch_hi, args.n_rows));
+            if (!valid) m = 0u;
+          } else {
+            const int64_t word = rc >> 5;
+            const bool word_ok = valid && word < args.nw && rc < args.n_rows;
+            const uint32_t sel = word_ok ? args.selbm[bh * args.nw + word] : 0xffffffffu;
+            const float pr = rc < args.n_rows ? args.page_res[(int64_t)b * args.n_pages + rc / PAGE] : 0.f;
+            const float add = p1[hg] * pr;
+            const float* eta = args.eta + (int64_t)b * args.N + rc;
+#pragma unroll
+            for (int k = 0; k < 32; ++k) {
+              const float e = rc + k < args.n_rows ? eta[k] : 0.f;
+              const float T = args.lam * (v[k] + add + p2[hg] * e);
+              v[k] = T;
+              m |= (T > th[hg] ? 1u : 0u) << k;
             }
-            const uint32_t m = __ballot_sync(0xffffffffu, pass);
-            if (lane == j) m_lane = m;
+            m &= range_mask(rc, args.arch_lo, min(args.arch_hi, args.n_rows)) & ~sel;
+            if (!word_ok) m = 0u;
+            if (!emit && word_ok) args.firebm[bh * args.nw + word] = m;
           }
+          msk[c] = m;
+          cnt += __popc(m);
         }
-        mine[cc] = m_lane;
-        if (MODE == 2 && !emit && lane < hn && word_ok) args.firebm[(bh0 + c + lane) * args.nw + word] = m_lane;
-      }
-      if (emit) {
-        // reserve room for every chunk first (the atomics overlap), then read the scores again and scatter
+        if (emit) {
+          // reserve the head's room for this tile, then stage each chunk that has hits and visit only its set bits
+          int pos = cnt ? atomicAdd(&args.cand_cnt[bh], cnt) : 0;
 #pragma unroll
-        for (int cc = 0; cc < NCH; ++cc) {
-          if (cc * 32 >= H) break;
-          const int cnt = __popc(mine[cc]);
-          base[cc] = cnt ? atomicAdd(&args.cand_cnt[bh0 + cc * 32 + lane], cnt) : 0;
-        }
-#pragma unroll
-        for (int cc = 0; cc < NCH; ++cc) {
-          const int c = cc * 32;
-          if (c >= H) break;
-          const int hn = min(32, H - c);
-#pragma unroll
-          for (int half = 0; half < 2; ++half) {
-            if (16 * half >= hn) break;
-            float v[16];
-            tmem_ld16(tbase + c + 16 * half, v);
+          for (int c = 0; c < NC; ++c) {
+            if (!__any_sync(0xffffffffu, msk[c] != 0u)) continue;
+            float v[32];
+            tmem_ld_chunk<MH>(taddr + (MH == 128 ? 32 * c : 64 * c), v);
             tmem_wait_ld();
+            const int rc = row0 + (MH == 128 ? 32 * c : 64 * c + 32 * (lane >> 4));
+            if (MODE == 2) {
+              const float pr = args.page_res[(int64_t)b * args.n_pages + rc / PAGE];
+              const float add = p1[hg] * pr;
+              const float* eta = args.eta + (int64_t)b * args.N + rc;
 #pragma unroll
-            for (int jj = 0; jj < 16; ++jj) {
-              const int j = 16 * half + jj;
-              const uint32_t m = __shfl_sync(0xffffffffu, mine[cc], j);
-              const int bj = __shfl_sync(0xffffffffu, base[cc], j);
-              if ((m >> lane) & 1u) {
-                const int pos = bj + __popc(m & ((1u << lane) - 1u));
-                float val = v[jj];
-                if (MODE == 2) val = args.lam * (v[jj] + prm[2 * H + c + j] * row_add + prm[H + c + j] * row_eta);
-                if (pos < args.capc) args.cand[(bh0 + c + j) * args.capc + pos] = make_int2(row, __float_as_int(val));
+              for (int k = 0; k < 32; ++k) {
+                const float e = rc + k < args.n_rows ? eta[k] : 0.f;
+                v[k] = args.lam * (v[k] + add + p2[hg] * e);
+              }
+            }
+            uint32_t m = msk[c];
+            if (m) {
+#pragma unroll
+              for (int k = 0; k < 8; ++k)
+                reinterpret_cast<float4*>(my_stg)[k ^ (lane & 7)] =
+                    make_float4(v[4 * k], v[4 * k + 1], v[4 * k + 2], v[4 * k + 3]);
+              while (m) {
+                const int k = __ffs(m) - 1;
+                m &= m - 1;
+                const float val = my_stg[(((k >> 2) ^ (lane & 7)) << 2) | (k & 3)];
+                if (pos < args.capc) args.cand[bh * args.capc + pos] = make_int2(rc + k, __float_as_int(val));
+                ++pos;
               }
             }
           }
@@ -320,7 +357,7 @@ __global__ void __launch_bounds__((2 + 4 * G) * 32, 1) k_score_tc(const __grid_c
   tmem_fence_before();
   __syncthreads();
   tmem_fence_after();
-  if (warp == 1) tmem_dealloc(tmem_base, args.tmem_cols);
+  if (warp == 1) tmem_dealloc(tmem_base, 512);
   if (threadIdx.x == 0 && abort_flag) raise_status(args.status, VK_ERR_TIMEOUT);
 }
 
@@ -372,22 +409,26 @@ cudaError_t launch_score_tc(const vk_view& v, int row_offset, int row_stride, in
   args.tiles_per_seq = (n_rows + TC_M - 1) / TC_M;
   args.total_tiles = (int64_t)args.tiles_per_seq * v.B;
   args.n_pages = (v.N + PAGE - 1) / PAGE;
-  const int G = v.H <= 128 ? 4 : 2;                   // G accumulators of H columns fit in 512 TMEM columns
-  uint32_t cols = 32;
-  while (cols < (uint32_t)(G * v.H)) cols <<= 1;
-  args.tmem_cols = cols;
+  args.tmem_cols = 512;
   const int grid = (int)std::min<int64_t>(args.total_tiles, 152);
-  const size_t smem = TcSmem(v.H).total;
-  auto pick = [&](auto kernel, int g) -> cudaError_t {
+  const int m = args.mode;
+  auto go = [&](auto kernel, size_t smem, int g) -> cudaError_t {
     cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
     if (grid > 0) kernel<<<grid, (2 + 4 * g) * 32, smem, st>>>(kmap, qmap, args);
     return cudaSuccess;
   };
   cudaError_t e;
-  const int m = args.mode;
-  if (G == 4) e = m == 0 ? pick(k_score_tc<4, 0>, 4) : m == 1 ? pick(k_score_tc<4, 1>, 4) : pick(k_score_tc<4, 2>, 4);
-  else e = m == 0 ? pick(k_score_tc<2, 0>, 2) : m == 1 ? pick(k_score_tc<2, 1>, 2) : pick(k_score_tc<2, 2>, 2);
+  if (v.H <= 64) {
+    const size_t sm = TcSmem<64, 1>::total;
+    e = m == 0 ? go(k_score_tc<64, 1, 0>, sm, 4) : m == 1 ? go(k_score_tc<64, 1, 1>, sm, 4) : go(k_score_tc<64, 1, 2>, sm, 4);
+  } else if (v.H <= 128) {
+    const size_t sm = TcSmem<128, 1>::total;
+    e = m == 0 ? go(k_score_tc<128, 1, 0>, sm, 4) : m == 1 ? go(k_score_tc<128, 1, 1>, sm, 4) : go(k_score_tc<128, 1, 2>, sm, 4);
+  } else {
+    const size_t sm = TcSmem<128, 2>::total;
+    e = m == 0 ? go(k_score_tc<128, 2, 0>, sm, 2) : m == 1 ? go(k_score_tc<128, 2, 1>, sm, 2) : go(k_score_tc<128, 2, 2>, sm, 2);
+  }
   if (e != cudaSuccess) return e;
   if (grid > 0) count_launches(1);
   return cudaGetLastError();
