@@ -103,6 +103,65 @@ struct RecomputedKeys {
   }
 };
 
+// Block-wide AND and OR of one value per thread (scratch: 2 x 32 words). Every thread gets both.
+__device__ __forceinline__ void block_and_or(uint32_t& a, uint32_t& o, uint32_t* scratch) {
+  a = __reduce_and_sync(0xffffffffu, a);
+  o = __reduce_or_sync(0xffffffffu, o);
+  const int w = threadIdx.x >> 5, nwarp = blockDim.x >> 5;
+  __syncthreads();
+  if ((threadIdx.x & 31) == 0) { scratch[w] = a; scratch[32 + w] = o; }
+  __syncthreads();
+  a = 0xffffffffu;
+  o = 0u;
+  for (int i = 0; i < nwarp; ++i) { a &= scratch[i]; o |= scratch[32 + i]; }
+}
+
+// The k-th largest of n keys (1 <= k <= n) by radix select in 8-bit digits that start at the keys' highest
+// differing bit (bits above it are common to all keys, so they take no pass and pile into no single bin).
+// Returns the key; *need_out = how many keys equal to it are among the k; *ties_out = how many keys equal it.
+// Called by the whole block.
+template <class KeyAt>
+__device__ uint32_t radix_kth_desc(const KeyAt& key_at, int n, unsigned int k, unsigned int* hist, uint32_t* scratch,
+                                   unsigned int* need_out, unsigned int* ties_out) {
+  __shared__ unsigned int s_digit, s_above, s_cnt;
+  uint32_t kand = 0xffffffffu, kor = 0u;
+  for (int i = threadIdx.x; i < n; i += blockDim.x) { const uint32_t key = key_at(i); kand &= key; kor |= key; }
+  block_and_or(kand, kor, scratch);
+  const uint32_t diff = kand ^ kor;
+  if (diff == 0u) {                                   // all keys equal
+    *need_out = k;
+    *ties_out = (unsigned int)n;
+    return kand;
+  }
+  int hb = 31 - __clz(diff);                          // highest differing bit
+  uint32_t prefix = hb == 31 ? 0u : (kand & ~((2u << hb) - 1u));
+  uint32_t mask = hb == 31 ? 0u : ~((2u << hb) - 1u);
+  unsigned int need = k, ties = 0;
+  while (true) {
+    const int shift = max(hb - 7, 0);
+    const uint32_t dmask = (2u << (hb - shift)) - 1u;   // digit of hb - shift + 1 <= 8 bits
+    for (int i = threadIdx.x; i < 256; i += blockDim.x) hist[i] = 0;
+    __syncthreads();
+    for (int i = threadIdx.x; i < n; i += blockDim.x) {
+      const uint32_t key = key_at(i);
+      if ((key & mask) == prefix) atomicAdd(&hist[(key >> shift) & dmask], 1u);
+    }
+    __syncthreads();
+    if (threadIdx.x < 32) pick_digit_desc(hist, need, &s_digit, &s_above, &s_cnt);
+    __syncthreads();
+    prefix |= s_digit << shift;
+    mask |= dmask << shift;
+    need -= s_above;
+    ties = s_cnt;
+    __syncthreads();
+    if (shift == 0) break;
+    hb = shift - 1;
+  }
+  *need_out = need;
+  *ties_out = ties;
+  return prefix;
+}
+
 // Ordered per-head selection over positions [0, N) (one CTA): the k largest keys of the archive [lo, hi) by
 // (key desc, position asc), plus -- unless `append` -- every position outside the archive (sinks, window).
 // Writes the ascending id list (after count[bh] entries when appending), the bitmap words, count and kth.
@@ -205,7 +264,7 @@ __global__ void __launch_bounds__(CAND_THREADS) k_theta(int ns, int off, int str
   extern __shared__ __align__(16) unsigned char smem[];
   uint32_t* keys = reinterpret_cast<uint32_t*>(smem);         // the archive samples' keys, [n_arch]
   __shared__ unsigned int hist[256];
-  __shared__ unsigned int s_digit, s_above;
+  __shared__ uint32_t scratch[64];
   __shared__ int n_arch;
   const int64_t bh = blockIdx.x;
   const float* a = sample + bh * (int64_t)ns;
@@ -220,22 +279,8 @@ __global__ void __launch_bounds__(CAND_THREADS) k_theta(int ns, int off, int str
     if (threadIdx.x == 0) theta[bh] = -INFINITY;      // emit every archive row
     return;
   }
-  unsigned int prefix = 0, mask = 0, need = (unsigned int)j;
-  for (int shift = 24; shift >= 0; shift -= 8) {
-    for (int i = threadIdx.x; i < 256; i += blockDim.x) hist[i] = 0;
-    __syncthreads();
-    for (int i = threadIdx.x; i < na; i += blockDim.x) {
-      const uint32_t key = keys[i];
-      if ((key & mask) == prefix) atomicAdd(&hist[(key >> shift) & 255u], 1u);
-    }
-    __syncthreads();
-    if (threadIdx.x < 32) pick_digit_desc(hist, need, &s_digit, &s_above, nullptr);
-    __syncthreads();
-    prefix |= s_digit << shift;
-    need -= s_above;
-    mask |= 255u << shift;
-    __syncthreads();
-  }
+  unsigned int need_eq, ties;
+  const uint32_t prefix = radix_kth_desc([&](int i) { return keys[i]; }, na, (unsigned int)j, hist, scratch, &need_eq, &ties);
   if (threadIdx.x == 0) theta[bh] = funkey(prefix);
 }
 
@@ -252,21 +297,21 @@ cudaError_t launch_theta(int B, int H, int ns, int off, int stride, int lo, int 
 // Selection from a head's candidate list (every archive row with score >= theta, in arbitrary order). When the
 // list holds at least k and at most capc entries it contains the whole top-k, which is found by a radix select
 // (ties by smaller position, via a second select on the positions of the tied keys); the selected rows, the
-// sinks and the window become the head's bitmap and ascending id list. The list is staged in shared memory when
+// sinks and the window become the head's bitmap and ascending id list. Its keys are staged in shared memory when
 // it has at most smem_cap entries and read from global memory otherwise. When the list is too short or too long
 // (theta landed too high or too low) or with VK_FLAG_FORCE_FALLBACK, the head takes the exact ordered selection
 // over scores recomputed from the RoPE columns. With `append` (the top_j of the fired rows, whose list can never
 // overflow) only candidates are selected, no sinks or window, and the ids are appended after count[b,h].
-__global__ void __launch_bounds__(CAND_THREADS) k_select_cand(
+__global__ void __launch_bounds__(CAND_THREADS, 4) k_select_cand(
     int H, int N, int lo, int hi, long long k_all, const long long* __restrict__ k_per_head,
     const int* __restrict__ cand_cnt, const int2* __restrict__ cand, int capc, int smem_cap, int force_fallback,
     const __nv_bfloat16* __restrict__ rope, int64_t rld, int64_t rbs, const float* __restrict__ qt,
     int32_t* __restrict__ idx, int32_t* __restrict__ count, int cap, int append, float* __restrict__ kth,
     uint32_t* __restrict__ bitmap, long long nw, int* status) {
   extern __shared__ __align__(16) unsigned char smem[];
-  uint32_t* skey = reinterpret_cast<uint32_t*>(smem);          // [smem_cap]
-  int32_t* spos = reinterpret_cast<int32_t*>(skey + smem_cap); // [smem_cap]
+  uint32_t* skey = reinterpret_cast<uint32_t*>(smem);          // [smem_cap] keys (positions stay in global memory)
   __shared__ unsigned int hist[256];
+  __shared__ uint32_t scratch[64];
   __shared__ unsigned int s_prefix, s_need, s_digit, s_above, s_cnt;
   __shared__ float qts[D_ROPE];
   __shared__ int scan_scratch[33];
@@ -294,36 +339,17 @@ __global__ void __launch_bounds__(CAND_THREADS) k_select_cand(
   const bool staged = c <= smem_cap;
   const int2* g = cand + bh * (int64_t)capc;
   if (staged) {
-    for (int i = threadIdx.x; i < c; i += blockDim.x) {
-      const int2 e = g[i];
-      spos[i] = e.x;
-      skey[i] = fkey(__int_as_float(e.y));
-    }
+    for (int i = threadIdx.x; i < c; i += blockDim.x) skey[i] = fkey(__int_as_float(g[i].y));
     __syncthreads();
   }
   auto key_at = [&](int i) -> uint32_t { return staged ? skey[i] : fkey(__int_as_float(g[i].y)); };
-  auto pos_at = [&](int i) -> uint32_t { return staged ? (uint32_t)spos[i] : (uint32_t)g[i].x; };
+  auto pos_at = [&](int i) -> uint32_t { return (uint32_t)g[i].x; };
 
   // radix select of the k-th largest key among the c candidates
-  unsigned int prefix = 0, mask = 0, need = (unsigned int)k, ties = 0;
+  unsigned int prefix = 0, need = (unsigned int)k, ties = 0;
   uint32_t pos_cut = 0xffffffffu;
   if (k > 0) {
-    for (int shift = 24; shift >= 0; shift -= 8) {
-      for (int i = threadIdx.x; i < 256; i += blockDim.x) hist[i] = 0;
-      __syncthreads();
-      for (int i = threadIdx.x; i < c; i += blockDim.x) {
-        const uint32_t key = key_at(i);
-        if ((key & mask) == prefix) atomicAdd(&hist[(key >> shift) & 255u], 1u);
-      }
-      __syncthreads();
-      if (threadIdx.x < 32) pick_digit_desc(hist, need, &s_digit, &s_above, &s_cnt);
-      __syncthreads();
-      prefix |= s_digit << shift;
-      need -= s_above;
-      ties = s_cnt;                                   // after the last pass: the keys equal to tau
-      mask |= 255u << shift;
-      __syncthreads();
-    }
+    prefix = radix_kth_desc(key_at, c, (unsigned int)k, hist, scratch, &need, &ties);
     if (ties > need) {
       // among keys equal to tau keep the `need` smallest positions: find the need-th smallest of them
       unsigned int pprefix = 0, pmask = 0, pneed = need;
@@ -348,7 +374,7 @@ __global__ void __launch_bounds__(CAND_THREADS) k_select_cand(
   const uint32_t tau = prefix;
   // bitmap (built in shared memory when it fits): clear, then set sinks and window (tier 1) and the selected
   // candidates, then write it out
-  uint32_t* wbm = nw <= SEL_SMEM_BITMAP_WORDS ? reinterpret_cast<uint32_t*>(spos + smem_cap) : bm;
+  uint32_t* wbm = nw <= SEL_SMEM_BITMAP_WORDS ? skey + smem_cap : bm;
   for (long long w = threadIdx.x; w < nw; w += blockDim.x) wbm[w] = 0u;
   __syncthreads();
   if (!append) {
@@ -392,7 +418,7 @@ cudaError_t launch_select_cand(int B, int H, int N, int lo, int hi, int64_t k, c
                                const float* qt, int32_t* idx, int32_t* count, int cap, int append, float* kth,
                                uint32_t* bitmap, int64_t nw, int* status, cudaStream_t st) {
   const int smem_cap = capc < 12288 ? capc : 12288;
-  const size_t smem = (size_t)smem_cap * 8 + (nw <= SEL_SMEM_BITMAP_WORDS ? (size_t)nw * 4 : 0);
+  const size_t smem = (size_t)smem_cap * 4 + (nw <= SEL_SMEM_BITMAP_WORDS ? (size_t)nw * 4 : 0);
   cudaError_t e = cudaFuncSetAttribute(k_select_cand, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
   k_select_cand<<<B * H, CAND_THREADS, smem, st>>>(
