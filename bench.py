@@ -50,6 +50,25 @@ def dist_env():
     return rank, world, local
 
 
+def rank_seed(rank: int) -> int:
+    """Seed of a rank's own sequences: every rank draws a different, reproducible batch."""
+    return 1000 + 7919 * rank
+
+
+def max_over_ranks(ms: float, pg, device) -> float:
+    """The slowest rank's time (the job finishes when its last rank does); a no-op on one process."""
+    if pg is None:
+        return ms
+    t = torch.tensor([ms], dtype=torch.float64, device=device)
+    pg.all_reduce(t, op=pg.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_throughput(seqs_per_rank: int, world: int, ms_per_step: float) -> float:
+    """Whole-job query-tokens/s: every rank's sequences (one query token each) over the slowest rank's step."""
+    return seqs_per_rank * world / (ms_per_step * 1e-3)
+
+
 def workload_config(B, n_gpus):
     return {"workload": f"sparse MLA decode step: H={H}, N={N}, rho=1/32, r={R}, window={WINDOW}, bf16 cache "
                         f"[512 latent + 64 RoPE], {N_PLANTED} planted rows/seq, B={B} sequences per GPU",
@@ -221,7 +240,7 @@ def run_native(args):
         pg.barrier()
     vk.lib()
     B = args.batch
-    wl = datagen.make_workload(B, H, N, seed=1000 + 7919 * rank, n_planted=N_PLANTED, planted_hi=N - WINDOW,
+    wl = datagen.make_workload(B, H, N, seed=rank_seed(rank), n_planted=N_PLANTED, planted_hi=N - WINDOW,
                                device=dev)
     view = vk.make_view(wl.cache, wl.q_latent, wl.q_rope)
     params = vk.make_params(RHO, r=R, window=WINDOW)
@@ -263,10 +282,7 @@ def run_native(args):
         for i in range(6):
             stage_ms[i] += evs[i].elapsed_time(evs[i + 1])
         total_ms_events += evs[0].elapsed_time(evs[6])
-    if pg:
-        t = torch.tensor([elapsed_ms], device=dev)
-        pg.all_reduce(t, op=pg.ReduceOp.MAX)
-        elapsed_ms = float(t.item())
+    elapsed_ms = max_over_ranks(elapsed_ms, pg, dev)
     clk = clocks.stop()
     vk.vk_profile_set_events([])
     assert vk.vk_poll_status(buf.ws) == vk.VK_OK
@@ -320,24 +336,20 @@ def run_native(args):
     e1.record(stream)
     torch.cuda.synchronize()
     e2e_ms = e0.elapsed_time(e1)
-    if pg:
-        t = torch.tensor([e2e_ms], device=dev)
-        pg.all_reduce(t, op=pg.ReduceOp.MAX)
-        e2e_ms = float(t.item())
+    e2e_ms = max_over_ranks(e2e_ms, pg, dev)
     assert torch.isfinite(lseh).all()
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         cpu = oracle_baseline(wl.cache, wl.q_latent, wl.q_rope)
 
-    total_seqs = B * world
     line = {
-        "metric": METRIC, "value": total_seqs / (ms_step * 1e-3), "unit": UNIT, "n_gpus": world,
+        "metric": METRIC, "value": job_throughput(B, world, ms_step), "unit": UNIT, "n_gpus": world,
         "steps": args.steps, "warmup": max(3, args.warmup), "ms_per_step": ms_step, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
         "data": "synthetic (seeded Gaussian MLA cache, bf16)", "config": workload_config(B, world),
         "roofline": roof, "cpu_baseline": cpu,
-        "e2e": {"value": total_seqs / (e2e_ms / args.steps * 1e-3), "unit": UNIT, "h2d_bytes_per_step": h2d,
+        "e2e": {"value": job_throughput(B, world, e2e_ms / args.steps), "unit": UNIT, "h2d_bytes_per_step": h2d,
                 "d2h_bytes_per_step": d2h},
         "gpu_launches": int(launches), "clocks": clk,
         "step": {"device_ms_per_step": dev_ms_step, "algorithmic_bytes": step_b,

@@ -126,7 +126,8 @@ int vk_select(const vk_view* view, const vk_params* params, const float* scores,
 /* Absorbed-MLA attention over caller-given sets idx[b,h,0:count[b,h]) (distinct positions in [0,N); an
  * id out of range is skipped and flags VK_ERR_INVALID_ARG in the device status). out [B,H,512] fp32,
  * lse [B,H] and smax [B,H] (s*, the max logit) fp32; lse and smax may be NULL. An empty set gives
- * out = 0 and lse = smax = -inf. */
+ * out = 0 and lse = smax = -inf. For bf16 caches the rows are read in 64-row tiles and rows no head
+ * selected enter the product with weight 0, so every one of the N cached rows must hold finite values. */
 int vk_sparse_attn(const vk_view* view, const vk_params* params, const int32_t* idx, const int32_t* count,
                    int32_t cap, float* out, float* lse, float* smax, void* ws, size_t ws_bytes, void* stream);
 
