@@ -449,10 +449,9 @@ __global__ void __launch_bounds__(AT_THREADS, 1) k_attn_tc(const __grid_constant
         const float e0 = ((w >> c) & 1u) ? ex2(fmaf(sv[c], L, -m)) : 0.f;
         const float e1 = ((w >> (c + 1)) & 1u) ? ex2(fmaf(sv[c + 1], L, -m)) : 0.f;
         const __nv_bfloat162 pb = __floats2bfloat162_rn(e0, e1);
-        const uint32_t bits = *reinterpret_cast<const uint32_t*>(&pb);
-        ls0 += __uint_as_float(bits << 16);            // the rounded values: what the tensor core multiplies
-        ls1 += __uint_as_float(bits & 0xffff0000u);
-        pk[c >> 1] = bits;
+        ls0 += e0;
+        ls1 += e1;
+        pk[c >> 1] = *reinterpret_cast<const uint32_t*>(&pb);
       }
       lsum += ls0 + ls1;
       // publish this group's rescale factors (by tile parity: a warp that runs ahead writes the other buffer)

@@ -103,6 +103,50 @@ struct RecomputedKeys {
   }
 };
 
+// Ascending ids of the set bits of wbm[0, nw), written to out[base ...] (entries past cap are dropped). Each warp
+// takes a contiguous range of words, counts its bits, one barrier shares the warps' totals, then every warp
+// writes its ids with warp-level prefix sums over 32-word chunks. Returns base + the number of set bits. Called
+// by the whole block (blockDim a multiple of 32, at most 1024); scratch holds 32 ints.
+__device__ __forceinline__ int bitmap_to_ids(const uint32_t* wbm, long long nw, int32_t* out, int base, int cap,
+                                             int* scratch) {
+  const int lane = threadIdx.x & 31, w = threadIdx.x >> 5, nwarp = blockDim.x >> 5;
+  const long long per = ((nw + nwarp - 1) / nwarp + 31) / 32 * 32;   // words per warp, whole chunks
+  const long long w0 = (long long)w * per, w1 = min(nw, w0 + per);
+  int cnt = 0;
+  for (long long i = w0 + lane; i < w1; i += 32) cnt += __popc(wbm[i]);
+  cnt = __reduce_add_sync(0xffffffffu, cnt);
+  __syncthreads();                                   // scratch may still be read by an earlier caller
+  if (lane == 0) scratch[w] = cnt;
+  __syncthreads();
+  int pos = base, total = 0;
+  for (int i = 0; i < nwarp; ++i) {
+    const int c = scratch[i];
+    if (i < w) pos += c;
+    total += c;
+  }
+  for (long long c0 = w0; c0 < w1; c0 += 32) {
+    const long long i = c0 + lane;
+    const uint32_t word = i < w1 ? wbm[i] : 0u;
+    const int n = __popc(word);
+    int incl = n;
+#pragma unroll
+    for (int d = 1; d < 32; d <<= 1) {
+      const int y = __shfl_up_sync(0xffffffffu, incl, d);
+      if (lane >= d) incl += y;
+    }
+    int p = pos + incl - n;
+    uint32_t bits = word;
+    while (bits) {
+      const int b = __ffs(bits) - 1;
+      bits &= bits - 1;
+      if (p < cap) out[p] = (int32_t)(i * 32 + b);
+      ++p;
+    }
+    pos += __shfl_sync(0xffffffffu, incl, 31);
+  }
+  return base + total;
+}
+
 // Block-wide AND and OR of one value per thread (scratch: 2 x 32 words). Every thread gets both.
 __device__ __forceinline__ void block_and_or(uint32_t& a, uint32_t& o, uint32_t* scratch) {
   a = __reduce_and_sync(0xffffffffu, a);
@@ -391,21 +435,7 @@ __global__ void __launch_bounds__(CAND_THREADS, 4) k_select_cand(
   if (wbm != bm)
     for (long long w = threadIdx.x; w < nw; w += blockDim.x) bm[w] = wbm[w];
   // ascending ids from the bitmap
-  int base = append ? count[bh] : 0;
-  for (long long c0 = 0; c0 < nw; c0 += blockDim.x) {
-    const long long w = c0 + threadIdx.x;
-    const uint32_t word = (w < nw) ? wbm[w] : 0u;
-    int tot;
-    int pos = base + block_exclusive_scan(__popc(word), scan_scratch, &tot);
-    uint32_t bits = word;
-    while (bits) {
-      const int i = __ffs(bits) - 1;
-      bits &= bits - 1;
-      if (pos < cap) out[pos] = (int32_t)(w * 32 + i);
-      ++pos;
-    }
-    base += tot;
-  }
+  const int base = bitmap_to_ids(wbm, nw, out, append ? count[bh] : 0, cap, scan_scratch);
   if (threadIdx.x == 0) {
     count[bh] = base;
     if (kth && !append) kth[bh] = k > 0 ? funkey(tau) : INFINITY;
@@ -436,22 +466,8 @@ __global__ void __launch_bounds__(SEL_THREADS) k_bitmap_to_list(int N, const uin
                                                                 int32_t* __restrict__ count, int cap, int* status) {
   __shared__ int scan_scratch[33];
   const int64_t bh = blockIdx.x;
-  int base = count[bh];
   int32_t* out = idx + bh * (int64_t)cap;
-  for (long long c = 0; c < nw; c += blockDim.x) {
-    const long long w = c + threadIdx.x;
-    const uint32_t word = (w < nw) ? bitmap[bh * nw + w] : 0u;
-    int tot;
-    int pos = base + block_exclusive_scan(__popc(word), scan_scratch, &tot);
-    uint32_t bits = word;
-    while (bits) {
-      const int i = __ffs(bits) - 1;
-      bits &= bits - 1;
-      if (pos < cap) out[pos] = (int32_t)(w * 32 + i);
-      ++pos;
-    }
-    base += tot;
-  }
+  const int base = bitmap_to_ids(bitmap + bh * nw, nw, out, count[bh], cap, scan_scratch);
   __syncthreads();
   if (threadIdx.x == 0) {
     if (base > cap) raise_status(status, VK_ERR_CAPACITY);
