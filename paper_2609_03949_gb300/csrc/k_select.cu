@@ -162,11 +162,12 @@ __device__ __forceinline__ void block_and_or(uint32_t& a, uint32_t& o, uint32_t*
 
 // The k-th largest of n keys (1 <= k <= n) by radix select in 8-bit digits that start at the keys' highest
 // differing bit (bits above it are common to all keys, so they take no pass and pile into no single bin).
-// Returns the key; *need_out = how many keys equal to it are among the k; *ties_out = how many keys equal it.
-// Called by the whole block.
+// With max_passes < 4 the result is the lower bound of the bucket reached (a key <= the k-th largest).
+// Returns the key; *need_out = how many keys equal to it are among the k (exact result only); *ties_out = how
+// many keys fall in its final bucket. Called by the whole block.
 template <class KeyAt>
 __device__ uint32_t radix_kth_desc(const KeyAt& key_at, int n, unsigned int k, unsigned int* hist, uint32_t* scratch,
-                                   unsigned int* need_out, unsigned int* ties_out) {
+                                   unsigned int* need_out, unsigned int* ties_out, int max_passes = 8) {
   __shared__ unsigned int s_digit, s_above, s_cnt;
   uint32_t kand = 0xffffffffu, kor = 0u;
   for (int i = threadIdx.x; i < n; i += blockDim.x) { const uint32_t key = key_at(i); kand &= key; kor |= key; }
@@ -181,7 +182,7 @@ __device__ uint32_t radix_kth_desc(const KeyAt& key_at, int n, unsigned int k, u
   uint32_t prefix = hb == 31 ? 0u : (kand & ~((2u << hb) - 1u));
   uint32_t mask = hb == 31 ? 0u : ~((2u << hb) - 1u);
   unsigned int need = k, ties = 0;
-  while (true) {
+  for (int pass = 0;; ++pass) {
     const int shift = max(hb - 7, 0);
     const uint32_t dmask = (2u << (hb - shift)) - 1u;   // digit of hb - shift + 1 <= 8 bits
     for (int i = threadIdx.x; i < 256; i += blockDim.x) hist[i] = 0;
@@ -198,7 +199,7 @@ __device__ uint32_t radix_kth_desc(const KeyAt& key_at, int n, unsigned int k, u
     need -= s_above;
     ties = s_cnt;
     __syncthreads();
-    if (shift == 0) break;
+    if (shift == 0 || pass + 1 >= max_passes) break;
     hb = shift - 1;
   }
   *need_out = need;
@@ -324,7 +325,10 @@ __global__ void __launch_bounds__(CAND_THREADS) k_theta(int ns, int off, int str
     return;
   }
   unsigned int need_eq, ties;
-  const uint32_t prefix = radix_kth_desc([&](int i) { return keys[i]; }, na, (unsigned int)j, hist, scratch, &need_eq, &ties);
+  // two digits below the samples' first differing bit pin the j-th largest to a bucket of 2^-16 of their key
+  // range; its lower bound is theta (a little below the exact order statistic: a few more candidates pass)
+  const uint32_t prefix =
+      radix_kth_desc([&](int i) { return keys[i]; }, na, (unsigned int)j, hist, scratch, &need_eq, &ties, 2);
   if (threadIdx.x == 0) theta[bh] = funkey(prefix);
 }
 
