@@ -345,19 +345,20 @@ cudaError_t launch_theta(int B, int H, int ns, int off, int stride, int lo, int 
 // Selection from a head's candidate list (every archive row with score >= theta, in arbitrary order). When the
 // list holds at least k and at most capc entries it contains the whole top-k, which is found by a radix select
 // (ties by smaller position, via a second select on the positions of the tied keys); the selected rows, the
-// sinks and the window become the head's bitmap and ascending id list. Its keys are staged in shared memory when
-// it has at most smem_cap entries and read from global memory otherwise. When the list is too short or too long
+// sinks and the window become the head's bitmap and ascending id list. The keys are read from the list (L2-resident
+// after the scoring pass) on every radix pass: shared memory holds only the bitmap, so 8 blocks fit per SM and
+// hide each other's latency. When the list is too short or too long
 // (theta landed too high or too low) or with VK_FLAG_FORCE_FALLBACK, the head takes the exact ordered selection
 // over scores recomputed from the RoPE columns. With `append` (the top_j of the fired rows, whose list can never
 // overflow) only candidates are selected, no sinks or window, and the ids are appended after count[b,h].
-__global__ void __launch_bounds__(CAND_THREADS, 4) k_select_cand(
+__global__ void __launch_bounds__(CAND_THREADS, 8) k_select_cand(
     int H, int N, int lo, int hi, long long k_all, const long long* __restrict__ k_per_head,
-    const int* __restrict__ cand_cnt, const int2* __restrict__ cand, int capc, int smem_cap, int force_fallback,
+    const int* __restrict__ cand_cnt, const int2* __restrict__ cand, int capc, int force_fallback,
     const __nv_bfloat16* __restrict__ rope, int64_t rld, int64_t rbs, const float* __restrict__ qt,
     int32_t* __restrict__ idx, int32_t* __restrict__ count, int cap, int append, float* __restrict__ kth,
     uint32_t* __restrict__ bitmap, long long nw, int* status) {
   extern __shared__ __align__(16) unsigned char smem[];
-  uint32_t* skey = reinterpret_cast<uint32_t*>(smem);          // [smem_cap] keys (positions stay in global memory)
+  uint32_t* sbm = reinterpret_cast<uint32_t*>(smem);           // the head's bitmap words, when they fit
   __shared__ unsigned int hist[256];
   __shared__ uint32_t scratch[64];
   __shared__ unsigned int s_prefix, s_need, s_digit, s_above, s_cnt;
@@ -384,13 +385,8 @@ __global__ void __launch_bounds__(CAND_THREADS, 4) k_select_cand(
     return;
   }
 
-  const bool staged = c <= smem_cap;
   const int2* g = cand + bh * (int64_t)capc;
-  if (staged) {
-    for (int i = threadIdx.x; i < c; i += blockDim.x) skey[i] = fkey(__int_as_float(g[i].y));
-    __syncthreads();
-  }
-  auto key_at = [&](int i) -> uint32_t { return staged ? skey[i] : fkey(__int_as_float(g[i].y)); };
+  auto key_at = [&](int i) -> uint32_t { return fkey(__int_as_float(g[i].y)); };
   auto pos_at = [&](int i) -> uint32_t { return (uint32_t)g[i].x; };
 
   // radix select of the k-th largest key among the c candidates
@@ -422,7 +418,7 @@ __global__ void __launch_bounds__(CAND_THREADS, 4) k_select_cand(
   const uint32_t tau = prefix;
   // bitmap (built in shared memory when it fits): clear, then set sinks and window (tier 1) and the selected
   // candidates, then write it out
-  uint32_t* wbm = nw <= SEL_SMEM_BITMAP_WORDS ? skey + smem_cap : bm;
+  uint32_t* wbm = nw <= SEL_SMEM_BITMAP_WORDS ? sbm : bm;
   for (long long w = threadIdx.x; w < nw; w += blockDim.x) wbm[w] = 0u;
   __syncthreads();
   if (!append) {
@@ -451,12 +447,11 @@ cudaError_t launch_select_cand(int B, int H, int N, int lo, int hi, int64_t k, c
                                const int* cand_cnt, const int2* cand, int capc, int force_fallback, const vk_view& v,
                                const float* qt, int32_t* idx, int32_t* count, int cap, int append, float* kth,
                                uint32_t* bitmap, int64_t nw, int* status, cudaStream_t st) {
-  const int smem_cap = capc < 12288 ? capc : 12288;
-  const size_t smem = (size_t)smem_cap * 4 + (nw <= SEL_SMEM_BITMAP_WORDS ? (size_t)nw * 4 : 0);
+  const size_t smem = nw <= SEL_SMEM_BITMAP_WORDS ? (size_t)nw * 4 : 0;
   cudaError_t e = cudaFuncSetAttribute(k_select_cand, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
   k_select_cand<<<B * H, CAND_THREADS, smem, st>>>(
-      H, N, lo, hi, (long long)k, reinterpret_cast<const long long*>(k_per_head), cand_cnt, cand, capc, smem_cap,
+      H, N, lo, hi, (long long)k, reinterpret_cast<const long long*>(k_per_head), cand_cnt, cand, capc,
       force_fallback, static_cast<const __nv_bfloat16*>(v.rope), v.rope_ld, v.rope_bstride, qt, idx, count, cap,
       append, kth, bitmap, (long long)nw, status);
   count_launches(1);
