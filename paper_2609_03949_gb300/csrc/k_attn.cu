@@ -282,7 +282,6 @@ __global__ void __launch_bounds__(AT_THREADS, 1) k_attn(
       if (lane == 0) { raise_status(status, VK_ERR_TIMEOUT); abort_flag = 1; }
       break;
     }
-    const uint32_t uni = hdr_union[s];
     const T* stage = rows + (int64_t)s * AT_BLK * ROWE;
 #pragma unroll
     for (int i = 0; i < AT_HPW; ++i) {

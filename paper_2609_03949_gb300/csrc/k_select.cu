@@ -214,7 +214,7 @@ template <class Keys>
 __device__ void select_ordered(const Keys& key_of, int N, int lo, int hi, long long k, int32_t* out, int32_t* count_bh,
                                int cap, int append, float* kth_bh, uint32_t* bitmap_bh, long long nw, int* status) {
   __shared__ unsigned int hist[256];
-  __shared__ unsigned int s_prefix, s_need, s_digit, s_above, s_cnt;
+  __shared__ unsigned int s_prefix, s_need, s_digit, s_above;
   __shared__ int scan_scratch[33];
   unsigned int prefix = 0, mask = 0, need = (unsigned int)k;
   if (k > 0) {
@@ -307,18 +307,29 @@ cudaError_t launch_select_dense(int B, int H, int N, const float* scores, const 
 __global__ void __launch_bounds__(CAND_THREADS) k_theta(int ns, int off, int stride, int lo, int hi, int j,
                                                         const float* __restrict__ sample, float* __restrict__ theta) {
   extern __shared__ __align__(16) unsigned char smem[];
-  uint32_t* keys = reinterpret_cast<uint32_t*>(smem);         // the archive samples' keys, [n_arch]
+  uint32_t* keys = reinterpret_cast<uint32_t*>(smem);         // the archive samples' keys
   __shared__ unsigned int hist[256];
   __shared__ uint32_t scratch[64];
-  __shared__ int n_arch;
   const int64_t bh = blockIdx.x;
   const float* a = sample + bh * (int64_t)ns;
   // sampled positions off + stride * i inside [lo, hi) are a contiguous index range [i0, i1)
   const int i0 = lo > off ? (lo - off + stride - 1) / stride : 0;
   const int i1 = min(ns, hi > off ? (hi - off + stride - 1) / stride : 0);
   const int na = max(0, i1 - i0);
-  for (int i = threadIdx.x; i < na; i += blockDim.x) keys[i] = fkey(a[i0 + i]);
-  if (threadIdx.x == 0) n_arch = na;
+  // all of a thread's loads in flight at once (the block is otherwise latency-bound on them)
+  for (int i = threadIdx.x; i < na; i += 16 * blockDim.x) {
+    float v[16];
+#pragma unroll
+    for (int r = 0; r < 16; ++r) {
+      const int e = i + r * blockDim.x;
+      v[r] = e < na ? a[i0 + e] : 0.f;
+    }
+#pragma unroll
+    for (int r = 0; r < 16; ++r) {
+      const int e = i + r * blockDim.x;
+      if (e < na) keys[e] = fkey(v[r]);
+    }
+  }
   __syncthreads();
   if (j <= 0 || j > na) {
     if (threadIdx.x == 0) theta[bh] = -INFINITY;      // emit every archive row
@@ -361,7 +372,7 @@ __global__ void __launch_bounds__(CAND_THREADS, 8) k_select_cand(
   uint32_t* sbm = reinterpret_cast<uint32_t*>(smem);           // the head's bitmap words, when they fit
   __shared__ unsigned int hist[256];
   __shared__ uint32_t scratch[64];
-  __shared__ unsigned int s_prefix, s_need, s_digit, s_above, s_cnt;
+  __shared__ unsigned int s_digit, s_above;
   __shared__ float qts[D_ROPE];
   __shared__ int scan_scratch[33];
   const int64_t bh = blockIdx.x;
