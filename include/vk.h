@@ -87,6 +87,10 @@ typedef struct {
 #define VK_FLAG_FORCE_FALLBACK 0x1u
 /* Use the materialised-score selection path even where the fused path would run (for tests). */
 #define VK_FLAG_FORCE_DENSE 0x2u
+/* Test hook for failure detection (bf16 caches): one attention CTA withholds its first tile's loads, so its
+ * bounded waits expire after about a second, it reports VK_ERR_TIMEOUT in the device status word and every
+ * role of that CTA winds down; vk_poll_status then returns VK_ERR_TIMEOUT. No other call uses it. */
+#define VK_FLAG_TEST_TIMEOUT 0x4u
 
 /* The per-cache index built once by vk_build_digest (Sec. 4.2 index entry with sketch rank 0). */
 typedef struct {

@@ -357,10 +357,11 @@ size_t attn_smem_bytes(int dtype, int H, int split_len) {
 }
 
 cudaError_t launch_attn(const vk_view& v, float lam, const uint32_t* bitmap, int64_t nw, int nsplit, int split_len,
-                        int slot0, int nslot, float* part_o, float* part_ml, int* status, cudaStream_t st) {
-  // bf16 caches: logits on the tensor cores (k_attn_tc.cu); fp32 caches: the SIMT kernel below
+                        int slot0, int nslot, float* part_o, float* part_ml, uint32_t flags, int* status,
+                        cudaStream_t st) {
+  // bf16 caches: both contractions on the tensor cores (k_attn_tc.cu); fp32 caches: the SIMT kernel below
   if (attn_tc_supported(v))
-    return launch_attn_tc(v, lam, bitmap, nw, nsplit, split_len, slot0, nslot, part_o, part_ml, status, st);
+    return launch_attn_tc(v, lam, bitmap, nw, nsplit, split_len, slot0, nslot, part_o, part_ml, flags, status, st);
   dim3 grid(nsplit, (v.H + HG - 1) / HG, v.B);
   const int nst = attn_stages(v.dtype, v.H);
   const size_t smem = attn_smem_bytes(v.dtype, v.H, split_len);

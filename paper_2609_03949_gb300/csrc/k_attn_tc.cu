@@ -75,6 +75,7 @@ struct AttnTcArgs {
   const uint32_t* bitmap;
   float* part_o;
   float* part_ml;
+  int hold_first;        // VK_FLAG_TEST_TIMEOUT: CTA (0,0,0) withholds its first tile's loads
   int* status;
 };
 
@@ -247,7 +248,9 @@ __global__ void __launch_bounds__(AT_THREADS, 1) k_attn_tc(const __grid_constant
       if (lane == 0) unis[ws] = uni;
       __syncwarp();
       if (lane == 0) mbar_arrive(&wfull[ws]);
-      if (uni) {
+      if (uni && args.hold_first && t == 0 && blockIdx.x == 0 && blockIdx.y == 0 && blockIdx.z == 0) {
+        ++u;                                           // test hook: these loads are never issued
+      } else if (uni) {
         const int s = u & 1, use = u >> 1;
         const int pos0 = p0 + t * AT_T;
         unsigned char* xs = sx + s * AT_TILE;
@@ -580,7 +583,8 @@ static bool make_map3(CUtensorMap* map, const void* base, uint64_t cols, uint64_
 }
 
 cudaError_t launch_attn_tc(const vk_view& v, float lam, const uint32_t* bitmap, int64_t nw, int nsplit, int split_len,
-                           int slot0, int nslot, float* part_o, float* part_ml, int* status, cudaStream_t st) {
+                           int slot0, int nslot, float* part_o, float* part_ml, uint32_t flags, int* status,
+                           cudaStream_t st) {
   if (!encode2()) return cudaErrorNotSupported;
   if (split_len % AT_T != 0) return cudaErrorInvalidValue;
   CUtensorMap lmap, rmap, qlmap, qrmap;
@@ -601,6 +605,7 @@ cudaError_t launch_attn_tc(const vk_view& v, float lam, const uint32_t* bitmap, 
   a.bitmap = bitmap;
   a.part_o = part_o;
   a.part_ml = part_ml;
+  a.hold_first = (flags & VK_FLAG_TEST_TIMEOUT) ? 1 : 0;
   a.status = status;
   const size_t smem = AtSmem::total + 1024;
   cudaError_t e = cudaFuncSetAttribute(k_attn_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);

@@ -88,7 +88,8 @@ int check_params(const vk_view* v, const vk_params* p) {
   if (p->trigger != VK_TRIG_OFF && p->trigger != VK_TRIG_CS) return fail(VK_ERR_INVALID_ARG, "trigger = %d is unknown", p->trigger);
   if (!(p->z_eff >= 0.f) || !std::isfinite(p->z_eff)) return fail(VK_ERR_INVALID_ARG, "z_eff must be finite and >= 0");
   if (p->top_j < 0) return fail(VK_ERR_INVALID_ARG, "top_j must be >= 0");
-  if (p->flags & ~(VK_FLAG_FORCE_FALLBACK | VK_FLAG_FORCE_DENSE)) return fail(VK_ERR_INVALID_ARG, "unknown flags 0x%x", p->flags);
+  if (p->flags & ~(VK_FLAG_FORCE_FALLBACK | VK_FLAG_FORCE_DENSE | VK_FLAG_TEST_TIMEOUT))
+    return fail(VK_ERR_INVALID_ARG, "unknown flags 0x%x", p->flags);
   return VK_OK;
 }
 
@@ -326,7 +327,7 @@ int vk_sparse_attn(const vk_view* view, const vk_params* params, const int32_t* 
   float* po = at<float>(ws, L.off_part_o);
   float* pml = at<float>(ws, L.off_part_ml);
   VK_CUDA(vk::launch_list_to_bitmap(view->B, view->H, view->N, idx, count, cap, bm, L.nw, status, st), "list_to_bitmap");
-  VK_CUDA(vk::launch_attn(*view, params->sm_scale, bm, L.nw, (int)L.nsplit, (int)L.split_len, 0, (int)L.nsplit, po, pml,
+  VK_CUDA(vk::launch_attn(*view, params->sm_scale, bm, L.nw, (int)L.nsplit, (int)L.split_len, 0, (int)L.nsplit, po, pml, params->flags,
                           status, st), "attention");
   VK_CUDA(vk::launch_combine(view->B, view->H, (int)L.nsplit, (int)L.nsplit, po, pml, out, lse, smax, st), "combine");
   return VK_OK;
@@ -411,7 +412,7 @@ int vk_decode_step(const vk_view* view, const vk_params* params, const vk_index*
             "select");
   }
   prof(3, st);
-  VK_CUDA(vk::launch_attn(v, params->sm_scale, selbm, L.nw, ns, (int)L.split_len, 0, nslot, po, pml, status, st),
+  VK_CUDA(vk::launch_attn(v, params->sm_scale, selbm, L.nw, ns, (int)L.split_len, 0, nslot, po, pml, params->flags, status, st),
           "attention");
   prof(4, st);
   if (two_tier) {
@@ -460,7 +461,7 @@ int vk_decode_step(const vk_view* view, const vk_params* params, const vk_index*
         VK_CUDA(vk::launch_bitmap_to_list(B, H, N, firebm, L.nw, idx, count, cap, status, st), "fired list");
       }
     }
-    VK_CUDA(vk::launch_attn(v, params->sm_scale, firebm, L.nw, ns, (int)L.split_len, ns, nslot, po, pml, status, st),
+    VK_CUDA(vk::launch_attn(v, params->sm_scale, firebm, L.nw, ns, (int)L.split_len, ns, nslot, po, pml, 0u, status, st),
             "fired attention");
   }
   prof(5, st);

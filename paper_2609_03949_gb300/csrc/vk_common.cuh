@@ -107,10 +107,11 @@ cudaError_t launch_list_to_bitmap(int B, int H, int N, const int32_t* idx, const
 size_t attn_smem_bytes(int dtype, int H, int split_len);
 bool attn_tc_supported(const vk_view& v);
 cudaError_t launch_attn_tc(const vk_view& v, float lam, const uint32_t* bitmap, int64_t nw, int nsplit, int split_len,
-                           int slot0, int nslot, float* part_o, float* part_ml, int* status, cudaStream_t st);
+                           int slot0, int nslot, float* part_o, float* part_ml, uint32_t flags, int* status,
+                           cudaStream_t st);
 cudaError_t launch_attn(const vk_view& v, float lam, const uint32_t* bitmap, int64_t nw, int nsplit,
-                        int split_len, int slot0, int nslot, float* part_o, float* part_ml, int* status,
-                        cudaStream_t st);
+                        int split_len, int slot0, int nslot, float* part_o, float* part_ml, uint32_t flags,
+                        int* status, cudaStream_t st);
 cudaError_t launch_smax_reduce(int B, int H, int nsplit, int nslot, const float* part_ml, float* smax,
                                cudaStream_t st);
 cudaError_t launch_combine(int B, int H, int nslot, int nslot_tier1, const float* part_o, const float* part_ml,

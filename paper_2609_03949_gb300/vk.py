@@ -18,7 +18,7 @@ VK_OK, VK_ERR_INVALID_ARG, VK_ERR_UNSUPPORTED, VK_ERR_WORKSPACE = 0, -1, -2, -3
 VK_ERR_CAPACITY, VK_ERR_CUDA, VK_ERR_TIMEOUT = -4, -5, -6
 VK_BF16, VK_F32 = 0, 1
 VK_TRIG_OFF, VK_TRIG_CS = 0, 1
-VK_FLAG_FORCE_FALLBACK, VK_FLAG_FORCE_DENSE = 0x1, 0x2
+VK_FLAG_FORCE_FALLBACK, VK_FLAG_FORCE_DENSE, VK_FLAG_TEST_TIMEOUT = 0x1, 0x2, 0x4
 D_LATENT, D_ROPE, PAGE = 512, 64, 64
 DEFAULT_SM_SCALE = 1.0 / math.sqrt(192.0)
 

@@ -286,3 +286,20 @@ def test_selection_paths(flags, trigger, top_j):
     # the threshold-candidate path, its exact fallback and the materialised-score path all meet the oracle
     wl = datagen.make_workload(2, 64, 20000, seed=17, n_planted=16, planted_hi=20000 - 256, device="cuda")
     run_case(wl, rho=1 / 32, window=256, n_sink=2, trigger=trigger, z_eff=0.7, top_j=top_j, flags=flags)
+
+
+def test_bounded_wait_reports_timeout():
+    # Failure detection without a GPU fault: the test hook withholds one CTA's first tile; that CTA's bounded waits
+    # give up after about a second, the status word reads VK_ERR_TIMEOUT and the context stays usable.
+    wl = datagen.make_workload(2, 64, 8192, seed=23, device="cuda")
+    step = GpuStep(wl, rho=1 / 32, window=256, n_sink=4, flags=vk.VK_FLAG_TEST_TIMEOUT)
+    g = step.run()
+    assert g["status"] == vk.VK_ERR_TIMEOUT
+    assert vk.vk_poll_status(step.buf.ws) == vk.VK_OK         # reading the status clears it
+    clean = GpuStep(wl, rho=1 / 32, window=256, n_sink=4)
+    h = clean.run()
+    assert h["status"] == vk.VK_OK
+    # the tier-1 selection ran before the withheld attention tile and is unaffected
+    np.testing.assert_array_equal(g["idx"], h["idx"])
+    hi = oracle.HostInputs(wl)
+    check_outputs(hi, LAM, h)
