@@ -159,15 +159,20 @@ def union_rows(idx: torch.Tensor, count: torch.Tensor, n: int) -> int:
 
 
 def kernel_traffic(kernel: str):
-    """DRAM bytes per launch from the committed ncu summary, if the kernel's source is unchanged since."""
+    """DRAM bytes per launch from the committed ncu summary, if the kernel's sources are unchanged since."""
     path = os.path.join(ROOT, "profiles", "traffic.json")
     if not os.path.exists(path):
         return None
     d = json.load(open(path)).get(kernel)
     if not d:
         return None
-    src = os.path.join(ROOT, d["source"])
-    if not os.path.exists(src) or hashlib.sha256(open(src, "rb").read()).hexdigest()[:16] != d["source_sha"]:
+    srcs = [os.path.join(ROOT, f) for f in d["sources"]]
+    if not all(os.path.exists(f) for f in srcs):
+        return None
+    h = hashlib.sha256()
+    for f in srcs:
+        h.update(open(f, "rb").read())
+    if h.hexdigest()[:16] != d["source_sha"]:
         return None
     return float(d["bytes_per_launch"]) * d.get("scale_to_bench", 1.0)
 

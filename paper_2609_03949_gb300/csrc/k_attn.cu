@@ -356,12 +356,12 @@ size_t attn_smem_bytes(int dtype, int H, int split_len) {
   return AttnSmem(dtype == VK_BF16 ? 2 : 4, min(H, HG), attn_stages(dtype, H)).total;
 }
 
-cudaError_t launch_attn(const vk_view& v, float lam, const uint32_t* bitmap, int64_t nw, int nsplit, int split_len,
-                        int slot0, int nslot, float* part_o, float* part_ml, uint32_t flags, int* status,
-                        cudaStream_t st) {
-  // bf16 caches: both contractions on the tensor cores (k_attn_tc.cu); fp32 caches: the SIMT kernel below
-  if (attn_tc_supported(v))
-    return launch_attn_tc(v, lam, bitmap, nw, nsplit, split_len, slot0, nslot, part_o, part_ml, flags, status, st);
+cudaError_t launch_attn(const vk_view& v, float lam, const uint32_t* bitmap, int64_t nw, const AttnGeom& g, int slot0,
+                        int nslot, float* part_o, float* part_ml, uint32_t flags, int* status, cudaStream_t st) {
+  // bf16 caches: both contractions on the tensor cores, persistent layout (k_attn_tc.cu); fp32 caches: the SIMT
+  // kernel below, split layout
+  if (g.G > 0) return launch_attn_tc(v, lam, bitmap, nw, g, slot0, nslot, part_o, part_ml, flags, status, st);
+  const int nsplit = g.nsplit, split_len = g.split_len;
   dim3 grid(nsplit, (v.H + HG - 1) / HG, v.B);
   const int nst = attn_stages(v.dtype, v.H);
   const size_t smem = attn_smem_bytes(v.dtype, v.H, split_len);
@@ -389,44 +389,50 @@ cudaError_t launch_attn(const vk_view& v, float lam, const uint32_t* bitmap, int
 }
 
 // ---------------------------------------------------------------------------------------------- s* and merge
-__global__ void k_smax_reduce(int BH, int H, int nsplit, int nslot, const float* __restrict__ part_ml,
+// s*_h of the tier-1 set: the max over the written tier-1 slots of (b, h).
+__global__ void k_smax_reduce(int BH, int H, const AttnGeom g, int nslot, const float* __restrict__ part_ml,
                               float* __restrict__ smax) {
   const int i = blockIdx.x * blockDim.x + threadIdx.x;
   if (i >= BH) return;
   const int b = i / H, h = i % H;
+  const int nv = attn_nvalid(g, (long long)b * g.n_hg + h / HG);
   float m = -INFINITY;
-  for (int s = 0; s < nsplit; ++s) m = fmaxf(m, part_ml[(((int64_t)b * nslot + s) * H + h) * 2]);
+  for (int s = 0; s < nv; ++s) m = fmaxf(m, part_ml[(((int64_t)b * nslot + s) * H + h) * 2]);
   smax[i] = m;
 }
 
-cudaError_t launch_smax_reduce(int B, int H, int nsplit, int nslot, const float* part_ml, float* smax,
+cudaError_t launch_smax_reduce(int B, int H, const AttnGeom& g, int nslot, const float* part_ml, float* smax,
                                cudaStream_t st) {
-  k_smax_reduce<<<(B * H + 255) / 256, 256, 0, st>>>(B * H, H, nsplit, nslot, part_ml, smax);
+  k_smax_reduce<<<(B * H + 255) / 256, 256, 0, st>>>(B * H, H, g, nslot, part_ml, smax);
   count_launches(1);
   return cudaGetLastError();
 }
 
-// One warp per (b, h): o = sum_s e^{m_s - m} o_s / sum_s e^{m_s - m} l_s, lse = m + log(sum), and s* = the
-// max over the first nslot_tier1 slots.
-__global__ void k_combine(int BH, int H, int nslot, int nslot_tier1, const float* __restrict__ part_o,
+// One warp per (b, h): o = sum_s e^{m_s - m} o_s / sum_s e^{m_s - m} l_s over the written slots of both tiers,
+// lse = m + log(sum), and s* = the max over the tier-1 slots. Slot s of the list is tier-1 slot s for s < nv, else
+// fired slot g.nslot + s - nv (only when nslot covers two tiers).
+__global__ void k_combine(int BH, int H, const AttnGeom g, int nslot, const float* __restrict__ part_o,
                           const float* __restrict__ part_ml, float* __restrict__ out, float* __restrict__ lse,
                           float* __restrict__ smax) {
   const int wid = (blockIdx.x * blockDim.x + threadIdx.x) >> 5, lane = threadIdx.x & 31;
   if (wid >= BH) return;
   const int b = wid / H, h = wid % H;
+  const int nv = attn_nvalid(g, (long long)b * g.n_hg + h / HG);
+  const int nlist = nslot > g.nslot ? 2 * nv : nv;
+  auto slot_of = [&](int s) { return s < nv ? s : g.nslot + s - nv; };
   float m = -INFINITY, m1 = -INFINITY;
-  for (int s = 0; s < nslot; ++s) {
-    const float ms = part_ml[(((int64_t)b * nslot + s) * H + h) * 2];
+  for (int s = 0; s < nlist; ++s) {
+    const float ms = part_ml[(((int64_t)b * nslot + slot_of(s)) * H + h) * 2];
     m = fmaxf(m, ms);
-    if (s < nslot_tier1) m1 = fmaxf(m1, ms);
+    if (s < nv) m1 = fmaxf(m1, ms);
   }
   float acc[16];
 #pragma unroll
   for (int t = 0; t < 16; ++t) acc[t] = 0.f;
   float l = 0.f;
   if (m > -INFINITY) {
-    for (int s = 0; s < nslot; ++s) {
-      const int64_t base = ((int64_t)b * nslot + s) * H + h;
+    for (int s = 0; s < nlist; ++s) {
+      const int64_t base = ((int64_t)b * nslot + slot_of(s)) * H + h;
       const float ms = part_ml[base * 2], ls = part_ml[base * 2 + 1];
       if (!(ls > 0.f)) continue;
       const float w = __expf(ms - m);
@@ -453,11 +459,10 @@ __global__ void k_combine(int BH, int H, int nslot, int nslot_tier1, const float
   }
 }
 
-cudaError_t launch_combine(int B, int H, int nslot, int nslot_tier1, const float* part_o, const float* part_ml,
+cudaError_t launch_combine(int B, int H, const AttnGeom& g, int nslot, const float* part_o, const float* part_ml,
                            float* out, float* lse, float* smax, cudaStream_t st) {
   const int BH = B * H, threads = 256;
-  k_combine<<<(BH * 32 + threads - 1) / threads, threads, 0, st>>>(BH, H, nslot, nslot_tier1, part_o, part_ml, out,
-                                                                  lse, smax);
+  k_combine<<<(BH * 32 + threads - 1) / threads, threads, 0, st>>>(BH, H, g, nslot, part_o, part_ml, out, lse, smax);
   count_launches(1);
   return cudaGetLastError();
 }

@@ -1,18 +1,21 @@
 // k_attn_tc.cu -- gather + absorbed-MLA attention for bf16 caches, both contractions on the tensor cores.
 //
-// Per CTA: one sequence b, one range of positions (a multiple of 64 long), one group of <= 64 heads. Positions are
-// walked in tiles of 64 rows; a tile that no head of the group selects is neither loaded nor computed. Per tile:
+// Persistent: one CTA per SM. The work is B * n_hg segments (sequence b, group of <= 64 heads), each walked in tiles
+// of 64 rows; the segments' tiles, flattened segment-major, are cut into one equal contiguous range per CTA, so a
+// CTA covers the end of one segment, whole segments and the start of another. A tile that no head of its group
+// selects is neither loaded nor computed. Per tile:
 //   warp 0 (producer)  stages the heads' two 32-bit selection words of the tile, then TMA-loads its 64 rows x 576
 //                      columns (128-byte swizzle, one 8 KB block per 64 columns) as five groups -- the RoPE block
 //                      first, then four pairs of latent blocks, each as soon as the tile before it in that slot has
-//                      released it -- into one of two tile slots;
+//                      released it -- into one of two tile slots; at a segment's first tile it loads the segment's
+//                      queries once the previous segment's S products are done with the query buffer;
 //   warps 1, 7 (S)     S = Q . X^T on tcgen05 (M = 64 heads, N = 64 rows, K = 576: 36 instructions) in two halves,
 //                      each issued by its own thread as one burst once its blocks have landed, into their own
 //                      accumulators (double-buffered); with M = 64 the logit of head 16 g + i and row j sits in TMEM
 //                      lane 32 g + i, column j, and the softmax adds the two halves;
 //   warp 6 (O^T)       once the softmax warps have written P^T, O^T += X_lat^T . P^T (M = 128 latent dims x 4
 //                      blocks, N = 64 heads, K = 64 rows: 16 instructions) into the O^T accumulator, which stays in
-//                      tensor memory for the whole range. X_lat^T is read straight from the tile slot as an MN-major
+//                      tensor memory for the whole segment. X_lat^T is read straight from the tile slot as an MN-major
 //                      operand (the next 64 dims one 8 KB block away), so each latent row is staged in shared memory
 //                      once and feeds both contractions. Two issuing threads, so neither contraction waits behind
 //                      the other's issue;
@@ -23,8 +26,11 @@
 //                      swizzle). m_h is a running max that only moves when a tile's max exceeds it by more than 8
 //                      (log2 units; the head's O^T column and sum are then rescaled in tensor memory), so rescaling
 //                      is rare and P stays <= 256. The exact max is tracked beside it, and at the end the head's sum
-//                      and output are re-based on it, so the partial carries the true max logit.
-// The partial (max, sum, out) of each range is merged by the LSE combine (Lemma 1). Rows inside a loaded tile that
+//                      and output are re-based on it, so the partial carries the true max logit. At a segment's end
+//                      they write its partial and hand the O^T accumulator back to the O^T issuer.
+// The partials (max, sum, out) of a segment, one per CTA it spans, are merged by the LSE combine (Lemma 1): with
+// every CTA resident for the whole launch there is no tail of partly filled waves, and a long segment yields a
+// few partials instead of one per fixed-length split. Rows inside a loaded tile that
 // no head selected still enter the O^T product with weight 0, so every row in [0, N) must hold finite values.
 // All waits are bounded: a wait that gives up raises VK_ERR_TIMEOUT and every role drains and leaves.
 #include <cuda.h>
@@ -51,7 +57,7 @@ constexpr uint32_t AT_SB_COL = 384;                    // S (latent 256..511) bu
 constexpr uint32_t AT_O_COL = 128;                     // O^T block j: columns 128 + 64 j .. + 63
 
 // Shared memory, from a 1024-byte aligned base. Barriers: xfull/xrel [2 slots][5 groups], sfull/sfree [2],
-// wfull/wfree [2], pfull, pfree, qfull, mdone, gbar [2], ebar, adone, bdone.
+// wfull/wfree [2], pfull, pfree, qfull, qfree, gbar [2], ebar, odone, ofree, sdone [2].
 struct AtSmem {
   static constexpr uint32_t q = 0;
   static constexpr uint32_t x = q + AT_TILE;
@@ -62,20 +68,21 @@ struct AtSmem {
   static constexpr uint32_t anyw = fac + 2 * 64 * 4;   // [2][4] u32
   static constexpr uint32_t misc = anyw + 2 * 4 * 4;   // TMEM base, abort flag
   static constexpr uint32_t bars = (misc + 8 + 7) & ~7u;
-  static constexpr uint32_t nbars = 2 * AT_NG * 2 + 2 * 4 + 4 + 3 + 2;
+  static constexpr uint32_t nbars = 2 * AT_NG * 2 + 2 * 4 + 4 + 3 + 4;
   static constexpr uint32_t total = bars + nbars * 8;
 };
 static_assert(AtSmem::total + 1024 <= 232448, "attention shared memory exceeds the 227 KB opt-in limit");
 
 struct AttnTcArgs {
   int H, N;
-  int split_len, slot0, nslot;
+  AttnGeom g;            // persistent layout: G = gridDim.x ranges over total = B * n_hg * T tiles
+  int slot0, nslot;
   int64_t nw;
   float lam_log2e;
   const uint32_t* bitmap;
   float* part_o;
   float* part_ml;
-  int hold_first;        // VK_FLAG_TEST_TIMEOUT: CTA (0,0,0) withholds its first tile's loads
+  int hold_first;        // VK_FLAG_TEST_TIMEOUT: CTA 0 withholds its first tile's loads
   int* status;
 };
 
@@ -133,6 +140,24 @@ __device__ __forceinline__ bool warp_wait_(uint64_t* bar, uint32_t parity, volat
   return __shfl_sync(0xffffffffu, w, 0);
 }
 
+// Position of a flattened tile: its row tile kt within the segment and the segment's (sequence b, head group hg).
+// Stepped without divisions (the per-tile bookkeeping sits on the issuing threads' critical path).
+struct TilePos {
+  int kt, hg, b;
+  __device__ __forceinline__ void init(long long t, int T, int n_hg) {
+    const long long seg = t / T;
+    kt = (int)(t - seg * T);
+    b = (int)(seg / n_hg);
+    hg = (int)(seg - (long long)b * n_hg);
+  }
+  __device__ __forceinline__ void next(int T, int n_hg) {
+    if (++kt == T) {
+      kt = 0;
+      if (++hg == n_hg) { hg = 0; ++b; }
+    }
+  }
+};
+
 __global__ void __launch_bounds__(AT_THREADS, 1) k_attn_tc(const __grid_constant__ CUtensorMap lmap,
                                                          const __grid_constant__ CUtensorMap rmap,
                                                          const __grid_constant__ CUtensorMap qlmap,
@@ -158,19 +183,22 @@ __global__ void __launch_bounds__(AT_THREADS, 1) k_attn_tc(const __grid_constant
   uint64_t* wfree = wfull + 2;                // [2]
   uint64_t* pfull = wfree + 2;
   uint64_t* pfree = pfull + 1;
-  uint64_t* qfull = pfree + 1;
-  uint64_t* mdone = qfull + 1;
-  uint64_t* gbar = mdone + 1;                 // [2] softmax-group syncs, by tile parity
-  uint64_t* ebar = gbar + 2;                  // softmax-group sync before the epilogue
-  uint64_t* adone = ebar + 1;                 // O^T issuer's final commit
-  uint64_t* bdone = adone + 1;                // second S issuer's final commit
+  uint64_t* qfull = pfree + 1;                // a segment's queries landed (one phase per segment)
+  uint64_t* qfree = qfull + 1;                // both S issuers are done with the previous segment's queries
+  uint64_t* gbar = qfree + 1;                 // [2] softmax-group syncs, by tile parity
+  uint64_t* ebar = gbar + 2;                  // softmax-group syncs of a segment's epilogue (two per segment)
+  uint64_t* odone = ebar + 1;                 // the segment's O^T products are complete (O^T issuer's commit)
+  uint64_t* ofree = odone + 1;                // the softmax warps have read the segment's O^T out of tensor memory
+  uint64_t* sdone = ofree + 1;                // [2] each S issuer's final commit
 
-  const int split = blockIdx.x, hg = blockIdx.y, b = blockIdx.z;
-  const int H = args.H;
-  const int h0 = hg * 64, nh = min(64, H - h0);
-  const int p0 = split * args.split_len, p1 = min(args.N, p0 + args.split_len);
-  const int ntile = p1 > p0 ? (p1 - p0 + AT_T - 1) / AT_T : 0;    // p0 is a multiple of 64
+  const AttnGeom& geo = args.g;
+  const int H = args.H, T = geo.T;
+  const long long t0 = geo.total * blockIdx.x / gridDim.x, t1 = geo.total * (blockIdx.x + 1) / gridDim.x;
+  const int ntile = (int)(t1 - t0);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  // a segment's first tile, or the first of this CTA's range, starts a new segment for every role
+  TilePos tp;
+  tp.init(t0, T, geo.n_hg);
 
   if (threadIdx.x == 0) {
     *abort_flag = 0;
@@ -181,14 +209,15 @@ __global__ void __launch_bounds__(AT_THREADS, 1) k_attn_tc(const __grid_constant
       mbar_init(&wfull[i], 1);
       mbar_init(&wfree[i], AT_SMX + 3);
       mbar_init(&gbar[i], AT_SMX);
+      mbar_init(&sdone[i], 1);
     }
     mbar_init(pfull, AT_SMX);
     mbar_init(pfree, 1);
     mbar_init(qfull, 1);
-    mbar_init(mdone, 1);
+    mbar_init(qfree, 2);
     mbar_init(ebar, AT_SMX);
-    mbar_init(adone, 1);
-    mbar_init(bdone, 1);
+    mbar_init(odone, 1);
+    mbar_init(ofree, AT_SMX);
     mbar_fence_init();
   }
   if (warp == 1) tmem_alloc(tmem_slot, AT_TMEM_COLS);
@@ -199,27 +228,22 @@ __global__ void __launch_bounds__(AT_THREADS, 1) k_attn_tc(const __grid_constant
 
   if (warp == 0) {
     // ------------------------------------------------------------------ producer
-    const uint32_t* bm = args.bitmap + ((int64_t)b * H + h0) * args.nw;
     int last_use[2 * AT_NG];                           // last load issued per (slot, group), for the drain
 #pragma unroll
     for (int i = 0; i < 2 * AT_NG; ++i) last_use[i] = -1;
-    bool qissued = false;
-    if (lane == 0 && ntile > 0) {
-      mbar_arrive_expect_tx(qfull, AT_TILE);
-      const int qrow = b * H + h0;   // rows past the group's heads belong to other heads (or are zero-filled): unused
-      for (int k = 0; k < 8; ++k) tma_load_3d_(sq + k * AT_KBLK, &qlmap, 64 * k, qrow, 0, qfull);
-      tma_load_3d_(sq + 8 * AT_KBLK, &qrmap, 0, qrow, 0, qfull);
-      qissued = true;
-    }
-    // selection words of tile t: the lane holds heads lane and lane + 32, rows 0..31 and 32..63 of the tile
-    auto fetch = [&](int t, uint4& w) {
+    int nq = 0;                                        // query loads issued
+    // selection words of tile i (at position fp): the lane holds heads lane and lane + 32, rows 0..31 and 32..63
+    TilePos fp = tp;
+    auto fetch = [&](int i, uint4& w) {
       w = make_uint4(0u, 0u, 0u, 0u);
-      if (t >= ntile) return;
-      const int pos0 = p0 + t * AT_T;
+      if (i >= ntile) return;
+      const int b = fp.b, h0 = fp.hg * 64, nh = min(64, H - h0);
+      const int pos0 = fp.kt * AT_T;
       const int64_t wi = pos0 >> 5;
-      const int left = p1 - pos0;                      // >= 1
+      const int left = args.N - pos0;                  // >= 1
       const uint32_t m0 = left >= 32 ? 0xffffffffu : ((1u << left) - 1u);
       const uint32_t m1 = left >= 64 ? 0xffffffffu : (left <= 32 ? 0u : ((1u << (left - 32)) - 1u));
+      const uint32_t* bm = args.bitmap + ((int64_t)b * H + h0) * args.nw;
       if (lane < nh) {
         const uint32_t* r = bm + (int64_t)lane * args.nw + wi;
         w.x = r[0] & m0;
@@ -233,12 +257,14 @@ __global__ void __launch_bounds__(AT_THREADS, 1) k_attn_tc(const __grid_constant
     };
     uint4 cur, nxt;
     fetch(0, cur);
+    fp.next(T, geo.n_hg);
     int u = 0;                                         // tiles loaded so far
     bool ok = true;
-    for (int t = 0; t < ntile; ++t) {
-      fetch(t + 1, nxt);
-      const int ws = t & 1;
-      if (t >= 2 && !warp_wait_(&wfree[ws], ((t >> 1) - 1) & 1, abort_flag, lane)) { ok = false; break; }
+    for (int i = 0; i < ntile; ++i, tp.next(T, geo.n_hg)) {
+      fetch(i + 1, nxt);
+      fp.next(T, geo.n_hg);
+      const int ws = i & 1;
+      if (i >= 2 && !warp_wait_(&wfree[ws], ((i >> 1) - 1) & 1, abort_flag, lane)) { ok = false; break; }
       uint32_t* wd = words + ws * 128;
       wd[lane * 2] = cur.x;
       wd[lane * 2 + 1] = cur.y;
@@ -248,38 +274,52 @@ __global__ void __launch_bounds__(AT_THREADS, 1) k_attn_tc(const __grid_constant
       if (lane == 0) unis[ws] = uni;
       __syncwarp();
       if (lane == 0) mbar_arrive(&wfull[ws]);
-      if (uni && args.hold_first && t == 0 && blockIdx.x == 0 && blockIdx.y == 0 && blockIdx.z == 0) {
+      const int b = tp.b, h0 = tp.hg * 64;
+      bool lok = true;
+      if (uni && args.hold_first && i == 0 && blockIdx.x == 0) {
         ++u;                                           // test hook: these loads are never issued
       } else if (uni) {
         const int s = u & 1, use = u >> 1;
-        const int pos0 = p0 + t * AT_T;
+        const int pos0 = tp.kt * AT_T;
         unsigned char* xs = sx + s * AT_TILE;
-        bool lok = true;
         if (lane == 0) {
-          for (int i = 0; i < AT_NG; ++i) {
-            const int g = i == 0 ? 4 : i - 1;          // RoPE block first (its slot part is released first)
-            uint64_t* fb = &xfull[s * AT_NG + g];
-            if (use > 0 && !mbar_wait(&xrel[s * AT_NG + g], (use - 1) & 1, abort_flag)) { lok = false; break; }
-            if (g == 4) {
+          for (int g = 0; g < AT_NG; ++g) {
+            const int grp = g == 0 ? 4 : g - 1;        // RoPE block first (its slot part is released first)
+            uint64_t* fb = &xfull[s * AT_NG + grp];
+            if (use > 0 && !mbar_wait(&xrel[s * AT_NG + grp], (use - 1) & 1, abort_flag)) { lok = false; break; }
+            if (grp == 4) {
               mbar_arrive_expect_tx(fb, AT_KBLK);
               tma_load_3d_(xs + 8 * AT_KBLK, &rmap, 0, pos0, b, fb);
             } else {
               mbar_arrive_expect_tx(fb, 2 * AT_KBLK);
-              tma_load_3d_(xs + (2 * g) * AT_KBLK, &lmap, 128 * g, pos0, b, fb);
-              tma_load_3d_(xs + (2 * g + 1) * AT_KBLK, &lmap, 128 * g + 64, pos0, b, fb);
+              tma_load_3d_(xs + (2 * grp) * AT_KBLK, &lmap, 128 * grp, pos0, b, fb);
+              tma_load_3d_(xs + (2 * grp + 1) * AT_KBLK, &lmap, 128 * grp + 64, pos0, b, fb);
             }
-            last_use[s * AT_NG + g] = use;
+            last_use[s * AT_NG + grp] = use;
           }
         }
-        if (!__shfl_sync(0xffffffffu, lok, 0)) { ok = false; break; }
         ++u;
       }
+      if ((i == 0 || tp.kt == 0) && lane == 0 && lok) {
+        // the segment's queries, once both S issuers are done with the previous segment's
+        if (nq > 0 && !mbar_wait(qfree, (nq - 1) & 1, abort_flag)) {
+          lok = false;
+        } else {
+          const int qrow = b * H + h0;   // rows past the group's heads belong to other heads (or are zero-filled)
+          mbar_arrive_expect_tx(qfull, AT_TILE);
+          for (int k = 0; k < 8; ++k) tma_load_3d_(sq + k * AT_KBLK, &qlmap, 64 * k, qrow, 0, qfull);
+          tma_load_3d_(sq + 8 * AT_KBLK, &qrmap, 0, qrow, 0, qfull);
+          ++nq;
+        }
+      }
+      if (!__shfl_sync(0xffffffffu, lok, 0)) { ok = false; break; }
       cur = nxt;
     }
     if (!ok && lane == 0) { raise_status(args.status, VK_ERR_TIMEOUT); *abort_flag = 1; }
-    // drain: every load issued must have landed before the CTA leaves (only matters after an abort)
+    // drain: every load issued must have landed before the CTA leaves (only matters after an abort; a query load
+    // is issued only after the previous one was consumed, so the last is the only one that can be in flight)
     if (lane == 0) {
-      if (qissued) mbar_wait(qfull, 0, nullptr);
+      if (nq > 0) mbar_wait(qfull, (nq - 1) & 1, nullptr);
       for (int i = 0; i < 2 * AT_NG; ++i)
         if (last_use[i] >= 0) mbar_wait(&xfull[i], last_use[i] & 1, nullptr);
     }
@@ -293,13 +333,18 @@ __global__ void __launch_bounds__(AT_THREADS, 1) k_attn_tc(const __grid_constant
       const uint32_t idesc_s =
           (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(AT_T >> 3) << 17) | ((uint32_t)(64 >> 4) << 24);
       const uint64_t qd = sdesc_(smem_addr(sq), 16);
-      uint64_t* done_bar = half == 0 ? mdone : bdone;
-      bool ok = mbar_wait(qfull, 0, abort_flag);
-      int u = 0;
-      for (int t = 0; t < ntile && ok; ++t) {
-        if (!mbar_wait(&wfull[t & 1], (t >> 1) & 1, abort_flag)) { ok = false; break; }
-        const uint32_t uni = unis[t & 1];
-        mbar_arrive(&wfree[t & 1]);
+      uint64_t* done_bar = &sdone[half];
+      bool ok = true;
+      int u = 0, nq = 0;
+      for (int i = 0; i < ntile; ++i, tp.next(T, geo.n_hg)) {
+        if (!mbar_wait(&wfull[i & 1], (i >> 1) & 1, abort_flag)) { ok = false; break; }
+        const uint32_t uni = unis[i & 1];
+        mbar_arrive(&wfree[i & 1]);
+        if (i == 0 || tp.kt == 0) {
+          if (nq > 0) mma_commit_(qfree);            // every S of the previous segment issued: its queries may go
+          if (!mbar_wait(qfull, nq & 1, abort_flag)) { ok = false; break; }
+          ++nq;
+        }
         if (!uni) continue;
         const int s = u & 1, use = u >> 1;
         if (use > 0 && !mbar_wait(&sfree[s], (use - 1) & 1, abort_flag)) { ok = false; break; }
@@ -341,18 +386,29 @@ __global__ void __launch_bounds__(AT_THREADS, 1) k_attn_tc(const __grid_constant
     // ------------------------------------------------------------------ O^T issuer
     // Issues each loaded tile's O^T += X_lat^T . P^T as soon as its P^T is written; its commits release the tile's
     // latent blocks for the next load into the slot. (A commit tracks this thread's own MMAs; the tile's S, issued
-    // by the other thread, completed before its softmax could start.)
+    // by the other thread, completed before its softmax could start.) At a segment boundary it commits odone (the
+    // epilogue may read O^T) and waits for ofree before the next segment's first product overwrites it.
     if (lane == 0 && ntile > 0) {
       // O^T: M = 128 dims, N = 64 heads, A = X_lat^T MN-major (bit 15), B = P^T K-major
       const uint32_t idesc_o =
           (1u << 4) | (1u << 7) | (1u << 10) | (1u << 15) | ((uint32_t)(64 >> 3) << 17) | ((uint32_t)(128 >> 4) << 24);
       const uint64_t pd = sdesc_(smem_addr(sp), 16);
       bool ok = true;
-      int u = 0;
-      for (int t = 0; t < ntile; ++t) {
-        if (!mbar_wait(&wfull[t & 1], (t >> 1) & 1, abort_flag)) { ok = false; break; }
-        const uint32_t uni = unis[t & 1];
-        mbar_arrive(&wfree[t & 1]);
+      int u = 0, useg = 0, nseg = 0, ncommit = 0;
+      for (int i = 0; i < ntile; ++i, tp.next(T, geo.n_hg)) {
+        if (!mbar_wait(&wfull[i & 1], (i >> 1) & 1, abort_flag)) { ok = false; break; }
+        const uint32_t uni = unis[i & 1];
+        mbar_arrive(&wfree[i & 1]);
+        if (i == 0 || tp.kt == 0) {
+          if (nseg > 0) {
+            mma_commit_(odone);
+            ++ncommit;
+            if (!mbar_wait(ofree, (nseg - 1) & 1, abort_flag)) { ok = false; break; }
+            tmem_fence_after();                        // the epilogue's reads of O^T came first
+          }
+          ++nseg;
+          useg = 0;
+        }
         if (!uni) continue;
         if (!mbar_wait(pfull, u & 1, abort_flag)) { ok = false; break; }
         tmem_fence_after();                            // P^T and any O^T rescale come from the softmax warps
@@ -363,15 +419,19 @@ __global__ void __launch_bounds__(AT_THREADS, 1) k_attn_tc(const __grid_constant
 #pragma unroll
           for (int ks = 0; ks < 4; ++ks)
             mma_bf16_(tmem + AT_O_COL + 64 * j, xd + (uint64_t)((2 * j * AT_KBLK + ks * 2048) >> 4),
-                      pd + (uint64_t)(ks * 2), idesc_o, (u > 0 || ks > 0) ? 1u : 0u);
+                      pd + (uint64_t)(ks * 2), idesc_o, (useg > 0 || ks > 0) ? 1u : 0u);
           mma_commit_(&xrel[s * AT_NG + j]);           // latent blocks 2j, 2j+1 of this slot are free again
         }
         mma_commit_(pfree);                            // P^T free, O^T up to date
         ++u;
+        ++useg;
       }
-      mma_commit_(adone);
+      if (nseg > 0) {
+        mma_commit_(odone);                            // the last segment's O^T is complete
+        ++ncommit;
+      }
       if (!ok) { raise_status(args.status, VK_ERR_TIMEOUT); *abort_flag = 1; }
-      mbar_wait(adone, 0, nullptr);
+      if (ncommit > 0) mbar_wait(odone, (ncommit - 1) & 1, nullptr);
     }
   } else {
     // ------------------------------------------------------------------ softmax
@@ -384,15 +444,79 @@ __global__ void __launch_bounds__(AT_THREADS, 1) k_attn_tc(const __grid_constant
     const float L = args.lam_log2e;
     const uint32_t lrow = tmem + ((uint32_t)(32 * q) << 16);
     float m = -INFINITY, mex = -INFINITY, lsum = 0.f;  // lsum: this half's share of the head's sum
-    int u = 0;
+    int u = 0, useg = 0, nseg = 0;
+    int sb = 0, shg = 0;                               // the current segment's sequence and head group
     bool ok = true;
-    for (int t = 0; t < ntile; ++t) {
-      const int ws = t & 1;
-      if (!warp_wait_(&wfull[ws], (t >> 1) & 1, abort_flag, lane)) { ok = false; break; }
-      const uint32_t uni = unis[ws];
-      const uint32_t w = words[ws * 128 + hl * 2 + hh];
+    // A segment's partial: re-base each head on its exact max, write (max, sum) and the output (unnormalised),
+    // then release the O^T accumulator. The re-basing factors go through the parity buffer the last tile did not
+    // use; a second group sync keeps the next tile from overwriting them while a warp still reads.
+    auto epilogue = [&]() -> bool {
+      if (!warp_wait_(odone, (nseg - 1) & 1, abort_flag, lane)) return false;   // the segment's O^T is complete
+      float lt = lsum + __shfl_xor_sync(0xffffffffu, lsum, 16);                // both halves of the head
+      float ff = 1.f;
+      if (mex != -INFINITY && m != mex) ff = ex2(m - mex);
+      lt *= ff;
+      float* facf = fac + (u & 1) * 64;
+      if (own) facf[hl] = ff;
       __syncwarp();
-      if (lane == 0) mbar_arrive(&wfree[ws]);
+      if (lane == 0) mbar_arrive(ebar);
+      if (!warp_wait_(ebar, 0, abort_flag, lane)) return false;
+      tmem_fence_after();
+      const int h0 = shg * 64, nh = min(64, H - h0);
+      const int slot = (int)blockIdx.x - attn_cta_of(geo, ((long long)sb * geo.n_hg + shg) * T);
+      const int64_t hbase = ((int64_t)sb * args.nslot + args.slot0 + slot) * H + h0;
+      constexpr float LN2 = 0.6931471805599453f;
+      if (own && hl < nh) {
+        args.part_ml[(hbase + hl) * 2] = mex * LN2;
+        args.part_ml[(hbase + hl) * 2 + 1] = lt;
+      }
+      // O^T block j on this warp's lanes: dims 128 j + 32 q + lane; columns: heads
+#pragma unroll 1
+      for (int j = 0; j < 4; ++j) {
+        const int dim = 128 * j + 32 * q + lane;
+#pragma unroll 1
+        for (int c = 0; c < 64; c += 32) {
+          float v[32];
+          if (useg > 0) {
+            tmem_ld32_(lrow + AT_O_COL + 64 * j + c, v);
+            tmem_wait_ld();
+          } else {
+#pragma unroll
+            for (int i = 0; i < 32; ++i) v[i] = 0.f;
+          }
+#pragma unroll
+          for (int i = 0; i < 32; ++i)
+            if (c + i < nh) args.part_o[(hbase + c + i) * D_LAT + dim] = v[i] * facf[c + i];
+        }
+      }
+      tmem_fence_before();
+      __syncwarp();
+      if (lane == 0) { mbar_arrive(ofree); mbar_arrive(ebar); }
+      return warp_wait_(ebar, 1, abort_flag, lane);
+    };
+    // one pass past the last tile closes the last segment: the epilogue has a single (inlined) call site, which
+    // keeps the loop's code small (instruction fetch is shared with the issuing warps' loops)
+    for (int i = 0; i <= ntile; ++i, tp.next(T, geo.n_hg)) {
+      const int ws = i & 1;
+      uint32_t uni = 0u, w = 0u;
+      const bool fresh = i == ntile || i == 0 || tp.kt == 0;
+      if (i < ntile) {
+        if (!warp_wait_(&wfull[ws], (i >> 1) & 1, abort_flag, lane)) { ok = false; break; }
+        uni = unis[ws];
+        w = words[ws * 128 + hl * 2 + hh];
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&wfree[ws]);
+      }
+      if (fresh) {
+        if (nseg > 0 && !epilogue()) { ok = false; break; }
+        if (i == ntile) break;
+        ++nseg;
+        sb = tp.b;
+        shg = tp.hg;
+        useg = 0;
+        m = mex = -INFINITY;
+        lsum = 0.f;
+      }
       if (!uni) continue;
       const int s = u & 1, use = u >> 1, par = u & 1;
       if (!warp_wait_(&sfull[s], use & 1, abort_flag, lane)) { ok = false; break; }
@@ -495,51 +619,9 @@ __global__ void __launch_bounds__(AT_THREADS, 1) k_attn_tc(const __grid_constant
       __syncwarp();
       if (lane == 0) mbar_arrive(pfull);
       ++u;
+      ++useg;
     }
-    // the last O^T product
-    if (ok && u > 0) ok = warp_wait_(pfree, (u - 1) & 1, abort_flag, lane);
-    lsum += __shfl_xor_sync(0xffffffffu, lsum, 16);    // both halves of the head
-    if (ok) {
-      // re-base each head on its exact max; the factors go through the parity buffer the last tile did not use
-      float ff = 1.f;
-      if (mex != -INFINITY && m != mex) ff = ex2(m - mex);
-      lsum *= ff;
-      float* facf = fac + (u & 1) * 64;
-      if (own) facf[hl] = ff;
-      __syncwarp();
-      if (lane == 0) mbar_arrive(ebar);
-      ok = warp_wait_(ebar, 0, abort_flag, lane);
-    }
-    if (ok) {
-      tmem_fence_after();
-      const float* facf = fac + (u & 1) * 64;
-      const int slot = args.slot0 + split;
-      const int64_t hbase = ((int64_t)b * args.nslot + slot) * H + h0;
-      constexpr float LN2 = 0.6931471805599453f;
-      if (own && hl < nh) {
-        args.part_ml[(hbase + hl) * 2] = mex * LN2;
-        args.part_ml[(hbase + hl) * 2 + 1] = lsum;
-      }
-      // O^T block j on this warp's lanes: dims 128 j + 32 q + lane; columns: heads
-#pragma unroll 1
-      for (int j = 0; j < 4; ++j) {
-        const int dim = 128 * j + 32 * q + lane;
-#pragma unroll 1
-        for (int c = 0; c < 64; c += 32) {
-          float v[32];
-          if (u > 0) {
-            tmem_ld32_(lrow + AT_O_COL + 64 * j + c, v);
-            tmem_wait_ld();
-          } else {
-#pragma unroll
-            for (int i = 0; i < 32; ++i) v[i] = 0.f;
-          }
-#pragma unroll
-          for (int i = 0; i < 32; ++i)
-            if (c + i < nh) args.part_o[(hbase + c + i) * D_LAT + dim] = v[i] * facf[c + i];
-        }
-      }
-    } else if (lane == 0) {
+    if (!ok && lane == 0) {
       raise_status(args.status, VK_ERR_TIMEOUT);
       *abort_flag = 1;
     }
@@ -582,11 +664,13 @@ static bool make_map3(CUtensorMap* map, const void* base, uint64_t cols, uint64_
                    CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-cudaError_t launch_attn_tc(const vk_view& v, float lam, const uint32_t* bitmap, int64_t nw, int nsplit, int split_len,
+cudaError_t launch_attn_tc(const vk_view& v, float lam, const uint32_t* bitmap, int64_t nw, const AttnGeom& g,
                            int slot0, int nslot, float* part_o, float* part_ml, uint32_t flags, int* status,
                            cudaStream_t st) {
   if (!encode2()) return cudaErrorNotSupported;
-  if (split_len % AT_T != 0) return cudaErrorInvalidValue;
+  if (g.G < 1 || g.G > g.total || g.T != (v.N + AT_T - 1) / AT_T || g.n_hg != (v.H + 63) / 64 ||
+      g.total != (long long)v.B * g.n_hg * g.T)
+    return cudaErrorInvalidValue;
   CUtensorMap lmap, rmap, qlmap, qrmap;
   // cache rows: latent [B][N][512] and RoPE [B][N][64]; queries: [B*H][512] and [B*H][64]; 64-row boxes
   if (!make_map3(&lmap, v.latent, D_LAT, v.N, v.B, v.latent_ld, v.latent_bstride, AT_T) ||
@@ -597,7 +681,7 @@ cudaError_t launch_attn_tc(const vk_view& v, float lam, const uint32_t* bitmap, 
   AttnTcArgs a{};
   a.H = v.H;
   a.N = v.N;
-  a.split_len = split_len;
+  a.g = g;
   a.slot0 = slot0;
   a.nslot = nslot;
   a.nw = nw;
@@ -610,8 +694,7 @@ cudaError_t launch_attn_tc(const vk_view& v, float lam, const uint32_t* bitmap, 
   const size_t smem = AtSmem::total + 1024;
   cudaError_t e = cudaFuncSetAttribute(k_attn_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
-  dim3 grid(nsplit, (v.H + 63) / 64, v.B);
-  k_attn_tc<<<grid, AT_THREADS, smem, st>>>(lmap, rmap, qlmap, qrmap, a);
+  k_attn_tc<<<g.G, AT_THREADS, smem, st>>>(lmap, rmap, qlmap, qrmap, a);
   count_launches(1);
   return cudaGetLastError();
 }

@@ -45,7 +45,7 @@ int cuda_fail(cudaError_t e, const char* where) {
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
 constexpr int64_t MAX_N = (1 << 24) - 1;
-constexpr int NUM_SMS_TARGET = 152;   // GB300 SMs; attention splits are sized in whole waves
+constexpr int NUM_SMS_TARGET = 152;   // GB300 SMs: the attention's CTA count
 
 int check_view(const vk_view* v) {
   if (!v) return fail(VK_ERR_INVALID_ARG, "view is NULL");
@@ -129,6 +129,35 @@ void choose_splits(const vk_view& v, int64_t* nsplit, int64_t* split_len) {
   *nsplit = (N + best_len - 1) / best_len;
 }
 
+}  // namespace
+
+namespace vk {
+// Partial-result layout of the attention kernel that runs for this view: the persistent layout for the
+// tensor-core kernel, the split layout for the fp32 kernel. Persistent: one CTA per SM, but at least 4 tiles per
+// CTA -- a partial (64 heads x 512 fp32 = 128 KB) costs more traffic than a tile (72 KB), so small problems take
+// fewer, longer ranges.
+AttnGeom attn_geom(const vk_view& v) {
+  AttnGeom g{};
+  g.n_hg = (v.H + HG - 1) / HG;
+  g.T = (v.N + 63) / 64;
+  g.total = (long long)v.B * g.n_hg * g.T;
+  if (attn_tc_supported(v)) {
+    g.G = (int)std::min<long long>(std::max<long long>(1, g.total / 4), NUM_SMS_TARGET);
+    g.nslot = 1;
+    for (long long s = 0; s < (long long)v.B * g.n_hg; ++s) g.nslot = std::max(g.nslot, attn_nvalid(g, s));
+  } else {
+    int64_t ns = 0, len = 0;
+    choose_splits(v, &ns, &len);
+    g.nsplit = (int)ns;
+    g.split_len = (int)len;
+    g.nslot = (int)ns;
+  }
+  return g;
+}
+}  // namespace vk
+
+namespace {
+
 // Fused selection parameters: a strided sample of about 2048+ archive rows per head gives theta = its j-th
 // largest score, with j chosen so that ~1.5 k + 8 samples' worth of archive rows pass; the candidate list has
 // room for twice that (+2048) before the exact fallback takes over.
@@ -152,7 +181,7 @@ VkLayout make_layout(const vk_view& v, const vk_params& p) {
   L.B = v.B; L.H = v.H; L.N = v.N;
   L.nw = (v.N + 31) / 32;
   L.n_hg = (v.H + vk::HG - 1) / vk::HG;
-  choose_splits(v, &L.nsplit, &L.split_len);
+  L.ag = vk::attn_geom(v);
   L.two_tier = p.trigger != VK_TRIG_OFF;
   L.tc = vk::score_tc_supported(v, p.r);
   L.fused = L.tc && !(p.flags & VK_FLAG_FORCE_DENSE);
@@ -162,7 +191,7 @@ VkLayout make_layout(const vk_view& v, const vk_params& p) {
   if (L.fused) fused_params(v.N, lo, hi, k, &L);
   L.fcap = (L.fused && L.two_tier && p.top_j > 0) ? std::max<int64_t>(1, hi - lo) : 0;
   const int64_t BH = (int64_t)v.B * v.H;
-  const int64_t nslot = L.nsplit * (L.two_tier ? 2 : 1);
+  const int64_t nslot = (int64_t)L.ag.nslot * (L.two_tier ? 2 : 1);
   size_t off = 0;
   auto take = [&](size_t bytes) { size_t o = off; off = align_up(off + bytes, 256); return o; };
   L.off_status = take(256);
@@ -327,9 +356,9 @@ int vk_sparse_attn(const vk_view* view, const vk_params* params, const int32_t* 
   float* po = at<float>(ws, L.off_part_o);
   float* pml = at<float>(ws, L.off_part_ml);
   VK_CUDA(vk::launch_list_to_bitmap(view->B, view->H, view->N, idx, count, cap, bm, L.nw, status, st), "list_to_bitmap");
-  VK_CUDA(vk::launch_attn(*view, params->sm_scale, bm, L.nw, (int)L.nsplit, (int)L.split_len, 0, (int)L.nsplit, po, pml, params->flags,
-                          status, st), "attention");
-  VK_CUDA(vk::launch_combine(view->B, view->H, (int)L.nsplit, (int)L.nsplit, po, pml, out, lse, smax, st), "combine");
+  VK_CUDA(vk::launch_attn(*view, params->sm_scale, bm, L.nw, L.ag, 0, L.ag.nslot, po, pml, params->flags, status, st),
+          "attention");
+  VK_CUDA(vk::launch_combine(view->B, view->H, L.ag, L.ag.nslot, po, pml, out, lse, smax, st), "combine");
   return VK_OK;
 }
 
@@ -359,7 +388,7 @@ int vk_decode_step(const vk_view* view, const vk_params* params, const vk_index*
   uint32_t* selbm = at<uint32_t>(ws, L.off_selbm);
   float* po = at<float>(ws, L.off_part_o);
   float* pml = at<float>(ws, L.off_part_ml);
-  const int ns = (int)L.nsplit, nslot = two_tier ? 2 * ns : ns;
+  const int ns = L.ag.nslot, nslot = two_tier ? 2 * ns : ns;
 
   const int lo = S, hi = N - W;
   prof(0, st);
@@ -412,14 +441,14 @@ int vk_decode_step(const vk_view* view, const vk_params* params, const vk_index*
             "select");
   }
   prof(3, st);
-  VK_CUDA(vk::launch_attn(v, params->sm_scale, selbm, L.nw, ns, (int)L.split_len, 0, nslot, po, pml, params->flags, status, st),
+  VK_CUDA(vk::launch_attn(v, params->sm_scale, selbm, L.nw, L.ag, 0, nslot, po, pml, params->flags, status, st),
           "attention");
   prof(4, st);
   if (two_tier) {
     float* smax1 = at<float>(ws, L.off_smax1);
     int64_t* nfired = at<int64_t>(ws, L.off_nfired);
     uint32_t* firebm = at<uint32_t>(ws, L.off_firebm);
-    VK_CUDA(vk::launch_smax_reduce(B, H, ns, nslot, pml, smax1, st), "smax");
+    VK_CUDA(vk::launch_smax_reduce(B, H, L.ag, nslot, pml, smax1, st), "smax");
     if (L.fused) {
       vk::ScoreTcArgs t{};
       t.mode = 2;
@@ -461,11 +490,11 @@ int vk_decode_step(const vk_view* view, const vk_params* params, const vk_index*
         VK_CUDA(vk::launch_bitmap_to_list(B, H, N, firebm, L.nw, idx, count, cap, status, st), "fired list");
       }
     }
-    VK_CUDA(vk::launch_attn(v, params->sm_scale, firebm, L.nw, ns, (int)L.split_len, ns, nslot, po, pml, 0u, status, st),
+    VK_CUDA(vk::launch_attn(v, params->sm_scale, firebm, L.nw, L.ag, ns, nslot, po, pml, 0u, status, st),
             "fired attention");
   }
   prof(5, st);
-  VK_CUDA(vk::launch_combine(B, H, nslot, ns, po, pml, out, lse, smax, st), "combine");
+  VK_CUDA(vk::launch_combine(B, H, L.ag, nslot, po, pml, out, lse, smax, st), "combine");
   prof(6, st);
   return VK_OK;
 }

@@ -68,14 +68,39 @@ __device__ __forceinline__ int block_exclusive_scan(int v, int* scratch, int* to
   return prefix;
 }
 
+// ------------------------------------------------------------------------------------------ attention partials
+// Where the attention writes its partial results (part_o [B][nslot][H][512], part_ml [B][nslot][H][2]). The work
+// is made of B * n_hg segments (sequence, head group of 64), each of T = ceil(N / 64) row tiles.
+//  * split layout (fp32 kernel, G = 0): every segment is cut into nsplit ranges of split_len positions, one CTA
+//    each, and all nsplit slots of every segment are written;
+//  * persistent layout (tensor-core kernel, G > 0): the segments' tiles are flattened segment-major and cut into
+//    G equal contiguous ranges, one CTA each; a segment owns one slot per CTA its tiles fall in, numbered from 0
+//    by CTA, so segment s has attn_nvalid(s) written slots.
+// nslot is the slot count of one tier (the largest attn_nvalid); the fired rows of the two-tier path use slots
+// nslot .. 2 nslot - 1 the same way.
+struct AttnGeom {
+  int nslot;
+  int nsplit, split_len;     // split layout
+  int G, T, n_hg;            // persistent layout
+  long long total;           // B * n_hg * T
+};
+// The CTA of the persistent layout whose range holds flattened tile t: ranges are [c total / G, (c+1) total / G).
+__host__ __device__ inline int attn_cta_of(const AttnGeom& g, long long t) {
+  return (int)(((t + 1) * (long long)g.G - 1) / g.total);
+}
+// Written slots of segment s (per tier).
+__host__ __device__ inline int attn_nvalid(const AttnGeom& g, long long s) {
+  if (g.G == 0) return g.nslot;
+  return attn_cta_of(g, (s + 1) * g.T - 1) - attn_cta_of(g, s * g.T) + 1;
+}
+
 }  // namespace vk
 
 // ------------------------------------------------------------------------------------------ workspace
 // Byte offsets of every scratch region inside the caller's workspace, for one set of shapes.
 struct VkLayout {
   int64_t B, H, N, nw;          // nw = 32-bit words per head bitmap
-  int64_t nsplit;               // attention splits per sequence (per tier)
-  int64_t split_len;            // positions per split (multiple of 32)
+  vk::AttnGeom ag;              // where the attention writes its partials
   int64_t n_hg;                 // head groups of 64
   bool dense_scores;            // materialised [B,H,N] scores are part of the layout
   bool two_tier;
@@ -106,15 +131,15 @@ cudaError_t launch_list_to_bitmap(int B, int H, int N, const int32_t* idx, const
                                   uint32_t* bitmap, int64_t nw, int* status, cudaStream_t st);
 size_t attn_smem_bytes(int dtype, int H, int split_len);
 bool attn_tc_supported(const vk_view& v);
-cudaError_t launch_attn_tc(const vk_view& v, float lam, const uint32_t* bitmap, int64_t nw, int nsplit, int split_len,
+AttnGeom attn_geom(const vk_view& v);
+cudaError_t launch_attn_tc(const vk_view& v, float lam, const uint32_t* bitmap, int64_t nw, const AttnGeom& g,
                            int slot0, int nslot, float* part_o, float* part_ml, uint32_t flags, int* status,
                            cudaStream_t st);
-cudaError_t launch_attn(const vk_view& v, float lam, const uint32_t* bitmap, int64_t nw, int nsplit,
-                        int split_len, int slot0, int nslot, float* part_o, float* part_ml, uint32_t flags,
-                        int* status, cudaStream_t st);
-cudaError_t launch_smax_reduce(int B, int H, int nsplit, int nslot, const float* part_ml, float* smax,
+cudaError_t launch_attn(const vk_view& v, float lam, const uint32_t* bitmap, int64_t nw, const AttnGeom& g, int slot0,
+                        int nslot, float* part_o, float* part_ml, uint32_t flags, int* status, cudaStream_t st);
+cudaError_t launch_smax_reduce(int B, int H, const AttnGeom& g, int nslot, const float* part_ml, float* smax,
                                cudaStream_t st);
-cudaError_t launch_combine(int B, int H, int nslot, int nslot_tier1, const float* part_o, const float* part_ml,
+cudaError_t launch_combine(int B, int H, const AttnGeom& g, int nslot, const float* part_o, const float* part_ml,
                            float* out, float* lse, float* smax, cudaStream_t st);
 cudaError_t launch_trigger_dense(int B, int H, int N, int W, int n_sink, float lam, float z_eff, int top_j,
                                  float* scores, const float* qcn, const float* qrn, const float* eta,

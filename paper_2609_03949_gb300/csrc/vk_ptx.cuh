@@ -65,9 +65,15 @@ __device__ __forceinline__ bool mbar_test_wait(uint64_t* bar, uint32_t parity) {
 }
 
 // Wait until the phase with this parity has completed. Returns false if it gave up (after kWaitNs, or earlier
-// once *abort is set by another warp that gave up).
+// once *abort is set by another warp that gave up). The first test is inlined; the polling loop is one out-of-line
+// copy per translation unit: inlined at every call site it made the warp-specialised kernels' code large enough
+// for instruction fetch to stall their hot loops.
+static __device__ __noinline__ bool mbar_wait_slow(uint64_t* bar, uint32_t parity, volatile int* abort);
 __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volatile int* abort) {
   if (mbar_try_wait(bar, parity)) return true;
+  return mbar_wait_slow(bar, parity, abort);
+}
+static __device__ __noinline__ bool mbar_wait_slow(uint64_t* bar, uint32_t parity, volatile int* abort) {
   const uint64_t t0 = global_ns();
   for (uint32_t it = 1;; ++it) {
     if (mbar_try_wait(bar, parity)) return true;
