@@ -105,10 +105,13 @@ struct RecomputedKeys {
 
 // Ascending ids of the set bits of wbm[0, nw), written to out[base ...] (entries past cap are dropped). Each warp
 // takes a contiguous range of words, counts its bits, one barrier shares the warps' totals, then every warp
-// writes its ids with warp-level prefix sums over 32-word chunks. Returns base + the number of set bits. Called
-// by the whole block (blockDim a multiple of 32, at most 1024); scratch holds 32 ints.
+// writes its ids in groups of eight 32-word chunks: the eight chunks' warp prefix sums run interleaved (one scan
+// latency per group, not per chunk), then each lane writes the ids of its word in every chunk -- a sparse word bit
+// by bit, a full word (the window, sinks) by the whole warp, one id per lane. Returns base + the number of set
+// bits. Called by the whole block (blockDim a multiple of 32, at most 1024); scratch holds 32 ints.
 __device__ __forceinline__ int bitmap_to_ids(const uint32_t* wbm, long long nw, int32_t* out, int base, int cap,
                                              int* scratch) {
+  constexpr int GC = 8;                              // chunks per group
   const int lane = threadIdx.x & 31, w = threadIdx.x >> 5, nwarp = blockDim.x >> 5;
   const long long per = ((nw + nwarp - 1) / nwarp + 31) / 32 * 32;   // words per warp, whole chunks
   const long long w0 = (long long)w * per, w1 = min(nw, w0 + per);
@@ -124,25 +127,46 @@ __device__ __forceinline__ int bitmap_to_ids(const uint32_t* wbm, long long nw, 
     if (i < w) pos += c;
     total += c;
   }
-  for (long long c0 = w0; c0 < w1; c0 += 32) {
-    const long long i = c0 + lane;
-    const uint32_t word = i < w1 ? wbm[i] : 0u;
-    const int n = __popc(word);
-    int incl = n;
+  for (long long g0 = w0; g0 < w1; g0 += 32 * GC) {
+    uint32_t wv[GC];
+    int n[GC], inc[GC];
+#pragma unroll
+    for (int j = 0; j < GC; ++j) {
+      const long long i = g0 + 32 * j + lane;
+      wv[j] = i < w1 ? wbm[i] : 0u;
+      n[j] = __popc(wv[j]);
+      inc[j] = n[j];
+    }
 #pragma unroll
     for (int d = 1; d < 32; d <<= 1) {
-      const int y = __shfl_up_sync(0xffffffffu, incl, d);
-      if (lane >= d) incl += y;
+#pragma unroll
+      for (int j = 0; j < GC; ++j) {
+        const int y = __shfl_up_sync(0xffffffffu, inc[j], d);
+        if (lane >= d) inc[j] += y;
+      }
     }
-    int p = pos + incl - n;
-    uint32_t bits = word;
-    while (bits) {
-      const int b = __ffs(bits) - 1;
-      bits &= bits - 1;
-      if (p < cap) out[p] = (int32_t)(i * 32 + b);
-      ++p;
+#pragma unroll
+    for (int j = 0; j < GC; ++j) {
+      const long long c0 = g0 + 32 * j;
+      const int p0 = pos + inc[j] - n[j];
+      const bool full = wv[j] == 0xffffffffu;
+      int p = p0;
+      uint32_t bits = full ? 0u : wv[j];
+      while (bits) {
+        const int b = __ffs(bits) - 1;
+        bits &= bits - 1;
+        if (p < cap) out[p] = (int32_t)((c0 + lane) * 32 + b);
+        ++p;
+      }
+      uint32_t fl = __ballot_sync(0xffffffffu, full);
+      while (fl) {
+        const int src = __ffs(fl) - 1;
+        fl &= fl - 1;
+        const int ps = __shfl_sync(0xffffffffu, p0, src) + lane;
+        if (ps < cap) out[ps] = (int32_t)((c0 + src) * 32 + lane);
+      }
+      pos += __shfl_sync(0xffffffffu, inc[j], 31);
     }
-    pos += __shfl_sync(0xffffffffu, incl, 31);
   }
   return base + total;
 }
@@ -164,18 +188,23 @@ __device__ __forceinline__ void block_and_or(uint32_t& a, uint32_t& o, uint32_t*
 // differing bit (bits above it are common to all keys, so they take no pass and pile into no single bin).
 // With max_passes < 4 the result is the lower bound of the bucket reached (a key <= the k-th largest).
 // Returns the key; *need_out = how many keys equal to it are among the k (exact result only); *ties_out = how
-// many keys fall in its final bucket. Called by the whole block.
-template <class KeyAt>
-__device__ uint32_t radix_kth_desc(const KeyAt& key_at, int n, unsigned int k, unsigned int* hist, uint32_t* scratch,
-                                   unsigned int* need_out, unsigned int* ties_out, int max_passes = 8) {
+// many keys fall in its final bucket. Called by the whole block; each_key(f) calls f(key) for every key this
+// thread holds (in registers, shared or global memory). With mask_out, the select stops as soon as the bucket
+// holding the k-th largest key holds exactly the keys still needed: the k largest are then the keys whose bits
+// under *mask_out are >= the returned prefix (*need_out == *ties_out).
+template <class EachKey>
+__device__ uint32_t radix_kth_desc(const EachKey& each_key, int n, unsigned int k, unsigned int* hist,
+                                   uint32_t* scratch, unsigned int* need_out, unsigned int* ties_out,
+                                   int max_passes = 8, uint32_t* mask_out = nullptr) {
   __shared__ unsigned int s_digit, s_above, s_cnt;
   uint32_t kand = 0xffffffffu, kor = 0u;
-  for (int i = threadIdx.x; i < n; i += blockDim.x) { const uint32_t key = key_at(i); kand &= key; kor |= key; }
+  each_key([&](uint32_t key) { kand &= key; kor |= key; });
   block_and_or(kand, kor, scratch);
   const uint32_t diff = kand ^ kor;
   if (diff == 0u) {                                   // all keys equal
     *need_out = k;
     *ties_out = (unsigned int)n;
+    if (mask_out) *mask_out = 0xffffffffu;
     return kand;
   }
   int hb = 31 - __clz(diff);                          // highest differing bit
@@ -187,10 +216,9 @@ __device__ uint32_t radix_kth_desc(const KeyAt& key_at, int n, unsigned int k, u
     const uint32_t dmask = (2u << (hb - shift)) - 1u;   // digit of hb - shift + 1 <= 8 bits
     for (int i = threadIdx.x; i < 256; i += blockDim.x) hist[i] = 0;
     __syncthreads();
-    for (int i = threadIdx.x; i < n; i += blockDim.x) {
-      const uint32_t key = key_at(i);
+    each_key([&](uint32_t key) {
       if ((key & mask) == prefix) atomicAdd(&hist[(key >> shift) & dmask], 1u);
-    }
+    });
     __syncthreads();
     if (threadIdx.x < 32) pick_digit_desc(hist, need, &s_digit, &s_above, &s_cnt);
     __syncthreads();
@@ -199,11 +227,12 @@ __device__ uint32_t radix_kth_desc(const KeyAt& key_at, int n, unsigned int k, u
     need -= s_above;
     ties = s_cnt;
     __syncthreads();
-    if (shift == 0 || pass + 1 >= max_passes) break;
+    if (shift == 0 || pass + 1 >= max_passes || (mask_out && ties == need)) break;
     hb = shift - 1;
   }
   *need_out = need;
   *ties_out = ties;
+  if (mask_out) *mask_out = mask;
   return prefix;
 }
 
@@ -303,11 +332,12 @@ cudaError_t launch_select_dense(int B, int H, int N, const float* scores, const 
 // ---------------------------------------------------------------------------------------------- fused path
 // Threshold from a strided sample of the archive: theta[b,h] = the j-th largest sampled score, so that about
 // j * stride archive rows score >= theta (chosen well above k). The candidate pass then emits only those rows.
-// sample[(b*H + h) * ns + i] is the score of position off + stride * i.
+// sample[(b*H + h) * ns + i] is the score of position off + stride * i. Up to THETA_R x 256 archive samples are
+// held in registers (THETA_R per thread, loaded together); more go through shared memory (ns x 4 bytes).
+constexpr int THETA_R = 16;
 __global__ void __launch_bounds__(CAND_THREADS) k_theta(int ns, int off, int stride, int lo, int hi, int j,
                                                         const float* __restrict__ sample, float* __restrict__ theta) {
   extern __shared__ __align__(16) unsigned char smem[];
-  uint32_t* keys = reinterpret_cast<uint32_t*>(smem);         // the archive samples' keys
   __shared__ unsigned int hist[256];
   __shared__ uint32_t scratch[64];
   const int64_t bh = blockIdx.x;
@@ -316,21 +346,6 @@ __global__ void __launch_bounds__(CAND_THREADS) k_theta(int ns, int off, int str
   const int i0 = lo > off ? (lo - off + stride - 1) / stride : 0;
   const int i1 = min(ns, hi > off ? (hi - off + stride - 1) / stride : 0);
   const int na = max(0, i1 - i0);
-  // all of a thread's loads in flight at once (the block is otherwise latency-bound on them)
-  for (int i = threadIdx.x; i < na; i += 16 * blockDim.x) {
-    float v[16];
-#pragma unroll
-    for (int r = 0; r < 16; ++r) {
-      const int e = i + r * blockDim.x;
-      v[r] = e < na ? a[i0 + e] : 0.f;
-    }
-#pragma unroll
-    for (int r = 0; r < 16; ++r) {
-      const int e = i + r * blockDim.x;
-      if (e < na) keys[e] = fkey(v[r]);
-    }
-  }
-  __syncthreads();
   if (j <= 0 || j > na) {
     if (threadIdx.x == 0) theta[bh] = -INFINITY;      // emit every archive row
     return;
@@ -338,14 +353,48 @@ __global__ void __launch_bounds__(CAND_THREADS) k_theta(int ns, int off, int str
   unsigned int need_eq, ties;
   // two digits below the samples' first differing bit pin the j-th largest to a bucket of 2^-16 of their key
   // range; its lower bound is theta (a little below the exact order statistic: a few more candidates pass)
-  const uint32_t prefix =
-      radix_kth_desc([&](int i) { return keys[i]; }, na, (unsigned int)j, hist, scratch, &need_eq, &ties, 2);
+  uint32_t prefix;
+  if (na <= THETA_R * CAND_THREADS) {
+    uint32_t kr[THETA_R];
+#pragma unroll
+    for (int r = 0; r < THETA_R; ++r) {
+      const int e = threadIdx.x + r * CAND_THREADS;
+      kr[r] = fkey(e < na ? a[i0 + e] : 0.f);
+    }
+    auto each_key = [&](auto f) {
+#pragma unroll
+      for (int r = 0; r < THETA_R; ++r)
+        if (threadIdx.x + r * CAND_THREADS < na) f(kr[r]);
+    };
+    prefix = radix_kth_desc(each_key, na, (unsigned int)j, hist, scratch, &need_eq, &ties, 2);
+  } else {
+    uint32_t* keys = reinterpret_cast<uint32_t*>(smem);         // the archive samples' keys
+    for (int i = threadIdx.x; i < na; i += 16 * CAND_THREADS) {
+      float v[16];
+#pragma unroll
+      for (int r = 0; r < 16; ++r) {
+        const int e = i + r * CAND_THREADS;
+        v[r] = e < na ? a[i0 + e] : 0.f;
+      }
+#pragma unroll
+      for (int r = 0; r < 16; ++r) {
+        const int e = i + r * CAND_THREADS;
+        if (e < na) keys[e] = fkey(v[r]);
+      }
+    }
+    __syncthreads();
+    auto each_key = [&](auto f) {
+      for (int i = threadIdx.x; i < na; i += CAND_THREADS) f(keys[i]);
+    };
+    prefix = radix_kth_desc(each_key, na, (unsigned int)j, hist, scratch, &need_eq, &ties, 2);
+  }
   if (threadIdx.x == 0) theta[bh] = funkey(prefix);
 }
 
 cudaError_t launch_theta(int B, int H, int ns, int off, int stride, int lo, int hi, int j, const float* sample,
                          float* theta, cudaStream_t st) {
-  const size_t smem = (size_t)ns * 4;
+  // shared memory only when the samples outgrow the registers (na <= ns)
+  const size_t smem = ns > THETA_R * CAND_THREADS ? (size_t)ns * 4 : 0;
   cudaError_t e = cudaFuncSetAttribute(k_theta, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
   k_theta<<<B * H, CAND_THREADS, smem, st>>>(ns, off, stride, lo, hi, j, sample, theta);
@@ -353,68 +402,34 @@ cudaError_t launch_theta(int B, int H, int ns, int off, int stride, int lo, int 
   return cudaGetLastError();
 }
 
-// Selection from a head's candidate list (every archive row with score >= theta, in arbitrary order). When the
-// list holds at least k and at most capc entries it contains the whole top-k, which is found by a radix select
-// (ties by smaller position, via a second select on the positions of the tied keys); the selected rows, the
-// sinks and the window become the head's bitmap and ascending id list. The keys are read from the list (L2-resident
-// after the scoring pass) on every radix pass: shared memory holds only the bitmap, so 8 blocks fit per SM and
-// hide each other's latency. When the list is too short or too long
-// (theta landed too high or too low) or with VK_FLAG_FORCE_FALLBACK, the head takes the exact ordered selection
-// over scores recomputed from the RoPE columns. With `append` (the top_j of the fired rows, whose list can never
-// overflow) only candidates are selected, no sinks or window, and the ids are appended after count[b,h].
-__global__ void __launch_bounds__(CAND_THREADS, 8) k_select_cand(
-    int H, int N, int lo, int hi, long long k_all, const long long* __restrict__ k_per_head,
-    const int* __restrict__ cand_cnt, const int2* __restrict__ cand, int capc, int force_fallback,
-    const __nv_bfloat16* __restrict__ rope, int64_t rld, int64_t rbs, const float* __restrict__ qt,
-    int32_t* __restrict__ idx, int32_t* __restrict__ count, int cap, int append, float* __restrict__ kth,
-    uint32_t* __restrict__ bitmap, long long nw, int* status) {
-  extern __shared__ __align__(16) unsigned char smem[];
-  uint32_t* sbm = reinterpret_cast<uint32_t*>(smem);           // the head's bitmap words, when they fit
+// The selection proper from a head's candidates: the k-th largest key tau by radix select, then -- when more
+// keys equal tau than are needed -- the `need` smallest positions among the tied ones by a second radix select
+// on positions; the selected rows (plus sinks and window unless appending) become the head's bitmap and its
+// ascending id list. each_kp(f) calls f(key, position) for every candidate this thread holds.
+template <class EachKP>
+__device__ void select_from_candidates(const EachKP& each_kp, int c, long long k, int N, int lo, int hi, int append,
+                                       uint32_t* sbm, uint32_t* bm, long long nw, int32_t* out, int32_t* count_bh,
+                                       int cap, float* kth_bh, int* status) {
   __shared__ unsigned int hist[256];
   __shared__ uint32_t scratch[64];
   __shared__ unsigned int s_digit, s_above;
-  __shared__ float qts[D_ROPE];
   __shared__ int scan_scratch[33];
-  const int64_t bh = blockIdx.x;
-  const int b = (int)(bh / H);
-  long long k = k_all;
-  if (k_per_head) k = min(k, k_per_head[bh]);
-  const int c = cand_cnt[bh];
-  if (append) k = min(k, (long long)c);
-  uint32_t* bm = bitmap + bh * nw;
-  int32_t* out = idx + bh * (int64_t)cap;
-
-  if (force_fallback || c < k || c > capc) {
-    if (append) {                       // cannot happen: the fired list has room for the whole archive
-      if (threadIdx.x == 0) raise_status(status, VK_ERR_CAPACITY);
-      return;
-    }
-    for (int i = threadIdx.x; i < D_ROPE; i += blockDim.x) qts[i] = qt[bh * D_ROPE + i];
-    __syncthreads();
-    RecomputedKeys keys{rope + (int64_t)b * rbs, rld, qts};
-    select_ordered(keys, N, lo, hi, k, out, count + bh, cap, 0, kth ? kth + bh : nullptr, bm, nw, status);
-    return;
-  }
-
-  const int2* g = cand + bh * (int64_t)capc;
-  auto key_at = [&](int i) -> uint32_t { return fkey(__int_as_float(g[i].y)); };
-  auto pos_at = [&](int i) -> uint32_t { return (uint32_t)g[i].x; };
-
-  // radix select of the k-th largest key among the c candidates
+  auto each_key = [&](auto f) { each_kp([&](uint32_t key, uint32_t) { f(key); }); };
   unsigned int prefix = 0, need = (unsigned int)k, ties = 0;
   uint32_t pos_cut = 0xffffffffu;
+  uint32_t kmask = 0xffffffffu;   // the bits of a key compared with the threshold
   if (k > 0) {
-    prefix = radix_kth_desc(key_at, c, (unsigned int)k, hist, scratch, &need, &ties);
+    // without a k-th key to report, stop once the bucket of the k-th key is taken whole
+    prefix = radix_kth_desc(each_key, c, (unsigned int)k, hist, scratch, &need, &ties, 8, kth_bh ? nullptr : &kmask);
     if (ties > need) {
       // among keys equal to tau keep the `need` smallest positions: find the need-th smallest of them
       unsigned int pprefix = 0, pmask = 0, pneed = need;
       for (int shift = 24; shift >= 0; shift -= 8) {
         for (int i = threadIdx.x; i < 256; i += blockDim.x) hist[i] = 0;
         __syncthreads();
-        for (int i = threadIdx.x; i < c; i += blockDim.x) {
-          const uint32_t p = pos_at(i);
-          if (key_at(i) == prefix && (p & pmask) == pprefix) atomicAdd(&hist[(p >> shift) & 255u], 1u);
-        }
+        each_kp([&](uint32_t key, uint32_t p) {
+          if (key == prefix && (p & pmask) == pprefix) atomicAdd(&hist[(p >> shift) & 255u], 1u);
+        });
         __syncthreads();
         if (threadIdx.x < 32) pick_digit_asc(hist, pneed, &s_digit, &s_above);
         __syncthreads();
@@ -429,7 +444,7 @@ __global__ void __launch_bounds__(CAND_THREADS, 8) k_select_cand(
   const uint32_t tau = prefix;
   // bitmap (built in shared memory when it fits): clear, then set sinks and window (tier 1) and the selected
   // candidates, then write it out
-  uint32_t* wbm = nw <= SEL_SMEM_BITMAP_WORDS ? sbm : bm;
+  uint32_t* wbm = sbm ? sbm : bm;
   for (long long w = threadIdx.x; w < nw; w += blockDim.x) wbm[w] = 0u;
   __syncthreads();
   if (!append) {
@@ -437,20 +452,91 @@ __global__ void __launch_bounds__(CAND_THREADS, 8) k_select_cand(
     for (int u = hi + threadIdx.x; u < N; u += blockDim.x) atomicOr(&wbm[u >> 5], 1u << (u & 31));
   }
   if (k > 0) {
-    for (int i = threadIdx.x; i < c; i += blockDim.x) {
-      const uint32_t key = key_at(i), p = pos_at(i);
-      if (key > tau || (key == tau && p <= pos_cut)) atomicOr(&wbm[p >> 5], 1u << (p & 31));
-    }
+    each_kp([&](uint32_t key, uint32_t p) {
+      const uint32_t km = key & kmask;
+      if (km > tau || (km == tau && p <= pos_cut)) atomicOr(&wbm[p >> 5], 1u << (p & 31));
+    });
   }
   __syncthreads();
   if (wbm != bm)
     for (long long w = threadIdx.x; w < nw; w += blockDim.x) bm[w] = wbm[w];
   // ascending ids from the bitmap
-  const int base = bitmap_to_ids(wbm, nw, out, append ? count[bh] : 0, cap, scan_scratch);
+  const int base = bitmap_to_ids(wbm, nw, out, append ? *count_bh : 0, cap, scan_scratch);
   if (threadIdx.x == 0) {
-    count[bh] = base;
-    if (kth && !append) kth[bh] = k > 0 ? funkey(tau) : INFINITY;
+    *count_bh = base;
+    if (kth_bh && !append) *kth_bh = k > 0 ? funkey(tau) : INFINITY;
     if (base > cap) raise_status(status, VK_ERR_CAPACITY);
+  }
+}
+
+// Selection from a head's candidate list (every archive row with score >= theta, in arbitrary order). When the
+// list holds at least k and at most capc entries it contains the whole top-k (select_from_candidates). The keys
+// of lists of up to CAND_R x 256 entries are loaded once into registers (CAND_R per thread, all loads in flight
+// together) and every radix pass runs on them; longer lists are re-read from memory (L2-resident after the
+// scoring pass) on every pass. The block is latency-bound, so the launch bounds ask for 8 resident blocks per SM
+// even though the compiler then keeps part of the state in local memory: for 4096 heads of ~3.2k candidates
+// that measured 0.097 ms, against 0.106 ms at 4 blocks per SM without spills and 0.105 ms with the keys in
+// shared memory instead. When the list is too short or too long (theta landed too high or too low) or with
+// VK_FLAG_FORCE_FALLBACK, the head takes the exact ordered selection over scores recomputed from the RoPE
+// columns. With `append` (the top_j of the fired rows, whose list can never overflow) only candidates are
+// selected, no sinks or window, and the ids are appended after count[b,h].
+constexpr int CAND_R = 16;
+__global__ void __launch_bounds__(CAND_THREADS, 8) k_select_cand(
+    int H, int N, int lo, int hi, long long k_all, const long long* __restrict__ k_per_head,
+    const int* __restrict__ cand_cnt, const int2* __restrict__ cand, int capc, int force_fallback,
+    const __nv_bfloat16* __restrict__ rope, int64_t rld, int64_t rbs, const float* __restrict__ qt,
+    int32_t* __restrict__ idx, int32_t* __restrict__ count, int cap, int append, float* __restrict__ kth,
+    uint32_t* __restrict__ bitmap, long long nw, int* status) {
+  extern __shared__ __align__(16) unsigned char smem[];
+  uint32_t* sbm = nw <= SEL_SMEM_BITMAP_WORDS ? reinterpret_cast<uint32_t*>(smem) : nullptr;   // bitmap words
+  __shared__ float qts[D_ROPE];
+  const int64_t bh = blockIdx.x;
+  const int b = (int)(bh / H);
+  long long k = k_all;
+  if (k_per_head) k = min(k, k_per_head[bh]);
+  const int c = cand_cnt[bh];
+  if (append) k = min(k, (long long)c);
+  uint32_t* bm = bitmap + bh * nw;
+  int32_t* out = idx + bh * (int64_t)cap;
+  float* kth_bh = kth ? kth + bh : nullptr;
+
+  if (force_fallback || c < k || c > capc) {
+    if (append) {                       // cannot happen: the fired list has room for the whole archive
+      if (threadIdx.x == 0) raise_status(status, VK_ERR_CAPACITY);
+      return;
+    }
+    for (int i = threadIdx.x; i < D_ROPE; i += blockDim.x) qts[i] = qt[bh * D_ROPE + i];
+    __syncthreads();
+    RecomputedKeys keys{rope + (int64_t)b * rbs, rld, qts};
+    select_ordered(keys, N, lo, hi, k, out, count + bh, cap, 0, kth_bh, bm, nw, status);
+    return;
+  }
+
+  const int2* g = cand + bh * (int64_t)capc;
+  if (c <= CAND_R * CAND_THREADS) {
+    // keys in registers; a position is read back from the list only where a pass needs it (ties, marking)
+    uint32_t kr[CAND_R];
+#pragma unroll
+    for (int r = 0; r < CAND_R; ++r) {
+      const int i = threadIdx.x + r * CAND_THREADS;
+      kr[r] = fkey(i < c ? __int_as_float(g[i].y) : 0.f);
+    }
+    auto each_kp = [&](auto f) {
+#pragma unroll
+      for (int r = 0; r < CAND_R; ++r) {
+        const int i = threadIdx.x + r * CAND_THREADS;
+        if (i < c) f(kr[r], (uint32_t)g[i].x);
+      }
+    };
+    select_from_candidates(each_kp, c, k, N, lo, hi, append, sbm, bm, nw, out, count + bh, cap, kth_bh, status);
+  } else {
+    auto each_kp = [&](auto f) {
+      for (int i = threadIdx.x; i < c; i += CAND_THREADS) {
+        const int2 e = g[i];
+        f(fkey(__int_as_float(e.y)), (uint32_t)e.x);
+      }
+    };
+    select_from_candidates(each_kp, c, k, N, lo, hi, append, sbm, bm, nw, out, count + bh, cap, kth_bh, status);
   }
 }
 
