@@ -153,6 +153,9 @@ __global__ void __launch_bounds__((2 + 4 * (4 / NHG)) * 32, 1) k_score_tc(const 
   const int n = (int)(t1 - t0);
   const int tps = args.tiles_per_seq;
   const int b_first = (int)(t0 / tps);
+  const int kt_first = (int)(t0 - (int64_t)b_first * tps);
+  // (sequence, tile within it) of the range's tiles, stepped without divisions: a 64-bit division per tile on
+  // the producer's or the MMA issuer's thread is slower than the tile's whole TMA + MMA work
   constexpr uint32_t DCOLS = NHG * TC_M;                 // columns per accumulator
 
   if (threadIdx.x == 0) {
@@ -170,10 +173,9 @@ __global__ void __launch_bounds__((2 + 4 * (4 / NHG)) * 32, 1) k_score_tc(const 
   if (warp == 0) {
     // ------------------------------------------------------------------ TMA producer
     if (lane == 0 && n > 0) {
-      int prev_b = -1;
-      for (int i = 0; i < n; ++i) {
-        const int64_t t = t0 + i;
-        const int b = (int)(t / tps), row0 = (int)(t % tps) * TC_M;
+      int prev_b = -1, b = b_first, kt = kt_first;
+      for (int i = 0; i < n; ++i, kt = kt + 1 == tps ? (++b, 0) : kt + 1) {
+        const int row0 = kt * TC_M;
         if (b != prev_b) {
           const int qi = (b - b_first) & 1, quse = (b - b_first) >> 1;
           if (quse > 0 && !mbar_wait(&q_empty[qi], (quse - 1) & 1, &abort_flag)) { abort_flag = 1; break; }
@@ -192,10 +194,8 @@ __global__ void __launch_bounds__((2 + 4 * (4 / NHG)) * 32, 1) k_score_tc(const 
     // ------------------------------------------------------------------ MMA issuer
     if (lane == 0 && n > 0) {
       constexpr uint32_t idesc = mma_idesc_bf16(MH, TC_M);
-      int prev_b = -1;
-      for (int i = 0; i < n; ++i) {
-        const int64_t t = t0 + i;
-        const int b = (int)(t / tps);
+      int prev_b = -1, b = b_first, kt = kt_first;
+      for (int i = 0; i < n; ++i, kt = kt + 1 == tps ? (++b, 0) : kt + 1) {
         const int qi = (b - b_first) & 1;
         if (b != prev_b) {
           if (!mbar_wait(&q_full[qi], ((b - b_first) >> 1) & 1, &abort_flag)) { abort_flag = 1; break; }
@@ -216,7 +216,7 @@ __global__ void __launch_bounds__((2 + 4 * (4 / NHG)) * 32, 1) k_score_tc(const 
                      bd + (uint64_t)((32 * k) >> 4), idesc, k > 0 ? 1u : 0u);
         mma_commit(&a_empty[s]);
         mma_commit(&d_full[ds]);
-        const bool last_of_seq = (i + 1 == n) || ((t + 1) / tps != b);
+        const bool last_of_seq = (i + 1 == n) || kt + 1 == tps;
         if (last_of_seq) mma_commit(&q_empty[qi]);
       }
     }
@@ -229,9 +229,10 @@ __global__ void __launch_bounds__((2 + 4 * (4 / NHG)) * 32, 1) k_score_tc(const 
     float* my_stg = stg + (ew * 32 + lane) * 32;          // this thread's staging row (128 B, 16-byte swizzled)
     int prev_b = -1;
     float th[NHG], p1[NHG], p2[NHG];                      // per head: theta, or (s*, |(O Qr)[r:]|, z |Qc|)
-    for (int i = g; i < n; i += G) {
-      const int64_t t = t0 + i;
-      const int b = (int)(t / tps), row0 = (int)(t % tps) * TC_M;
+    int b = b_first, kt = kt_first + g;
+    for (int i = g; i < n; i += G, kt += G) {
+      while (kt >= tps) { kt -= tps; ++b; }
+      const int row0 = kt * TC_M;
       if (b != prev_b) {
 #pragma unroll
         for (int hg = 0; hg < NHG; ++hg) {
