@@ -48,7 +48,6 @@ constexpr int AT_SMX = 4;                              // softmax warps (one per
 constexpr int AT_THREADS = (4 + AT_SMX) * 32;   // producer, S issuer, softmax x4, O^T issuer, S issuer
 constexpr uint32_t AT_KBLK = 64 * 128;                 // one 64-column block of 64 rows (or 64 heads): 8 KB
 constexpr uint32_t AT_TILE = 9 * AT_KBLK;              // 73,728: one tile slot, and the queries
-constexpr uint32_t AT_P = 64 * 128;                    // P^T: 64 heads x 64 rows, bf16
 constexpr int AT_NG = 5;                               // load groups per tile: latent pairs 0..3, RoPE block 4
 constexpr float AT_TAU = 8.f;                          // log2 slack before a running max moves
 constexpr uint32_t AT_TMEM_COLS = 512;
@@ -57,18 +56,19 @@ constexpr uint32_t AT_SB_COL = 384;                    // S (latent 256..511) bu
 constexpr uint32_t AT_O_COL = 128;                     // O^T block j: columns 128 + 64 j .. + 63
 
 // Shared memory, from a 1024-byte aligned base. Barriers: xfull/xrel [2 slots][5 groups], sfull/sfree [2],
-// wfull/wfree [2], pfull, pfree, qfull, qfree, gbar [2], ebar, odone, ofree, sdone [2].
+// wfull/wfree [2], pfull, pfree [2], qfull, qfree, gbar [2], ebar, odone, ofree, sdone [2]. P^T has no region of its
+// own: a tile's P^T (64 heads x 64 rows, bf16, 8 KB) is written over its slot's RoPE block once S has read it.
 struct AtSmem {
   static constexpr uint32_t q = 0;
   static constexpr uint32_t x = q + AT_TILE;
   static constexpr uint32_t p = x + 2 * AT_TILE;
-  static constexpr uint32_t words = p + AT_P;          // [2][64 heads][2] u32
+  static constexpr uint32_t words = p;                 // [2][64 heads][2] u32
   static constexpr uint32_t uni = words + 2 * 64 * 2 * 4;
   static constexpr uint32_t fac = uni + 2 * 4;         // [2][64] f32
   static constexpr uint32_t anyw = fac + 2 * 64 * 4;   // [2][4] u32
   static constexpr uint32_t misc = anyw + 2 * 4 * 4;   // TMEM base, abort flag
   static constexpr uint32_t bars = (misc + 8 + 7) & ~7u;
-  static constexpr uint32_t nbars = 2 * AT_NG * 2 + 2 * 4 + 4 + 3 + 4;
+  static constexpr uint32_t nbars = 2 * AT_NG * 2 + 2 * 4 + 5 + 3 + 4;
   static constexpr uint32_t total = bars + nbars * 8;
 };
 static_assert(AtSmem::total + 1024 <= 232448, "attention shared memory exceeds the 227 KB opt-in limit");
@@ -167,7 +167,6 @@ __global__ void __launch_bounds__(AT_THREADS, 1) k_attn_tc(const __grid_constant
   unsigned char* smem = reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   unsigned char* sq = smem + AtSmem::q;
   unsigned char* sx = smem + AtSmem::x;
-  unsigned char* sp = smem + AtSmem::p;
   uint32_t* words = reinterpret_cast<uint32_t*>(smem + AtSmem::words);
   uint32_t* unis = reinterpret_cast<uint32_t*>(smem + AtSmem::uni);
   float* fac = reinterpret_cast<float*>(smem + AtSmem::fac);
@@ -182,8 +181,8 @@ __global__ void __launch_bounds__(AT_THREADS, 1) k_attn_tc(const __grid_constant
   uint64_t* wfull = sfree + 2;                // [2]
   uint64_t* wfree = wfull + 2;                // [2]
   uint64_t* pfull = wfree + 2;
-  uint64_t* pfree = pfull + 1;
-  uint64_t* qfull = pfree + 1;                // a segment's queries landed (one phase per segment)
+  uint64_t* pfree = pfull + 1;                // [2] a tile's O^T product is complete, by tile parity
+  uint64_t* qfull = pfree + 2;                // a segment's queries landed (one phase per segment)
   uint64_t* qfree = qfull + 1;                // both S issuers are done with the previous segment's queries
   uint64_t* gbar = qfree + 1;                 // [2] softmax-group syncs, by tile parity
   uint64_t* ebar = gbar + 2;                  // softmax-group syncs of a segment's epilogue (two per segment)
@@ -212,7 +211,8 @@ __global__ void __launch_bounds__(AT_THREADS, 1) k_attn_tc(const __grid_constant
       mbar_init(&sdone[i], 1);
     }
     mbar_init(pfull, AT_SMX);
-    mbar_init(pfree, 1);
+    mbar_init(&pfree[0], 1);
+    mbar_init(&pfree[1], 1);
     mbar_init(qfull, 1);
     mbar_init(qfree, 2);
     mbar_init(ebar, AT_SMX);
@@ -284,7 +284,7 @@ __global__ void __launch_bounds__(AT_THREADS, 1) k_attn_tc(const __grid_constant
         unsigned char* xs = sx + s * AT_TILE;
         if (lane == 0) {
           for (int g = 0; g < AT_NG; ++g) {
-            const int grp = g == 0 ? 4 : g - 1;        // RoPE block first (its slot part is released first)
+            const int grp = g;                         // latent pairs 0..3 in release order, then the RoPE block
             uint64_t* fb = &xfull[s * AT_NG + grp];
             if (use > 0 && !mbar_wait(&xrel[s * AT_NG + grp], (use - 1) & 1, abort_flag)) { lok = false; break; }
             if (grp == 4) {
@@ -326,7 +326,10 @@ __global__ void __launch_bounds__(AT_THREADS, 1) k_attn_tc(const __grid_constant
   } else if (warp == 1 || warp == 3 + AT_SMX) {
     // ------------------------------------------------------------------ S issuers
     // Two threads issue the two halves of the K = 576 contraction into their own accumulators (the softmax adds
-    // them): warp 1 the RoPE block and latent dims 0..255 (20 instructions), warp 7 latent dims 256..511 (16).
+    // them): warp 1 latent dims 0..255 (16 instructions), warp 7 latent dims 256..511 and the RoPE block (20). The
+    // groups land in the order the previous tile's O^T product releases them: latent pairs 0..3, then the RoPE
+    // block, which holds that tile's P^T until its O^T is done. (A 24/12 split, the short part after the last
+    // group to land, measured slower.)
     const int half = warp == 1 ? 0 : 1;
     if (lane == 0 && ntile > 0) {
       // S: M = 64 heads, N = 64 rows, A = Q and B = X, both K-major
@@ -352,26 +355,25 @@ __global__ void __launch_bounds__(AT_THREADS, 1) k_attn_tc(const __grid_constant
         // this half's load groups first, then its instructions as one branch-free burst: control flow between
         // tcgen05.mma issues costs the issuing thread far more than the instructions themselves
         if (half == 0) {
-          ok = mbar_wait(&xfull[s * AT_NG + 4], use & 1, abort_flag) && mbar_wait(&xfull[s * AT_NG + 0], use & 1, abort_flag) &&
-               mbar_wait(&xfull[s * AT_NG + 1], use & 1, abort_flag);
+          ok = mbar_wait(&xfull[s * AT_NG + 0], use & 1, abort_flag) && mbar_wait(&xfull[s * AT_NG + 1], use & 1, abort_flag);
           if (!ok) break;
           // operands land by TMA and are observed through the mbarrier: no tensor-memory fence is needed
           const uint32_t d = tmem + AT_S_COL + 64 * s;
 #pragma unroll
-          for (int j = 0; j < 20; ++j) {
-            const int kb = j < 4 ? 8 : (j - 4) >> 2;
-            const uint64_t off = (uint64_t)((kb * AT_KBLK + 32 * (j & 3)) >> 4);
+          for (int j = 0; j < 16; ++j) {
+            const uint64_t off = (uint64_t)(((j >> 2) * AT_KBLK + 32 * (j & 3)) >> 4);
             mma_bf16_(d, qd + off, xd + off, idesc_s, j > 0 ? 1u : 0u);
           }
           mma_commit_(&sfull[s]);
-          mma_commit_(&xrel[s * AT_NG + 4]);           // the RoPE block is read by S only
         } else {
-          ok = mbar_wait(&xfull[s * AT_NG + 2], use & 1, abort_flag) && mbar_wait(&xfull[s * AT_NG + 3], use & 1, abort_flag);
+          ok = mbar_wait(&xfull[s * AT_NG + 2], use & 1, abort_flag) && mbar_wait(&xfull[s * AT_NG + 3], use & 1, abort_flag) &&
+               mbar_wait(&xfull[s * AT_NG + 4], use & 1, abort_flag);
           if (!ok) break;
           const uint32_t d = tmem + AT_SB_COL + 64 * s;
 #pragma unroll
-          for (int j = 0; j < 16; ++j) {
-            const uint64_t off = (uint64_t)(((4 + (j >> 2)) * AT_KBLK + 32 * (j & 3)) >> 4);
+          for (int j = 0; j < 20; ++j) {
+            const int kb = j < 16 ? 4 + (j >> 2) : 8;
+            const uint64_t off = (uint64_t)((kb * AT_KBLK + 32 * (j & 3)) >> 4);
             mma_bf16_(d, qd + off, xd + off, idesc_s, j > 0 ? 1u : 0u);
           }
           mma_commit_(&sfull[s]);
@@ -392,7 +394,6 @@ __global__ void __launch_bounds__(AT_THREADS, 1) k_attn_tc(const __grid_constant
       // O^T: M = 128 dims, N = 64 heads, A = X_lat^T MN-major (bit 15), B = P^T K-major
       const uint32_t idesc_o =
           (1u << 4) | (1u << 7) | (1u << 10) | (1u << 15) | ((uint32_t)(64 >> 3) << 17) | ((uint32_t)(128 >> 4) << 24);
-      const uint64_t pd = sdesc_(smem_addr(sp), 16);
       bool ok = true;
       int u = 0, useg = 0, nseg = 0, ncommit = 0;
       for (int i = 0; i < ntile; ++i, tp.next(T, geo.n_hg)) {
@@ -414,6 +415,7 @@ __global__ void __launch_bounds__(AT_THREADS, 1) k_attn_tc(const __grid_constant
         tmem_fence_after();                            // P^T and any O^T rescale come from the softmax warps
         const int s = u & 1;
         const uint64_t xd = sdesc_(smem_addr(sx + s * AT_TILE), AT_KBLK);
+        const uint64_t pd = sdesc_(smem_addr(sx + s * AT_TILE + 8 * AT_KBLK), 16);   // this tile's P^T
 #pragma unroll
         for (int j = 0; j < 4; ++j) {
 #pragma unroll
@@ -422,7 +424,8 @@ __global__ void __launch_bounds__(AT_THREADS, 1) k_attn_tc(const __grid_constant
                       pd + (uint64_t)(ks * 2), idesc_o, (useg > 0 || ks > 0) ? 1u : 0u);
           mma_commit_(&xrel[s * AT_NG + j]);           // latent blocks 2j, 2j+1 of this slot are free again
         }
-        mma_commit_(pfree);                            // P^T free, O^T up to date
+        mma_commit_(&xrel[s * AT_NG + 4]);             // P^T read: the RoPE block may be reloaded
+        mma_commit_(&pfree[u & 1]);                    // O^T up to date through this tile
         ++u;
         ++useg;
       }
@@ -585,12 +588,13 @@ __global__ void __launch_bounds__(AT_THREADS, 1) k_attn_tc(const __grid_constant
       const uint32_t need = __ballot_sync(0xffffffffu, own && f != 1.f);
       if (own) fac[par * 64 + hl] = f;
       if (lane == 0) anyw[par * 4 + q] = need;
-      // the previous tile's O^T product must be complete: it reads P^T, and O^T may be rescaled now
-      if (u > 0 && !warp_wait_(pfree, (u - 1) & 1, abort_flag, lane)) { ok = false; break; }
       __syncwarp();
       if (lane == 0) mbar_arrive(&gbar[par]);
       if (!warp_wait_(&gbar[par], use & 1, abort_flag, lane)) { ok = false; break; }
       if (anyw[par * 4] | anyw[par * 4 + 1] | anyw[par * 4 + 2] | anyw[par * 4 + 3]) {
+        // a rescale of O^T needs the previous tile's O^T product complete (u > 0: a head's first selected row
+        // never rescales, so the first tile of a segment never gets here)
+        if (!warp_wait_(&pfree[(u - 1) & 1], ((u - 1) >> 1) & 1, abort_flag, lane)) { ok = false; break; }
         tmem_fence_after();
         for (int h = 0; h < 64; ++h) {
           const float fh = fac[par * 64 + h];
@@ -607,8 +611,9 @@ __global__ void __launch_bounds__(AT_THREADS, 1) k_attn_tc(const __grid_constant
         tmem_wait_st();
       }
       {
-        // P^T row hl, rows 32 hh .. + 31 of the tile: four 16-byte chunks, 128-byte swizzle
-        unsigned char* row = sp + hl * 128;
+        // P^T row hl, rows 32 hh .. + 31 of the tile: four 16-byte chunks, 128-byte swizzle, over the slot's RoPE
+        // block (S has read it: sfull)
+        unsigned char* row = sx + s * AT_TILE + 8 * AT_KBLK + hl * 128;
 #pragma unroll
         for (int i = 0; i < 4; ++i)
           *reinterpret_cast<uint4*>(row + (((4 * hh + i) ^ (hl & 7)) * 16)) =
