@@ -56,7 +56,7 @@ constexpr uint32_t AT_SB_COL = 384;                    // S (latent 256..511) bu
 constexpr uint32_t AT_O_COL = 128;                     // O^T block j: columns 128 + 64 j .. + 63
 
 // Shared memory, from a 1024-byte aligned base. Barriers: xfull/xrel [2 slots][5 groups], sfull/sfree [2],
-// wfull/wfree [2], pfull, pfree [2], qfull, qfree, gbar [2], ebar, odone, ofree, sdone [2]. P^T has no region of its
+// wfull/wfree [2], pfull [2], pfree [2], qfull, qfree, gbar [2], ebar, odone, ofree, sdone [2]. P^T has no region of its
 // own: a tile's P^T (64 heads x 64 rows, bf16, 8 KB) is written over its slot's RoPE block once S has read it.
 struct AtSmem {
   static constexpr uint32_t q = 0;
@@ -68,7 +68,7 @@ struct AtSmem {
   static constexpr uint32_t anyw = fac + 2 * 64 * 4;   // [2][4] u32
   static constexpr uint32_t misc = anyw + 2 * 4 * 4;   // TMEM base, abort flag
   static constexpr uint32_t bars = (misc + 8 + 7) & ~7u;
-  static constexpr uint32_t nbars = 2 * AT_NG * 2 + 2 * 4 + 5 + 3 + 4;
+  static constexpr uint32_t nbars = 2 * AT_NG * 2 + 2 * 4 + 6 + 3 + 4;
   static constexpr uint32_t total = bars + nbars * 8;
 };
 static_assert(AtSmem::total + 1024 <= 232448, "attention shared memory exceeds the 227 KB opt-in limit");
@@ -180,8 +180,10 @@ __global__ void __launch_bounds__(AT_THREADS, 1) k_attn_tc(const __grid_constant
   uint64_t* sfree = sfull + 2;                // [2]
   uint64_t* wfull = sfree + 2;                // [2]
   uint64_t* wfree = wfull + 2;                // [2]
+  // [2] a tile's P^T is written, by slot. One barrier per slot: the softmax warps do not wait for the O^T product
+  // between tiles, so a single barrier could complete twice before the O^T issuer looked at it.
   uint64_t* pfull = wfree + 2;
-  uint64_t* pfree = pfull + 1;                // [2] a tile's O^T product is complete, by tile parity
+  uint64_t* pfree = pfull + 2;                // [2] a tile's O^T product is complete, by tile parity
   uint64_t* qfull = pfree + 2;                // a segment's queries landed (one phase per segment)
   uint64_t* qfree = qfull + 1;                // both S issuers are done with the previous segment's queries
   uint64_t* gbar = qfree + 1;                 // [2] softmax-group syncs, by tile parity
@@ -210,9 +212,10 @@ __global__ void __launch_bounds__(AT_THREADS, 1) k_attn_tc(const __grid_constant
       mbar_init(&gbar[i], AT_SMX);
       mbar_init(&sdone[i], 1);
     }
-    mbar_init(pfull, AT_SMX);
-    mbar_init(&pfree[0], 1);
-    mbar_init(&pfree[1], 1);
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(&pfull[i], AT_SMX);
+      mbar_init(&pfree[i], 1);
+    }
     mbar_init(qfull, 1);
     mbar_init(qfree, 2);
     mbar_init(ebar, AT_SMX);
@@ -411,9 +414,9 @@ __global__ void __launch_bounds__(AT_THREADS, 1) k_attn_tc(const __grid_constant
           useg = 0;
         }
         if (!uni) continue;
-        if (!mbar_wait(pfull, u & 1, abort_flag)) { ok = false; break; }
-        tmem_fence_after();                            // P^T and any O^T rescale come from the softmax warps
         const int s = u & 1;
+        if (!mbar_wait(&pfull[s], (u >> 1) & 1, abort_flag)) { ok = false; break; }
+        tmem_fence_after();                            // P^T and any O^T rescale come from the softmax warps
         const uint64_t xd = sdesc_(smem_addr(sx + s * AT_TILE), AT_KBLK);
         const uint64_t pd = sdesc_(smem_addr(sx + s * AT_TILE + 8 * AT_KBLK), 16);   // this tile's P^T
 #pragma unroll
@@ -622,7 +625,7 @@ __global__ void __launch_bounds__(AT_THREADS, 1) k_attn_tc(const __grid_constant
       fence_async_smem_();
       tmem_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive(pfull);
+      if (lane == 0) mbar_arrive(&pfull[s]);
       ++u;
       ++useg;
     }
