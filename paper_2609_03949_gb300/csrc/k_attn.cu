@@ -459,10 +459,95 @@ __global__ void k_combine(int BH, int H, const AttnGeom g, int nslot, const floa
   }
 }
 
+// The same merge for many slots per (b, h) (small batches: one sequence's tiles spread over up to 152 CTAs): one
+// block of CMB_WARPS warps per (b, h). The block finds the max over the slots, each warp sums every CMB_WARPS-th
+// slot (lanes over the 512 dims), and the warps' sums are added through shared memory -- the slots' loads run
+// CMB_WARPS wide instead of one slot after another.
+constexpr int CMB_WARPS = 8;
+__global__ void __launch_bounds__(CMB_WARPS * 32) k_combine_wide(int H, const AttnGeom g, int nslot,
+                                                                 const float* __restrict__ part_o,
+                                                                 const float* __restrict__ part_ml,
+                                                                 float* __restrict__ out, float* __restrict__ lse,
+                                                                 float* __restrict__ smax) {
+  __shared__ float red_m[CMB_WARPS], red_m1[CMB_WARPS], red_l[CMB_WARPS];
+  __shared__ float4 red_acc[CMB_WARPS][32][4];
+  const int bh = blockIdx.x, b = bh / H, h = bh % H;
+  const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int nv = attn_nvalid(g, (long long)b * g.n_hg + h / HG);
+  const int nlist = nslot > g.nslot ? 2 * nv : nv;
+  auto slot_of = [&](int s) { return s < nv ? s : g.nslot + s - nv; };
+  float m = -INFINITY, m1 = -INFINITY;
+  for (int s = threadIdx.x; s < nlist; s += blockDim.x) {
+    const float ms = part_ml[(((int64_t)b * nslot + slot_of(s)) * H + h) * 2];
+    m = fmaxf(m, ms);
+    if (s < nv) m1 = fmaxf(m1, ms);
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, o));
+    m1 = fmaxf(m1, __shfl_xor_sync(0xffffffffu, m1, o));
+  }
+  if (lane == 0) { red_m[w] = m; red_m1[w] = m1; }
+  __syncthreads();
+  m = red_m[0];
+  m1 = red_m1[0];
+#pragma unroll
+  for (int i = 1; i < CMB_WARPS; ++i) { m = fmaxf(m, red_m[i]); m1 = fmaxf(m1, red_m1[i]); }
+  float acc[16];
+#pragma unroll
+  for (int t = 0; t < 16; ++t) acc[t] = 0.f;
+  float l = 0.f;
+  if (m > -INFINITY) {
+    for (int s = w; s < nlist; s += CMB_WARPS) {
+      const int64_t base = ((int64_t)b * nslot + slot_of(s)) * H + h;
+      const float ms = part_ml[base * 2], ls = part_ml[base * 2 + 1];
+      if (!(ls > 0.f)) continue;
+      const float wt = __expf(ms - m);
+      l = fmaf(wt, ls, l);
+      const float4* src = reinterpret_cast<const float4*>(part_o + base * D_LAT + lane * 16);
+#pragma unroll
+      for (int t = 0; t < 4; ++t) {
+        const float4 x = src[t];
+        acc[4 * t] = fmaf(wt, x.x, acc[4 * t]);
+        acc[4 * t + 1] = fmaf(wt, x.y, acc[4 * t + 1]);
+        acc[4 * t + 2] = fmaf(wt, x.z, acc[4 * t + 2]);
+        acc[4 * t + 3] = fmaf(wt, x.w, acc[4 * t + 3]);
+      }
+    }
+  }
+#pragma unroll
+  for (int t = 0; t < 4; ++t) red_acc[w][lane][t] = make_float4(acc[4 * t], acc[4 * t + 1], acc[4 * t + 2], acc[4 * t + 3]);
+  if (lane == 0) red_l[w] = l;
+  __syncthreads();
+  if (w != 0) return;
+  float lt = 0.f;
+#pragma unroll
+  for (int i = 0; i < CMB_WARPS; ++i) lt += red_l[i];
+  const float inv = lt > 0.f ? 1.f / lt : 0.f;
+  float4* dst = reinterpret_cast<float4*>(out + (int64_t)bh * D_LAT + lane * 16);
+#pragma unroll
+  for (int t = 0; t < 4; ++t) {
+    float4 a = red_acc[0][lane][t];
+#pragma unroll
+    for (int i = 1; i < CMB_WARPS; ++i) {
+      const float4 x = red_acc[i][lane][t];
+      a.x += x.x; a.y += x.y; a.z += x.z; a.w += x.w;
+    }
+    dst[t] = make_float4(a.x * inv, a.y * inv, a.z * inv, a.w * inv);
+  }
+  if (lane == 0) {
+    if (lse) lse[bh] = lt > 0.f ? m + logf(lt) : -INFINITY;
+    if (smax) smax[bh] = m1;
+  }
+}
+
 cudaError_t launch_combine(int B, int H, const AttnGeom& g, int nslot, const float* part_o, const float* part_ml,
                            float* out, float* lse, float* smax, cudaStream_t st) {
   const int BH = B * H, threads = 256;
-  k_combine<<<(BH * 32 + threads - 1) / threads, threads, 0, st>>>(BH, H, g, nslot, part_o, part_ml, out, lse, smax);
+  if (nslot > CMB_WARPS)
+    k_combine_wide<<<BH, CMB_WARPS * 32, 0, st>>>(H, g, nslot, part_o, part_ml, out, lse, smax);
+  else
+    k_combine<<<(BH * 32 + threads - 1) / threads, threads, 0, st>>>(BH, H, g, nslot, part_o, part_ml, out, lse, smax);
   count_launches(1);
   return cudaGetLastError();
 }
