@@ -125,6 +125,7 @@ EDGES = [
     dict(B=2, H=64, N=2048, rho=1.0, window=0),            # dense
     dict(B=2, H=64, N=3000, rho=1 / 8, window=64, dtype="f32"),
     dict(B=1, H=256, N=2048, rho=1 / 8, window=64),
+    dict(B=300, H=16, N=100, rho=1 / 4, window=8),         # attention CTAs that span several whole segments
 ]
 
 
@@ -138,6 +139,14 @@ def test_edge_cases(case):
     res = run_case(wl, **c)
     if c["rho"] == 1.0 and c.get("window", 0) == 0:
         assert np.all(res["gpu"]["count"] == N)
+
+
+def test_two_tier_many_partials():
+    # one sequence spread over 64 attention CTAs per tier: the combine merges 64 tier-1 and 64 fired partials per
+    # head (the block-per-head merge); most fired tiles are empty, so many CTAs close segments with no tile
+    wl = datagen.make_workload(1, 64, 16384, seed=41, n_planted=16, planted_hi=16384 - 256, device="cuda")
+    res = run_case(wl, rho=1 / 32, window=256, trigger=1, z_eff=0.6)
+    assert res["fired"] > 0
 
 
 def test_two_tier_sinks_and_capacity():
