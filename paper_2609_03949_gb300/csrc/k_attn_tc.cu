@@ -23,9 +23,11 @@
 //                      and 32..63 of the tile. They read the head's logits, mask them with its selection words,
 //                      and write P^T[h][row] = 2^(s lambda log2(e) - m_h)
 //                      (0 where the head did not select the row) in bf16 into shared memory (K-major, 128-byte
-//                      swizzle). m_h is a running max that only moves when a tile's max exceeds it by more than 8
-//                      (log2 units; the head's O^T column and sum are then rescaled in tensor memory), so rescaling
-//                      is rare and P stays <= 256. The exact max is tracked beside it, and at the end the head's sum
+//                      swizzle). m_h is a running max that only moves when a tile's max exceeds it by more than 32
+//                      (log2 units), so P stays <= 2^32 and a rescale is rare: the O^T issuer sees it in the tile's
+//                      published flags and has the four softmax warps scale the head's O^T column in tensor memory
+//                      (each its quarter of the dims) before the tile's product; there is no per-tile sync of the
+//                      softmax warps otherwise. The exact max is tracked beside it, and at the end the head's sum
 //                      and output are re-based on it, so the partial carries the true max logit. At a segment's end
 //                      they write its partial and hand the O^T accumulator back to the O^T issuer.
 // The partials (max, sum, out) of a segment, one per CTA it spans, are merged by the LSE combine (Lemma 1): with
@@ -49,14 +51,14 @@ constexpr int AT_THREADS = (4 + AT_SMX) * 32;   // producer, S issuer, softmax x
 constexpr uint32_t AT_KBLK = 64 * 128;                 // one 64-column block of 64 rows (or 64 heads): 8 KB
 constexpr uint32_t AT_TILE = 9 * AT_KBLK;              // 73,728: one tile slot, and the queries
 constexpr int AT_NG = 5;                               // load groups per tile: latent pairs 0..3, RoPE block 4
-constexpr float AT_TAU = 8.f;                          // log2 slack before a running max moves
+constexpr float AT_TAU = 32.f;                         // log2 slack before a running max moves (P <= 2^32)
 constexpr uint32_t AT_TMEM_COLS = 512;
 constexpr uint32_t AT_S_COL = 0;                       // S (RoPE + latent 0..255) buffers: columns 0..63, 64..127
 constexpr uint32_t AT_SB_COL = 384;                    // S (latent 256..511) buffers: columns 384..447, 448..511
 constexpr uint32_t AT_O_COL = 128;                     // O^T block j: columns 128 + 64 j .. + 63
 
 // Shared memory, from a 1024-byte aligned base. Barriers: xfull/xrel [2 slots][5 groups], sfull/sfree [2],
-// wfull/wfree [2], pfull [2], pfree [2], qfull, qfree, gbar [2], ebar, odone, ofree, sdone [2]. P^T has no region of its
+// wfull/wfree [2], pfull [2], pfree [2], qfull, qfree, rdone, odec [2], ebar, odone, ofree, sdone [2]. P^T has no region of its
 // own: a tile's P^T (64 heads x 64 rows, bf16, 8 KB) is written over its slot's RoPE block once S has read it.
 struct AtSmem {
   static constexpr uint32_t q = 0;
@@ -66,9 +68,9 @@ struct AtSmem {
   static constexpr uint32_t uni = words + 2 * 64 * 2 * 4;
   static constexpr uint32_t fac = uni + 2 * 4;         // [2][64] f32
   static constexpr uint32_t anyw = fac + 2 * 64 * 4;   // [2][4] u32
-  static constexpr uint32_t misc = anyw + 2 * 4 * 4;   // TMEM base, abort flag
-  static constexpr uint32_t bars = (misc + 8 + 7) & ~7u;
-  static constexpr uint32_t nbars = 2 * AT_NG * 2 + 2 * 4 + 6 + 3 + 4;
+  static constexpr uint32_t misc = anyw + 2 * 4 * 4;   // TMEM base, abort flag, rescale request (tile, count)
+  static constexpr uint32_t bars = (misc + 16 + 7) & ~7u;
+  static constexpr uint32_t nbars = 2 * AT_NG * 2 + 2 * 4 + 6 + 4 + 4;
   static constexpr uint32_t total = bars + nbars * 8;
 };
 static_assert(AtSmem::total + 1024 <= 232448, "attention shared memory exceeds the 227 KB opt-in limit");
@@ -140,6 +142,42 @@ __device__ __forceinline__ bool warp_wait_(uint64_t* bar, uint32_t parity, volat
   return __shfl_sync(0xffffffffu, w, 0);
 }
 
+// A rescale request of the O^T issuer (tile r: some head's running max moved there), served by one softmax warp
+// (warp-collective): once O^T(r - 1) is complete, scale the warp's quarter of the dims (TMEM lanes lrow..) of every
+// such head's O^T column by its factor in fac[r & 1], then report on rdone. Out of line: it is rare.
+static __device__ __noinline__ bool attn_handle_request(volatile int* rq_tile, uint64_t* pfree, uint64_t* rdone,
+                                                        const float* fac, uint32_t lrow, volatile int* abort_flag,
+                                                        int lane) {
+  int r = 0;
+  if (lane == 0) {
+    __threadfence_block();                             // the count was read first; the tile was written first
+    r = *rq_tile;
+  }
+  r = __shfl_sync(0xffffffffu, r, 0);
+  __syncwarp();
+  __threadfence_block();                               // the factors were published before the request
+  if (!warp_wait_(&pfree[(r - 1) & 1], ((r - 1) >> 1) & 1, abort_flag, lane)) return false;
+  tmem_fence_after();
+  const float* fr = fac + (r & 1) * 64;
+  for (int h = 0; h < 64; ++h) {
+    const float fh = fr[h];
+    if (fh != 1.f) {
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        const uint32_t a = lrow + AT_O_COL + 64 * j + h;
+        const float v = tmem_ld1_(a);
+        tmem_wait_ld();
+        tmem_st1_(a, v * fh);
+      }
+    }
+  }
+  tmem_wait_st();
+  tmem_fence_before();
+  __syncwarp();
+  if (lane == 0) mbar_arrive(rdone);
+  return true;
+}
+
 // Position of a flattened tile: its row tile kt within the segment and the segment's (sequence b, head group hg).
 // Stepped without divisions (the per-tile bookkeeping sits on the issuing threads' critical path).
 struct TilePos {
@@ -173,6 +211,8 @@ __global__ void __launch_bounds__(AT_THREADS, 1) k_attn_tc(const __grid_constant
   uint32_t* anyw = reinterpret_cast<uint32_t*>(smem + AtSmem::anyw);
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + AtSmem::misc);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + AtSmem::misc + 4);
+  volatile int* rq_tile = reinterpret_cast<volatile int*>(smem + AtSmem::misc + 8);    // tile of the last request
+  volatile int* rq_count = reinterpret_cast<volatile int*>(smem + AtSmem::misc + 12);  // requests made so far
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + AtSmem::bars);
   uint64_t* xfull = bars;                     // [2][5]
   uint64_t* xrel = bars + 2 * AT_NG;          // [2][5]
@@ -186,8 +226,9 @@ __global__ void __launch_bounds__(AT_THREADS, 1) k_attn_tc(const __grid_constant
   uint64_t* pfree = pfull + 2;                // [2] a tile's O^T product is complete, by tile parity
   uint64_t* qfull = pfree + 2;                // a segment's queries landed (one phase per segment)
   uint64_t* qfree = qfull + 1;                // both S issuers are done with the previous segment's queries
-  uint64_t* gbar = qfree + 1;                 // [2] softmax-group syncs, by tile parity
-  uint64_t* ebar = gbar + 2;                  // softmax-group syncs of a segment's epilogue (two per segment)
+  uint64_t* rdone = qfree + 1;                // the softmax warps have applied a requested O^T rescale
+  uint64_t* odec = rdone + 1;                 // [2] the O^T issuer has seen a tile's P^T (and asked for any rescale)
+  uint64_t* ebar = odec + 2;                  // softmax-group syncs of a segment's epilogue (two per segment)
   uint64_t* odone = ebar + 1;                 // the segment's O^T products are complete (O^T issuer's commit)
   uint64_t* ofree = odone + 1;                // the softmax warps have read the segment's O^T out of tensor memory
   uint64_t* sdone = ofree + 1;                // [2] each S issuer's final commit
@@ -203,13 +244,14 @@ __global__ void __launch_bounds__(AT_THREADS, 1) k_attn_tc(const __grid_constant
 
   if (threadIdx.x == 0) {
     *abort_flag = 0;
+    *rq_tile = -1;
+    *rq_count = 0;
     for (int i = 0; i < 2 * AT_NG; ++i) { mbar_init(&xfull[i], 1); mbar_init(&xrel[i], 1); }
     for (int i = 0; i < 2; ++i) {
       mbar_init(&sfull[i], 2);                    // one commit from each S issuer
       mbar_init(&sfree[i], AT_SMX);
       mbar_init(&wfull[i], 1);
       mbar_init(&wfree[i], AT_SMX + 3);
-      mbar_init(&gbar[i], AT_SMX);
       mbar_init(&sdone[i], 1);
     }
     for (int i = 0; i < 2; ++i) {
@@ -218,6 +260,9 @@ __global__ void __launch_bounds__(AT_THREADS, 1) k_attn_tc(const __grid_constant
     }
     mbar_init(qfull, 1);
     mbar_init(qfree, 2);
+    mbar_init(rdone, AT_SMX);
+    mbar_init(&odec[0], 1);
+    mbar_init(&odec[1], 1);
     mbar_init(ebar, AT_SMX);
     mbar_init(odone, 1);
     mbar_init(ofree, AT_SMX);
@@ -398,7 +443,7 @@ __global__ void __launch_bounds__(AT_THREADS, 1) k_attn_tc(const __grid_constant
       const uint32_t idesc_o =
           (1u << 4) | (1u << 7) | (1u << 10) | (1u << 15) | ((uint32_t)(64 >> 3) << 17) | ((uint32_t)(128 >> 4) << 24);
       bool ok = true;
-      int u = 0, useg = 0, nseg = 0, ncommit = 0;
+      int u = 0, useg = 0, nseg = 0, ncommit = 0, nreq = 0;
       for (int i = 0; i < ntile; ++i, tp.next(T, geo.n_hg)) {
         if (!mbar_wait(&wfull[i & 1], (i >> 1) & 1, abort_flag)) { ok = false; break; }
         const uint32_t uni = unis[i & 1];
@@ -416,6 +461,17 @@ __global__ void __launch_bounds__(AT_THREADS, 1) k_attn_tc(const __grid_constant
         if (!uni) continue;
         const int s = u & 1;
         if (!mbar_wait(&pfull[s], (u >> 1) & 1, abort_flag)) { ok = false; break; }
+        if (anyw[s * 4] | anyw[s * 4 + 1] | anyw[s * 4 + 2] | anyw[s * 4 + 3]) {
+          // a head's running max moved on this tile: the softmax warps rescale its O^T column (each its quarter of
+          // the dims) before this tile's product is added; they look for the request when they see odec
+          *rq_tile = u;
+          __threadfence_block();
+          *rq_count = ++nreq;
+          mbar_arrive(&odec[s]);
+          if (!mbar_wait(rdone, (nreq - 1) & 1, abort_flag)) { ok = false; break; }
+        } else {
+          mbar_arrive(&odec[s]);
+        }
         tmem_fence_after();                            // P^T and any O^T rescale come from the softmax warps
         const uint64_t xd = sdesc_(smem_addr(sx + s * AT_TILE), AT_KBLK);
         const uint64_t pd = sdesc_(smem_addr(sx + s * AT_TILE + 8 * AT_KBLK), 16);   // this tile's P^T
@@ -452,11 +508,26 @@ __global__ void __launch_bounds__(AT_THREADS, 1) k_attn_tc(const __grid_constant
     float m = -INFINITY, mex = -INFINITY, lsum = 0.f;  // lsum: this half's share of the head's sum
     int u = 0, useg = 0, nseg = 0;
     int sb = 0, shg = 0;                               // the current segment's sequence and head group
+    int handled = 0;                                   // rescale requests applied by this warp
     bool ok = true;
+    // Before a wait that may depend on O^T(t) -- S(t + 2) reuses its slot, the epilogue needs it done -- take the
+    // O^T issuer's decision on tile t (odec) and serve its rescale request if it made one. Cheap when there is none
+    // (the usual case: a head's running max moves only by more than AT_TAU).
+    auto check = [&](int t) -> bool {
+      if (!warp_wait_(&odec[t & 1], (t >> 1) & 1, abort_flag, lane)) return false;
+      int pend = 0;
+      if (lane == 0) pend = *rq_count != handled;
+      if (__shfl_sync(0xffffffffu, pend, 0)) {
+        if (!attn_handle_request(rq_tile, pfree, rdone, fac, lrow, abort_flag, lane)) return false;
+        ++handled;
+      }
+      return true;
+    };
     // A segment's partial: re-base each head on its exact max, write (max, sum) and the output (unnormalised),
     // then release the O^T accumulator. The re-basing factors go through the parity buffer the last tile did not
     // use; a second group sync keeps the next tile from overwriting them while a warp still reads.
     auto epilogue = [&]() -> bool {
+      if ((u >= 2 && !check(u - 2)) || (u >= 1 && !check(u - 1))) return false;
       if (!warp_wait_(odone, (nseg - 1) & 1, abort_flag, lane)) return false;   // the segment's O^T is complete
       float lt = lsum + __shfl_xor_sync(0xffffffffu, lsum, 16);                // both halves of the head
       float ff = 1.f;
@@ -525,6 +596,7 @@ __global__ void __launch_bounds__(AT_THREADS, 1) k_attn_tc(const __grid_constant
       }
       if (!uni) continue;
       const int s = u & 1, use = u >> 1, par = u & 1;
+      if (u >= 2 && !check(u - 2)) { ok = false; break; }
       if (!warp_wait_(&sfull[s], use & 1, abort_flag, lane)) { ok = false; break; }
       tmem_fence_after();
       float sv[32];
@@ -587,32 +659,11 @@ __global__ void __launch_bounds__(AT_THREADS, 1) k_attn_tc(const __grid_constant
         pk[c >> 1] = *reinterpret_cast<const uint32_t*>(&pb);
       }
       lsum += ls0 + ls1;
-      // publish this group's rescale factors (by tile parity: a warp that runs ahead writes the other buffer)
+      // publish this group's rescale factors (by tile parity); the O^T issuer reads them after pfull and, when a
+      // head needs one, has every softmax warp apply them (handle_request) before this tile's product
       const uint32_t need = __ballot_sync(0xffffffffu, own && f != 1.f);
       if (own) fac[par * 64 + hl] = f;
       if (lane == 0) anyw[par * 4 + q] = need;
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&gbar[par]);
-      if (!warp_wait_(&gbar[par], use & 1, abort_flag, lane)) { ok = false; break; }
-      if (anyw[par * 4] | anyw[par * 4 + 1] | anyw[par * 4 + 2] | anyw[par * 4 + 3]) {
-        // a rescale of O^T needs the previous tile's O^T product complete (u > 0: a head's first selected row
-        // never rescales, so the first tile of a segment never gets here)
-        if (!warp_wait_(&pfree[(u - 1) & 1], ((u - 1) >> 1) & 1, abort_flag, lane)) { ok = false; break; }
-        tmem_fence_after();
-        for (int h = 0; h < 64; ++h) {
-          const float fh = fac[par * 64 + h];
-          if (fh != 1.f) {
-#pragma unroll
-            for (int j = 0; j < 4; ++j) {
-              const uint32_t a = lrow + AT_O_COL + 64 * j + h;
-              const float v = tmem_ld1_(a);
-              tmem_wait_ld();
-              tmem_st1_(a, v * fh);
-            }
-          }
-        }
-        tmem_wait_st();
-      }
       {
         // P^T row hl, rows 32 hh .. + 31 of the tile: four 16-byte chunks, 128-byte swizzle, over the slot's RoPE
         // block (S has read it: sfull)

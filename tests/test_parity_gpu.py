@@ -312,3 +312,29 @@ def test_bounded_wait_reports_timeout():
     np.testing.assert_array_equal(g["idx"], h["idx"])
     hi = oracle.HostInputs(wl)
     check_outputs(hi, LAM, h)
+
+
+@pytest.mark.parametrize("c", [60.0, 200.0])
+def test_attention_rescale_on_logit_jump(c):
+    # A row whose logit jumps tens of log2 units above the rows attended before it (in the same attention CTA)
+    # moves the running max by more than the kernel's slack: the O^T accumulator is rescaled mid-segment (by
+    # 2^-40..-50 for c = 60; underflowing to 0 for c = 200). The output must still match the oracle.
+    wl = datagen.make_workload(1, 64, 4096, seed=29, device="cuda")
+    qr0 = wl.q_rope[0, 0].float()
+    wl.cache[0, 200, 512:] = (c * qr0 / qr0.norm()).to(wl.cache.dtype)
+    hi = oracle.HostInputs(wl)
+    ids = sorted(set(range(0, 4096, 3)) | {200})
+    cap = len(ids)
+    idx = np.tile(np.array(ids, np.int32), (1, 64, 1))
+    cnt = np.full((1, 64), cap, np.int32)
+    view = vk.make_view(wl.cache, wl.q_latent, wl.q_rope)
+    p = vk.make_params(1 / 8)
+    ws = vk.alloc_workspace(view, p, cap)
+    out = torch.empty(1, 64, 512, device="cuda")
+    lse = torch.empty(1, 64, device="cuda")
+    smax = torch.empty(1, 64, device="cuda")
+    vk.vk_sparse_attn(view, p, torch.from_numpy(idx).cuda(), torch.from_numpy(cnt).cuda(), out, lse, smax, ws)
+    assert vk.vk_poll_status(ws) == vk.VK_OK
+    g = dict(out=out.cpu().double().numpy(), lse=lse.cpu().double().numpy())
+    r = check_outputs(hi, LAM, g, idx, cnt)
+    np.testing.assert_allclose(smax.cpu().double().numpy(), r["smax"], rtol=1e-4, atol=1e-4)
