@@ -485,6 +485,7 @@ __global__ void __launch_bounds__(CAND_THREADS, 8) k_select_cand(
     int H, int N, int lo, int hi, long long k_all, const long long* __restrict__ k_per_head,
     const int* __restrict__ cand_cnt, const int2* __restrict__ cand, int capc, int force_fallback,
     const __nv_bfloat16* __restrict__ rope, int64_t rld, int64_t rbs, const float* __restrict__ qt,
+    const __nv_bfloat16* __restrict__ qrope,
     int32_t* __restrict__ idx, int32_t* __restrict__ count, int cap, int append, float* __restrict__ kth,
     uint32_t* __restrict__ bitmap, long long nw, int* status) {
   extern __shared__ __align__(16) unsigned char smem[];
@@ -505,7 +506,9 @@ __global__ void __launch_bounds__(CAND_THREADS, 8) k_select_cand(
       if (threadIdx.x == 0) raise_status(status, VK_ERR_CAPACITY);
       return;
     }
-    for (int i = threadIdx.x; i < D_ROPE; i += blockDim.x) qts[i] = qt[bh * D_ROPE + i];
+    // the scoring query: qt from the query prep when it ran, else (r = 64: no rotation) the RoPE query itself
+    for (int i = threadIdx.x; i < D_ROPE; i += blockDim.x)
+      qts[i] = qt ? qt[bh * D_ROPE + i] : __bfloat162float(qrope[bh * D_ROPE + i]);
     __syncthreads();
     RecomputedKeys keys{rope + (int64_t)b * rbs, rld, qts};
     select_ordered(keys, N, lo, hi, k, out, count + bh, cap, 0, kth_bh, bm, nw, status);
@@ -549,7 +552,8 @@ cudaError_t launch_select_cand(int B, int H, int N, int lo, int hi, int64_t k, c
   if (e != cudaSuccess) return e;
   k_select_cand<<<B * H, CAND_THREADS, smem, st>>>(
       H, N, lo, hi, (long long)k, reinterpret_cast<const long long*>(k_per_head), cand_cnt, cand, capc,
-      force_fallback, static_cast<const __nv_bfloat16*>(v.rope), v.rope_ld, v.rope_bstride, qt, idx, count, cap,
+      force_fallback, static_cast<const __nv_bfloat16*>(v.rope), v.rope_ld, v.rope_bstride, qt,
+      static_cast<const __nv_bfloat16*>(v.q_rope), idx, count, cap,
       append, kth, bitmap, (long long)nw, status);
   count_launches(1);
   return cudaGetLastError();

@@ -392,7 +392,10 @@ int vk_decode_step(const vk_view* view, const vk_params* params, const vk_index*
 
   const int lo = S, hi = N - W;
   prof(0, st);
-  VK_CUDA(vk::launch_qprep(v, params->r, index ? index->rot : nullptr, qt, qcn, qrn, st), "qprep");
+  // the query prep feeds the materialised-score path and the trigger; the fused path at r = 64 scores with the
+  // RoPE query as it is (its exact fallback reads it directly)
+  const bool qprep = !L.fused || two_tier;
+  if (qprep) VK_CUDA(vk::launch_qprep(v, params->r, index ? index->rot : nullptr, qt, qcn, qrn, st), "qprep");
   prof(1, st);
   if (L.fused) {
     // threshold from a strided sample, then one scoring pass that keeps only the rows above it
@@ -422,7 +425,8 @@ int vk_decode_step(const vk_view* view, const vk_params* params, const vk_index*
     }
     prof(2, st);
     VK_CUDA(vk::launch_select_cand(B, H, N, lo, hi, k, nullptr, ccnt, cand, (int)L.capc,
-                                   (params->flags & VK_FLAG_FORCE_FALLBACK) ? 1 : 0, v, qt, idx, count, cap, 0, nullptr,
+                                   (params->flags & VK_FLAG_FORCE_FALLBACK) ? 1 : 0, v, qprep ? qt : nullptr, idx, count,
+                                   cap, 0, nullptr,
                                    selbm, L.nw, status, st), "select (candidates)");
   } else {
     if (L.tc) {
