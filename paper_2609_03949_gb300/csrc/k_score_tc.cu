@@ -11,7 +11,8 @@
 //   G groups of 4 warps  epilogue, group g taking tiles i = g (mod G). The thread of head h reads its logits in
 //                        32-row chunks (tcgen05.ld 16x32bx2 for M = 64, 32x32b for M = 128), so a chunk's
 //                        threshold test is directly the head's 32-bit bitmap word of those rows:
-//                        mode 0  write fp32 scores [B][H][ld] (also used on a strided row sample),
+//                        mode 0  write scores [B][H][ld], fp32 (or bf16 for the strided row sample that only
+//                                feeds the threshold estimate),
 //                        mode 1  emit (u, a) for archive rows with a >= theta[b,h] into per-head candidate lists:
 //                                one atomic per thread and tile reserves the room, then the chunk is staged in
 //                                shared memory and only its set bits are visited,
@@ -272,7 +273,27 @@ __global__ void __launch_bounds__((2 + 4 * (4 / NHG)) * 32, 1) k_score_tc(const 
           tmem_wait_ld();
           const int rc = row0 + (MH == 128 ? 32 * c : 64 * c + 32 * (lane >> 4));   // first row of the chunk
           uint32_t m = 0u;
-          if (MODE == 0) {
+          if (MODE == 0 && args.scores_bf16) {
+            if (valid) {
+              __nv_bfloat16* dst = reinterpret_cast<__nv_bfloat16*>(args.scores) + bh * args.scores_ld + rc;
+              if (rc + 32 <= args.n_rows && ((bh * args.scores_ld + rc) & 7) == 0) {
+#pragma unroll
+                for (int k = 0; k < 4; ++k) {
+                  uint32_t w[4];
+#pragma unroll
+                  for (int e = 0; e < 4; ++e) {
+                    const __nv_bfloat162 pb = __floats2bfloat162_rn(v[8 * k + 2 * e], v[8 * k + 2 * e + 1]);
+                    w[e] = *reinterpret_cast<const uint32_t*>(&pb);
+                  }
+                  reinterpret_cast<uint4*>(dst)[k] = make_uint4(w[0], w[1], w[2], w[3]);
+                }
+              } else {
+#pragma unroll
+                for (int k = 0; k < 32; ++k)
+                  if (rc + k < args.n_rows) dst[k] = __float2bfloat16_rn(v[k]);
+              }
+            }
+          } else if (MODE == 0) {
             if (valid) {
               float* dst = args.scores + bh * args.scores_ld + rc;
               if (rc + 32 <= args.n_rows && ((bh * args.scores_ld + rc) & 3) == 0) {

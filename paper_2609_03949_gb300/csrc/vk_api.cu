@@ -205,7 +205,7 @@ VkLayout make_layout(const vk_view& v, const vk_params& p) {
   L.off_firebm = take(L.two_tier ? sizeof(uint32_t) * BH * L.nw : 0);
   L.off_part_o = take(sizeof(float) * v.B * nslot * v.H * vk::D_LAT);
   L.off_part_ml = take(sizeof(float) * v.B * nslot * v.H * 2);
-  L.off_sample = take(L.fused ? sizeof(float) * BH * L.ns : 0);
+  L.off_sample = take(L.fused ? sizeof(uint16_t) * BH * L.ns : 0);     // bf16 sample scores
   L.off_theta = take(L.fused ? sizeof(float) * BH : 0);
   L.off_ccnt = take(L.fused ? sizeof(int) * BH : 0);
   L.off_cand = take(L.fused ? sizeof(int2) * BH * L.capc : 0);
@@ -409,6 +409,7 @@ int vk_decode_step(const vk_view* view, const vk_params* params, const vk_index*
       a.mode = 0;
       a.scores = sample;
       a.scores_ld = L.ns;
+      a.scores_bf16 = 1;
       a.status = status;
       VK_CUDA(vk::launch_score_tc(v, (int)L.soff, (int)L.ss, (int)L.ns, a, st), "sample scores");
       VK_CUDA(vk::launch_theta(B, H, (int)L.ns, (int)L.soff, (int)L.ss, lo, hi, (int)L.j, sample, theta, st), "theta");

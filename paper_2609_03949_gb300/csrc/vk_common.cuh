@@ -145,7 +145,7 @@ cudaError_t launch_trigger_dense(int B, int H, int N, int W, int n_sink, float l
                                  float* scores, const float* qcn, const float* qrn, const float* eta,
                                  const float* page_res, const float* smax1, const uint32_t* selbm,
                                  uint32_t* firebm, int64_t nw, int64_t* nfired, cudaStream_t st);
-cudaError_t launch_theta(int B, int H, int ns, int off, int stride, int lo, int hi, int j, const float* sample,
+cudaError_t launch_theta(int B, int H, int ns, int off, int stride, int lo, int hi, int j, const void* sample,
                          float* theta, cudaStream_t st);
 cudaError_t launch_select_cand(int B, int H, int N, int lo, int hi, int64_t k, const int64_t* k_per_head,
                                const int* cand_cnt, const int2* cand, int capc, int force_fallback, const vk_view& v,

@@ -11,9 +11,10 @@ struct ScoreTcArgs {
   uint32_t tmem_cols;
   // epilogue mode: 0 dense scores, 1 threshold candidates, 2 trigger
   int mode;
-  // mode 0: scores[(b*H + h) * scores_ld + row]
+  // mode 0: scores[(b*H + h) * scores_ld + row], fp32; or, with scores_bf16, bf16 (rounded to nearest even)
   float* scores;
   int64_t scores_ld;
+  int scores_bf16;
   // modes 1, 2: archive [arch_lo, arch_hi) in positions
   int arch_lo, arch_hi;
   // mode 1: emit rows with a >= theta[b*H + h]
