@@ -19,8 +19,10 @@
 //                      operand (the next 64 dims one 8 KB block away), so each latent row is staged in shared memory
 //                      once and feeds both contractions. Two issuing threads, so neither contraction waits behind
 //                      the other's issue;
-//   warps 2..5         softmax: lanes i and 16 + i of the warp on TMEM lane quarter g own head 16 g + i, rows 0..31
-//                      and 32..63 of the tile. They read the head's logits, mask them with its selection words,
+//   warps 2..5, 8..11  softmax, two warps per TMEM lane quarter g (warp % 4): warps 2..5 take rows 0..31 of the
+//                      tile, warps 8..11 rows 32..63; lanes i and 16 + i own head 16 g + i, 16 rows each. The two
+//                      warps of a quarter agree on each tile's max per head through shared memory. They read the
+//                      head's logits, mask them with its selection word,
 //                      and write P^T[h][row] = 2^(s lambda log2(e) - m_h)
 //                      (0 where the head did not select the row) in bf16 into shared memory (K-major, 128-byte
 //                      swizzle). m_h is a running max that only moves when a tile's max exceeds it by more than 32
@@ -46,8 +48,9 @@
 namespace vk {
 
 constexpr int AT_T = 64;                               // rows per tile
-constexpr int AT_SMX = 4;                              // softmax warps (one per TMEM lane quarter)
-constexpr int AT_THREADS = (4 + AT_SMX) * 32;   // producer, S issuer, softmax x4, O^T issuer, S issuer
+constexpr int AT_SMX = 8;                              // softmax warps: two per TMEM lane quarter (rows 0..31, 32..63)
+constexpr int AT_THREADS = (4 + AT_SMX) * 32;   // producer, S issuer, softmax x4, O^T issuer, S issuer, softmax x4
+constexpr int AT_W_OT = 6, AT_W_SB = 7;               // the O^T issuer and the second S issuer
 constexpr uint32_t AT_KBLK = 64 * 128;                 // one 64-column block of 64 rows (or 64 heads): 8 KB
 constexpr uint32_t AT_TILE = 9 * AT_KBLK;              // 73,728: one tile slot, and the queries
 constexpr int AT_NG = 5;                               // load groups per tile: latent pairs 0..3, RoPE block 4
@@ -68,9 +71,11 @@ struct AtSmem {
   static constexpr uint32_t uni = words + 2 * 64 * 2 * 4;
   static constexpr uint32_t fac = uni + 2 * 4;         // [2][64] f32
   static constexpr uint32_t anyw = fac + 2 * 64 * 4;   // [2][4] u32
-  static constexpr uint32_t misc = anyw + 2 * 4 * 4;   // TMEM base, abort flag, rescale request (tile, count)
+  static constexpr uint32_t tmax = anyw + 2 * 4 * 4;   // [2][2][64] f32: each row half's tile max per head
+  static constexpr uint32_t lpart = tmax + 2 * 2 * 64 * 4;   // [64] f32: the second row half's sum, at the end
+  static constexpr uint32_t misc = lpart + 64 * 4;     // TMEM base, abort flag, rescale request (tile, count)
   static constexpr uint32_t bars = (misc + 16 + 7) & ~7u;
-  static constexpr uint32_t nbars = 2 * AT_NG * 2 + 2 * 4 + 6 + 4 + 4;
+  static constexpr uint32_t nbars = 2 * AT_NG * 2 + 2 * 4 + 6 + 4 + 4 + 8;
   static constexpr uint32_t total = bars + nbars * 8;
 };
 static_assert(AtSmem::total + 1024 <= 232448, "attention shared memory exceeds the 227 KB opt-in limit");
@@ -208,6 +213,8 @@ __global__ void __launch_bounds__(AT_THREADS, 1) k_attn_tc(const __grid_constant
   uint32_t* words = reinterpret_cast<uint32_t*>(smem + AtSmem::words);
   uint32_t* unis = reinterpret_cast<uint32_t*>(smem + AtSmem::uni);
   float* fac = reinterpret_cast<float*>(smem + AtSmem::fac);
+  float* tmaxs = reinterpret_cast<float*>(smem + AtSmem::tmax);
+  float* lparts = reinterpret_cast<float*>(smem + AtSmem::lpart);
   uint32_t* anyw = reinterpret_cast<uint32_t*>(smem + AtSmem::anyw);
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + AtSmem::misc);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + AtSmem::misc + 4);
@@ -232,6 +239,7 @@ __global__ void __launch_bounds__(AT_THREADS, 1) k_attn_tc(const __grid_constant
   uint64_t* odone = ebar + 1;                 // the segment's O^T products are complete (O^T issuer's commit)
   uint64_t* ofree = odone + 1;                // the softmax warps have read the segment's O^T out of tensor memory
   uint64_t* sdone = ofree + 1;                // [2] each S issuer's final commit
+  uint64_t* hbar = sdone + 2;                 // [2][4] the two row halves of a lane quarter agree on a tile's max
 
   const AttnGeom& geo = args.g;
   const int H = args.H, T = geo.T;
@@ -260,7 +268,8 @@ __global__ void __launch_bounds__(AT_THREADS, 1) k_attn_tc(const __grid_constant
     }
     mbar_init(qfull, 1);
     mbar_init(qfree, 2);
-    mbar_init(rdone, AT_SMX);
+    mbar_init(rdone, 4);
+    for (int i = 0; i < 8; ++i) mbar_init(&hbar[i], 2);
     mbar_init(&odec[0], 1);
     mbar_init(&odec[1], 1);
     mbar_init(ebar, AT_SMX);
@@ -371,7 +380,7 @@ __global__ void __launch_bounds__(AT_THREADS, 1) k_attn_tc(const __grid_constant
       for (int i = 0; i < 2 * AT_NG; ++i)
         if (last_use[i] >= 0) mbar_wait(&xfull[i], last_use[i] & 1, nullptr);
     }
-  } else if (warp == 1 || warp == 3 + AT_SMX) {
+  } else if (warp == 1 || warp == AT_W_SB) {
     // ------------------------------------------------------------------ S issuers
     // Two threads issue the two halves of the K = 576 contraction into their own accumulators (the softmax adds
     // them): warp 1 latent dims 0..255 (16 instructions), warp 7 latent dims 256..511 and the RoPE block (20). The
@@ -432,7 +441,7 @@ __global__ void __launch_bounds__(AT_THREADS, 1) k_attn_tc(const __grid_constant
       if (!ok) { raise_status(args.status, VK_ERR_TIMEOUT); *abort_flag = 1; }
       mbar_wait(done_bar, 0, nullptr);                 // nothing this thread issued may outlive the CTA
     }
-  } else if (warp == 2 + AT_SMX) {
+  } else if (warp == AT_W_OT) {
     // ------------------------------------------------------------------ O^T issuer
     // Issues each loaded tile's O^T += X_lat^T . P^T as soon as its P^T is written; its commits release the tile's
     // latent blocks for the next load into the slot. (A commit tracks this thread's own MMAs; the tile's S, issued
@@ -497,10 +506,13 @@ __global__ void __launch_bounds__(AT_THREADS, 1) k_attn_tc(const __grid_constant
     }
   } else {
     // ------------------------------------------------------------------ softmax
-    // Head hl = 16 q + (lane % 16); lanes 0..15 take rows 0..31 of the tile, lanes 16..31 rows 32..63 (one
-    // tcgen05.ld 16x32bx2 gives each half its 32 columns of the same 16 TMEM lanes).
+    // Two warps per TMEM lane quarter: warps 2..5 take rows 0..31 of the tile (rh = 0), warps 8..11 rows 32..63.
+    // Head hl = 16 q + (lane % 16); lanes 0..15 take the first 16 of the warp's rows, lanes 16..31 the next 16 (one
+    // tcgen05.ld 16x32bx2 gives each half its 16 columns of the same 16 TMEM lanes). The two warps of a quarter
+    // agree on each tile's max per head (hbar); the rh = 0 warps publish the rescale factors and serve rescales.
     const int q = warp & 3;                            // TMEM lane quarter of this warp
-    const int hh = lane >> 4;                          // which half of the tile's rows
+    const int rh = warp >= 8 ? 1 : 0;                  // which 32 rows of the tile
+    const int hh = lane >> 4;                          // which 16 of them
     const int hl = 16 * q + (lane & 15);               // this lane's head
     const bool own = hh == 0;                          // the lane that publishes per-head values
     const float L = args.lam_log2e;
@@ -514,6 +526,7 @@ __global__ void __launch_bounds__(AT_THREADS, 1) k_attn_tc(const __grid_constant
     // O^T issuer's decision on tile t (odec) and serve its rescale request if it made one. Cheap when there is none
     // (the usual case: a head's running max moves only by more than AT_TAU).
     auto check = [&](int t) -> bool {
+      if (rh) return true;                             // the rh = 0 warps serve requests
       if (!warp_wait_(&odec[t & 1], (t >> 1) & 1, abort_flag, lane)) return false;
       int pend = 0;
       if (lane == 0) pend = *rq_count != handled;
@@ -529,27 +542,28 @@ __global__ void __launch_bounds__(AT_THREADS, 1) k_attn_tc(const __grid_constant
     auto epilogue = [&]() -> bool {
       if ((u >= 2 && !check(u - 2)) || (u >= 1 && !check(u - 1))) return false;
       if (!warp_wait_(odone, (nseg - 1) & 1, abort_flag, lane)) return false;   // the segment's O^T is complete
-      float lt = lsum + __shfl_xor_sync(0xffffffffu, lsum, 16);                // both halves of the head
+      float lt = lsum + __shfl_xor_sync(0xffffffffu, lsum, 16);                // this warp's 32 rows
       float ff = 1.f;
       if (mex != -INFINITY && m != mex) ff = ex2(m - mex);
-      lt *= ff;
       float* facf = fac + (u & 1) * 64;
-      if (own) facf[hl] = ff;
+      if (own && rh == 0) facf[hl] = ff;
+      if (own && rh == 1) lparts[hl] = lt;
       __syncwarp();
       if (lane == 0) mbar_arrive(ebar);
       if (!warp_wait_(ebar, 0, abort_flag, lane)) return false;
+      lt = (lt + lparts[hl]) * ff;                                               // both row halves (rh = 0 uses it)
       tmem_fence_after();
       const int h0 = shg * 64, nh = min(64, H - h0);
       const int slot = (int)blockIdx.x - attn_cta_of(geo, ((long long)sb * geo.n_hg + shg) * T);
       const int64_t hbase = ((int64_t)sb * args.nslot + args.slot0 + slot) * H + h0;
       constexpr float LN2 = 0.6931471805599453f;
-      if (own && hl < nh) {
+      if (own && rh == 0 && hl < nh) {
         args.part_ml[(hbase + hl) * 2] = mex * LN2;
         args.part_ml[(hbase + hl) * 2 + 1] = lt;
       }
-      // O^T block j on this warp's lanes: dims 128 j + 32 q + lane; columns: heads
+      // O^T block j on this warp's lanes: dims 128 j + 32 q + lane; columns: heads (blocks 2 rh, 2 rh + 1)
 #pragma unroll 1
-      for (int j = 0; j < 4; ++j) {
+      for (int j = 2 * rh; j < 2 * rh + 2; ++j) {
         const int dim = 128 * j + 32 * q + lane;
 #pragma unroll 1
         for (int c = 0; c < 64; c += 32) {
@@ -580,7 +594,7 @@ __global__ void __launch_bounds__(AT_THREADS, 1) k_attn_tc(const __grid_constant
       if (i < ntile) {
         if (!warp_wait_(&wfull[ws], (i >> 1) & 1, abort_flag, lane)) { ok = false; break; }
         uni = unis[ws];
-        w = words[ws * 128 + hl * 2 + hh];
+        w = words[ws * 128 + hl * 2 + rh];            // this warp's 32 rows of the head
         __syncwarp();
         if (lane == 0) mbar_arrive(&wfree[ws]);
       }
@@ -599,46 +613,47 @@ __global__ void __launch_bounds__(AT_THREADS, 1) k_attn_tc(const __grid_constant
       if (u >= 2 && !check(u - 2)) { ok = false; break; }
       if (!warp_wait_(&sfull[s], use & 1, abort_flag, lane)) { ok = false; break; }
       tmem_fence_after();
-      float sv[32];
+      float sv[16];
       {
         uint32_t* r = reinterpret_cast<uint32_t*>(sv);
         asm volatile(
-            "tcgen05.ld.sync.aligned.16x32bx2.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16,%17,"
-            "%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32], 32;\n"
+            "tcgen05.ld.sync.aligned.16x32bx2.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16], 16;\n"
             : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
-              "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]),
-              "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]),
-              "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
-            : "r"(lrow + AT_S_COL + 64 * s)
+              "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
+            : "r"(lrow + AT_S_COL + 64 * s + 32 * rh)
             : "memory");
-        float sb[32];
+        float sb[16];
         uint32_t* rb = reinterpret_cast<uint32_t*>(sb);
         asm volatile(
-            "tcgen05.ld.sync.aligned.16x32bx2.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16,%17,"
-            "%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32], 32;\n"
+            "tcgen05.ld.sync.aligned.16x32bx2.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16], 16;\n"
             : "=r"(rb[0]), "=r"(rb[1]), "=r"(rb[2]), "=r"(rb[3]), "=r"(rb[4]), "=r"(rb[5]), "=r"(rb[6]), "=r"(rb[7]),
               "=r"(rb[8]), "=r"(rb[9]), "=r"(rb[10]), "=r"(rb[11]), "=r"(rb[12]), "=r"(rb[13]), "=r"(rb[14]),
-              "=r"(rb[15]), "=r"(rb[16]), "=r"(rb[17]), "=r"(rb[18]), "=r"(rb[19]), "=r"(rb[20]), "=r"(rb[21]),
-              "=r"(rb[22]), "=r"(rb[23]), "=r"(rb[24]), "=r"(rb[25]), "=r"(rb[26]), "=r"(rb[27]), "=r"(rb[28]),
-              "=r"(rb[29]), "=r"(rb[30]), "=r"(rb[31])
-            : "r"(lrow + AT_SB_COL + 64 * s)
+              "=r"(rb[15])
+            : "r"(lrow + AT_SB_COL + 64 * s + 32 * rh)
             : "memory");
         tmem_wait_ld();
 #pragma unroll
-        for (int c = 0; c < 32; ++c) sv[c] += sb[c];
+        for (int c = 0; c < 16; ++c) sv[c] += sb[c];
       }
       tmem_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(&sfree[s]);
-      // the head's tile max over its selected rows (lambda log2(e) > 0 commutes with max)
+      // the head's tile max over its selected rows (lambda log2(e) > 0 commutes with max): this warp's 32 rows, then
+      // the other row half's through shared memory
+      const uint32_t w16 = (w >> (16 * hh)) & 0xffffu;
       float mr0 = -INFINITY, mr1 = -INFINITY;
 #pragma unroll
-      for (int c = 0; c < 32; c += 2) {
-        if ((w >> c) & 1u) mr0 = fmaxf(mr0, sv[c]);
-        if ((w >> (c + 1)) & 1u) mr1 = fmaxf(mr1, sv[c + 1]);
+      for (int c = 0; c < 16; c += 2) {
+        if ((w16 >> c) & 1u) mr0 = fmaxf(mr0, sv[c]);
+        if ((w16 >> (c + 1)) & 1u) mr1 = fmaxf(mr1, sv[c + 1]);
       }
       float mr = fmaxf(mr0, mr1);
       mr = fmaxf(mr, __shfl_xor_sync(0xffffffffu, mr, 16));
+      if (own) tmaxs[(par * 2 + rh) * 64 + hl] = mr;
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&hbar[par * 4 + q]);
+      if (!warp_wait_(&hbar[par * 4 + q], (u >> 1) & 1, abort_flag, lane)) { ok = false; break; }
+      mr = fmaxf(mr, tmaxs[(par * 2 + (rh ^ 1)) * 64 + hl]);
       const float mt = mr * L;
       mex = fmaxf(mex, mt);
       float f = 1.f;
@@ -647,30 +662,33 @@ __global__ void __launch_bounds__(AT_THREADS, 1) k_attn_tc(const __grid_constant
         m = mt;
         lsum *= f;
       }
-      uint32_t pk[16];
+      uint32_t pk[8];
       float ls0 = 0.f, ls1 = 0.f;
 #pragma unroll
-      for (int c = 0; c < 32; c += 2) {
-        const float e0 = ((w >> c) & 1u) ? ex2(fmaf(sv[c], L, -m)) : 0.f;
-        const float e1 = ((w >> (c + 1)) & 1u) ? ex2(fmaf(sv[c + 1], L, -m)) : 0.f;
+      for (int c = 0; c < 16; c += 2) {
+        const float e0 = ((w16 >> c) & 1u) ? ex2(fmaf(sv[c], L, -m)) : 0.f;
+        const float e1 = ((w16 >> (c + 1)) & 1u) ? ex2(fmaf(sv[c + 1], L, -m)) : 0.f;
         const __nv_bfloat162 pb = __floats2bfloat162_rn(e0, e1);
         ls0 += e0;
         ls1 += e1;
         pk[c >> 1] = *reinterpret_cast<const uint32_t*>(&pb);
       }
       lsum += ls0 + ls1;
-      // publish this group's rescale factors (by tile parity); the O^T issuer reads them after pfull and, when a
-      // head needs one, has every softmax warp apply them (handle_request) before this tile's product
-      const uint32_t need = __ballot_sync(0xffffffffu, own && f != 1.f);
-      if (own) fac[par * 64 + hl] = f;
-      if (lane == 0) anyw[par * 4 + q] = need;
+      // publish this group's rescale factors (by tile parity; both row halves hold the same ones, rh = 0 publishes);
+      // the O^T issuer reads them after pfull and, when a head needs one, has the rh = 0 softmax warps apply them
+      // (handle_request) before this tile's product
+      if (rh == 0) {
+        const uint32_t need = __ballot_sync(0xffffffffu, own && f != 1.f);
+        if (own) fac[par * 64 + hl] = f;
+        if (lane == 0) anyw[par * 4 + q] = need;
+      }
       {
-        // P^T row hl, rows 32 hh .. + 31 of the tile: four 16-byte chunks, 128-byte swizzle, over the slot's RoPE
-        // block (S has read it: sfull)
+        // P^T row hl, rows 32 rh + 16 hh .. + 15 of the tile: two 16-byte chunks, 128-byte swizzle, over the slot's
+        // RoPE block (S has read it: sfull)
         unsigned char* row = sx + s * AT_TILE + 8 * AT_KBLK + hl * 128;
 #pragma unroll
-        for (int i = 0; i < 4; ++i)
-          *reinterpret_cast<uint4*>(row + (((4 * hh + i) ^ (hl & 7)) * 16)) =
+        for (int i = 0; i < 2; ++i)
+          *reinterpret_cast<uint4*>(row + (((4 * rh + 2 * hh + i) ^ (hl & 7)) * 16)) =
               make_uint4(pk[4 * i], pk[4 * i + 1], pk[4 * i + 2], pk[4 * i + 3]);
       }
       fence_async_smem_();
