@@ -20,9 +20,9 @@
 //                      once and feeds both contractions. Two issuing threads, so neither contraction waits behind
 //                      the other's issue;
 //   warps 2..5, 8..11  softmax, two warps per TMEM lane quarter g (warp % 4): warps 2..5 take rows 0..31 of the
-//                      tile, warps 8..11 rows 32..63; lanes i and 16 + i own head 16 g + i, 16 rows each. The two
-//                      warps of a quarter agree on each tile's max per head through shared memory. They read the
-//                      head's logits, mask them with its selection word,
+//                      tile, warps 8..11 rows 32..63; lanes i and 16 + i own head 16 g + i, 16 rows each. Both
+//                      warps of a quarter read all 64 of the head's logits, so each finds the same tile max without
+//                      an exchange. They mask the logits with the head's selection words,
 //                      and write P^T[h][row] = 2^(s lambda log2(e) - m_h)
 //                      (0 where the head did not select the row) in bf16 into shared memory (K-major, 128-byte
 //                      swizzle). m_h is a running max that only moves when a tile's max exceeds it by more than 32
@@ -71,11 +71,10 @@ struct AtSmem {
   static constexpr uint32_t uni = words + 2 * 64 * 2 * 4;
   static constexpr uint32_t fac = uni + 2 * 4;         // [2][64] f32
   static constexpr uint32_t anyw = fac + 2 * 64 * 4;   // [2][4] u32
-  static constexpr uint32_t tmax = anyw + 2 * 4 * 4;   // [2][2][64] f32: each row half's tile max per head
-  static constexpr uint32_t lpart = tmax + 2 * 2 * 64 * 4;   // [64] f32: the second row half's sum, at the end
+  static constexpr uint32_t lpart = anyw + 2 * 4 * 4;  // [64] f32: the second row half's sum, at the end
   static constexpr uint32_t misc = lpart + 64 * 4;     // TMEM base, abort flag, rescale request (tile, count)
   static constexpr uint32_t bars = (misc + 16 + 7) & ~7u;
-  static constexpr uint32_t nbars = 2 * AT_NG * 2 + 2 * 4 + 6 + 4 + 4 + 8;
+  static constexpr uint32_t nbars = 2 * AT_NG * 2 + 2 * 4 + 6 + 4 + 4;
   static constexpr uint32_t total = bars + nbars * 8;
 };
 static_assert(AtSmem::total + 1024 <= 232448, "attention shared memory exceeds the 227 KB opt-in limit");
@@ -147,6 +146,18 @@ __device__ __forceinline__ bool warp_wait_(uint64_t* bar, uint32_t parity, volat
   return __shfl_sync(0xffffffffu, w, 0);
 }
 
+// 16 columns of the M = 64 accumulator's 16 TMEM lanes: lanes 0..15 of the warp get columns col .. col + 15, lanes
+// 16..31 columns col + 16 .. col + 31 of the same TMEM lanes (asynchronous until tmem_wait_ld).
+__device__ __forceinline__ void tmem_ld16x2_(uint32_t taddr, float* v) {
+  uint32_t* r = reinterpret_cast<uint32_t*>(v);
+  asm volatile(
+      "tcgen05.ld.sync.aligned.16x32bx2.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16], 16;\n"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]), "=r"(r[8]),
+        "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
+      : "r"(taddr)
+      : "memory");
+}
+
 // A rescale request of the O^T issuer (tile r: some head's running max moved there), served by one softmax warp
 // (warp-collective): once O^T(r - 1) is complete, scale the warp's quarter of the dims (TMEM lanes lrow..) of every
 // such head's O^T column by its factor in fac[r & 1], then report on rdone. Out of line: it is rare.
@@ -213,7 +224,6 @@ __global__ void __launch_bounds__(AT_THREADS, 1) k_attn_tc(const __grid_constant
   uint32_t* words = reinterpret_cast<uint32_t*>(smem + AtSmem::words);
   uint32_t* unis = reinterpret_cast<uint32_t*>(smem + AtSmem::uni);
   float* fac = reinterpret_cast<float*>(smem + AtSmem::fac);
-  float* tmaxs = reinterpret_cast<float*>(smem + AtSmem::tmax);
   float* lparts = reinterpret_cast<float*>(smem + AtSmem::lpart);
   uint32_t* anyw = reinterpret_cast<uint32_t*>(smem + AtSmem::anyw);
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + AtSmem::misc);
@@ -239,7 +249,6 @@ __global__ void __launch_bounds__(AT_THREADS, 1) k_attn_tc(const __grid_constant
   uint64_t* odone = ebar + 1;                 // the segment's O^T products are complete (O^T issuer's commit)
   uint64_t* ofree = odone + 1;                // the softmax warps have read the segment's O^T out of tensor memory
   uint64_t* sdone = ofree + 1;                // [2] each S issuer's final commit
-  uint64_t* hbar = sdone + 2;                 // [2][4] the two row halves of a lane quarter agree on a tile's max
 
   const AttnGeom& geo = args.g;
   const int H = args.H, T = geo.T;
@@ -269,7 +278,6 @@ __global__ void __launch_bounds__(AT_THREADS, 1) k_attn_tc(const __grid_constant
     mbar_init(qfull, 1);
     mbar_init(qfree, 2);
     mbar_init(rdone, 4);
-    for (int i = 0; i < 8; ++i) mbar_init(&hbar[i], 2);
     mbar_init(&odec[0], 1);
     mbar_init(&odec[1], 1);
     mbar_init(ebar, AT_SMX);
@@ -508,8 +516,8 @@ __global__ void __launch_bounds__(AT_THREADS, 1) k_attn_tc(const __grid_constant
     // ------------------------------------------------------------------ softmax
     // Two warps per TMEM lane quarter: warps 2..5 take rows 0..31 of the tile (rh = 0), warps 8..11 rows 32..63.
     // Head hl = 16 q + (lane % 16); lanes 0..15 take the first 16 of the warp's rows, lanes 16..31 the next 16 (one
-    // tcgen05.ld 16x32bx2 gives each half its 16 columns of the same 16 TMEM lanes). The two warps of a quarter
-    // agree on each tile's max per head (hbar); the rh = 0 warps publish the rescale factors and serve rescales.
+    // tcgen05.ld 16x32bx2 gives each half its 16 columns of the same 16 TMEM lanes). Both warps of a quarter take
+    // each tile's max over all 64 rows; the rh = 0 warps publish the rescale factors and serve rescales.
     const int q = warp & 3;                            // TMEM lane quarter of this warp
     const int rh = warp >= 8 ? 1 : 0;                  // which 32 rows of the tile
     const int hh = lane >> 4;                          // which 16 of them
@@ -589,12 +597,13 @@ __global__ void __launch_bounds__(AT_THREADS, 1) k_attn_tc(const __grid_constant
     // keeps the loop's code small (instruction fetch is shared with the issuing warps' loops)
     for (int i = 0; i <= ntile; ++i, tp.next(T, geo.n_hg)) {
       const int ws = i & 1;
-      uint32_t uni = 0u, w = 0u;
+      uint32_t uni = 0u, w = 0u, wo = 0u;
       const bool fresh = i == ntile || i == 0 || tp.kt == 0;
       if (i < ntile) {
         if (!warp_wait_(&wfull[ws], (i >> 1) & 1, abort_flag, lane)) { ok = false; break; }
         uni = unis[ws];
         w = words[ws * 128 + hl * 2 + rh];            // this warp's 32 rows of the head
+        wo = words[ws * 128 + hl * 2 + (rh ^ 1)];     // the other 32
         __syncwarp();
         if (lane == 0) mbar_arrive(&wfree[ws]);
       }
@@ -613,47 +622,36 @@ __global__ void __launch_bounds__(AT_THREADS, 1) k_attn_tc(const __grid_constant
       if (u >= 2 && !check(u - 2)) { ok = false; break; }
       if (!warp_wait_(&sfull[s], use & 1, abort_flag, lane)) { ok = false; break; }
       tmem_fence_after();
-      float sv[16];
+      // this warp's 16 rows per lane (sv) and the other row half's (ov), both S halves added: each warp of a quarter
+      // takes the whole tile's max itself, so both reach the same running max without an exchange
+      float sv[16], ov[16];
       {
-        uint32_t* r = reinterpret_cast<uint32_t*>(sv);
-        asm volatile(
-            "tcgen05.ld.sync.aligned.16x32bx2.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16], 16;\n"
-            : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
-              "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
-            : "r"(lrow + AT_S_COL + 64 * s + 32 * rh)
-            : "memory");
-        float sb[16];
-        uint32_t* rb = reinterpret_cast<uint32_t*>(sb);
-        asm volatile(
-            "tcgen05.ld.sync.aligned.16x32bx2.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16], 16;\n"
-            : "=r"(rb[0]), "=r"(rb[1]), "=r"(rb[2]), "=r"(rb[3]), "=r"(rb[4]), "=r"(rb[5]), "=r"(rb[6]), "=r"(rb[7]),
-              "=r"(rb[8]), "=r"(rb[9]), "=r"(rb[10]), "=r"(rb[11]), "=r"(rb[12]), "=r"(rb[13]), "=r"(rb[14]),
-              "=r"(rb[15])
-            : "r"(lrow + AT_SB_COL + 64 * s + 32 * rh)
-            : "memory");
+        float sb[16], ob[16];
+        const uint32_t c0 = lrow + 64 * s + 32 * rh, c1 = lrow + 64 * s + 32 * (rh ^ 1);
+        tmem_ld16x2_(c0 + AT_S_COL, sv);
+        tmem_ld16x2_(c0 + AT_SB_COL, sb);
+        tmem_ld16x2_(c1 + AT_S_COL, ov);
+        tmem_ld16x2_(c1 + AT_SB_COL, ob);
         tmem_wait_ld();
 #pragma unroll
-        for (int c = 0; c < 16; ++c) sv[c] += sb[c];
+        for (int c = 0; c < 16; ++c) {
+          sv[c] += sb[c];
+          ov[c] += ob[c];
+        }
       }
       tmem_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(&sfree[s]);
-      // the head's tile max over its selected rows (lambda log2(e) > 0 commutes with max): this warp's 32 rows, then
-      // the other row half's through shared memory
-      const uint32_t w16 = (w >> (16 * hh)) & 0xffffu;
+      // the head's tile max over its selected rows (lambda log2(e) > 0 commutes with max)
+      const uint32_t w16 = (w >> (16 * hh)) & 0xffffu, o16 = (wo >> (16 * hh)) & 0xffffu;
       float mr0 = -INFINITY, mr1 = -INFINITY;
 #pragma unroll
-      for (int c = 0; c < 16; c += 2) {
+      for (int c = 0; c < 16; ++c) {
         if ((w16 >> c) & 1u) mr0 = fmaxf(mr0, sv[c]);
-        if ((w16 >> (c + 1)) & 1u) mr1 = fmaxf(mr1, sv[c + 1]);
+        if ((o16 >> c) & 1u) mr1 = fmaxf(mr1, ov[c]);
       }
       float mr = fmaxf(mr0, mr1);
       mr = fmaxf(mr, __shfl_xor_sync(0xffffffffu, mr, 16));
-      if (own) tmaxs[(par * 2 + rh) * 64 + hl] = mr;
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&hbar[par * 4 + q]);
-      if (!warp_wait_(&hbar[par * 4 + q], (u >> 1) & 1, abort_flag, lane)) { ok = false; break; }
-      mr = fmaxf(mr, tmaxs[(par * 2 + (rh ^ 1)) * 64 + hl]);
       const float mt = mr * L;
       mex = fmaxf(mex, mt);
       float f = 1.f;
