@@ -19,10 +19,11 @@
 //                      operand (the next 64 dims one 8 KB block away), so each latent row is staged in shared memory
 //                      once and feeds both contractions. Two issuing threads, so neither contraction waits behind
 //                      the other's issue;
-//   warps 2..5, 8..11  softmax, two warps per TMEM lane quarter g (warp % 4): warps 2..5 take rows 0..31 of the
-//                      tile, warps 8..11 rows 32..63; lanes i and 16 + i own head 16 g + i, 16 rows each. Both
-//                      warps of a quarter read all 64 of the head's logits, so each finds the same tile max without
-//                      an exchange. They mask the logits with the head's selection words,
+//   warps 2..5, 8..11  softmax, two warps per TMEM lane quarter g (warp % 4); lanes i and 16 + i own head 16 g + i,
+//                      and lane half t = 0, 1 reads rows 32 t .. 32 t + 31. Both warps of a quarter read all 64 of
+//                      the head's logits, so each finds the same tile max without an exchange; warps 2..5 then
+//                      write rows 32 t .. + 15, warps 8..11 rows 32 t + 16 .. + 31. They mask the logits with the
+//                      head's selection words,
 //                      and write P^T[h][row] = 2^(s lambda log2(e) - m_h)
 //                      (0 where the head did not select the row) in bf16 into shared memory (K-major, 128-byte
 //                      swizzle). m_h is a running max that only moves when a tile's max exceeds it by more than 32
@@ -146,18 +147,20 @@ __device__ __forceinline__ bool warp_wait_(uint64_t* bar, uint32_t parity, volat
   return __shfl_sync(0xffffffffu, w, 0);
 }
 
-// 16 columns of the M = 64 accumulator's 16 TMEM lanes: lanes 0..15 of the warp get columns col .. col + 15, lanes
-// 16..31 columns col + 16 .. col + 31 of the same TMEM lanes (asynchronous until tmem_wait_ld).
-__device__ __forceinline__ void tmem_ld16x2_(uint32_t taddr, float* v) {
+// 32 columns of the M = 64 accumulator's 16 TMEM lanes: lanes 0..15 of the warp get columns col .. col + 31, lanes
+// 16..31 columns col + 32 .. col + 63 of the same TMEM lanes (asynchronous until tmem_wait_ld).
+__device__ __forceinline__ void tmem_ld32x2_(uint32_t taddr, float* v) {
   uint32_t* r = reinterpret_cast<uint32_t*>(v);
   asm volatile(
-      "tcgen05.ld.sync.aligned.16x32bx2.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16], 16;\n"
+      "tcgen05.ld.sync.aligned.16x32bx2.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
+      "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32], 32;\n"
       : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]), "=r"(r[8]),
-        "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
+        "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]), "=r"(r[16]),
+        "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]),
+        "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
       : "r"(taddr)
       : "memory");
 }
-
 // A rescale request of the O^T issuer (tile r: some head's running max moved there), served by one softmax warp
 // (warp-collective): once O^T(r - 1) is complete, scale the warp's quarter of the dims (TMEM lanes lrow..) of every
 // such head's O^T column by its factor in fac[r & 1], then report on rdone. Out of line: it is rare.
@@ -514,18 +517,18 @@ __global__ void __launch_bounds__(AT_THREADS, 1) k_attn_tc(const __grid_constant
     }
   } else {
     // ------------------------------------------------------------------ softmax
-    // Two warps per TMEM lane quarter: warps 2..5 take rows 0..31 of the tile (rh = 0), warps 8..11 rows 32..63.
-    // Head hl = 16 q + (lane % 16); lanes 0..15 take the first 16 of the warp's rows, lanes 16..31 the next 16 (one
-    // tcgen05.ld 16x32bx2 gives each half its 16 columns of the same 16 TMEM lanes). Both warps of a quarter take
-    // each tile's max over all 64 rows; the rh = 0 warps publish the rescale factors and serve rescales.
+    // Two warps per TMEM lane quarter. Head hl = 16 q + (lane % 16); one tcgen05.ld 16x32bx2 per S half gives lanes
+    // 0..15 the head's rows 0..31 and lanes 16..31 its rows 32..63, so both warps of a quarter see the whole tile and
+    // take its max alone. Of its 32 rows a lane writes P for 16: rows 32 hh + 16 rh .. + 15 (rh = 0 for warps 2..5,
+    // 1 for warps 8..11). The rh = 0 warps publish the rescale factors and serve rescales.
     const int q = warp & 3;                            // TMEM lane quarter of this warp
-    const int rh = warp >= 8 ? 1 : 0;                  // which 32 rows of the tile
-    const int hh = lane >> 4;                          // which 16 of them
+    const int rh = warp >= 8 ? 1 : 0;                  // which 16 of the lane's 32 rows this warp writes
+    const int hh = lane >> 4;                          // which 32 rows of the tile the lane reads
     const int hl = 16 * q + (lane & 15);               // this lane's head
     const bool own = hh == 0;                          // the lane that publishes per-head values
     const float L = args.lam_log2e;
     const uint32_t lrow = tmem + ((uint32_t)(32 * q) << 16);
-    float m = -INFINITY, mex = -INFINITY, lsum = 0.f;  // lsum: this half's share of the head's sum
+    float m = -INFINITY, mex = -INFINITY, lsum = 0.f;  // lsum: this warp's share of the head's sum
     int u = 0, useg = 0, nseg = 0;
     int sb = 0, shg = 0;                               // the current segment's sequence and head group
     int handled = 0;                                   // rescale requests applied by this warp
@@ -559,7 +562,7 @@ __global__ void __launch_bounds__(AT_THREADS, 1) k_attn_tc(const __grid_constant
       __syncwarp();
       if (lane == 0) mbar_arrive(ebar);
       if (!warp_wait_(ebar, 0, abort_flag, lane)) return false;
-      lt = (lt + lparts[hl]) * ff;                                               // both row halves (rh = 0 uses it)
+      lt = (lt + lparts[hl]) * ff;                                               // both warps' rows (rh = 0 uses it)
       tmem_fence_after();
       const int h0 = shg * 64, nh = min(64, H - h0);
       const int slot = (int)blockIdx.x - attn_cta_of(geo, ((long long)sb * geo.n_hg + shg) * T);
@@ -597,13 +600,12 @@ __global__ void __launch_bounds__(AT_THREADS, 1) k_attn_tc(const __grid_constant
     // keeps the loop's code small (instruction fetch is shared with the issuing warps' loops)
     for (int i = 0; i <= ntile; ++i, tp.next(T, geo.n_hg)) {
       const int ws = i & 1;
-      uint32_t uni = 0u, w = 0u, wo = 0u;
+      uint32_t uni = 0u, w = 0u;
       const bool fresh = i == ntile || i == 0 || tp.kt == 0;
       if (i < ntile) {
         if (!warp_wait_(&wfull[ws], (i >> 1) & 1, abort_flag, lane)) { ok = false; break; }
         uni = unis[ws];
-        w = words[ws * 128 + hl * 2 + rh];            // this warp's 32 rows of the head
-        wo = words[ws * 128 + hl * 2 + (rh ^ 1)];     // the other 32
+        w = words[ws * 128 + hl * 2 + hh];            // rows 32 hh .. 32 hh + 31 of the head
         __syncwarp();
         if (lane == 0) mbar_arrive(&wfree[ws]);
       }
@@ -624,34 +626,32 @@ __global__ void __launch_bounds__(AT_THREADS, 1) k_attn_tc(const __grid_constant
       tmem_fence_after();
       // this warp's 16 rows per lane (sv) and the other row half's (ov), both S halves added: each warp of a quarter
       // takes the whole tile's max itself, so both reach the same running max without an exchange
-      float sv[16], ov[16];
+      float sv[32];
       {
-        float sb[16], ob[16];
-        const uint32_t c0 = lrow + 64 * s + 32 * rh, c1 = lrow + 64 * s + 32 * (rh ^ 1);
-        tmem_ld16x2_(c0 + AT_S_COL, sv);
-        tmem_ld16x2_(c0 + AT_SB_COL, sb);
-        tmem_ld16x2_(c1 + AT_S_COL, ov);
-        tmem_ld16x2_(c1 + AT_SB_COL, ob);
+        float sb[32];
+        const uint32_t c0 = lrow + 64 * s;
+        tmem_ld32x2_(c0 + AT_S_COL, sv);
+        tmem_ld32x2_(c0 + AT_SB_COL, sb);
         tmem_wait_ld();
 #pragma unroll
-        for (int c = 0; c < 16; ++c) {
-          sv[c] += sb[c];
-          ov[c] += ob[c];
-        }
+        for (int c = 0; c < 32; ++c) sv[c] += sb[c];
       }
       tmem_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(&sfree[s]);
-      // the head's tile max over its selected rows (lambda log2(e) > 0 commutes with max)
-      const uint32_t w16 = (w >> (16 * hh)) & 0xffffu, o16 = (wo >> (16 * hh)) & 0xffffu;
       float mr0 = -INFINITY, mr1 = -INFINITY;
 #pragma unroll
-      for (int c = 0; c < 16; ++c) {
-        if ((w16 >> c) & 1u) mr0 = fmaxf(mr0, sv[c]);
-        if ((o16 >> c) & 1u) mr1 = fmaxf(mr1, ov[c]);
+      for (int c = 0; c < 32; c += 2) {
+        if ((w >> c) & 1u) mr0 = fmaxf(mr0, sv[c]);
+        if ((w >> (c + 1)) & 1u) mr1 = fmaxf(mr1, sv[c + 1]);
       }
       float mr = fmaxf(mr0, mr1);
       mr = fmaxf(mr, __shfl_xor_sync(0xffffffffu, mr, 16));
+      // this warp's P rows: 32 hh + 16 rh .. + 15
+      const uint32_t w16 = (w >> (16 * rh)) & 0xffffu;
+      float pv[16];
+#pragma unroll
+      for (int c = 0; c < 16; ++c) pv[c] = rh ? sv[16 + c] : sv[c];
       const float mt = mr * L;
       mex = fmaxf(mex, mt);
       float f = 1.f;
@@ -664,15 +664,15 @@ __global__ void __launch_bounds__(AT_THREADS, 1) k_attn_tc(const __grid_constant
       float ls0 = 0.f, ls1 = 0.f;
 #pragma unroll
       for (int c = 0; c < 16; c += 2) {
-        const float e0 = ((w16 >> c) & 1u) ? ex2(fmaf(sv[c], L, -m)) : 0.f;
-        const float e1 = ((w16 >> (c + 1)) & 1u) ? ex2(fmaf(sv[c + 1], L, -m)) : 0.f;
+        const float e0 = ((w16 >> c) & 1u) ? ex2(fmaf(pv[c], L, -m)) : 0.f;
+        const float e1 = ((w16 >> (c + 1)) & 1u) ? ex2(fmaf(pv[c + 1], L, -m)) : 0.f;
         const __nv_bfloat162 pb = __floats2bfloat162_rn(e0, e1);
         ls0 += e0;
         ls1 += e1;
         pk[c >> 1] = *reinterpret_cast<const uint32_t*>(&pb);
       }
       lsum += ls0 + ls1;
-      // publish this group's rescale factors (by tile parity; both row halves hold the same ones, rh = 0 publishes);
+      // publish this group's rescale factors (by tile parity; both warps of the quarter hold the same ones, rh = 0 publishes);
       // the O^T issuer reads them after pfull and, when a head needs one, has the rh = 0 softmax warps apply them
       // (handle_request) before this tile's product
       if (rh == 0) {
@@ -681,12 +681,12 @@ __global__ void __launch_bounds__(AT_THREADS, 1) k_attn_tc(const __grid_constant
         if (lane == 0) anyw[par * 4 + q] = need;
       }
       {
-        // P^T row hl, rows 32 rh + 16 hh .. + 15 of the tile: two 16-byte chunks, 128-byte swizzle, over the slot's
+        // P^T row hl, rows 32 hh + 16 rh .. + 15 of the tile: two 16-byte chunks, 128-byte swizzle, over the slot's
         // RoPE block (S has read it: sfull)
         unsigned char* row = sx + s * AT_TILE + 8 * AT_KBLK + hl * 128;
 #pragma unroll
         for (int i = 0; i < 2; ++i)
-          *reinterpret_cast<uint4*>(row + (((4 * rh + 2 * hh + i) ^ (hl & 7)) * 16)) =
+          *reinterpret_cast<uint4*>(row + (((4 * hh + 2 * rh + i) ^ (hl & 7)) * 16)) =
               make_uint4(pk[4 * i], pk[4 * i + 1], pk[4 * i + 2], pk[4 * i + 3]);
       }
       fence_async_smem_();
