@@ -274,7 +274,8 @@ def run_native(args):
     torch.cuda.synchronize()
     assert vk.vk_poll_status(buf.ws) == vk.VK_OK
     step_events = [[torch.cuda.Event(enable_timing=True) for _ in range(7)] for _ in range(args.steps)]
-    for evs in step_events:          # create the underlying cudaEvent_t handles outside the timed region
+    step_brackets = [[torch.cuda.Event(enable_timing=True) for _ in range(2)] for _ in range(args.steps)]
+    for evs in step_events + step_brackets:   # create the underlying cudaEvent_t handles outside the timed region
         for e in evs:
             e.record(stream)
     torch.cuda.synchronize()
@@ -288,33 +289,44 @@ def run_native(args):
     if pg:
         pg.barrier()
     torch.cuda.synchronize()
+    # pass 1, the headline: the steps alone (no stage events), bracketed by events on the launching stream;
+    # with an L2 flush between steps, each step is bracketed by its own pair so that the flushes stay outside
     launches0 = vk.vk_profile_launches()
     clocks.mark(True)
     t_start.record(stream)
-    for evs in step_events:
+    for sb, se in step_brackets:
         if flush is not None:
             flush.fill_(1)
-        vk.vk_profile_set_events(evs)    # this step records its stage boundaries into its own events
+            sb.record(stream)
         buf.run(view, params)
+        if flush is not None:
+            se.record(stream)
     t_end.record(stream)
     torch.cuda.synchronize()
     clocks.mark(False)
     launches = vk.vk_profile_launches() - launches0
     elapsed_ms = t_start.elapsed_time(t_end)
+    if flush is not None:
+        elapsed_ms = sum(sb.elapsed_time(se) for sb, se in step_brackets)
+    elapsed_ms = max_over_ranks(elapsed_ms, pg, dev)
+    clk = clocks.stop()
+    ms_step = elapsed_ms / args.steps
+    assert vk.vk_poll_status(buf.ws) == vk.VK_OK
+    # pass 2, the breakdown: the same steps again, each recording its stage boundaries into its own events
     stage_ms = np.zeros(6)
     total_ms_events = 0.0
+    for evs in step_events:
+        if flush is not None:
+            flush.fill_(1)
+        vk.vk_profile_set_events(evs)
+        buf.run(view, params)
+    torch.cuda.synchronize()
+    vk.vk_profile_set_events([])
     for evs in step_events:
         for i in range(6):
             stage_ms[i] += evs[i].elapsed_time(evs[i + 1])
         total_ms_events += evs[0].elapsed_time(evs[6])
-    elapsed_ms = max_over_ranks(elapsed_ms, pg, dev)
-    clk = clocks.stop()
-    vk.vk_profile_set_events([])
     assert vk.vk_poll_status(buf.ws) == vk.VK_OK
-    # kernel-time per step: the events bracket only the library's launches (host gaps between steps excluded)
-    ms_step = elapsed_ms / args.steps
-    if flush is not None:                # the flushes are inside [t_start, t_end]: time the steps by their events
-        ms_step = max_over_ranks(total_ms_events / args.steps, pg, dev)
     dev_ms_step = total_ms_events / args.steps
     stage_ms /= args.steps
 
@@ -336,36 +348,63 @@ def run_native(args):
             "algorithmic_bytes_per_launch": stage_bytes[dom],
             "ms_per_launch": dom_ms}
 
-    # ---- end to end through the public C entry point with host buffers (pinned)
+    # ---- end to end through the public C entry point with host buffers (pinned). Every step copies its queries
+    # in from pinned host memory and its outputs back; the copies run on their own streams and overlap the
+    # neighbouring steps' kernels (two query/output buffer sets, ordered by events), as a serving loop would.
     qlh = wl.q_latent.cpu().pin_memory()
     qrh = wl.q_rope.cpu().pin_memory()
-    outh = torch.empty_like(buf.out, device="cpu").pin_memory()
-    lseh = torch.empty_like(buf.lse, device="cpu").pin_memory()
+    qls = [torch.empty_like(wl.q_latent) for _ in range(2)]
+    qrs = [torch.empty_like(wl.q_rope) for _ in range(2)]
+    views = [vk.make_view(wl.cache, qls[k], qrs[k]) for k in range(2)]
+    bufs = [buf, vk.DecodeBuffers(views[1], params, device=dev)]
+    outh = [torch.empty_like(buf.out, device="cpu").pin_memory() for _ in range(2)]
+    lseh = [torch.empty_like(buf.lse, device="cpu").pin_memory() for _ in range(2)]
     h2d = qlh.numel() * qlh.element_size() + qrh.numel() * qrh.element_size()
-    d2h = outh.numel() * outh.element_size() + lseh.numel() * lseh.element_size()
-    for _ in range(3):
-        wl.q_latent.copy_(qlh, non_blocking=True)
-        wl.q_rope.copy_(qrh, non_blocking=True)
-        buf.run(view, params)
-        outh.copy_(buf.out, non_blocking=True)
-        lseh.copy_(buf.lse, non_blocking=True)
+    d2h = outh[0].numel() * outh[0].element_size() + lseh[0].numel() * lseh[0].element_size()
+    s_in = torch.cuda.Stream(dev)
+    s_out = torch.cuda.Stream(dev)
+    ev_in = [torch.cuda.Event() for _ in range(2)]      # queries of buffer k landed
+    ev_comp = [torch.cuda.Event() for _ in range(2)]    # step on buffer k done
+    ev_out = [torch.cuda.Event() for _ in range(2)]     # outputs of buffer k copied out
+
+    def e2e_steps(n):
+        for i in range(n):
+            k = i & 1
+            if i >= 2:
+                s_in.wait_event(ev_comp[k])              # step i - 2 has read these query buffers
+            with torch.cuda.stream(s_in):
+                qls[k].copy_(qlh, non_blocking=True)
+                qrs[k].copy_(qrh, non_blocking=True)
+                ev_in[k].record(s_in)
+            stream.wait_event(ev_in[k])
+            if i >= 2:
+                stream.wait_event(ev_out[k])             # step i - 2's outputs are out of these buffers
+            bufs[k].run(views[k], params)
+            ev_comp[k].record(stream)
+            s_out.wait_event(ev_comp[k])
+            with torch.cuda.stream(s_out):
+                outh[k].copy_(bufs[k].out, non_blocking=True)
+                lseh[k].copy_(bufs[k].lse, non_blocking=True)
+                ev_out[k].record(s_out)
+        for k in range(min(n, 2)):
+            stream.wait_event(ev_out[k])
+
+    e2e_steps(3)
     torch.cuda.synchronize()
     if pg:
         pg.barrier()
     e0 = torch.cuda.Event(enable_timing=True)
     e1 = torch.cuda.Event(enable_timing=True)
     e0.record(stream)
-    for _ in range(args.steps):
-        wl.q_latent.copy_(qlh, non_blocking=True)
-        wl.q_rope.copy_(qrh, non_blocking=True)
-        buf.run(view, params)
-        outh.copy_(buf.out, non_blocking=True)
-        lseh.copy_(buf.lse, non_blocking=True)
+    s_in.wait_event(e0)
+    s_out.wait_event(e0)
+    e2e_steps(args.steps)
     e1.record(stream)
     torch.cuda.synchronize()
     e2e_ms = e0.elapsed_time(e1)
     e2e_ms = max_over_ranks(e2e_ms, pg, dev)
-    assert torch.isfinite(lseh).all()
+    assert all(torch.isfinite(t).all() for t in lseh)
+    assert vk.vk_poll_status(bufs[1].ws) == vk.VK_OK
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
