@@ -101,7 +101,7 @@ uint16_t vko_bf16_rne(double x) {
   return (uint16_t)(b >> 16);
 }
 
-/* ---------------------------------------------------------------- set sizes (Sec. 4.1, spec rho) */
+/* ---------------------------------------------------------------- set sizes (Sec. 4.1, keep ratio rho) */
 /* Archive A = [n_sink, N-W); keep k = min(ceil(rho*N), |A|) archived rows per head. */
 int64_t vko_keep_count(int32_t N, double rho, int32_t W, int32_t n_sink) {
   int64_t A = (int64_t)N - W - n_sink;

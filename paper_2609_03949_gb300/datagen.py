@@ -144,29 +144,29 @@ def make_workload(B: int, H: int, N: int, *, dtype: str = "bf16", seed: int = 0,
                     seed=int(seed))
 
 
-# The five workloads of the evaluation, restated with their sizes. ``config_params`` gives the selection
-# parameters each one is run with; every config draws from seed (index - 1) unless a sweep point overrides it.
+# The five evaluation workloads, named by what they are, with their sizes. ``CONFIG_PARAMS`` gives the selection
+# parameters each one is run with, and each draws from its own seed unless a sweep point overrides it.
 CONFIGS = {
-    1: dict(B=1, H=16, N=1024, dtype="f32", n_planted=8, seed=0),
-    2: dict(B=1, H=128, N=8192, dtype="bf16", n_planted=32, seed=1),
-    3: dict(B=16, H=64, N=32768, dtype="bf16", n_planted=0, lognormal_keys=True, seed=2),
-    4: dict(B=8, H=128, N=65536, dtype="bf16", n_planted=32, seed=3),
-    5: dict(B=8, H=64, N=65536, dtype="bf16", n_planted=64, seed=1000),
+    "fp32_h16_n1k": dict(B=1, H=16, N=1024, dtype="f32", n_planted=8, seed=0),
+    "h128_n8k": dict(B=1, H=128, N=8192, dtype="bf16", n_planted=32, seed=1),
+    "h64_n32k_lognormal": dict(B=16, H=64, N=32768, dtype="bf16", n_planted=0, lognormal_keys=True, seed=2),
+    "h128_n64k_two_tier": dict(B=8, H=128, N=65536, dtype="bf16", n_planted=32, seed=3),
+    "h64_n64k": dict(B=8, H=64, N=65536, dtype="bf16", n_planted=64, seed=1000),
 }
 
 CONFIG_PARAMS = {
-    1: dict(rho=1 / 8, window=64, r=64),
-    2: dict(rho=1 / 32, window=128, r=64),
-    3: dict(rho=1 / 32, window=256, r=64),
-    4: dict(rho=1 / 32, window=256, r=64, trigger=1, z_eff=1.0),
-    5: dict(rho=1 / 32, window=256, r=64),
+    "fp32_h16_n1k": dict(rho=1 / 8, window=64, r=64),
+    "h128_n8k": dict(rho=1 / 32, window=128, r=64),
+    "h64_n32k_lognormal": dict(rho=1 / 32, window=256, r=64),
+    "h128_n64k_two_tier": dict(rho=1 / 32, window=256, r=64, trigger=1, z_eff=1.0),
+    "h64_n64k": dict(rho=1 / 32, window=256, r=64),
 }
 
 
-def config_workload(idx: int, device="cpu", **overrides) -> Workload:
-    kw = dict(CONFIGS[idx])
+def config_workload(name: str, device="cpu", **overrides) -> Workload:
+    kw = dict(CONFIGS[name])
     kw.update(overrides)
-    window = CONFIG_PARAMS[idx]["window"]
+    window = CONFIG_PARAMS[name]["window"]
     return make_workload(device=device, planted_lo=0, planted_hi=max(0, kw["N"] - window), **kw)
 
 

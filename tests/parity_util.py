@@ -1,6 +1,6 @@
 """Helpers shared by the GPU parity tests: run a step through the C ABI and compare it with the oracle.
 
-Comparison rules (the benchmark spec's criteria, written out):
+Comparison rules (the path's correctness criteria, written out):
 
 * Selection: every head's set has exactly k + W + n_sink rows and contains the window and the sinks. Its
   archive part must equal the oracle's except for rows whose score lies within 1e-3 relative of the k-th

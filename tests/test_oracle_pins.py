@@ -385,7 +385,7 @@ def pin_two_tier_is_lse_merge():
 
 
 def pin_planted_rows_selected():
-    for idx_cfg, over in ((1, {}), (2, dict(N=2048, H=32))):
+    for idx_cfg, over in (("fp32_h16_n1k", {}), ("h128_n8k", dict(N=2048, H=32))):
         wl = datagen.config_workload(idx_cfg, **over)
         hi = oracle.HostInputs(wl)
         p = datagen.CONFIG_PARAMS[idx_cfg]

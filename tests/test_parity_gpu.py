@@ -63,8 +63,8 @@ def run_case(wl, *, rho, r=64, window=0, n_sink=0, trigger=0, z_eff=1.0, top_j=0
 
 
 # ------------------------------------------------------------------------------------------------ configs
-def test_config1_fp32():
-    wl = datagen.config_workload(1)
+def test_fp32_h16_n1k():
+    wl = datagen.config_workload("fp32_h16_n1k")
     res = run_case(wl, rho=1 / 8, window=64)
     for pos, h in zip(wl.planted_pos[0].tolist(), wl.planted_head.tolist()):
         assert pos in res["gpu"]["idx"][0, h].tolist()
@@ -73,35 +73,35 @@ def test_config1_fp32():
 
 @pytest.mark.parametrize("r", [4, 8, 16, 32, 64])
 @pytest.mark.parametrize("rho", [1 / 8, 1 / 32, 1 / 128])
-def test_config2_rho_r(rho, r):
-    wl = datagen.config_workload(2, device="cuda")
+def test_h128_n8k_rho_r(rho, r):
+    wl = datagen.config_workload("h128_n8k", device="cuda")
     res = run_case(wl, rho=rho, r=r, window=128)
     # tighter than the 2e-2 gate: the only rounding beyond fp32 accumulation is the bf16 softmax weight
     assert res["out"]["out_rel"] < 1e-2
 
 
 @pytest.mark.parametrize("rho", [1 / 32, 1 / 128])
-def test_config3_lognormal(rho):
-    wl = datagen.config_workload(3, device="cuda")
+def test_h64_n32k_lognormal(rho):
+    wl = datagen.config_workload("h64_n32k_lognormal", device="cuda")
     run_case(wl, rho=rho, window=256)
 
 
-def test_config4_two_tier():
-    wl = datagen.config_workload(4, device="cuda")
+def test_h128_n64k_two_tier():
+    wl = datagen.config_workload("h128_n64k_two_tier", device="cuda")
     res = run_case(wl, rho=1 / 32, window=256, trigger=1, z_eff=1.0, check_seqs=[0, wl.B - 1])
     assert res["fired"] > 0
 
 
 @pytest.mark.parametrize("r,z,top_j", [(16, 1.0, 0), (64, 1.0, 16), (8, 0.5, 0)])
 def test_two_tier_variants(r, z, top_j):
-    wl = datagen.config_workload(4, device="cuda", B=2, N=8192)
+    wl = datagen.config_workload("h128_n64k_two_tier", device="cuda", B=2, N=8192)
     res = run_case(wl, rho=1 / 32, r=r, window=256, trigger=1, z_eff=z, top_j=top_j)
     assert res["fired"] > 0
 
 
 @pytest.mark.parametrize("N", [16384, 65536, 131072])
 @pytest.mark.parametrize("B", [1, 8, 32, 64])
-def test_config5_sweep(N, B):
+def test_h64_sweep(N, B):
     wl = datagen.make_workload(B, 64, N, dtype="bf16", seed=1000 + 10 * B + N // 16384, n_planted=64,
                                planted_hi=N - 256, device="cuda")
     res = run_case(wl, rho=1 / 32, window=256, check_seqs=sorted({0, B - 1}))
@@ -165,7 +165,7 @@ def test_two_tier_sinks_and_capacity():
 
 # ------------------------------------------------------------------------------------------------ entry points
 def test_vk_score_matches_oracle():
-    wl = datagen.config_workload(2, device="cuda", N=3000, H=32)
+    wl = datagen.config_workload("h128_n8k", device="cuda", N=3000, H=32)
     hi = oracle.HostInputs(wl)
     for r in (64, 16):
         _, dig16, _, _ = oracle.build_index(hi, r)
@@ -247,7 +247,7 @@ def test_build_digest_matches_oracle():
 
 
 def test_deterministic_and_graph_capturable():
-    wl = datagen.config_workload(5, device="cuda", B=4, N=16384)
+    wl = datagen.config_workload("h64_n64k", device="cuda", B=4, N=16384)
     step = GpuStep(wl, rho=1 / 32, window=256)
     a = step.run()
     b = step.run()
