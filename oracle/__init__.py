@@ -25,7 +25,7 @@ D_LATENT, D_ROPE, PAGE = 512, 64, 64
 
 # Deliberate mistakes the "known-bad first" tests plant in the oracle (see vk_oracle.c).
 MUT_NONE, MUT_TIE_LARGER, MUT_DROP_WINDOW, MUT_SCALE_SQUARED = 0, 1, 2, 3
-MUT_ROT_TRANSPOSE, MUT_DROP_ROPE, MUT_TRIGGER_NO_Z = 4, 5, 6
+MUT_ROT_TRANSPOSE, MUT_DROP_ROPE, MUT_TRIGGER_NO_Z, MUT_SIGMA_ONE_SIDED = 4, 5, 6, 7
 
 
 def build(force: bool = False) -> str:
@@ -63,6 +63,9 @@ def lib():
         L.vko_trigger.argtypes = [VP, I32, P, D, D, I32, P, P, P, P, P, I32, P, I32, I32, I32, P, P]
         L.vko_decode_step.argtypes = [VP, D, I32, I32, I32, D, I32, D, I32, P, P, I32, P, P, P, P, P, P]
         L.vko_decode_step.restype = ctypes.c_int
+        L.vko_sigma.argtypes = [P, I64, I32, I32, P]
+        L.vko_sigma_select.argtypes = [P, I64, I32, I32, I64, P]
+        L.vko_sigma_select.restype = I64
         L.vko_set_mutation.argtypes = [ctypes.c_int]
         L.vko_num_threads.restype = ctypes.c_int
         del F
@@ -199,3 +202,27 @@ def decode_step(hi: HostInputs, *, rho: float, r: int = 64, window: int = 0, n_s
                                float(z_eff), int(top_j), _ptr(hi.rot), _ptr(dg), cap, _ptr(out), _ptr(lse),
                                _ptr(smax), _ptr(idx), _ptr(count), _ptr(kth))
     return dict(out=out, lse=lse, smax=smax, idx=idx, count=count, kth=kth, rc=int(rc))
+
+
+# ------------------------------------------------------------------------------------------------ sigma selector
+def sigma(branch: np.ndarray, T: int = 4096, kappa: int = 16) -> np.ndarray:
+    """Low-pass residual norms of the RoPE branch (Sec. 4.1, Eq. 3) over fixed blocks of T rows.
+
+    ``branch`` is [N, 64] (any float dtype; used in fp64). Returns sigma [N] in fp64; rows past the last whole
+    block (the open tail) get -1.
+    """
+    r = np.ascontiguousarray(np.asarray(branch, dtype=np.float64))
+    assert r.ndim == 2 and r.shape[1] == D_ROPE
+    out = np.empty(r.shape[0], dtype=np.float64)
+    lib().vko_sigma(_ptr(r), r.shape[0], int(T), int(kappa), _ptr(out))
+    return out
+
+
+def sigma_select(sig: np.ndarray, T: int, n_sink: int, m: int) -> np.ndarray:
+    """The sigma selector's attended set (Sec. 4.1): sinks, the open tail, and the top-m closed rows by sigma
+    (ties: the smaller position). Returns the ascending ids."""
+    s = np.ascontiguousarray(np.asarray(sig, dtype=np.float64))
+    out = np.empty(max(1, s.shape[0]), dtype=np.int32)
+    c = lib().vko_sigma_select(_ptr(s), s.shape[0], int(T), int(n_sink), int(m), _ptr(out))
+    return out[:c].copy()
+

@@ -43,6 +43,7 @@ enum {
   MUT_ROT_TRANSPOSE = 4,  /* the digest rotation is applied as O^T */
   MUT_DROP_ROPE = 5,      /* attention logits drop the RoPE summand */
   MUT_TRIGGER_NO_Z = 6,   /* trigger ignores the certificate term */
+  MUT_SIGMA_ONE_SIDED = 7, /* sigma's inverse DFT drops the factor 2 of the bins that stand for a conjugate pair */
 };
 static int g_mutation = MUT_NONE;
 void vko_set_mutation(int m) { g_mutation = m; }
@@ -364,6 +365,92 @@ int vko_decode_step(const vko_view* v, double rho, int32_t r, int32_t W, int32_t
   }
   free(a);
   return rc;
+}
+
+/* ---------------------------------------------------------------- sigma selector (Sec. 4.1, Eq. 3) */
+/* The query-independent ranking of the paper's tier 1. The branch vectors r_u (the 64 RoPE-branch columns of each
+   row, fp64, [N][64] row-major) are cut into fixed blocks of T rows; only whole blocks [jT, (j+1)T) are closed.
+   Within a closed block, for each of the 64 dims, the sequence-axis DFT X_k = sum_u r_u e^{-2 pi i k u / T} is kept
+   on bins 0 <= k < kappa (and k <= T/2, the one-sided spectrum of a real signal) and inverted:
+     low_u = (1/T) sum_{k kept} w_k (A_k cos(2 pi k u / T) + B_k sin(2 pi k u / T)),
+   A_k = sum_u r_u cos(2 pi k u / T), B_k = sum_u r_u sin(2 pi k u / T), w_0 = 1, w_{T/2} = 1 (T even), else w_k = 2
+   (bin k stands for itself and its conjugate T - k). sigma_u = || r_u - low_u ||_2 over the 64 dims. The sums are
+   written out (no FFT). Rows past the last closed block (the open tail) get sigma = -1. */
+void vko_sigma(const double* r, int64_t N, int32_t T, int32_t kappa, double* sigma) {
+  const int64_t nb = N / T;
+  int32_t nk = kappa < T / 2 + 1 ? kappa : T / 2 + 1;      /* kept bins */
+  if (nk < 0) nk = 0;
+  const double TWO_PI = 6.283185307179586476925286766559;
+  double* cs = (double*)malloc(sizeof(double) * (size_t)nk * (size_t)T);
+  double* sn = (double*)malloc(sizeof(double) * (size_t)nk * (size_t)T);
+  for (int32_t k = 0; k < nk; ++k)
+    for (int32_t u = 0; u < T; ++u) {
+      const double ang = TWO_PI * (double)(((int64_t)k * u) % T) / (double)T;   /* reduced exactly before cos/sin */
+      cs[(size_t)k * T + u] = cos(ang);
+      sn[(size_t)k * T + u] = sin(ang);
+    }
+  for (int64_t u = nb * (int64_t)T; u < N; ++u) sigma[u] = -1.0;
+#pragma omp parallel for schedule(static)
+  for (int64_t j = 0; j < nb; ++j) {
+    const double* rb = r + (size_t)j * T * D_ROPE;
+    double* res2 = (double*)calloc((size_t)T, sizeof(double));   /* squared residual per row */
+    double* low = (double*)malloc(sizeof(double) * (size_t)T);
+    for (int d = 0; d < D_ROPE; ++d) {
+      for (int32_t u = 0; u < T; ++u) low[u] = 0.0;
+      for (int32_t k = 0; k < nk; ++k) {
+        double A = 0.0, B = 0.0;
+        for (int32_t u = 0; u < T; ++u) {
+          const double x = rb[(size_t)u * D_ROPE + d];
+          A += x * cs[(size_t)k * T + u];
+          B += x * sn[(size_t)k * T + u];
+        }
+        double w = (k == 0 || 2 * k == T) ? 1.0 : 2.0;
+        if (g_mutation == MUT_SIGMA_ONE_SIDED) w = 1.0;
+        for (int32_t u = 0; u < T; ++u) low[u] += w * (A * cs[(size_t)k * T + u] + B * sn[(size_t)k * T + u]);
+      }
+      for (int32_t u = 0; u < T; ++u) {
+        const double e = rb[(size_t)u * D_ROPE + d] - low[u] / (double)T;
+        res2[u] += e * e;
+      }
+    }
+    for (int32_t u = 0; u < T; ++u) sigma[(size_t)j * T + u] = sqrt(res2[u]);
+    free(res2);
+    free(low);
+  }
+  free(cs);
+  free(sn);
+}
+
+/* The attended set of the sigma selector (Sec. 4.1): the sinks [0, n_sink), the open tail (rows past the last
+   closed block of T rows), and the m closed rows outside the sinks with the largest sigma (ties: the smaller
+   position). m is clamped to the number of such rows. Writes the ascending ids to out (room for N) and returns
+   their count. */
+static const double* g_sig;
+static int cmp_sigma(const void* x, const void* y) {
+  const int64_t a = *(const int64_t*)x, b = *(const int64_t*)y;
+  if (g_sig[a] > g_sig[b]) return -1;
+  if (g_sig[a] < g_sig[b]) return 1;
+  return (a > b) - (a < b);
+}
+int64_t vko_sigma_select(const double* sigma, int64_t N, int32_t T, int32_t n_sink, int64_t m, int32_t* out) {
+  const int64_t closed = (N / T) * (int64_t)T;
+  const int64_t lo = n_sink < closed ? n_sink : closed;
+  int64_t nc = closed - lo;
+  if (m > nc) m = nc;
+  if (m < 0) m = 0;
+  int64_t* ord = (int64_t*)malloc(sizeof(int64_t) * (size_t)(nc > 0 ? nc : 1));
+  for (int64_t i = 0; i < nc; ++i) ord[i] = lo + i;
+  g_sig = sigma;
+  qsort(ord, (size_t)nc, sizeof(int64_t), cmp_sigma);
+  unsigned char* keep = (unsigned char*)calloc((size_t)(N > 0 ? N : 1), 1);
+  for (int64_t i = 0; i < N; ++i) keep[i] = (i < n_sink || i >= closed) ? 1 : 0;
+  for (int64_t i = 0; i < m; ++i) keep[ord[i]] = 1;
+  int64_t c = 0;
+  for (int64_t i = 0; i < N; ++i)
+    if (keep[i]) out[c++] = (int32_t)i;
+  free(ord);
+  free(keep);
+  return c;
 }
 
 int vko_num_threads(void) {
