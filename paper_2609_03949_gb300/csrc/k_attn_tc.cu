@@ -28,7 +28,7 @@
 //                      (0 where the head did not select the row) in bf16 into shared memory (K-major, 128-byte
 //                      swizzle). m_h is a running max that only moves when a tile's max exceeds it by more than 32
 //                      (log2 units), so P stays <= 2^32 and a rescale is rare: the O^T issuer sees it in the tile's
-//                      published flags and has the four softmax warps scale the head's O^T column in tensor memory
+//                      published flags and has softmax warps 2..5 scale the head's O^T column in tensor memory
 //                      (each its quarter of the dims) before the tile's product; there is no per-tile sync of the
 //                      softmax warps otherwise. The exact max is tracked beside it, and at the end the head's sum
 //                      and output are re-based on it, so the partial carries the true max logit. At a segment's end
