@@ -432,7 +432,7 @@ cudaError_t launch_score_tc(const vk_view& v, int row_offset, int row_stride, in
   args.total_tiles = (int64_t)args.tiles_per_seq * v.B;
   args.n_pages = (v.N + PAGE - 1) / PAGE;
   args.tmem_cols = 512;
-  const int grid = (int)std::min<int64_t>(args.total_tiles, 152);
+  const int grid = (int)std::min<int64_t>(args.total_tiles, sm_count());   // persistent: one CTA per SM
   const int m = args.mode;
   auto go = [&](auto kernel, size_t smem, int g) -> cudaError_t {
     cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);

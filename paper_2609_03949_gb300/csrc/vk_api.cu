@@ -45,7 +45,6 @@ int cuda_fail(cudaError_t e, const char* where) {
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
 constexpr int64_t MAX_N = (1 << 24) - 1;
-constexpr int NUM_SMS_TARGET = 152;   // GB300 SMs: the attention's CTA count
 
 int check_view(const vk_view* v) {
   if (!v) return fail(VK_ERR_INVALID_ARG, "view is NULL");
@@ -108,21 +107,22 @@ int check_index(const vk_view* v, const vk_params* p, const vk_index* ix, bool n
 size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
 // Positions per attention split, a multiple of 64 (the attention tile). One attention CTA is resident per SM,
-// so the split count is chosen to fill the 152 SMs in whole waves: maximise (work) / (waves x 152 x positions
-// per CTA), preferring longer splits (fewer partials to merge) when two counts are equally good.
+// so the split count is chosen to fill the SMs in whole waves: maximise (work) / (waves x SMs x positions per
+// CTA), preferring longer splits (fewer partials to merge) when two counts are equally good.
 void choose_splits(const vk_view& v, int64_t* nsplit, int64_t* split_len) {
   const int64_t per_pos = (int64_t)v.B * ((v.H + vk::HG - 1) / vk::HG);
   const int64_t N = v.N;
   const int64_t lo = std::max<int64_t>(1, (N + 16383) / 16384);
   const int64_t hi = std::max<int64_t>(lo, std::min<int64_t>((N + 255) / 256, 2048));
+  const int64_t sms = vk::sm_count();
   double best = -1.0;
   int64_t best_len = ((N + 63) / 64) * 64;
   for (int64_t ns = lo; ns <= hi; ++ns) {
     const int64_t len = ((N + ns - 1) / ns + 63) / 64 * 64;
     const int64_t ns_eff = (N + len - 1) / len;
     const int64_t ctas = per_pos * ns_eff;
-    const int64_t waves = (ctas + NUM_SMS_TARGET - 1) / NUM_SMS_TARGET;
-    const double eff = (double)(per_pos * N) / ((double)waves * NUM_SMS_TARGET * len);
+    const int64_t waves = (ctas + sms - 1) / sms;
+    const double eff = (double)(per_pos * N) / ((double)waves * sms * len);
     if (eff > best + 1e-9) { best = eff; best_len = len; }
   }
   *split_len = best_len;
@@ -136,13 +136,29 @@ namespace vk {
 // tensor-core kernel, the split layout for the fp32 kernel. Persistent: one CTA per SM, but at least 4 tiles per
 // CTA -- a partial (64 heads x 512 fp32 = 128 KB) costs more traffic than a tile (72 KB), so small problems take
 // fewer, longer ranges.
+int sm_count() {
+  static int cached[64] = {0};
+  int dev = 0, n = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) {
+    cudaGetLastError();
+    return 152;
+  }
+  if (cached[dev] > 0) return cached[dev];
+  if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0) {
+    cudaGetLastError();
+    n = 152;
+  }
+  cached[dev] = n;
+  return n;
+}
+
 AttnGeom attn_geom(const vk_view& v) {
   AttnGeom g{};
   g.n_hg = (v.H + HG - 1) / HG;
   g.T = (v.N + 63) / 64;
   g.total = (long long)v.B * g.n_hg * g.T;
   if (attn_tc_supported(v)) {
-    g.G = (int)std::min<long long>(std::max<long long>(1, g.total / 4), NUM_SMS_TARGET);
+    g.G = (int)std::min<long long>(std::max<long long>(1, g.total / 4), sm_count());
     g.nslot = 1;
     for (long long s = 0; s < (long long)v.B * g.n_hg; ++s) g.nslot = std::max(g.nslot, attn_nvalid(g, s));
   } else {

@@ -131,6 +131,9 @@ cudaError_t launch_list_to_bitmap(int B, int H, int N, const int32_t* idx, const
                                   uint32_t* bitmap, int64_t nw, int* status, cudaStream_t st);
 size_t attn_smem_bytes(int dtype, int H, int split_len);
 bool attn_tc_supported(const vk_view& v);
+// SMs of the current device (152 on GB300; also the value used when it cannot be read): the persistent kernels'
+// CTA count, one per SM.
+int sm_count();
 AttnGeom attn_geom(const vk_view& v);
 cudaError_t launch_attn_tc(const vk_view& v, float lam, const uint32_t* bitmap, int64_t nw, const AttnGeom& g,
                            int slot0, int nslot, float* part_o, float* part_ml, uint32_t flags, int* status,
