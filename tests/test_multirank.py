@@ -42,7 +42,7 @@ def _rank_main(rank: int, world: int, port: int, out: dict) -> None:
 def test_two_ranks_host_logic():
     world = 2
     port = _free_port()
-    with mp.Manager() as mgr:
+    with mp.get_context("spawn").Manager() as mgr:    # no fork: the test process may already run threads
         out = mgr.dict()
         mp.start_processes(_rank_main, args=(world, port, out), nprocs=world, start_method="spawn", join=True)
         res = dict(out)
