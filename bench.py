@@ -5,8 +5,12 @@ sequence, rho = 1/32, r = 64, recent window 256, 64 planted rows per sequence, a
 decode sequences per GPU (weak scaling: every rank owns its own 64 sequences). Metric: decode query-tokens/s
 per layer (one query token per sequence per step).
 
-Prints one JSON line (rank 0). `python bench.py --impl reference` times the CPU oracle on the same workload
-instead (a bounded sample of sequences per step), on the host cores.
+Prints one JSON line (rank 0). `value` times the steps alone (device events on the launching stream); a second
+pass of the same steps records the library's stage events for the breakdown and the roofline of the dominant
+kernel. `e2e` runs the steps through the same entry point with each step's queries copied in from pinned host
+memory and its outputs copied back, on copy streams that overlap the neighbouring steps. `python bench.py --impl
+reference` times the CPU oracle on the same workload instead (a bounded sample of sequences per step), on the host
+cores.
 """
 from __future__ import annotations
 
