@@ -160,8 +160,9 @@ int vk_workspace_init(void* ws, size_t ws_bytes, void* stream);
  *     allocates nothing itself (no cudaMalloc, no allocating library routine).
  *   - Problems whose vk_workspace_bytes() exceeds VK_NOALLOC_SCRATCH_BYTES are rejected with
  *     VK_ERR_WORKSPACE; bad arguments are refused exactly as vk_decode_step refuses them.
- *   - The first call on each device looks up the array's device address (cudaGetSymbolAddress) and caches
- *     it; make that first call before any stream capture on that device.
+ *   - Every call looks up the array's device address on the current device (cudaGetSymbolAddress); the
+ *     first call on a device may also load the library's device code there, so make that first call before
+ *     any stream capture on that device.
  *   - Every call on a device shares the one array and it keeps the last call's contents; the call clears
  *     the status word it needs at zero. Calls that overlap on the GPU (other streams, other host threads,
  *     without ordering between them) race on the array and corrupt each other's results.

@@ -61,6 +61,8 @@ def lib():
         L.vko_select.argtypes = [I32, I32, I32, P, I64, I32, I32, I32, P, P, P]
         L.vko_attention.argtypes = [VP, D, P, P, I32, P, P, P]
         L.vko_trigger.argtypes = [VP, I32, P, D, D, I32, P, P, P, P, P, I32, P, I32, I32, I32, P, P]
+        L.vko_page_norms.argtypes = [VP, P, P]
+        L.vko_trigger_page.argtypes = [VP, D, D, I32, P, P, P, P, I32, P, I32, I32, I32, P, P]
         L.vko_decode_step.argtypes = [VP, D, I32, I32, I32, D, I32, D, I32, P, P, I32, P, P, P, P, P, P]
         L.vko_decode_step.restype = ctypes.c_int
         L.vko_sigma.argtypes = [P, I64, I32, I32, P]
@@ -182,10 +184,39 @@ def trigger(hi: HostInputs, r: int, lam: float, z_eff: float, top_j: int, a: np.
     return fidx, fcount
 
 
+def page_norms(hi: HostInputs):
+    """(page_knorm [B,P], page_eta [B,P]): per 64-row page the largest |K_u| (64 RoPE dims) and |L_u|."""
+    P = (hi.N + PAGE - 1) // PAGE
+    pk = np.zeros((hi.B, P), np.float64)
+    pe = np.zeros((hi.B, P), np.float64)
+    lib().vko_page_norms(ctypes.byref(hi.view), _ptr(pk), _ptr(pe))
+    return pk, pe
+
+
+def trigger_page(hi: HostInputs, lam: float, z_eff: float, top_j: int, page_knorm: np.ndarray,
+                 page_eta: np.ndarray, idx: np.ndarray, count: np.ndarray, smax: np.ndarray, window: int,
+                 n_sink: int = 0):
+    """(fired idx [B,H,N] int32, fired count [B,H]) of the page-level trigger (reading B): archived rows outside
+    S_h of every page whose bound lam (|qr| page_knorm + z_eff |qc| page_eta) beats s*_h."""
+    idx = np.ascontiguousarray(idx, dtype=np.int32)
+    count = np.ascontiguousarray(count, dtype=np.int32)
+    smax = np.ascontiguousarray(smax, dtype=np.float64)
+    pk = np.ascontiguousarray(page_knorm, dtype=np.float64)
+    pe = np.ascontiguousarray(page_eta, dtype=np.float64)
+    capf = hi.N
+    fidx = np.full((hi.B, hi.H, capf), -1, np.int32)
+    fcount = np.zeros((hi.B, hi.H), np.int32)
+    lib().vko_trigger_page(ctypes.byref(hi.view), float(lam), float(z_eff), int(top_j), _ptr(pk), _ptr(pe),
+                           _ptr(idx), _ptr(count), idx.shape[-1], _ptr(smax), window, n_sink, capf, _ptr(fidx),
+                           _ptr(fcount))
+    return fidx, fcount
+
+
 def decode_step(hi: HostInputs, *, rho: float, r: int = 64, window: int = 0, n_sink: int = 0,
                 sm_scale: float | None = None, trigger: int = 0, z_eff: float = 1.0, top_j: int = 0,
                 digest_bf16: np.ndarray | None = None, cap: int | None = None):
-    """Whole step. Returns dict(out, lse, smax, idx, count, kth, rc)."""
+    """Whole step (trigger: 0 off, 1 row-level reading A, 2 page-level reading B).
+    Returns dict(out, lse, smax, idx, count, kth, rc)."""
     lam = (1.0 / math.sqrt(192.0)) if sm_scale is None else float(sm_scale)
     if cap is None:
         cap = hi.N if trigger else max(1, keep_count(hi.N, rho, window, n_sink) + window + n_sink)

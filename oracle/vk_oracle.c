@@ -19,7 +19,8 @@
  *   - ties in the top-k go to the smaller position;
  *   - the trigger is row level: Eq. 4 with sketch rank 0 (the content summand is bounded by
  *     Cauchy-Schwarz with eta_u = |L_u|), plus a page-level bound on the RoPE dims that the width-r
- *     digest does not cover.
+ *     digest does not cover (reading A); reading B admits whole 64-row pages by a page-level bound on
+ *     both summands.
  */
 #include <math.h>
 #include <stdint.h>
@@ -325,10 +326,83 @@ void vko_trigger(const vko_view* v, int32_t r, const float* rot, double lam, dou
   }
 }
 
+/* ---------------------------------------------------------------- page-level trigger (reading B) */
+/* Per 64-row page P: the largest RoPE-key norm max_{u in P} |K_u| (all 64 stored dims) and the largest latent
+ * norm max_{u in P} eta_u = max |L_u|. Cauchy-Schwarz on both summands of the logit gives, for every row u of P
+ * and any query, s(u) = lambda (qc . L_u + qr . K_u) <= lambda (|qr| max_P |K_u| + |qc| max_P eta_u) (Lemma 2
+ * with the sketch rank 0, applied to the page's extreme norms instead of the row's own). */
+void vko_page_norms(const vko_view* v, double* page_knorm, double* page_eta) {
+  const int64_t N = v->N, P = (N + PAGE - 1) / PAGE;
+#pragma omp parallel for schedule(static)
+  for (int b = 0; b < v->B; ++b) {
+    for (int64_t p = 0; p < P; ++p) { page_knorm[(int64_t)b * P + p] = 0.0; page_eta[(int64_t)b * P + p] = 0.0; }
+    for (int64_t u = 0; u < N; ++u) {
+      double kk = 0.0, ll = 0.0;
+      for (int j = 0; j < D_ROPE; ++j) kk += K(v, b, u, j) * K(v, b, u, j);
+      for (int j = 0; j < D_LAT; ++j) ll += L(v, b, u, j) * L(v, b, u, j);
+      double* pk = &page_knorm[(int64_t)b * P + u / PAGE];
+      double* pe = &page_eta[(int64_t)b * P + u / PAGE];
+      if (sqrt(kk) > *pk) *pk = sqrt(kk);
+      if (sqrt(ll) > *pe) *pe = sqrt(ll);
+    }
+  }
+}
+
+/* Reading B of the recall trigger: a whole archived page is admitted when its page-level bound
+ *     Bp = lambda * (|qr_h| * page_knorm[P] + z_eff * |qc_h| * page_eta[P])
+ * beats s*_h; its archived rows outside S_h fire. With z_eff >= 1 this is sound (no row left out can beat s*).
+ * With top_j > 0 only the top_j fired rows by (Bp desc, position asc) are kept. Fired ids in ascending position. */
+void vko_trigger_page(const vko_view* v, double lam, double z_eff, int32_t top_j, const double* page_knorm,
+                      const double* page_eta, const int32_t* idx, const int32_t* count, int32_t cap,
+                      const double* smax, int32_t W, int32_t n_sink, int32_t capf, int32_t* fidx, int32_t* fcount) {
+  const int64_t N = v->N, P = (N + PAGE - 1) / PAGE;
+#pragma omp parallel for collapse(2) schedule(dynamic)
+  for (int b = 0; b < v->B; ++b) {
+    for (int h = 0; h < v->H; ++h) {
+      double qrn = 0.0, qcn = 0.0;
+      for (int j = 0; j < D_ROPE; ++j) qrn += QR(v, b, h, j) * QR(v, b, h, j);
+      for (int j = 0; j < D_LAT; ++j) qcn += QC(v, b, h, j) * QC(v, b, h, j);
+      qrn = sqrt(qrn);
+      qcn = sqrt(qcn);
+      double zz = (g_mutation == MUT_TRIGGER_NO_Z) ? 0.0 : z_eff;
+      char* in_set = (char*)calloc((size_t)N + 1, 1);
+      const int32_t* set = &idx[((int64_t)b * v->H + h) * cap];
+      int32_t n = count[b * v->H + h];
+      if (n > cap) n = cap;
+      for (int32_t i = 0; i < n; ++i) in_set[set[i]] = 1;
+      const double sstar = smax[b * v->H + h];
+      int64_t lo = n_sink, hi = N - W;
+      item* fired = (item*)malloc(sizeof(item) * (size_t)(hi > lo ? hi - lo : 1));
+      int64_t nf = 0;
+      for (int64_t u = lo; u < hi; ++u) {
+        if (in_set[u]) continue;
+        const int64_t pg = (int64_t)b * P + u / PAGE;
+        const double bound = lam * (qrn * page_knorm[pg] + zz * qcn * page_eta[pg]);
+        if (bound > sstar) { fired[nf].key = bound; fired[nf].u = (int32_t)u; ++nf; }
+      }
+      if (top_j > 0 && nf > top_j) {
+        qsort(fired, (size_t)nf, sizeof(item), by_key_desc_pos_asc);
+        nf = top_j;
+      }
+      char* mark = (char*)calloc((size_t)N + 1, 1);
+      for (int64_t i = 0; i < nf; ++i) mark[fired[i].u] = 1;
+      int32_t c = 0;
+      int32_t* out = &fidx[((int64_t)b * v->H + h) * capf];
+      for (int64_t u = 0; u < N; ++u)
+        if (mark[u]) { if (c < capf) out[c] = (int32_t)u; ++c; }
+      fcount[b * v->H + h] = c;
+      free(mark);
+      free(fired);
+      free(in_set);
+    }
+  }
+}
+
 /* ---------------------------------------------------------------- one decode step */
 /* Score -> select -> attend; in two-tier mode also index -> trigger -> attend over S u F, which equals
- * the LSE merge of the two partial softmaxes (Lemma 1). idx lists S_h (ascending) followed by F_h
- * (ascending); count = |S_h| + |F_h|. Returns 0, or -4 when a list does not fit in cap. */
+ * the LSE merge of the two partial softmaxes (Lemma 1). trigger: 0 off, 1 the row-level rule (reading A),
+ * 2 the page-level rule (reading B). idx lists S_h (ascending) followed by F_h (ascending);
+ * count = |S_h| + |F_h|. Returns 0, or -4 when a list does not fit in cap. */
 int vko_decode_step(const vko_view* v, double rho, int32_t r, int32_t W, int32_t n_sink, double lam,
                     int32_t trigger, double z_eff, int32_t top_j, const float* rot, const uint16_t* digest,
                     int32_t cap, double* out, double* lse, double* smax, int32_t* idx, int32_t* count,
@@ -349,7 +423,16 @@ int vko_decode_step(const vko_view* v, double rho, int32_t r, int32_t W, int32_t
     int32_t capf = (int32_t)N;
     int32_t* fidx = (int32_t*)malloc(sizeof(int32_t) * (size_t)(BH * capf));
     int32_t* fcount = (int32_t*)malloc(sizeof(int32_t) * (size_t)BH);
-    vko_trigger(v, r, rot, lam, z_eff, top_j, a, eta, pres, idx, count, cap, smax, W, n_sink, capf, fidx, fcount);
+    if (trigger == 2) {
+      double* pk = (double*)malloc(sizeof(double) * (size_t)(v->B * P));
+      double* pe = (double*)malloc(sizeof(double) * (size_t)(v->B * P));
+      vko_page_norms(v, pk, pe);
+      vko_trigger_page(v, lam, z_eff, top_j, pk, pe, idx, count, cap, smax, W, n_sink, capf, fidx, fcount);
+      free(pk);
+      free(pe);
+    } else {
+      vko_trigger(v, r, rot, lam, z_eff, top_j, a, eta, pres, idx, count, cap, smax, W, n_sink, capf, fidx, fcount);
+    }
     for (int64_t i = 0; i < BH; ++i) {
       int32_t* dst = &idx[i * cap];
       int32_t c = count[i];

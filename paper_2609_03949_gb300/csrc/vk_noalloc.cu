@@ -10,9 +10,10 @@
 // GPU (at the latest at this entry point's first call there) and keeps until the process exits. Its size is
 // VK_NOALLOC_SCRATCH_BYTES; problems whose workspace (vk_workspace_bytes) is larger are rejected.
 // Host code cannot use the array's name as a device address: the name is a host-side shadow. The device
-// address is looked up once per device with cudaGetSymbolAddress, with that device current, and cached.
+// address is looked up with cudaGetSymbolAddress on every call, with the caller's device current: the lookup is
+// cheap, and a cached address could outlive its module (after cudaDeviceReset the runtime loads the library's
+// code again, and the array may then sit elsewhere).
 #include <cstdio>
-#include <mutex>
 
 #include "vk_common.cuh"
 
@@ -20,24 +21,13 @@ namespace {
 
 static __device__ __align__(256) unsigned char g_noalloc_scratch[VK_NOALLOC_SCRATCH_BYTES];
 
-constexpr int kMaxDevices = 64;
-void* g_scratch_addr[kMaxDevices] = {};
-std::mutex g_scratch_mu;
-
-// Device address of g_noalloc_scratch on the current device (looked up on the first call per device).
+// Device address of g_noalloc_scratch on the current device, looked up afresh (the first lookup on a device
+// loads the library's device code there if that has not happened yet).
 cudaError_t scratch_address(void** out) {
-  int dev = 0;
-  cudaError_t e = cudaGetDevice(&dev);
+  void* p = nullptr;
+  const cudaError_t e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
   if (e != cudaSuccess) return e;
-  if (dev < 0 || dev >= kMaxDevices) return cudaErrorInvalidDevice;
-  std::lock_guard<std::mutex> lock(g_scratch_mu);
-  if (!g_scratch_addr[dev]) {
-    void* p = nullptr;
-    e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
-    if (e != cudaSuccess) return e;
-    g_scratch_addr[dev] = p;
-  }
-  *out = g_scratch_addr[dev];
+  *out = p;
   return cudaSuccess;
 }
 

@@ -337,6 +337,78 @@ def pin_trigger_top_j():
         assert fj[0, h, :cj[0, h]].tolist() == sorted(fired[order[:5]].tolist())
 
 
+def pin_page_norms():
+    # per 64-row page: the largest |K_u| over all 64 RoPE dims and the largest |L_u| (numpy norms, ragged tail)
+    hi, wl = small_random(B=2, N=150, dtype="bf16")
+    pk, pe = oracle.page_norms(hi)
+    kn = np.linalg.norm(f64(wl.rope), axis=-1)
+    ln = np.linalg.norm(f64(wl.latent), axis=-1)
+    for b in range(2):
+        for p in range(3):
+            assert pk[b, p] == pytest.approx(kn[b, p * 64:(p + 1) * 64].max(), rel=1e-14)
+            assert pe[b, p] == pytest.approx(ln[b, p * 64:(p + 1) * 64].max(), rel=1e-14)
+
+
+def _page_hand_case():
+    # four pages; page 3 is the recent window. Page p holds RoPE keys of norm <= p + 1 (largest on its last row)
+    # and latent rows of norm <= 0.5 (p + 1); qr = e_0 (|qr| = 1), |qc| = 2.
+    N, W = 256, 64
+    cache = np.zeros((1, N, 576))
+    for u in range(N):
+        p = u // 64
+        f = (u % 64 + 1) / 64.0
+        cache[0, u, 512 + 1] = (p + 1) * f            # K_u = (p + 1) f e_1: qr . K_u = 0, |K_u| = (p + 1) f
+        cache[0, u, 3] = 0.5 * (p + 1) * f            # |L_u| = 0.5 (p + 1) f
+    qc = np.zeros((1, 1, 512))
+    qc[0, 0, 7] = 2.0
+    qr = np.zeros((1, 1, 64))
+    qr[0, 0, 0] = 1.0
+    hi, wl = host(cache, qc, qr)
+    idx = np.arange(N - W, N, dtype=np.int32)[None, None, :]      # S = the window only
+    cnt = np.array([[W]], np.int32)
+    return hi, wl, idx, cnt, N, W
+
+
+def pin_page_trigger_hand():
+    # reading B: page p fires (all its archived rows outside S) iff lam (|qr| max|K| + z |qc| max eta) > s*
+    hi, wl, idx, cnt, N, W = _page_hand_case()
+    pk, pe = oracle.page_norms(hi)
+    for z in (1.0, 0.5):
+        bound = [LAM * ((p + 1) + z * 2.0 * 0.5 * (p + 1)) for p in range(3)]
+        for s_star, want_pages in ((bound[1] * (1 - 1e-9), (1, 2)), (bound[1] * (1 + 1e-9), (2,)),
+                                   (bound[0] * (1 - 1e-9), (0, 1, 2)), (bound[2] * (1 + 1e-9), ())):
+            fidx, fcnt = oracle.trigger_page(hi, LAM, z, 0, pk, pe, idx, cnt, np.array([[s_star]]), W)
+            want = [u for p in want_pages for u in range(64 * p, 64 * p + 64)]
+            assert fidx[0, 0, :fcnt[0, 0]].tolist() == want, (z, s_star)
+    # top_j: the highest page bound first, then the smaller position
+    fidx, fcnt = oracle.trigger_page(hi, LAM, 1.0, 70, pk, pe, idx, cnt, np.array([[0.0]]), W)
+    assert fidx[0, 0, :fcnt[0, 0]].tolist() == list(range(64, 70)) + list(range(128, 192))
+
+
+def pin_page_trigger_sound_and_contains_row_level():
+    # with z_eff = 1 no row left out of S u F beats s* (Lemma 2 on the page's extreme norms); at r = 64 every row
+    # the row-level rule fires also fires under the page rule (its trigger score is at most the page bound); z = 0
+    # reduces the bound to lam |qr| max|K|
+    hi, wl, a, eta, pres, idx, cnt, smax, fidx, fcnt, k = _trigger_case(64, 1.0)
+    pk, pe = oracle.page_norms(hi)
+    s = exact_logits(wl)[0]
+    qrn = np.linalg.norm(f64(wl.q_rope)[0], axis=1)
+    for z in (1.0, 0.3, 0.0):
+        fb, cb = oracle.trigger_page(hi, LAM, z, 0, pk, pe, idx, cnt, smax, 40)
+        fa, ca = oracle.trigger(hi, 64, LAM, z, 0, a, eta, pres, idx, cnt, smax, 40)
+        for h in range(wl.H):
+            S = set(idx[0, h, :cnt[0, h]].tolist())
+            FB = set(fb[0, h, :cb[0, h]].tolist())
+            assert FB.isdisjoint(S)
+            assert set(fa[0, h, :ca[0, h]].tolist()) <= FB
+            if z == 1.0:
+                out_rows = np.array(sorted(set(range(wl.N)) - S - FB), dtype=int)
+                assert np.all(s[h, out_rows] <= smax[0, h] + 1e-9)
+            if z == 0.0:
+                want = [u for u in range(0, wl.N - 40) if u not in S and LAM * qrn[h] * pk[0, u // 64] > smax[0, h]]
+                assert fb[0, h, :cb[0, h]].tolist() == want
+
+
 def pin_index_norms():
     hi, wl = small_random(B=2, N=150, dtype="bf16")
     for r in (8, 64):
@@ -399,7 +471,8 @@ PINS = [pin_keep_count, pin_scores_r64_matmul, pin_digest_orientation_permutatio
         pin_select_ramp, pin_select_all_equal_ties, pin_select_window_only, pin_select_bruteforce_lexsort,
         pin_select_count_invariant, pin_attention_dense_rho1, pin_attention_constant_rows,
         pin_attention_hull_and_permutation, pin_attention_single_row_and_uniform, pin_attention_leakage_bound,
-        pin_trigger_sound, pin_trigger_z0_and_monotone, pin_trigger_top_j, pin_index_norms, pin_bf16_rne,
+        pin_trigger_sound, pin_trigger_z0_and_monotone, pin_trigger_top_j, pin_page_norms, pin_page_trigger_hand,
+        pin_page_trigger_sound_and_contains_row_level, pin_index_norms, pin_bf16_rne,
         pin_two_tier_is_lse_merge, pin_planted_rows_selected]
 
 
@@ -419,6 +492,7 @@ def test_pin(pin):
     (oracle.MUT_ROT_TRANSPOSE, pin_digest_haar_matches_numpy),
     (oracle.MUT_DROP_ROPE, pin_attention_dense_rho1),
     (oracle.MUT_TRIGGER_NO_Z, pin_trigger_sound),
+    (oracle.MUT_TRIGGER_NO_Z, pin_page_trigger_hand),
 ])
 def test_planted_mistakes_are_caught(mutation, pin):
     oracle.set_mutation(mutation)
