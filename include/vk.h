@@ -16,6 +16,8 @@
  *   trigger (two-tier) F_h = { u in A \ S_h : lambda (a[h,u] + |(O Qr_h)[r:]| P_res[u/64]
  *           + z_eff |Qc_h| eta_u) > s*_h }, optionally the top_j of them (Eq. 4 with sketch rank 0,
  *           Lemma 2; the fetch of rows that beat the tier-1 max), attended too and merged by LSE.
+ *           Reading B admits whole 64-row pages instead: every archived row outside S_h of a page P with
+ *           lambda (|Qr_h| max_P |K_u| + z_eff |Qc_h| max_P eta_u) > s*_h (Lemma 2 on the page's extreme norms).
  *
  * Conventions
  *   - Every pointer in vk_view / vk_index and every output is DEVICE memory owned by the caller.
@@ -54,8 +56,13 @@ typedef enum {
 typedef enum { VK_BF16 = 0, VK_F32 = 1 } vk_dtype;
 
 typedef enum {
-  VK_TRIG_OFF = 0,  /* tier 1 only: the top-k plus window (plus sinks) */
-  VK_TRIG_CS = 1    /* two-tier: also fetch the archived rows whose Cauchy-Schwarz trigger score beats s* */
+  VK_TRIG_OFF = 0,     /* tier 1 only: the top-k plus window (plus sinks) */
+  VK_TRIG_CS = 1,      /* two-tier, row level (reading A): fetch the archived rows whose Cauchy-Schwarz trigger
+                          score (Eq. 4 with sketch rank 0) beats s* */
+  VK_TRIG_CS_PAGE = 2  /* two-tier, page level (reading B): fetch every archived row of each 64-row page whose
+                          page-level bound lambda (|Qr| max|K| + z_eff |Qc| max eta) beats s*; needs
+                          index->page_knorm and index->page_eta. With top_j, the top_j fired rows by (page bound
+                          desc, position asc) */
 } vk_trigger;
 
 /* The cache and the query of one decode step. */
@@ -91,6 +98,10 @@ typedef struct {
  * bounded waits expire after about a second, it reports VK_ERR_TIMEOUT in the device status word and every
  * role of that CTA winds down; vk_poll_status then returns VK_ERR_TIMEOUT. No other call uses it. */
 #define VK_FLAG_TEST_TIMEOUT 0x4u
+/* Turn off the page skip of the row-level trigger scan (for tests; the fired sets are the same either way).
+ * With index->page_knorm and index->page_eta given, the r = 64 scan of VK_TRIG_CS skips every 128-row tile in which
+ * no head's page bound lambda (|Qr_h| max|K| + z_eff |Qc_h| max eta) reaches s*_h: no row there can fire. */
+#define VK_FLAG_NO_PAGE_SKIP 0x8u
 
 /* The per-cache index built once by vk_build_digest (Sec. 4.2 index entry with sketch rank 0). */
 typedef struct {
@@ -98,6 +109,9 @@ typedef struct {
   const float* eta;         /* [B, N] |L_u|_2; needed only by the trigger */
   const float* page_res;    /* [B, ceil(N/64)] max over the page of |(O K_u)[r:64]| (0 when r = 64); trigger only */
   const float* rot;         /* [64, 64] row-major orthogonal O; NULL iff r = 64 */
+  const float* page_knorm;  /* [B, ceil(N/64)] max over the page of |K_u| (all 64 RoPE dims); VK_TRIG_CS_PAGE needs
+                               it, VK_TRIG_CS uses it for the page skip; may be NULL otherwise */
+  const float* page_eta;    /* [B, ceil(N/64)] max over the page of eta_u; with page_knorm */
 } vk_index;
 
 /* k = min(ceil(rho*N), N - W - n_sink): archived rows kept per head (-1 on bad arguments). */
@@ -111,10 +125,10 @@ int32_t vk_min_cap(const vk_view* view, const vk_params* params);
 size_t vk_workspace_bytes(const vk_view* view, const vk_params* params, int32_t cap);
 
 /* Index build (the compression-time work of Sec. 4.2): for every row, digest = bf16((O K_u)[0:r]) when
- * r < 64, eta_u = |L_u|_2, and per 64-row page the max of |(O K_u)[r:64]|. Any output may be NULL to skip
- * it. rot64: [64,64] row-major fp32 orthogonal matrix (device); may be NULL when r = 64. */
+ * r < 64, eta_u = |L_u|_2, and per 64-row page the max of |(O K_u)[r:64]|, of |K_u| and of eta_u. Any output
+ * may be NULL to skip it. rot64: [64,64] row-major fp32 orthogonal matrix (device); may be NULL when r = 64. */
 int vk_build_digest(const vk_view* view, const vk_params* params, const float* rot64, void* digest, float* eta,
-                    float* page_res, void* stream);
+                    float* page_res, float* page_knorm, float* page_eta, void* stream);
 
 /* Score every cached row: scores[b,h,u] = a[h,u] (unscaled) as fp32, [B, H, N] contiguous. The RoPE columns
  * are read when r = 64, the index's digest otherwise. ws holds the rotated queries. */
@@ -135,8 +149,8 @@ int vk_select(const vk_view* view, const vk_params* params, const float* scores,
 int vk_sparse_attn(const vk_view* view, const vk_params* params, const int32_t* idx, const int32_t* count,
                    int32_t cap, float* out, float* lse, float* smax, void* ws, size_t ws_bytes, void* stream);
 
-/* The whole step: score, select, attend, and with params->trigger = VK_TRIG_CS also the trigger scan, the
- * attention over the fired rows and the LSE merge. out [B,H,512], lse [B,H]; smax [B,H] (s* of the tier-1
+/* The whole step: score, select, attend, and with params->trigger = VK_TRIG_CS (or VK_TRIG_CS_PAGE) also the
+ * trigger scan (or the page-bound test), the attention over the fired rows and the LSE merge. out [B,H,512], lse [B,H]; smax [B,H] (s* of the tier-1
  * set; may be NULL). idx[b,h,:] lists S_h (ascending) followed by F_h (ascending) and count[b,h] is
  * |S_h| + |F_h|; fired rows that do not fit in cap are still attended (out/lse stay exact) but are left
  * out of the list, and VK_ERR_CAPACITY is raised in the device status. index may be NULL when r = 64

@@ -18,6 +18,10 @@
 //                                shared memory and only its set bits are visited,
 //                        mode 2  trigger: T = lambda (a + |(O Qr)[r:]| page_res + z |Qc| eta) > s*_h for archive
 //                                rows outside S_h -> 32-row words of the fired bitmap (or candidates for top_j).
+//                                With the page norm maxima given, a tile in which no head's page bound can reach
+//                                s*_h (page_may_fire) is skipped: the producer warp decides per tile, loads nothing
+//                                and tells the MMA issuer to issue nothing; the epilogue, applying the same test per
+//                                head and page, writes empty words without reading the accumulator.
 // Every mbarrier wait is bounded; a wait that gives up raises VK_ERR_TIMEOUT and the CTA winds down.
 #include <cuda.h>
 #include <cudaTypedefs.h>
@@ -105,6 +109,15 @@ __device__ __forceinline__ void tmem_ld_chunk(uint32_t taddr, float* v) {
   }
 }
 
+// Whether a row of a 64-row page can fire for a head: its trigger score lambda (a + z |Qc| eta_u) is at most the page
+// bound lambda (|Qr| max|K_u| + z |Qc| max eta_u) (Cauchy-Schwarz, a = Qr . K_u); the bound is inflated by 2^-10 so
+// that the fp32 rounding of the scores and norms cannot turn a skip into a missed row. Rounded operations are
+// explicit so that the producer and the epilogue reach the same decision bit for bit.
+__device__ __forceinline__ bool page_may_fire(float lam, float qrf, float zqc, float sstar, float pk, float pe) {
+  const float bound = __fmul_rn(__fmul_rn(lam, __fadd_rn(__fmul_rn(qrf, pk), __fmul_rn(zqc, pe))), 1.0f + 0x1p-10f);
+  return !(bound <= sstar);
+}
+
 // Bits of the rows [lo, hi) within the 32 rows starting at r0.
 __device__ __forceinline__ uint32_t range_mask(int r0, int lo, int hi) {
   const int a = max(lo - r0, 0), e = min(hi - r0, 32);
@@ -147,6 +160,8 @@ __global__ void __launch_bounds__((2 + 4 * (4 / NHG)) * 32, 1) k_score_tc(const 
   uint64_t* d_empty = d_full + G;                        // [G]
   __shared__ uint32_t tmem_base;
   __shared__ int abort_flag;
+  __shared__ int skip_stage[TC_STAGES];                  // mode 2 page skip: the ring stage's tile was not loaded
+  const bool page_skip = MODE == 2 && args.page_knorm != nullptr;
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int64_t total = args.total_tiles;
@@ -171,7 +186,69 @@ __global__ void __launch_bounds__((2 + 4 * (4 / NHG)) * 32, 1) k_score_tc(const 
   __syncthreads();
   tmem_fence_after();
 
-  if (warp == 0) {
+  if (warp == 0 && page_skip) {
+    // ------------------------------------------------------------------ TMA producer with the page skip
+    // The whole warp walks the tiles: lane l holds heads l + 32 j (their |Qr|, z |Qc| and s*), the tile is skipped
+    // when no head may fire on either of its two pages; lane 0 issues the copies.
+    constexpr int NJ = NHG * MH / 32;
+    float hq[NJ], hz[NJ], hs[NJ];
+    bool ok = n > 0;
+    int prev_b = -1, b = b_first, kt = kt_first;
+    for (int i = 0; i < n && ok; ++i, kt = kt + 1 == tps ? (++b, 0) : kt + 1) {
+      const int row0 = kt * TC_M;
+      bool lok = true;
+      if (b != prev_b) {
+        if (lane == 0) {
+          const int qi = (b - b_first) & 1, quse = (b - b_first) >> 1;
+          if (quse > 0 && !mbar_wait(&q_empty[qi], (quse - 1) & 1, &abort_flag)) {
+            lok = false;
+          } else {
+            mbar_arrive_expect_tx(&q_full[qi], (uint32_t)H * 128u);
+            tma_load_2d(sq + qi * L::qbuf, &qmap, 0, b * H, &q_full[qi]);
+          }
+        }
+#pragma unroll
+        for (int j = 0; j < NJ; ++j) {
+          const int hh = lane + 32 * j;
+          hq[j] = hz[j] = 0.f;
+          hs[j] = INFINITY;                              // a head past H never fires
+          if (hh < H) {
+            const int64_t bh = (int64_t)b * H + hh;
+            hq[j] = args.qrf[bh];
+            hz[j] = args.qcn[bh] * args.z;
+            hs[j] = args.smax1[bh];
+          }
+        }
+        prev_b = b;
+      }
+      const int64_t pg = (int64_t)b * args.n_pages + row0 / PAGE;
+      const bool two = row0 + PAGE < args.n_rows;
+      const float pk0 = args.page_knorm[pg], pe0 = args.page_eta[pg];
+      const float pk1 = two ? args.page_knorm[pg + 1] : 0.f, pe1 = two ? args.page_eta[pg + 1] : 0.f;
+      bool may = false;
+#pragma unroll
+      for (int j = 0; j < NJ; ++j)
+        may = may || page_may_fire(args.lam, hq[j], hz[j], hs[j], pk0, pe0) ||
+              (two && page_may_fire(args.lam, hq[j], hz[j], hs[j], pk1, pe1));
+      const bool skip = !__any_sync(0xffffffffu, may);
+      if (lane == 0 && lok) {
+        const int s = i % TC_STAGES, use = i / TC_STAGES;
+        if ((use > 0 && !mbar_wait(&a_empty[s], (use - 1) & 1, &abort_flag)) || abort_flag) {
+          lok = false;
+        } else {
+          skip_stage[s] = skip ? 1 : 0;                  // published by the arrive below (release)
+          if (skip) {
+            mbar_arrive(&a_full[s]);
+          } else {
+            mbar_arrive_expect_tx(&a_full[s], TC_TILE_BYTES);
+            tma_load_3d(sa + s * TC_TILE_BYTES, &kmap, 0, row0, b, &a_full[s]);
+          }
+        }
+      }
+      ok = __shfl_sync(0xffffffffu, lok, 0);
+    }
+    if (n > 0 && !ok && lane == 0) abort_flag = 1;
+  } else if (warp == 0) {
     // ------------------------------------------------------------------ TMA producer
     if (lane == 0 && n > 0) {
       int prev_b = -1, b = b_first, kt = kt_first;
@@ -209,12 +286,14 @@ __global__ void __launch_bounds__((2 + 4 * (4 / NHG)) * 32, 1) k_score_tc(const 
         tmem_fence_after();                              // the epilogue's reads of this accumulator came first
         const uint64_t bd = sw128_desc(smem_addr(sa + s * TC_TILE_BYTES));
         const uint64_t ad = sw128_desc(smem_addr(sq + qi * L::qbuf));
+        if (!(page_skip && skip_stage[s])) {             // a skipped tile: no product (the epilogue ignores it)
 #pragma unroll
-        for (int hg = 0; hg < NHG; ++hg)
+          for (int hg = 0; hg < NHG; ++hg)
 #pragma unroll
-          for (int k = 0; k < 4; ++k)
-            mma_bf16(tmem_base + ds * DCOLS + hg * TC_M, ad + (uint64_t)((hg * MH * 128 + 32 * k) >> 4),
-                     bd + (uint64_t)((32 * k) >> 4), idesc, k > 0 ? 1u : 0u);
+            for (int k = 0; k < 4; ++k)
+              mma_bf16(tmem_base + ds * DCOLS + hg * TC_M, ad + (uint64_t)((hg * MH * 128 + 32 * k) >> 4),
+                       bd + (uint64_t)((32 * k) >> 4), idesc, k > 0 ? 1u : 0u);
+        }
         mma_commit(&a_empty[s]);
         mma_commit(&d_full[ds]);
         const bool last_of_seq = (i + 1 == n) || kt + 1 == tps;
@@ -229,7 +308,7 @@ __global__ void __launch_bounds__((2 + 4 * (4 / NHG)) * 32, 1) k_score_tc(const 
     constexpr int NC = MH == 128 ? 4 : 2;                 // 32-row chunks per thread and tile
     float* my_stg = stg + (ew * 32 + lane) * 32;          // this thread's staging row (128 B, 16-byte swizzled)
     int prev_b = -1;
-    float th[NHG], p1[NHG], p2[NHG];                      // per head: theta, or (s*, |(O Qr)[r:]|, z |Qc|)
+    float th[NHG], p1[NHG], p2[NHG], p3[NHG];             // per head: theta, or (s*, |(O Qr)[r:]|, z |Qc|, |Qr|)
     int b = b_first, kt = kt_first + g;
     for (int i = g; i < n; i += G, kt += G) {
       while (kt >= tps) { kt -= tps; ++b; }
@@ -238,7 +317,7 @@ __global__ void __launch_bounds__((2 + 4 * (4 / NHG)) * 32, 1) k_score_tc(const 
 #pragma unroll
         for (int hg = 0; hg < NHG; ++hg) {
           const int hh = hg * 128 + (MH == 128 ? 32 * quarter + lane : 16 * quarter + (lane & 15));
-          th[hg] = p1[hg] = p2[hg] = 0.f;
+          th[hg] = p1[hg] = p2[hg] = p3[hg] = 0.f;
           if (hh < H) {
             const int64_t bh = (int64_t)b * H + hh;
             if (MODE == 1) th[hg] = args.theta[bh];
@@ -246,6 +325,7 @@ __global__ void __launch_bounds__((2 + 4 * (4 / NHG)) * 32, 1) k_score_tc(const 
               th[hg] = args.smax1[bh];
               p1[hg] = args.qrn[bh];
               p2[hg] = args.qcn[bh] * args.z;
+              if (page_skip) p3[hg] = args.qrf[bh];
             }
           }
         }
@@ -314,18 +394,26 @@ __global__ void __launch_bounds__((2 + 4 * (4 / NHG)) * 32, 1) k_score_tc(const 
           } else {
             const int64_t word = rc >> 5;
             const bool word_ok = valid && word < args.nw && rc < args.n_rows;
-            const uint32_t sel = word_ok ? args.selbm[bh * args.nw + word] : 0xffffffffu;
-            const float pr = rc < args.n_rows ? args.page_res[(int64_t)b * args.n_pages + rc / PAGE] : 0.f;
-            const float add = p1[hg] * pr;
-            const float* eta = args.eta + (int64_t)b * args.N + rc;
+            // the page test is the producer's, per head: where it fails no row can fire (and a tile that every
+            // head fails was skipped, its accumulator stale)
+            const bool may = !page_skip || (rc < args.n_rows &&
+                             page_may_fire(args.lam, p3[hg], p2[hg], th[hg],
+                                           args.page_knorm[(int64_t)b * args.n_pages + rc / PAGE],
+                                           args.page_eta[(int64_t)b * args.n_pages + rc / PAGE]));
+            if (may) {
+              const uint32_t sel = word_ok ? args.selbm[bh * args.nw + word] : 0xffffffffu;
+              const float pr = rc < args.n_rows ? args.page_res[(int64_t)b * args.n_pages + rc / PAGE] : 0.f;
+              const float add = p1[hg] * pr;
+              const float* eta = args.eta + (int64_t)b * args.N + rc;
 #pragma unroll
-            for (int k = 0; k < 32; ++k) {
-              const float e = rc + k < args.n_rows ? eta[k] : 0.f;
-              const float T = args.lam * (v[k] + add + p2[hg] * e);
-              v[k] = T;
-              m |= (T > th[hg] ? 1u : 0u) << k;
+              for (int k = 0; k < 32; ++k) {
+                const float e = rc + k < args.n_rows ? eta[k] : 0.f;
+                const float T = args.lam * (v[k] + add + p2[hg] * e);
+                v[k] = T;
+                m |= (T > th[hg] ? 1u : 0u) << k;
+              }
+              m &= range_mask(rc, args.arch_lo, min(args.arch_hi, args.n_rows)) & ~sel;
             }
-            m &= range_mask(rc, args.arch_lo, min(args.arch_hi, args.n_rows)) & ~sel;
             if (!word_ok) m = 0u;
             if (!emit && word_ok) args.firebm[bh * args.nw + word] = m;
           }

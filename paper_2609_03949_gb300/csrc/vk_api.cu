@@ -84,10 +84,11 @@ int check_params(const vk_view* v, const vk_params* p) {
   if (p->n_sink < 0 || p->n_sink > v->N - p->window)
     return fail(VK_ERR_INVALID_ARG, "n_sink = %d is outside [0, N - window]", p->n_sink);
   if (!(p->sm_scale > 0.f) || !std::isfinite(p->sm_scale)) return fail(VK_ERR_INVALID_ARG, "sm_scale must be finite and > 0");
-  if (p->trigger != VK_TRIG_OFF && p->trigger != VK_TRIG_CS) return fail(VK_ERR_INVALID_ARG, "trigger = %d is unknown", p->trigger);
+  if (p->trigger != VK_TRIG_OFF && p->trigger != VK_TRIG_CS && p->trigger != VK_TRIG_CS_PAGE)
+    return fail(VK_ERR_INVALID_ARG, "trigger = %d is unknown", p->trigger);
   if (!(p->z_eff >= 0.f) || !std::isfinite(p->z_eff)) return fail(VK_ERR_INVALID_ARG, "z_eff must be finite and >= 0");
   if (p->top_j < 0) return fail(VK_ERR_INVALID_ARG, "top_j must be >= 0");
-  if (p->flags & ~(VK_FLAG_FORCE_FALLBACK | VK_FLAG_FORCE_DENSE | VK_FLAG_TEST_TIMEOUT))
+  if (p->flags & ~(VK_FLAG_FORCE_FALLBACK | VK_FLAG_FORCE_DENSE | VK_FLAG_TEST_TIMEOUT | VK_FLAG_NO_PAGE_SKIP))
     return fail(VK_ERR_INVALID_ARG, "unknown flags 0x%x", p->flags);
   return VK_OK;
 }
@@ -97,8 +98,14 @@ int check_index(const vk_view* v, const vk_params* p, const vk_index* ix, bool n
     if (!ix || !ix->digest || !ix->rot) return fail(VK_ERR_INVALID_ARG, "r < 64 needs index->digest and index->rot");
     if (!aligned16(ix->digest) || !aligned16(ix->rot)) return fail(VK_ERR_INVALID_ARG, "index pointers must be 16-byte aligned");
   }
-  if (need_trigger) {
+  if (need_trigger && p->trigger == VK_TRIG_CS) {
     if (!ix || !ix->eta || !ix->page_res) return fail(VK_ERR_INVALID_ARG, "the trigger needs index->eta and index->page_res");
+    if ((ix->page_knorm == nullptr) != (ix->page_eta == nullptr))
+      return fail(VK_ERR_INVALID_ARG, "index->page_knorm and index->page_eta go together");
+  }
+  if (need_trigger && p->trigger == VK_TRIG_CS_PAGE) {
+    if (!ix || !ix->page_knorm || !ix->page_eta)
+      return fail(VK_ERR_INVALID_ARG, "the page trigger needs index->page_knorm and index->page_eta");
   }
   (void)v;
   return VK_OK;
@@ -205,7 +212,8 @@ VkLayout make_layout(const vk_view& v, const vk_params& p) {
   const int64_t lo = p.n_sink, hi = (int64_t)v.N - p.window;
   const int64_t k = keep_count(v.N, p.rho, p.window, p.n_sink);
   if (L.fused) fused_params(v.N, lo, hi, k, &L);
-  L.fcap = (L.fused && L.two_tier && p.top_j > 0) ? std::max<int64_t>(1, hi - lo) : 0;
+  const bool page_trig = p.trigger == VK_TRIG_CS_PAGE;
+  L.fcap = ((L.fused || page_trig) && L.two_tier && p.top_j > 0) ? std::max<int64_t>(1, hi - lo) : 0;
   const int64_t BH = (int64_t)v.B * v.H;
   const int64_t nslot = (int64_t)L.ag.nslot * (L.two_tier ? 2 : 1);
   size_t off = 0;
@@ -214,6 +222,7 @@ VkLayout make_layout(const vk_view& v, const vk_params& p) {
   L.off_qt = take(sizeof(float) * BH * vk::D_ROPE);
   L.off_qcn = take(sizeof(float) * BH);
   L.off_qrn = take(sizeof(float) * BH);
+  L.off_qrf = take(sizeof(float) * BH);
   L.off_smax1 = take(sizeof(float) * BH);
   L.off_nfired = take(sizeof(int64_t) * BH);
   L.off_scores = take(L.dense_scores ? sizeof(float) * BH * v.N : 0);
@@ -287,16 +296,18 @@ size_t vk_workspace_bytes(const vk_view* view, const vk_params* params, int32_t 
 }
 
 int vk_build_digest(const vk_view* view, const vk_params* params, const float* rot64, void* digest, float* eta,
-                    float* page_res, void* stream) {
+                    float* page_res, float* page_knorm, float* page_eta, void* stream) {
   g_err[0] = 0;
   int rc;
   if ((rc = check_view(view)) != VK_OK || (rc = check_params(view, params)) != VK_OK) return rc;
   if (params->r < vk::D_ROPE && (digest || page_res) && !rot64)
     return fail(VK_ERR_INVALID_ARG, "r < 64 needs rot64 for the digest and page_res");
-  if ((digest && !aligned16(digest)) || (eta && !aligned16(eta)) || (page_res && !aligned16(page_res)))
+  if ((digest && !aligned16(digest)) || (eta && !aligned16(eta)) || (page_res && !aligned16(page_res)) ||
+      (page_knorm && !aligned16(page_knorm)) || (page_eta && !aligned16(page_eta)))
     return fail(VK_ERR_INVALID_ARG, "outputs must be 16-byte aligned");
   cudaStream_t st = static_cast<cudaStream_t>(stream);
-  VK_CUDA(vk::launch_build_digest(*view, params->r, rot64, static_cast<__nv_bfloat16*>(digest), eta, page_res, st),
+  VK_CUDA(vk::launch_build_digest(*view, params->r, rot64, static_cast<__nv_bfloat16*>(digest), eta, page_res,
+                                  page_knorm, page_eta, st),
           "build_digest");
   return VK_OK;
 }
@@ -330,7 +341,7 @@ int vk_score(const vk_view* view, const vk_params* params, const vk_index* index
     return VK_OK;
   }
   VK_CUDA(vk::launch_qprep(*view, params->r, index ? index->rot : nullptr, qt, at<float>(ws, L.off_qcn),
-                           at<float>(ws, L.off_qrn), st), "qprep");
+                           at<float>(ws, L.off_qrn), at<float>(ws, L.off_qrf), st), "qprep");
   VK_CUDA(vk::launch_score_simt(*view, params->r, qt,
                                 static_cast<const __nv_bfloat16*>(index ? index->digest : nullptr), scores, st),
           "score");
@@ -400,6 +411,7 @@ int vk_decode_step(const vk_view* view, const vk_params* params, const vk_index*
   float* qt = at<float>(ws, L.off_qt);
   float* qcn = at<float>(ws, L.off_qcn);
   float* qrn = at<float>(ws, L.off_qrn);
+  float* qrf = at<float>(ws, L.off_qrf);
   float* scores = at<float>(ws, L.off_scores);
   uint32_t* selbm = at<uint32_t>(ws, L.off_selbm);
   float* po = at<float>(ws, L.off_part_o);
@@ -411,7 +423,7 @@ int vk_decode_step(const vk_view* view, const vk_params* params, const vk_index*
   // the query prep feeds the materialised-score path and the trigger; the fused path at r = 64 scores with the
   // RoPE query as it is (its exact fallback reads it directly)
   const bool qprep = !L.fused || two_tier;
-  if (qprep) VK_CUDA(vk::launch_qprep(v, params->r, index ? index->rot : nullptr, qt, qcn, qrn, st), "qprep");
+  if (qprep) VK_CUDA(vk::launch_qprep(v, params->r, index ? index->rot : nullptr, qt, qcn, qrn, qrf, st), "qprep");
   prof(1, st);
   if (L.fused) {
     // threshold from a strided sample, then one scoring pass that keeps only the rows above it
@@ -470,7 +482,20 @@ int vk_decode_step(const vk_view* view, const vk_params* params, const vk_index*
     int64_t* nfired = at<int64_t>(ws, L.off_nfired);
     uint32_t* firebm = at<uint32_t>(ws, L.off_firebm);
     VK_CUDA(vk::launch_smax_reduce(B, H, L.ag, nslot, pml, smax1, st), "smax");
-    if (L.fused) {
+    if (params->trigger == VK_TRIG_CS_PAGE) {
+      // reading B: whole pages by their page-level bound (no scan of the scores)
+      int* fcnt = params->top_j > 0 ? at<int>(ws, L.off_fcnt) : nullptr;
+      int2* fcand = params->top_j > 0 ? at<int2>(ws, L.off_fcand) : nullptr;
+      VK_CUDA(vk::launch_trigger_page(B, H, N, W, S, params->sm_scale, params->z_eff, qcn, qrf, index->page_knorm,
+                                      index->page_eta, smax1, selbm, firebm, L.nw, params->top_j, fcnt, fcand,
+                                      (int)L.fcap, st), "page trigger");
+      if (params->top_j > 0) {
+        VK_CUDA(vk::launch_select_cand(B, H, N, lo, hi, params->top_j, nullptr, fcnt, fcand, (int)L.fcap, 0, v, qt, idx,
+                                       count, cap, 1, nullptr, firebm, L.nw, status, st), "top_j");
+      } else {
+        VK_CUDA(vk::launch_bitmap_to_list(B, H, N, firebm, L.nw, idx, count, cap, status, st), "fired list");
+      }
+    } else if (L.fused) {
       vk::ScoreTcArgs t{};
       t.mode = 2;
       t.arch_lo = lo;
@@ -487,6 +512,11 @@ int vk_decode_step(const vk_view* view, const vk_params* params, const vk_index*
       t.nw = L.nw;
       t.top_j = params->top_j;
       t.status = status;
+      if (index->page_knorm && !(params->flags & VK_FLAG_NO_PAGE_SKIP)) {
+        t.qrf = qrf;
+        t.page_knorm = index->page_knorm;
+        t.page_eta = index->page_eta;
+      }
       if (params->top_j > 0) {
         int* fcnt = at<int>(ws, L.off_fcnt);
         int2* fcand = at<int2>(ws, L.off_fcand);

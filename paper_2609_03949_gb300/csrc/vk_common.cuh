@@ -108,8 +108,8 @@ struct VkLayout {
   bool fused;                   // threshold-candidate selection (no materialised scores)
   int64_t ss, soff, ns, j;      // fused: sample stride, offset, rows per sequence, order statistic for theta
   int64_t capc;                 // fused: candidate capacity per head
-  int64_t fcap;                 // two-tier top_j on the fused path: fired-candidate capacity per head
-  size_t off_status, off_qt, off_qcn, off_qrn, off_smax1, off_nfired, off_scores, off_selbm, off_firebm,
+  int64_t fcap;                 // two-tier top_j (fused path or page trigger): fired-candidate capacity per head
+  size_t off_status, off_qt, off_qcn, off_qrn, off_qrf, off_smax1, off_nfired, off_scores, off_selbm, off_firebm,
       off_part_o, off_part_ml, off_sample, off_theta, off_ccnt, off_cand, off_fcnt, off_fcand, total;
 };
 
@@ -117,7 +117,7 @@ struct VkLayout {
 // Every launcher enqueues on `st`, counts its kernel launches and returns cudaGetLastError().
 namespace vk {
 void count_launches(int n);
-cudaError_t launch_qprep(const vk_view& v, int r, const float* rot, float* qt, float* qcn, float* qrn,
+cudaError_t launch_qprep(const vk_view& v, int r, const float* rot, float* qt, float* qcn, float* qrn, float* qrf,
                          cudaStream_t st);
 cudaError_t launch_score_simt(const vk_view& v, int r, const float* qt, const __nv_bfloat16* digest,
                               float* scores, cudaStream_t st);
@@ -126,7 +126,11 @@ cudaError_t launch_select_dense(int B, int H, int N, const float* scores, const 
                                 int append_from_count, float* kth, uint32_t* bitmap, int64_t nw, int* status,
                                 cudaStream_t st);
 cudaError_t launch_build_digest(const vk_view& v, int r, const float* rot, __nv_bfloat16* digest, float* eta,
-                                float* page_res, cudaStream_t st);
+                                float* page_res, float* page_knorm, float* page_eta, cudaStream_t st);
+cudaError_t launch_trigger_page(int B, int H, int N, int W, int n_sink, float lam, float z_eff, const float* qcn,
+                                const float* qrf, const float* page_knorm, const float* page_eta, const float* smax1,
+                                const uint32_t* selbm, uint32_t* firebm, int64_t nw, int top_j, int* fcnt,
+                                int2* fcand, int fcap, cudaStream_t st);
 cudaError_t launch_list_to_bitmap(int B, int H, int N, const int32_t* idx, const int32_t* count, int cap,
                                   uint32_t* bitmap, int64_t nw, int* status, cudaStream_t st);
 size_t attn_smem_bytes(int dtype, int H, int split_len);

@@ -30,6 +30,9 @@ struct ScoreTcArgs {
   uint32_t* firebm;
   int64_t nw;
   int top_j;
+  // mode 2 page skip (when page_knorm != NULL): a 128-row tile is neither loaded nor multiplied when, for every head
+  // and both of its pages, lam * (qrf * page_knorm + z * qcn * page_eta) cannot reach smax1 (page_may_fire)
+  const float *qrf, *page_knorm, *page_eta;
   int* status;
 };
 

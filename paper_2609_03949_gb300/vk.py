@@ -17,8 +17,8 @@ LIB_PATH = os.path.join(_HERE, "libvk.so")
 VK_OK, VK_ERR_INVALID_ARG, VK_ERR_UNSUPPORTED, VK_ERR_WORKSPACE = 0, -1, -2, -3
 VK_ERR_CAPACITY, VK_ERR_CUDA, VK_ERR_TIMEOUT = -4, -5, -6
 VK_BF16, VK_F32 = 0, 1
-VK_TRIG_OFF, VK_TRIG_CS = 0, 1
-VK_FLAG_FORCE_FALLBACK, VK_FLAG_FORCE_DENSE, VK_FLAG_TEST_TIMEOUT = 0x1, 0x2, 0x4
+VK_TRIG_OFF, VK_TRIG_CS, VK_TRIG_CS_PAGE = 0, 1, 2
+VK_FLAG_FORCE_FALLBACK, VK_FLAG_FORCE_DENSE, VK_FLAG_TEST_TIMEOUT, VK_FLAG_NO_PAGE_SKIP = 0x1, 0x2, 0x4, 0x8
 D_LATENT, D_ROPE, PAGE = 512, 64, 64
 DEFAULT_SM_SCALE = 1.0 / math.sqrt(192.0)
 
@@ -44,7 +44,7 @@ class vk_params(ctypes.Structure):
 
 class vk_index(ctypes.Structure):
     _fields_ = [("digest", ctypes.c_void_p), ("eta", ctypes.c_void_p), ("page_res", ctypes.c_void_p),
-                ("rot", ctypes.c_void_p)]
+                ("rot", ctypes.c_void_p), ("page_knorm", ctypes.c_void_p), ("page_eta", ctypes.c_void_p)]
 
 
 _lib = None
@@ -63,7 +63,7 @@ def lib():
             "vk_keep_count": ([I32, D, I32, I32], I64),
             "vk_min_cap": ([VP, PP], I32),
             "vk_workspace_bytes": ([VP, PP, I32], SZ),
-            "vk_build_digest": ([VP, PP, P, P, P, P, P], ctypes.c_int),
+            "vk_build_digest": ([VP, PP, P, P, P, P, P, P, P], ctypes.c_int),
             "vk_score": ([VP, PP, IP, P, P, SZ, P], ctypes.c_int),
             "vk_select": ([VP, PP, P, P, P, P, I32, P, SZ, P], ctypes.c_int),
             "vk_sparse_attn": ([VP, PP, P, P, I32, P, P, P, P, SZ, P], ctypes.c_int),
@@ -135,8 +135,9 @@ def make_params(rho: float, r: int = 64, window: int = 0, n_sink: int = 0, sm_sc
                      top_j=top_j, flags=flags)
 
 
-def make_index(digest=None, eta=None, page_res=None, rot=None) -> vk_index:
-    return vk_index(digest=_ptr(digest), eta=_ptr(eta), page_res=_ptr(page_res), rot=_ptr(rot))
+def make_index(digest=None, eta=None, page_res=None, rot=None, page_knorm=None, page_eta=None) -> vk_index:
+    return vk_index(digest=_ptr(digest), eta=_ptr(eta), page_res=_ptr(page_res), rot=_ptr(rot),
+                    page_knorm=_ptr(page_knorm), page_eta=_ptr(page_eta))
 
 
 # ------------------------------------------------------------------------------------------------ entry points
@@ -159,9 +160,10 @@ def vk_workspace_init(ws: torch.Tensor, stream=None) -> None:
     _check(lib().vk_workspace_init(_ptr(ws), ws.numel() * ws.element_size(), _stream(stream)))
 
 
-def vk_build_digest(view, params, rot, digest=None, eta=None, page_res=None, stream=None) -> None:
+def vk_build_digest(view, params, rot, digest=None, eta=None, page_res=None, page_knorm=None, page_eta=None,
+                    stream=None) -> None:
     _check(lib().vk_build_digest(ctypes.byref(view), ctypes.byref(params), _ptr(rot), _ptr(digest), _ptr(eta),
-                                 _ptr(page_res), _stream(stream)))
+                                 _ptr(page_res), _ptr(page_knorm), _ptr(page_eta), _stream(stream)))
 
 
 def vk_score(view, params, index: vk_index | None, scores: torch.Tensor, ws: torch.Tensor, stream=None) -> None:

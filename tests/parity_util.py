@@ -46,13 +46,17 @@ class GpuStep:
         self.rot = self.wl.rot.contiguous()
         self.eta = torch.empty(B, N, dtype=torch.float32, device="cuda")
         self.page_res = torch.empty(B, P, dtype=torch.float32, device="cuda")
+        self.page_knorm = torch.empty(B, P, dtype=torch.float32, device="cuda")
+        self.page_eta = torch.empty(B, P, dtype=torch.float32, device="cuda")
         self.digest = None
         if r < 64:
             # the oracle's bf16 digest feeds both sides, so the scores are compared on identical inputs
             assert digest_bf16 is not None
             self.digest = torch.from_numpy(digest_bf16.astype(np.int16)).view(torch.bfloat16).cuda().contiguous()
-        vk.vk_build_digest(self.view, self.params, self.rot, None, self.eta, self.page_res)
-        self.index = vk.make_index(self.digest, self.eta, self.page_res, self.rot if r < 64 else None)
+        vk.vk_build_digest(self.view, self.params, self.rot, None, self.eta, self.page_res, self.page_knorm,
+                           self.page_eta)
+        self.index = vk.make_index(self.digest, self.eta, self.page_res, self.rot if r < 64 else None,
+                                   self.page_knorm, self.page_eta)
         self.buf = vk.DecodeBuffers(self.view, self.params, cap=cap)
 
     def run(self):
@@ -171,3 +175,50 @@ def check_fired(a, eta, pres, wl, lam, z_eff, r, smax_ref, S_idx, S_cnt, gF, W, 
     return swaps
 
 
+
+
+def check_fired_page(hi, wl, lam, z_eff, smax_ref, S_idx, S_cnt, gF, W, n_sink, top_j=0):
+    """Fired sets of the page-level trigger (reading B) vs the oracle's rule: the archived rows outside S_h of every
+    page with lam (|qr| max|K| + z_eff |qc| max eta) > s*. Exact outside the tie band around s* (and, with top_j,
+    around the top_j-th page bound); inside a band the GPU's choice must still be valid. Returns the band swaps."""
+    pk, pe = oracle.page_norms(hi)
+    B, H, N = wl.B, wl.H, wl.N
+    qrn = np.linalg.norm(wl.q_rope.double().cpu().numpy(), axis=-1)
+    qcn = np.linalg.norm(wl.q_latent.double().cpu().numpy(), axis=-1)
+    swaps = 0
+    for b in range(B):
+        for h in range(H):
+            inS = np.zeros(N, bool)
+            inS[S_idx[b, h, :S_cnt[b, h]]] = True
+            u = np.arange(n_sink, N - W)
+            u = u[~inS[u]]
+            Bp = lam * (qrn[b, h] * pk[b, u // 64] + z_eff * qcn[b, h] * pe[b, u // 64])
+            Bmap = dict(zip(u.tolist(), Bp.tolist()))
+            s = float(smax_ref[b, h])
+            eps_s = band(s, np.array([s]))
+            got = list(gF[b][h])
+            assert got == sorted(set(got)), "fired ids must be ascending and distinct"
+            for x in got:
+                assert x in Bmap, f"b={b} h={h}: fired row {x} is not an unselected archive row"
+                assert Bmap[x] > s - eps_s, f"b={b} h={h} u={x}: page bound below s* - band"
+            fired = u[Bp > s]
+            if top_j == 0 or len(fired) <= top_j:
+                diff = set(fired.tolist()).symmetric_difference(got)
+                for x in diff:
+                    assert abs(Bmap[x] - s) <= eps_s, f"b={b} h={h} u={x}: bound {Bmap[x]} s*={s} outside the band"
+                swaps += len(diff)
+                continue
+            assert len(got) == top_j, (b, h, len(got), top_j)
+            Bf = np.sort(Bp[Bp > s])[::-1]
+            thr = float(Bf[top_j - 1])
+            eps_t = band(thr, Bf)
+            gotset = set(got)
+            for x in got:
+                assert Bmap[x] >= thr - eps_t, f"b={b} h={h} u={x}: kept below the top_j cut"
+            for x in fired.tolist():
+                if x not in gotset:
+                    assert Bmap[x] <= thr + eps_t, f"b={b} h={h} u={x}: dropped above the top_j cut"
+            # among rows of equal page bound the smaller positions are kept
+            strict = [x for x in got if Bmap[x] > thr + eps_t]
+            assert len(strict) <= top_j
+    return swaps

@@ -113,6 +113,12 @@ def test_cap_workspace_and_index_are_checked(vk):
     assert call_decode(vk, v, vk.make_params(1 / 8, window=16, trigger=1)) == vk.VK_ERR_INVALID_ARG
     idx = vk.make_index(eta=FAKE, page_res=None)
     assert call_decode(vk, v, vk.make_params(1 / 8, window=16, trigger=1), index=idx) == vk.VK_ERR_INVALID_ARG
+    # the page skip's two page arrays go together; the page trigger needs both
+    idx = vk.make_index(eta=FAKE, page_res=FAKE, page_knorm=FAKE)
+    assert call_decode(vk, v, vk.make_params(1 / 8, window=16, trigger=1), index=idx) == vk.VK_ERR_INVALID_ARG
+    idx = vk.make_index(eta=FAKE, page_res=FAKE, page_eta=FAKE)
+    assert call_decode(vk, v, vk.make_params(1 / 8, window=16, trigger=2), index=idx) == vk.VK_ERR_INVALID_ARG
+    assert call_decode(vk, v, vk.make_params(1 / 8, window=16, trigger=3)) == vk.VK_ERR_INVALID_ARG
     assert call_decode(vk, v, p, out=FAKE + 4) == vk.VK_ERR_INVALID_ARG
 
 
@@ -124,6 +130,8 @@ def test_other_entry_points_refuse(vk):
     assert L.vk_sparse_attn(ctypes.byref(v), ctypes.byref(p), FAKE, FAKE, 10, FAKE, None, None, None, 0,
                             None) == vk.VK_ERR_WORKSPACE
     assert L.vk_build_digest(ctypes.byref(v), ctypes.byref(vk.make_params(1 / 8, r=8)), None, FAKE, None, None,
+                             None, None, None) == vk.VK_ERR_INVALID_ARG
+    assert L.vk_build_digest(ctypes.byref(v), ctypes.byref(p), None, None, None, None, FAKE + 4, None,
                              None) == vk.VK_ERR_INVALID_ARG
     assert L.vk_poll_status(None, None) == vk.VK_ERR_WORKSPACE
     assert L.vk_workspace_init(None, 0, None) == vk.VK_ERR_WORKSPACE

@@ -14,7 +14,7 @@ import oracle
 from paper_2609_03949_gb300 import datagen
 from paper_2609_03949_gb300 import vk
 
-from parity_util import GpuStep, check_fired, check_outputs, check_selection
+from parity_util import GpuStep, check_fired, check_fired_page, check_outputs, check_selection
 
 pytestmark = pytest.mark.gpu
 LAM = vk.DEFAULT_SM_SCALE
@@ -55,8 +55,12 @@ def run_case(wl, *, rho, r=64, window=0, n_sink=0, trigger=0, z_eff=1.0, top_j=0
     np.testing.assert_allclose(g["smax"], smax_ref, rtol=1e-4, atol=1e-4)
     _, _, eta, pres = oracle.build_index(hi, r)
     gF = [[g["idx"][b, h, nS:g["count"][b, h]].tolist() for h in range(wl.H)] for b in range(len(seqs))]
-    res["swaps"] = check_fired(a, eta, pres, sub, LAM, z_eff, r, smax_ref, g["idx"], np.full_like(g["count"], nS), gF,
-                               window, n_sink, top_j)
+    if trigger == vk.VK_TRIG_CS_PAGE:
+        res["swaps"] = check_fired_page(hi, sub, LAM, z_eff, smax_ref, g["idx"], np.full_like(g["count"], nS), gF,
+                                        window, n_sink, top_j)
+    else:
+        res["swaps"] = check_fired(a, eta, pres, sub, LAM, z_eff, r, smax_ref, g["idx"], np.full_like(g["count"], nS),
+                                   gF, window, n_sink, top_j)
     res["out"] = check_outputs(hi, LAM, g)
     res["fired"] = int((g["count"] - nS).sum())
     return res
@@ -97,6 +101,60 @@ def test_two_tier_variants(r, z, top_j):
     wl = datagen.config_workload("h128_n64k_two_tier", device="cuda", B=2, N=8192)
     res = run_case(wl, rho=1 / 32, r=r, window=256, trigger=1, z_eff=z, top_j=top_j)
     assert res["fired"] > 0
+
+
+@pytest.mark.parametrize("top_j,z", [(0, 1.0), (0, 0.05), (40, 0.05)])
+def test_h128_n64k_page_trigger(top_j, z):
+    # reading B at config 4's shape (two sequences checked): whole pages admitted by their page-level bound. With the
+    # sound z_eff = 1 nearly every page fires on this data; z_eff = 0.05 leaves a mix of fired and quiet pages.
+    wl = datagen.config_workload("h128_n64k_two_tier", device="cuda")
+    res = run_case(wl, rho=1 / 32, window=256, trigger=vk.VK_TRIG_CS_PAGE, z_eff=z, top_j=top_j,
+                   check_seqs=[0, wl.B - 1])
+    assert res["fired"] > 0
+
+
+@pytest.mark.parametrize("r,top_j", [(64, 0), (16, 0), (64, 7)])
+def test_page_trigger_variants(r, top_j):
+    wl = datagen.config_workload("h128_n64k_two_tier", device="cuda", B=2, N=8192)
+    res = run_case(wl, rho=1 / 32, r=r, window=256, n_sink=3, trigger=vk.VK_TRIG_CS_PAGE, z_eff=0.05, top_j=top_j)
+    assert res["fired"] > 0
+
+
+def _skippable_workload():
+    # every head finds a strong row in its recent window (K = 4.5 Qr_h / |Qr_h|, so s*_h >~ 4.5 |Qr_h| lambda), while the
+    # RoPE keys of rows 1024 .. 5119 are scaled by 1/40: on those pages no head's bound can reach s*, so the r = 64
+    # trigger scan skips their tiles
+    wl = datagen.make_workload(2, 64, 8192, seed=51, n_planted=0, device="cuda")
+    wl.cache[:, 1024:5120, 512:] = (wl.cache[:, 1024:5120, 512:].float() / 40).to(wl.cache.dtype)
+    for b in range(wl.B):
+        for h in range(64):
+            qr = wl.q_rope[b, h].float()
+            wl.cache[b, 8192 - 1 - h, 512:] = (4.5 * qr / qr.norm()).to(wl.cache.dtype)
+    return wl
+
+
+@pytest.mark.parametrize("top_j", [0, 5])
+def test_page_skip_keeps_fired_sets(top_j):
+    # the sound page skip of the row-level scan changes cost, not results: with and without it the fired sets and
+    # outputs are identical, and both meet the oracle
+    wl = _skippable_workload()
+    hi = oracle.HostInputs(wl)
+    pk, pe = oracle.page_norms(hi)
+    qrn = np.linalg.norm(wl.q_rope.double().cpu().numpy(), axis=-1)
+    qcn = np.linalg.norm(wl.q_latent.double().cpu().numpy(), axis=-1)
+    res = run_case(wl, rho=1 / 32, window=256, trigger=vk.VK_TRIG_CS, z_eff=0.25, top_j=top_j)
+    # the workload really has tiles that every head skips: both pages of the tile stay below every head's s*
+    smax = res["gpu"]["smax"]
+    bound = LAM * (qrn[:, :, None] * pk[:, None, :] + 0.25 * qcn[:, :, None] * pe[:, None, :])   # [B,H,P]
+    quiet = np.all(bound * (1 + 2.0 ** -10) <= smax[:, :, None], axis=1)                        # [B,P]
+    tile_quiet = quiet[:, 0::2] & quiet[:, 1::2]
+    assert tile_quiet.sum() >= 20, tile_quiet.sum()
+    on = GpuStep(wl, rho=1 / 32, window=256, trigger=vk.VK_TRIG_CS, z_eff=0.25, top_j=top_j).run()
+    off = GpuStep(wl, rho=1 / 32, window=256, trigger=vk.VK_TRIG_CS, z_eff=0.25, top_j=top_j,
+                  flags=vk.VK_FLAG_NO_PAGE_SKIP).run()
+    for key in ("idx", "count", "out", "lse"):
+        np.testing.assert_array_equal(on[key], off[key])
+    assert on["status"] == vk.VK_OK and off["status"] == vk.VK_OK
 
 
 @pytest.mark.parametrize("N", [16384, 65536, 131072])
