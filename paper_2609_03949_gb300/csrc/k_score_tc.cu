@@ -34,9 +34,6 @@
 
 namespace vk {
 
-constexpr int TC_M = 128;                        // rows per tile (MMA N)
-constexpr int TC_STAGES = 7;
-constexpr uint32_t TC_TILE_BYTES = TC_M * 128;   // 128 rows x 64 bf16
 
 __device__ __forceinline__ void tma_load_3d(void* dst, const CUtensorMap* map, int x, int y, int z, uint64_t* bar) {
   asm volatile(
@@ -126,25 +123,45 @@ __device__ __forceinline__ uint32_t range_mask(int r0, int lo, int hi) {
   return upto & ~((1u << a) - 1u);
 }
 
-// Shared memory from a 1024-aligned base: the ring, two query buffers of NHG x MH rows, G x 128 staging rows of
-// 128 B (modes 1, 2), barriers.
-template <int MH, int NHG>
-struct TcSmem {
-  static constexpr int G = 4 / NHG;
-  static constexpr uint32_t a = 0;
-  static constexpr uint32_t q = a + TC_STAGES * TC_TILE_BYTES;
+// One configuration of the kernel: TM rows per tile (the MMA's N: 64 or 128), G epilogue groups of WPQ warps per
+// tensor-memory lane quarter (a tile's 32-row chunks of a head are split among them), NACC accumulators of
+// NHG x TM tensor-memory columns (all 512 columns), a ring of STAGES tiles (96 to 112 KB). Shared memory from a
+// 1024-aligned base: the ring, two query buffers of NHG x MH rows, 128 B of staging per epilogue thread (modes 1,
+// 2), barriers.
+template <int MH, int NHG, int TM_, int G_, int WPQ_ = 1>
+struct TcCfg {
+  static constexpr int TM = TM_;
+  static constexpr int G = G_;
+  static constexpr int WPQ = WPQ_;
+  static constexpr uint32_t DCOLS = NHG * TM;            // columns per accumulator
+  static constexpr int NACC = 512 / DCOLS;
+  static constexpr uint32_t TILE = TM * 128;             // TM rows x 64 bf16
+  static constexpr int NC = MH == 128 ? TM / 32 : TM / 64;   // 32-row chunks per lane and tile
+  static constexpr int NCT = NC / WPQ;                   // of which one epilogue thread takes
+  static constexpr int EW = 4 * G * WPQ;                 // epilogue warps
+  static constexpr int THREADS = (2 + EW) * 32;
   static constexpr uint32_t qbuf = NHG * MH * 128;
+  static constexpr uint32_t STG = EW * 32 * 128;
+  // as many ring stages (up to 7 of 16 KB, or 14 of 8 KB) as fit beside the queries and the staging rows
+  static constexpr int STAGES_FIT = (int)((224u * 1024u - 2 * qbuf - STG) / TILE);
+  static constexpr int STAGES = STAGES_FIT < (TM == 128 ? 7 : 14) ? STAGES_FIT : (TM == 128 ? 7 : 14);
+  static constexpr uint32_t a = 0;
+  static constexpr uint32_t q = a + STAGES * TILE;
   static constexpr uint32_t stg = q + 2 * qbuf;
-  static constexpr uint32_t bars = stg + G * 128 * 128;
-  static constexpr uint32_t total = bars + (2 * TC_STAGES + 4 + 2 * G) * 8 + 1024;
+  static constexpr uint32_t bars = stg + STG;
+  static constexpr uint32_t total = bars + (2 * STAGES + 4 + 2 * NACC) * 8 + 1024;
+  static_assert(G <= NACC, "every epilogue group needs an accumulator of its own");
+  static_assert(NC % WPQ == 0 && STAGES >= 4, "configuration");
+  static_assert(total <= 232448, "scoring shared memory exceeds the 227 KB opt-in limit");
 };
 
-template <int MH, int NHG, int MODE>
-__global__ void __launch_bounds__((2 + 4 * (4 / NHG)) * 32, 1) k_score_tc(const __grid_constant__ CUtensorMap kmap,
-                                                                        const __grid_constant__ CUtensorMap qmap,
-                                                                        const ScoreTcArgs args) {
-  constexpr int G = 4 / NHG;
-  using L = TcSmem<MH, NHG>;
+template <int MH, int NHG, int MODE, int TM_, int G_, int WPQ_>
+__global__ void __launch_bounds__(TcCfg<MH, NHG, TM_, G_, WPQ_>::THREADS, 1)
+    k_score_tc(const __grid_constant__ CUtensorMap kmap, const __grid_constant__ CUtensorMap qmap,
+               const ScoreTcArgs args) {
+  using L = TcCfg<MH, NHG, TM_, G_, WPQ_>;
+  constexpr int G = L::G, TC_M = L::TM, TC_STAGES = L::STAGES, NACC = L::NACC;
+  constexpr uint32_t TC_TILE_BYTES = L::TILE;
   extern __shared__ __align__(1024) unsigned char smem_raw[];
   unsigned char* smem = reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   const int H = args.H;
@@ -156,8 +173,8 @@ __global__ void __launch_bounds__((2 + 4 * (4 / NHG)) * 32, 1) k_score_tc(const 
   uint64_t* a_empty = bars + TC_STAGES;
   uint64_t* q_full = bars + 2 * TC_STAGES;              // [2]
   uint64_t* q_empty = q_full + 2;                        // [2]
-  uint64_t* d_full = q_empty + 2;                        // [G]
-  uint64_t* d_empty = d_full + G;                        // [G]
+  uint64_t* d_full = q_empty + 2;                        // [NACC]
+  uint64_t* d_empty = d_full + NACC;                     // [NACC]
   __shared__ uint32_t tmem_base;
   __shared__ int abort_flag;
   __shared__ int skip_stage[TC_STAGES];                  // mode 2 page skip: the ring stage's tile was not loaded
@@ -172,13 +189,13 @@ __global__ void __launch_bounds__((2 + 4 * (4 / NHG)) * 32, 1) k_score_tc(const 
   const int kt_first = (int)(t0 - (int64_t)b_first * tps);
   // (sequence, tile within it) of the range's tiles, stepped without divisions: a 64-bit division per tile on
   // the producer's or the MMA issuer's thread is slower than the tile's whole TMA + MMA work
-  constexpr uint32_t DCOLS = NHG * TC_M;                 // columns per accumulator
+  constexpr uint32_t DCOLS = L::DCOLS;
 
   if (threadIdx.x == 0) {
     abort_flag = 0;
     for (int s = 0; s < TC_STAGES; ++s) { mbar_init(&a_full[s], 1); mbar_init(&a_empty[s], 1); }
     for (int i = 0; i < 2; ++i) { mbar_init(&q_full[i], 1); mbar_init(&q_empty[i], 1); }
-    for (int i = 0; i < G; ++i) { mbar_init(&d_full[i], 1); mbar_init(&d_empty[i], 4); }
+    for (int i = 0; i < NACC; ++i) { mbar_init(&d_full[i], 1); mbar_init(&d_empty[i], 4 * L::WPQ); }
     mbar_fence_init();
   }
   if (warp == 1) tmem_alloc(&tmem_base, 512);
@@ -222,7 +239,7 @@ __global__ void __launch_bounds__((2 + 4 * (4 / NHG)) * 32, 1) k_score_tc(const 
         prev_b = b;
       }
       const int64_t pg = (int64_t)b * args.n_pages + row0 / PAGE;
-      const bool two = row0 + PAGE < args.n_rows;
+      const bool two = TC_M > PAGE && row0 + PAGE < args.n_rows;
       const float pk0 = args.page_knorm[pg], pe0 = args.page_eta[pg];
       const float pk1 = two ? args.page_knorm[pg + 1] : 0.f, pe1 = two ? args.page_eta[pg + 1] : 0.f;
       bool may = false;
@@ -280,7 +297,7 @@ __global__ void __launch_bounds__((2 + 4 * (4 / NHG)) * 32, 1) k_score_tc(const 
           prev_b = b;
         }
         const int s = i % TC_STAGES, use = i / TC_STAGES;
-        const int ds = i % G, duse = i / G;
+        const int ds = i % NACC, duse = i / NACC;
         if (!mbar_wait(&a_full[s], use & 1, &abort_flag)) { abort_flag = 1; break; }
         if (duse > 0 && !mbar_wait(&d_empty[ds], (duse - 1) & 1, &abort_flag)) { abort_flag = 1; break; }
         tmem_fence_after();                              // the epilogue's reads of this accumulator came first
@@ -302,10 +319,11 @@ __global__ void __launch_bounds__((2 + 4 * (4 / NHG)) * 32, 1) k_score_tc(const 
     }
   } else {
     // ------------------------------------------------------------------ epilogue
-    const int ew = warp - 2;                              // 0 .. 4G-1
-    const int g = ew >> 2;                                // group: tiles i = g (mod G), accumulator g
+    const int ew = warp - 2;                              // 0 .. EW-1
+    const int g = ew / (4 * L::WPQ);                      // group: tiles i = g (mod G), accumulator i mod NACC
+    const int sub = (ew % (4 * L::WPQ)) >> 2;             // which of the group's warps on this lane quarter
     const int quarter = warp & 3;                         // TMEM lane quarter this warp may read
-    constexpr int NC = MH == 128 ? 4 : 2;                 // 32-row chunks per thread and tile
+    constexpr int NCT = L::NCT;                           // 32-row chunks per thread and tile: sub + WPQ j
     float* my_stg = stg + (ew * 32 + lane) * 32;          // this thread's staging row (128 B, 16-byte swizzled)
     int prev_b = -1;
     float th[NHG], p1[NHG], p2[NHG], p3[NHG];             // per head: theta, or (s*, |(O Qr)[r:]|, z |Qc|, |Qr|)
@@ -331,8 +349,8 @@ __global__ void __launch_bounds__((2 + 4 * (4 / NHG)) * 32, 1) k_score_tc(const 
         }
         prev_b = b;
       }
-      const int duse = i / G;
-      if (!mbar_wait(&d_full[g], duse & 1, &abort_flag)) {
+      const int ds = i % NACC, duse = i / NACC;
+      if (!mbar_wait(&d_full[ds], duse & 1, &abort_flag)) {
         if (lane == 0) { raise_status(args.status, VK_ERR_TIMEOUT); abort_flag = 1; }
         break;
       }
@@ -342,12 +360,14 @@ __global__ void __launch_bounds__((2 + 4 * (4 / NHG)) * 32, 1) k_score_tc(const 
         const int hh = hg * 128 + (MH == 128 ? 32 * quarter + lane : 16 * quarter + (lane & 15));
         const bool valid = hh < H;
         const int64_t bh = (int64_t)b * H + hh;
-        const uint32_t taddr = tmem_base + ((uint32_t)(32 * quarter) << 16) + g * DCOLS + hg * TC_M;
+        const uint32_t taddr = tmem_base + ((uint32_t)(32 * quarter) << 16) + ds * DCOLS + hg * TC_M;
         const bool emit = MODE == 1 || (MODE == 2 && args.top_j > 0);
-        uint32_t msk[NC];
+        uint32_t msk[NCT];
+        float keep[NCT == 1 ? 32 : 1];                    // one chunk per thread: its values, kept for the emission
         int cnt = 0;
 #pragma unroll
-        for (int c = 0; c < NC; ++c) {
+        for (int j = 0; j < NCT; ++j) {
+          const int c = sub + L::WPQ * j;
           float v[32];
           tmem_ld_chunk<MH>(taddr + (MH == 128 ? 32 * c : 64 * c), v);
           tmem_wait_ld();
@@ -417,20 +437,30 @@ __global__ void __launch_bounds__((2 + 4 * (4 / NHG)) * 32, 1) k_score_tc(const 
             if (!word_ok) m = 0u;
             if (!emit && word_ok) args.firebm[bh * args.nw + word] = m;
           }
-          msk[c] = m;
+          msk[j] = m;
           cnt += __popc(m);
+          if constexpr (NCT == 1) {
+#pragma unroll
+            for (int k = 0; k < 32; ++k) keep[k] = v[k];
+          }
         }
         if (emit) {
           // reserve the head's room for this tile, then stage each chunk that has hits and visit only its set bits
           int pos = cnt ? atomicAdd(&args.cand_cnt[bh], cnt) : 0;
 #pragma unroll
-          for (int c = 0; c < NC; ++c) {
-            if (!__any_sync(0xffffffffu, msk[c] != 0u)) continue;
+          for (int j = 0; j < NCT; ++j) {
+            const int c = sub + L::WPQ * j;
+            if (!__any_sync(0xffffffffu, msk[j] != 0u)) continue;
             float v[32];
-            tmem_ld_chunk<MH>(taddr + (MH == 128 ? 32 * c : 64 * c), v);
-            tmem_wait_ld();
             const int rc = row0 + (MH == 128 ? 32 * c : 64 * c + 32 * (lane >> 4));
-            if (MODE == 2) {
+            if constexpr (NCT == 1) {
+#pragma unroll
+              for (int k = 0; k < 32; ++k) v[k] = keep[k];
+            } else {
+              tmem_ld_chunk<MH>(taddr + (MH == 128 ? 32 * c : 64 * c), v);
+              tmem_wait_ld();
+            }
+            if (MODE == 2 && NCT > 1) {
               const float pr = args.page_res[(int64_t)b * args.n_pages + rc / PAGE];
               const float add = p1[hg] * pr;
               const float* eta = args.eta + (int64_t)b * args.N + rc;
@@ -440,7 +470,7 @@ __global__ void __launch_bounds__((2 + 4 * (4 / NHG)) * 32, 1) k_score_tc(const 
                 v[k] = args.lam * (v[k] + add + p2[hg] * e);
               }
             }
-            uint32_t m = msk[c];
+            uint32_t m = msk[j];
             if (m) {
 #pragma unroll
               for (int k = 0; k < 8; ++k)
@@ -459,7 +489,7 @@ __global__ void __launch_bounds__((2 + 4 * (4 / NHG)) * 32, 1) k_score_tc(const 
       }
       tmem_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive(&d_empty[g]);
+      if (lane == 0) mbar_arrive(&d_empty[ds]);
     }
   }
 
@@ -489,15 +519,19 @@ bool score_tc_supported(const vk_view& v, int r) {
          (v.rope_ld * 2) % 16 == 0 && (v.rope_bstride * 2) % 16 == 0 && encode_fn() != nullptr;
 }
 
-cudaError_t launch_score_tc(const vk_view& v, int row_offset, int row_stride, int n_rows, ScoreTcArgs args,
-                            cudaStream_t st) {
+// Configurations (MH, NHG, TM, G, WPQ): 128-row tiles and 4 / NHG epilogue groups of one warp per lane quarter.
+// Measured slower for the candidate pass (sample, theta and candidates at B = 64, N = 65536, H = 64: 0.21 ms):
+// 64-row tiles with six groups over eight accumulators (0.29 ms), and three groups of two warps per lane quarter,
+// each thread one 32-row chunk kept in registers from the compare to the emission (0.23 ms).
+template <int MH, int NHG, int MODE, int TM, int G, int WPQ>
+static cudaError_t launch_cfg(const vk_view& v, const __nv_bfloat16* rope, int row_stride, int n_rows,
+                              ScoreTcArgs args, cudaStream_t st) {
+  using L = TcCfg<MH, NHG, TM, G, WPQ>;
   auto encode = encode_fn();
-  if (!encode) return cudaErrorNotSupported;
   CUtensorMap kmap, qmap;
-  const auto* rope = static_cast<const __nv_bfloat16*>(v.rope) + (int64_t)row_offset * v.rope_ld;
   cuuint64_t kdims[3] = {(cuuint64_t)D_ROPE, (cuuint64_t)n_rows, (cuuint64_t)v.B};
   cuuint64_t kstr[2] = {(cuuint64_t)(v.rope_ld * row_stride * 2), (cuuint64_t)(v.rope_bstride * 2)};
-  cuuint32_t kbox[3] = {D_ROPE, TC_M, 1};
+  cuuint32_t kbox[3] = {D_ROPE, (cuuint32_t)TM, 1};
   cuuint32_t es3[3] = {1, 1, 1};
   // each row contributes one 128-byte segment 1152 bytes apart: no L2 promotion, so DRAM reads only those bytes
   if (encode(&kmap, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<__nv_bfloat16*>(rope), kdims, kstr, kbox, es3,
@@ -516,32 +550,37 @@ cudaError_t launch_score_tc(const vk_view& v, int row_offset, int row_stride, in
   args.H = v.H;
   args.N = v.N;
   args.n_rows = n_rows;
-  args.tiles_per_seq = (n_rows + TC_M - 1) / TC_M;
+  args.tiles_per_seq = (n_rows + TM - 1) / TM;
   args.total_tiles = (int64_t)args.tiles_per_seq * v.B;
   args.n_pages = (v.N + PAGE - 1) / PAGE;
   args.tmem_cols = 512;
   const int grid = (int)std::min<int64_t>(args.total_tiles, sm_count());   // persistent: one CTA per SM
-  const int m = args.mode;
-  auto go = [&](auto kernel, size_t smem, int g) -> cudaError_t {
-    cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    if (e != cudaSuccess) return e;
-    if (grid > 0) kernel<<<grid, (2 + 4 * g) * 32, smem, st>>>(kmap, qmap, args);
-    return cudaSuccess;
-  };
-  cudaError_t e;
-  if (v.H <= 64) {
-    const size_t sm = TcSmem<64, 1>::total;
-    e = m == 0 ? go(k_score_tc<64, 1, 0>, sm, 4) : m == 1 ? go(k_score_tc<64, 1, 1>, sm, 4) : go(k_score_tc<64, 1, 2>, sm, 4);
-  } else if (v.H <= 128) {
-    const size_t sm = TcSmem<128, 1>::total;
-    e = m == 0 ? go(k_score_tc<128, 1, 0>, sm, 4) : m == 1 ? go(k_score_tc<128, 1, 1>, sm, 4) : go(k_score_tc<128, 1, 2>, sm, 4);
-  } else {
-    const size_t sm = TcSmem<128, 2>::total;
-    e = m == 0 ? go(k_score_tc<128, 2, 0>, sm, 2) : m == 1 ? go(k_score_tc<128, 2, 1>, sm, 2) : go(k_score_tc<128, 2, 2>, sm, 2);
-  }
+  auto kernel = k_score_tc<MH, NHG, MODE, TM, G, WPQ>;
+  cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)L::total);
   if (e != cudaSuccess) return e;
-  if (grid > 0) count_launches(1);
+  if (grid > 0) {
+    kernel<<<grid, L::THREADS, L::total, st>>>(kmap, qmap, args);
+    count_launches(1);
+  }
   return cudaGetLastError();
+}
+
+template <int MH, int NHG>
+static cudaError_t launch_heads(const vk_view& v, const __nv_bfloat16* rope, int row_stride, int n_rows,
+                                const ScoreTcArgs& args, cudaStream_t st) {
+  constexpr int G4 = 4 / NHG;
+  if (args.mode == 0) return launch_cfg<MH, NHG, 0, 128, G4, 1>(v, rope, row_stride, n_rows, args, st);
+  if (args.mode == 2) return launch_cfg<MH, NHG, 2, 128, G4, 1>(v, rope, row_stride, n_rows, args, st);
+  return launch_cfg<MH, NHG, 1, 128, G4, 1>(v, rope, row_stride, n_rows, args, st);
+}
+
+cudaError_t launch_score_tc(const vk_view& v, int row_offset, int row_stride, int n_rows, ScoreTcArgs args,
+                            cudaStream_t st) {
+  if (!encode_fn()) return cudaErrorNotSupported;
+  const auto* rope = static_cast<const __nv_bfloat16*>(v.rope) + (int64_t)row_offset * v.rope_ld;
+  if (v.H <= 64) return launch_heads<64, 1>(v, rope, row_stride, n_rows, args, st);
+  if (v.H <= 128) return launch_heads<128, 1>(v, rope, row_stride, n_rows, args, st);
+  return launch_heads<128, 2>(v, rope, row_stride, n_rows, args, st);
 }
 
 }  // namespace vk

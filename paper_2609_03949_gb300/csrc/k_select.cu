@@ -336,14 +336,14 @@ cudaError_t launch_select_dense(int B, int H, int N, const float* scores, const 
 // candidates pass; the candidates themselves carry fp32 scores). Up to THETA_R x 256 archive samples are
 // held in registers (THETA_R per thread, loaded together); more go through shared memory (ns x 4 bytes).
 constexpr int THETA_R = 16;
-__global__ void __launch_bounds__(CAND_THREADS) k_theta(int ns, int off, int stride, int lo, int hi, int j,
+__global__ void __launch_bounds__(CAND_THREADS) k_theta(int ns, int ld, int off, int stride, int lo, int hi, int j,
                                                         const __nv_bfloat16* __restrict__ sample,
                                                         float* __restrict__ theta) {
   extern __shared__ __align__(16) unsigned char smem[];
   __shared__ unsigned int hist[256];
   __shared__ uint32_t scratch[64];
   const int64_t bh = blockIdx.x;
-  const __nv_bfloat16* a = sample + bh * (int64_t)ns;
+  const __nv_bfloat16* a = sample + bh * (int64_t)ld;
   // sampled positions off + stride * i inside [lo, hi) are a contiguous index range [i0, i1)
   const int i0 = lo > off ? (lo - off + stride - 1) / stride : 0;
   const int i1 = min(ns, hi > off ? (hi - off + stride - 1) / stride : 0);
@@ -393,13 +393,13 @@ __global__ void __launch_bounds__(CAND_THREADS) k_theta(int ns, int off, int str
   if (threadIdx.x == 0) theta[bh] = funkey(prefix);
 }
 
-cudaError_t launch_theta(int B, int H, int ns, int off, int stride, int lo, int hi, int j, const void* sample,
+cudaError_t launch_theta(int B, int H, int ns, int ld, int off, int stride, int lo, int hi, int j, const void* sample,
                          float* theta, cudaStream_t st) {
   // shared memory only when the samples outgrow the registers (na <= ns)
   const size_t smem = ns > THETA_R * CAND_THREADS ? (size_t)ns * 4 : 0;
   cudaError_t e = cudaFuncSetAttribute(k_theta, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
-  k_theta<<<B * H, CAND_THREADS, smem, st>>>(ns, off, stride, lo, hi, j,
+  k_theta<<<B * H, CAND_THREADS, smem, st>>>(ns, ld, off, stride, lo, hi, j,
                                              static_cast<const __nv_bfloat16*>(sample), theta);
   count_launches(1);
   return cudaGetLastError();

@@ -189,6 +189,7 @@ void fused_params(int64_t N, int64_t lo, int64_t hi, int64_t k, VkLayout* L) {
   L->ss = A >= 32768 ? 16 : std::max<int64_t>(1, A / 2048);
   L->soff = L->ss / 2;
   L->ns = N > L->soff ? (N - L->soff + L->ss - 1) / L->ss : 0;
+  L->sld = (L->ns + 7) / 8 * 8;            // sample rows start on 16-byte boundaries
   int64_t n_arch = 0;                      // sampled rows inside the archive
   for (int64_t i = 0; i < L->ns; ++i) {
     const int64_t u = L->soff + L->ss * i;
@@ -230,7 +231,7 @@ VkLayout make_layout(const vk_view& v, const vk_params& p) {
   L.off_firebm = take(L.two_tier ? sizeof(uint32_t) * BH * L.nw : 0);
   L.off_part_o = take(sizeof(float) * v.B * nslot * v.H * vk::D_LAT);
   L.off_part_ml = take(sizeof(float) * v.B * nslot * v.H * 2);
-  L.off_sample = take(L.fused ? sizeof(uint16_t) * BH * L.ns : 0);     // bf16 sample scores
+  L.off_sample = take(L.fused ? sizeof(uint16_t) * BH * L.sld : 0);    // bf16 sample scores
   L.off_theta = take(L.fused ? sizeof(float) * BH : 0);
   L.off_ccnt = take(L.fused ? sizeof(int) * BH : 0);
   L.off_cand = take(L.fused ? sizeof(int2) * BH * L.capc : 0);
@@ -436,11 +437,12 @@ int vk_decode_step(const vk_view* view, const vk_params* params, const vk_index*
       vk::ScoreTcArgs a{};
       a.mode = 0;
       a.scores = sample;
-      a.scores_ld = L.ns;
+      a.scores_ld = L.sld;
       a.scores_bf16 = 1;
       a.status = status;
       VK_CUDA(vk::launch_score_tc(v, (int)L.soff, (int)L.ss, (int)L.ns, a, st), "sample scores");
-      VK_CUDA(vk::launch_theta(B, H, (int)L.ns, (int)L.soff, (int)L.ss, lo, hi, (int)L.j, sample, theta, st), "theta");
+      VK_CUDA(vk::launch_theta(B, H, (int)L.ns, (int)L.sld, (int)L.soff, (int)L.ss, lo, hi, (int)L.j, sample, theta, st),
+              "theta");
       vk::ScoreTcArgs c{};
       c.mode = 1;
       c.theta = theta;
@@ -455,8 +457,8 @@ int vk_decode_step(const vk_view* view, const vk_params* params, const vk_index*
     prof(2, st);
     VK_CUDA(vk::launch_select_cand(B, H, N, lo, hi, k, nullptr, ccnt, cand, (int)L.capc,
                                    (params->flags & VK_FLAG_FORCE_FALLBACK) ? 1 : 0, v, qprep ? qt : nullptr, idx, count,
-                                   cap, 0, nullptr,
-                                   selbm, L.nw, status, st), "select (candidates)");
+                                   cap, 0, nullptr, selbm, L.nw, status, st),
+            "select (candidates)");
   } else {
     if (L.tc) {
       vk::ScoreTcArgs a{};

@@ -106,7 +106,8 @@ struct VkLayout {
   bool two_tier;
   bool tc;                      // bf16, r = 64, H % 16 == 0: scoring on tcgen05
   bool fused;                   // threshold-candidate selection (no materialised scores)
-  int64_t ss, soff, ns, j;      // fused: sample stride, offset, rows per sequence, order statistic for theta
+  int64_t ss, soff, ns, sld, j; // fused: sample stride, offset, rows per sequence, row stride (ns rounded up to 8),
+                                //        order statistic for theta
   int64_t capc;                 // fused: candidate capacity per head
   int64_t fcap;                 // two-tier top_j (fused path or page trigger): fired-candidate capacity per head
   size_t off_status, off_qt, off_qcn, off_qrn, off_qrf, off_smax1, off_nfired, off_scores, off_selbm, off_firebm,
@@ -152,7 +153,7 @@ cudaError_t launch_trigger_dense(int B, int H, int N, int W, int n_sink, float l
                                  float* scores, const float* qcn, const float* qrn, const float* eta,
                                  const float* page_res, const float* smax1, const uint32_t* selbm,
                                  uint32_t* firebm, int64_t nw, int64_t* nfired, cudaStream_t st);
-cudaError_t launch_theta(int B, int H, int ns, int off, int stride, int lo, int hi, int j, const void* sample,
+cudaError_t launch_theta(int B, int H, int ns, int ld, int off, int stride, int lo, int hi, int j, const void* sample,
                          float* theta, cudaStream_t st);
 cudaError_t launch_select_cand(int B, int H, int N, int lo, int hi, int64_t k, const int64_t* k_per_head,
                                const int* cand_cnt, const int2* cand, int capc, int force_fallback, const vk_view& v,
