@@ -185,6 +185,31 @@ int vk_workspace_init(void* ws, size_t ws_bytes, void* stream);
 int vk_decode_step_noalloc(const vk_view* view, const vk_params* params, const vk_index* index, float* out,
                            float* lse, float* smax, int32_t* idx, int32_t* count, int32_t cap, void* stream);
 
+/* ---------------------------------------------------------------------------------------------------------------
+ * The sigma selector of tier 1 (Sec. 4.1, Eq. 3; Corollary 1): a query-independent ranking of cached rows by how
+ * far their 64-wide RoPE branch lies from its low-pass reconstruction. Rows are cut into fixed blocks of T rows
+ * (4096 in the paper); within each closed block, per RoPE dim, the sequence-axis DFT is kept on bins
+ * 0 .. kappa-1 (the one-sided spectrum of a real signal) and inverted, and sigma_u = |r_u - low_u|_2 over the 64
+ * dims. A block's sigma depends on that block alone, so a stream of closes gives the same values as one pass. */
+
+/* Workspace bytes of vk_sigma for a block length T and bandwidth kappa; 0 on bad arguments (T a positive multiple
+ * of 128, 1 <= kappa <= 64). The workspace starts with the device status word read by vk_poll_status. */
+size_t vk_sigma_workspace_bytes(int32_t T, int32_t kappa);
+
+/* sigma [B, N] fp32 (device) for every row of every sequence of the view (only its RoPE columns are read; bf16
+ * caches, VK_ERR_UNSUPPORTED otherwise). Rows past the last whole block of T rows (the open tail) get -1. The two
+ * contractions per block run on the tensor cores with the low-pass basis and its coefficients rounded to bf16
+ * (fp32 accumulation): sigma is exact to about 1e-4 relative. */
+int vk_sigma(const vk_view* view, int32_t T, int32_t kappa, float* sigma, void* ws, size_t ws_bytes, void* stream);
+
+/* The sigma selector's attended set of every sequence (Sec. 4.1: sinks, the open tail, and the top m closed rows):
+ * the sinks [0, min(n_sink, closed)), the rows past the last whole block of T rows, and the m closed rows outside
+ * the sinks with the largest sigma (ties: the smaller position; m is clamped to the rows available), listed in
+ * ascending position in idx[b, 0:count[b]) (idx [B, cap] int32, count [B] int32; device). sigma [B, N] as written
+ * by vk_sigma. cap must hold the whole set. ws: at least 256 bytes (the device status word). */
+int vk_sigma_select(int32_t B, int32_t N, int32_t T, const float* sigma, int32_t n_sink, int64_t m, int32_t* idx,
+                    int32_t* count, int32_t cap, void* ws, size_t ws_bytes, void* stream);
+
 /* Wait for `stream`, read the device status word at the start of ws (VK_OK or a device-side error of the
  * calls since the last poll) and clear it. */
 int vk_poll_status(void* ws, void* stream);

@@ -552,6 +552,48 @@ int vk_decode_step(const vk_view* view, const vk_params* params, const vk_index*
   return VK_OK;
 }
 
+size_t vk_sigma_workspace_bytes(int32_t T, int32_t kappa) {
+  if (T < 128 || T % 128 != 0 || kappa < 1 || kappa > 64) return 0;
+  return vk::sigma_workspace_bytes(T, kappa);
+}
+
+int vk_sigma(const vk_view* view, int32_t T, int32_t kappa, float* sigma, void* ws, size_t ws_bytes, void* stream) {
+  g_err[0] = 0;
+  int rc;
+  if ((rc = check_view(view)) != VK_OK) return rc;
+  if (T < 128 || T % 128 != 0) return fail(VK_ERR_INVALID_ARG, "T = %d must be a positive multiple of 128", T);
+  if (kappa < 1 || kappa > 64) return fail(VK_ERR_INVALID_ARG, "kappa = %d is outside [1, 64]", kappa);
+  if (view->dtype != VK_BF16) return fail(VK_ERR_UNSUPPORTED, "the sigma kernel reads bf16 caches");
+  if (!sigma) return fail(VK_ERR_INVALID_ARG, "sigma is NULL");
+  const size_t need = vk::sigma_workspace_bytes(T, kappa);
+  if (!ws || (reinterpret_cast<uintptr_t>(ws) & 255u) != 0 || ws_bytes < need)
+    return fail(VK_ERR_WORKSPACE, "the sigma workspace needs %zu bytes, 256-byte aligned", need);
+  VK_CUDA(vk::launch_sigma(*view, T, kappa, sigma, ws, static_cast<cudaStream_t>(stream)), "sigma");
+  return VK_OK;
+}
+
+int vk_sigma_select(int32_t B, int32_t N, int32_t T, const float* sigma, int32_t n_sink, int64_t m, int32_t* idx,
+                    int32_t* count, int32_t cap, void* ws, size_t ws_bytes, void* stream) {
+  g_err[0] = 0;
+  if (B < 1 || N < 1 || N > MAX_N) return fail(VK_ERR_INVALID_ARG, "B >= 1 and 1 <= N <= %lld required", (long long)MAX_N);
+  if (T < 1) return fail(VK_ERR_INVALID_ARG, "T must be >= 1");
+  if (n_sink < 0 || m < 0) return fail(VK_ERR_INVALID_ARG, "n_sink and m must be >= 0");
+  if (!sigma || !idx || !count) return fail(VK_ERR_INVALID_ARG, "sigma, idx and count must be non-NULL");
+  const int64_t closed = (int64_t)(N / T) * T;
+  const int64_t sinks = std::min<int64_t>(n_sink, closed);
+  const int64_t k = std::min<int64_t>(m, closed - sinks);
+  if ((int64_t)cap < sinks + k + (N - closed))
+    return fail(VK_ERR_INVALID_ARG, "cap = %d < sinks + m + open tail = %lld", cap, (long long)(sinks + k + N - closed));
+  if (!ws || ws_bytes < 256 || (reinterpret_cast<uintptr_t>(ws) & 255u) != 0)
+    return fail(VK_ERR_WORKSPACE, "a 256-byte aligned workspace of at least 256 bytes is needed (status word)");
+  // the selection of the per-head path with one "head" per sequence: the open tail is always kept like the recent
+  // window, the sinks like the sinks, and the top m of the closed rows by (sigma desc, position asc)
+  VK_CUDA(vk::launch_select_dense(B, 1, N, sigma, nullptr, k, (int)(N - closed), (int)sinks, idx, count, cap, 0,
+                                  nullptr, nullptr, 0, static_cast<int*>(ws), static_cast<cudaStream_t>(stream)),
+          "sigma select");
+  return VK_OK;
+}
+
 int vk_poll_status(void* ws, void* stream) {
   g_err[0] = 0;
   if (!ws) return fail(VK_ERR_WORKSPACE, "workspace is NULL");

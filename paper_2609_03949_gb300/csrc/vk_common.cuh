@@ -165,4 +165,8 @@ cudaError_t launch_score_tc(const vk_view& v, int row_offset, int row_stride, in
                             cudaStream_t st);
 cudaError_t launch_bitmap_to_list(int B, int H, int N, const uint32_t* bitmap, int64_t nw, int32_t* idx,
                                   int32_t* count, int cap, int* status, cudaStream_t st);
+// sigma selector (k_sigma.cu): workspace = status word + the two bf16 copies of the low-pass basis
+int sigma_basis_cols(int kappa);
+size_t sigma_workspace_bytes(int T, int kappa);
+cudaError_t launch_sigma(const vk_view& v, int T, int kappa, float* sigma, void* ws, cudaStream_t st);
 }  // namespace vk

@@ -67,6 +67,16 @@ class Workload:
             q_rope=self.q_rope[bs].contiguous(), planted_pos=self.planted_pos[bs].contiguous())
 
 
+def _slice_rows(self, n: int) -> "Workload":
+    """The same sequences cut to their first ``n`` cached rows (an earlier point of the same stream)."""
+    pp = self.planted_pos.clone()
+    pp[pp >= n] = -1
+    return dataclasses.replace(self, N=n, cache=self.cache[:, :n].contiguous(), planted_pos=pp)
+
+
+Workload.slice_rows = _slice_rows
+
+
 def haar_orthogonal(seed: int) -> np.ndarray:
     """Haar-distributed 64x64 orthogonal matrix: QR of a seeded Gaussian with sign(diag R) > 0 (fp64)."""
     rng = np.random.default_rng(seed)

@@ -74,6 +74,9 @@ def lib():
             "vk_profile_set_events": ([ctypes.POINTER(ctypes.c_void_p), I32], ctypes.c_int),
             "vk_profile_launches": ([], I64),
             "vk_last_error": ([], ctypes.c_char_p),
+            "vk_sigma_workspace_bytes": ([I32, I32], SZ),
+            "vk_sigma": ([VP, I32, I32, P, P, SZ, P], ctypes.c_int),
+            "vk_sigma_select": ([I32, I32, I32, P, I32, I64, P, P, I32, P, SZ, P], ctypes.c_int),
         }
         for name, (args, res) in sig.items():
             fn = getattr(L, name)
@@ -87,8 +90,8 @@ def exported_symbols():
     """Names of the C entry points declared in include/vk.h."""
     return ["vk_keep_count", "vk_min_cap", "vk_workspace_bytes", "vk_build_digest", "vk_score", "vk_select",
             "vk_sparse_attn", "vk_decode_step", "vk_decode_step_noalloc", "vk_workspace_init", "vk_poll_status",
-            "vk_profile_set_events",
-            "vk_profile_launches", "vk_last_error"]
+            "vk_profile_set_events", "vk_profile_launches", "vk_last_error", "vk_sigma_workspace_bytes", "vk_sigma",
+            "vk_sigma_select"]
 
 
 def _check(rc: int):
@@ -242,3 +245,28 @@ class DecodeBuffers:
 
     def run(self, view, params, index=None, stream=None):
         vk_decode_step(view, params, index, self.out, self.lse, self.smax, self.idx, self.count, self.ws, stream)
+
+
+# ------------------------------------------------------------------------------------------------ sigma selector
+def vk_sigma_workspace_bytes(T: int, kappa: int) -> int:
+    n = int(lib().vk_sigma_workspace_bytes(T, kappa))
+    if n == 0:
+        raise VkError(VK_ERR_INVALID_ARG, f"bad sigma parameters T={T} kappa={kappa}")
+    return n
+
+
+def vk_sigma(view, T: int, kappa: int, sigma, ws, stream=None) -> None:
+    _check(lib().vk_sigma(ctypes.byref(view), T, kappa, _ptr(sigma), _ptr(ws), ws.numel() * ws.element_size(),
+                          _stream(stream)))
+
+
+def vk_sigma_select(B: int, N: int, T: int, sigma, n_sink: int, m: int, idx, count, ws, stream=None) -> None:
+    _check(lib().vk_sigma_select(B, N, T, _ptr(sigma), n_sink, m, _ptr(idx), _ptr(count), idx.shape[-1], _ptr(ws),
+                                 ws.numel() * ws.element_size(), _stream(stream)))
+
+
+def alloc_bytes(n: int, device="cuda") -> torch.Tensor:
+    """A zeroed, 256-byte aligned device buffer of n bytes (allocated by torch)."""
+    buf = torch.zeros(n + 256, dtype=torch.uint8, device=device)
+    off = (-buf.data_ptr()) % 256
+    return buf[off:off + n]

@@ -135,3 +135,22 @@ def test_other_entry_points_refuse(vk):
                              None) == vk.VK_ERR_INVALID_ARG
     assert L.vk_poll_status(None, None) == vk.VK_ERR_WORKSPACE
     assert L.vk_workspace_init(None, 0, None) == vk.VK_ERR_WORKSPACE
+
+
+def test_sigma_entry_points_refuse(vk):
+    L = vk.lib()
+    v = fake_view(vk, N=20000)
+    assert L.vk_sigma_workspace_bytes(4096, 16) > 0
+    assert L.vk_sigma_workspace_bytes(4000, 16) == 0          # T must be a multiple of 128
+    assert L.vk_sigma_workspace_bytes(4096, 65) == 0          # kappa in [1, 64]
+    nb = L.vk_sigma_workspace_bytes(4096, 16)
+    assert L.vk_sigma(ctypes.byref(v), 4000, 16, FAKE, FAKE, nb, None) == vk.VK_ERR_INVALID_ARG
+    assert L.vk_sigma(ctypes.byref(v), 4096, 0, FAKE, FAKE, nb, None) == vk.VK_ERR_INVALID_ARG
+    assert L.vk_sigma(ctypes.byref(v), 4096, 16, FAKE, FAKE, nb - 1, None) == vk.VK_ERR_WORKSPACE
+    assert L.vk_sigma(ctypes.byref(v), 4096, 16, None, FAKE, nb, None) == vk.VK_ERR_INVALID_ARG
+    assert L.vk_sigma(ctypes.byref(fake_view(vk, N=20000, dtype=1)), 4096, 16, FAKE, FAKE, nb, None) == \
+        vk.VK_ERR_UNSUPPORTED
+    # the attended set must fit: sinks + m + open tail (20000 rows: 4 closed blocks, a tail of 3616)
+    assert L.vk_sigma_select(2, 20000, 4096, FAKE, 4, 100, FAKE, FAKE, 3616 + 104 - 1, FAKE, 256, None) == \
+        vk.VK_ERR_INVALID_ARG
+    assert L.vk_sigma_select(2, 20000, 4096, FAKE, 4, 100, FAKE, FAKE, 3720, FAKE, 255, None) == vk.VK_ERR_WORKSPACE
