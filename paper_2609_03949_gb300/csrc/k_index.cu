@@ -16,9 +16,9 @@ __host__ __device__ __forceinline__ const T* tptr(const void* p) { return reinte
 // ---------------------------------------------------------------------------------------------- query prep
 // One warp per (b, h); lane l owns RoPE coordinates l and l + 32.
 template <typename T>
-__global__ void k_qprep(const T* __restrict__ q_latent, const T* __restrict__ q_rope, int BH, int r,
+__global__ void k_qprep(const T* __restrict__ q_latent, const T* __restrict__ q_rope, int BH, int H, int r,
                         const float* __restrict__ rot, float* __restrict__ qt, float* __restrict__ qcn,
-                        float* __restrict__ qrn, float* __restrict__ qrf) {
+                        float* __restrict__ qrn, float* __restrict__ qrf, __nv_bfloat16* __restrict__ qhl) {
   const int warp = (blockIdx.x * blockDim.x + threadIdx.x) >> 5, lane = threadIdx.x & 31;
   if (warp >= BH) return;
   const T* qc = q_latent + (int64_t)warp * D_LAT;
@@ -47,6 +47,18 @@ __global__ void k_qprep(const T* __restrict__ q_latent, const T* __restrict__ q_
   for (int o = 16; o; o >>= 1) res += __shfl_xor_sync(0xffffffffu, res, o);
   qt[(int64_t)warp * D_ROPE + lane] = y0;
   qt[(int64_t)warp * D_ROPE + lane + 32] = y1;
+  if (qhl && r < D_ROPE) {
+    // the tensor-core query operand: high part bf16(y), low part bf16(y - high), zero past r (up to 16)
+    const int kp = r < 16 ? 16 : r, b = warp / H, h = warp - b * H;
+    __nv_bfloat16* hi = qhl + ((int64_t)(2 * b) * H + h) * kp;
+    __nv_bfloat16* lo = qhl + ((int64_t)(2 * b + 1) * H + h) * kp;
+    for (int j = lane; j < kp; j += 32) {
+      const float y = j < r ? (j < 32 ? y0 : y1) : 0.f;
+      const __nv_bfloat16 yh = __float2bfloat16_rn(y);
+      hi[j] = yh;
+      lo[j] = __float2bfloat16_rn(y - __bfloat162float(yh));
+    }
+  }
   if (lane == 0) {
     qcn[warp] = sqrtf(ss);
     qrn[warp] = sqrtf(res);
@@ -55,14 +67,14 @@ __global__ void k_qprep(const T* __restrict__ q_latent, const T* __restrict__ q_
 }
 
 cudaError_t launch_qprep(const vk_view& v, int r, const float* rot, float* qt, float* qcn, float* qrn, float* qrf,
-                         cudaStream_t st) {
+                         __nv_bfloat16* qhl, cudaStream_t st) {
   const int BH = v.B * v.H, threads = 256, blocks = (BH * 32 + threads - 1) / threads;
   if (v.dtype == VK_BF16)
     k_qprep<__nv_bfloat16><<<blocks, threads, 0, st>>>(tptr<__nv_bfloat16>(v.q_latent), tptr<__nv_bfloat16>(v.q_rope),
-                                                       BH, r, rot, qt, qcn, qrn, qrf);
+                                                       BH, v.H, r, rot, qt, qcn, qrn, qrf, qhl);
   else
-    k_qprep<float><<<blocks, threads, 0, st>>>(tptr<float>(v.q_latent), tptr<float>(v.q_rope), BH, r, rot, qt, qcn,
-                                               qrn, qrf);
+    k_qprep<float><<<blocks, threads, 0, st>>>(tptr<float>(v.q_latent), tptr<float>(v.q_rope), BH, v.H, r, rot, qt,
+                                               qcn, qrn, qrf, qhl);
   count_launches(1);
   return cudaGetLastError();
 }

@@ -1,8 +1,11 @@
-// k_score_tc.cu -- RoPE-branch scoring on the 5th-generation tensor cores (tcgen05), bf16, r = 64.
+// k_score_tc.cu -- RoPE-branch scoring on the 5th-generation tensor cores (tcgen05), bf16, r in {8, 16, 32, 64}.
 //
 // a[h,u] = Qr_h . K_u for every cached row (Eq. 4's exact summand): per sequence the [H x 64] query times the
-// [64 x N] RoPE slice, a dense contraction at H flop per byte. One CTA per SM walks a contiguous range of
-// 128-row tiles:
+// [64 x N] RoPE slice, a dense contraction at H flop per byte. For a width-r digest D_u (r = 32, 16, 8) it is
+// (O Qr_h)[0:r] . D_u: the rotated query is fp32, so it enters as two bf16 parts (high and the rounding rest),
+// two products accumulated in fp32, and the digest tile is read with the swizzle its row width allows (64, 32 or
+// 16 bytes; at r = 8 the second 8 columns of the K = 16 product are the query's zero padding). One CTA per SM
+// walks a contiguous range of 128-row tiles:
 //   warp 0 (one thread)  TMA: the tile's 128 x 64 bf16 slice (128 B of every 1152-B row, 128-byte swizzle) into a
 //                        7-stage ring, and the sequence's H x 64 query when the sequence changes;
 //   warp 1 (one thread)  D = Q . K^T on tcgen05: M = 64 heads (H <= 64) or 128 per head group, N = 128 rows,
@@ -59,7 +62,19 @@ __device__ __forceinline__ uint64_t sw128_desc(uint32_t saddr) {
          ((uint64_t)1u << 46) | ((uint64_t)2u << 61);
 }
 
-// Instruction descriptor of tcgen05.mma kind::f16: fp32 accumulate (bits 4-5 = 1), A and B bf16 (7-9, 10-12 = 1),
+// K-major operand descriptor for rows of ROWB bytes: 128, 64 and 32 take the matching swizzle (8-row atoms of
+// 8 x ROWB bytes, the next 8 rows ROWB x 8 bytes on); 16 is the unswizzled layout of 8-row x 16-byte core matrices
+// 128 bytes apart, whose leading offset (the next 8 columns along K) is 0: the r = 8 digest's K = 16 product reads
+// its 8 columns twice, against the query's 8 values and its 8 zeros.
+template <int ROWB>
+__device__ __forceinline__ uint64_t kmajor_desc(uint32_t saddr) {
+  constexpr uint64_t layout = ROWB == 128 ? 2 : ROWB == 64 ? 4 : ROWB == 32 ? 6 : 0;
+  constexpr uint64_t lbo = ROWB == 16 ? 0 : 1;
+  constexpr uint64_t sbo = (uint64_t)(8 * ROWB) >> 4;
+  return (uint64_t)((saddr >> 4) & 0x3FFFu) | (lbo << 16) | (sbo << 32) | ((uint64_t)1u << 46) | (layout << 61);
+}
+
+// Instruction descriptor of tcgen05.mma kind::f16// Instruction descriptor of tcgen05.mma kind::f16: fp32 accumulate (bits 4-5 = 1), A and B bf16 (7-9, 10-12 = 1),
 // both K-major, N >> 3 at bits 17-22, M >> 4 at bits 24-28.
 __host__ __device__ constexpr uint32_t mma_idesc_bf16(int M, int N) {
   return (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(N >> 3) << 17) | ((uint32_t)(M >> 4) << 24);
@@ -128,23 +143,29 @@ __device__ __forceinline__ uint32_t range_mask(int r0, int lo, int hi) {
 // NHG x TM tensor-memory columns (all 512 columns), a ring of STAGES tiles (96 to 112 KB). Shared memory from a
 // 1024-aligned base: the ring, two query buffers of NHG x MH rows, 128 B of staging per epilogue thread (modes 1,
 // 2), barriers.
-template <int MH, int NHG, int TM_, int G_, int WPQ_ = 1>
+template <int MH, int NHG, int TM_, int G_, int WPQ_ = 1, int RW_ = 64>
 struct TcCfg {
   static constexpr int TM = TM_;
   static constexpr int G = G_;
   static constexpr int WPQ = WPQ_;
+  static constexpr int RW = RW_;                         // score width: the RoPE columns (64) or a digest width
+  static constexpr int KP = RW < 16 ? 16 : RW;           // the product's K (r = 8 padded to 16 on the query side)
+  static constexpr int QPARTS = RW == 64 ? 1 : 2;        // bf16 query parts: the RoPE query, or high + low
+  static constexpr uint32_t QROW = KP * 2;               // bytes per query row
+  static constexpr uint32_t QPART = NHG * MH * QROW;     // one query part
   static constexpr uint32_t DCOLS = NHG * TM;            // columns per accumulator
   static constexpr int NACC = 512 / DCOLS;
-  static constexpr uint32_t TILE = TM * 128;             // TM rows x 64 bf16
+  static constexpr uint32_t TILE = TM * RW * 2;          // TM rows x RW bf16
   static constexpr int NC = MH == 128 ? TM / 32 : TM / 64;   // 32-row chunks per lane and tile
   static constexpr int NCT = NC / WPQ;                   // of which one epilogue thread takes
   static constexpr int EW = 4 * G * WPQ;                 // epilogue warps
   static constexpr int THREADS = (2 + EW) * 32;
-  static constexpr uint32_t qbuf = NHG * MH * 128;
+  static constexpr uint32_t qbuf = QPARTS * QPART;
   static constexpr uint32_t STG = EW * 32 * 128;
-  // as many ring stages (up to 7 of 16 KB, or 14 of 8 KB) as fit beside the queries and the staging rows
+  // as many ring stages as fit beside the queries and the staging rows, up to 112 KB of tiles (28 at most)
   static constexpr int STAGES_FIT = (int)((224u * 1024u - 2 * qbuf - STG) / TILE);
-  static constexpr int STAGES = STAGES_FIT < (TM == 128 ? 7 : 14) ? STAGES_FIT : (TM == 128 ? 7 : 14);
+  static constexpr int STAGES_CAP = (int)(112u * 1024u / TILE) < 28 ? (int)(112u * 1024u / TILE) : 28;
+  static constexpr int STAGES = STAGES_FIT < STAGES_CAP ? STAGES_FIT : STAGES_CAP;
   static constexpr uint32_t a = 0;
   static constexpr uint32_t q = a + STAGES * TILE;
   static constexpr uint32_t stg = q + 2 * qbuf;
@@ -155,11 +176,11 @@ struct TcCfg {
   static_assert(total <= 232448, "scoring shared memory exceeds the 227 KB opt-in limit");
 };
 
-template <int MH, int NHG, int MODE, int TM_, int G_, int WPQ_>
-__global__ void __launch_bounds__(TcCfg<MH, NHG, TM_, G_, WPQ_>::THREADS, 1)
+template <int MH, int NHG, int MODE, int TM_, int G_, int WPQ_, int RW_>
+__global__ void __launch_bounds__(TcCfg<MH, NHG, TM_, G_, WPQ_, RW_>::THREADS, 1)
     k_score_tc(const __grid_constant__ CUtensorMap kmap, const __grid_constant__ CUtensorMap qmap,
                const ScoreTcArgs args) {
-  using L = TcCfg<MH, NHG, TM_, G_, WPQ_>;
+  using L = TcCfg<MH, NHG, TM_, G_, WPQ_, RW_>;
   constexpr int G = L::G, TC_M = L::TM, TC_STAGES = L::STAGES, NACC = L::NACC;
   constexpr uint32_t TC_TILE_BYTES = L::TILE;
   extern __shared__ __align__(1024) unsigned char smem_raw[];
@@ -178,7 +199,7 @@ __global__ void __launch_bounds__(TcCfg<MH, NHG, TM_, G_, WPQ_>::THREADS, 1)
   __shared__ uint32_t tmem_base;
   __shared__ int abort_flag;
   __shared__ int skip_stage[TC_STAGES];                  // mode 2 page skip: the ring stage's tile was not loaded
-  const bool page_skip = MODE == 2 && args.page_knorm != nullptr;
+  const bool page_skip = MODE == 2 && L::RW == 64 && args.page_knorm != nullptr;
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int64_t total = args.total_tiles;
@@ -220,8 +241,9 @@ __global__ void __launch_bounds__(TcCfg<MH, NHG, TM_, G_, WPQ_>::THREADS, 1)
           if (quse > 0 && !mbar_wait(&q_empty[qi], (quse - 1) & 1, &abort_flag)) {
             lok = false;
           } else {
-            mbar_arrive_expect_tx(&q_full[qi], (uint32_t)H * 128u);
-            tma_load_2d(sq + qi * L::qbuf, &qmap, 0, b * H, &q_full[qi]);
+            mbar_arrive_expect_tx(&q_full[qi], (uint32_t)H * L::QROW * L::QPARTS);
+            for (int part = 0; part < L::QPARTS; ++part)
+              tma_load_2d(sq + qi * L::qbuf + part * L::QPART, &qmap, 0, (b * L::QPARTS + part) * H, &q_full[qi]);
           }
         }
 #pragma unroll
@@ -274,8 +296,9 @@ __global__ void __launch_bounds__(TcCfg<MH, NHG, TM_, G_, WPQ_>::THREADS, 1)
         if (b != prev_b) {
           const int qi = (b - b_first) & 1, quse = (b - b_first) >> 1;
           if (quse > 0 && !mbar_wait(&q_empty[qi], (quse - 1) & 1, &abort_flag)) { abort_flag = 1; break; }
-          mbar_arrive_expect_tx(&q_full[qi], (uint32_t)H * 128u);
-          tma_load_2d(sq + qi * L::qbuf, &qmap, 0, b * H, &q_full[qi]);
+          mbar_arrive_expect_tx(&q_full[qi], (uint32_t)H * L::QROW * L::QPARTS);
+          for (int part = 0; part < L::QPARTS; ++part)
+            tma_load_2d(sq + qi * L::qbuf + part * L::QPART, &qmap, 0, (b * L::QPARTS + part) * H, &q_full[qi]);
           prev_b = b;
         }
         const int s = i % TC_STAGES, use = i / TC_STAGES;
@@ -301,15 +324,19 @@ __global__ void __launch_bounds__(TcCfg<MH, NHG, TM_, G_, WPQ_>::THREADS, 1)
         if (!mbar_wait(&a_full[s], use & 1, &abort_flag)) { abort_flag = 1; break; }
         if (duse > 0 && !mbar_wait(&d_empty[ds], (duse - 1) & 1, &abort_flag)) { abort_flag = 1; break; }
         tmem_fence_after();                              // the epilogue's reads of this accumulator came first
-        const uint64_t bd = sw128_desc(smem_addr(sa + s * TC_TILE_BYTES));
-        const uint64_t ad = sw128_desc(smem_addr(sq + qi * L::qbuf));
+        const uint64_t bd = kmajor_desc<L::RW * 2>(smem_addr(sa + s * TC_TILE_BYTES));
         if (!(page_skip && skip_stage[s])) {             // a skipped tile: no product (the epilogue ignores it)
 #pragma unroll
           for (int hg = 0; hg < NHG; ++hg)
 #pragma unroll
-            for (int k = 0; k < 4; ++k)
-              mma_bf16(tmem_base + ds * DCOLS + hg * TC_M, ad + (uint64_t)((hg * MH * 128 + 32 * k) >> 4),
-                       bd + (uint64_t)((32 * k) >> 4), idesc, k > 0 ? 1u : 0u);
+            for (int part = 0; part < L::QPARTS; ++part) {
+              const uint64_t ad =
+                  kmajor_desc<L::QROW>(smem_addr(sq + qi * L::qbuf + part * L::QPART + hg * MH * L::QROW));
+#pragma unroll
+              for (int k = 0; k < L::KP / 16; ++k)
+                mma_bf16(tmem_base + ds * DCOLS + hg * TC_M, ad + (uint64_t)((32 * k) >> 4),
+                         bd + (uint64_t)(L::RW >= 16 ? (32 * k) >> 4 : 0), idesc, (part > 0 || k > 0) ? 1u : 0u);
+            }
         }
         mma_commit(&a_empty[s]);
         mma_commit(&d_full[ds]);
@@ -515,35 +542,43 @@ static PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
 }
 
 bool score_tc_supported(const vk_view& v, int r) {
-  return v.dtype == VK_BF16 && r == D_ROPE && v.H % 16 == 0 && v.H >= 16 && v.H <= 256 &&
-         (v.rope_ld * 2) % 16 == 0 && (v.rope_bstride * 2) % 16 == 0 && encode_fn() != nullptr;
+  return v.dtype == VK_BF16 && (r == 8 || r == 16 || r == 32 || r == D_ROPE) && v.H % 16 == 0 && v.H >= 16 &&
+         v.H <= 256 && (v.rope_ld * 2) % 16 == 0 && (v.rope_bstride * 2) % 16 == 0 && encode_fn() != nullptr;
 }
 
 // Configurations (MH, NHG, TM, G, WPQ): 128-row tiles and 4 / NHG epilogue groups of one warp per lane quarter.
 // Measured slower for the candidate pass (sample, theta and candidates at B = 64, N = 65536, H = 64: 0.21 ms):
 // 64-row tiles with six groups over eight accumulators (0.29 ms), and three groups of two warps per lane quarter,
 // each thread one 32-row chunk kept in registers from the compare to the emission (0.23 ms).
-template <int MH, int NHG, int MODE, int TM, int G, int WPQ>
-static cudaError_t launch_cfg(const vk_view& v, const __nv_bfloat16* rope, int row_stride, int n_rows,
-                              ScoreTcArgs args, cudaStream_t st) {
-  using L = TcCfg<MH, NHG, TM, G, WPQ>;
+static CUtensorMapSwizzle swizzle_for(int row_bytes) {
+  return row_bytes == 128 ? CU_TENSOR_MAP_SWIZZLE_128B
+         : row_bytes == 64 ? CU_TENSOR_MAP_SWIZZLE_64B
+         : row_bytes == 32 ? CU_TENSOR_MAP_SWIZZLE_32B
+                           : CU_TENSOR_MAP_SWIZZLE_NONE;
+}
+
+template <int MH, int NHG, int MODE, int TM, int G, int WPQ, int RW>
+static cudaError_t launch_cfg(const vk_view& v, const void* keys, int64_t key_ld, int64_t key_bstride,
+                              const void* qsrc, int row_stride, int n_rows, ScoreTcArgs args, cudaStream_t st) {
+  using L = TcCfg<MH, NHG, TM, G, WPQ, RW>;
   auto encode = encode_fn();
   CUtensorMap kmap, qmap;
-  cuuint64_t kdims[3] = {(cuuint64_t)D_ROPE, (cuuint64_t)n_rows, (cuuint64_t)v.B};
-  cuuint64_t kstr[2] = {(cuuint64_t)(v.rope_ld * row_stride * 2), (cuuint64_t)(v.rope_bstride * 2)};
-  cuuint32_t kbox[3] = {D_ROPE, (cuuint32_t)TM, 1};
+  cuuint64_t kdims[3] = {(cuuint64_t)RW, (cuuint64_t)n_rows, (cuuint64_t)v.B};
+  cuuint64_t kstr[2] = {(cuuint64_t)(key_ld * row_stride * 2), (cuuint64_t)(key_bstride * 2)};
+  cuuint32_t kbox[3] = {(cuuint32_t)RW, (cuuint32_t)TM, 1};
   cuuint32_t es3[3] = {1, 1, 1};
-  // each row contributes one 128-byte segment 1152 bytes apart: no L2 promotion, so DRAM reads only those bytes
-  if (encode(&kmap, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<__nv_bfloat16*>(rope), kdims, kstr, kbox, es3,
-             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_NONE,
+  // RoPE rows: one 128-byte segment per 1152-byte row, no L2 promotion, so DRAM reads only those bytes
+  if (encode(&kmap, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(keys), kdims, kstr, kbox, es3,
+             CU_TENSOR_MAP_INTERLEAVE_NONE, swizzle_for(RW * 2),
+             RW == 64 ? CU_TENSOR_MAP_L2_PROMOTION_NONE : CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
     return cudaErrorInvalidValue;
-  cuuint64_t qdims[2] = {(cuuint64_t)D_ROPE, (cuuint64_t)v.B * v.H};
-  cuuint64_t qstr[1] = {(cuuint64_t)D_ROPE * 2};
-  cuuint32_t qbox[2] = {D_ROPE, (cuuint32_t)v.H};
+  cuuint64_t qdims[2] = {(cuuint64_t)L::KP, (cuuint64_t)v.B * v.H * L::QPARTS};
+  cuuint64_t qstr[1] = {(cuuint64_t)L::QROW};
+  cuuint32_t qbox[2] = {(cuuint32_t)L::KP, (cuuint32_t)v.H};
   cuuint32_t es2[2] = {1, 1};
-  if (encode(&qmap, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(v.q_rope), qdims, qstr, qbox, es2,
-             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+  if (encode(&qmap, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(qsrc), qdims, qstr, qbox, es2,
+             CU_TENSOR_MAP_INTERLEAVE_NONE, swizzle_for(L::QROW), CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
     return cudaErrorInvalidValue;
   args.B = v.B;
@@ -555,7 +590,7 @@ static cudaError_t launch_cfg(const vk_view& v, const __nv_bfloat16* rope, int r
   args.n_pages = (v.N + PAGE - 1) / PAGE;
   args.tmem_cols = 512;
   const int grid = (int)std::min<int64_t>(args.total_tiles, sm_count());   // persistent: one CTA per SM
-  auto kernel = k_score_tc<MH, NHG, MODE, TM, G, WPQ>;
+  auto kernel = k_score_tc<MH, NHG, MODE, TM, G, WPQ, RW>;
   cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)L::total);
   if (e != cudaSuccess) return e;
   if (grid > 0) {
@@ -565,22 +600,40 @@ static cudaError_t launch_cfg(const vk_view& v, const __nv_bfloat16* rope, int r
   return cudaGetLastError();
 }
 
-template <int MH, int NHG>
-static cudaError_t launch_heads(const vk_view& v, const __nv_bfloat16* rope, int row_stride, int n_rows,
-                                const ScoreTcArgs& args, cudaStream_t st) {
+template <int MH, int NHG, int RW>
+static cudaError_t launch_heads(const vk_view& v, const void* keys, int64_t key_ld, int64_t key_bstride,
+                                const void* qsrc, int row_stride, int n_rows, const ScoreTcArgs& args,
+                                cudaStream_t st) {
   constexpr int G4 = 4 / NHG;
-  if (args.mode == 0) return launch_cfg<MH, NHG, 0, 128, G4, 1>(v, rope, row_stride, n_rows, args, st);
-  if (args.mode == 2) return launch_cfg<MH, NHG, 2, 128, G4, 1>(v, rope, row_stride, n_rows, args, st);
-  return launch_cfg<MH, NHG, 1, 128, G4, 1>(v, rope, row_stride, n_rows, args, st);
+  if (args.mode == 0)
+    return launch_cfg<MH, NHG, 0, 128, G4, 1, RW>(v, keys, key_ld, key_bstride, qsrc, row_stride, n_rows, args, st);
+  if (args.mode == 2)
+    return launch_cfg<MH, NHG, 2, 128, G4, 1, RW>(v, keys, key_ld, key_bstride, qsrc, row_stride, n_rows, args, st);
+  return launch_cfg<MH, NHG, 1, 128, G4, 1, RW>(v, keys, key_ld, key_bstride, qsrc, row_stride, n_rows, args, st);
 }
 
-cudaError_t launch_score_tc(const vk_view& v, int row_offset, int row_stride, int n_rows, ScoreTcArgs args,
-                            cudaStream_t st) {
+template <int RW>
+static cudaError_t launch_width(const vk_view& v, const void* keys, int64_t key_ld, int64_t key_bstride,
+                                const void* qsrc, int row_stride, int n_rows, const ScoreTcArgs& args,
+                                cudaStream_t st) {
+  if (v.H <= 64) return launch_heads<64, 1, RW>(v, keys, key_ld, key_bstride, qsrc, row_stride, n_rows, args, st);
+  if (v.H <= 128) return launch_heads<128, 1, RW>(v, keys, key_ld, key_bstride, qsrc, row_stride, n_rows, args, st);
+  return launch_heads<128, 2, RW>(v, keys, key_ld, key_bstride, qsrc, row_stride, n_rows, args, st);
+}
+
+cudaError_t launch_score_tc(const vk_view& v, int r, const void* digest, const void* qhl, int row_offset,
+                            int row_stride, int n_rows, ScoreTcArgs args, cudaStream_t st) {
   if (!encode_fn()) return cudaErrorNotSupported;
-  const auto* rope = static_cast<const __nv_bfloat16*>(v.rope) + (int64_t)row_offset * v.rope_ld;
-  if (v.H <= 64) return launch_heads<64, 1>(v, rope, row_stride, n_rows, args, st);
-  if (v.H <= 128) return launch_heads<128, 1>(v, rope, row_stride, n_rows, args, st);
-  return launch_heads<128, 2>(v, rope, row_stride, n_rows, args, st);
+  if (r == D_ROPE) {
+    const auto* rope = static_cast<const __nv_bfloat16*>(v.rope) + (int64_t)row_offset * v.rope_ld;
+    return launch_width<64>(v, rope, v.rope_ld, v.rope_bstride, v.q_rope, row_stride, n_rows, args, st);
+  }
+  const auto* dig = static_cast<const __nv_bfloat16*>(digest) + (int64_t)row_offset * r;
+  const int64_t bs = (int64_t)v.N * r;
+  if (r == 32) return launch_width<32>(v, dig, r, bs, qhl, row_stride, n_rows, args, st);
+  if (r == 16) return launch_width<16>(v, dig, r, bs, qhl, row_stride, n_rows, args, st);
+  if (r == 8) return launch_width<8>(v, dig, r, bs, qhl, row_stride, n_rows, args, st);
+  return cudaErrorInvalidValue;
 }
 
 }  // namespace vk

@@ -78,22 +78,24 @@ __device__ __forceinline__ void pick_digit_asc(const unsigned int* hist, unsigne
   }
 }
 
-// Key sources for the ordered selection: scores stored in memory, or recomputed from the RoPE columns
-// (the exact fallback of the fused path: a[u] = qt . K_u in fp32, qt already in shared memory).
+// Key sources for the ordered selection: scores stored in memory, or recomputed from the RoPE columns or the digest
+// (the exact fallback of the fused path: a[u] = qt[0:r] . key_u[0:r] in fp32, qt already in shared memory).
 struct StoredKeys {
   const float* a;
   __device__ __forceinline__ float operator()(int u) const { return a[u]; }
 };
 struct RecomputedKeys {
-  const __nv_bfloat16* rope;    // this sequence's RoPE rows
+  const __nv_bfloat16* rows;    // this sequence's RoPE rows (r = 64) or digest rows
   int64_t ld;
   const float* qt;              // 64 floats in shared memory
+  int r;                        // key width, a multiple of 8
   __device__ __forceinline__ float operator()(int u) const {
-    const uint4* r = reinterpret_cast<const uint4*>(rope + (int64_t)u * ld);
+    const uint4* rp = reinterpret_cast<const uint4*>(rows + (int64_t)u * ld);
     float acc = 0.f;
 #pragma unroll
     for (int i = 0; i < 8; ++i) {
-      const uint4 w = r[i];
+      if (8 * i >= r) break;
+      const uint4 w = rp[i];
       acc = fmaf(qt[8 * i + 0], bf_lo(w.x), acc); acc = fmaf(qt[8 * i + 1], bf_hi(w.x), acc);
       acc = fmaf(qt[8 * i + 2], bf_lo(w.y), acc); acc = fmaf(qt[8 * i + 3], bf_hi(w.y), acc);
       acc = fmaf(qt[8 * i + 4], bf_lo(w.z), acc); acc = fmaf(qt[8 * i + 5], bf_hi(w.z), acc);
@@ -487,7 +489,7 @@ constexpr int CAND_R = 16;
 __global__ void __launch_bounds__(CAND_THREADS, 8) k_select_cand(
     int H, int N, int lo, int hi, long long k_all, const long long* __restrict__ k_per_head,
     const int* __restrict__ cand_cnt, const int2* __restrict__ cand, int capc, int force_fallback,
-    const __nv_bfloat16* __restrict__ rope, int64_t rld, int64_t rbs, const float* __restrict__ qt,
+    const __nv_bfloat16* __restrict__ rope, int64_t rld, int64_t rbs, int r, const float* __restrict__ qt,
     const __nv_bfloat16* __restrict__ qrope,
     int32_t* __restrict__ idx, int32_t* __restrict__ count, int cap, int append, float* __restrict__ kth,
     uint32_t* __restrict__ bitmap, long long nw, int* status) {
@@ -513,7 +515,7 @@ __global__ void __launch_bounds__(CAND_THREADS, 8) k_select_cand(
     for (int i = threadIdx.x; i < D_ROPE; i += blockDim.x)
       qts[i] = qt ? qt[bh * D_ROPE + i] : __bfloat162float(qrope[bh * D_ROPE + i]);
     __syncthreads();
-    RecomputedKeys keys{rope + (int64_t)b * rbs, rld, qts};
+    RecomputedKeys keys{rope + (int64_t)b * rbs, rld, qts, r};
     select_ordered(keys, N, lo, hi, k, out, count + bh, cap, 0, kth_bh, bm, nw, status);
     return;
   }
@@ -548,14 +550,16 @@ __global__ void __launch_bounds__(CAND_THREADS, 8) k_select_cand(
 
 cudaError_t launch_select_cand(int B, int H, int N, int lo, int hi, int64_t k, const int64_t* k_per_head,
                                const int* cand_cnt, const int2* cand, int capc, int force_fallback, const vk_view& v,
-                               const float* qt, int32_t* idx, int32_t* count, int cap, int append, float* kth,
-                               uint32_t* bitmap, int64_t nw, int* status, cudaStream_t st) {
+                               int r, const void* digest, const float* qt, int32_t* idx, int32_t* count, int cap,
+                               int append, float* kth, uint32_t* bitmap, int64_t nw, int* status, cudaStream_t st) {
   const size_t smem = nw <= SEL_SMEM_BITMAP_WORDS ? (size_t)nw * 4 : 0;
   cudaError_t e = cudaFuncSetAttribute(k_select_cand, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
   k_select_cand<<<B * H, CAND_THREADS, smem, st>>>(
       H, N, lo, hi, (long long)k, reinterpret_cast<const long long*>(k_per_head), cand_cnt, cand, capc,
-      force_fallback, static_cast<const __nv_bfloat16*>(v.rope), v.rope_ld, v.rope_bstride, qt,
+      force_fallback,
+      r == D_ROPE ? static_cast<const __nv_bfloat16*>(v.rope) : static_cast<const __nv_bfloat16*>(digest),
+      r == D_ROPE ? v.rope_ld : (int64_t)r, r == D_ROPE ? v.rope_bstride : (int64_t)v.N * r, r, qt,
       static_cast<const __nv_bfloat16*>(v.q_rope), idx, count, cap,
       append, kth, bitmap, (long long)nw, status);
   count_launches(1);

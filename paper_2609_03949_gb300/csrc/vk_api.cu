@@ -221,6 +221,7 @@ VkLayout make_layout(const vk_view& v, const vk_params& p) {
   auto take = [&](size_t bytes) { size_t o = off; off = align_up(off + bytes, 256); return o; };
   L.off_status = take(256);
   L.off_qt = take(sizeof(float) * BH * vk::D_ROPE);
+  L.off_qhl = take(sizeof(uint16_t) * BH * 2 * 32);                   // bf16 query parts of a digest (r <= 32)
   L.off_qcn = take(sizeof(float) * BH);
   L.off_qrn = take(sizeof(float) * BH);
   L.off_qrf = take(sizeof(float) * BH);
@@ -332,17 +333,20 @@ int vk_score(const vk_view* view, const vk_params* params, const vk_index* index
   if ((rc = check_ws(L, ws, ws_bytes)) != VK_OK) return rc;
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   float* qt = at<float>(ws, L.off_qt);
+  __nv_bfloat16* qhl = at<__nv_bfloat16>(ws, L.off_qhl);
+  if (!L.tc || params->r < vk::D_ROPE)
+    VK_CUDA(vk::launch_qprep(*view, params->r, index ? index->rot : nullptr, qt, at<float>(ws, L.off_qcn),
+                             at<float>(ws, L.off_qrn), at<float>(ws, L.off_qrf), L.tc ? qhl : nullptr, st), "qprep");
   if (L.tc) {
     vk::ScoreTcArgs a{};
     a.mode = 0;
     a.scores = scores;
     a.scores_ld = view->N;
     a.status = at<int>(ws, L.off_status);
-    VK_CUDA(vk::launch_score_tc(*view, 0, 1, view->N, a, st), "score (tcgen05)");
+    VK_CUDA(vk::launch_score_tc(*view, params->r, index ? index->digest : nullptr, qhl, 0, 1, view->N, a, st),
+            "score (tcgen05)");
     return VK_OK;
   }
-  VK_CUDA(vk::launch_qprep(*view, params->r, index ? index->rot : nullptr, qt, at<float>(ws, L.off_qcn),
-                           at<float>(ws, L.off_qrn), at<float>(ws, L.off_qrf), st), "qprep");
   VK_CUDA(vk::launch_score_simt(*view, params->r, qt,
                                 static_cast<const __nv_bfloat16*>(index ? index->digest : nullptr), scores, st),
           "score");
@@ -413,6 +417,9 @@ int vk_decode_step(const vk_view* view, const vk_params* params, const vk_index*
   float* qcn = at<float>(ws, L.off_qcn);
   float* qrn = at<float>(ws, L.off_qrn);
   float* qrf = at<float>(ws, L.off_qrf);
+  __nv_bfloat16* qhl = at<__nv_bfloat16>(ws, L.off_qhl);
+  const void* digest = index ? index->digest : nullptr;
+  const int r = params->r;
   float* scores = at<float>(ws, L.off_scores);
   uint32_t* selbm = at<uint32_t>(ws, L.off_selbm);
   float* po = at<float>(ws, L.off_part_o);
@@ -421,10 +428,11 @@ int vk_decode_step(const vk_view* view, const vk_params* params, const vk_index*
 
   const int lo = S, hi = N - W;
   prof(0, st);
-  // the query prep feeds the materialised-score path and the trigger; the fused path at r = 64 scores with the
-  // RoPE query as it is (its exact fallback reads it directly)
-  const bool qprep = !L.fused || two_tier;
-  if (qprep) VK_CUDA(vk::launch_qprep(v, params->r, index ? index->rot : nullptr, qt, qcn, qrn, qrf, st), "qprep");
+  // the query prep feeds the materialised-score path, the trigger and digest scoring on the tensor cores (the bf16
+  // query parts); the fused path at r = 64 scores with the RoPE query as it is (its exact fallback reads it directly)
+  const bool qprep = !L.fused || two_tier || r < vk::D_ROPE;
+  if (qprep)
+    VK_CUDA(vk::launch_qprep(v, r, index ? index->rot : nullptr, qt, qcn, qrn, qrf, L.tc ? qhl : nullptr, st), "qprep");
   prof(1, st);
   if (L.fused) {
     // threshold from a strided sample, then one scoring pass that keeps only the rows above it
@@ -440,7 +448,7 @@ int vk_decode_step(const vk_view* view, const vk_params* params, const vk_index*
       a.scores_ld = L.sld;
       a.scores_bf16 = 1;
       a.status = status;
-      VK_CUDA(vk::launch_score_tc(v, (int)L.soff, (int)L.ss, (int)L.ns, a, st), "sample scores");
+      VK_CUDA(vk::launch_score_tc(v, r, digest, qhl, (int)L.soff, (int)L.ss, (int)L.ns, a, st), "sample scores");
       VK_CUDA(vk::launch_theta(B, H, (int)L.ns, (int)L.sld, (int)L.soff, (int)L.ss, lo, hi, (int)L.j, sample, theta, st),
               "theta");
       vk::ScoreTcArgs c{};
@@ -452,12 +460,12 @@ int vk_decode_step(const vk_view* view, const vk_params* params, const vk_index*
       c.cand = cand;
       c.capc = (int)L.capc;
       c.status = status;
-      VK_CUDA(vk::launch_score_tc(v, 0, 1, N, c, st), "score (candidates)");
+      VK_CUDA(vk::launch_score_tc(v, r, digest, qhl, 0, 1, N, c, st), "score (candidates)");
     }
     prof(2, st);
     VK_CUDA(vk::launch_select_cand(B, H, N, lo, hi, k, nullptr, ccnt, cand, (int)L.capc,
-                                   (params->flags & VK_FLAG_FORCE_FALLBACK) ? 1 : 0, v, qprep ? qt : nullptr, idx, count,
-                                   cap, 0, nullptr, selbm, L.nw, status, st),
+                                   (params->flags & VK_FLAG_FORCE_FALLBACK) ? 1 : 0, v, r, digest, qprep ? qt : nullptr,
+                                   idx, count, cap, 0, nullptr, selbm, L.nw, status, st),
             "select (candidates)");
   } else {
     if (L.tc) {
@@ -466,7 +474,7 @@ int vk_decode_step(const vk_view* view, const vk_params* params, const vk_index*
       a.scores = scores;
       a.scores_ld = N;
       a.status = status;
-      VK_CUDA(vk::launch_score_tc(v, 0, 1, N, a, st), "score (tcgen05)");
+      VK_CUDA(vk::launch_score_tc(v, r, digest, qhl, 0, 1, N, a, st), "score (tcgen05)");
     } else {
       VK_CUDA(vk::launch_score_simt(v, params->r, qt, static_cast<const __nv_bfloat16*>(index ? index->digest : nullptr),
                                     scores, st), "score");
@@ -492,8 +500,8 @@ int vk_decode_step(const vk_view* view, const vk_params* params, const vk_index*
                                       index->page_eta, smax1, selbm, firebm, L.nw, params->top_j, fcnt, fcand,
                                       (int)L.fcap, st), "page trigger");
       if (params->top_j > 0) {
-        VK_CUDA(vk::launch_select_cand(B, H, N, lo, hi, params->top_j, nullptr, fcnt, fcand, (int)L.fcap, 0, v, qt, idx,
-                                       count, cap, 1, nullptr, firebm, L.nw, status, st), "top_j");
+        VK_CUDA(vk::launch_select_cand(B, H, N, lo, hi, params->top_j, nullptr, fcnt, fcand, (int)L.fcap, 0, v, r, digest,
+                                       qt, idx, count, cap, 1, nullptr, firebm, L.nw, status, st), "top_j");
       } else {
         VK_CUDA(vk::launch_bitmap_to_list(B, H, N, firebm, L.nw, idx, count, cap, status, st), "fired list");
       }
@@ -526,11 +534,11 @@ int vk_decode_step(const vk_view* view, const vk_params* params, const vk_index*
         t.cand_cnt = fcnt;
         t.cand = fcand;
         t.capc = (int)L.fcap;
-        VK_CUDA(vk::launch_score_tc(v, 0, 1, N, t, st), "trigger (candidates)");
-        VK_CUDA(vk::launch_select_cand(B, H, N, lo, hi, params->top_j, nullptr, fcnt, fcand, (int)L.fcap, 0, v, qt, idx,
-                                       count, cap, 1, nullptr, firebm, L.nw, status, st), "top_j");
+        VK_CUDA(vk::launch_score_tc(v, r, digest, qhl, 0, 1, N, t, st), "trigger (candidates)");
+        VK_CUDA(vk::launch_select_cand(B, H, N, lo, hi, params->top_j, nullptr, fcnt, fcand, (int)L.fcap, 0, v, r, digest,
+                                       qt, idx, count, cap, 1, nullptr, firebm, L.nw, status, st), "top_j");
       } else {
-        VK_CUDA(vk::launch_score_tc(v, 0, 1, N, t, st), "trigger");
+        VK_CUDA(vk::launch_score_tc(v, r, digest, qhl, 0, 1, N, t, st), "trigger");
         VK_CUDA(vk::launch_bitmap_to_list(B, H, N, firebm, L.nw, idx, count, cap, status, st), "fired list");
       }
     } else {

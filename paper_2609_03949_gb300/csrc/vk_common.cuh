@@ -110,7 +110,7 @@ struct VkLayout {
                                 //        order statistic for theta
   int64_t capc;                 // fused: candidate capacity per head
   int64_t fcap;                 // two-tier top_j (fused path or page trigger): fired-candidate capacity per head
-  size_t off_status, off_qt, off_qcn, off_qrn, off_qrf, off_smax1, off_nfired, off_scores, off_selbm, off_firebm,
+  size_t off_status, off_qt, off_qhl, off_qcn, off_qrn, off_qrf, off_smax1, off_nfired, off_scores, off_selbm, off_firebm,
       off_part_o, off_part_ml, off_sample, off_theta, off_ccnt, off_cand, off_fcnt, off_fcand, total;
 };
 
@@ -118,8 +118,10 @@ struct VkLayout {
 // Every launcher enqueues on `st`, counts its kernel launches and returns cudaGetLastError().
 namespace vk {
 void count_launches(int n);
+// qhl (may be NULL; r < 64): the rotated query's first r values as bf16 high and low parts, [B][2][H][max(r, 16)]
+// with zeros past r, the query operand of the tensor-core digest scoring.
 cudaError_t launch_qprep(const vk_view& v, int r, const float* rot, float* qt, float* qcn, float* qrn, float* qrf,
-                         cudaStream_t st);
+                         __nv_bfloat16* qhl, cudaStream_t st);
 cudaError_t launch_score_simt(const vk_view& v, int r, const float* qt, const __nv_bfloat16* digest,
                               float* scores, cudaStream_t st);
 cudaError_t launch_select_dense(int B, int H, int N, const float* scores, const int64_t* k_per_head,
@@ -157,12 +159,14 @@ cudaError_t launch_theta(int B, int H, int ns, int ld, int off, int stride, int 
                          float* theta, cudaStream_t st);
 cudaError_t launch_select_cand(int B, int H, int N, int lo, int hi, int64_t k, const int64_t* k_per_head,
                                const int* cand_cnt, const int2* cand, int capc, int force_fallback, const vk_view& v,
-                               const float* qt, int32_t* idx, int32_t* count, int cap, int append, float* kth,
-                               uint32_t* bitmap, int64_t nw, int* status, cudaStream_t st);
+                               int r, const void* digest, const float* qt, int32_t* idx, int32_t* count, int cap,
+                               int append, float* kth, uint32_t* bitmap, int64_t nw, int* status, cudaStream_t st);
 struct ScoreTcArgs;
 bool score_tc_supported(const vk_view& v, int r);
-cudaError_t launch_score_tc(const vk_view& v, int row_offset, int row_stride, int n_rows, ScoreTcArgs args,
-                            cudaStream_t st);
+// r = 64 reads the RoPE columns and the RoPE query; r in {8, 16, 32} the [B, N, r] digest and the query prep's
+// bf16 high and low parts qhl [B][2][H][max(r, 16)]. Rows row_offset + row_stride i, i < n_rows, of every sequence.
+cudaError_t launch_score_tc(const vk_view& v, int r, const void* digest, const void* qhl, int row_offset,
+                            int row_stride, int n_rows, ScoreTcArgs args, cudaStream_t st);
 cudaError_t launch_bitmap_to_list(int B, int H, int N, const uint32_t* bitmap, int64_t nw, int32_t* idx,
                                   int32_t* count, int cap, int* status, cudaStream_t st);
 // sigma selector (k_sigma.cu): workspace = status word + the two bf16 copies of the low-pass basis

@@ -356,6 +356,16 @@ def test_selection_paths(flags, trigger, top_j):
     run_case(wl, rho=1 / 32, window=256, n_sink=2, trigger=trigger, z_eff=0.7, top_j=top_j, flags=flags)
 
 
+@pytest.mark.parametrize("r", [8, 16, 32])
+@pytest.mark.parametrize("flags,trigger,top_j", [(0, 0, 0), (vk.VK_FLAG_FORCE_FALLBACK, 0, 0), (0, 1, 0), (0, 1, 6)],
+                         ids=["fused", "fallback", "trigger", "trigger-top_j"])
+def test_digest_selection_paths(r, flags, trigger, top_j):
+    # width-r digests on the tensor cores (query as bf16 high + low parts): the threshold-candidate selection, its
+    # exact fallback over recomputed digest scores, and the trigger scan all meet the oracle
+    wl = datagen.make_workload(2, 64, 20000, seed=19 + r, n_planted=16, planted_hi=20000 - 256, device="cuda")
+    run_case(wl, rho=1 / 32, r=r, window=256, n_sink=2, trigger=trigger, z_eff=0.6, top_j=top_j, flags=flags)
+
+
 def test_bounded_wait_reports_timeout():
     # Failure detection without a GPU fault: the test hook withholds one CTA's first tile; that CTA's bounded waits
     # give up after about a second, the status word reads VK_ERR_TIMEOUT and the context stays usable.
