@@ -26,6 +26,7 @@ D_LATENT, D_ROPE, PAGE = 512, 64, 64
 # Deliberate mistakes the "known-bad first" tests plant in the oracle (see vk_oracle.c).
 MUT_NONE, MUT_TIE_LARGER, MUT_DROP_WINDOW, MUT_SCALE_SQUARED = 0, 1, 2, 3
 MUT_ROT_TRANSPOSE, MUT_DROP_ROPE, MUT_TRIGGER_NO_Z, MUT_SIGMA_ONE_SIDED = 4, 5, 6, 7
+MUT_PCA_ASCENDING = 8
 
 
 def build(force: bool = False) -> str:
@@ -68,6 +69,9 @@ def lib():
         L.vko_sigma.argtypes = [P, I64, I32, I32, P]
         L.vko_sigma_select.argtypes = [P, I64, I32, I32, I64, P]
         L.vko_sigma_select.restype = I64
+        L.vko_second_moment.argtypes = [VP, P]
+        L.vko_sym_eig.argtypes = [P, P, P]
+        L.vko_pca_basis.argtypes = [VP, P, P]
         L.vko_set_mutation.argtypes = [ctypes.c_int]
         L.vko_num_threads.restype = ctypes.c_int
         del F
@@ -257,3 +261,28 @@ def sigma_select(sig: np.ndarray, T: int, n_sink: int, m: int) -> np.ndarray:
     c = lib().vko_sigma_select(_ptr(s), s.shape[0], int(T), int(n_sink), int(m), _ptr(out))
     return out[:c].copy()
 
+
+
+# ------------------------------------------------------------------------------------------------ PCA digest basis
+def second_moment(hi: HostInputs) -> np.ndarray:
+    """sum over every row of every sequence of K_u K_u^T, [64, 64] fp64."""
+    M = np.zeros((D_ROPE, D_ROPE), np.float64)
+    lib().vko_second_moment(ctypes.byref(hi.view), _ptr(M))
+    return M
+
+
+def sym_eig(M: np.ndarray):
+    """(eigenvalues desc [64], eigenvectors as rows [64, 64]) of a symmetric 64x64 matrix by cyclic Jacobi."""
+    A = np.ascontiguousarray(M, dtype=np.float64)
+    eig = np.zeros(D_ROPE, np.float64)
+    vec = np.zeros((D_ROPE, D_ROPE), np.float64)
+    lib().vko_sym_eig(_ptr(A), _ptr(eig), _ptr(vec))
+    return eig, vec
+
+
+def pca_basis(hi: HostInputs):
+    """(eigenvalues desc, rotation [64, 64] whose rows are the RoPE branch's principal directions)."""
+    eig = np.zeros(D_ROPE, np.float64)
+    rot = np.zeros((D_ROPE, D_ROPE), np.float64)
+    lib().vko_pca_basis(ctypes.byref(hi.view), _ptr(eig), _ptr(rot))
+    return eig, rot

@@ -45,6 +45,7 @@ enum {
   MUT_DROP_ROPE = 5,      /* attention logits drop the RoPE summand */
   MUT_TRIGGER_NO_Z = 6,   /* trigger ignores the certificate term */
   MUT_SIGMA_ONE_SIDED = 7, /* sigma's inverse DFT drops the factor 2 of the bins that stand for a conjugate pair */
+  MUT_PCA_ASCENDING = 8,   /* the PCA basis is ordered by increasing eigenvalue */
 };
 static int g_mutation = MUT_NONE;
 void vko_set_mutation(int m) { g_mutation = m; }
@@ -534,6 +535,93 @@ int64_t vko_sigma_select(const double* sigma, int64_t N, int32_t T, int32_t n_si
   free(ord);
   free(keep);
   return c;
+}
+
+/* ---------------------------------------------------------------- PCA-truncated digest (appendix ablation) */
+/* The branch-width ablation keeps the leading principal directions of the RoPE branch instead of the first
+ * coordinates after a random rotation. The basis is the eigenvector set of the (uncentred) second-moment matrix
+ * M = sum over every row of every sequence of K_u K_u^T (64 x 64, fp64), by decreasing eigenvalue: the rows of the
+ * returned rotation, so that digest = (O K_u)[0:r] keeps the most branch energy. Eigenvectors come from the cyclic
+ * Jacobi method (a rotation zeroes each off-diagonal pair in turn, sweeps repeat until the off-diagonal mass is
+ * negligible); each is signed so that its entry of largest magnitude is positive. eig receives the eigenvalues. */
+void vko_second_moment(const vko_view* v, double* M) {
+  for (int i = 0; i < D_ROPE * D_ROPE; ++i) M[i] = 0.0;
+  for (int b = 0; b < v->B; ++b)
+    for (int64_t u = 0; u < v->N; ++u) {
+      double k[D_ROPE];
+      for (int j = 0; j < D_ROPE; ++j) k[j] = K(v, b, u, j);
+      for (int i = 0; i < D_ROPE; ++i)
+        for (int j = 0; j < D_ROPE; ++j) M[i * D_ROPE + j] += k[i] * k[j];
+    }
+}
+
+void vko_sym_eig(const double* M_in, double* eig, double* vec /* [64][64], row i = eigenvector i */) {
+  const int n = D_ROPE;
+  double A[D_ROPE * D_ROPE], V[D_ROPE * D_ROPE];
+  for (int i = 0; i < n * n; ++i) A[i] = M_in[i];
+  for (int i = 0; i < n; ++i)
+    for (int j = 0; j < n; ++j) V[i * n + j] = (i == j) ? 1.0 : 0.0;
+  double total = 0.0;
+  for (int i = 0; i < n * n; ++i) total += A[i] * A[i];
+  for (int sweep = 0; sweep < 100; ++sweep) {
+    double off = 0.0;
+    for (int i = 0; i < n; ++i)
+      for (int j = 0; j < n; ++j)
+        if (i != j) off += A[i * n + j] * A[i * n + j];
+    if (off <= 1e-30 * total) break;
+    for (int p = 0; p < n - 1; ++p)
+      for (int q = p + 1; q < n; ++q) {
+        const double apq = A[p * n + q];
+        if (apq == 0.0) continue;
+        /* the rotation in the (p, q) plane that zeroes A[p][q] */
+        const double theta = (A[q * n + q] - A[p * n + p]) / (2.0 * apq);
+        const double t = (theta >= 0.0 ? 1.0 : -1.0) / (fabs(theta) + sqrt(theta * theta + 1.0));
+        const double c = 1.0 / sqrt(t * t + 1.0), sn = t * c;
+        for (int k = 0; k < n; ++k) {            /* A <- A J (columns p, q) */
+          const double akp = A[k * n + p], akq = A[k * n + q];
+          A[k * n + p] = c * akp - sn * akq;
+          A[k * n + q] = sn * akp + c * akq;
+        }
+        for (int k = 0; k < n; ++k) {            /* A <- J^T A (rows p, q) */
+          const double apk = A[p * n + k], aqk = A[q * n + k];
+          A[p * n + k] = c * apk - sn * aqk;
+          A[q * n + k] = sn * apk + c * aqk;
+        }
+        for (int k = 0; k < n; ++k) {            /* V <- V J: column j of V is eigenvector j */
+          const double vkp = V[k * n + p], vkq = V[k * n + q];
+          V[k * n + p] = c * vkp - sn * vkq;
+          V[k * n + q] = sn * vkp + c * vkq;
+        }
+      }
+  }
+  /* order by eigenvalue, descending (ties: the lower index first) */
+  int ord[D_ROPE];
+  for (int i = 0; i < n; ++i) ord[i] = i;
+  for (int i = 1; i < n; ++i) {
+    const int x = ord[i];
+    int j = i - 1;
+    const int asc = g_mutation == MUT_PCA_ASCENDING;
+    while (j >= 0 && (asc ? A[ord[j] * n + ord[j]] > A[x * n + x] : A[ord[j] * n + ord[j]] < A[x * n + x])) {
+      ord[j + 1] = ord[j];
+      --j;
+    }
+    ord[j + 1] = x;
+  }
+  for (int i = 0; i < n; ++i) {
+    const int c = ord[i];
+    eig[i] = A[c * n + c];
+    int big = 0;
+    for (int k = 1; k < n; ++k)
+      if (fabs(V[k * n + c]) > fabs(V[big * n + c])) big = k;
+    const double sg = V[big * n + c] < 0.0 ? -1.0 : 1.0;
+    for (int k = 0; k < n; ++k) vec[i * n + k] = sg * V[k * n + c];
+  }
+}
+
+void vko_pca_basis(const vko_view* v, double* eig, double* rot) {
+  double M[D_ROPE * D_ROPE];
+  vko_second_moment(v, M);
+  vko_sym_eig(M, eig, rot);
 }
 
 int vko_num_threads(void) {
