@@ -186,6 +186,16 @@ int vk_decode_step_noalloc(const vk_view* view, const vk_params* params, const v
                            float* lse, float* smax, int32_t* idx, int32_t* count, int32_t cap, void* stream);
 
 /* ---------------------------------------------------------------------------------------------------------------
+ * The PCA digest basis (the appendix's branch-width ablation: principal directions of the branch instead of a
+ * random rotation). rot [64, 64] row-major fp32 (device): the eigenvectors of M = sum over every row of every
+ * sequence of the view of K_u K_u^T, by decreasing eigenvalue, each signed so that its largest entry is positive;
+ * usable as index->rot and as vk_build_digest's rot64, so that the width-r digest keeps the most branch energy.
+ * eig [64] fp32 (device, may be NULL): the eigenvalues. M is accumulated on the tensor cores (bf16 rows, fp32 per
+ * CTA, fp64 across CTAs); the 64 x 64 eigenproblem is solved by cyclic Jacobi in fp64. bf16 caches only. */
+size_t vk_pca_workspace_bytes(void);
+int vk_pca_basis(const vk_view* view, float* rot, float* eig, void* ws, size_t ws_bytes, void* stream);
+
+/* ---------------------------------------------------------------------------------------------------------------
  * The sigma selector of tier 1 (Sec. 4.1, Eq. 3; Corollary 1): a query-independent ranking of cached rows by how
  * far their 64-wide RoPE branch lies from its low-pass reconstruction. Rows are cut into fixed blocks of T rows
  * (4096 in the paper); within each closed block, per RoPE dim, the sequence-axis DFT is kept on bins

@@ -560,6 +560,20 @@ int vk_decode_step(const vk_view* view, const vk_params* params, const vk_index*
   return VK_OK;
 }
 
+size_t vk_pca_workspace_bytes(void) { return vk::pca_workspace_bytes(); }
+
+int vk_pca_basis(const vk_view* view, float* rot, float* eig, void* ws, size_t ws_bytes, void* stream) {
+  g_err[0] = 0;
+  int rc;
+  if ((rc = check_view(view)) != VK_OK) return rc;
+  if (view->dtype != VK_BF16) return fail(VK_ERR_UNSUPPORTED, "the PCA basis kernel reads bf16 caches");
+  if (!rot || !aligned16(rot)) return fail(VK_ERR_INVALID_ARG, "rot must be a 16-byte aligned pointer");
+  if (!ws || (reinterpret_cast<uintptr_t>(ws) & 255u) != 0 || ws_bytes < vk::pca_workspace_bytes())
+    return fail(VK_ERR_WORKSPACE, "the PCA workspace needs %zu bytes, 256-byte aligned", vk::pca_workspace_bytes());
+  VK_CUDA(vk::launch_pca_basis(*view, rot, eig, ws, static_cast<cudaStream_t>(stream)), "pca basis");
+  return VK_OK;
+}
+
 size_t vk_sigma_workspace_bytes(int32_t T, int32_t kappa) {
   if (T < 128 || T % 128 != 0 || kappa < 1 || kappa > 64) return 0;
   return vk::sigma_workspace_bytes(T, kappa);

@@ -169,6 +169,9 @@ cudaError_t launch_score_tc(const vk_view& v, int r, const void* digest, const v
                             int row_stride, int n_rows, ScoreTcArgs args, cudaStream_t st);
 cudaError_t launch_bitmap_to_list(int B, int H, int N, const uint32_t* bitmap, int64_t nw, int32_t* idx,
                                   int32_t* count, int cap, int* status, cudaStream_t st);
+// PCA digest basis (k_pca.cu): workspace = status word + the fp64 second moment
+size_t pca_workspace_bytes();
+cudaError_t launch_pca_basis(const vk_view& v, float* rot, float* eig, void* ws, cudaStream_t st);
 // sigma selector (k_sigma.cu): workspace = status word + the two bf16 copies of the low-pass basis
 int sigma_basis_cols(int kappa);
 size_t sigma_workspace_bytes(int T, int kappa);

@@ -75,6 +75,8 @@ def lib():
             "vk_profile_launches": ([], I64),
             "vk_last_error": ([], ctypes.c_char_p),
             "vk_sigma_workspace_bytes": ([I32, I32], SZ),
+            "vk_pca_workspace_bytes": ([], SZ),
+            "vk_pca_basis": ([VP, P, P, P, SZ, P], ctypes.c_int),
             "vk_sigma": ([VP, I32, I32, P, P, SZ, P], ctypes.c_int),
             "vk_sigma_select": ([I32, I32, I32, P, I32, I64, P, P, I32, P, SZ, P], ctypes.c_int),
         }
@@ -91,7 +93,7 @@ def exported_symbols():
     return ["vk_keep_count", "vk_min_cap", "vk_workspace_bytes", "vk_build_digest", "vk_score", "vk_select",
             "vk_sparse_attn", "vk_decode_step", "vk_decode_step_noalloc", "vk_workspace_init", "vk_poll_status",
             "vk_profile_set_events", "vk_profile_launches", "vk_last_error", "vk_sigma_workspace_bytes", "vk_sigma",
-            "vk_sigma_select"]
+            "vk_sigma_select", "vk_pca_workspace_bytes", "vk_pca_basis"]
 
 
 def _check(rc: int):
@@ -270,3 +272,12 @@ def alloc_bytes(n: int, device="cuda") -> torch.Tensor:
     buf = torch.zeros(n + 256, dtype=torch.uint8, device=device)
     off = (-buf.data_ptr()) % 256
     return buf[off:off + n]
+
+
+# ------------------------------------------------------------------------------------------------ PCA digest basis
+def vk_pca_basis(view, rot, eig=None, ws=None, stream=None) -> None:
+    """Principal directions of the view's RoPE branch as the rows of rot [64, 64] fp32 (eigenvalues into eig)."""
+    if ws is None:
+        ws = alloc_bytes(int(lib().vk_pca_workspace_bytes()))
+    _check(lib().vk_pca_basis(ctypes.byref(view), _ptr(rot), _ptr(eig), _ptr(ws), ws.numel() * ws.element_size(),
+                              _stream(stream)))
