@@ -26,7 +26,7 @@ D_LATENT, D_ROPE, PAGE = 512, 64, 64
 # Deliberate mistakes the "known-bad first" tests plant in the oracle (see vk_oracle.c).
 MUT_NONE, MUT_TIE_LARGER, MUT_DROP_WINDOW, MUT_SCALE_SQUARED = 0, 1, 2, 3
 MUT_ROT_TRANSPOSE, MUT_DROP_ROPE, MUT_TRIGGER_NO_Z, MUT_SIGMA_ONE_SIDED = 4, 5, 6, 7
-MUT_PCA_ASCENDING = 8
+MUT_PCA_ASCENDING, MUT_CONFORMAL_FLOOR = 8, 9
 
 
 def build(force: bool = False) -> str:
@@ -72,6 +72,14 @@ def lib():
         L.vko_second_moment.argtypes = [VP, P]
         L.vko_sym_eig.argtypes = [P, P, P]
         L.vko_pca_basis.argtypes = [VP, P, P]
+        L.vko_tau_s.argtypes = [D]
+        L.vko_tau_s.restype = D
+        L.vko_min_hard.argtypes = [D]
+        L.vko_min_hard.restype = I64
+        L.vko_conformal_quantile.argtypes = [P, I64, D, D]
+        L.vko_conformal_quantile.restype = D
+        L.vko_calib_zq.argtypes = [VP, I32, P, D, P, P, P, P, P, I32, P, P]
+        L.vko_calib_zq.restype = I64
         L.vko_set_mutation.argtypes = [ctypes.c_int]
         L.vko_num_threads.restype = ctypes.c_int
         del F
@@ -286,3 +294,33 @@ def pca_basis(hi: HostInputs):
     rot = np.zeros((D_ROPE, D_ROPE), np.float64)
     lib().vko_pca_basis(ctypes.byref(hi.view), _ptr(eig), _ptr(rot))
     return eig, rot
+
+
+# ------------------------------------------------------------------------------------------------ conformal z
+def tau_s(tau: float) -> float:
+    return float(lib().vko_tau_s(float(tau)))
+
+
+def min_hard(tau: float) -> int:
+    return int(lib().vko_min_hard(float(tau)))
+
+
+def conformal_quantile(zq, tau: float = 0.9, z_max: float = 8.0) -> float:
+    """z from the hard queries' required inflations (the ceil((n+1) tau_s)-th smallest, clamped to [0, z_max])."""
+    v = np.ascontiguousarray(np.asarray(zq, dtype=np.float64).ravel())
+    return float(lib().vko_conformal_quantile(_ptr(v) if v.size else 0, v.size, float(tau), float(z_max)))
+
+
+def calib_zq(hi: HostInputs, r: int, lam: float, a: np.ndarray, eta: np.ndarray, page_res: np.ndarray,
+             idx: np.ndarray, count: np.ndarray):
+    """(zq [B,H] with NaN where the query is not hard, ustar [B,H], n_hard) for every (b, h) as a calibration query."""
+    a = np.ascontiguousarray(a, dtype=np.float64)
+    eta = np.ascontiguousarray(eta, dtype=np.float64)
+    page_res = np.ascontiguousarray(page_res, dtype=np.float64)
+    idx = np.ascontiguousarray(idx, dtype=np.int32)
+    count = np.ascontiguousarray(count, dtype=np.int32)
+    zq = np.zeros((hi.B, hi.H), np.float64)
+    ustar = np.zeros((hi.B, hi.H), np.int32)
+    n = lib().vko_calib_zq(ctypes.byref(hi.view), int(r), _ptr(hi.rot), float(lam), _ptr(a), _ptr(eta), _ptr(page_res),
+                           _ptr(idx), _ptr(count), idx.shape[-1], _ptr(zq), _ptr(ustar))
+    return zq, ustar, int(n)

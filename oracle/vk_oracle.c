@@ -46,6 +46,7 @@ enum {
   MUT_TRIGGER_NO_Z = 6,   /* trigger ignores the certificate term */
   MUT_SIGMA_ONE_SIDED = 7, /* sigma's inverse DFT drops the factor 2 of the bins that stand for a conjugate pair */
   MUT_PCA_ASCENDING = 8,   /* the PCA basis is ordered by increasing eigenvalue */
+  MUT_CONFORMAL_FLOOR = 9, /* the conformal order statistic takes floor((n+1) tau_s) instead of the ceiling */
 };
 static int g_mutation = MUT_NONE;
 void vko_set_mutation(int m) { g_mutation = m; }
@@ -622,6 +623,95 @@ void vko_pca_basis(const vko_view* v, double* eig, double* rot) {
   double M[D_ROPE * D_ROPE];
   vko_second_moment(v, M);
   vko_sym_eig(M, eig, rot);
+}
+
+/* ---------------------------------------------------------------- conformal z (Sec. 4.2; Sec. 5) */
+/* The trigger's certificate multiplier z from calibration queries. One recall target tau fixes the rest: the gate's
+ * false-close budget alpha = (1 - tau)/2, the scan-level target tau_s = tau/(1 - alpha), the smallest calibration set
+ * that can certify it min_hard = ceil(tau_s/(1 - tau_s)), and z = the ceil((n+1) tau_s)-th smallest required inflation
+ * over n hard queries, clamped to Z_max. (Ceilings are taken 1e-9 below the exact value so that a ratio that is an
+ * integer in exact arithmetic is not pushed up by rounding.) */
+double vko_tau_s(double tau) {
+  const double alpha = (1.0 - tau) / 2.0;
+  return tau / (1.0 - alpha);
+}
+
+int64_t vko_min_hard(double tau) {
+  const double ts = vko_tau_s(tau);
+  return (int64_t)ceil(ts / (1.0 - ts) - 1e-9);
+}
+
+static int cmp_double(const void* x, const void* y) {
+  const double a = *(const double*)x, b = *(const double*)y;
+  return (a > b) - (a < b);
+}
+
+/* z from the required inflations zq[0, n) of the hard queries: Z_max when n < min_hard or the order statistic's
+ * index exceeds n, else the k-th smallest (k = ceil((n+1) tau_s), 1-based); the result is clamped to [0, Z_max]. */
+double vko_conformal_quantile(const double* zq, int64_t n, double tau, double z_max) {
+  if (n < vko_min_hard(tau)) return z_max;
+  const double x = (double)(n + 1) * vko_tau_s(tau);
+  const int64_t k = (g_mutation == MUT_CONFORMAL_FLOOR) ? (int64_t)floor(x) : (int64_t)ceil(x - 1e-9);
+  if (k > n || k < 1) return z_max;
+  double* v = (double*)malloc(sizeof(double) * (size_t)n);
+  for (int64_t i = 0; i < n; ++i) v[i] = zq[i];
+  qsort(v, (size_t)n, sizeof(double), cmp_double);
+  double z = v[k - 1];
+  free(v);
+  if (z > z_max) z = z_max;
+  if (z < 0.0) z = 0.0;
+  return z;
+}
+
+/* Every (b, h) is one calibration query. Its exact logits over all N cached rows give the causal argmax u* (ties: the
+ * smaller position); the query is hard when u* lies outside its attended set S_h (idx/count), so that only the recall
+ * tier can bring it back. For a hard query the required inflation is the z at which u*'s trigger score reaches the
+ * tier-1 maximum s* = max over S_h: with sketch rank 0 the index part is idx_t = lambda (a[h,u*] +
+ * |(O qr_h)[r:]| page_res[page(u*)]) and the certificate scale cert_t = lambda |qc_h| eta_u* / sqrt(d_c), d_c = 512,
+ * so zq = (s* - idx_t) / cert_t. a, eta, page_res as from vko_scores and vko_build_index. zq[b,h] gets NaN for a query
+ * that is not hard; ustar[b,h] the argmax row. Returns the number of hard queries. */
+int64_t vko_calib_zq(const vko_view* v, int32_t r, const float* rot, double lam, const double* a, const double* eta,
+                     const double* page_res, const int32_t* idx, const int32_t* count, int32_t cap, double* zq,
+                     int32_t* ustar) {
+  const int64_t N = v->N, P = (N + PAGE - 1) / PAGE;
+  int64_t n_hard = 0;
+#pragma omp parallel for collapse(2) schedule(dynamic) reduction(+ : n_hard)
+  for (int b = 0; b < v->B; ++b) {
+    for (int h = 0; h < v->H; ++h) {
+      const int64_t bh = (int64_t)b * v->H + h;
+      char* in_set = (char*)calloc((size_t)N + 1, 1);
+      int32_t n = count[bh];
+      if (n > cap) n = cap;
+      for (int32_t i = 0; i < n; ++i) in_set[idx[bh * cap + i]] = 1;
+      double best = -INFINITY, sstar = -INFINITY;
+      int64_t us = 0;
+      for (int64_t u = 0; u < N; ++u) {
+        const double s_u = logit(v, b, h, u, lam);
+        if (s_u > best) { best = s_u; us = u; }
+        if (in_set[u] && s_u > sstar) sstar = s_u;
+      }
+      ustar[bh] = (int32_t)us;
+      if (in_set[us]) {
+        zq[bh] = NAN;
+      } else {
+        double q[D_ROPE], qt[D_ROPE], qres = 0.0, qcn = 0.0;
+        for (int j = 0; j < D_ROPE; ++j) q[j] = QR(v, b, h, j);
+        if (r < D_ROPE) {
+          rotate64(rot, q, qt);
+          for (int j = r; j < D_ROPE; ++j) qres += qt[j] * qt[j];
+          qres = sqrt(qres);
+        }
+        for (int j = 0; j < D_LAT; ++j) qcn += QC(v, b, h, j) * QC(v, b, h, j);
+        qcn = sqrt(qcn);
+        const double idx_t = lam * (a[bh * N + us] + qres * page_res[(int64_t)b * P + us / PAGE]);
+        const double cert_t = lam * qcn * eta[(int64_t)b * N + us] / sqrt((double)D_LAT);
+        zq[bh] = (sstar - idx_t) / cert_t;
+        ++n_hard;
+      }
+      free(in_set);
+    }
+  }
+  return n_hard;
 }
 
 int vko_num_threads(void) {
