@@ -186,6 +186,23 @@ int vk_decode_step_noalloc(const vk_view* view, const vk_params* params, const v
                            float* lse, float* smax, int32_t* idx, int32_t* count, int32_t cap, void* stream);
 
 /* ---------------------------------------------------------------------------------------------------------------
+ * Conformal calibration of the trigger's z (Sec. 4.2, Sec. 5 "Recommended configuration"). Every (b, h) of the
+ * view is one calibration query, with its attended set S_h given as vk_decode_step lists it (idx, count, cap; the
+ * tier-1 part of a step with the same params). A query is hard when its exact argmax row over all cached rows (ties:
+ * the smaller position) lies outside S_h; its required inflation is zq = (s* - idx_t) / cert_t, s* the max logit
+ * over S_h, idx_t = lambda (a[h,u*] + |(O Qr_h)[r:]| page_res[page(u*)]), cert_t = lambda |Qc_h| eta_u* / sqrt(512)
+ * (the sketch-rank-0 index part and certificate of Eq. 4). With alpha = (1 - tau)/2, tau_s = tau / (1 - alpha) and
+ * min_hard = ceil(tau_s / (1 - tau_s)), z is the ceil((n+1) tau_s)-th smallest zq over the n hard queries, z_max
+ * when n < min_hard or that index passes n, clamped to [0, z_max]. Outputs (device): zq [B, H] fp32, NaN where the
+ * query is not hard; z_out[3] = {z, z_eff = z / sqrt(512) (the decode step's z_eff), n_hard}. index needs eta and
+ * page_res (and the digest and rotation when r < 64); bf16 caches only (the argmax runs on the tensor-core
+ * attention over every row); B * H <= 16384 (one block sorts the zq). */
+size_t vk_conformal_workspace_bytes(const vk_view* view, const vk_params* params);
+int vk_conformal_z(const vk_view* view, const vk_params* params, const vk_index* index, const int32_t* idx,
+                   const int32_t* count, int32_t cap, float tau, float z_max, float* zq, float* z_out, void* ws,
+                   size_t ws_bytes, void* stream);
+
+/* ---------------------------------------------------------------------------------------------------------------
  * The PCA digest basis (the appendix's branch-width ablation: principal directions of the branch instead of a
  * random rotation). rot [64, 64] row-major fp32 (device): the eigenvectors of M = sum over every row of every
  * sequence of the view of K_u K_u^T, by decreasing eigenvalue, each signed so that its largest entry is positive;

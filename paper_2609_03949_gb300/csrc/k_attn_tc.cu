@@ -91,6 +91,7 @@ struct AttnTcArgs {
   float* part_ml;
   int hold_first;        // VK_FLAG_TEST_TIMEOUT: CTA 0 withholds its first tile's loads
   int* status;
+  int* part_arg;         // ARG instantiation: the row of each partial's max logit, [B][nslot][H]
 };
 
 __device__ __forceinline__ void tma_load_3d_(void* dst, const CUtensorMap* map, int x, int y, int z, uint64_t* bar) {
@@ -215,6 +216,9 @@ struct TilePos {
   }
 };
 
+// ARG (the calibration's instantiation) also tracks, per head, the row of the exact max logit (ties: the smaller
+// row) and writes it beside each partial; the decode step's instantiation does not.
+template <bool ARG>
 __global__ void __launch_bounds__(AT_THREADS, 1) k_attn_tc(const __grid_constant__ CUtensorMap lmap,
                                                          const __grid_constant__ CUtensorMap rmap,
                                                          const __grid_constant__ CUtensorMap qlmap,
@@ -529,6 +533,7 @@ __global__ void __launch_bounds__(AT_THREADS, 1) k_attn_tc(const __grid_constant
     const float L = args.lam_log2e;
     const uint32_t lrow = tmem + ((uint32_t)(32 * q) << 16);
     float m = -INFINITY, mex = -INFINITY, lsum = 0.f;  // lsum: this warp's share of the head's sum
+    int mpos = 0;                                      // ARG: the row of mex
     int u = 0, useg = 0, nseg = 0;
     int sb = 0, shg = 0;                               // the current segment's sequence and head group
     int handled = 0;                                   // rescale requests applied by this warp
@@ -571,6 +576,7 @@ __global__ void __launch_bounds__(AT_THREADS, 1) k_attn_tc(const __grid_constant
       if (own && rh == 0 && hl < nh) {
         args.part_ml[(hbase + hl) * 2] = mex * LN2;
         args.part_ml[(hbase + hl) * 2 + 1] = lt;
+        if constexpr (ARG) args.part_arg[hbase + hl] = mpos;
       }
       // O^T block j on this warp's lanes: dims 128 j + 32 q + lane; columns: heads (blocks 2 rh, 2 rh + 1)
 #pragma unroll 1
@@ -617,6 +623,7 @@ __global__ void __launch_bounds__(AT_THREADS, 1) k_attn_tc(const __grid_constant
         shg = tp.hg;
         useg = 0;
         m = mex = -INFINITY;
+        mpos = 0;
         lsum = 0.f;
       }
       if (!uni) continue;
@@ -639,21 +646,41 @@ __global__ void __launch_bounds__(AT_THREADS, 1) k_attn_tc(const __grid_constant
       tmem_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(&sfree[s]);
-      float mr0 = -INFINITY, mr1 = -INFINITY;
+      float mr;
+      int rpos = 0;                                    // ARG: the tile row of mr
+      if constexpr (ARG) {
+        float best = -INFINITY;
+        int bp = 0;
 #pragma unroll
-      for (int c = 0; c < 32; c += 2) {
-        if ((w >> c) & 1u) mr0 = fmaxf(mr0, sv[c]);
-        if ((w >> (c + 1)) & 1u) mr1 = fmaxf(mr1, sv[c + 1]);
+        for (int c = 0; c < 32; ++c)
+          if (((w >> c) & 1u) && sv[c] > best) { best = sv[c]; bp = 32 * hh + c; }
+        const float ob = __shfl_xor_sync(0xffffffffu, best, 16);
+        const int op = __shfl_xor_sync(0xffffffffu, bp, 16);
+        // the lower row half wins ties: its rows come first
+        const bool mine = hh == 0 ? best >= ob : best > ob;
+        mr = mine ? best : ob;
+        rpos = mine ? bp : op;
+      } else {
+        float mr0 = -INFINITY, mr1 = -INFINITY;
+#pragma unroll
+        for (int c = 0; c < 32; c += 2) {
+          if ((w >> c) & 1u) mr0 = fmaxf(mr0, sv[c]);
+          if ((w >> (c + 1)) & 1u) mr1 = fmaxf(mr1, sv[c + 1]);
+        }
+        mr = fmaxf(mr0, mr1);
+        mr = fmaxf(mr, __shfl_xor_sync(0xffffffffu, mr, 16));
       }
-      float mr = fmaxf(mr0, mr1);
-      mr = fmaxf(mr, __shfl_xor_sync(0xffffffffu, mr, 16));
       // this warp's P rows: 32 hh + 16 rh .. + 15
       const uint32_t w16 = (w >> (16 * rh)) & 0xffffu;
       float pv[16];
 #pragma unroll
       for (int c = 0; c < 16; ++c) pv[c] = rh ? sv[16 + c] : sv[c];
       const float mt = mr * L;
-      mex = fmaxf(mex, mt);
+      if constexpr (ARG) {
+        if (mt > mex) { mex = mt; mpos = tp.kt * AT_T + rpos; }   // an earlier tile keeps a tie
+      } else {
+        mex = fmaxf(mex, mt);
+      }
       float f = 1.f;
       if (mt > m + AT_TAU) {                           // includes the head's first selected row (m = -inf)
         if (m != -INFINITY) f = ex2(m - mt);
@@ -741,7 +768,7 @@ static bool make_map3(CUtensorMap* map, const void* base, uint64_t cols, uint64_
 
 cudaError_t launch_attn_tc(const vk_view& v, float lam, const uint32_t* bitmap, int64_t nw, const AttnGeom& g,
                            int slot0, int nslot, float* part_o, float* part_ml, uint32_t flags, int* status,
-                           cudaStream_t st) {
+                           cudaStream_t st, int* part_arg) {
   if (!encode2()) return cudaErrorNotSupported;
   if (g.G < 1 || g.G > g.total || g.T != (v.N + AT_T - 1) / AT_T || g.n_hg != (v.H + 63) / 64 ||
       g.total != (long long)v.B * g.n_hg * g.T)
@@ -766,10 +793,12 @@ cudaError_t launch_attn_tc(const vk_view& v, float lam, const uint32_t* bitmap, 
   a.part_ml = part_ml;
   a.hold_first = (flags & VK_FLAG_TEST_TIMEOUT) ? 1 : 0;
   a.status = status;
+  a.part_arg = part_arg;
   const size_t smem = AtSmem::total + 1024;
-  cudaError_t e = cudaFuncSetAttribute(k_attn_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  auto kernel = part_arg ? k_attn_tc<true> : k_attn_tc<false>;
+  cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
-  k_attn_tc<<<g.G, AT_THREADS, smem, st>>>(lmap, rmap, qlmap, qrmap, a);
+  kernel<<<g.G, AT_THREADS, smem, st>>>(lmap, rmap, qlmap, qrmap, a);
   count_launches(1);
   return cudaGetLastError();
 }

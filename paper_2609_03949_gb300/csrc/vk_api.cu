@@ -560,6 +560,77 @@ int vk_decode_step(const vk_view* view, const vk_params* params, const vk_index*
   return VK_OK;
 }
 
+namespace {
+// The calibration reuses a two-tier step's layout (tier-1 partials in slots 0 .., the all-rows pass in the second
+// half, the all-rows bitmap in the fired bitmap's place) plus the argmax rows of the all-rows partials.
+vk_params calib_params(const vk_params& p) {
+  vk_params q = p;
+  q.trigger = VK_TRIG_CS;
+  q.top_j = 0;
+  q.flags = 0;
+  return q;
+}
+size_t calib_arg_offset(const VkLayout& L) { return align_up(L.total, 256); }
+size_t calib_bytes(const VkLayout& L, const vk_view& v) {
+  return calib_arg_offset(L) + sizeof(int) * (size_t)v.B * 2 * L.ag.nslot * v.H;
+}
+}  // namespace
+
+size_t vk_conformal_workspace_bytes(const vk_view* view, const vk_params* params) {
+  if (check_view(view) != VK_OK || check_params(view, params) != VK_OK) return 0;
+  const vk_params q = calib_params(*params);
+  return calib_bytes(make_layout(*view, q), *view);
+}
+
+int vk_conformal_z(const vk_view* view, const vk_params* params, const vk_index* index, const int32_t* idx,
+                   const int32_t* count, int32_t cap, float tau, float z_max, float* zq, float* z_out, void* ws,
+                   size_t ws_bytes, void* stream) {
+  g_err[0] = 0;
+  int rc;
+  if ((rc = check_view(view)) != VK_OK || (rc = check_params(view, params)) != VK_OK) return rc;
+  const vk_params q = calib_params(*params);
+  if ((rc = check_index(view, &q, index, true)) != VK_OK) return rc;
+  if (!vk::attn_tc_supported(*view)) return fail(VK_ERR_UNSUPPORTED, "the calibration's argmax pass reads bf16 caches");
+  if (!(tau > 0.f && tau < 1.f)) return fail(VK_ERR_INVALID_ARG, "tau = %g is outside (0, 1)", tau);
+  if (!(z_max >= 0.f) || !std::isfinite(z_max)) return fail(VK_ERR_INVALID_ARG, "z_max must be finite and >= 0");
+  if (!idx || !count || cap < 1 || !zq || !z_out) return fail(VK_ERR_INVALID_ARG, "idx, count, zq, z_out needed, cap >= 1");
+  const int64_t BH = (int64_t)view->B * view->H;
+  if (vk::conformal_smem_bytes(BH) > (size_t)vk::SMEM_BUDGET)
+    return fail(VK_ERR_UNSUPPORTED, "B * H = %lld calibration queries exceed one block's sort", (long long)BH);
+  const VkLayout L = make_layout(*view, q);
+  const size_t need = calib_bytes(L, *view);
+  if (!ws || (reinterpret_cast<uintptr_t>(ws) & 255u) != 0 || ws_bytes < need)
+    return fail(VK_ERR_WORKSPACE, "the calibration workspace needs %zu bytes, 256-byte aligned", need);
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  const vk_view& v = *view;
+  int* status = at<int>(ws, L.off_status);
+  float* qt = at<float>(ws, L.off_qt);
+  float* qcn = at<float>(ws, L.off_qcn);
+  float* qrn = at<float>(ws, L.off_qrn);
+  float* smax1 = at<float>(ws, L.off_smax1);
+  uint32_t* selbm = at<uint32_t>(ws, L.off_selbm);
+  uint32_t* allbm = at<uint32_t>(ws, L.off_firebm);
+  float* po = at<float>(ws, L.off_part_o);
+  float* pml = at<float>(ws, L.off_part_ml);
+  int* parg = at<int>(ws, calib_arg_offset(L));
+  const int ns = L.ag.nslot, nslot = 2 * ns;
+  const double alpha = (1.0 - (double)tau) / 2.0, tau_s = (double)tau / (1.0 - alpha);
+  const int min_hard = (int)std::ceil(tau_s / (1.0 - tau_s) - 1e-9);
+  VK_CUDA(vk::launch_qprep(v, q.r, index->rot, qt, qcn, qrn, at<float>(ws, L.off_qrf), nullptr, st), "qprep");
+  // s*: the max logit over each query's attended set
+  VK_CUDA(vk::launch_list_to_bitmap(v.B, v.H, v.N, idx, count, cap, selbm, L.nw, status, st), "list_to_bitmap");
+  VK_CUDA(vk::launch_attn(v, q.sm_scale, selbm, L.nw, L.ag, 0, nslot, po, pml, 0u, status, st), "attention (S)");
+  VK_CUDA(vk::launch_smax_reduce(v.B, v.H, L.ag, nslot, pml, smax1, st), "smax");
+  // the exact max logit over every row and its row
+  VK_CUDA(cudaMemsetAsync(allbm, 0xff, sizeof(uint32_t) * BH * L.nw, st), "all rows");
+  VK_CUDA(vk::launch_attn_tc(v, q.sm_scale, allbm, L.nw, L.ag, ns, nslot, po, pml, 0u, status, st, parg),
+          "attention (all rows)");
+  VK_CUDA(vk::launch_calib(v, q.r, L.ag, ns, nslot, pml, parg, smax1, selbm, L.nw, qt, qcn, qrn, index->digest,
+                           index->eta, index->page_res, q.sm_scale, tau_s, min_hard, z_max, zq, z_out, st),
+          "conformal z");
+  return VK_OK;
+}
+
 size_t vk_pca_workspace_bytes(void) { return vk::pca_workspace_bytes(); }
 
 int vk_pca_basis(const vk_view* view, float* rot, float* eig, void* ws, size_t ws_bytes, void* stream) {

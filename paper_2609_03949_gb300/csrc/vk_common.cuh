@@ -142,9 +142,11 @@ bool attn_tc_supported(const vk_view& v);
 // CTA count, one per SM.
 int sm_count();
 AttnGeom attn_geom(const vk_view& v);
+// part_arg (bf16 caches, may be NULL): also the row of every partial's max logit, [B][nslot][H] (the calibration's
+// argmax over the attended rows).
 cudaError_t launch_attn_tc(const vk_view& v, float lam, const uint32_t* bitmap, int64_t nw, const AttnGeom& g,
                            int slot0, int nslot, float* part_o, float* part_ml, uint32_t flags, int* status,
-                           cudaStream_t st);
+                           cudaStream_t st, int* part_arg = nullptr);
 cudaError_t launch_attn(const vk_view& v, float lam, const uint32_t* bitmap, int64_t nw, const AttnGeom& g, int slot0,
                         int nslot, float* part_o, float* part_ml, uint32_t flags, int* status, cudaStream_t st);
 cudaError_t launch_smax_reduce(int B, int H, const AttnGeom& g, int nslot, const float* part_ml, float* smax,
@@ -169,6 +171,14 @@ cudaError_t launch_score_tc(const vk_view& v, int r, const void* digest, const v
                             int row_stride, int n_rows, ScoreTcArgs args, cudaStream_t st);
 cudaError_t launch_bitmap_to_list(int B, int H, int N, const uint32_t* bitmap, int64_t nw, int32_t* idx,
                                   int32_t* count, int cap, int* status, cudaStream_t st);
+// conformal calibration (k_calib.cu): per-query required inflations zq [B,H] from the all-rows argmax partials
+// (slots slot0 ..), then z_out = {z, z_eff, n_hard}
+size_t conformal_smem_bytes(int64_t BH);
+cudaError_t launch_calib(const vk_view& v, int r, const AttnGeom& g, int slot0, int nslot, const float* part_ml,
+                         const int* part_arg, const float* smax1, const uint32_t* selbm, int64_t nw, const float* qt,
+                         const float* qcn, const float* qrn, const void* digest, const float* eta,
+                         const float* page_res, float lam, double tau_s, int min_hard, float z_max, float* zq,
+                         float* z_out, cudaStream_t st);
 // PCA digest basis (k_pca.cu): workspace = status word + the fp64 second moment
 size_t pca_workspace_bytes();
 cudaError_t launch_pca_basis(const vk_view& v, float* rot, float* eig, void* ws, cudaStream_t st);

@@ -76,6 +76,8 @@ def lib():
             "vk_last_error": ([], ctypes.c_char_p),
             "vk_sigma_workspace_bytes": ([I32, I32], SZ),
             "vk_pca_workspace_bytes": ([], SZ),
+            "vk_conformal_workspace_bytes": ([VP, PP], SZ),
+            "vk_conformal_z": ([VP, PP, IP, P, P, I32, ctypes.c_float, ctypes.c_float, P, P, P, SZ, P], ctypes.c_int),
             "vk_pca_basis": ([VP, P, P, P, SZ, P], ctypes.c_int),
             "vk_sigma": ([VP, I32, I32, P, P, SZ, P], ctypes.c_int),
             "vk_sigma_select": ([I32, I32, I32, P, I32, I64, P, P, I32, P, SZ, P], ctypes.c_int),
@@ -93,7 +95,8 @@ def exported_symbols():
     return ["vk_keep_count", "vk_min_cap", "vk_workspace_bytes", "vk_build_digest", "vk_score", "vk_select",
             "vk_sparse_attn", "vk_decode_step", "vk_decode_step_noalloc", "vk_workspace_init", "vk_poll_status",
             "vk_profile_set_events", "vk_profile_launches", "vk_last_error", "vk_sigma_workspace_bytes", "vk_sigma",
-            "vk_sigma_select", "vk_pca_workspace_bytes", "vk_pca_basis"]
+            "vk_sigma_select", "vk_pca_workspace_bytes", "vk_pca_basis", "vk_conformal_workspace_bytes",
+            "vk_conformal_z"]
 
 
 def _check(rc: int):
@@ -281,3 +284,18 @@ def vk_pca_basis(view, rot, eig=None, ws=None, stream=None) -> None:
         ws = alloc_bytes(int(lib().vk_pca_workspace_bytes()))
     _check(lib().vk_pca_basis(ctypes.byref(view), _ptr(rot), _ptr(eig), _ptr(ws), ws.numel() * ws.element_size(),
                               _stream(stream)))
+
+
+# ------------------------------------------------------------------------------------------------ conformal z
+def vk_conformal_z(view, params, index, idx, count, zq, z_out, tau: float = 0.9, z_max: float = 8.0, ws=None,
+                   stream=None) -> None:
+    """Calibrate the trigger's z from every (b, h) as a calibration query (S_h given by idx/count)."""
+    if ws is None:
+        n = int(lib().vk_conformal_workspace_bytes(ctypes.byref(view), ctypes.byref(params)))
+        if n == 0:
+            raise VkError(VK_ERR_INVALID_ARG, lib().vk_last_error().decode())
+        ws = alloc_bytes(n)
+    _check(lib().vk_conformal_z(ctypes.byref(view), ctypes.byref(params), ctypes.byref(index), _ptr(idx), _ptr(count),
+                                idx.shape[-1], float(tau), float(z_max), _ptr(zq), _ptr(z_out), _ptr(ws),
+                                ws.numel() * ws.element_size(), _stream(stream)))
+    return ws
