@@ -14,11 +14,17 @@ template <typename T>
 __host__ __device__ __forceinline__ const T* tptr(const void* p) { return reinterpret_cast<const T*>(p); }
 
 // ---------------------------------------------------------------------------------------------- query prep
-// One warp per (b, h); lane l owns RoPE coordinates l and l + 32.
+// One warp per (b, h); lane l owns RoPE coordinates l and l + 32. With a digest the block first stages the 64 x 64
+// rotation in shared memory (transposed and padded, so that the lanes' reads of one column hit distinct banks).
 template <typename T>
 __global__ void k_qprep(const T* __restrict__ q_latent, const T* __restrict__ q_rope, int BH, int H, int r,
                         const float* __restrict__ rot, float* __restrict__ qt, float* __restrict__ qcn,
                         float* __restrict__ qrn, float* __restrict__ qrf, __nv_bfloat16* __restrict__ qhl) {
+  __shared__ float rot_t[D_ROPE][D_ROPE + 1];        // rot_t[i][j] = O[j][i]
+  if (r < D_ROPE) {
+    for (int e = threadIdx.x; e < D_ROPE * D_ROPE; e += blockDim.x) rot_t[e % D_ROPE][e / D_ROPE] = rot[e];
+    __syncthreads();
+  }
   const int warp = (blockIdx.x * blockDim.x + threadIdx.x) >> 5, lane = threadIdx.x & 31;
   if (warp >= BH) return;
   const T* qc = q_latent + (int64_t)warp * D_LAT;
@@ -35,8 +41,8 @@ __global__ void k_qprep(const T* __restrict__ q_latent, const T* __restrict__ q_
     y0 = 0.f; y1 = 0.f;
     for (int i = 0; i < D_ROPE; ++i) {
       float qi = __shfl_sync(0xffffffffu, i < 32 ? q0 : q1, i & 31);
-      y0 = fmaf(rot[lane * D_ROPE + i], qi, y0);
-      y1 = fmaf(rot[(lane + 32) * D_ROPE + i], qi, y1);
+      y0 = fmaf(rot_t[i][lane], qi, y0);
+      y1 = fmaf(rot_t[i][lane + 32], qi, y1);
     }
   }
   float res = 0.f;
@@ -87,6 +93,11 @@ __global__ void k_build_digest(const T* __restrict__ latent, int64_t lld, int64_
                                const float* __restrict__ rot, __nv_bfloat16* __restrict__ digest,
                                float* __restrict__ eta, float* __restrict__ page_res, float* __restrict__ page_knorm,
                                float* __restrict__ page_eta) {
+  __shared__ float rot_t[D_ROPE][D_ROPE + 1];        // rot_t[i][j] = O[j][i] (staged once per block)
+  if (r < D_ROPE) {
+    for (int e = threadIdx.x; e < D_ROPE * D_ROPE; e += blockDim.x) rot_t[e % D_ROPE][e / D_ROPE] = rot[e];
+    __syncthreads();
+  }
   const int64_t row = (int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
   const int lane = threadIdx.x & 31;
   if (row >= total_rows) return;
@@ -113,8 +124,8 @@ __global__ void k_build_digest(const T* __restrict__ latent, int64_t lld, int64_
     float y0 = 0.f, y1 = 0.f;
     for (int i = 0; i < D_ROPE; ++i) {
       float ki = __shfl_sync(0xffffffffu, i < 32 ? k0 : k1, i & 31);
-      y0 = fmaf(rot[lane * D_ROPE + i], ki, y0);
-      y1 = fmaf(rot[(lane + 32) * D_ROPE + i], ki, y1);
+      y0 = fmaf(rot_t[i][lane], ki, y0);
+      y1 = fmaf(rot_t[i][lane + 32], ki, y1);
     }
     if (digest) {
       if (lane < r) digest[row * r + lane] = __float2bfloat16_rn(y0);

@@ -10,9 +10,10 @@
 //   phase 1  C^T [64 dims x mp] = R^T Phi, accumulated over the block's 128-row chunks: A = the R chunk read
 //            MN-major straight from its TMA tile, B = the Phi^T chunk; M = 64, N = mp, K = 128 per chunk;
 //   phase 2  low [128 rows x 64 dims] = Phi_chunk C: A = the Phi chunk, B = C rounded to bf16 by the epilogue into
-//            shared memory; M = 128, N = 64, K = mp. The epilogue (one thread per row) reads the row's low part
-//            from tensor memory and the row itself from global memory (phase 1 read it just before, so it comes
-//            from L2), and writes sigma.
+//            shared memory; M = 128, N = 64, K = mp, into one of four tensor-memory buffers. The R chunk is loaded
+//            again (phase 1 read it just before, so it comes from L2) into a ring of its own, and the epilogue (one
+//            thread per row) takes the row's low part from tensor memory and the row from shared memory, and
+//            writes sigma.
 // Roles: warp 0 TMA producer, warp 1 MMA issuer, warps 2..5 epilogue (one per tensor-memory lane quarter).
 // Phi is built in the workspace in bf16 twice: Phi^T [mp][T] and Phi [T][mp] (mp = 64 for kappa <= 32, else 128).
 // Rows past the last closed block (the open tail) get sigma = -1. Every wait is bounded.
@@ -37,9 +38,12 @@ struct SgCfg {
   static constexpr uint32_t PHT = 2 * MP * 128;          // Phi^T chunk: two 64-row K blocks of MP x 128 B
   static constexpr uint32_t STAGE = SG_RBYTES + PHT;     // phase 1 stage (phase 2 uses the first MP / 64 x 16 KB)
   static constexpr int STAGES = MP == 64 ? 4 : 3;
+  static constexpr int R2 = MP == 64 ? 4 : 3;            // phase 2 ring of R chunks for the epilogue
+  static constexpr int NL = 4;                           // tensor-memory buffers of the phase 2 product
   static constexpr uint32_t cbuf = STAGES * STAGE;       // C as the phase 2 B operand: MP / 64 blocks of 64 x 128 B
-  static constexpr uint32_t bars = cbuf + 64 * MP * 2;
-  static constexpr uint32_t total = bars + (2 * STAGES + 6) * 8 + 1024;
+  static constexpr uint32_t r2 = cbuf + 64 * MP * 2;
+  static constexpr uint32_t bars = r2 + R2 * SG_RBYTES;
+  static constexpr uint32_t total = bars + (2 * STAGES + 2 * R2 + 2 + 2 * NL) * 8 + 1024;
   static_assert(total <= 232448, "sigma shared memory exceeds the 227 KB opt-in limit");
 };
 
@@ -131,25 +135,29 @@ __global__ void __launch_bounds__(SG_THREADS, 1) k_sigma(const __grid_constant__
   uint64_t* empty = bars + L::STAGES;      // [STAGES]
   uint64_t* c_full = empty + L::STAGES;    // phase 1 of an item is complete
   uint64_t* c_ready = c_full + 1;          // the epilogue has written C (bf16) for phase 2
-  uint64_t* l_full = c_ready + 1;          // [2] a phase 2 chunk's low part is in tensor memory
-  uint64_t* l_empty = l_full + 2;          // [2] the epilogue has read it
+  uint64_t* l_full = c_ready + 1;          // [NL] a phase 2 chunk's low part is in tensor memory
+  uint64_t* l_empty = l_full + L::NL;      // [NL] the epilogue has read it
+  uint64_t* r_full = l_empty + L::NL;      // [R2] a phase 2 R chunk has landed
+  uint64_t* r_empty = r_full + L::R2;      // [R2] the epilogue is done with it
+  unsigned char* rbuf = smem + L::r2;
   __shared__ uint32_t tmem_base;
   __shared__ int abort_flag;
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const long long i0 = args.items * blockIdx.x / gridDim.x, i1 = args.items * (blockIdx.x + 1) / gridDim.x;
   const int nchunk = args.T / SG_CH;
-  constexpr uint32_t C_COL = 0, L_COL = 128;               // tensor memory: C^T, then two 64-column low buffers
+  constexpr uint32_t C_COL = 0, L_COL = 128;               // tensor memory: C^T, then four 64-column low buffers
 
   if (threadIdx.x == 0) {
     abort_flag = 0;
     for (int s = 0; s < L::STAGES; ++s) { mbar_init(&full[s], 1); mbar_init(&empty[s], 1); }
     mbar_init(c_full, 1);
     mbar_init(c_ready, 4);
-    for (int i = 0; i < 2; ++i) { mbar_init(&l_full[i], 1); mbar_init(&l_empty[i], 4); }
+    for (int i = 0; i < L::NL; ++i) { mbar_init(&l_full[i], 1); mbar_init(&l_empty[i], 4); }
+    for (int i = 0; i < L::R2; ++i) { mbar_init(&r_full[i], 1); mbar_init(&r_empty[i], 4); }
     mbar_fence_init();
   }
-  if (warp == 1) tmem_alloc(&tmem_base, 256);
+  if (warp == 1) tmem_alloc(&tmem_base, 512);
   tmem_fence_before();
   __syncthreads();
   tmem_fence_after();
@@ -158,7 +166,7 @@ __global__ void __launch_bounds__(SG_THREADS, 1) k_sigma(const __grid_constant__
   if (warp == 0) {
     // ------------------------------------------------------------------ producer
     if (lane == 0) {
-      int n = 0;                                          // loads issued (ring position)
+      int n = 0, n2 = 0;                                  // loads issued into the ring and into the R ring
       bool ok = true;
       for (long long it = i0; it < i1 && ok; ++it) {
         const int b = (int)(it / args.nb), blk = (int)(it - (long long)b * args.nb);
@@ -176,6 +184,11 @@ __global__ void __launch_bounds__(SG_THREADS, 1) k_sigma(const __grid_constant__
             } else {
               mbar_arrive_expect_tx(&full[s], (uint32_t)MP * 256u);
               for (int kb = 0; kb < MP / 64; ++kb) sg_tma_2d(st + kb * 16384, &pmap, 64 * kb, u0, &full[s]);
+              const int s2 = n2 % L::R2, use2 = n2 / L::R2;
+              if (use2 > 0 && !mbar_wait(&r_empty[s2], (use2 - 1) & 1, &abort_flag)) { ok = false; ++n; break; }
+              mbar_arrive_expect_tx(&r_full[s2], SG_RBYTES);
+              sg_tma_3d(rbuf + s2 * SG_RBYTES, &rmap, 0, blk * args.T + u0, b, &r_full[s2]);
+              ++n2;
             }
           }
         }
@@ -183,6 +196,7 @@ __global__ void __launch_bounds__(SG_THREADS, 1) k_sigma(const __grid_constant__
       if (!ok) abort_flag = 1;
       // drain: the last load of every stage has landed before the CTA may leave (already true unless it aborted)
       for (int k = std::max(0, n - L::STAGES); k < n; ++k) mbar_wait(&full[k % L::STAGES], (k / L::STAGES) & 1, nullptr);
+      for (int k = std::max(0, n2 - L::R2); k < n2; ++k) mbar_wait(&r_full[k % L::R2], (k / L::R2) & 1, nullptr);
     }
   } else if (warp == 1) {
     // ------------------------------------------------------------------ MMA issuer
@@ -216,7 +230,7 @@ __global__ void __launch_bounds__(SG_THREADS, 1) k_sigma(const __grid_constant__
         const uint32_t cba = smem_addr(cb);
         for (int c = 0; c < nchunk; ++c, ++n, ++nl) {
           const int s = n % L::STAGES, use = n / L::STAGES;
-          const int lb = nl & 1, luse = nl >> 1;
+          const int lb = nl % L::NL, luse = nl / L::NL;
           if (!mbar_wait(&full[s], use & 1, &abort_flag)) { ok = false; break; }
           if (luse > 0 && !mbar_wait(&l_empty[lb], (luse - 1) & 1, &abort_flag)) { ok = false; break; }
           tmem_fence_after();
@@ -275,10 +289,15 @@ __global__ void __launch_bounds__(SG_THREADS, 1) k_sigma(const __grid_constant__
       tmem_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(c_ready);
-      // phase 2: one row per thread
+      // phase 2: one row per thread; the row from the R ring (128-byte swizzle: chunk k of row x sits at k ^ (x & 7))
       for (int c = 0; c < nchunk; ++c, ++nl) {
-        const int lb = nl & 1, luse = nl >> 1;
-        if (!warp_wait_sg(&l_full[lb], luse & 1, &abort_flag, lane)) { ok = false; break; }
+        const int lb = nl % L::NL, luse = nl / L::NL;
+        const int s2 = nl % L::R2, use2 = nl / L::R2;
+        if (!warp_wait_sg(&l_full[lb], luse & 1, &abort_flag, lane) ||
+            !warp_wait_sg(&r_full[s2], use2 & 1, &abort_flag, lane)) {
+          ok = false;
+          break;
+        }
         tmem_fence_after();
         float lo[64];
         sg_ld32(tmem + lq + L_COL + 64 * lb, lo);
@@ -287,12 +306,18 @@ __global__ void __launch_bounds__(SG_THREADS, 1) k_sigma(const __grid_constant__
         tmem_fence_before();
         __syncwarp();
         if (lane == 0) mbar_arrive(&l_empty[lb]);
-        const int u = blk * args.T + c * SG_CH + 32 * q + lane;
-        const uint4* rr = reinterpret_cast<const uint4*>(args.rope + (int64_t)b * args.rbs + (int64_t)u * args.rld);
+        const int x = 32 * q + lane;                      // row within the chunk
+        const int u = blk * args.T + c * SG_CH + x;
+        const unsigned char* rrow = rbuf + s2 * SG_RBYTES + x * 128;
+        uint4 rv[8];
+#pragma unroll
+        for (int k = 0; k < 8; ++k) rv[k] = *reinterpret_cast<const uint4*>(rrow + ((k ^ (x & 7)) * 16));
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&r_empty[s2]);
         float acc = 0.f;
 #pragma unroll
         for (int k = 0; k < 8; ++k) {
-          const uint4 w = rr[k];
+          const uint4 w = rv[k];
           const uint32_t ww[4] = {w.x, w.y, w.z, w.w};
 #pragma unroll
           for (int e = 0; e < 4; ++e) {
@@ -313,7 +338,7 @@ __global__ void __launch_bounds__(SG_THREADS, 1) k_sigma(const __grid_constant__
   __syncthreads();
   if (warp == 1) {
     tmem_fence_after();
-    tmem_dealloc(tmem, 256);
+    tmem_dealloc(tmem, 512);
   }
 }
 
