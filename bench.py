@@ -1,16 +1,18 @@
 """Benchmark of the sparse MLA decode step (VestigeKV hot path) on GB300.
 
-Workload: a Kimi-K2-shaped layer (64 heads, 512 latent + 64 RoPE, bf16 cache), N = 65536 cached rows per
-sequence, rho = 1/32, r = 64, recent window 256, 64 planted rows per sequence, a batch of 64 independent
-decode sequences per GPU (weak scaling: every rank owns its own 64 sequences). Metric: decode query-tokens/s
-per layer (one query token per sequence per step).
+Default workload (the metric's): a Kimi-K2-shaped layer (64 heads, 512 latent + 64 RoPE, bf16 cache), N = 65536
+cached rows per sequence, rho = 1/32, r = 64, recent window 256, 64 planted rows per sequence, a batch of 64
+independent decode sequences per GPU (weak scaling: every rank owns its own 64 sequences). Metric: decode
+query-tokens/s per layer (one query token per sequence per step). ``--config`` selects one of the other evaluation
+workloads of datagen.CONFIGS instead (the fp32 tiny layer, the DeepSeek-V2-shaped layers, the log-normal-key layer,
+the two-tier layer), with its own selection parameters.
 
 Prints one JSON line (rank 0). `value` times the steps alone (device events on the launching stream); a second
 pass of the same steps records the library's stage events for the breakdown and the roofline of the dominant
 kernel. `e2e` runs the steps through the same entry point with each step's queries copied in from pinned host
-memory and its outputs copied back, on copy streams that overlap the neighbouring steps. `python bench.py --impl
-reference` times the CPU oracle on the same workload instead (a bounded sample of sequences per step), on the host
-cores.
+memory and its outputs copied back, on copy streams that overlap the neighbouring steps. On the default workload the
+line also carries the sigma selector kernel's throughput over the same cache. `python bench.py --impl reference`
+times the CPU oracle on the same workload instead (a bounded sample of sequences per step), on the host cores.
 """
 from __future__ import annotations
 
@@ -29,12 +31,54 @@ sys.path.insert(0, ROOT)
 import numpy as np  # noqa: E402
 import torch  # noqa: E402
 
-H, N, RHO, WINDOW, R, N_PLANTED = 64, 65536, 1 / 32, 256, 64, 64
-B_PER_GPU = 64
-METRIC = "decode query-tokens/s per layer at N=64K, rho=1/32"
-N_DEFAULT = N
+from paper_2609_03949_gb300 import datagen  # noqa: E402
+
+DEFAULT_CONFIG = "h64_n64k"
+B_PER_GPU = 64                 # sequences per GPU on the default workload
+N_DEFAULT = 65536
 UNIT = "query-tokens/s"
 STAGES = ["qprep", "score", "select", "attn", "trigger", "combine"]
+
+
+class Workload:
+    """The benchmarked workload: sizes, selection parameters and the metric's name."""
+
+    def __init__(self, name: str, B: int | None, N: int | None, rho: float | None, r: int | None):
+        self.name = name
+        c, p = datagen.CONFIGS[name], datagen.CONFIG_PARAMS[name]
+        self.H, self.dtype = c["H"], c["dtype"]
+        self.B = B if B is not None else (B_PER_GPU if name == DEFAULT_CONFIG else c["B"])
+        self.N = N if N is not None else (N_DEFAULT if name == DEFAULT_CONFIG else c["N"])
+        self.rho = rho if rho is not None else p["rho"]
+        self.r = r if r is not None else p["r"]
+        self.window = p["window"]
+        self.trigger = p.get("trigger", 0)
+        self.z_eff = p.get("z_eff", 1.0)
+        self.n_planted = c["n_planted"]
+        self.lognormal = c.get("lognormal_keys", False)
+        self.seed = c["seed"]
+        n = self.N
+        nk = f"{n // 1024}K" if n % 1024 == 0 else str(n)
+        rho_s = f"1/{round(1 / self.rho)}" if self.rho < 1 else "1"
+        self.metric = f"decode query-tokens/s per layer at N={nk}, rho={rho_s}"
+        if name != DEFAULT_CONFIG:
+            self.metric += f" ({name})"
+
+    def describe(self, n_gpus: int) -> dict:
+        B, N = self.B, self.N
+        esz = 2 if self.dtype == "bf16" else 4
+        rows = B * N * 576 * esz
+        return {"workload": f"sparse MLA decode step: {self.name}, H={self.H}, N={N}, rho={self.rho:g}, r={self.r}, "
+                            f"window={self.window}, {self.dtype} cache [512 latent + 64 RoPE]"
+                            f"{', two-tier trigger z_eff=%g' % self.z_eff if self.trigger else ''}, "
+                            f"{self.n_planted} planted rows/seq, B={B} sequences per GPU",
+                "heads": self.H, "context": N, "rho": self.rho, "r": self.r, "window": self.window,
+                "batch_per_gpu": B, "global_batch": B * n_gpus, "trigger": self.trigger,
+                "parallelism": f"independent sequences x{n_gpus} (no collective)",
+                "l2": (f"inputs larger than L2: each step streams a {rows / 1e9:.1f} GB cache per GPU (L2 is 129 MB)"
+                       if rows >= 4 * 129e6 else
+                       f"L2 flushed before every step (512 MB write outside the step's events; the cache is "
+                       f"{rows / 1e6:.0f} MB)")}
 
 
 def parse():
@@ -43,21 +87,16 @@ def parse():
     ap.add_argument("--steps", type=int, default=50)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="native", choices=["native", "reference"])
-    ap.add_argument("--batch", type=int, default=B_PER_GPU)
+    ap.add_argument("--config", default=DEFAULT_CONFIG, choices=sorted(datagen.CONFIGS),
+                    help="evaluation workload (default: the metric's, H=64, N=65536, rho=1/32, B=64)")
+    ap.add_argument("--batch", type=int, default=None)
+    ap.add_argument("--context", type=int, default=None, help="cached rows per sequence")
+    ap.add_argument("--rho", type=float, default=None)
+    ap.add_argument("--r", type=int, default=None, help="score width: 64 or a digest width")
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--context", type=int, default=N_DEFAULT,
-                    help="cached rows per sequence (default 65536, the workload the metric is quoted on)")
     args = ap.parse_args()
-    set_context(args.context)
+    args.wl = Workload(args.config, args.batch, args.context, args.rho, args.r)
     return args
-
-
-def set_context(n: int):
-    """Other context lengths for sweeps: the metric names its N."""
-    global N, METRIC
-    N = n
-    METRIC = (f"decode query-tokens/s per layer at N={n // 1024}K, rho=1/32" if n % 1024 == 0
-              else f"decode query-tokens/s per layer at N={n}, rho=1/32")
 
 
 def dist_env():
@@ -84,17 +123,6 @@ def max_over_ranks(ms: float, pg, device) -> float:
 def job_throughput(seqs_per_rank: int, world: int, ms_per_step: float) -> float:
     """Whole-job query-tokens/s: every rank's sequences (one query token each) over the slowest rank's step."""
     return seqs_per_rank * world / (ms_per_step * 1e-3)
-
-
-def workload_config(B, n_gpus):
-    return {"workload": f"sparse MLA decode step: H={H}, N={N}, rho=1/32, r={R}, window={WINDOW}, bf16 cache "
-                        f"[512 latent + 64 RoPE], {N_PLANTED} planted rows/seq, B={B} sequences per GPU",
-            "heads": H, "context": N, "rho": RHO, "r": R, "window": WINDOW, "batch_per_gpu": B,
-            "global_batch": B * n_gpus, "parallelism": f"independent sequences x{n_gpus} (no collective)",
-            "l2": (f"inputs larger than L2: each step streams a {B * N * 1152 / 1e9:.1f} GB cache per GPU (L2 is 129 MB)"
-                   if B * N * 1152 >= 4 * 129e6 else
-                   f"L2 flushed before every step (512 MB write outside the step's events; the cache is "
-                   f"{B * N * 1152 / 1e6:.0f} MB)")}
 
 
 def peaks():
@@ -198,27 +226,46 @@ def kernel_traffic(kernel: str):
 
 
 # ------------------------------------------------------------------------------------------------ CPU oracle
-def oracle_baseline(cache_dev, ql_dev, qr_dev, budget_s=12.0, max_seqs=1024):
-    """The CPU oracle, as it stands, on a bounded sample of this workload's sequences (host cores)."""
+def make_host_workload(w: Workload, B: int, seed: int, device="cpu"):
+    return datagen.config_workload(w.name, device=device, B=B, N=w.N, seed=seed)
+
+
+def oracle_step(hi, digest, w: Workload):
     import oracle
-    from paper_2609_03949_gb300 import datagen
-    done, t_total = 0, 0.0
-    while done < max_seqs and (t_total < budget_s or done == 0):
-        b = done % cache_dev.shape[0]
-        wl = datagen.Workload(B=1, H=H, N=N, dtype="bf16", cache=cache_dev[b:b + 1].cpu(),
-                              q_latent=ql_dev[b:b + 1].cpu(), q_rope=qr_dev[b:b + 1].cpu(),
-                              rot=torch.eye(64), planted_pos=torch.zeros(1, 0, dtype=torch.int64),
-                              planted_head=torch.zeros(0, dtype=torch.int64), seed=0)
-        hi = oracle.HostInputs(wl)
-        t0 = time.perf_counter()
-        oracle.decode_step(hi, rho=RHO, window=WINDOW)
-        t_total += time.perf_counter() - t0
-        done += 1
-        if done == 1 and t_total * max_seqs > 4 * budget_s:
-            max_seqs = max(1, int(budget_s / t_total))
-    return {"value": done / t_total, "unit": UNIT, "cores": oracle.num_threads(), "kind": "oracle",
-            "sample": f"{done} sequence(s) of the bench workload (N={N}, H={H}) through the fp64 C oracle's "
-                      f"whole decode step, {t_total:.1f} s"}
+    return oracle.decode_step(hi, rho=w.rho, r=w.r, window=w.window, trigger=w.trigger, z_eff=w.z_eff,
+                              digest_bf16=digest)
+
+
+def oracle_inputs(wl, w: Workload):
+    import oracle
+    hi = oracle.HostInputs(wl)
+    dig = oracle.build_index(hi, w.r)[1] if w.r < 64 else None
+    return hi, dig
+
+
+def oracle_baseline(wl_dev, w: Workload, threads: int | None = None, budget_s=12.0, max_seqs=1024):
+    """The CPU oracle, as it stands, on a bounded sample of this workload's sequences (host cores, or `threads`)."""
+    import oracle
+    if threads:
+        oracle.set_threads(threads)
+    try:
+        done, t_total = 0, 0.0
+        while done < max_seqs and (t_total < budget_s or done == 0):
+            b = done % wl_dev.B
+            hi, dig = oracle_inputs(wl_dev.slice_batch([b]), w)
+            t0 = time.perf_counter()
+            oracle_step(hi, dig, w)
+            t_total += time.perf_counter() - t0
+            done += 1
+            if done == 1 and t_total * max_seqs > 4 * budget_s:
+                max_seqs = max(1, int(budget_s / t_total))
+        cores = oracle.num_threads()
+    finally:
+        if threads:
+            oracle.set_threads(os.cpu_count() or 1)
+    return {"value": done / t_total, "unit": UNIT, "cores": cores, "kind": "oracle",
+            "sample": f"{done} sequence(s) of the bench workload ({w.name}, N={w.N}, H={w.H}) through the fp64 C "
+                      f"oracle's whole decode step, {t_total:.1f} s"}
 
 
 def run_reference(args):
@@ -226,28 +273,53 @@ def run_reference(args):
     if rank != 0:
         return
     import oracle
-    from paper_2609_03949_gb300 import datagen
-    wl = datagen.make_workload(2, H, N, seed=1000, n_planted=N_PLANTED, planted_hi=N - WINDOW, device="cpu")
-    his = [oracle.HostInputs(wl.slice_batch([b])) for b in range(wl.B)]
+    w = args.wl
+    wl = make_host_workload(w, 2, seed=w.seed)
+    inputs = [oracle_inputs(wl.slice_batch([b]), w) for b in range(wl.B)]
     warm = max(3, args.warmup)
     for i in range(warm):
-        oracle.decode_step(his[i % 2], rho=RHO, window=WINDOW)
+        oracle_step(*inputs[i % 2], w)
     t0 = time.perf_counter()
     for i in range(args.steps):
-        oracle.decode_step(his[i % 2], rho=RHO, window=WINDOW)
+        oracle_step(*inputs[i % 2], w)
     dt = time.perf_counter() - t0
     value = args.steps / dt
-    line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus, "steps": args.steps,
+    line = {"metric": w.metric, "value": value, "unit": UNIT, "n_gpus": args.gpus, "steps": args.steps,
             "warmup": warm, "ms_per_step": 1e3 * dt / args.steps, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic (seeded, bf16 storage)",
-            "impl": "reference", "config": workload_config(args.batch, args.gpus),
+            "impl": "reference", "config": w.describe(args.gpus),
             "cpu_baseline": {"value": value, "unit": UNIT, "cores": oracle.num_threads(), "kind": "oracle",
-                             "sample": f"each step: 1 sequence (N={N}, H={H}) through the fp64 C oracle"},
+                             "sample": f"each step: 1 sequence (N={w.N}, H={w.H}) through the fp64 C oracle"},
             "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
 
 
 # ------------------------------------------------------------------------------------------------ native
+def sigma_throughput(vk, view, B, N, stream, hbm_peak, T=4096, kappa=16, reps=5):
+    """The sigma selector kernel over the bench cache (every closed block of T rows): its time and the algorithmic
+    bytes (each row's 64 RoPE columns read once, 128 B) against the copy bandwidth."""
+    if (N // T) == 0:
+        return None
+    ws = vk.alloc_bytes(vk.vk_sigma_workspace_bytes(T, kappa))
+    sig = torch.empty(B, N, device="cuda")
+    for _ in range(2):
+        vk.vk_sigma(view, T, kappa, sig, ws)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    torch.cuda.synchronize()
+    e0.record(stream)
+    for _ in range(reps):
+        vk.vk_sigma(view, T, kappa, sig, ws)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    ms = e0.elapsed_time(e1) / reps
+    assert vk.vk_poll_status(ws) == vk.VK_OK
+    byts = B * (N // T) * T * 128
+    gbs = byts / (ms * 1e-3) / 1e9
+    return {"kernel": "k_sigma", "T": T, "kappa": kappa, "blocks": B * (N // T), "ms": ms,
+            "algorithmic_bytes": byts, "achieved_gbs": gbs, "frac_of_peak": gbs / hbm_peak,
+            "bound": "hbm (two bf16 contractions of 64 x 31 per row: 32 flop/B, below the tensor ridge)"}
+
+
 def run_native(args):
     rank, world, local = dist_env()
     if args.gpus != world and world > 1:
@@ -259,23 +331,34 @@ def run_native(args):
         import torch.distributed as dist
         dist.init_process_group("nccl", device_id=dev)
         pg = dist
-    from paper_2609_03949_gb300 import _build, datagen, vk
+    from paper_2609_03949_gb300 import _build, vk
     if rank == 0 or not os.path.exists(vk.LIB_PATH):
         _build.build()
     if pg:
         pg.barrier()
     vk.lib()
-    B = args.batch
-    wl = datagen.make_workload(B, H, N, seed=rank_seed(rank), n_planted=N_PLANTED, planted_hi=N - WINDOW,
-                               device=dev)
+    w = args.wl
+    B, N, H = w.B, w.N, w.H
+    seed = rank_seed(rank) if w.name == DEFAULT_CONFIG else w.seed + 7919 * rank
+    wl = make_host_workload(w, B, seed=seed, device=dev)
     view = vk.make_view(wl.cache, wl.q_latent, wl.q_rope)
-    params = vk.make_params(RHO, r=R, window=WINDOW)
+    params = vk.make_params(w.rho, r=w.r, window=w.window, trigger=w.trigger, z_eff=w.z_eff)
+    # the per-cache index (built once, off the step): digest for r < 64, norms for the trigger
+    index = None
+    if w.r < 64 or w.trigger:
+        P = (N + 63) // 64
+        dig = torch.empty(B, N, w.r, dtype=torch.bfloat16, device=dev) if w.r < 64 else None
+        rot = wl.rot.contiguous()
+        eta = torch.empty(B, N, device=dev)
+        pres, pk, pe = (torch.empty(B, P, device=dev) for _ in range(3))
+        vk.vk_build_digest(view, params, rot, dig, eta, pres, pk, pe)
+        index = vk.make_index(dig, eta, pres, rot if w.r < 64 else None, pk, pe)
     buf = vk.DecodeBuffers(view, params, device=dev)
     stream = torch.cuda.current_stream(dev)
 
     # ---- device-timed region: inputs resident in HBM, per-stage CUDA events on the launching stream
     for _ in range(max(3, args.warmup)):
-        buf.run(view, params)
+        buf.run(view, params, index)
     torch.cuda.synchronize()
     assert vk.vk_poll_status(buf.ws) == vk.VK_OK
     step_events = [[torch.cuda.Event(enable_timing=True) for _ in range(7)] for _ in range(args.steps)]
@@ -284,8 +367,9 @@ def run_native(args):
         for e in evs:
             e.record(stream)
     torch.cuda.synchronize()
+    esz = 2 if w.dtype == "bf16" else 4
     # a cache that L2 could hold is evicted between steps by a 512 MB write outside the steps' events
-    flush = torch.empty(512 << 20, dtype=torch.uint8, device=dev) if B * N * 1152 < 4 * 129e6 else None
+    flush = torch.empty(512 << 20, dtype=torch.uint8, device=dev) if B * N * 576 * esz < 4 * 129e6 else None
     clocks = ClockSampler(local)
     clocks.start()
     time.sleep(0.3)
@@ -303,7 +387,7 @@ def run_native(args):
         if flush is not None:
             flush.fill_(1)
             sb.record(stream)
-        buf.run(view, params)
+        buf.run(view, params, index)
         if flush is not None:
             se.record(stream)
     t_end.record(stream)
@@ -324,7 +408,7 @@ def run_native(args):
         if flush is not None:
             flush.fill_(1)
         vk.vk_profile_set_events(evs)
-        buf.run(view, params)
+        buf.run(view, params, index)
     torch.cuda.synchronize()
     vk.vk_profile_set_events([])
     for evs in step_events:
@@ -335,23 +419,25 @@ def run_native(args):
     dev_ms_step = total_ms_events / args.steps
     stage_ms /= args.steps
 
-    # ---- algorithmic bytes (union of the heads' selections, per sequence, summed)
-    from paper_2609_03949_gb300.bytes_model import step_bytes
-    U = union_rows(buf.idx, buf.count, N)
-    score_bytes = B * N * 2 * R
-    attn_bytes = U * 1152
-    step_b = step_bytes(N, B, R, "bf16", U)
+    # ---- algorithmic bytes (distinct rows gathered per sequence, summed; the trigger's scan and new fired rows)
+    from paper_2609_03949_gb300.bytes_model import row_bytes, score_bytes_per_row, step_bytes
+    k = vk.vk_keep_count(N, w.rho, w.window, 0)
+    nS = k + w.window
+    U1 = union_rows(buf.idx[..., :nS], torch.minimum(buf.count, torch.tensor(nS, device=dev)), N)
+    U = union_rows(buf.idx, buf.count, N) if w.trigger else U1
+    step_b = step_bytes(N, B, w.r, w.dtype, U1, bool(w.trigger), U - U1)
     hbm_peak, peak_kind = peaks()
-    stage_bytes = {"score": score_bytes, "attn": attn_bytes}
-    dom = max(("score", "attn"), key=lambda s: stage_ms[STAGES.index(s)])
+    sb = score_bytes_per_row(w.r, w.dtype)
+    stage_bytes = {"score": B * N * sb, "attn": U1 * row_bytes(w.dtype),
+                   "trigger": B * N * (sb + 4) + (U - U1) * row_bytes(w.dtype)}
+    cands = ["score", "attn"] + (["trigger"] if w.trigger else [])
+    dom = max(cands, key=lambda st: stage_ms[STAGES.index(st)])
     dom_ms = stage_ms[STAGES.index(dom)]
-    kname = {"score": "score", "attn": "attn"}[dom]
     achieved = stage_bytes[dom] / (dom_ms * 1e-3) / 1e9
-    roof = {"bound": "hbm", "kernel": kname, "achieved": achieved, "peak": hbm_peak, "unit": "GB/s",
+    roof = {"bound": "hbm", "kernel": dom, "achieved": achieved, "peak": hbm_peak, "unit": "GB/s",
             "frac": achieved / hbm_peak, "peak_kind": f"{peak_kind} copy bandwidth",
-            "traffic": kernel_traffic(kname) if (B, N) == (B_PER_GPU, N_DEFAULT) else None,
-            "algorithmic_bytes_per_launch": stage_bytes[dom],
-            "ms_per_launch": dom_ms}
+            "traffic": kernel_traffic(dom) if (w.name, B, N) == (DEFAULT_CONFIG, B_PER_GPU, N_DEFAULT) else None,
+            "algorithmic_bytes_per_launch": stage_bytes[dom], "ms_per_launch": dom_ms}
 
     # ---- end to end through the public C entry point with host buffers (pinned). Every step copies its queries
     # in from pinned host memory and its outputs back; the copies run on their own streams and overlap the
@@ -384,7 +470,7 @@ def run_native(args):
             stream.wait_event(ev_in[k])
             if i >= 2:
                 stream.wait_event(ev_out[k])             # step i - 2's outputs are out of these buffers
-            bufs[k].run(views[k], params)
+            bufs[k].run(views[k], params, index)
             ev_comp[k].record(stream)
             s_out.wait_event(ev_comp[k])
             with torch.cuda.stream(s_out):
@@ -411,23 +497,30 @@ def run_native(args):
     assert all(torch.isfinite(t).all() for t in lseh)
     assert vk.vk_poll_status(bufs[1].ws) == vk.VK_OK
 
-    cpu = None
+    sigma = None
+    if w.name == DEFAULT_CONFIG and w.dtype == "bf16":
+        sigma = sigma_throughput(vk, view, B, N, stream, hbm_peak)
+
+    cpu = cpu1 = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        cpu = oracle_baseline(wl.cache, wl.q_latent, wl.q_rope)
+        cpu = oracle_baseline(wl, w)
+        cpu1 = oracle_baseline(wl, w, threads=1, budget_s=6.0)
 
     line = {
-        "metric": METRIC, "value": job_throughput(B, world, ms_step), "unit": UNIT, "n_gpus": world,
+        "metric": w.metric, "value": job_throughput(B, world, ms_step), "unit": UNIT, "n_gpus": world,
         "steps": args.steps, "warmup": max(3, args.warmup), "ms_per_step": ms_step, "higher_is_better": True,
-        "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
-        "data": "synthetic (seeded Gaussian MLA cache, bf16)", "config": workload_config(B, world),
-        "roofline": roof, "cpu_baseline": cpu,
+        "scaling": "weak", "vs_baseline": None, "dtype": w.dtype,
+        "data": f"synthetic (seeded Gaussian MLA cache, {w.dtype})", "config": w.describe(world),
+        "roofline": roof, "cpu_baseline": cpu, "cpu_baseline_single_thread": cpu1,
         "e2e": {"value": job_throughput(B, world, e2e_ms / args.steps), "unit": UNIT, "h2d_bytes_per_step": h2d,
                 "d2h_bytes_per_step": d2h},
         "gpu_launches": int(launches), "clocks": clk,
         "step": {"device_ms_per_step": dev_ms_step, "algorithmic_bytes": step_b,
                  "hbm_gbs": step_b / (ms_step * 1e-3) / 1e9, "frac_of_peak": step_b / (ms_step * 1e-3) / 1e9 / hbm_peak,
-                 "union_rows_per_seq": U / B, "union_frac": U / (B * N),
-                 "stage_ms": {s: float(stage_ms[i]) for i, s in enumerate(STAGES)}},
+                 "union_rows_per_seq": U1 / B, "union_frac": U1 / (B * N),
+                 "fired_new_rows_per_seq": (U - U1) / B,
+                 "stage_ms": {st: float(stage_ms[i]) for i, st in enumerate(STAGES)}},
+        "sigma": sigma,
     }
     if rank == 0:
         print(json.dumps(line), flush=True)

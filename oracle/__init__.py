@@ -82,6 +82,7 @@ def lib():
         L.vko_calib_zq.restype = I64
         L.vko_set_mutation.argtypes = [ctypes.c_int]
         L.vko_num_threads.restype = ctypes.c_int
+        L.vko_set_threads.argtypes = [ctypes.c_int]
         del F
         _lib = L
     return _lib
@@ -119,6 +120,11 @@ def set_mutation(m: int) -> None:
 
 def num_threads() -> int:
     return int(lib().vko_num_threads())
+
+
+def set_threads(n: int) -> None:
+    """OpenMP threads of the oracle's (b, h) loops from now on."""
+    lib().vko_set_threads(int(n))
 
 
 def keep_count(N: int, rho: float, window: int, n_sink: int = 0) -> int:

@@ -714,6 +714,14 @@ int64_t vko_calib_zq(const vko_view* v, int32_t r, const float* rot, double lam,
   return n_hard;
 }
 
+void vko_set_threads(int n) {
+#ifdef _OPENMP
+  if (n > 0) omp_set_num_threads(n);
+#else
+  (void)n;
+#endif
+}
+
 int vko_num_threads(void) {
 #ifdef _OPENMP
   return omp_get_max_threads();
