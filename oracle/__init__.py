@@ -26,7 +26,7 @@ D_LATENT, D_ROPE, PAGE = 512, 64, 64
 # Deliberate mistakes the "known-bad first" tests plant in the oracle (see vk_oracle.c).
 MUT_NONE, MUT_TIE_LARGER, MUT_DROP_WINDOW, MUT_SCALE_SQUARED = 0, 1, 2, 3
 MUT_ROT_TRANSPOSE, MUT_DROP_ROPE, MUT_TRIGGER_NO_Z, MUT_SIGMA_ONE_SIDED = 4, 5, 6, 7
-MUT_PCA_ASCENDING, MUT_CONFORMAL_FLOOR = 8, 9
+MUT_PCA_ASCENDING, MUT_CONFORMAL_FLOOR, MUT_SKETCH_QNORM = 8, 9, 10
 
 
 def build(force: bool = False) -> str:
@@ -61,10 +61,10 @@ def lib():
         L.vko_scores.argtypes = [VP, I32, P, P, P]
         L.vko_select.argtypes = [I32, I32, I32, P, I64, I32, I32, I32, P, P, P]
         L.vko_attention.argtypes = [VP, D, P, P, I32, P, P, P]
-        L.vko_trigger.argtypes = [VP, I32, P, D, D, I32, P, P, P, P, P, I32, P, I32, I32, I32, P, P]
+        L.vko_trigger.argtypes = [VP, I32, P, D, D, I32, P, P, P, I32, P, P, P, P, P, I32, P, I32, I32, I32, P, P]
         L.vko_page_norms.argtypes = [VP, P, P]
         L.vko_trigger_page.argtypes = [VP, D, D, I32, P, P, P, P, I32, P, I32, I32, I32, P, P]
-        L.vko_decode_step.argtypes = [VP, D, I32, I32, I32, D, I32, D, I32, P, P, I32, P, P, P, P, P, P]
+        L.vko_decode_step.argtypes = [VP, D, I32, I32, I32, D, I32, D, I32, P, P, I32, P, P, I32, P, P, P, P, P, P]
         L.vko_decode_step.restype = ctypes.c_int
         L.vko_sigma.argtypes = [P, I64, I32, I32, P]
         L.vko_sigma_select.argtypes = [P, I64, I32, I32, I64, P]
@@ -80,6 +80,10 @@ def lib():
         L.vko_conformal_quantile.restype = D
         L.vko_calib_zq.argtypes = [VP, I32, P, D, P, P, P, P, P, I32, P, P]
         L.vko_calib_zq.restype = I64
+        L.vko_sketch_basis.argtypes = [P, I64, I32, P, P]
+        L.vko_sketch_basis.restype = ctypes.c_int
+        L.vko_build_sketch.argtypes = [VP, I32, P, P, P, P]
+        L.vko_sketch_query.argtypes = [VP, I32, P, P, P]
         L.vko_set_mutation.argtypes = [ctypes.c_int]
         L.vko_num_threads.restype = ctypes.c_int
         L.vko_set_threads.argtypes = [ctypes.c_int]
@@ -185,8 +189,11 @@ def attention(hi: HostInputs, lam: float, idx: np.ndarray, count: np.ndarray):
 
 def trigger(hi: HostInputs, r: int, lam: float, z_eff: float, top_j: int, a: np.ndarray, eta: np.ndarray,
             page_res: np.ndarray, idx: np.ndarray, count: np.ndarray, smax: np.ndarray, window: int,
-            n_sink: int = 0):
-    """(fired idx [B,H,N] int32, fired count [B,H]) of the row-level Cauchy-Schwarz trigger."""
+            n_sink: int = 0, sketch=None):
+    """(fired idx [B,H,N] int32, fired count [B,H]) of the row-level Cauchy-Schwarz trigger.
+
+    ``sketch`` = (s16 [B,N,r_sk] bf16 bits, p [B,H,r_sk], rho [B,H]) adds the rank-r_sk content sketch term; eta
+    must then be the sketch residual norms (``build_sketch``)."""
     a = np.ascontiguousarray(a, dtype=np.float64)
     idx = np.ascontiguousarray(idx, dtype=np.int32)
     count = np.ascontiguousarray(count, dtype=np.int32)
@@ -196,9 +203,15 @@ def trigger(hi: HostInputs, r: int, lam: float, z_eff: float, top_j: int, a: np.
     capf = hi.N
     fidx = np.full((hi.B, hi.H, capf), -1, np.int32)
     fcount = np.zeros((hi.B, hi.H), np.int32)
+    r_sk, s16, p, rho = 0, None, None, None
+    if sketch is not None:
+        s16 = np.ascontiguousarray(sketch[0], dtype=np.uint16)
+        p = np.ascontiguousarray(sketch[1], dtype=np.float64)
+        rho = np.ascontiguousarray(sketch[2], dtype=np.float64)
+        r_sk = s16.shape[-1]
     lib().vko_trigger(ctypes.byref(hi.view), r, _ptr(hi.rot), float(lam), float(z_eff), int(top_j), _ptr(a),
-                      _ptr(eta), _ptr(page_res), _ptr(idx), _ptr(count), idx.shape[-1], _ptr(smax), window,
-                      n_sink, capf, _ptr(fidx), _ptr(fcount))
+                      _ptr(eta), _ptr(page_res), r_sk, _ptr(s16), _ptr(p), _ptr(rho), _ptr(idx), _ptr(count),
+                      idx.shape[-1], _ptr(smax), window, n_sink, capf, _ptr(fidx), _ptr(fcount))
     return fidx, fcount
 
 
@@ -232,9 +245,11 @@ def trigger_page(hi: HostInputs, lam: float, z_eff: float, top_j: int, page_knor
 
 def decode_step(hi: HostInputs, *, rho: float, r: int = 64, window: int = 0, n_sink: int = 0,
                 sm_scale: float | None = None, trigger: int = 0, z_eff: float = 1.0, top_j: int = 0,
-                digest_bf16: np.ndarray | None = None, cap: int | None = None):
-    """Whole step (trigger: 0 off, 1 row-level reading A, 2 page-level reading B).
-    Returns dict(out, lse, smax, idx, count, kth, rc)."""
+                digest_bf16: np.ndarray | None = None, cap: int | None = None, sketch_basis=None,
+                sketch_bf16: np.ndarray | None = None):
+    """Whole step (trigger: 0 off, 1 row-level reading A, 2 page-level reading B). ``sketch_basis`` [r_sk, 512]
+    turns on the rank-r_sk content sketch of the row-level trigger (``sketch_bf16`` [B,N,r_sk]: the stored entries,
+    else the bf16 rounding of the exact projection). Returns dict(out, lse, smax, idx, count, kth, rc)."""
     lam = (1.0 / math.sqrt(192.0)) if sm_scale is None else float(sm_scale)
     if cap is None:
         cap = hi.N if trigger else max(1, keep_count(hi.N, rho, window, n_sink) + window + n_sink)
@@ -247,9 +262,12 @@ def decode_step(hi: HostInputs, *, rho: float, r: int = 64, window: int = 0, n_s
     dg = None if digest_bf16 is None else np.ascontiguousarray(digest_bf16, dtype=np.uint16)
     if r < D_ROPE and dg is None:
         raise ValueError("a width-r digest needs the stored bf16 digest")
+    vb = None if sketch_basis is None else np.ascontiguousarray(sketch_basis, dtype=np.float64)
+    r_sk = 0 if vb is None else vb.shape[0]
+    s16 = None if sketch_bf16 is None else np.ascontiguousarray(sketch_bf16, dtype=np.uint16)
     rc = lib().vko_decode_step(ctypes.byref(hi.view), float(rho), r, window, n_sink, lam, int(trigger),
-                               float(z_eff), int(top_j), _ptr(hi.rot), _ptr(dg), cap, _ptr(out), _ptr(lse),
-                               _ptr(smax), _ptr(idx), _ptr(count), _ptr(kth))
+                               float(z_eff), int(top_j), _ptr(hi.rot), _ptr(dg), r_sk, _ptr(vb), _ptr(s16), cap,
+                               _ptr(out), _ptr(lse), _ptr(smax), _ptr(idx), _ptr(count), _ptr(kth))
     return dict(out=out, lse=lse, smax=smax, idx=idx, count=count, kth=kth, rc=int(rc))
 
 
@@ -300,6 +318,41 @@ def pca_basis(hi: HostInputs):
     rot = np.zeros((D_ROPE, D_ROPE), np.float64)
     lib().vko_pca_basis(ctypes.byref(hi.view), _ptr(eig), _ptr(rot))
     return eig, rot
+
+
+# ------------------------------------------------------------------------------------------------ content sketch
+def sketch_basis(q, r_sk: int):
+    """(basis [r_sk, 512] whose rows are the leading eigenvectors of sum_i q_i q_i^T, eigenvalues [r_sk]) from
+    queries q [n, 512] (Sec. 4.2: V_r from the context's own queries)."""
+    qq = np.ascontiguousarray(np.asarray(q, dtype=np.float64).reshape(-1, D_LATENT))
+    vb = np.zeros((r_sk, D_LATENT), np.float64)
+    eig = np.zeros(r_sk, np.float64)
+    rc = lib().vko_sketch_basis(_ptr(qq), qq.shape[0], int(r_sk), _ptr(vb), _ptr(eig))
+    if rc != 0:
+        raise ValueError(f"no rank-{r_sk} basis from {qq.shape[0]} queries")
+    return vb, eig
+
+
+def build_sketch(hi: HostInputs, vb):
+    """(s fp64 [B,N,r_sk], s bf16 bits [B,N,r_sk], eta [B,N]): the sketch index entry of every cached row and its
+    residual norm |L_u - V_r s_u|."""
+    vb = np.ascontiguousarray(vb, dtype=np.float64)
+    r_sk = vb.shape[0]
+    s = np.zeros((hi.B, hi.N, r_sk), np.float64)
+    s16 = np.zeros((hi.B, hi.N, r_sk), np.uint16)
+    eta = np.zeros((hi.B, hi.N), np.float64)
+    lib().vko_build_sketch(ctypes.byref(hi.view), r_sk, _ptr(vb), _ptr(s), _ptr(s16), _ptr(eta))
+    return s, s16, eta
+
+
+def sketch_query(hi: HostInputs, vb):
+    """(p [B,H,r_sk], rho [B,H]): the queries' sketch coordinates and residual norms."""
+    vb = np.ascontiguousarray(vb, dtype=np.float64)
+    r_sk = vb.shape[0]
+    p = np.zeros((hi.B, hi.H, max(r_sk, 1)), np.float64)
+    rho = np.zeros((hi.B, hi.H), np.float64)
+    lib().vko_sketch_query(ctypes.byref(hi.view), r_sk, _ptr(vb), _ptr(p), _ptr(rho))
+    return p[..., :r_sk], rho
 
 
 # ------------------------------------------------------------------------------------------------ conformal z

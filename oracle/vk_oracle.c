@@ -17,10 +17,10 @@
  *   - the cache holds rows 0..N-1; the query sits at position N; the recent window is [N-W, N);
  *   - the archive is A = [n_sink, N-W); k = min(ceil(rho*N), |A|) rows are kept from it per head;
  *   - ties in the top-k go to the smaller position;
- *   - the trigger is row level: Eq. 4 with sketch rank 0 (the content summand is bounded by
- *     Cauchy-Schwarz with eta_u = |L_u|), plus a page-level bound on the RoPE dims that the width-r
- *     digest does not cover (reading A); reading B admits whole 64-row pages by a page-level bound on
- *     both summands.
+ *   - the trigger is row level: Eq. 4, with the content summand either bounded whole by Cauchy-Schwarz
+ *     (sketch rank 0, eta_u = |L_u|) or split into a rank-r_sk sketch term and a residual bound, plus a
+ *     page-level bound on the RoPE dims that the width-r digest does not cover (reading A); reading B
+ *     admits whole 64-row pages by a page-level bound on both summands (sketch rank 0 only).
  */
 #include <math.h>
 #include <stdint.h>
@@ -47,6 +47,7 @@ enum {
   MUT_SIGMA_ONE_SIDED = 7, /* sigma's inverse DFT drops the factor 2 of the bins that stand for a conjugate pair */
   MUT_PCA_ASCENDING = 8,   /* the PCA basis is ordered by increasing eigenvalue */
   MUT_CONFORMAL_FLOOR = 9, /* the conformal order statistic takes floor((n+1) tau_s) instead of the ceiling */
+  MUT_SKETCH_QNORM = 10,   /* with a content sketch, the certificate keeps |qc_h| instead of the residual norm */
 };
 static int g_mutation = MUT_NONE;
 void vko_set_mutation(int m) { g_mutation = m; }
@@ -274,11 +275,15 @@ void vko_attention(const vko_view* v, double lam, const int32_t* idx, const int3
  * not already attended is
  *     T = lambda * (a[h,u] + |(O qr_h)[r:]| * page_res[page(u)] + z_eff * |qc_h| * eta_u)
  * and the row fires when T > s*_h, the attended set's max logit. With top_j > 0 only the top_j fired
- * rows by (T desc, position asc) are kept. Fired ids are listed in ascending position. */
+ * rows by (T desc, position asc) are kept. Fired ids are listed in ascending position.
+ * With a rank-r_sk content sketch (r_sk > 0: sk16 the stored bf16 entries [B][N][r_sk], p [B][H][r_sk] and rho [B][H]
+ * from vko_sketch_query, eta the sketch residual norms from vko_build_sketch) the content summand is the sketch term
+ * plus the residual bound of Lemma 1:
+ *     T = lambda * (a[h,u] + |(O qr_h)[r:]| * page_res[page(u)] + p_h . s_u + z_eff * rho_h * eta_u). */
 void vko_trigger(const vko_view* v, int32_t r, const float* rot, double lam, double z_eff, int32_t top_j,
-                 const double* a, const double* eta, const double* page_res, const int32_t* idx,
-                 const int32_t* count, int32_t cap, const double* smax, int32_t W, int32_t n_sink,
-                 int32_t capf, int32_t* fidx, int32_t* fcount) {
+                 const double* a, const double* eta, const double* page_res, int32_t r_sk, const uint16_t* sk16,
+                 const double* p, const double* rho, const int32_t* idx, const int32_t* count, int32_t cap,
+                 const double* smax, int32_t W, int32_t n_sink, int32_t capf, int32_t* fidx, int32_t* fcount) {
   const int64_t N = v->N, P = (N + PAGE - 1) / PAGE;
 #pragma omp parallel for collapse(2) schedule(dynamic)
   for (int b = 0; b < v->B; ++b) {
@@ -293,6 +298,8 @@ void vko_trigger(const vko_view* v, int32_t r, const float* rot, double lam, dou
       for (int j = 0; j < D_LAT; ++j) qcn += QC(v, b, h, j) * QC(v, b, h, j);
       qcn = sqrt(qcn);
       double zz = (g_mutation == MUT_TRIGGER_NO_Z) ? 0.0 : z_eff;
+      const int64_t bh = (int64_t)b * v->H + h;
+      const double cert = (r_sk > 0 && g_mutation != MUT_SKETCH_QNORM) ? rho[bh] : qcn;
 
       char* in_set = (char*)calloc((size_t)N + 1, 1);
       const int32_t* set = &idx[((int64_t)b * v->H + h) * cap];
@@ -307,7 +314,9 @@ void vko_trigger(const vko_view* v, int32_t r, const float* rot, double lam, dou
       int64_t nf = 0;
       for (int64_t u = lo; u < hi; ++u) {
         if (in_set[u]) continue;
-        double t = lam * (s[u] + qres * page_res[(int64_t)b * P + u / PAGE] + zz * qcn * eta[(int64_t)b * N + u]);
+        double skt = 0.0;
+        for (int j = 0; j < r_sk; ++j) skt += p[bh * r_sk + j] * from_bf16(sk16[((int64_t)b * N + u) * r_sk + j]);
+        double t = lam * (s[u] + qres * page_res[(int64_t)b * P + u / PAGE] + skt + zz * cert * eta[(int64_t)b * N + u]);
         if (t > sstar) { fired[nf].key = t; fired[nf].u = (int32_t)u; ++nf; }
       }
       if (top_j > 0 && nf > top_j) {
@@ -401,16 +410,23 @@ void vko_trigger_page(const vko_view* v, double lam, double z_eff, int32_t top_j
 }
 
 /* ---------------------------------------------------------------- one decode step */
+/* The content sketch's index and query parts (defined with the sketch, below). */
+void vko_build_sketch(const vko_view* v, int32_t r_sk, const double* vb, double* s, uint16_t* s16, double* eta);
+void vko_sketch_query(const vko_view* v, int32_t r_sk, const double* vb, double* p, double* rho);
+
 /* Score -> select -> attend; in two-tier mode also index -> trigger -> attend over S u F, which equals
  * the LSE merge of the two partial softmaxes (Lemma 1). trigger: 0 off, 1 the row-level rule (reading A),
- * 2 the page-level rule (reading B). idx lists S_h (ascending) followed by F_h (ascending);
- * count = |S_h| + |F_h|. Returns 0, or -4 when a list does not fit in cap. */
+ * 2 the page-level rule (reading B). With r_sk > 0 the row-level rule uses the rank-r_sk content sketch of basis
+ * vb [r_sk][512]; sketch16 is the stored index entry (NULL: the bf16 rounding of vb L_u). idx lists S_h (ascending)
+ * followed by F_h (ascending); count = |S_h| + |F_h|. Returns 0, -1 for a sketch with the page-level rule, or -4
+ * when a list does not fit in cap. */
 int vko_decode_step(const vko_view* v, double rho, int32_t r, int32_t W, int32_t n_sink, double lam,
                     int32_t trigger, double z_eff, int32_t top_j, const float* rot, const uint16_t* digest,
-                    int32_t cap, double* out, double* lse, double* smax, int32_t* idx, int32_t* count,
-                    double* kth) {
+                    int32_t r_sk, const double* vb, const uint16_t* sketch16, int32_t cap, double* out,
+                    double* lse, double* smax, int32_t* idx, int32_t* count, double* kth) {
   const int64_t BH = (int64_t)v->B * v->H, N = v->N, P = (N + PAGE - 1) / PAGE;
   int rc = 0;
+  if (r_sk > 0 && trigger == 2) return -1;
   double* a = (double*)malloc(sizeof(double) * (size_t)(BH * N));
   vko_scores(v, r, rot, digest, a);
   int64_t k = vko_keep_count(v->N, rho, W, n_sink);
@@ -432,8 +448,21 @@ int vko_decode_step(const vko_view* v, double rho, int32_t r, int32_t W, int32_t
       vko_trigger_page(v, lam, z_eff, top_j, pk, pe, idx, count, cap, smax, W, n_sink, capf, fidx, fcount);
       free(pk);
       free(pe);
+    } else if (r_sk > 0) {
+      uint16_t* own16 = NULL;
+      if (!sketch16) own16 = (uint16_t*)malloc(sizeof(uint16_t) * (size_t)(v->B * N * r_sk));
+      vko_build_sketch(v, r_sk, vb, NULL, own16, eta);
+      double* pq = (double*)malloc(sizeof(double) * (size_t)(BH * r_sk));
+      double* rq = (double*)malloc(sizeof(double) * (size_t)BH);
+      vko_sketch_query(v, r_sk, vb, pq, rq);
+      vko_trigger(v, r, rot, lam, z_eff, top_j, a, eta, pres, r_sk, sketch16 ? sketch16 : own16, pq, rq, idx, count,
+                  cap, smax, W, n_sink, capf, fidx, fcount);
+      free(rq);
+      free(pq);
+      free(own16);
     } else {
-      vko_trigger(v, r, rot, lam, z_eff, top_j, a, eta, pres, idx, count, cap, smax, W, n_sink, capf, fidx, fcount);
+      vko_trigger(v, r, rot, lam, z_eff, top_j, a, eta, pres, 0, NULL, NULL, NULL, idx, count, cap, smax, W, n_sink,
+                  capf, fidx, fcount);
     }
     for (int64_t i = 0; i < BH; ++i) {
       int32_t* dst = &idx[i * cap];
@@ -556,9 +585,11 @@ void vko_second_moment(const vko_view* v, double* M) {
     }
 }
 
-void vko_sym_eig(const double* M_in, double* eig, double* vec /* [64][64], row i = eigenvector i */) {
-  const int n = D_ROPE;
-  double A[D_ROPE * D_ROPE], V[D_ROPE * D_ROPE];
+/* Eigenvalues (descending; ties: the lower index first) and eigenvectors (rows of vec, each signed so that its entry
+ * of largest magnitude is positive) of a symmetric n x n matrix by the cyclic Jacobi method. */
+static void jacobi_eig(int n, const double* M_in, double* eig, double* vec) {
+  double* A = (double*)malloc(sizeof(double) * (size_t)n * n);
+  double* V = (double*)malloc(sizeof(double) * (size_t)n * n);
   for (int i = 0; i < n * n; ++i) A[i] = M_in[i];
   for (int i = 0; i < n; ++i)
     for (int j = 0; j < n; ++j) V[i * n + j] = (i == j) ? 1.0 : 0.0;
@@ -596,7 +627,7 @@ void vko_sym_eig(const double* M_in, double* eig, double* vec /* [64][64], row i
       }
   }
   /* order by eigenvalue, descending (ties: the lower index first) */
-  int ord[D_ROPE];
+  int* ord = (int*)malloc(sizeof(int) * (size_t)n);
   for (int i = 0; i < n; ++i) ord[i] = i;
   for (int i = 1; i < n; ++i) {
     const int x = ord[i];
@@ -617,12 +648,130 @@ void vko_sym_eig(const double* M_in, double* eig, double* vec /* [64][64], row i
     const double sg = V[big * n + c] < 0.0 ? -1.0 : 1.0;
     for (int k = 0; k < n; ++k) vec[i * n + k] = sg * V[k * n + c];
   }
+  free(ord);
+  free(V);
+  free(A);
+}
+
+void vko_sym_eig(const double* M_in, double* eig, double* vec /* [64][64], row i = eigenvector i */) {
+  jacobi_eig(D_ROPE, M_in, eig, vec);
 }
 
 void vko_pca_basis(const vko_view* v, double* eig, double* rot) {
   double M[D_ROPE * D_ROPE];
   vko_second_moment(v, M);
   vko_sym_eig(M, eig, rot);
+}
+
+/* ---------------------------------------------------------------- content sketch (Sec. 4.2, Eq. 4, Lemma 1) */
+/* A rank-r_sk sketch of the content summand. V_r is r_sk orthonormal directions of the 512-wide content space, stored
+ * as the rows of vb [r_sk][512]. Lemma 1 splits the content logit of query q and row L as
+ *     q . L = (V_r^T q) . (V_r^T L) + delta,   |delta| <= |(I - V_r V_r^T) q| |(I - V_r V_r^T) L|,
+ * so the index keeps per row s_u = V_r^T L_u (stored in bf16) and eta_u = |(I - V_r V_r^T) L_u|, and the trigger
+ * takes per query p_h = V_r^T qc_h and rho_h = |(I - V_r V_r^T) qc_h|.
+ *
+ * The basis comes from the context's own queries: the r_sk leading eigenvectors of their uncentred second moment
+ * M = sum_i q_i q_i^T (q [n][512]), by decreasing eigenvalue, each signed so that its entry of largest magnitude is
+ * positive. With fewer queries than 512 the same vectors come from the n x n Gram matrix G[i][j] = q_i . q_j: an
+ * eigenvector g of G with eigenvalue mu > 0 gives M's eigenvector sum_i g_i q_i / sqrt(mu), with the same eigenvalue
+ * (M = Q^T Q and G = Q Q^T share their nonzero spectrum). eig receives the r_sk eigenvalues. Returns 0, or -1 when
+ * r_sk is not in [1, 512] or the queries span fewer than r_sk directions. */
+int vko_sketch_basis(const double* q, int64_t n, int32_t r_sk, double* vb, double* eig) {
+  if (r_sk < 1 || r_sk > D_LAT || n < 1) return -1;
+  const int gram = n < D_LAT;
+  const int m = gram ? (int)n : D_LAT;
+  if (r_sk > m) return -1;
+  double* A = (double*)malloc(sizeof(double) * (size_t)m * m);
+  double* ev = (double*)malloc(sizeof(double) * (size_t)m);
+  double* vec = (double*)malloc(sizeof(double) * (size_t)m * m);
+  if (gram) {
+    for (int i = 0; i < m; ++i)
+      for (int j = 0; j < m; ++j) {
+        double acc = 0.0;
+        for (int d = 0; d < D_LAT; ++d) acc += q[(int64_t)i * D_LAT + d] * q[(int64_t)j * D_LAT + d];
+        A[i * m + j] = acc;
+      }
+  } else {
+    for (int i = 0; i < m * m; ++i) A[i] = 0.0;
+    for (int64_t t = 0; t < n; ++t)
+      for (int i = 0; i < D_LAT; ++i)
+        for (int j = 0; j < D_LAT; ++j) A[i * m + j] += q[t * D_LAT + i] * q[t * D_LAT + j];
+  }
+  jacobi_eig(m, A, ev, vec);
+  int rc = 0;
+  for (int k = 0; k < r_sk; ++k) {
+    eig[k] = ev[k];
+    double* out = vb + (int64_t)k * D_LAT;
+    if (gram) {
+      if (!(ev[k] > 0.0)) { rc = -1; break; }
+      for (int d = 0; d < D_LAT; ++d) {
+        double acc = 0.0;
+        for (int i = 0; i < m; ++i) acc += vec[k * m + i] * q[(int64_t)i * D_LAT + d];
+        out[d] = acc / sqrt(ev[k]);
+      }
+      int big = 0;
+      for (int d = 1; d < D_LAT; ++d)
+        if (fabs(out[d]) > fabs(out[big])) big = d;
+      if (out[big] < 0.0)
+        for (int d = 0; d < D_LAT; ++d) out[d] = -out[d];
+    } else {
+      for (int d = 0; d < D_LAT; ++d) out[d] = vec[k * m + d];
+    }
+  }
+  free(vec);
+  free(ev);
+  free(A);
+  return rc;
+}
+
+/* Index entry of every cached row: s_u = V_r^T L_u (s fp64 and s16 its bf16 RNE rounding, [B][N][r_sk], either may be
+ * NULL) and eta_u = |L_u - V_r s_u| with the unrounded s_u ([B][N]). At r_sk = 0, eta_u = |L_u|. */
+void vko_build_sketch(const vko_view* v, int32_t r_sk, const double* vb, double* s, uint16_t* s16, double* eta) {
+  const int64_t N = v->N;
+#pragma omp parallel for schedule(static)
+  for (int b = 0; b < v->B; ++b) {
+    double l[D_LAT], res[D_LAT];
+    double* sk = (double*)malloc(sizeof(double) * (size_t)(r_sk > 0 ? r_sk : 1));
+    for (int64_t u = 0; u < N; ++u) {
+      for (int d = 0; d < D_LAT; ++d) { l[d] = L(v, b, u, d); res[d] = l[d]; }
+      for (int j = 0; j < r_sk; ++j) {
+        double acc = 0.0;
+        for (int d = 0; d < D_LAT; ++d) acc += vb[(int64_t)j * D_LAT + d] * l[d];
+        sk[j] = acc;
+      }
+      for (int j = 0; j < r_sk; ++j)
+        for (int d = 0; d < D_LAT; ++d) res[d] -= sk[j] * vb[(int64_t)j * D_LAT + d];
+      double e = 0.0;
+      for (int d = 0; d < D_LAT; ++d) e += res[d] * res[d];
+      eta[(int64_t)b * N + u] = sqrt(e);
+      const int64_t o = ((int64_t)b * N + u) * r_sk;
+      for (int j = 0; j < r_sk; ++j) {
+        if (s) s[o + j] = sk[j];
+        if (s16) s16[o + j] = vko_bf16_rne(sk[j]);
+      }
+    }
+    free(sk);
+  }
+}
+
+/* Query side of the sketch: p_h = V_r^T qc_h ([B][H][r_sk]) and rho_h = |qc_h - V_r p_h| ([B][H]). */
+void vko_sketch_query(const vko_view* v, int32_t r_sk, const double* vb, double* p, double* rho) {
+  for (int b = 0; b < v->B; ++b)
+    for (int h = 0; h < v->H; ++h) {
+      double q[D_LAT], res[D_LAT];
+      const int64_t bh = (int64_t)b * v->H + h;
+      for (int d = 0; d < D_LAT; ++d) { q[d] = QC(v, b, h, d); res[d] = q[d]; }
+      for (int j = 0; j < r_sk; ++j) {
+        double acc = 0.0;
+        for (int d = 0; d < D_LAT; ++d) acc += vb[(int64_t)j * D_LAT + d] * q[d];
+        p[bh * r_sk + j] = acc;
+      }
+      for (int j = 0; j < r_sk; ++j)
+        for (int d = 0; d < D_LAT; ++d) res[d] -= p[bh * r_sk + j] * vb[(int64_t)j * D_LAT + d];
+      double e = 0.0;
+      for (int d = 0; d < D_LAT; ++d) e += res[d] * res[d];
+      rho[bh] = sqrt(e);
+    }
 }
 
 /* ---------------------------------------------------------------- conformal z (Sec. 4.2; Sec. 5) */

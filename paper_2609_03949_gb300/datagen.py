@@ -11,6 +11,10 @@ Recipe (one decode step of one attention layer, B independent sequences):
 * RoPE keys: N(0,1)^64 vectors rotated at their position u (interleaved pairs (2i, 2i+1), frequency
   10000^(-2i/64)); ``lognormal_keys`` rescales each key to norm 8*exp(0.5*xi), xi ~ N(0,1), before rotating;
 * absorbed query latent part ~ N(0,1)^512 per head; RoPE part N(0,1)^64 rotated at position N;
+* ``query_rank`` k > 0 makes the content queries low-rank plus noise, as a model's queries are: q = sqrt((1-nu) 512/k)
+  U g + sqrt(nu) eps, U the first k rows of a seeded Haar 512x512 rotation, g ~ N(0,1)^k, eps ~ N(0,1)^512, nu =
+  ``query_noise`` (E|q|^2 = 512 as in the isotropic case); ``prefix_queries`` draws the context's earlier queries
+  from the same law (the sketch basis is computed from them);
 * planted rows: ``n_planted`` distinct archive positions per sequence; planted row p targets head p mod H and
   stores the key 4 * q_rope[h] / |q_rope[h]| (a stored, already-rotated value);
 * everything stored as bf16 by round-to-nearest-even from fp32, or kept fp32;
@@ -45,6 +49,8 @@ class Workload:
     planted_pos: torch.Tensor     # [B, n_planted] int64 positions (may be empty)
     planted_head: torch.Tensor    # [n_planted] int64 target head of each planted row
     seed: int
+    query_rank: int = 0           # > 0: content queries low-rank plus noise (see the module notes)
+    query_noise: float = 0.0
 
     @property
     def latent(self) -> torch.Tensor:
@@ -77,10 +83,31 @@ def _slice_rows(self, n: int) -> "Workload":
 Workload.slice_rows = _slice_rows
 
 
-def haar_orthogonal(seed: int) -> np.ndarray:
-    """Haar-distributed 64x64 orthogonal matrix: QR of a seeded Gaussian with sign(diag R) > 0 (fp64)."""
+def _spiked_queries(n: int, query_rank: int, query_noise: float, basis_seed: int, gen: torch.Generator,
+                    device) -> torch.Tensor:
+    """n content queries [n, 512] (fp32): sqrt((1-nu) 512/k) U g + sqrt(nu) eps (see the module notes)."""
+    U = torch.from_numpy(haar_orthogonal(basis_seed, D_LATENT)[:query_rank]).float().to(device)
+    g = torch.randn(n, query_rank, generator=gen, device=device)
+    eps = torch.randn(n, D_LATENT, generator=gen, device=device)
+    return math.sqrt((1.0 - query_noise) * D_LATENT / query_rank) * (g @ U) + math.sqrt(query_noise) * eps
+
+
+def prefix_queries(wl: "Workload", n: int, seed_offset: int = 1) -> torch.Tensor:
+    """n earlier content queries of the same context [n, 512], in the workload's storage dtype: the same law as its
+    decode queries (the same subspace U when ``query_rank`` > 0), independent draws."""
+    gen = torch.Generator(device="cpu")
+    gen.manual_seed(int(wl.seed) * 7 + 1_000_003 * int(seed_offset))
+    if wl.query_rank > 0:
+        q = _spiked_queries(n, wl.query_rank, wl.query_noise, wl.seed + 15485863, gen, "cpu")
+    else:
+        q = torch.randn(n, D_LATENT, generator=gen)
+    return q.to(torch.bfloat16 if wl.dtype == "bf16" else torch.float32)
+
+
+def haar_orthogonal(seed: int, n: int = D_ROPE) -> np.ndarray:
+    """Haar-distributed n x n orthogonal matrix (default 64): QR of a seeded Gaussian with sign(diag R) > 0 (fp64)."""
     rng = np.random.default_rng(seed)
-    g = rng.standard_normal((D_ROPE, D_ROPE))
+    g = rng.standard_normal((n, n))
     q, r = np.linalg.qr(g)
     q = q * np.sign(np.diag(r))[None, :]
     return q
@@ -104,7 +131,7 @@ def _rotate_pairs(x: torch.Tensor, cos: torch.Tensor, sin: torch.Tensor) -> torc
 
 def make_workload(B: int, H: int, N: int, *, dtype: str = "bf16", seed: int = 0, n_planted: int = 0,
                   lognormal_keys: bool = False, planted_lo: int = 0, planted_hi: int | None = None,
-                  device: str | torch.device = "cpu") -> Workload:
+                  query_rank: int = 0, query_noise: float = 0.05, device: str | torch.device = "cpu") -> Workload:
     """Draw one decode step's cache and queries.
 
     Planted rows go to distinct positions in [planted_lo, planted_hi) (the archive range of the caller's
@@ -124,6 +151,10 @@ def make_workload(B: int, H: int, N: int, *, dtype: str = "bf16", seed: int = 0,
     sin_q = torch.from_numpy(sin_q).float().to(device)
 
     q_latent = torch.randn(B, H, D_LATENT, generator=gen, device=device)
+    if query_rank > 0:   # drawn from a generator of their own, so the cache is the same as with isotropic queries
+        gq = torch.Generator(device=device)
+        gq.manual_seed(int(seed) + 31337)
+        q_latent = _spiked_queries(B * H, query_rank, query_noise, seed + 15485863, gq, device).view(B, H, D_LATENT)
     q_rope = _rotate_pairs(torch.randn(B, H, D_ROPE, generator=gen, device=device), cos_q, sin_q)
 
     hi = N if planted_hi is None else planted_hi
@@ -151,7 +182,7 @@ def make_workload(B: int, H: int, N: int, *, dtype: str = "bf16", seed: int = 0,
     rot = torch.from_numpy(haar_orthogonal(seed + 7919)).float().to(device)
     return Workload(B=B, H=H, N=N, dtype=dtype, cache=cache, q_latent=q_latent.to(store),
                     q_rope=q_rope.to(store), rot=rot, planted_pos=planted_pos, planted_head=planted_head,
-                    seed=int(seed))
+                    seed=int(seed), query_rank=int(query_rank), query_noise=float(query_noise if query_rank else 0.0))
 
 
 # The five evaluation workloads, named by what they are, with their sizes. ``CONFIG_PARAMS`` gives the selection
