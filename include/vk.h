@@ -58,7 +58,7 @@ typedef enum { VK_BF16 = 0, VK_F32 = 1 } vk_dtype;
 typedef enum {
   VK_TRIG_OFF = 0,     /* tier 1 only: the top-k plus window (plus sinks) */
   VK_TRIG_CS = 1,      /* two-tier, row level (reading A): fetch the archived rows whose Cauchy-Schwarz trigger
-                          score (Eq. 4 with sketch rank 0) beats s* */
+                          score (Eq. 4, with sketch rank 0 or params->r_sk) beats s* */
   VK_TRIG_CS_PAGE = 2  /* two-tier, page level (reading B): fetch every archived row of each 64-row page whose
                           page-level bound lambda (|Qr| max|K| + z_eff |Qc| max eta) beats s*; needs
                           index->page_knorm and index->page_eta. With top_j, the top_j fired rows by (page bound
@@ -88,6 +88,9 @@ typedef struct {
   float z_eff;              /* trigger certificate multiplier z / sqrt(d_c - r_sk); 1 = the sound bound */
   int32_t top_j;            /* keep only the top_j fired rows per head; 0 = uncapped */
   uint32_t flags;           /* VK_FLAG_* below; 0 for normal use */
+  int32_t r_sk;             /* content sketch rank of the row-level trigger (Sec. 4.2, Eq. 4): 0 (the content
+                               summand bounded whole, eta_u = |L_u|), or 16, 32, 64 with index->sketch and
+                               index->sketch_basis; VK_TRIG_CS only */
 } vk_params;
 
 /* Force the exact fallback of the fused selection on every head (for tests; results are unchanged). */
@@ -112,6 +115,9 @@ typedef struct {
   const float* page_knorm;  /* [B, ceil(N/64)] max over the page of |K_u| (all 64 RoPE dims); VK_TRIG_CS_PAGE needs
                                it, VK_TRIG_CS uses it for the page skip; may be NULL otherwise */
   const float* page_eta;    /* [B, ceil(N/64)] max over the page of eta_u; with page_knorm */
+  const void* sketch;       /* [B, N, r_sk] bf16 contiguous, s_u = V_r^T L_u rounded to nearest even (vk_build_sketch);
+                               with r_sk > 0, when eta must be the sketch residual |L_u - V_r s_u| */
+  const float* sketch_basis;/* [r_sk, 512] fp32: the rows are V_r's orthonormal directions (vk_sketch_basis) */
 } vk_index;
 
 /* k = min(ceil(rho*N), N - W - n_sink): archived rows kept per head (-1 on bad arguments). */
@@ -129,6 +135,25 @@ size_t vk_workspace_bytes(const vk_view* view, const vk_params* params, int32_t 
  * may be NULL to skip it. rot64: [64,64] row-major fp32 orthogonal matrix (device); may be NULL when r = 64. */
 int vk_build_digest(const vk_view* view, const vk_params* params, const float* rot64, void* digest, float* eta,
                     float* page_res, float* page_knorm, float* page_eta, void* stream);
+
+/* Content sketch of the index (Sec. 4.2, Eq. 4, Lemma 1): for every row s_u = V_r^T L_u (r_sk values, stored in bf16
+ * by round-to-nearest-even into sketch [B, N, r_sk]) and eta_u = |L_u - V_r s_u| (fp32 [B, N], with the unrounded s_u).
+ * basis: [r_sk, 512] fp32 (device), orthonormal rows. r_sk in {16, 32, 64}. Either output may be NULL. By Lemma 1,
+ * qc . L_u differs from (V_r^T qc) . s_u by at most |(I - V_r V_r^T) qc| eta_u. The paper's index keeps this entry
+ * for every archived row; the trigger of vk_decode_step reads it when params->r_sk > 0. */
+int vk_build_sketch(const vk_view* view, int32_t r_sk, const float* basis, void* sketch, float* eta, void* stream);
+
+/* Workspace bytes of vk_sketch_basis; 0 on bad arguments. */
+size_t vk_sketch_basis_workspace_bytes(int64_t n, int32_t r_sk);
+
+/* The sketch basis from n queries of the context (Sec. 4.2: V_r from the context's own prefix queries): the r_sk
+ * leading eigenvectors of their uncentred second moment sum_i q_i q_i^T, by decreasing eigenvalue, each signed so that
+ * its entry of largest magnitude is positive, as the rows of basis [r_sk, 512] fp32, and their eigenvalues in eig
+ * [r_sk] fp32 (device; eig may be NULL). queries: [n, 512] contiguous, dtype a vk_dtype (device). r_sk in {16, 32,
+ * 64}, n >= r_sk. The moment is accumulated in fp32 and its leading subspace found by orthogonal iteration with a
+ * Rayleigh-Ritz step in fp64: directions whose eigenvalues are close are accurate as a subspace, not one by one. */
+int vk_sketch_basis(const void* queries, int32_t dtype, int64_t n, int32_t r_sk, float* basis, float* eig, void* ws,
+                    size_t ws_bytes, void* stream);
 
 /* Score every cached row: scores[b,h,u] = a[h,u] (unscaled) as fp32, [B, H, N] contiguous. The RoPE columns
  * are read when r = 64, the index's digest otherwise. ws holds the rotated queries. */
@@ -196,7 +221,8 @@ int vk_decode_step_noalloc(const vk_view* view, const vk_params* params, const v
  * when n < min_hard or that index passes n, clamped to [0, z_max]. Outputs (device): zq [B, H] fp32, NaN where the
  * query is not hard; z_out[3] = {z, z_eff = z / sqrt(512) (the decode step's z_eff), n_hard}. index needs eta and
  * page_res (and the digest and rotation when r < 64); bf16 caches only (the argmax runs on the tensor-core
- * attention over every row); B * H <= 16384 (one block sorts the zq). */
+ * attention over every row); B * H <= 16384 (one block sorts the zq). params->r_sk must be 0 (VK_ERR_UNSUPPORTED
+ * otherwise): the calibration computes the sketch-rank-0 certificate. */
 size_t vk_conformal_workspace_bytes(const vk_view* view, const vk_params* params);
 int vk_conformal_z(const vk_view* view, const vk_params* params, const vk_index* index, const int32_t* idx,
                    const int32_t* count, int32_t cap, float tau, float z_max, float* zq, float* z_out, void* ws,

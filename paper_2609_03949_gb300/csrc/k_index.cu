@@ -5,7 +5,8 @@
 // page_res[page] = max_u |(O K_u)[r:64]|, and the page maxima of |K_u| and eta_u (the page-level bound).
 // Page trigger (reading B): every archived row outside S_h of a page whose bound beats s*_h fires.
 // SIMT scoring: a[h,u] = qt_h[0:r] . key_u[0:r] (fp32) for fp32 caches, digests and small problems.
-// Dense trigger (Eq. 4, Lemma 2): T = lambda (a + |(O Qr)[r:]| page_res + z_eff |Qc| eta) > s*_h.
+// Dense trigger (Eq. 4, Lemma 2): T = lambda (a + |(O Qr)[r:]| page_res + z_eff |Qc| eta) > s*_h; with a content
+// sketch, T = lambda (a + |(O Qr)[r:]| page_res + p_h . s_u + z_eff rho_h eta_u) (rho_h passed as |Qc|).
 #include "vk_common.cuh"
 
 namespace vk {
@@ -237,7 +238,8 @@ __global__ void k_trigger_dense(int H, int N, int W, int n_sink, float lam, floa
                                 const float* __restrict__ qrn, const float* __restrict__ eta,
                                 const float* __restrict__ page_res, const float* __restrict__ smax1,
                                 const uint32_t* __restrict__ selbm, uint32_t* __restrict__ firebm, int64_t nw,
-                                long long* __restrict__ nfired) {
+                                long long* __restrict__ nfired, int r_sk, const __nv_bfloat16* __restrict__ sketch,
+                                const float* __restrict__ skp) {
   const int64_t bh = blockIdx.y;
   const int64_t w = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
   if (w >= nw) return;
@@ -254,7 +256,9 @@ __global__ void k_trigger_dense(int H, int N, int W, int n_sink, float lam, floa
     bool fire = false;
     float t = -INFINITY;
     if (arch && !((sel >> i) & 1u)) {
-      t = lam * (a[u] + cq * page_res[b * P + u / PAGE] + cz * eta[b * N + u]);
+      float skt = 0.f;                               // the content sketch term p_h . s_u (Eq. 4), r_sk > 0
+      for (int j = 0; j < r_sk; ++j) skt = fmaf(skp[bh * r_sk + j], __bfloat162float(sketch[(b * N + u) * r_sk + j]), skt);
+      t = lam * (a[u] + cq * page_res[b * P + u / PAGE] + skt + cz * eta[b * N + u]);
       fire = t > sstar;
     }
     if (fire) bits |= 1u << i;
@@ -267,12 +271,14 @@ __global__ void k_trigger_dense(int H, int N, int W, int n_sink, float lam, floa
 cudaError_t launch_trigger_dense(int B, int H, int N, int W, int n_sink, float lam, float z_eff, int top_j,
                                  float* scores, const float* qcn, const float* qrn, const float* eta,
                                  const float* page_res, const float* smax1, const uint32_t* selbm,
-                                 uint32_t* firebm, int64_t nw, int64_t* nfired, cudaStream_t st) {
+                                 uint32_t* firebm, int64_t nw, int64_t* nfired, cudaStream_t st, int r_sk,
+                                 const void* sketch, const float* skp) {
   cudaError_t e = cudaMemsetAsync(nfired, 0, sizeof(int64_t) * B * H, st);
   if (e != cudaSuccess) return e;
   dim3 grid((unsigned)((nw + 127) / 128), B * H);
   k_trigger_dense<<<grid, 128, 0, st>>>(H, N, W, n_sink, lam, z_eff, top_j, scores, qcn, qrn, eta, page_res, smax1,
-                                        selbm, firebm, nw, reinterpret_cast<long long*>(nfired));
+                                        selbm, firebm, nw, reinterpret_cast<long long*>(nfired), r_sk,
+                                        static_cast<const __nv_bfloat16*>(sketch), skp);
   count_launches(1);
   return cudaGetLastError();
 }

@@ -317,4 +317,13 @@ cudaError_t launch_pca_basis(const vk_view& v, float* rot, float* eig, void* ws,
   return cudaGetLastError();
 }
 
+cudaError_t launch_sym_eig64(const double* A, float* vec, float* eig, cudaStream_t st) {
+  const size_t jsmem = 2 * 64 * 65 * sizeof(double);
+  cudaError_t e = cudaFuncSetAttribute(k_pca_jacobi, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)jsmem);
+  if (e != cudaSuccess) return e;
+  k_pca_jacobi<<<1, JC_THREADS, jsmem, st>>>(A, vec, eig);
+  count_launches(1);
+  return cudaGetLastError();
+}
+
 }  // namespace vk

@@ -21,6 +21,11 @@
 //                                shared memory and only its set bits are visited,
 //                        mode 2  trigger: T = lambda (a + |(O Qr)[r:]| page_res + z |Qc| eta) > s*_h for archive
 //                                rows outside S_h -> 32-row words of the fired bitmap (or candidates for top_j).
+//                                With a rank-SK content sketch (Eq. 4), each stage also holds the tile's sketch
+//                                rows s_u (TMA, [TM x SK] bf16) and the query buffer the bf16 high and low parts of
+//                                p_h = V^T Qc_h, so that p_h . s_u accumulates into the same tensor-memory
+//                                accumulator as a (SK/16 x 2 more instructions); the certificate's |Qc| is then the
+//                                sketch residual norm, passed in its place.
 //                                With the page norm maxima given, a tile in which no head's page bound can reach
 //                                s*_h (page_may_fire) is skipped: the producer warp decides per tile, loads nothing
 //                                and tells the MMA issuer to issue nothing; the epilogue, applying the same test per
@@ -141,9 +146,9 @@ __device__ __forceinline__ uint32_t range_mask(int r0, int lo, int hi) {
 // One configuration of the kernel: TM rows per tile (the MMA's N: 64 or 128), G epilogue groups of WPQ warps per
 // tensor-memory lane quarter (a tile's 32-row chunks of a head are split among them), NACC accumulators of
 // NHG x TM tensor-memory columns (all 512 columns), a ring of STAGES tiles (96 to 112 KB). Shared memory from a
-// 1024-aligned base: the ring, two query buffers of NHG x MH rows, 128 B of staging per epilogue thread (modes 1,
-// 2), barriers.
-template <int MH, int NHG, int TM_, int G_, int WPQ_ = 1, int RW_ = 64>
+// 1024-aligned base: the ring, two query buffers of NHG x MH rows (one with a sketch, whose query parts take the
+// room), 128 B of staging per epilogue thread (modes 1, 2), barriers. SK: the content sketch width (mode 2), or 0.
+template <int MH, int NHG, int TM_, int G_, int WPQ_ = 1, int RW_ = 64, int SK_ = 0>
 struct TcCfg {
   static constexpr int TM = TM_;
   static constexpr int G = G_;
@@ -155,32 +160,41 @@ struct TcCfg {
   static constexpr uint32_t QPART = NHG * MH * QROW;     // one query part
   static constexpr uint32_t DCOLS = NHG * TM;            // columns per accumulator
   static constexpr int NACC = 512 / DCOLS;
-  static constexpr uint32_t TILE = TM * RW * 2;          // TM rows x RW bf16
+  static constexpr int SK = SK_;
+  static constexpr uint32_t KTILE = TM * RW * 2;         // TM rows x RW bf16
+  static constexpr uint32_t TILE = KTILE + TM * SK * 2;  // ... then TM rows x SK bf16 of sketch
+  static constexpr uint32_t SQPART = NHG * MH * SK * 2;  // one bf16 part of the sketch query p
   static constexpr int NC = MH == 128 ? TM / 32 : TM / 64;   // 32-row chunks per lane and tile
   static constexpr int NCT = NC / WPQ;                   // of which one epilogue thread takes
   static constexpr int EW = 4 * G * WPQ;                 // epilogue warps
   static constexpr int THREADS = (2 + EW) * 32;
-  static constexpr uint32_t qbuf = QPARTS * QPART;
+  static constexpr int QB = SK > 0 ? 1 : 2;              // query buffers
+  static constexpr uint32_t qbuf = QPARTS * QPART + 2 * SQPART;
   static constexpr uint32_t STG = EW * 32 * 128;
-  // as many ring stages as fit beside the queries and the staging rows, up to 112 KB of tiles (28 at most)
-  static constexpr int STAGES_FIT = (int)((224u * 1024u - 2 * qbuf - STG) / TILE);
-  static constexpr int STAGES_CAP = (int)(112u * 1024u / TILE) < 28 ? (int)(112u * 1024u / TILE) : 28;
+  // as many ring stages as fit beside the queries and the staging rows, up to 112 KB of tiles (160 KB with the
+  // sketch's wider stages; 28 at most)
+  static constexpr uint32_t RING_CAP = (SK > 0 ? 160u : 112u) * 1024u;
+  static constexpr int STAGES_FIT = (int)((224u * 1024u - QB * qbuf - STG) / TILE);
+  static constexpr int STAGES_CAP = (int)(RING_CAP / TILE) < 28 ? (int)(RING_CAP / TILE) : 28;
   static constexpr int STAGES = STAGES_FIT < STAGES_CAP ? STAGES_FIT : STAGES_CAP;
   static constexpr uint32_t a = 0;
   static constexpr uint32_t q = a + STAGES * TILE;
-  static constexpr uint32_t stg = q + 2 * qbuf;
+  static constexpr uint32_t stg = q + QB * qbuf;
   static constexpr uint32_t bars = stg + STG;
   static constexpr uint32_t total = bars + (2 * STAGES + 4 + 2 * NACC) * 8 + 1024;
   static_assert(G <= NACC, "every epilogue group needs an accumulator of its own");
   static_assert(NC % WPQ == 0 && STAGES >= 4, "configuration");
+  static_assert(TILE % 1024 == 0 && qbuf % 1024 == 0 && (SK == 0 || SK == 16 || SK == 32 || SK == 64), "alignment");
   static_assert(total <= 232448, "scoring shared memory exceeds the 227 KB opt-in limit");
 };
 
-template <int MH, int NHG, int MODE, int TM_, int G_, int WPQ_, int RW_>
-__global__ void __launch_bounds__(TcCfg<MH, NHG, TM_, G_, WPQ_, RW_>::THREADS, 1)
+template <int MH, int NHG, int MODE, int TM_, int G_, int WPQ_, int RW_, int SK_>
+__global__ void __launch_bounds__(TcCfg<MH, NHG, TM_, G_, WPQ_, RW_, SK_>::THREADS, 1)
     k_score_tc(const __grid_constant__ CUtensorMap kmap, const __grid_constant__ CUtensorMap qmap,
+               const __grid_constant__ CUtensorMap smap, const __grid_constant__ CUtensorMap sqmap,
                const ScoreTcArgs args) {
-  using L = TcCfg<MH, NHG, TM_, G_, WPQ_, RW_>;
+  using L = TcCfg<MH, NHG, TM_, G_, WPQ_, RW_, SK_>;
+  static_assert(SK_ == 0 || MODE == 2, "the sketch belongs to the trigger");
   constexpr int G = L::G, TC_M = L::TM, TC_STAGES = L::STAGES, NACC = L::NACC;
   constexpr uint32_t TC_TILE_BYTES = L::TILE;
   extern __shared__ __align__(1024) unsigned char smem_raw[];
@@ -199,7 +213,7 @@ __global__ void __launch_bounds__(TcCfg<MH, NHG, TM_, G_, WPQ_, RW_>::THREADS, 1
   __shared__ uint32_t tmem_base;
   __shared__ int abort_flag;
   __shared__ int skip_stage[TC_STAGES];                  // mode 2 page skip: the ring stage's tile was not loaded
-  const bool page_skip = MODE == 2 && L::RW == 64 && args.page_knorm != nullptr;
+  const bool page_skip = MODE == 2 && L::RW == 64 && L::SK == 0 && args.page_knorm != nullptr;
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int64_t total = args.total_tiles;
@@ -237,7 +251,7 @@ __global__ void __launch_bounds__(TcCfg<MH, NHG, TM_, G_, WPQ_, RW_>::THREADS, 1
       bool lok = true;
       if (b != prev_b) {
         if (lane == 0) {
-          const int qi = (b - b_first) & 1, quse = (b - b_first) >> 1;
+          const int qi = (b - b_first) % L::QB, quse = (b - b_first) / L::QB;
           if (quse > 0 && !mbar_wait(&q_empty[qi], (quse - 1) & 1, &abort_flag)) {
             lok = false;
           } else {
@@ -294,11 +308,16 @@ __global__ void __launch_bounds__(TcCfg<MH, NHG, TM_, G_, WPQ_, RW_>::THREADS, 1
       for (int i = 0; i < n; ++i, kt = kt + 1 == tps ? (++b, 0) : kt + 1) {
         const int row0 = kt * TC_M;
         if (b != prev_b) {
-          const int qi = (b - b_first) & 1, quse = (b - b_first) >> 1;
+          const int qi = (b - b_first) % L::QB, quse = (b - b_first) / L::QB;
           if (quse > 0 && !mbar_wait(&q_empty[qi], (quse - 1) & 1, &abort_flag)) { abort_flag = 1; break; }
-          mbar_arrive_expect_tx(&q_full[qi], (uint32_t)H * L::QROW * L::QPARTS);
+          mbar_arrive_expect_tx(&q_full[qi], (uint32_t)H * (L::QROW * L::QPARTS + 4u * L::SK));
           for (int part = 0; part < L::QPARTS; ++part)
             tma_load_2d(sq + qi * L::qbuf + part * L::QPART, &qmap, 0, (b * L::QPARTS + part) * H, &q_full[qi]);
+          if constexpr (L::SK > 0) {
+            for (int part = 0; part < 2; ++part)
+              tma_load_2d(sq + qi * L::qbuf + L::QPARTS * L::QPART + part * L::SQPART, &sqmap, 0, (b * 2 + part) * H,
+                          &q_full[qi]);
+          }
           prev_b = b;
         }
         const int s = i % TC_STAGES, use = i / TC_STAGES;
@@ -306,6 +325,7 @@ __global__ void __launch_bounds__(TcCfg<MH, NHG, TM_, G_, WPQ_, RW_>::THREADS, 1
         if (abort_flag) break;
         mbar_arrive_expect_tx(&a_full[s], TC_TILE_BYTES);
         tma_load_3d(sa + s * TC_TILE_BYTES, &kmap, 0, row0, b, &a_full[s]);
+        if constexpr (L::SK > 0) tma_load_3d(sa + s * TC_TILE_BYTES + L::KTILE, &smap, 0, row0, b, &a_full[s]);
       }
     }
   } else if (warp == 1) {
@@ -314,9 +334,9 @@ __global__ void __launch_bounds__(TcCfg<MH, NHG, TM_, G_, WPQ_, RW_>::THREADS, 1
       constexpr uint32_t idesc = mma_idesc_bf16(MH, TC_M);
       int prev_b = -1, b = b_first, kt = kt_first;
       for (int i = 0; i < n; ++i, kt = kt + 1 == tps ? (++b, 0) : kt + 1) {
-        const int qi = (b - b_first) & 1;
+        const int qi = (b - b_first) % L::QB;
         if (b != prev_b) {
-          if (!mbar_wait(&q_full[qi], ((b - b_first) >> 1) & 1, &abort_flag)) { abort_flag = 1; break; }
+          if (!mbar_wait(&q_full[qi], ((b - b_first) / L::QB) & 1, &abort_flag)) { abort_flag = 1; break; }
           prev_b = b;
         }
         const int s = i % TC_STAGES, use = i / TC_STAGES;
@@ -337,6 +357,21 @@ __global__ void __launch_bounds__(TcCfg<MH, NHG, TM_, G_, WPQ_, RW_>::THREADS, 1
                 mma_bf16(tmem_base + ds * DCOLS + hg * TC_M, ad + (uint64_t)((32 * k) >> 4),
                          bd + (uint64_t)(L::RW >= 16 ? (32 * k) >> 4 : 0), idesc, (part > 0 || k > 0) ? 1u : 0u);
             }
+          if constexpr (L::SK > 0) {
+            // + p_h . s_u: the sketch rows after the key tile, the query's high and low parts after its key parts
+            const uint64_t sd = kmajor_desc<L::SK * 2>(smem_addr(sa + s * TC_TILE_BYTES + L::KTILE));
+#pragma unroll
+            for (int hg = 0; hg < NHG; ++hg)
+#pragma unroll
+              for (int part = 0; part < 2; ++part) {
+                const uint64_t ad = kmajor_desc<L::SK * 2>(smem_addr(sq + qi * L::qbuf + L::QPARTS * L::QPART +
+                                                                     part * L::SQPART + hg * MH * L::SK * 2));
+#pragma unroll
+                for (int k = 0; k < L::SK / 16; ++k)
+                  mma_bf16(tmem_base + ds * DCOLS + hg * TC_M, ad + (uint64_t)((32 * k) >> 4),
+                           sd + (uint64_t)((32 * k) >> 4), idesc, 1u);
+              }
+          }
         }
         mma_commit(&a_empty[s]);
         mma_commit(&d_full[ds]);
@@ -557,12 +592,12 @@ static CUtensorMapSwizzle swizzle_for(int row_bytes) {
                            : CU_TENSOR_MAP_SWIZZLE_NONE;
 }
 
-template <int MH, int NHG, int MODE, int TM, int G, int WPQ, int RW>
+template <int MH, int NHG, int MODE, int TM, int G, int WPQ, int RW, int SK = 0>
 static cudaError_t launch_cfg(const vk_view& v, const void* keys, int64_t key_ld, int64_t key_bstride,
                               const void* qsrc, int row_stride, int n_rows, ScoreTcArgs args, cudaStream_t st) {
-  using L = TcCfg<MH, NHG, TM, G, WPQ, RW>;
+  using L = TcCfg<MH, NHG, TM, G, WPQ, RW, SK>;
   auto encode = encode_fn();
-  CUtensorMap kmap, qmap;
+  CUtensorMap kmap, qmap, smap, sqmap;
   cuuint64_t kdims[3] = {(cuuint64_t)RW, (cuuint64_t)n_rows, (cuuint64_t)v.B};
   cuuint64_t kstr[2] = {(cuuint64_t)(key_ld * row_stride * 2), (cuuint64_t)(key_bstride * 2)};
   cuuint32_t kbox[3] = {(cuuint32_t)RW, (cuuint32_t)TM, 1};
@@ -581,6 +616,26 @@ static cudaError_t launch_cfg(const vk_view& v, const void* keys, int64_t key_ld
              CU_TENSOR_MAP_INTERLEAVE_NONE, swizzle_for(L::QROW), CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
     return cudaErrorInvalidValue;
+  smap = kmap;
+  sqmap = qmap;
+  if constexpr (SK > 0) {
+    // sketch rows [B][N][SK] (all N rows: the trigger scans with row stride 1) and the query parts [B][2][H][SK]
+    if (row_stride != 1 || !args.sketch || !args.sketch_q) return cudaErrorInvalidValue;
+    cuuint64_t sdims[3] = {(cuuint64_t)SK, (cuuint64_t)n_rows, (cuuint64_t)v.B};
+    cuuint64_t sstr[2] = {(cuuint64_t)SK * 2, (cuuint64_t)v.N * SK * 2};
+    cuuint32_t sbox[3] = {(cuuint32_t)SK, (cuuint32_t)TM, 1};
+    if (encode(&smap, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(args.sketch), sdims, sstr, sbox, es3,
+               CU_TENSOR_MAP_INTERLEAVE_NONE, swizzle_for(SK * 2), CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+      return cudaErrorInvalidValue;
+    cuuint64_t pdims[2] = {(cuuint64_t)SK, (cuuint64_t)v.B * 2 * v.H};
+    cuuint64_t pstr[1] = {(cuuint64_t)SK * 2};
+    cuuint32_t pbox[2] = {(cuuint32_t)SK, (cuuint32_t)v.H};
+    if (encode(&sqmap, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(args.sketch_q), pdims, pstr, pbox, es2,
+               CU_TENSOR_MAP_INTERLEAVE_NONE, swizzle_for(SK * 2), CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+      return cudaErrorInvalidValue;
+  }
   args.B = v.B;
   args.H = v.H;
   args.N = v.N;
@@ -590,11 +645,11 @@ static cudaError_t launch_cfg(const vk_view& v, const void* keys, int64_t key_ld
   args.n_pages = (v.N + PAGE - 1) / PAGE;
   args.tmem_cols = 512;
   const int grid = (int)std::min<int64_t>(args.total_tiles, sm_count());   // persistent: one CTA per SM
-  auto kernel = k_score_tc<MH, NHG, MODE, TM, G, WPQ, RW>;
+  auto kernel = k_score_tc<MH, NHG, MODE, TM, G, WPQ, RW, SK>;
   cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)L::total);
   if (e != cudaSuccess) return e;
   if (grid > 0) {
-    kernel<<<grid, L::THREADS, L::total, st>>>(kmap, qmap, args);
+    kernel<<<grid, L::THREADS, L::total, st>>>(kmap, qmap, smap, sqmap, args);
     count_launches(1);
   }
   return cudaGetLastError();
@@ -605,6 +660,18 @@ static cudaError_t launch_heads(const vk_view& v, const void* keys, int64_t key_
                                 const void* qsrc, int row_stride, int n_rows, const ScoreTcArgs& args,
                                 cudaStream_t st) {
   constexpr int G4 = 4 / NHG;
+  if (args.mode == 2 && args.r_sk > 0) {
+    // with the sketch: two epilogue groups and one query buffer leave room for four or more stages of key + sketch
+    if constexpr (NHG == 1 && RW == 64) {
+      if (args.r_sk == 64)
+        return launch_cfg<MH, 1, 2, 128, 2, 1, 64, 64>(v, keys, key_ld, key_bstride, qsrc, row_stride, n_rows, args, st);
+      if (args.r_sk == 32)
+        return launch_cfg<MH, 1, 2, 128, 2, 1, 64, 32>(v, keys, key_ld, key_bstride, qsrc, row_stride, n_rows, args, st);
+      if (args.r_sk == 16)
+        return launch_cfg<MH, 1, 2, 128, 2, 1, 64, 16>(v, keys, key_ld, key_bstride, qsrc, row_stride, n_rows, args, st);
+    }
+    return cudaErrorInvalidValue;
+  }
   if (args.mode == 0)
     return launch_cfg<MH, NHG, 0, 128, G4, 1, RW>(v, keys, key_ld, key_bstride, qsrc, row_stride, n_rows, args, st);
   if (args.mode == 2)

@@ -90,6 +90,10 @@ int check_params(const vk_view* v, const vk_params* p) {
   if (p->top_j < 0) return fail(VK_ERR_INVALID_ARG, "top_j must be >= 0");
   if (p->flags & ~(VK_FLAG_FORCE_FALLBACK | VK_FLAG_FORCE_DENSE | VK_FLAG_TEST_TIMEOUT | VK_FLAG_NO_PAGE_SKIP))
     return fail(VK_ERR_INVALID_ARG, "unknown flags 0x%x", p->flags);
+  if (p->r_sk != 0 && p->r_sk != 16 && p->r_sk != 32 && p->r_sk != 64)
+    return fail(VK_ERR_INVALID_ARG, "r_sk = %d is not in {0, 16, 32, 64}", p->r_sk);
+  if (p->r_sk > 0 && p->trigger != VK_TRIG_CS)
+    return fail(VK_ERR_INVALID_ARG, "the content sketch (r_sk = %d) belongs to the row-level trigger VK_TRIG_CS", p->r_sk);
   return VK_OK;
 }
 
@@ -102,6 +106,12 @@ int check_index(const vk_view* v, const vk_params* p, const vk_index* ix, bool n
     if (!ix || !ix->eta || !ix->page_res) return fail(VK_ERR_INVALID_ARG, "the trigger needs index->eta and index->page_res");
     if ((ix->page_knorm == nullptr) != (ix->page_eta == nullptr))
       return fail(VK_ERR_INVALID_ARG, "index->page_knorm and index->page_eta go together");
+  }
+  if (need_trigger && p->trigger == VK_TRIG_CS && p->r_sk > 0) {
+    if (!ix->sketch || !ix->sketch_basis)
+      return fail(VK_ERR_INVALID_ARG, "r_sk > 0 needs index->sketch and index->sketch_basis");
+    if (!aligned16(ix->sketch) || !aligned16(ix->sketch_basis))
+      return fail(VK_ERR_INVALID_ARG, "index->sketch and index->sketch_basis must be 16-byte aligned");
   }
   if (need_trigger && p->trigger == VK_TRIG_CS_PAGE) {
     if (!ix || !ix->page_knorm || !ix->page_eta)
@@ -208,7 +218,10 @@ VkLayout make_layout(const vk_view& v, const vk_params& p) {
   L.ag = vk::attn_geom(v);
   L.two_tier = p.trigger != VK_TRIG_OFF;
   L.tc = vk::score_tc_supported(v, p.r);
-  L.fused = L.tc && !(p.flags & VK_FLAG_FORCE_DENSE);
+  L.sketch = p.trigger == VK_TRIG_CS && p.r_sk > 0;
+  // the tensor-core trigger carries the sketch at r = 64 for up to 128 heads; otherwise the scores are materialised
+  // and the dense trigger adds the sketch term
+  L.fused = L.tc && !(p.flags & VK_FLAG_FORCE_DENSE) && !(L.sketch && (p.r != vk::D_ROPE || v.H > 128));
   L.dense_scores = !L.fused;
   const int64_t lo = p.n_sink, hi = (int64_t)v.N - p.window;
   const int64_t k = keep_count(v.N, p.rho, p.window, p.n_sink);
@@ -238,6 +251,9 @@ VkLayout make_layout(const vk_view& v, const vk_params& p) {
   L.off_cand = take(L.fused ? sizeof(int2) * BH * L.capc : 0);
   L.off_fcnt = take(L.fcap ? sizeof(int) * BH : 0);
   L.off_fcand = take(L.fcap ? sizeof(int2) * BH * L.fcap : 0);
+  L.off_skp = take(L.sketch ? sizeof(float) * BH * p.r_sk : 0);
+  L.off_skhl = take(L.sketch ? sizeof(uint16_t) * BH * 2 * p.r_sk : 0);
+  L.off_rho = take(L.sketch ? sizeof(float) * BH : 0);
   L.total = off;
   return L;
 }
@@ -492,6 +508,17 @@ int vk_decode_step(const vk_view* view, const vk_params* params, const vk_index*
     int64_t* nfired = at<int64_t>(ws, L.off_nfired);
     uint32_t* firebm = at<uint32_t>(ws, L.off_firebm);
     VK_CUDA(vk::launch_smax_reduce(B, H, L.ag, nslot, pml, smax1, st), "smax");
+    // with a content sketch the certificate's query norm is the sketch residual rho_h (Lemma 1), passed as |Qc|
+    const float* cq = qcn;
+    float* skp = nullptr;
+    void* skhl = nullptr;
+    if (L.sketch) {
+      float* rho = at<float>(ws, L.off_rho);
+      skp = at<float>(ws, L.off_skp);
+      skhl = at<uint16_t>(ws, L.off_skhl);
+      VK_CUDA(vk::launch_sketch_query(v, params->r_sk, index->sketch_basis, skp, skhl, rho, st), "sketch query");
+      cq = rho;
+    }
     if (params->trigger == VK_TRIG_CS_PAGE) {
       // reading B: whole pages by their page-level bound (no scan of the scores)
       int* fcnt = params->top_j > 0 ? at<int>(ws, L.off_fcnt) : nullptr;
@@ -510,7 +537,7 @@ int vk_decode_step(const vk_view* view, const vk_params* params, const vk_index*
       t.mode = 2;
       t.arch_lo = lo;
       t.arch_hi = hi;
-      t.qcn = qcn;
+      t.qcn = cq;
       t.qrn = qrn;
       t.eta = index->eta;
       t.page_res = index->page_res;
@@ -522,7 +549,11 @@ int vk_decode_step(const vk_view* view, const vk_params* params, const vk_index*
       t.nw = L.nw;
       t.top_j = params->top_j;
       t.status = status;
-      if (index->page_knorm && !(params->flags & VK_FLAG_NO_PAGE_SKIP)) {
+      if (L.sketch) {
+        t.r_sk = params->r_sk;
+        t.sketch = index->sketch;
+        t.sketch_q = skhl;
+      } else if (index->page_knorm && !(params->flags & VK_FLAG_NO_PAGE_SKIP)) {
         t.qrf = qrf;
         t.page_knorm = index->page_knorm;
         t.page_eta = index->page_eta;
@@ -542,8 +573,10 @@ int vk_decode_step(const vk_view* view, const vk_params* params, const vk_index*
         VK_CUDA(vk::launch_bitmap_to_list(B, H, N, firebm, L.nw, idx, count, cap, status, st), "fired list");
       }
     } else {
-      VK_CUDA(vk::launch_trigger_dense(B, H, N, W, S, params->sm_scale, params->z_eff, params->top_j, scores, qcn, qrn,
-                                       index->eta, index->page_res, smax1, selbm, firebm, L.nw, nfired, st), "trigger");
+      VK_CUDA(vk::launch_trigger_dense(B, H, N, W, S, params->sm_scale, params->z_eff, params->top_j, scores, cq, qrn,
+                                       index->eta, index->page_res, smax1, selbm, firebm, L.nw, nfired, st,
+                                       L.sketch ? params->r_sk : 0, L.sketch ? index->sketch : nullptr, skp),
+              "trigger");
       if (params->top_j > 0) {
         VK_CUDA(vk::launch_select_dense(B, H, N, scores, nfired, params->top_j, 0, 0, idx, count, cap, 1, nullptr, firebm,
                                         L.nw, status, st), "top_j");
@@ -588,6 +621,8 @@ int vk_conformal_z(const vk_view* view, const vk_params* params, const vk_index*
   g_err[0] = 0;
   int rc;
   if ((rc = check_view(view)) != VK_OK || (rc = check_params(view, params)) != VK_OK) return rc;
+  if (params->r_sk > 0)
+    return fail(VK_ERR_UNSUPPORTED, "the calibration computes the sketch-rank-0 certificate; r_sk must be 0");
   const vk_params q = calib_params(*params);
   if ((rc = check_index(view, &q, index, true)) != VK_OK) return rc;
   if (!vk::attn_tc_supported(*view)) return fail(VK_ERR_UNSUPPORTED, "the calibration's argmax pass reads bf16 caches");
@@ -642,6 +677,40 @@ int vk_pca_basis(const vk_view* view, float* rot, float* eig, void* ws, size_t w
   if (!ws || (reinterpret_cast<uintptr_t>(ws) & 255u) != 0 || ws_bytes < vk::pca_workspace_bytes())
     return fail(VK_ERR_WORKSPACE, "the PCA workspace needs %zu bytes, 256-byte aligned", vk::pca_workspace_bytes());
   VK_CUDA(vk::launch_pca_basis(*view, rot, eig, ws, static_cast<cudaStream_t>(stream)), "pca basis");
+  return VK_OK;
+}
+
+int vk_build_sketch(const vk_view* view, int32_t r_sk, const float* basis, void* sketch, float* eta, void* stream) {
+  g_err[0] = 0;
+  int rc;
+  if ((rc = check_view(view)) != VK_OK) return rc;
+  if (r_sk != 16 && r_sk != 32 && r_sk != 64) return fail(VK_ERR_INVALID_ARG, "r_sk = %d is not in {16, 32, 64}", r_sk);
+  if (!basis || !aligned16(basis)) return fail(VK_ERR_INVALID_ARG, "basis must be a 16-byte aligned pointer");
+  if ((sketch && !aligned16(sketch)) || (eta && !aligned16(eta)))
+    return fail(VK_ERR_INVALID_ARG, "sketch and eta must be 16-byte aligned");
+  if (!sketch && !eta) return VK_OK;
+  VK_CUDA(vk::launch_build_sketch(*view, r_sk, basis, sketch, eta, static_cast<cudaStream_t>(stream)), "build sketch");
+  return VK_OK;
+}
+
+size_t vk_sketch_basis_workspace_bytes(int64_t n, int32_t r_sk) {
+  if (n < 1 || (r_sk != 16 && r_sk != 32 && r_sk != 64) || n < r_sk) return 0;
+  return vk::sketch_basis_ws_bytes();
+}
+
+int vk_sketch_basis(const void* queries, int32_t dtype, int64_t n, int32_t r_sk, float* basis, float* eig, void* ws,
+                    size_t ws_bytes, void* stream) {
+  g_err[0] = 0;
+  if (r_sk != 16 && r_sk != 32 && r_sk != 64) return fail(VK_ERR_INVALID_ARG, "r_sk = %d is not in {16, 32, 64}", r_sk);
+  if (n < r_sk) return fail(VK_ERR_INVALID_ARG, "n = %lld queries cannot span r_sk = %d directions", (long long)n, r_sk);
+  if (dtype != VK_BF16 && dtype != VK_F32) return fail(VK_ERR_INVALID_ARG, "dtype = %d is unknown", dtype);
+  if (!queries || !aligned16(queries) || !basis || !aligned16(basis))
+    return fail(VK_ERR_INVALID_ARG, "queries and basis must be 16-byte aligned pointers");
+  if (!ws || (reinterpret_cast<uintptr_t>(ws) & 255u) != 0 || ws_bytes < vk::sketch_basis_ws_bytes())
+    return fail(VK_ERR_WORKSPACE, "the sketch-basis workspace needs %zu bytes, 256-byte aligned",
+                vk::sketch_basis_ws_bytes());
+  VK_CUDA(vk::launch_sketch_basis(queries, dtype, n, r_sk, basis, eig, ws, static_cast<cudaStream_t>(stream)),
+          "sketch basis");
   return VK_OK;
 }
 

@@ -111,7 +111,9 @@ struct VkLayout {
   int64_t capc;                 // fused: candidate capacity per head
   int64_t fcap;                 // two-tier top_j (fused path or page trigger): fired-candidate capacity per head
   size_t off_status, off_qt, off_qhl, off_qcn, off_qrn, off_qrf, off_smax1, off_nfired, off_scores, off_selbm, off_firebm,
-      off_part_o, off_part_ml, off_sample, off_theta, off_ccnt, off_cand, off_fcnt, off_fcand, total;
+      off_part_o, off_part_ml, off_sample, off_theta, off_ccnt, off_cand, off_fcnt, off_fcand, off_skp, off_skhl,
+      off_rho, total;
+  bool sketch;                  // row-level trigger with a content sketch (r_sk > 0)
 };
 
 // ------------------------------------------------------------------------------------------ launchers
@@ -156,7 +158,20 @@ cudaError_t launch_combine(int B, int H, const AttnGeom& g, int nslot, const flo
 cudaError_t launch_trigger_dense(int B, int H, int N, int W, int n_sink, float lam, float z_eff, int top_j,
                                  float* scores, const float* qcn, const float* qrn, const float* eta,
                                  const float* page_res, const float* smax1, const uint32_t* selbm,
-                                 uint32_t* firebm, int64_t nw, int64_t* nfired, cudaStream_t st);
+                                 uint32_t* firebm, int64_t nw, int64_t* nfired, cudaStream_t st, int r_sk = 0,
+                                 const void* sketch = nullptr, const float* skp = nullptr);
+// Content sketch (k_sketch.cu): the index entry of every row (sketch bf16 [B][N][r_sk], eta [B][N]), the query side
+// (p fp32 [B][H][r_sk], its bf16 high/low parts [B][2][H][r_sk], rho [B][H]), and the basis from n queries.
+cudaError_t launch_build_sketch(const vk_view& v, int r_sk, const float* basis, void* sketch, float* eta,
+                                cudaStream_t st);
+cudaError_t launch_sketch_query(const vk_view& v, int r_sk, const float* basis, float* p, void* phl, float* rho,
+                                cudaStream_t st);
+size_t sketch_basis_ws_bytes();
+cudaError_t launch_sketch_basis(const void* queries, int dtype, int64_t n, int r_sk, float* basis, float* eig,
+                                void* ws, cudaStream_t st);
+// The 64 x 64 fp64 symmetric eigensolver of the PCA basis (k_pca.cu): eigenvectors as rows of vec (fp32), by
+// decreasing eigenvalue.
+cudaError_t launch_sym_eig64(const double* A, float* vec, float* eig, cudaStream_t st);
 cudaError_t launch_theta(int B, int H, int ns, int ld, int off, int stride, int lo, int hi, int j, const void* sample,
                          float* theta, cudaStream_t st);
 cudaError_t launch_select_cand(int B, int H, int N, int lo, int hi, int64_t k, const int64_t* k_per_head,

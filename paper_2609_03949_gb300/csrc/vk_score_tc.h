@@ -33,6 +33,10 @@ struct ScoreTcArgs {
   // mode 2 page skip (when page_knorm != NULL): a 128-row tile is neither loaded nor multiplied when, for every head
   // and both of its pages, lam * (qrf * page_knorm + z * qcn * page_eta) cannot reach smax1 (page_may_fire)
   const float *qrf, *page_knorm, *page_eta;
+  // mode 2 content sketch (r_sk in {16, 32, 64}, r = 64, H <= 128): sketch rows [B][N][r_sk] bf16 and the query's bf16
+  // high and low parts of p = V^T Qc, [B][2][H][r_sk]; qcn then holds the sketch residual norms of the queries
+  int r_sk;
+  const void *sketch, *sketch_q;
   int* status;
 };
 

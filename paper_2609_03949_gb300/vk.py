@@ -39,12 +39,14 @@ class vk_view(ctypes.Structure):
 class vk_params(ctypes.Structure):
     _fields_ = [("rho", ctypes.c_double), ("r", ctypes.c_int32), ("window", ctypes.c_int32),
                 ("n_sink", ctypes.c_int32), ("sm_scale", ctypes.c_float), ("trigger", ctypes.c_int32),
-                ("z_eff", ctypes.c_float), ("top_j", ctypes.c_int32), ("flags", ctypes.c_uint32)]
+                ("z_eff", ctypes.c_float), ("top_j", ctypes.c_int32), ("flags", ctypes.c_uint32),
+                ("r_sk", ctypes.c_int32)]
 
 
 class vk_index(ctypes.Structure):
     _fields_ = [("digest", ctypes.c_void_p), ("eta", ctypes.c_void_p), ("page_res", ctypes.c_void_p),
-                ("rot", ctypes.c_void_p), ("page_knorm", ctypes.c_void_p), ("page_eta", ctypes.c_void_p)]
+                ("rot", ctypes.c_void_p), ("page_knorm", ctypes.c_void_p), ("page_eta", ctypes.c_void_p),
+                ("sketch", ctypes.c_void_p), ("sketch_basis", ctypes.c_void_p)]
 
 
 _lib = None
@@ -81,6 +83,9 @@ def lib():
             "vk_pca_basis": ([VP, P, P, P, SZ, P], ctypes.c_int),
             "vk_sigma": ([VP, I32, I32, P, P, SZ, P], ctypes.c_int),
             "vk_sigma_select": ([I32, I32, I32, P, I32, I64, P, P, I32, P, SZ, P], ctypes.c_int),
+            "vk_build_sketch": ([VP, I32, P, P, P, P], ctypes.c_int),
+            "vk_sketch_basis_workspace_bytes": ([I64, I32], SZ),
+            "vk_sketch_basis": ([P, I32, I64, I32, P, P, P, SZ, P], ctypes.c_int),
         }
         for name, (args, res) in sig.items():
             fn = getattr(L, name)
@@ -96,7 +101,7 @@ def exported_symbols():
             "vk_sparse_attn", "vk_decode_step", "vk_decode_step_noalloc", "vk_workspace_init", "vk_poll_status",
             "vk_profile_set_events", "vk_profile_launches", "vk_last_error", "vk_sigma_workspace_bytes", "vk_sigma",
             "vk_sigma_select", "vk_pca_workspace_bytes", "vk_pca_basis", "vk_conformal_workspace_bytes",
-            "vk_conformal_z"]
+            "vk_conformal_z", "vk_build_sketch", "vk_sketch_basis_workspace_bytes", "vk_sketch_basis"]
 
 
 def _check(rc: int):
@@ -138,14 +143,17 @@ def make_view(cache: torch.Tensor, q_latent: torch.Tensor, q_rope: torch.Tensor)
 
 
 def make_params(rho: float, r: int = 64, window: int = 0, n_sink: int = 0, sm_scale: float = DEFAULT_SM_SCALE,
-                trigger: int = VK_TRIG_OFF, z_eff: float = 1.0, top_j: int = 0, flags: int = 0) -> vk_params:
+                trigger: int = VK_TRIG_OFF, z_eff: float = 1.0, top_j: int = 0, flags: int = 0,
+                r_sk: int = 0) -> vk_params:
     return vk_params(rho=rho, r=r, window=window, n_sink=n_sink, sm_scale=sm_scale, trigger=trigger, z_eff=z_eff,
-                     top_j=top_j, flags=flags)
+                     top_j=top_j, flags=flags, r_sk=r_sk)
 
 
-def make_index(digest=None, eta=None, page_res=None, rot=None, page_knorm=None, page_eta=None) -> vk_index:
+def make_index(digest=None, eta=None, page_res=None, rot=None, page_knorm=None, page_eta=None, sketch=None,
+               sketch_basis=None) -> vk_index:
     return vk_index(digest=_ptr(digest), eta=_ptr(eta), page_res=_ptr(page_res), rot=_ptr(rot),
-                    page_knorm=_ptr(page_knorm), page_eta=_ptr(page_eta))
+                    page_knorm=_ptr(page_knorm), page_eta=_ptr(page_eta), sketch=_ptr(sketch),
+                    sketch_basis=_ptr(sketch_basis))
 
 
 # ------------------------------------------------------------------------------------------------ entry points
@@ -284,6 +292,28 @@ def vk_pca_basis(view, rot, eig=None, ws=None, stream=None) -> None:
         ws = alloc_bytes(int(lib().vk_pca_workspace_bytes()))
     _check(lib().vk_pca_basis(ctypes.byref(view), _ptr(rot), _ptr(eig), _ptr(ws), ws.numel() * ws.element_size(),
                               _stream(stream)))
+
+
+# ------------------------------------------------------------------------------------------------ content sketch
+def vk_build_sketch(view, r_sk: int, basis, sketch=None, eta=None, stream=None) -> None:
+    """Sketch index entry of every cached row: sketch [B, N, r_sk] bf16 = V_r^T L_u, eta [B, N] fp32 its residual."""
+    _check(lib().vk_build_sketch(ctypes.byref(view), int(r_sk), _ptr(basis), _ptr(sketch), _ptr(eta), _stream(stream)))
+
+
+def vk_sketch_basis(queries: torch.Tensor, r_sk: int, basis, eig=None, ws=None, stream=None):
+    """Sketch basis [r_sk, 512] fp32 (rows) from the context's queries [n, 512] (bf16 or fp32, contiguous)."""
+    q = queries
+    if q.dim() != 2 or q.shape[1] != D_LATENT or not q.is_contiguous():
+        raise ValueError("queries must be a contiguous [n, 512] tensor")
+    dt = VK_BF16 if q.dtype == torch.bfloat16 else VK_F32
+    if ws is None:
+        n = int(lib().vk_sketch_basis_workspace_bytes(q.shape[0], int(r_sk)))
+        if n == 0:
+            raise VkError(VK_ERR_INVALID_ARG, lib().vk_last_error().decode())
+        ws = alloc_bytes(n)
+    _check(lib().vk_sketch_basis(_ptr(q), dt, q.shape[0], int(r_sk), _ptr(basis), _ptr(eig), _ptr(ws),
+                                 ws.numel() * ws.element_size(), _stream(stream)))
+    return ws
 
 
 # ------------------------------------------------------------------------------------------------ conformal z

@@ -36,11 +36,14 @@ class GpuStep:
     """Inputs on the GPU plus the C-ABI call of one decode step."""
 
     def __init__(self, wl: datagen.Workload, *, rho, r=64, window=0, n_sink=0, trigger=0, z_eff=1.0, top_j=0,
-                 flags=0, digest_bf16: np.ndarray | None = None, cap=None):
+                 flags=0, digest_bf16: np.ndarray | None = None, cap=None, sketch=None):
+        """sketch = (stored bf16 entries [B,N,r_sk] uint16, basis [r_sk,512], residual norms eta [B,N]): the rank-r_sk
+        content sketch of the row-level trigger, taken from the oracle so that both sides score the same index."""
         self.wl = wl.to("cuda")
         self.view = vk.make_view(self.wl.cache, self.wl.q_latent, self.wl.q_rope)
+        r_sk = 0 if sketch is None else sketch[1].shape[0]
         self.params = vk.make_params(rho, r=r, window=window, n_sink=n_sink, trigger=trigger, z_eff=z_eff,
-                                     top_j=top_j, flags=flags)
+                                     top_j=top_j, flags=flags, r_sk=r_sk)
         B, N = wl.B, wl.N
         P = (N + 63) // 64
         self.rot = self.wl.rot.contiguous()
@@ -55,8 +58,13 @@ class GpuStep:
             self.digest = torch.from_numpy(digest_bf16.astype(np.int16)).view(torch.bfloat16).cuda().contiguous()
         vk.vk_build_digest(self.view, self.params, self.rot, None, self.eta, self.page_res, self.page_knorm,
                            self.page_eta)
+        self.sketch = self.basis = None
+        if sketch is not None:
+            self.sketch = torch.from_numpy(sketch[0].astype(np.int16)).view(torch.bfloat16).cuda().contiguous()
+            self.basis = torch.as_tensor(sketch[1], dtype=torch.float32).cuda().contiguous()
+            self.eta = torch.as_tensor(sketch[2], dtype=torch.float32).cuda().contiguous()
         self.index = vk.make_index(self.digest, self.eta, self.page_res, self.rot if r < 64 else None,
-                                   self.page_knorm, self.page_eta)
+                                   self.page_knorm, self.page_eta, self.sketch, self.basis)
         self.buf = vk.DecodeBuffers(self.view, self.params, cap=cap)
 
     def run(self):

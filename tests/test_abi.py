@@ -154,3 +154,27 @@ def test_sigma_entry_points_refuse(vk):
     assert L.vk_sigma_select(2, 20000, 4096, FAKE, 4, 100, FAKE, FAKE, 3616 + 104 - 1, FAKE, 256, None) == \
         vk.VK_ERR_INVALID_ARG
     assert L.vk_sigma_select(2, 20000, 4096, FAKE, 4, 100, FAKE, FAKE, 3720, FAKE, 255, None) == vk.VK_ERR_WORKSPACE
+
+
+def test_sketch_entry_points_refuse(vk):
+    L = vk.lib()
+    v = fake_view(vk)
+    # the sketch rank: 0, 16, 32 or 64, and only with the row-level trigger
+    assert call_decode(vk, v, vk.make_params(1 / 8, window=16, trigger=1, r_sk=24)) == vk.VK_ERR_INVALID_ARG
+    assert call_decode(vk, v, vk.make_params(1 / 8, window=16, trigger=0, r_sk=16)) == vk.VK_ERR_INVALID_ARG
+    assert call_decode(vk, v, vk.make_params(1 / 8, window=16, trigger=2, r_sk=16)) == vk.VK_ERR_INVALID_ARG
+    # with r_sk > 0 the index needs the stored sketch and its basis
+    idx = vk.make_index(eta=FAKE, page_res=FAKE)
+    assert call_decode(vk, v, vk.make_params(1 / 8, window=16, trigger=1, r_sk=16), index=idx) == vk.VK_ERR_INVALID_ARG
+    idx = vk.make_index(eta=FAKE, page_res=FAKE, sketch=FAKE, sketch_basis=FAKE + 4)
+    assert call_decode(vk, v, vk.make_params(1 / 8, window=16, trigger=1, r_sk=16), index=idx) == vk.VK_ERR_INVALID_ARG
+    assert L.vk_build_sketch(ctypes.byref(v), 8, FAKE, FAKE, FAKE, None) == vk.VK_ERR_INVALID_ARG
+    assert L.vk_build_sketch(ctypes.byref(v), 16, None, FAKE, FAKE, None) == vk.VK_ERR_INVALID_ARG
+    assert L.vk_build_sketch(ctypes.byref(v), 16, FAKE, FAKE + 2, None, None) == vk.VK_ERR_INVALID_ARG
+    nb = L.vk_sketch_basis_workspace_bytes(100, 32)
+    assert nb > 0
+    assert L.vk_sketch_basis_workspace_bytes(20, 32) == 0     # 20 queries cannot span 32 directions
+    assert L.vk_sketch_basis_workspace_bytes(100, 48) == 0
+    assert L.vk_sketch_basis(FAKE, 0, 20, 32, FAKE, None, FAKE, nb, None) == vk.VK_ERR_INVALID_ARG
+    assert L.vk_sketch_basis(FAKE, 3, 100, 32, FAKE, None, FAKE, nb, None) == vk.VK_ERR_INVALID_ARG
+    assert L.vk_sketch_basis(FAKE, 0, 100, 32, FAKE, None, FAKE, nb - 1, None) == vk.VK_ERR_WORKSPACE
