@@ -43,8 +43,10 @@ STAGES = ["qprep", "score", "select", "attn", "trigger", "combine"]
 class Workload:
     """The benchmarked workload: sizes, selection parameters and the metric's name."""
 
-    def __init__(self, name: str, B: int | None, N: int | None, rho: float | None, r: int | None):
+    def __init__(self, name: str, B: int | None, N: int | None, rho: float | None, r: int | None, r_sk: int = 0,
+                 query_rank: int = 0):
         self.name = name
+        self.r_sk, self.query_rank = r_sk, query_rank
         c, p = datagen.CONFIGS[name], datagen.CONFIG_PARAMS[name]
         self.H, self.dtype = c["H"], c["dtype"]
         self.B = B if B is not None else (B_PER_GPU if name == DEFAULT_CONFIG else c["B"])
@@ -63,6 +65,8 @@ class Workload:
         self.metric = f"decode query-tokens/s per layer at N={nk}, rho={rho_s}"
         if name != DEFAULT_CONFIG:
             self.metric += f" ({name})"
+        if r_sk:
+            self.metric += f" with a rank-{r_sk} content sketch"
 
     def describe(self, n_gpus: int) -> dict:
         B, N = self.B, self.N
@@ -70,7 +74,9 @@ class Workload:
         rows = B * N * 576 * esz
         return {"workload": f"sparse MLA decode step: {self.name}, H={self.H}, N={N}, rho={self.rho:g}, r={self.r}, "
                             f"window={self.window}, {self.dtype} cache [512 latent + 64 RoPE]"
-                            f"{', two-tier trigger z_eff=%g' % self.z_eff if self.trigger else ''}, "
+                            f"{', two-tier trigger z_eff=%g' % self.z_eff if self.trigger else ''}"
+                            f"{', content sketch r_sk=%d' % self.r_sk if self.r_sk else ''}"
+                            f"{', content queries of rank %d + 5%% noise' % self.query_rank if self.query_rank else ''}, "
                             f"{self.n_planted} planted rows/seq, B={B} sequences per GPU",
                 "heads": self.H, "context": N, "rho": self.rho, "r": self.r, "window": self.window,
                 "batch_per_gpu": B, "global_batch": B * n_gpus, "trigger": self.trigger,
@@ -93,9 +99,14 @@ def parse():
     ap.add_argument("--context", type=int, default=None, help="cached rows per sequence")
     ap.add_argument("--rho", type=float, default=None)
     ap.add_argument("--r", type=int, default=None, help="score width: 64 or a digest width")
+    ap.add_argument("--r-sk", type=int, default=0, help="content sketch rank of the trigger (16, 32, 64; 0 = none)")
+    ap.add_argument("--query-rank", type=int, default=0,
+                    help="content queries of this rank plus 5%% noise (the sketch basis comes from such prefix queries)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     args = ap.parse_args()
-    args.wl = Workload(args.config, args.batch, args.context, args.rho, args.r)
+    args.wl = Workload(args.config, args.batch, args.context, args.rho, args.r, args.r_sk, args.query_rank)
+    if args.wl.r_sk and not args.wl.trigger:
+        ap.error("--r-sk needs a two-tier workload (h128_n64k_two_tier)")
     return args
 
 
@@ -226,21 +237,36 @@ def kernel_traffic(kernel: str):
 
 
 # ------------------------------------------------------------------------------------------------ CPU oracle
+N_PREFIX = 512        # prefix queries the sketch basis is computed from
+
+
 def make_host_workload(w: Workload, B: int, seed: int, device="cpu"):
-    return datagen.config_workload(w.name, device=device, B=B, N=w.N, seed=seed)
+    return datagen.config_workload(w.name, device=device, B=B, N=w.N, seed=seed, query_rank=w.query_rank)
 
 
-def oracle_step(hi, digest, w: Workload):
+def oracle_step(hi, digest, w: Workload, basis=None):
     import oracle
     return oracle.decode_step(hi, rho=w.rho, r=w.r, window=w.window, trigger=w.trigger, z_eff=w.z_eff,
-                              digest_bf16=digest)
+                              digest_bf16=digest, sketch_basis=basis)
 
 
 def oracle_inputs(wl, w: Workload):
+    """(host inputs, stored digest, sketch basis) of the oracle's step; the basis from the workload's prefix queries
+    (N_PREFIX - 1 of them, so the oracle's Gram route applies)."""
     import oracle
     hi = oracle.HostInputs(wl)
     dig = oracle.build_index(hi, w.r)[1] if w.r < 64 else None
-    return hi, dig
+    basis = None
+    if w.r_sk:   # the prefix queries depend on the workload's seed alone: one basis per workload
+        key = (wl.seed, w.r_sk)
+        if key not in _ORACLE_BASIS:
+            q = datagen.prefix_queries(wl, N_PREFIX - 1).double().numpy()
+            _ORACLE_BASIS[key] = oracle.sketch_basis(q, w.r_sk)[0]
+        basis = _ORACLE_BASIS[key]
+    return hi, dig, basis
+
+
+_ORACLE_BASIS = {}
 
 
 def oracle_baseline(wl_dev, w: Workload, threads: int | None = None, budget_s=12.0, max_seqs=1024):
@@ -252,9 +278,9 @@ def oracle_baseline(wl_dev, w: Workload, threads: int | None = None, budget_s=12
         done, t_total = 0, 0.0
         while done < max_seqs and (t_total < budget_s or done == 0):
             b = done % wl_dev.B
-            hi, dig = oracle_inputs(wl_dev.slice_batch([b]), w)
+            hi, dig, basis = oracle_inputs(wl_dev.slice_batch([b]), w)
             t0 = time.perf_counter()
-            oracle_step(hi, dig, w)
+            oracle_step(hi, dig, w, basis)
             t_total += time.perf_counter() - t0
             done += 1
             if done == 1 and t_total * max_seqs > 4 * budget_s:
@@ -278,10 +304,10 @@ def run_reference(args):
     inputs = [oracle_inputs(wl.slice_batch([b]), w) for b in range(wl.B)]
     warm = max(3, args.warmup)
     for i in range(warm):
-        oracle_step(*inputs[i % 2], w)
+        oracle_step(*inputs[i % 2][:2], w, inputs[i % 2][2])
     t0 = time.perf_counter()
     for i in range(args.steps):
-        oracle_step(*inputs[i % 2], w)
+        oracle_step(*inputs[i % 2][:2], w, inputs[i % 2][2])
     dt = time.perf_counter() - t0
     value = args.steps / dt
     line = {"metric": w.metric, "value": value, "unit": UNIT, "n_gpus": args.gpus, "steps": args.steps,
@@ -342,7 +368,7 @@ def run_native(args):
     seed = rank_seed(rank) if w.name == DEFAULT_CONFIG else w.seed + 7919 * rank
     wl = make_host_workload(w, B, seed=seed, device=dev)
     view = vk.make_view(wl.cache, wl.q_latent, wl.q_rope)
-    params = vk.make_params(w.rho, r=w.r, window=w.window, trigger=w.trigger, z_eff=w.z_eff)
+    params = vk.make_params(w.rho, r=w.r, window=w.window, trigger=w.trigger, z_eff=w.z_eff, r_sk=w.r_sk)
     # the per-cache index (built once, off the step): digest for r < 64, norms for the trigger
     index = None
     if w.r < 64 or w.trigger:
@@ -352,7 +378,15 @@ def run_native(args):
         eta = torch.empty(B, N, device=dev)
         pres, pk, pe = (torch.empty(B, P, device=dev) for _ in range(3))
         vk.vk_build_digest(view, params, rot, dig, eta, pres, pk, pe)
-        index = vk.make_index(dig, eta, pres, rot if w.r < 64 else None, pk, pe)
+        sketch = basis = None
+        if w.r_sk:
+            # V from the context's prefix queries, then every row's sketch entry (eta becomes the sketch residual)
+            q = datagen.prefix_queries(wl, N_PREFIX - 1).to(dev).contiguous()
+            basis = torch.empty(w.r_sk, 512, device=dev)
+            vk.vk_sketch_basis(q, w.r_sk, basis)
+            sketch = torch.empty(B, N, w.r_sk, dtype=torch.bfloat16, device=dev)
+            vk.vk_build_sketch(view, w.r_sk, basis, sketch, eta)
+        index = vk.make_index(dig, eta, pres, rot if w.r < 64 else None, pk, pe, sketch, basis)
     buf = vk.DecodeBuffers(view, params, device=dev)
     stream = torch.cuda.current_stream(dev)
 
@@ -425,11 +459,11 @@ def run_native(args):
     nS = k + w.window
     U1 = union_rows(buf.idx[..., :nS], torch.minimum(buf.count, torch.tensor(nS, device=dev)), N)
     U = union_rows(buf.idx, buf.count, N) if w.trigger else U1
-    step_b = step_bytes(N, B, w.r, w.dtype, U1, bool(w.trigger), U - U1)
+    step_b = step_bytes(N, B, w.r, w.dtype, U1, bool(w.trigger), U - U1, w.r_sk)
     hbm_peak, peak_kind = peaks()
     sb = score_bytes_per_row(w.r, w.dtype)
     stage_bytes = {"score": B * N * sb, "attn": U1 * row_bytes(w.dtype),
-                   "trigger": B * N * (sb + 4) + (U - U1) * row_bytes(w.dtype)}
+                   "trigger": B * N * (sb + 4 + 2 * w.r_sk) + (U - U1) * row_bytes(w.dtype)}
     cands = ["score", "attn"] + (["trigger"] if w.trigger else [])
     dom = max(cands, key=lambda st: stage_ms[STAGES.index(st)])
     dom_ms = stage_ms[STAGES.index(dom)]

@@ -105,6 +105,10 @@ typedef struct {
  * With index->page_knorm and index->page_eta given, the r = 64 scan of VK_TRIG_CS skips every 128-row tile in which
  * no head's page bound lambda (|Qr_h| max|K| + z_eff |Qc_h| max eta) reaches s*_h: no row there can fire. */
 #define VK_FLAG_NO_PAGE_SKIP 0x8u
+/* Attend the fired rows with the tile pass even when every head fired few rows (for tests; the outputs are the same
+ * up to fp32 rounding). By default the step attends a head's fired rows with a per-head pass over its fired bitmap
+ * when no head fired more than 512 rows, and with the tile pass otherwise. */
+#define VK_FLAG_FIRED_TILES 0x10u
 
 /* The per-cache index built once by vk_build_digest (Sec. 4.2 index entry with sketch rank 0). */
 typedef struct {

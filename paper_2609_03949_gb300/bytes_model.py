@@ -37,15 +37,16 @@ def score_bytes_per_row(r: int, dtype: str) -> int:
 
 
 def step_bytes(N: int, B: int, r: int, dtype: str, union_rows: int, trigger: bool = False,
-               fired_new_rows: int = 0) -> int:
+               fired_new_rows: int = 0, r_sk: int = 0) -> int:
     """Algorithmic bytes of one decode step over B sequences of N cached rows.
 
     union_rows: total distinct rows gathered by tier-1 attention, summed over the batch.
     fired_new_rows: total fired rows not already in the tier-1 union, summed over the batch.
+    r_sk: the trigger scan also reads each row's bf16 content sketch (2 r_sk bytes).
     """
     total = B * N * score_bytes_per_row(r, dtype) + union_rows * row_bytes(dtype)
     if trigger:
-        total += B * N * (score_bytes_per_row(r, dtype) + 4) + fired_new_rows * row_bytes(dtype)
+        total += B * N * (score_bytes_per_row(r, dtype) + 4 + 2 * r_sk) + fired_new_rows * row_bytes(dtype)
     return int(total)
 
 

@@ -129,7 +129,8 @@ __global__ void __launch_bounds__(AT_THREADS, 1) k_attn(
     const T* __restrict__ latent, int64_t lld, int64_t lbs, const T* __restrict__ rope, int64_t rld, int64_t rbs,
     const T* __restrict__ q_latent, const T* __restrict__ q_rope, int H, int N, float lam_log2e,
     const uint32_t* __restrict__ bitmap, int64_t nw, int split_len, int slot0, int nslot, int qrows, int nst,
-    float* __restrict__ part_o, float* __restrict__ part_ml, int* status) {
+    float* __restrict__ part_o, float* __restrict__ part_ml, int* status, const int* __restrict__ skip) {
+  if (skip && *skip) return;                         // another kernel took this pass (the whole block leaves)
   using Slice = typename SliceOf<T>::type;
   constexpr int ROWE = D_LAT + D_ROPE;
   constexpr int ESZ = Elem<T>::bytes;
@@ -357,10 +358,11 @@ size_t attn_smem_bytes(int dtype, int H, int split_len) {
 }
 
 cudaError_t launch_attn(const vk_view& v, float lam, const uint32_t* bitmap, int64_t nw, const AttnGeom& g, int slot0,
-                        int nslot, float* part_o, float* part_ml, uint32_t flags, int* status, cudaStream_t st) {
+                        int nslot, float* part_o, float* part_ml, uint32_t flags, int* status, cudaStream_t st,
+                        const int* skip) {
   // bf16 caches: both contractions on the tensor cores, persistent layout (k_attn_tc.cu); fp32 caches: the SIMT
   // kernel below, split layout
-  if (g.G > 0) return launch_attn_tc(v, lam, bitmap, nw, g, slot0, nslot, part_o, part_ml, flags, status, st);
+  if (g.G > 0) return launch_attn_tc(v, lam, bitmap, nw, g, slot0, nslot, part_o, part_ml, flags, status, st, nullptr, skip);
   const int nsplit = g.nsplit, split_len = g.split_len;
   dim3 grid(nsplit, (v.H + HG - 1) / HG, v.B);
   const int nst = attn_stages(v.dtype, v.H);
@@ -374,7 +376,7 @@ cudaError_t launch_attn(const vk_view& v, float lam, const uint32_t* bitmap, int
     k_attn<T><<<grid, AT_THREADS, smem, st>>>(
         reinterpret_cast<const T*>(v.latent), v.latent_ld, v.latent_bstride, reinterpret_cast<const T*>(v.rope),
         v.rope_ld, v.rope_bstride, reinterpret_cast<const T*>(v.q_latent), reinterpret_cast<const T*>(v.q_rope), v.H,
-        v.N, lam_log2e, bitmap, nw, split_len, slot0, nslot, qrows, nst, part_o, part_ml, status);
+        v.N, lam_log2e, bitmap, nw, split_len, slot0, nslot, qrows, nst, part_o, part_ml, status, skip);
   } else {
     using T = float;
     cudaError_t e = cudaFuncSetAttribute(k_attn<T>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
@@ -382,7 +384,7 @@ cudaError_t launch_attn(const vk_view& v, float lam, const uint32_t* bitmap, int
     k_attn<T><<<grid, AT_THREADS, smem, st>>>(
         reinterpret_cast<const T*>(v.latent), v.latent_ld, v.latent_bstride, reinterpret_cast<const T*>(v.rope),
         v.rope_ld, v.rope_bstride, reinterpret_cast<const T*>(v.q_latent), reinterpret_cast<const T*>(v.q_rope), v.H,
-        v.N, lam_log2e, bitmap, nw, split_len, slot0, nslot, qrows, nst, part_o, part_ml, status);
+        v.N, lam_log2e, bitmap, nw, split_len, slot0, nslot, qrows, nst, part_o, part_ml, status, skip);
   }
   count_launches(1);
   return cudaGetLastError();
@@ -410,15 +412,18 @@ cudaError_t launch_smax_reduce(int B, int H, const AttnGeom& g, int nslot, const
 
 // One warp per (b, h): o = sum_s e^{m_s - m} o_s / sum_s e^{m_s - m} l_s over the written slots of both tiers,
 // lse = m + log(sum), and s* = the max over the tier-1 slots. Slot s of the list is tier-1 slot s for s < nv, else
-// fired slot g.nslot + s - nv (only when nslot covers two tiers).
-__global__ void k_combine(int BH, int H, const AttnGeom g, int nslot, const float* __restrict__ part_o,
+// fired slot g.nslot + s - nv (only when nslot covers two tiers): nf of them (the per-head fired pass writes one), or
+// nv when nf < 0; with `mode` given, *mode != 0 says the per-head pass ran (nf = 1), else the tile pass (nf = nv).
+__global__ void k_combine(int BH, int H, const AttnGeom g, int nslot, int nf, const int* __restrict__ mode,
+                          const float* __restrict__ part_o,
                           const float* __restrict__ part_ml, float* __restrict__ out, float* __restrict__ lse,
                           float* __restrict__ smax) {
   const int wid = (blockIdx.x * blockDim.x + threadIdx.x) >> 5, lane = threadIdx.x & 31;
   if (wid >= BH) return;
   const int b = wid / H, h = wid % H;
   const int nv = attn_nvalid(g, (long long)b * g.n_hg + h / HG);
-  const int nlist = nslot > g.nslot ? 2 * nv : nv;
+  const int nfe = mode ? (*mode ? 1 : -1) : nf;
+  const int nlist = nslot > g.nslot ? nv + (nfe < 0 ? nv : nfe) : nv;
   auto slot_of = [&](int s) { return s < nv ? s : g.nslot + s - nv; };
   float m = -INFINITY, m1 = -INFINITY;
   for (int s = 0; s < nlist; ++s) {
@@ -464,7 +469,8 @@ __global__ void k_combine(int BH, int H, const AttnGeom g, int nslot, const floa
 // slot (lanes over the 512 dims), and the warps' sums are added through shared memory -- the slots' loads run
 // CMB_WARPS wide instead of one slot after another.
 constexpr int CMB_WARPS = 8;
-__global__ void __launch_bounds__(CMB_WARPS * 32) k_combine_wide(int H, const AttnGeom g, int nslot,
+__global__ void __launch_bounds__(CMB_WARPS * 32) k_combine_wide(int H, const AttnGeom g, int nslot, int nf,
+                                                                 const int* __restrict__ mode,
                                                                  const float* __restrict__ part_o,
                                                                  const float* __restrict__ part_ml,
                                                                  float* __restrict__ out, float* __restrict__ lse,
@@ -474,7 +480,8 @@ __global__ void __launch_bounds__(CMB_WARPS * 32) k_combine_wide(int H, const At
   const int bh = blockIdx.x, b = bh / H, h = bh % H;
   const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int nv = attn_nvalid(g, (long long)b * g.n_hg + h / HG);
-  const int nlist = nslot > g.nslot ? 2 * nv : nv;
+  const int nfe = mode ? (*mode ? 1 : -1) : nf;
+  const int nlist = nslot > g.nslot ? nv + (nfe < 0 ? nv : nfe) : nv;
   auto slot_of = [&](int s) { return s < nv ? s : g.nslot + s - nv; };
   float m = -INFINITY, m1 = -INFINITY;
   for (int s = threadIdx.x; s < nlist; s += blockDim.x) {
@@ -542,12 +549,13 @@ __global__ void __launch_bounds__(CMB_WARPS * 32) k_combine_wide(int H, const At
 }
 
 cudaError_t launch_combine(int B, int H, const AttnGeom& g, int nslot, const float* part_o, const float* part_ml,
-                           float* out, float* lse, float* smax, cudaStream_t st) {
+                           float* out, float* lse, float* smax, cudaStream_t st, int nf, const int* mode) {
   const int BH = B * H, threads = 256;
   if (nslot > CMB_WARPS)
-    k_combine_wide<<<BH, CMB_WARPS * 32, 0, st>>>(H, g, nslot, part_o, part_ml, out, lse, smax);
+    k_combine_wide<<<BH, CMB_WARPS * 32, 0, st>>>(H, g, nslot, nf, mode, part_o, part_ml, out, lse, smax);
   else
-    k_combine<<<(BH * 32 + threads - 1) / threads, threads, 0, st>>>(BH, H, g, nslot, part_o, part_ml, out, lse, smax);
+    k_combine<<<(BH * 32 + threads - 1) / threads, threads, 0, st>>>(BH, H, g, nslot, nf, mode, part_o, part_ml, out, lse,
+                                                                     smax);
   count_launches(1);
   return cudaGetLastError();
 }

@@ -92,6 +92,7 @@ struct AttnTcArgs {
   int hold_first;        // VK_FLAG_TEST_TIMEOUT: CTA 0 withholds its first tile's loads
   int* status;
   int* part_arg;         // ARG instantiation: the row of each partial's max logit, [B][nslot][H]
+  const int* skip;       // when non-NULL and *skip != 0 the launch does nothing (another kernel took this pass)
 };
 
 __device__ __forceinline__ void tma_load_3d_(void* dst, const CUtensorMap* map, int x, int y, int z, uint64_t* bar) {
@@ -225,6 +226,7 @@ __global__ void __launch_bounds__(AT_THREADS, 1) k_attn_tc(const __grid_constant
                                                          const __grid_constant__ CUtensorMap qrmap,
                                                          const AttnTcArgs args) {
   extern __shared__ __align__(1024) unsigned char smem_raw[];
+  if (args.skip && *args.skip) return;               // every thread reads the same word: the whole CTA leaves
   unsigned char* smem = reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   unsigned char* sq = smem + AtSmem::q;
   unsigned char* sx = smem + AtSmem::x;
@@ -768,7 +770,7 @@ static bool make_map3(CUtensorMap* map, const void* base, uint64_t cols, uint64_
 
 cudaError_t launch_attn_tc(const vk_view& v, float lam, const uint32_t* bitmap, int64_t nw, const AttnGeom& g,
                            int slot0, int nslot, float* part_o, float* part_ml, uint32_t flags, int* status,
-                           cudaStream_t st, int* part_arg) {
+                           cudaStream_t st, int* part_arg, const int* skip) {
   if (!encode2()) return cudaErrorNotSupported;
   if (g.G < 1 || g.G > g.total || g.T != (v.N + AT_T - 1) / AT_T || g.n_hg != (v.H + 63) / 64 ||
       g.total != (long long)v.B * g.n_hg * g.T)
@@ -794,6 +796,7 @@ cudaError_t launch_attn_tc(const vk_view& v, float lam, const uint32_t* bitmap, 
   a.hold_first = (flags & VK_FLAG_TEST_TIMEOUT) ? 1 : 0;
   a.status = status;
   a.part_arg = part_arg;
+  a.skip = skip;
   const size_t smem = AtSmem::total + 1024;
   auto kernel = part_arg ? k_attn_tc<true> : k_attn_tc<false>;
   cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);

@@ -75,7 +75,7 @@ __global__ void __launch_bounds__(256) k_sketch_rows(int64_t rows, int N, int r_
 }
 
 template <typename T>
-__global__ void __launch_bounds__(256) k_sketch_query(int B, int H, int r_sk, const T* __restrict__ q_latent,
+__global__ void __launch_bounds__(512) k_sketch_query(int B, int H, int r_sk, const T* __restrict__ q_latent,
                                                       const float* __restrict__ basis, float* __restrict__ p,
                                                       __nv_bfloat16* __restrict__ phl, float* __restrict__ rho) {
   extern __shared__ float vb[];
@@ -322,17 +322,18 @@ cudaError_t launch_sketch_query(const vk_view& v, int r_sk, const float* basis, 
                                 cudaStream_t st) {
   const int64_t BH = (int64_t)v.B * v.H;
   const size_t smem = vb_smem(r_sk);
-  const int grid = (int)((BH + 7) / 8);
+  // 16 queries per block: each block stages the basis (up to 128 KB) once for 16 warps
+  const int grid = (int)((BH + 15) / 16);
   auto* hl = static_cast<__nv_bfloat16*>(phl);
   cudaError_t e;
   if (v.dtype == VK_BF16) {
     if ((e = allow_smem(k_sketch_query<__nv_bfloat16>, smem)) != cudaSuccess) return e;
-    k_sketch_query<__nv_bfloat16><<<grid, 256, smem, st>>>(v.B, v.H, r_sk,
+    k_sketch_query<__nv_bfloat16><<<grid, 512, smem, st>>>(v.B, v.H, r_sk,
                                                           static_cast<const __nv_bfloat16*>(v.q_latent), basis, p, hl,
                                                           rho);
   } else {
     if ((e = allow_smem(k_sketch_query<float>, smem)) != cudaSuccess) return e;
-    k_sketch_query<float><<<grid, 256, smem, st>>>(v.B, v.H, r_sk, static_cast<const float*>(v.q_latent), basis, p,
+    k_sketch_query<float><<<grid, 512, smem, st>>>(v.B, v.H, r_sk, static_cast<const float*>(v.q_latent), basis, p,
                                                   hl, rho);
   }
   count_launches(1);

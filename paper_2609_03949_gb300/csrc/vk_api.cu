@@ -88,7 +88,8 @@ int check_params(const vk_view* v, const vk_params* p) {
     return fail(VK_ERR_INVALID_ARG, "trigger = %d is unknown", p->trigger);
   if (!(p->z_eff >= 0.f) || !std::isfinite(p->z_eff)) return fail(VK_ERR_INVALID_ARG, "z_eff must be finite and >= 0");
   if (p->top_j < 0) return fail(VK_ERR_INVALID_ARG, "top_j must be >= 0");
-  if (p->flags & ~(VK_FLAG_FORCE_FALLBACK | VK_FLAG_FORCE_DENSE | VK_FLAG_TEST_TIMEOUT | VK_FLAG_NO_PAGE_SKIP))
+  if (p->flags & ~(VK_FLAG_FORCE_FALLBACK | VK_FLAG_FORCE_DENSE | VK_FLAG_TEST_TIMEOUT | VK_FLAG_NO_PAGE_SKIP |
+                   VK_FLAG_FIRED_TILES))
     return fail(VK_ERR_INVALID_ARG, "unknown flags 0x%x", p->flags);
   if (p->r_sk != 0 && p->r_sk != 16 && p->r_sk != 32 && p->r_sk != 64)
     return fail(VK_ERR_INVALID_ARG, "r_sk = %d is not in {0, 16, 32, 64}", p->r_sk);
@@ -254,6 +255,7 @@ VkLayout make_layout(const vk_view& v, const vk_params& p) {
   L.off_skp = take(L.sketch ? sizeof(float) * BH * p.r_sk : 0);
   L.off_skhl = take(L.sketch ? sizeof(uint16_t) * BH * 2 * p.r_sk : 0);
   L.off_rho = take(L.sketch ? sizeof(float) * BH : 0);
+  L.off_fmode = take(L.two_tier ? sizeof(int) : 0);
   L.total = off;
   return L;
 }
@@ -409,6 +411,9 @@ int vk_sparse_attn(const vk_view* view, const vk_params* params, const int32_t* 
   VK_CUDA(vk::launch_combine(view->B, view->H, L.ag, L.ag.nslot, po, pml, out, lse, smax, st), "combine");
   return VK_OK;
 }
+
+// Largest fired set per head for which the per-head pass over the fired rows beats the tile pass.
+constexpr int kFiredListMax = 512;
 
 int vk_decode_step(const vk_view* view, const vk_params* params, const vk_index* index, float* out, float* lse,
                    float* smax, int32_t* idx, int32_t* count, int32_t cap, void* ws, size_t ws_bytes, void* stream) {
@@ -584,11 +589,21 @@ int vk_decode_step(const vk_view* view, const vk_params* params, const vk_index*
         VK_CUDA(vk::launch_bitmap_to_list(B, H, N, firebm, L.nw, idx, count, cap, status, st), "fired list");
       }
     }
-    VK_CUDA(vk::launch_attn(v, params->sm_scale, firebm, L.nw, L.ag, ns, nslot, po, pml, 0u, status, st),
-            "fired attention");
+    // The fired rows: when every head fired at most kFiredListMax rows (the usual case: the tier fetches only rows
+    // that could still compete), one partial per (b, h) over its own fired bitmap, in the first fired slot; otherwise
+    // the tile pass, which shares each loaded tile among a group's heads. The choice is made on the device from the
+    // fired counts; the pass not chosen, and the merge, read the same flag.
+    int* fmode = at<int>(ws, L.off_fmode);
+    const int list_max = (params->flags & VK_FLAG_FIRED_TILES) ? -1 : kFiredListMax;
+    VK_CUDA(vk::launch_fired_mode((int64_t)B * H, count, (int)(k + W + S), list_max, fmode, st), "fired mode");
+    VK_CUDA(vk::launch_attn_list(v, params->sm_scale, firebm, L.nw, nslot, ns, po, pml, status, fmode, st),
+            "fired attention (per head)");
+    VK_CUDA(vk::launch_attn(v, params->sm_scale, firebm, L.nw, L.ag, ns, nslot, po, pml, 0u, status, st, fmode),
+            "fired attention (tiles)");
   }
   prof(5, st);
-  VK_CUDA(vk::launch_combine(B, H, L.ag, nslot, po, pml, out, lse, smax, st), "combine");
+  VK_CUDA(vk::launch_combine(B, H, L.ag, nslot, po, pml, out, lse, smax, st, -1,
+                             two_tier ? at<int>(ws, L.off_fmode) : nullptr), "combine");
   prof(6, st);
   return VK_OK;
 }

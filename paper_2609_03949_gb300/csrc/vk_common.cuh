@@ -112,7 +112,7 @@ struct VkLayout {
   int64_t fcap;                 // two-tier top_j (fused path or page trigger): fired-candidate capacity per head
   size_t off_status, off_qt, off_qhl, off_qcn, off_qrn, off_qrf, off_smax1, off_nfired, off_scores, off_selbm, off_firebm,
       off_part_o, off_part_ml, off_sample, off_theta, off_ccnt, off_cand, off_fcnt, off_fcand, off_skp, off_skhl,
-      off_rho, total;
+      off_rho, off_fmode, total;
   bool sketch;                  // row-level trigger with a content sketch (r_sk > 0)
 };
 
@@ -148,13 +148,22 @@ AttnGeom attn_geom(const vk_view& v);
 // argmax over the attended rows).
 cudaError_t launch_attn_tc(const vk_view& v, float lam, const uint32_t* bitmap, int64_t nw, const AttnGeom& g,
                            int slot0, int nslot, float* part_o, float* part_ml, uint32_t flags, int* status,
-                           cudaStream_t st, int* part_arg = nullptr);
+                           cudaStream_t st, int* part_arg = nullptr, const int* skip = nullptr);
+// skip (device, may be NULL): when *skip != 0 the launch does nothing (the fired rows' pass taken by k_attn_list)
 cudaError_t launch_attn(const vk_view& v, float lam, const uint32_t* bitmap, int64_t nw, const AttnGeom& g, int slot0,
-                        int nslot, float* part_o, float* part_ml, uint32_t flags, int* status, cudaStream_t st);
+                        int nslot, float* part_o, float* part_ml, uint32_t flags, int* status, cudaStream_t st,
+                        const int* skip = nullptr);
 cudaError_t launch_smax_reduce(int B, int H, const AttnGeom& g, int nslot, const float* part_ml, float* smax,
                                cudaStream_t st);
 cudaError_t launch_combine(int B, int H, const AttnGeom& g, int nslot, const float* part_o, const float* part_ml,
-                           float* out, float* lse, float* smax, cudaStream_t st);
+                           float* out, float* lse, float* smax, cudaStream_t st, int nf = -1,
+                           const int* mode = nullptr);
+// The fired rows' attention (k_attn_list.cu): one partial per (b, h) over the rows its fired bitmap [B][H][nw] marks,
+// into slot `slot` of the [B][nslot][H] partial layout; nothing when *mode == 0. launch_fired_mode sets mode[0] = 1 when
+// every head fired at most `limit` rows (count[i] - n0), else 0.
+cudaError_t launch_fired_mode(int64_t BH, const int32_t* count, int n0, int limit, int* mode, cudaStream_t st);
+cudaError_t launch_attn_list(const vk_view& v, float lam, const uint32_t* bitmap, int64_t nw, int nslot, int slot,
+                             float* part_o, float* part_ml, int* status, const int* mode, cudaStream_t st);
 cudaError_t launch_trigger_dense(int B, int H, int N, int W, int n_sink, float lam, float z_eff, int top_j,
                                  float* scores, const float* qcn, const float* qrn, const float* eta,
                                  const float* page_res, const float* smax1, const uint32_t* selbm,

@@ -19,6 +19,7 @@ VK_ERR_CAPACITY, VK_ERR_CUDA, VK_ERR_TIMEOUT = -4, -5, -6
 VK_BF16, VK_F32 = 0, 1
 VK_TRIG_OFF, VK_TRIG_CS, VK_TRIG_CS_PAGE = 0, 1, 2
 VK_FLAG_FORCE_FALLBACK, VK_FLAG_FORCE_DENSE, VK_FLAG_TEST_TIMEOUT, VK_FLAG_NO_PAGE_SKIP = 0x1, 0x2, 0x4, 0x8
+VK_FLAG_FIRED_TILES = 0x10
 D_LATENT, D_ROPE, PAGE = 512, 64, 64
 DEFAULT_SM_SCALE = 1.0 / math.sqrt(192.0)
 

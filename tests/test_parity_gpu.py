@@ -407,3 +407,17 @@ def test_attention_rescale_on_logit_jump(c):
     g = dict(out=out.cpu().double().numpy(), lse=lse.cpu().double().numpy())
     r = check_outputs(hi, LAM, g, idx, cnt)
     np.testing.assert_allclose(smax.cpu().double().numpy(), r["smax"], rtol=1e-4, atol=1e-4)
+
+
+@pytest.mark.parametrize("z,top_j", [(0.05, 0), (1.0, 0), (0.3, 12)])
+def test_fired_passes_agree(z, top_j):
+    """The fired rows' two passes (per head over its fired bitmap when no head fired more than 512 rows, else by
+    tiles) give the same outputs up to fp32 rounding, and both meet the oracle."""
+    wl = datagen.config_workload("h128_n64k_two_tier", device="cuda", B=2, N=8192)
+    a = run_case(wl, rho=1 / 32, window=256, trigger=1, z_eff=z, top_j=top_j)
+    b = run_case(wl, rho=1 / 32, window=256, trigger=1, z_eff=z, top_j=top_j, flags=vk.VK_FLAG_FIRED_TILES)
+    ga, gb = a["gpu"], b["gpu"]
+    np.testing.assert_array_equal(ga["idx"], gb["idx"])
+    np.testing.assert_array_equal(ga["count"], gb["count"])
+    np.testing.assert_allclose(ga["out"], gb["out"], rtol=1e-4, atol=1e-5)
+    np.testing.assert_allclose(ga["lse"], gb["lse"], rtol=1e-5, atol=1e-5)
