@@ -337,6 +337,9 @@ cudaError_t launch_select_dense(int B, int H, int N, const float* scores, const 
 // sample[(b*H + h) * ns + i] is the score of position off + stride * i, in bf16 (theta only steers how many
 // candidates pass; the candidates themselves carry fp32 scores). Up to THETA_R x 256 archive samples are
 // held in registers (THETA_R per thread, loaded together); more go through shared memory (ns x 4 bytes).
+// Measured slower at B = 64, N = 65536, H = 64 (36 us here): one warp per head with exact two-pass 8-bit histograms
+// of the 16-bit bf16 keys (43-47 us: a head's scores share a few exponents, so the first pass's shared-memory
+// atomics pile onto a few buckets), and the same with the lanes of a bucket aggregated by match_any (102 us).
 constexpr int THETA_R = 16;
 __global__ void __launch_bounds__(CAND_THREADS) k_theta(int ns, int ld, int off, int stride, int lo, int hi, int j,
                                                         const __nv_bfloat16* __restrict__ sample,
