@@ -193,3 +193,31 @@ def test_sketch_tightens_the_gpu_trigger():
     nS = oracle.keep_count(8192, 1 / 32, 128) + 128
     f0 = int((g0["count"] - nS).sum())
     assert f_sk < 0.5 * f0, (f_sk, f0)
+
+
+def test_sketch_fp32_cache():
+    """fp32 caches: materialised scores, the dense trigger scan with the sketch term, the fp32 per-head fired pass."""
+    wl = datagen.make_workload(1, 16, 2048, dtype="f32", seed=91, n_planted=0, query_rank=8)
+    rng = np.random.default_rng(91)
+    for h in range(0, 16, 3):
+        u = int(rng.integers(0, 1400))
+        qc = wl.q_latent[0, h].float()
+        wl.cache[0, u, :512] = 3.0 * qc / qc.norm()
+    fired, swaps = run_sketch_case(wl, r_sk=32, window=64, rho_keep=1 / 16, z_eff=0.5)
+    assert fired > 0
+    assert swaps <= max(2, fired // 100)
+
+
+def test_sketch_256_heads_dense_scan():
+    """More than 128 heads with a sketch: the step materialises the scores and the dense scan adds the sketch term."""
+    wl = sketch_workload(1, 256, 4096, seed=93, planted_frac=5)
+    fired, swaps = run_sketch_case(wl, r_sk=64, z_eff=0.5)
+    assert fired > 0
+    assert swaps <= max(2, fired // 100)
+
+
+@pytest.mark.parametrize("r,top_j", [(16, 5), (64, 3)])
+def test_sketch_top_j(r, top_j):
+    wl = sketch_workload(2, 64, 4096, seed=95 + r)
+    fired, _ = run_sketch_case(wl, r_sk=32, r=r, z_eff=0.3, top_j=top_j)
+    assert 0 < fired <= 2 * 64 * top_j
