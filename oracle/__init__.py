@@ -78,7 +78,7 @@ def lib():
         L.vko_min_hard.restype = I64
         L.vko_conformal_quantile.argtypes = [P, I64, D, D]
         L.vko_conformal_quantile.restype = D
-        L.vko_calib_zq.argtypes = [VP, I32, P, D, P, P, P, P, P, I32, P, P]
+        L.vko_calib_zq.argtypes = [VP, I32, P, D, P, P, P, I32, P, P, P, P, P, I32, P, P]
         L.vko_calib_zq.restype = I64
         L.vko_sketch_basis.argtypes = [P, I64, I32, P, P]
         L.vko_sketch_basis.restype = ctypes.c_int
@@ -371,8 +371,9 @@ def conformal_quantile(zq, tau: float = 0.9, z_max: float = 8.0) -> float:
 
 
 def calib_zq(hi: HostInputs, r: int, lam: float, a: np.ndarray, eta: np.ndarray, page_res: np.ndarray,
-             idx: np.ndarray, count: np.ndarray):
-    """(zq [B,H] with NaN where the query is not hard, ustar [B,H], n_hard) for every (b, h) as a calibration query."""
+             idx: np.ndarray, count: np.ndarray, sketch=None):
+    """(zq [B,H] with NaN where the query is not hard, ustar [B,H], n_hard) for every (b, h) as a calibration query.
+    ``sketch`` = (s16, p, rho) as for ``trigger``: the sketch term and certificate (eta then the sketch residual)."""
     a = np.ascontiguousarray(a, dtype=np.float64)
     eta = np.ascontiguousarray(eta, dtype=np.float64)
     page_res = np.ascontiguousarray(page_res, dtype=np.float64)
@@ -380,6 +381,13 @@ def calib_zq(hi: HostInputs, r: int, lam: float, a: np.ndarray, eta: np.ndarray,
     count = np.ascontiguousarray(count, dtype=np.int32)
     zq = np.zeros((hi.B, hi.H), np.float64)
     ustar = np.zeros((hi.B, hi.H), np.int32)
+    r_sk, s16, p, rho = 0, None, None, None
+    if sketch is not None:
+        s16 = np.ascontiguousarray(sketch[0], dtype=np.uint16)
+        p = np.ascontiguousarray(sketch[1], dtype=np.float64)
+        rho = np.ascontiguousarray(sketch[2], dtype=np.float64)
+        r_sk = s16.shape[-1]
     n = lib().vko_calib_zq(ctypes.byref(hi.view), int(r), _ptr(hi.rot), float(lam), _ptr(a), _ptr(eta), _ptr(page_res),
-                           _ptr(idx), _ptr(count), idx.shape[-1], _ptr(zq), _ptr(ustar))
+                           r_sk, _ptr(s16), _ptr(p), _ptr(rho), _ptr(idx), _ptr(count), idx.shape[-1], _ptr(zq),
+                           _ptr(ustar))
     return zq, ustar, int(n)

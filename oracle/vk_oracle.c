@@ -817,11 +817,13 @@ double vko_conformal_quantile(const double* zq, int64_t n, double tau, double z_
  * tier can bring it back. For a hard query the required inflation is the z at which u*'s trigger score reaches the
  * tier-1 maximum s* = max over S_h: with sketch rank 0 the index part is idx_t = lambda (a[h,u*] +
  * |(O qr_h)[r:]| page_res[page(u*)]) and the certificate scale cert_t = lambda |qc_h| eta_u* / sqrt(d_c), d_c = 512,
- * so zq = (s* - idx_t) / cert_t. a, eta, page_res as from vko_scores and vko_build_index. zq[b,h] gets NaN for a query
- * that is not hard; ustar[b,h] the argmax row. Returns the number of hard queries. */
+ * so zq = (s* - idx_t) / cert_t. With a rank-r_sk content sketch (sk16, p, rho as for vko_trigger, eta the sketch
+ * residual norms) the index part gains p_h . s_u* and the certificate is lambda rho_h eta_u* / sqrt(d_c - r_sk) (Eq. 4).
+ * a, eta, page_res as from vko_scores and vko_build_index (or vko_build_sketch). zq[b,h] gets NaN for a query that
+ * is not hard; ustar[b,h] the argmax row. Returns the number of hard queries. */
 int64_t vko_calib_zq(const vko_view* v, int32_t r, const float* rot, double lam, const double* a, const double* eta,
-                     const double* page_res, const int32_t* idx, const int32_t* count, int32_t cap, double* zq,
-                     int32_t* ustar) {
+                     const double* page_res, int32_t r_sk, const uint16_t* sk16, const double* p, const double* rho,
+                     const int32_t* idx, const int32_t* count, int32_t cap, double* zq, int32_t* ustar) {
   const int64_t N = v->N, P = (N + PAGE - 1) / PAGE;
   int64_t n_hard = 0;
 #pragma omp parallel for collapse(2) schedule(dynamic) reduction(+ : n_hard)
@@ -852,8 +854,11 @@ int64_t vko_calib_zq(const vko_view* v, int32_t r, const float* rot, double lam,
         }
         for (int j = 0; j < D_LAT; ++j) qcn += QC(v, b, h, j) * QC(v, b, h, j);
         qcn = sqrt(qcn);
-        const double idx_t = lam * (a[bh * N + us] + qres * page_res[(int64_t)b * P + us / PAGE]);
-        const double cert_t = lam * qcn * eta[(int64_t)b * N + us] / sqrt((double)D_LAT);
+        double skt = 0.0;
+        for (int j = 0; j < r_sk; ++j) skt += p[bh * r_sk + j] * from_bf16(sk16[((int64_t)b * N + us) * r_sk + j]);
+        const double idx_t = lam * (a[bh * N + us] + qres * page_res[(int64_t)b * P + us / PAGE] + skt);
+        const double cq = r_sk > 0 ? rho[bh] : qcn;
+        const double cert_t = lam * cq * eta[(int64_t)b * N + us] / sqrt((double)(D_LAT - r_sk));
         zq[bh] = (sstar - idx_t) / cert_t;
         ++n_hard;
       }

@@ -211,8 +211,45 @@ def pin_decode_step_composes():
     assert oracle.decode_step(hi, rho=rho_keep, window=W, trigger=2, sketch_basis=V)["rc"] == -1
 
 
+def pin_calibration_matches_sketch_trigger():
+    # hard queries (the argmax row's RoPE score is ordinary, so tier 1 leaves it out): the required inflation computed
+    # with the sketch puts the row exactly on s* in the sketch trigger at z_eff = zq / sqrt(512 - r_sk) -- just above
+    # it fires, just below it does not
+    # the planted row points along the query's residual outside span(V): its logit dominates but the sketch term
+    # cannot see it, so only the certificate can bring it back (a positive required inflation)
+    wl = datagen.make_workload(1, 4, 512, seed=33, query_rank=8, n_planted=0)
+    r_sk, W = 16, 32
+    V, _ = oracle.sketch_basis(datagen.prefix_queries(wl, 100).double().numpy(), r_sk)
+    for h in range(4):
+        qc = wl.q_latent[0, h].double().numpy()
+        res = qc - V.T @ (V @ qc)
+        wl.cache[0, 100 + 37 * h, :512] = torch.as_tensor(12.0 * res / np.linalg.norm(res)).to(wl.cache.dtype)
+    hi = oracle.HostInputs(wl)
+    a = oracle.scores(hi)
+    idx, cnt, _ = oracle.select(a, 8, W)
+    _, s16, eta = oracle.build_sketch(hi, V)
+    p, rho = oracle.sketch_query(hi, V)
+    pres = oracle.build_index(hi, 64)[3]
+    zq, ustar, n = oracle.calib_zq(hi, 64, LAM, a, eta, pres, idx, cnt, sketch=(s16, p, rho))
+    _, _, smax = oracle.attention(hi, LAM, idx, cnt)
+    checked = 0
+    for h in range(4):
+        if np.isnan(zq[0, h]) or zq[0, h] <= 0:
+            continue
+        for f, fires in ((1 + 1e-9, True), (1 - 1e-9, False)):
+            z_eff = f * zq[0, h] / math.sqrt(512 - r_sk)
+            fidx, fcnt = oracle.trigger(hi, 64, LAM, z_eff, 0, a, eta, pres, idx, cnt, smax, W, sketch=(s16, p, rho))
+            assert (int(ustar[0, h]) in fidx[0, h, :fcnt[0, h]].tolist()) == fires, (h, f)
+        checked += 1
+    assert checked >= 1 and n >= checked
+    # without the sketch the same queries need a different (rank-0) inflation
+    _, _, eta0, _ = oracle.build_index(hi, 64)
+    zq0, _, _ = oracle.calib_zq(hi, 64, LAM, a, eta0, pres, idx, cnt)
+    assert np.nanmax(np.abs(zq0 - zq)) > 1e-3
+
+
 PINS = [pin_basis_matches_eigh, pin_basis_known_spectrum, pin_basis_direct_route, pin_index_entry, pin_query_side, pin_trigger_hand_case,
-        pin_lemma1_soundness, pin_decode_step_composes]
+        pin_lemma1_soundness, pin_decode_step_composes, pin_calibration_matches_sketch_trigger]
 
 
 @pytest.mark.parametrize("pin", PINS, ids=lambda f: f.__name__)
