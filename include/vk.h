@@ -225,8 +225,9 @@ int vk_decode_step_noalloc(const vk_view* view, const vk_params* params, const v
  * when n < min_hard or that index passes n, clamped to [0, z_max]. Outputs (device): zq [B, H] fp32, NaN where the
  * query is not hard; z_out[3] = {z, z_eff = z / sqrt(512) (the decode step's z_eff), n_hard}. index needs eta and
  * page_res (and the digest and rotation when r < 64); bf16 caches only (the argmax runs on the tensor-core
- * attention over every row); B * H <= 16384 (one block sorts the zq). params->r_sk must be 0 (VK_ERR_UNSUPPORTED
- * otherwise): the calibration computes the sketch-rank-0 certificate. */
+ * attention over every row); B * H <= 16384 (one block sorts the zq). With params->r_sk > 0 (and the index's sketch
+ * and basis, eta the sketch residual) the index part gains p_h . s_u* and cert_t = lambda rho_h eta_u* /
+ * sqrt(512 - r_sk), the sketch certificate of Eq. 4; z_out[1] is then z / sqrt(512 - r_sk). */
 size_t vk_conformal_workspace_bytes(const vk_view* view, const vk_params* params);
 int vk_conformal_z(const vk_view* view, const vk_params* params, const vk_index* index, const int32_t* idx,
                    const int32_t* count, int32_t cap, float tau, float z_max, float* zq, float* z_out, void* ws,

@@ -5,9 +5,11 @@
 // when u* lies outside its attended set S_h. For a hard query the required inflation is
 //   zq = (s* - idx_t) / cert_t,  idx_t = lambda (a[h,u*] + |(O Qr_h)[r:]| page_res[page(u*)]),
 //                                cert_t = lambda |Qc_h| eta_u* / sqrt(d_c),  d_c = 512 (sketch rank 0),
-// with s* the max logit over S_h. z is then the ceil((n+1) tau_s)-th smallest zq over the n hard queries (tau_s =
-// tau / (1 - alpha), alpha = (1 - tau)/2), Z_max when n < min_hard = ceil(tau_s / (1 - tau_s)) or the index passes
-// n, clamped to [0, Z_max]; z_eff = z / sqrt(d_c) is the decode step's parameter.
+// with s* the max logit over S_h. With a rank-r_sk content sketch the index part gains p_h . s_u* and the certificate
+// is lambda rho_h eta_u* / sqrt(d_c - r_sk) (eta the sketch residual). z is then the ceil((n+1) tau_s)-th smallest zq
+// over the n hard queries (tau_s = tau / (1 - alpha), alpha = (1 - tau)/2), Z_max when n < min_hard =
+// ceil(tau_s / (1 - tau_s)) or the index passes n, clamped to [0, Z_max]; z_eff = z / sqrt(d_c - r_sk) is the decode
+// step's parameter.
 #include <cmath>
 
 #include "vk_common.cuh"
@@ -22,7 +24,9 @@ __global__ void k_calib_zq(int B, int H, int N, AttnGeom g, int slot0, int nslot
                            const float* __restrict__ qcn, const float* __restrict__ qrn,
                            const __nv_bfloat16* __restrict__ rope, int64_t rld, int64_t rbs,
                            const __nv_bfloat16* __restrict__ digest, const float* __restrict__ eta,
-                           const float* __restrict__ page_res, float lam, float* __restrict__ zq) {
+                           const float* __restrict__ page_res, float lam, int r_sk, const float* __restrict__ skp,
+                           const __nv_bfloat16* __restrict__ sketch, const float* __restrict__ rho,
+                           float* __restrict__ zq) {
   const int64_t bh = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
   if (bh >= (int64_t)B * H) return;
   const int b = (int)(bh / H), h = (int)(bh - (int64_t)b * H);
@@ -49,9 +53,12 @@ __global__ void k_calib_zq(int B, int H, int N, AttnGeom g, int slot0, int nslot
     const __nv_bfloat16* d = digest + ((int64_t)b * N + pos) * r;
     for (int j = 0; j < r; ++j) a = fmaf(q[j], __bfloat162float(d[j]), a);
   }
+  for (int j = 0; j < r_sk; ++j)
+    a = fmaf(skp[bh * r_sk + j], __bfloat162float(sketch[((int64_t)b * N + pos) * r_sk + j]), a);
   const int64_t P = (N + PAGE - 1) / PAGE;
   const float idx_t = lam * (a + qrn[bh] * page_res[(int64_t)b * P + pos / PAGE]);
-  const float cert_t = lam * qcn[bh] * eta[(int64_t)b * N + pos] * (1.0f / sqrtf((float)D_LAT));
+  const float cq = r_sk > 0 ? rho[bh] : qcn[bh];
+  const float cert_t = lam * cq * eta[(int64_t)b * N + pos] * (1.0f / sqrtf((float)(D_LAT - r_sk)));
   zq[bh] = (smax1[bh] - idx_t) / cert_t;
 }
 
@@ -60,7 +67,7 @@ __global__ void k_calib_zq(int B, int H, int N, AttnGeom g, int slot0, int nslot
 constexpr int CQ_THREADS = 1024;
 __global__ void __launch_bounds__(CQ_THREADS) k_conformal_quantile(int64_t BH, const float* __restrict__ zq,
                                                                  double tau_s, int min_hard, float z_max,
-                                                                 float* __restrict__ out) {
+                                                                 int r_sk, float* __restrict__ out) {
   extern __shared__ float vals[];
   __shared__ int cnt;
   if (threadIdx.x == 0) cnt = 0;
@@ -94,7 +101,7 @@ __global__ void __launch_bounds__(CQ_THREADS) k_conformal_quantile(int64_t BH, c
       if (k >= 1 && k <= n) z = fminf(fmaxf(vals[k - 1], 0.f), z_max);
     }
     out[0] = z;
-    out[1] = z * (1.0f / sqrtf((float)D_LAT));
+    out[1] = z * (1.0f / sqrtf((float)(D_LAT - r_sk)));
     out[2] = (float)n;
   }
 }
@@ -111,16 +118,17 @@ cudaError_t launch_calib(const vk_view& v, int r, const AttnGeom& g, int slot0, 
                          const int* part_arg, const float* smax1, const uint32_t* selbm, int64_t nw, const float* qt,
                          const float* qcn, const float* qrn, const void* digest, const float* eta,
                          const float* page_res, float lam, double tau_s, int min_hard, float z_max, float* zq,
-                         float* z_out, cudaStream_t st) {
+                         float* z_out, cudaStream_t st, int r_sk, const float* skp, const void* sketch,
+                         const float* rho) {
   const int64_t BH = (int64_t)v.B * v.H;
   k_calib_zq<<<(unsigned)((BH + 127) / 128), 128, 0, st>>>(
       v.B, v.H, v.N, g, slot0, nslot, part_ml, part_arg, smax1, selbm, nw, r, qt, qcn, qrn,
       static_cast<const __nv_bfloat16*>(v.rope), v.rope_ld, v.rope_bstride, static_cast<const __nv_bfloat16*>(digest),
-      eta, page_res, lam, zq);
+      eta, page_res, lam, r_sk, skp, static_cast<const __nv_bfloat16*>(sketch), rho, zq);
   const size_t smem = conformal_smem_bytes(BH);
   cudaError_t e = cudaFuncSetAttribute(k_conformal_quantile, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
-  k_conformal_quantile<<<1, CQ_THREADS, smem, st>>>(BH, zq, tau_s, min_hard, z_max, z_out);
+  k_conformal_quantile<<<1, CQ_THREADS, smem, st>>>(BH, zq, tau_s, min_hard, z_max, r_sk, z_out);
   count_launches(2);
   return cudaGetLastError();
 }

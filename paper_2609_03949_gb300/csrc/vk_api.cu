@@ -636,8 +636,6 @@ int vk_conformal_z(const vk_view* view, const vk_params* params, const vk_index*
   g_err[0] = 0;
   int rc;
   if ((rc = check_view(view)) != VK_OK || (rc = check_params(view, params)) != VK_OK) return rc;
-  if (params->r_sk > 0)
-    return fail(VK_ERR_UNSUPPORTED, "the calibration computes the sketch-rank-0 certificate; r_sk must be 0");
   const vk_params q = calib_params(*params);
   if ((rc = check_index(view, &q, index, true)) != VK_OK) return rc;
   if (!vk::attn_tc_supported(*view)) return fail(VK_ERR_UNSUPPORTED, "the calibration's argmax pass reads bf16 caches");
@@ -675,8 +673,17 @@ int vk_conformal_z(const vk_view* view, const vk_params* params, const vk_index*
   VK_CUDA(cudaMemsetAsync(allbm, 0xff, sizeof(uint32_t) * BH * L.nw, st), "all rows");
   VK_CUDA(vk::launch_attn_tc(v, q.sm_scale, allbm, L.nw, L.ag, ns, nslot, po, pml, 0u, status, st, parg),
           "attention (all rows)");
+  // with a content sketch: the queries' sketch coordinates and residual norms for the index part and certificate
+  float* skp = nullptr;
+  float* rho = nullptr;
+  if (L.sketch) {
+    skp = at<float>(ws, L.off_skp);
+    rho = at<float>(ws, L.off_rho);
+    VK_CUDA(vk::launch_sketch_query(v, q.r_sk, index->sketch_basis, skp, nullptr, rho, st), "sketch query");
+  }
   VK_CUDA(vk::launch_calib(v, q.r, L.ag, ns, nslot, pml, parg, smax1, selbm, L.nw, qt, qcn, qrn, index->digest,
-                           index->eta, index->page_res, q.sm_scale, tau_s, min_hard, z_max, zq, z_out, st),
+                           index->eta, index->page_res, q.sm_scale, tau_s, min_hard, z_max, zq, z_out, st,
+                           L.sketch ? q.r_sk : 0, skp, L.sketch ? index->sketch : nullptr, rho),
           "conformal z");
   return VK_OK;
 }

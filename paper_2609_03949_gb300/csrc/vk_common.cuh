@@ -202,7 +202,8 @@ cudaError_t launch_calib(const vk_view& v, int r, const AttnGeom& g, int slot0, 
                          const int* part_arg, const float* smax1, const uint32_t* selbm, int64_t nw, const float* qt,
                          const float* qcn, const float* qrn, const void* digest, const float* eta,
                          const float* page_res, float lam, double tau_s, int min_hard, float z_max, float* zq,
-                         float* z_out, cudaStream_t st);
+                         float* z_out, cudaStream_t st, int r_sk = 0, const float* skp = nullptr,
+                         const void* sketch = nullptr, const float* rho = nullptr);
 // PCA digest basis (k_pca.cu): workspace = status word + the fp64 second moment
 size_t pca_workspace_bytes();
 cudaError_t launch_pca_basis(const vk_view& v, float* rot, float* eig, void* ws, cudaStream_t st);

@@ -86,3 +86,48 @@ def test_conformal_z_matches_oracle(r, z_max):
     assert zo[0] == pytest.approx(oracle.conformal_quantile(gz[hard], 0.9, z_max), abs=1e-6)
     assert zo[0] == pytest.approx(oracle.conformal_quantile(rzq[~np.isnan(rzq)], 0.9, z_max), abs=2e-3 + 1e-3 * zo[0])
     assert zo[1] == pytest.approx(zo[0] / math.sqrt(512.0), rel=1e-6)
+
+
+@pytest.mark.parametrize("r_sk", [16, 64])
+def test_conformal_z_with_sketch(r_sk):
+    """Calibration with the rank-r_sk sketch certificate: queries of rank 8 plus noise; for a third of the heads a row
+    along the query's residual outside the basis span (only the certificate can bring it back), so those are hard."""
+    B, H, N, W = 2, 64, 8192, 256
+    wl = datagen.make_workload(B, H, N, seed=111 + r_sk, n_planted=0, query_rank=8)
+    V, _ = oracle.sketch_basis(datagen.prefix_queries(wl, 200).double().numpy(), r_sk)
+    rng = np.random.default_rng(r_sk)
+    for b in range(B):
+        for h in range(0, H, 3):
+            qc = wl.q_latent[b, h].double().numpy()
+            res = qc - V.T @ (V @ qc)
+            u = int(rng.integers(0, N - 512))
+            wl.cache[b, u, :512] = torch.as_tensor(12.0 * res / np.linalg.norm(res)).to(wl.cache.dtype)
+    hi = oracle.HostInputs(wl)
+    _, s16, eta = oracle.build_sketch(hi, V)
+    p, rho = oracle.sketch_query(hi, V)
+    # tier 1 without the trigger; the sketch index rides along for the calibration
+    step = GpuStep(wl, rho=1 / 32, window=W)
+    g = step.run()
+    assert g["status"] == vk.VK_OK
+    sk = torch.from_numpy(s16.astype(np.int16)).view(torch.bfloat16).cuda().contiguous()
+    basis = torch.as_tensor(V, dtype=torch.float32).cuda().contiguous()
+    eta_g = torch.as_tensor(eta, dtype=torch.float32).cuda().contiguous()
+    index = vk.make_index(None, eta_g, step.page_res, None, None, None, sk, basis)
+    params = vk.make_params(1 / 32, window=W, trigger=vk.VK_TRIG_CS, r_sk=r_sk)
+    zq = torch.empty(B, H, device="cuda")
+    z_out = torch.empty(3, device="cuda")
+    ws = vk.vk_conformal_z(step.view, params, index, step.buf.idx, step.buf.count, zq, z_out, tau=0.9, z_max=100.0)
+    torch.cuda.synchronize()
+    assert vk.vk_poll_status(ws) == vk.VK_OK
+    gz = zq.cpu().double().numpy()
+    zo = z_out.cpu().double().numpy()
+    a = oracle.scores(hi)
+    pres = oracle.build_index(hi, 64)[3]
+    rzq, _, n_ref = oracle.calib_zq(hi, 64, LAM, a, eta, pres, g["idx"], g["count"], sketch=(s16, p, rho))
+    hard = ~np.isnan(rzq)
+    assert hard.sum() >= oracle.min_hard(0.9)
+    np.testing.assert_array_equal(np.isnan(gz), np.isnan(rzq))
+    np.testing.assert_allclose(gz[hard], rzq[hard], rtol=1e-3, atol=2e-3)
+    assert zo[2] == hard.sum()
+    assert zo[0] == pytest.approx(oracle.conformal_quantile(rzq[hard], 0.9, 100.0), abs=2e-3 + 1e-3 * zo[0])
+    assert zo[1] == pytest.approx(zo[0] / math.sqrt(512.0 - r_sk), rel=1e-6)
