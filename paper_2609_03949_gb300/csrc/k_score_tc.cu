@@ -148,7 +148,7 @@ __device__ __forceinline__ uint32_t range_mask(int r0, int lo, int hi) {
 // NHG x TM tensor-memory columns (all 512 columns), a ring of STAGES tiles (96 to 112 KB). Shared memory from a
 // 1024-aligned base: the ring, two query buffers of NHG x MH rows (one with a sketch, whose query parts take the
 // room), 128 B of staging per epilogue thread (modes 1, 2), barriers. SK: the content sketch width (mode 2), or 0.
-template <int MH, int NHG, int TM_, int G_, int WPQ_ = 1, int RW_ = 64, int SK_ = 0>
+template <int MH, int NHG, int TM_, int G_, int WPQ_ = 1, int RW_ = 64, int SK_ = 0, int MODE_ = 0>
 struct TcCfg {
   static constexpr int TM = TM_;
   static constexpr int G = G_;
@@ -180,8 +180,12 @@ struct TcCfg {
   static constexpr uint32_t a = 0;
   static constexpr uint32_t q = a + STAGES * TILE;
   static constexpr uint32_t stg = q + QB * qbuf;
-  static constexpr uint32_t bars = stg + STG;
-  static constexpr uint32_t total = bars + (2 * STAGES + 4 + 2 * NACC) * 8 + 1024;
+  // mode 2: a ring of the tiles' eta rows (TM fp32 each), filled by the producer and released by the epilogue; it
+  // holds the tiles that sit in the stage ring and in the accumulators at once
+  static constexpr int E = MODE_ == 2 ? STAGES + NACC : 0;
+  static constexpr uint32_t eta = stg + STG;
+  static constexpr uint32_t bars = eta + E * TM * 4;
+  static constexpr uint32_t total = bars + (2 * STAGES + 4 + 2 * NACC + 2 * E) * 8 + 1024;
   static_assert(G <= NACC, "every epilogue group needs an accumulator of its own");
   static_assert(NC % WPQ == 0 && STAGES >= 4, "configuration");
   static_assert(TILE % 1024 == 0 && qbuf % 1024 == 0 && (SK == 0 || SK == 16 || SK == 32 || SK == 64), "alignment");
@@ -189,11 +193,11 @@ struct TcCfg {
 };
 
 template <int MH, int NHG, int MODE, int TM_, int G_, int WPQ_, int RW_, int SK_>
-__global__ void __launch_bounds__(TcCfg<MH, NHG, TM_, G_, WPQ_, RW_, SK_>::THREADS, 1)
+__global__ void __launch_bounds__(TcCfg<MH, NHG, TM_, G_, WPQ_, RW_, SK_, MODE>::THREADS, 1)
     k_score_tc(const __grid_constant__ CUtensorMap kmap, const __grid_constant__ CUtensorMap qmap,
                const __grid_constant__ CUtensorMap smap, const __grid_constant__ CUtensorMap sqmap,
-               const ScoreTcArgs args) {
-  using L = TcCfg<MH, NHG, TM_, G_, WPQ_, RW_, SK_>;
+               const __grid_constant__ CUtensorMap emap, const ScoreTcArgs args) {
+  using L = TcCfg<MH, NHG, TM_, G_, WPQ_, RW_, SK_, MODE>;
   static_assert(SK_ == 0 || MODE == 2, "the sketch belongs to the trigger");
   constexpr int G = L::G, TC_M = L::TM, TC_STAGES = L::STAGES, NACC = L::NACC;
   constexpr uint32_t TC_TILE_BYTES = L::TILE;
@@ -210,6 +214,10 @@ __global__ void __launch_bounds__(TcCfg<MH, NHG, TM_, G_, WPQ_, RW_, SK_>::THREA
   uint64_t* q_empty = q_full + 2;                        // [2]
   uint64_t* d_full = q_empty + 2;                        // [NACC]
   uint64_t* d_empty = d_full + NACC;                     // [NACC]
+  uint64_t* e_full = d_empty + NACC;                     // [E] mode 2: a tile's eta rows landed
+  uint64_t* e_empty = e_full + L::E;                     // [E] the epilogue is done with them
+  float* eta_s = reinterpret_cast<float*>(smem + L::eta);
+  const bool eta_tma = MODE == 2 && args.eta_tma;       // else the epilogue reads eta from global memory
   __shared__ uint32_t tmem_base;
   __shared__ int abort_flag;
   __shared__ int skip_stage[TC_STAGES];                  // mode 2 page skip: the ring stage's tile was not loaded
@@ -231,6 +239,7 @@ __global__ void __launch_bounds__(TcCfg<MH, NHG, TM_, G_, WPQ_, RW_, SK_>::THREA
     for (int s = 0; s < TC_STAGES; ++s) { mbar_init(&a_full[s], 1); mbar_init(&a_empty[s], 1); }
     for (int i = 0; i < 2; ++i) { mbar_init(&q_full[i], 1); mbar_init(&q_empty[i], 1); }
     for (int i = 0; i < NACC; ++i) { mbar_init(&d_full[i], 1); mbar_init(&d_empty[i], 4 * L::WPQ); }
+    for (int i = 0; i < L::E; ++i) { mbar_init(&e_full[i], 1); mbar_init(&e_empty[i], 4 * L::WPQ); }
     mbar_fence_init();
   }
   if (warp == 1) tmem_alloc(&tmem_base, 512);
@@ -296,6 +305,16 @@ __global__ void __launch_bounds__(TcCfg<MH, NHG, TM_, G_, WPQ_, RW_, SK_>::THREA
             mbar_arrive_expect_tx(&a_full[s], TC_TILE_BYTES);
             tma_load_3d(sa + s * TC_TILE_BYTES, &kmap, 0, row0, b, &a_full[s]);
           }
+          // the tile's eta rows (nothing to load for a skipped tile: its epilogue reads none)
+          const int e = i % L::E, euse = i / L::E;
+          if (euse > 0 && !mbar_wait(&e_empty[e], (euse - 1) & 1, &abort_flag)) {
+            lok = false;
+          } else if (eta_tma && !skip) {
+            mbar_arrive_expect_tx(&e_full[e], (uint32_t)TC_M * 4u);
+            tma_load_2d(eta_s + e * TC_M, &emap, row0, b, &e_full[e]);
+          } else {
+            mbar_arrive(&e_full[e]);
+          }
         }
       }
       ok = __shfl_sync(0xffffffffu, lok, 0);
@@ -326,6 +345,17 @@ __global__ void __launch_bounds__(TcCfg<MH, NHG, TM_, G_, WPQ_, RW_, SK_>::THREA
         mbar_arrive_expect_tx(&a_full[s], TC_TILE_BYTES);
         tma_load_3d(sa + s * TC_TILE_BYTES, &kmap, 0, row0, b, &a_full[s]);
         if constexpr (L::SK > 0) tma_load_3d(sa + s * TC_TILE_BYTES + L::KTILE, &smap, 0, row0, b, &a_full[s]);
+        if constexpr (MODE == 2) {
+          // the tile's eta rows, into a ring that the epilogue releases
+          const int e = i % L::E, euse = i / L::E;
+          if (euse > 0 && !mbar_wait(&e_empty[e], (euse - 1) & 1, &abort_flag)) { abort_flag = 1; break; }
+          if (eta_tma) {
+            mbar_arrive_expect_tx(&e_full[e], (uint32_t)TC_M * 4u);
+            tma_load_2d(eta_s + e * TC_M, &emap, row0, b, &e_full[e]);
+          } else {
+            mbar_arrive(&e_full[e]);
+          }
+        }
       }
     }
   } else if (warp == 1) {
@@ -412,10 +442,13 @@ __global__ void __launch_bounds__(TcCfg<MH, NHG, TM_, G_, WPQ_, RW_, SK_>::THREA
         prev_b = b;
       }
       const int ds = i % NACC, duse = i / NACC;
-      if (!mbar_wait(&d_full[ds], duse & 1, &abort_flag)) {
+      if (!mbar_wait(&d_full[ds], duse & 1, &abort_flag) ||
+          (MODE == 2 && !mbar_wait(&e_full[i % L::E], (i / L::E) & 1, &abort_flag))) {
         if (lane == 0) { raise_status(args.status, VK_ERR_TIMEOUT); abort_flag = 1; }
         break;
       }
+      // mode 2: the tile's eta rows in shared memory (zero past the last row), or in global memory
+      const float* eta_tile = eta_tma ? eta_s + (i % L::E) * TC_M : nullptr;
       tmem_fence_after();
 #pragma unroll
       for (int hg = 0; hg < NHG; ++hg) {
@@ -486,13 +519,23 @@ __global__ void __launch_bounds__(TcCfg<MH, NHG, TM_, G_, WPQ_, RW_, SK_>::THREA
               const uint32_t sel = word_ok ? args.selbm[bh * args.nw + word] : 0xffffffffu;
               const float pr = rc < args.n_rows ? args.page_res[(int64_t)b * args.n_pages + rc / PAGE] : 0.f;
               const float add = p1[hg] * pr;
-              const float* eta = args.eta + (int64_t)b * args.N + rc;
+              if (eta_tile) {                          // staged in shared memory by the producer
+                const float* etl = eta_tile + (rc - row0);
 #pragma unroll
-              for (int k = 0; k < 32; ++k) {
-                const float e = rc + k < args.n_rows ? eta[k] : 0.f;
-                const float T = args.lam * (v[k] + add + p2[hg] * e);
-                v[k] = T;
-                m |= (T > th[hg] ? 1u : 0u) << k;
+                for (int k = 0; k < 32; ++k) {
+                  const float T = args.lam * (v[k] + add + p2[hg] * etl[k]);
+                  v[k] = T;
+                  m |= (T > th[hg] ? 1u : 0u) << k;
+                }
+              } else {
+                const float* eta = args.eta + (int64_t)b * args.N + rc;
+#pragma unroll
+                for (int k = 0; k < 32; ++k) {
+                  const float e = rc + k < args.n_rows ? eta[k] : 0.f;
+                  const float T = args.lam * (v[k] + add + p2[hg] * e);
+                  v[k] = T;
+                  m |= (T > th[hg] ? 1u : 0u) << k;
+                }
               }
               m &= range_mask(rc, args.arch_lo, min(args.arch_hi, args.n_rows)) & ~sel;
             }
@@ -526,10 +569,15 @@ __global__ void __launch_bounds__(TcCfg<MH, NHG, TM_, G_, WPQ_, RW_, SK_>::THREA
               const float pr = args.page_res[(int64_t)b * args.n_pages + rc / PAGE];
               const float add = p1[hg] * pr;
               const float* eta = args.eta + (int64_t)b * args.N + rc;
+              if (eta_tile) {
 #pragma unroll
-              for (int k = 0; k < 32; ++k) {
-                const float e = rc + k < args.n_rows ? eta[k] : 0.f;
-                v[k] = args.lam * (v[k] + add + p2[hg] * e);
+                for (int k = 0; k < 32; ++k) v[k] = args.lam * (v[k] + add + p2[hg] * eta_tile[rc - row0 + k]);
+              } else {
+#pragma unroll
+                for (int k = 0; k < 32; ++k) {
+                  const float e = rc + k < args.n_rows ? eta[k] : 0.f;
+                  v[k] = args.lam * (v[k] + add + p2[hg] * e);
+                }
               }
             }
             uint32_t m = msk[j];
@@ -551,7 +599,10 @@ __global__ void __launch_bounds__(TcCfg<MH, NHG, TM_, G_, WPQ_, RW_, SK_>::THREA
       }
       tmem_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive(&d_empty[ds]);
+      if (lane == 0) {
+        mbar_arrive(&d_empty[ds]);
+        if (MODE == 2) mbar_arrive(&e_empty[i % L::E]);
+      }
     }
   }
 
@@ -595,9 +646,9 @@ static CUtensorMapSwizzle swizzle_for(int row_bytes) {
 template <int MH, int NHG, int MODE, int TM, int G, int WPQ, int RW, int SK = 0>
 static cudaError_t launch_cfg(const vk_view& v, const void* keys, int64_t key_ld, int64_t key_bstride,
                               const void* qsrc, int row_stride, int n_rows, ScoreTcArgs args, cudaStream_t st) {
-  using L = TcCfg<MH, NHG, TM, G, WPQ, RW, SK>;
+  using L = TcCfg<MH, NHG, TM, G, WPQ, RW, SK, MODE>;
   auto encode = encode_fn();
-  CUtensorMap kmap, qmap, smap, sqmap;
+  CUtensorMap kmap, qmap, smap, sqmap, emap;
   cuuint64_t kdims[3] = {(cuuint64_t)RW, (cuuint64_t)n_rows, (cuuint64_t)v.B};
   cuuint64_t kstr[2] = {(cuuint64_t)(key_ld * row_stride * 2), (cuuint64_t)(key_bstride * 2)};
   cuuint32_t kbox[3] = {(cuuint32_t)RW, (cuuint32_t)TM, 1};
@@ -618,6 +669,22 @@ static cudaError_t launch_cfg(const vk_view& v, const void* keys, int64_t key_ld
     return cudaErrorInvalidValue;
   smap = kmap;
   sqmap = qmap;
+  emap = kmap;
+  args.eta_tma = 0;
+  if constexpr (MODE == 2) {
+    // eta [B][N] fp32 as a 2D map, TM-row boxes (zero past N); its row stride must be a multiple of 16 bytes
+    if (row_stride == 1 && v.N % 4 == 0 && (reinterpret_cast<uintptr_t>(args.eta) & 15u) == 0) {
+      cuuint64_t edims[2] = {(cuuint64_t)v.N, (cuuint64_t)v.B};
+      cuuint64_t estr[1] = {(cuuint64_t)v.N * 4};
+      cuuint32_t ebox[2] = {(cuuint32_t)TM, 1};
+      cuuint32_t ees[2] = {1, 1};
+      if (encode(&emap, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2, const_cast<float*>(args.eta), edims, estr, ebox, ees,
+                 CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                 CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+        return cudaErrorInvalidValue;
+      args.eta_tma = 1;
+    }
+  }
   if constexpr (SK > 0) {
     // sketch rows [B][N][SK] (all N rows: the trigger scans with row stride 1) and the query parts [B][2][H][SK]
     if (row_stride != 1 || !args.sketch || !args.sketch_q) return cudaErrorInvalidValue;
@@ -649,7 +716,7 @@ static cudaError_t launch_cfg(const vk_view& v, const void* keys, int64_t key_ld
   cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)L::total);
   if (e != cudaSuccess) return e;
   if (grid > 0) {
-    kernel<<<grid, L::THREADS, L::total, st>>>(kmap, qmap, smap, sqmap, args);
+    kernel<<<grid, L::THREADS, L::total, st>>>(kmap, qmap, smap, sqmap, emap, args);
     count_launches(1);
   }
   return cudaGetLastError();

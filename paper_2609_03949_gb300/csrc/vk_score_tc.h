@@ -37,6 +37,8 @@ struct ScoreTcArgs {
   // high and low parts of p = V^T Qc, [B][2][H][r_sk]; qcn then holds the sketch residual norms of the queries
   int r_sk;
   const void *sketch, *sketch_q;
+  // mode 2, set by the launcher: the producer stages each tile's eta rows in shared memory by TMA (N % 4 == 0)
+  int eta_tma;
   int* status;
 };
 
