@@ -197,7 +197,7 @@ namespace {
 // room for twice that (+2048) before the exact fallback takes over.
 void fused_params(int64_t N, int64_t lo, int64_t hi, int64_t k, VkLayout* L) {
   const int64_t A = std::max<int64_t>(0, hi - lo);
-  L->ss = A >= 32768 ? 16 : std::max<int64_t>(1, A / 2048);
+  L->ss = A >= 49152 ? 32 : A >= 32768 ? 16 : std::max<int64_t>(1, A / 2048);
   L->soff = L->ss / 2;
   L->ns = N > L->soff ? (N - L->soff + L->ss - 1) / L->ss : 0;
   L->sld = (L->ns + 7) / 8 * 8;            // sample rows start on 16-byte boundaries
