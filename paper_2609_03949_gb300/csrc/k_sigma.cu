@@ -14,8 +14,11 @@
 //            again (phase 1 read it just before, so it comes from L2) into a ring of its own, and the epilogue (one
 //            thread per row) takes the row's low part from tensor memory and the row from shared memory, and
 //            writes sigma.
-// Roles: warp 0 TMA producer, warp 1 MMA issuer, warps 2..5 epilogue (one per tensor-memory lane quarter).
-// Phi is built in the workspace in bf16 twice: Phi^T [mp][T] and Phi [T][mp] (mp = 64 for kappa <= 32, else 128).
+// Roles: warp 0 TMA producer, warp 1 MMA issuer, warps 2..9 epilogue in two groups of four (one warp per
+// tensor-memory lane quarter each): group 0 writes C and takes the even phase 2 chunks, group 1 the odd ones.
+// Phi is built in the workspace in bf16 twice: Phi^T [mp][T] and Phi [T][mp] (mp = 32 for kappa <= 16, 64 for
+// kappa <= 32, else 128). At mp = 32 the phase 2 operands (the Phi chunk and C) have 64-byte rows and the 64-byte
+// swizzle, and the narrower stages let the ring hold six.
 // Rows past the last closed block (the open tail) get sigma = -1. Every wait is bounded.
 #include <cuda.h>
 #include <cudaTypedefs.h>
@@ -30,15 +33,16 @@ namespace vk {
 namespace {
 
 constexpr int SG_CH = 128;                 // rows per chunk
-constexpr int SG_THREADS = 6 * 32;
+constexpr int SG_THREADS = 10 * 32;
 constexpr uint32_t SG_RBYTES = SG_CH * 128;  // one chunk of R: 128 rows x 64 bf16
 
 template <int MP>
 struct SgCfg {
   static constexpr uint32_t PHT = 2 * MP * 128;          // Phi^T chunk: two 64-row K blocks of MP x 128 B
-  static constexpr uint32_t STAGE = SG_RBYTES + PHT;     // phase 1 stage (phase 2 uses the first MP / 64 x 16 KB)
-  static constexpr int STAGES = MP == 64 ? 4 : 3;
-  static constexpr int R2 = MP == 64 ? 4 : 3;            // phase 2 ring of R chunks for the epilogue
+  static constexpr uint32_t STAGE = SG_RBYTES + PHT;     // phase 1 stage (phase 2 uses its first 128 x MP x 2 B)
+  static constexpr int STAGES = MP == 32 ? 6 : MP == 64 ? 4 : 3;
+  static constexpr int R2 = MP == 128 ? 3 : 4;           // phase 2 ring of R chunks for the epilogue
+  static constexpr uint32_t ROW2 = MP == 32 ? 64 : 128;  // phase 2 operand row bytes (Phi chunk and C)
   static constexpr int NL = 4;                           // tensor-memory buffers of the phase 2 product
   static constexpr uint32_t cbuf = STAGES * STAGE;       // C as the phase 2 B operand: MP / 64 blocks of 64 x 128 B
   static constexpr uint32_t r2 = cbuf + 64 * MP * 2;
@@ -66,6 +70,16 @@ __device__ __forceinline__ void sg_tma_2d(void* dst, const CUtensorMap* map, int
 __device__ __forceinline__ uint64_t sg_desc(uint32_t saddr) {
   return (uint64_t)((saddr >> 4) & 0x3FFFu) | ((uint64_t)1u << 16) | ((uint64_t)(1024u >> 4) << 32) |
          ((uint64_t)1u << 46) | ((uint64_t)2u << 61);
+}
+// K-major operand with 64-byte rows, 64-byte swizzle: 8-row groups 512 B apart.
+__device__ __forceinline__ uint64_t sg_desc64(uint32_t saddr) {
+  return (uint64_t)((saddr >> 4) & 0x3FFFu) | ((uint64_t)1u << 16) | ((uint64_t)(512u >> 4) << 32) |
+         ((uint64_t)1u << 46) | ((uint64_t)4u << 61);
+}
+// The phase 2 descriptor for the operand width of MP.
+template <int MP>
+__device__ __forceinline__ uint64_t sg_desc2(uint32_t saddr) {
+  return MP == 32 ? sg_desc64(saddr) : sg_desc(saddr);
 }
 __device__ __forceinline__ void sg_mma(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc, uint32_t idesc, uint32_t acc) {
   asm volatile(
@@ -183,7 +197,7 @@ __global__ void __launch_bounds__(SG_THREADS, 1) k_sigma(const __grid_constant__
               sg_tma_2d(st + SG_RBYTES + MP * 128, &ptmap, u0 + 64, 0, &full[s]);
             } else {
               mbar_arrive_expect_tx(&full[s], (uint32_t)MP * 256u);
-              for (int kb = 0; kb < MP / 64; ++kb) sg_tma_2d(st + kb * 16384, &pmap, 64 * kb, u0, &full[s]);
+              for (int kb = 0; kb < (MP + 63) / 64; ++kb) sg_tma_2d(st + kb * 16384, &pmap, 64 * kb, u0, &full[s]);
               const int s2 = n2 % L::R2, use2 = n2 / L::R2;
               if (use2 > 0 && !mbar_wait(&r_empty[s2], (use2 - 1) & 1, &abort_flag)) { ok = false; ++n; break; }
               mbar_arrive_expect_tx(&r_full[s2], SG_RBYTES);
@@ -237,8 +251,8 @@ __global__ void __launch_bounds__(SG_THREADS, 1) k_sigma(const __grid_constant__
           const uint32_t st = smem_addr(smem + s * L::STAGE);
 #pragma unroll
           for (int j = 0; j < MP / 16; ++j) {
-            const uint64_t ad = sg_desc(st + (j >> 2) * 16384 + (j & 3) * 32);
-            const uint64_t bd = sg_desc(cba + (j >> 2) * 8192 + (j & 3) * 32);
+            const uint64_t ad = sg_desc2<MP>(st + (j >> 2) * 16384 + (j & 3) * 32);
+            const uint64_t bd = sg_desc2<MP>(cba + (j >> 2) * 8192 + (j & 3) * 32);
             sg_mma(tmem + L_COL + 64 * lb, ad, bd, idesc2, j > 0 ? 1u : 0u);
           }
           sg_commit(&empty[s]);
@@ -256,41 +270,49 @@ __global__ void __launch_bounds__(SG_THREADS, 1) k_sigma(const __grid_constant__
   } else {
     // ------------------------------------------------------------------ epilogue
     const int q = warp & 3;                               // tensor-memory lane quarter
+    const int eg = (warp - 2) >> 2;                       // epilogue group: 0 writes C, the groups split the chunks
     const uint32_t lq = (uint32_t)(32 * q) << 16;
-    int nit = 0, nl = 0;
+    int nit = 0;
     bool ok = true;
     for (long long it = i0; it < i1 && ok; ++it, ++nit) {
       const int b = (int)(it / args.nb), blk = (int)(it - (long long)b * args.nb);
-      if (!warp_wait_sg(c_full, nit & 1, &abort_flag, lane)) { ok = false; break; }
-      tmem_fence_after();
-      {
-        // C^T row d = 16 q + (lane % 16) (M = 64 layout), bins 32 (lane / 16) + 64 kb .. + 31 -> bf16 into the B
-        // operand of phase 2: row d of K block kb, 16-byte chunks 4 (lane / 16) .. + 3, 128-byte swizzle
-        const int d = 16 * q + (lane & 15), half = lane >> 4;
+      if (eg == 0) {
+        if (!warp_wait_sg(c_full, nit & 1, &abort_flag, lane)) { ok = false; break; }
+        tmem_fence_after();
+        {
+          // C^T row d = 16 q + (lane % 16) (M = 64 layout), bins 32 (lane / 16) + 64 kb .. + 31 -> bf16 into the B
+          // operand of phase 2: row d of K block kb, 16-byte chunks 4 (lane / 16) .. + 3, 128-byte swizzle (at MP = 32:
+          // 64-byte rows of the 32 bins, 64-byte swizzle, written by the lanes of the first half)
+          const int d = 16 * q + (lane & 15), half = lane >> 4;
 #pragma unroll
-        for (int kb = 0; kb < MP / 64; ++kb) {
-          float v[32];
-          sg_ld16x2(tmem + lq + C_COL + 64 * kb, v);
-          tmem_wait_ld();
-          unsigned char* row = cb + kb * 8192 + d * 128;
+          for (int kb = 0; kb < (MP + 63) / 64; ++kb) {
+            float v[32];
+            sg_ld16x2(tmem + lq + C_COL + 64 * kb, v);
+            tmem_wait_ld();
+            if (MP == 32 && half) continue;               // columns past the 32 bins
+            unsigned char* row = cb + kb * 8192 + d * L::ROW2;
 #pragma unroll
-          for (int k = 0; k < 4; ++k) {
-            uint32_t w[4];
+            for (int k = 0; k < 4; ++k) {
+              uint32_t w[4];
 #pragma unroll
-            for (int e = 0; e < 4; ++e) {
-              const __nv_bfloat162 pb = __floats2bfloat162_rn(v[8 * k + 2 * e], v[8 * k + 2 * e + 1]);
-              w[e] = *reinterpret_cast<const uint32_t*>(&pb);
+              for (int e = 0; e < 4; ++e) {
+                const __nv_bfloat162 pb = __floats2bfloat162_rn(v[8 * k + 2 * e], v[8 * k + 2 * e + 1]);
+                w[e] = *reinterpret_cast<const uint32_t*>(&pb);
+              }
+              const int chunk = MP == 32 ? (k ^ ((d >> 1) & 3)) : ((4 * half + k) ^ (d & 7));
+              *reinterpret_cast<uint4*>(row + chunk * 16) = make_uint4(w[0], w[1], w[2], w[3]);
             }
-            *reinterpret_cast<uint4*>(row + (((4 * half + k) ^ (d & 7)) * 16)) = make_uint4(w[0], w[1], w[2], w[3]);
           }
         }
+        fence_async_smem_sg();
+        tmem_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(c_ready);
       }
-      fence_async_smem_sg();
-      tmem_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(c_ready);
-      // phase 2: one row per thread; the row from the R ring (128-byte swizzle: chunk k of row x sits at k ^ (x & 7))
-      for (int c = 0; c < nchunk; ++c, ++nl) {
+      // phase 2: one row per thread; the row from the R ring (128-byte swizzle: chunk k of row x sits at k ^ (x & 7));
+      // chunk c of this item is the (nit * nchunk + c)-th phase 2 chunk of the CTA, taken by group c % 2
+      for (int c = eg; c < nchunk; c += 2) {
+        const int nl = nit * nchunk + c;
         const int lb = nl % L::NL, luse = nl / L::NL;
         const int s2 = nl % L::R2, use2 = nl / L::R2;
         if (!warp_wait_sg(&l_full[lb], luse & 1, &abort_flag, lane) ||
@@ -424,10 +446,10 @@ cudaError_t launch_sigma_mp(const vk_view& v, int T, int kappa, float* sigma, vo
   {
     cuuint64_t dims[2] = {(cuuint64_t)MP, (cuuint64_t)T};
     cuuint64_t str[1] = {(cuuint64_t)MP * 2};
-    cuuint32_t box[2] = {64, (cuuint32_t)SG_CH};
+    cuuint32_t box[2] = {(cuuint32_t)(MP < 64 ? MP : 64), (cuuint32_t)SG_CH};
     cuuint32_t es[2] = {1, 1};
     if (encode(&pmap, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, phi, dims, str, box, es, CU_TENSOR_MAP_INTERLEAVE_NONE,
-               CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+               MP == 32 ? CU_TENSOR_MAP_SWIZZLE_64B : CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
       return cudaErrorInvalidValue;
   }
@@ -453,7 +475,7 @@ cudaError_t launch_sigma_mp(const vk_view& v, int T, int kappa, float* sigma, vo
 
 }  // namespace
 
-int sigma_basis_cols(int kappa) { return kappa <= 32 ? 64 : 128; }
+int sigma_basis_cols(int kappa) { return kappa <= 16 ? 32 : kappa <= 32 ? 64 : 128; }
 
 size_t sigma_workspace_bytes(int T, int kappa) {
   return 256 + (size_t)2 * 2 * sigma_basis_cols(kappa) * (size_t)T;   // status word, Phi^T and Phi (bf16)
@@ -462,8 +484,10 @@ size_t sigma_workspace_bytes(int T, int kappa) {
 cudaError_t launch_sigma(const vk_view& v, int T, int kappa, float* sigma, void* ws, cudaStream_t st) {
   int* status = static_cast<int*>(ws);
   void* tables = static_cast<char*>(ws) + 256;
-  return sigma_basis_cols(kappa) == 64 ? launch_sigma_mp<64>(v, T, kappa, sigma, tables, status, st)
-                                       : launch_sigma_mp<128>(v, T, kappa, sigma, tables, status, st);
+  const int mp = sigma_basis_cols(kappa);
+  return mp == 32   ? launch_sigma_mp<32>(v, T, kappa, sigma, tables, status, st)
+         : mp == 64 ? launch_sigma_mp<64>(v, T, kappa, sigma, tables, status, st)
+                    : launch_sigma_mp<128>(v, T, kappa, sigma, tables, status, st);
 }
 
 }  // namespace vk
