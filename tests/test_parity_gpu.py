@@ -421,3 +421,34 @@ def test_fired_passes_agree(z, top_j):
     np.testing.assert_array_equal(ga["count"], gb["count"])
     np.testing.assert_allclose(ga["out"], gb["out"], rtol=1e-4, atol=1e-5)
     np.testing.assert_allclose(ga["lse"], gb["lse"], rtol=1e-5, atol=1e-5)
+
+
+@pytest.mark.parametrize("N,r,sketch", [(5003, 64, 0), (4097, 16, 0), (6001, 64, 32)])
+def test_two_tier_ragged_context(N, r, sketch):
+    """A context that is not a multiple of 4 rows: the trigger scan reads eta from global memory instead of staging
+    it by TMA (its row stride is no multiple of 16 bytes), and the last tile is ragged."""
+    H, W = 64, 128
+    if sketch:
+        wl = datagen.make_workload(1, H, N, seed=N + r, n_planted=8, planted_hi=N - W, query_rank=8)
+        hi = oracle.HostInputs(wl)
+        V, _ = oracle.sketch_basis(datagen.prefix_queries(wl, 150).double().numpy(), sketch)
+        _, s16, eta = oracle.build_sketch(hi, V)
+        p, rho = oracle.sketch_query(hi, V)
+        g = GpuStep(wl, rho=1 / 32, window=W, trigger=1, z_eff=0.2, sketch=(s16, V, eta)).run()
+        a = oracle.scores(hi)
+        k = oracle.keep_count(N, 1 / 32, W)
+        nS = k + W
+        check_selection(a, g["idx"], g["count"], k, W, 0)
+        _, _, smax = oracle.attention(hi, LAM, g["idx"][..., :nS], np.full_like(g["count"], nS))
+        pres = oracle.build_index(hi, 64)[3]
+        fidx, fcnt = oracle.trigger(hi, 64, LAM, 0.2, 0, a, eta, pres, g["idx"], np.full_like(g["count"], nS), smax, W,
+                                    sketch=(s16, p, rho))
+        for h in range(H):
+            got = set(g["idx"][0, h, nS:g["count"][0, h]].tolist())
+            ref = set(fidx[0, h, :fcnt[0, h]].tolist())
+            assert len(got ^ ref) <= 2, (h, sorted(got ^ ref)[:5])
+        check_outputs(hi, LAM, g)
+        return
+    wl = datagen.make_workload(1, H, N, seed=N + r, n_planted=8, planted_hi=N - W, device="cuda")
+    res = run_case(wl, rho=1 / 32, r=r, window=W, trigger=1, z_eff=0.3)
+    assert res["fired"] >= 0
