@@ -1,9 +1,11 @@
 // k_attn_tc.cu -- gather + absorbed-MLA attention for bf16 caches, both contractions on the tensor cores.
 //
 // Persistent: one CTA per SM. The work is B * n_hg segments (sequence b, group of <= 64 heads), each walked in tiles
-// of 64 rows; the segments' tiles, flattened segment-major, are cut into one equal contiguous range per CTA, so a
-// CTA covers the end of one segment, whole segments and the start of another. A tile that no head of its group
-// selects is neither loaded nor computed. Per tile:
+// of 64 rows. The B * T (sequence, row tile) positions are cut into equal contiguous ranges, and each range goes to
+// n_hg neighbouring CTAs, one per head group, so a CTA covers the end of one sequence, whole sequences and the
+// start of another for its group. The CTAs of a range read the same tiles at the same pace, so with two or more
+// head groups a tile comes from HBM about once and from L2 for the other groups. A tile that no head of the CTA's
+// group selects is neither loaded nor computed. Per tile:
 //   warp 0 (producer)  stages the heads' two 32-bit selection words of the tile, then TMA-loads its 64 rows x 576
 //                      columns (128-byte swizzle, one 8 KB block per 64 columns) as five groups -- the RoPE block
 //                      first, then four pairs of latent blocks, each as soon as the tile before it in that slot has
@@ -199,20 +201,19 @@ static __device__ __noinline__ bool attn_handle_request(volatile int* rq_tile, u
   return true;
 }
 
-// Position of a flattened tile: its row tile kt within the segment and the segment's (sequence b, head group hg).
-// Stepped without divisions (the per-tile bookkeeping sits on the issuing threads' critical path).
+// Position of a CTA's tile: the row tile kt of sequence b; the head group hg is the CTA's own. Stepped without
+// divisions (the per-tile bookkeeping sits on the issuing threads' critical path).
 struct TilePos {
   int kt, hg, b;
-  __device__ __forceinline__ void init(long long t, int T, int n_hg) {
-    const long long seg = t / T;
-    kt = (int)(t - seg * T);
-    b = (int)(seg / n_hg);
-    hg = (int)(seg - (long long)b * n_hg);
+  __device__ __forceinline__ void init(long long pos, int T, int group) {
+    b = (int)(pos / T);
+    kt = (int)(pos - (long long)b * T);
+    hg = group;
   }
-  __device__ __forceinline__ void next(int T, int n_hg) {
+  __device__ __forceinline__ void next(int T) {
     if (++kt == T) {
       kt = 0;
-      if (++hg == n_hg) { hg = 0; ++b; }
+      ++b;
     }
   }
 };
@@ -261,12 +262,16 @@ __global__ void __launch_bounds__(AT_THREADS, 1) k_attn_tc(const __grid_constant
 
   const AttnGeom& geo = args.g;
   const int H = args.H, T = geo.T;
-  const long long t0 = geo.total * blockIdx.x / gridDim.x, t1 = geo.total * (blockIdx.x + 1) / gridDim.x;
+  // this CTA: head group `grp` of position range `rng` (the groups of one range are neighbouring CTAs)
+  const int nranges = gridDim.x / geo.n_hg;
+  const int rng = blockIdx.x / geo.n_hg, grp = blockIdx.x - rng * geo.n_hg;
+  const long long npos = geo.total / geo.n_hg;
+  const long long t0 = npos * rng / nranges, t1 = npos * (rng + 1) / nranges;
   const int ntile = (int)(t1 - t0);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   // a segment's first tile, or the first of this CTA's range, starts a new segment for every role
   TilePos tp;
-  tp.init(t0, T, geo.n_hg);
+  tp.init(t0, T, grp);
 
   if (threadIdx.x == 0) {
     *abort_flag = 0;
@@ -331,12 +336,12 @@ __global__ void __launch_bounds__(AT_THREADS, 1) k_attn_tc(const __grid_constant
     };
     uint4 cur, nxt;
     fetch(0, cur);
-    fp.next(T, geo.n_hg);
+    fp.next(T);
     int u = 0;                                         // tiles loaded so far
     bool ok = true;
-    for (int i = 0; i < ntile; ++i, tp.next(T, geo.n_hg)) {
+    for (int i = 0; i < ntile; ++i, tp.next(T)) {
       fetch(i + 1, nxt);
-      fp.next(T, geo.n_hg);
+      fp.next(T);
       const int ws = i & 1;
       if (i >= 2 && !warp_wait_(&wfree[ws], ((i >> 1) - 1) & 1, abort_flag, lane)) { ok = false; break; }
       uint32_t* wd = words + ws * 128;
@@ -413,7 +418,7 @@ __global__ void __launch_bounds__(AT_THREADS, 1) k_attn_tc(const __grid_constant
       uint64_t* done_bar = &sdone[half];
       bool ok = true;
       int u = 0, nq = 0;
-      for (int i = 0; i < ntile; ++i, tp.next(T, geo.n_hg)) {
+      for (int i = 0; i < ntile; ++i, tp.next(T)) {
         if (!mbar_wait(&wfull[i & 1], (i >> 1) & 1, abort_flag)) { ok = false; break; }
         const uint32_t uni = unis[i & 1];
         mbar_arrive(&wfree[i & 1]);
@@ -470,7 +475,7 @@ __global__ void __launch_bounds__(AT_THREADS, 1) k_attn_tc(const __grid_constant
           (1u << 4) | (1u << 7) | (1u << 10) | (1u << 15) | ((uint32_t)(64 >> 3) << 17) | ((uint32_t)(128 >> 4) << 24);
       bool ok = true;
       int u = 0, useg = 0, nseg = 0, ncommit = 0, nreq = 0;
-      for (int i = 0; i < ntile; ++i, tp.next(T, geo.n_hg)) {
+      for (int i = 0; i < ntile; ++i, tp.next(T)) {
         if (!mbar_wait(&wfull[i & 1], (i >> 1) & 1, abort_flag)) { ok = false; break; }
         const uint32_t uni = unis[i & 1];
         mbar_arrive(&wfree[i & 1]);
@@ -572,7 +577,7 @@ __global__ void __launch_bounds__(AT_THREADS, 1) k_attn_tc(const __grid_constant
       lt = (lt + lparts[hl]) * ff;                                               // both warps' rows (rh = 0 uses it)
       tmem_fence_after();
       const int h0 = shg * 64, nh = min(64, H - h0);
-      const int slot = (int)blockIdx.x - attn_cta_of(geo, ((long long)sb * geo.n_hg + shg) * T);
+      const int slot = rng - attn_range_of(geo, ((long long)sb * geo.n_hg + shg) * T);
       const int64_t hbase = ((int64_t)sb * args.nslot + args.slot0 + slot) * H + h0;
       constexpr float LN2 = 0.6931471805599453f;
       if (own && rh == 0 && hl < nh) {
@@ -606,7 +611,7 @@ __global__ void __launch_bounds__(AT_THREADS, 1) k_attn_tc(const __grid_constant
     };
     // one pass past the last tile closes the last segment: the epilogue has a single (inlined) call site, which
     // keeps the loop's code small (instruction fetch is shared with the issuing warps' loops)
-    for (int i = 0; i <= ntile; ++i, tp.next(T, geo.n_hg)) {
+    for (int i = 0; i <= ntile; ++i, tp.next(T)) {
       const int ws = i & 1;
       uint32_t uni = 0u, w = 0u;
       const bool fresh = i == ntile || i == 0 || tp.kt == 0;
@@ -772,8 +777,8 @@ cudaError_t launch_attn_tc(const vk_view& v, float lam, const uint32_t* bitmap, 
                            int slot0, int nslot, float* part_o, float* part_ml, uint32_t flags, int* status,
                            cudaStream_t st, int* part_arg, const int* skip) {
   if (!encode2()) return cudaErrorNotSupported;
-  if (g.G < 1 || g.G > g.total || g.T != (v.N + AT_T - 1) / AT_T || g.n_hg != (v.H + 63) / 64 ||
-      g.total != (long long)v.B * g.n_hg * g.T)
+  if (g.G < 1 || g.G > g.total || g.G % g.n_hg != 0 || g.T != (v.N + AT_T - 1) / AT_T ||
+      g.n_hg != (v.H + 63) / 64 || g.total != (long long)v.B * g.n_hg * g.T)
     return cudaErrorInvalidValue;
   CUtensorMap lmap, rmap, qlmap, qrmap;
   // cache rows: latent [B][N][512] and RoPE [B][N][64]; queries: [B*H][512] and [B*H][64]; 64-row boxes

@@ -176,7 +176,10 @@ AttnGeom attn_geom(const vk_view& v) {
   g.T = (v.N + 63) / 64;
   g.total = (long long)v.B * g.n_hg * g.T;
   if (attn_tc_supported(v)) {
-    g.G = (int)std::min<long long>(std::max<long long>(1, g.total / 4), sm_count());
+    // P ranges of at least 4 positions, n_hg CTAs each, at most one CTA per SM where the groups allow
+    const long long P = std::min<long long>(std::max<long long>(1, (long long)v.B * g.T / 4),
+                                            std::max(1, sm_count() / g.n_hg));
+    g.G = (int)(P * g.n_hg);
     g.nslot = 1;
     for (long long s = 0; s < (long long)v.B * g.n_hg; ++s) g.nslot = std::max(g.nslot, attn_nvalid(g, s));
   } else {

@@ -73,25 +73,30 @@ __device__ __forceinline__ int block_exclusive_scan(int v, int* scratch, int* to
 // is made of B * n_hg segments (sequence, head group of 64), each of T = ceil(N / 64) row tiles.
 //  * split layout (fp32 kernel, G = 0): every segment is cut into nsplit ranges of split_len positions, one CTA
 //    each, and all nsplit slots of every segment are written;
-//  * persistent layout (tensor-core kernel, G > 0): the segments' tiles are flattened segment-major and cut into
-//    G equal contiguous ranges, one CTA each; a segment owns one slot per CTA its tiles fall in, numbered from 0
-//    by CTA, so segment s has attn_nvalid(s) written slots.
+//  * persistent layout (tensor-core kernel, G > 0): the B * T (sequence, row tile) positions, sequence-major, are
+//    cut into P = G / n_hg equal contiguous ranges, and CTA p * n_hg + c takes head group c of range p. The n_hg
+//    CTAs of a range walk the same rows in step, so the second head group's reads of a tile come from L2. A
+//    segment (tiles t = s T .. s T + T - 1, s = b n_hg + hg) owns one slot per range its tiles fall in, numbered
+//    from 0 by range, so segment s has attn_nvalid(s) written slots.
 // nslot is the slot count of one tier (the largest attn_nvalid); the fired rows of the two-tier path use slots
 // nslot .. 2 nslot - 1 the same way.
 struct AttnGeom {
   int nslot;
   int nsplit, split_len;     // split layout
-  int G, T, n_hg;            // persistent layout
+  int G, T, n_hg;            // persistent layout: G a multiple of n_hg
   long long total;           // B * n_hg * T
 };
-// The CTA of the persistent layout whose range holds flattened tile t: ranges are [c total / G, (c+1) total / G).
-__host__ __device__ inline int attn_cta_of(const AttnGeom& g, long long t) {
-  return (int)(((t + 1) * (long long)g.G - 1) / g.total);
+// The range of the persistent layout that holds tile t of segment t / T: ranges are [p npos / P, (p+1) npos / P)
+// over the npos = B * T positions.
+__host__ __device__ inline int attn_range_of(const AttnGeom& g, long long t) {
+  const long long s = t / g.T, kt = t - s * g.T;
+  const long long pos = (s / g.n_hg) * g.T + kt, npos = g.total / g.n_hg;
+  return (int)(((pos + 1) * (long long)(g.G / g.n_hg) - 1) / npos);
 }
 // Written slots of segment s (per tier).
 __host__ __device__ inline int attn_nvalid(const AttnGeom& g, long long s) {
   if (g.G == 0) return g.nslot;
-  return attn_cta_of(g, (s + 1) * g.T - 1) - attn_cta_of(g, s * g.T) + 1;
+  return attn_range_of(g, (s + 1) * g.T - 1) - attn_range_of(g, s * g.T) + 1;
 }
 
 }  // namespace vk
