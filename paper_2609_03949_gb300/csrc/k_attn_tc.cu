@@ -11,10 +11,10 @@
 //                      first, then four pairs of latent blocks, each as soon as the tile before it in that slot has
 //                      released it -- into one of two tile slots; at a segment's first tile it loads the segment's
 //                      queries once the previous segment's S products are done with the query buffer;
-//   warps 1, 7 (S)     S = Q . X^T on tcgen05 (M = 64 heads, N = 64 rows, K = 576: 36 instructions) in two halves,
-//                      each issued by its own thread as one burst once its blocks have landed, into their own
-//                      accumulators (double-buffered); with M = 64 the logit of head 16 g + i and row j sits in TMEM
-//                      lane 32 g + i, column j, and the softmax adds the two halves;
+//   warps 1, 7 (S)     S = Q . X^T on tcgen05 (M = 64 heads, N = 64 rows, K = 576: 36 instructions) in two parts
+//                      (24 + 12 instructions), each issued by its own thread, one burst per load group as the group
+//                      lands, into their own accumulators (double-buffered); with M = 64 the logit of head 16 g + i
+//                      and row j sits in TMEM lane 32 g + i, column j, and the softmax adds the two parts;
 //   warp 6 (O^T)       once the softmax warps have written P^T, O^T += X_lat^T . P^T (M = 128 latent dims x 4
 //                      blocks, N = 64 heads, K = 64 rows: 16 instructions) into the O^T accumulator, which stays in
 //                      tensor memory for the whole segment. X_lat^T is read straight from the tile slot as an MN-major
@@ -59,8 +59,8 @@ constexpr uint32_t AT_TILE = 9 * AT_KBLK;              // 73,728: one tile slot,
 constexpr int AT_NG = 5;                               // load groups per tile: latent pairs 0..3, RoPE block 4
 constexpr float AT_TAU = 32.f;                         // log2 slack before a running max moves (P <= 2^32)
 constexpr uint32_t AT_TMEM_COLS = 512;
-constexpr uint32_t AT_S_COL = 0;                       // S (RoPE + latent 0..255) buffers: columns 0..63, 64..127
-constexpr uint32_t AT_SB_COL = 384;                    // S (latent 256..511) buffers: columns 384..447, 448..511
+constexpr uint32_t AT_S_COL = 0;                       // S (latent 0..383) buffers: columns 0..63, 64..127
+constexpr uint32_t AT_SB_COL = 384;                    // S (latent 384..511 + RoPE) buffers: columns 384..447, 448..511
 constexpr uint32_t AT_O_COL = 128;                     // O^T block j: columns 128 + 64 j .. + 63
 
 // Shared memory, from a 1024-byte aligned base. Barriers: xfull/xrel [2 slots][5 groups], sfull/sfree [2],
@@ -404,11 +404,11 @@ __global__ void __launch_bounds__(AT_THREADS, 1) k_attn_tc(const __grid_constant
     }
   } else if (warp == 1 || warp == AT_W_SB) {
     // ------------------------------------------------------------------ S issuers
-    // Two threads issue the two halves of the K = 576 contraction into their own accumulators (the softmax adds
-    // them): warp 1 latent dims 0..255 (16 instructions), warp 7 latent dims 256..511 and the RoPE block (20). The
+    // Two threads issue the two parts of the K = 576 contraction into their own accumulators (the softmax adds
+    // them): warp 1 latent dims 0..383 (24 instructions), warp 7 latent dims 384..511 and the RoPE block (12). The
     // groups land in the order the previous tile's O^T product releases them: latent pairs 0..3, then the RoPE
-    // block, which holds that tile's P^T until its O^T is done. (A 24/12 split, the short part after the last
-    // group to land, measured slower.)
+    // block, which holds that tile's P^T until its O^T is done. Each thread issues a group's instructions as soon
+    // as that group has landed, so after the last group lands only its four instructions remain.
     const int half = warp == 1 ? 0 : 1;
     if (lane == 0 && ntile > 0) {
       // S: M = 64 heads, N = 64 rows, A = Q and B = X, both K-major
@@ -431,30 +431,43 @@ __global__ void __launch_bounds__(AT_THREADS, 1) k_attn_tc(const __grid_constant
         const int s = u & 1, use = u >> 1;
         if (use > 0 && !mbar_wait(&sfree[s], (use - 1) & 1, abort_flag)) { ok = false; break; }
         const uint64_t xd = sdesc_(smem_addr(sx + s * AT_TILE), 16);
-        // this half's load groups first, then its instructions as one branch-free burst: control flow between
-        // tcgen05.mma issues costs the issuing thread far more than the instructions themselves
+        // one branch-free burst per load group: control flow between tcgen05.mma issues costs the issuing thread far
+        // more than the instructions themselves, so the only test between bursts is the next group's wait
         if (half == 0) {
-          ok = mbar_wait(&xfull[s * AT_NG + 0], use & 1, abort_flag) && mbar_wait(&xfull[s * AT_NG + 1], use & 1, abort_flag);
-          if (!ok) break;
-          // operands land by TMA and are observed through the mbarrier: no tensor-memory fence is needed
           const uint32_t d = tmem + AT_S_COL + 64 * s;
 #pragma unroll
-          for (int j = 0; j < 16; ++j) {
-            const uint64_t off = (uint64_t)(((j >> 2) * AT_KBLK + 32 * (j & 3)) >> 4);
-            mma_bf16_(d, qd + off, xd + off, idesc_s, j > 0 ? 1u : 0u);
+          for (int g = 0; g < 3; ++g) {
+            if (!mbar_wait(&xfull[s * AT_NG + g], use & 1, abort_flag)) { ok = false; break; }
+#pragma unroll
+            for (int jj = 0; jj < 8; ++jj) {
+              const int j = 8 * g + jj;
+              const uint64_t off = (uint64_t)(((j >> 2) * AT_KBLK + 32 * (j & 3)) >> 4);
+              mma_bf16_(d, qd + off, xd + off, idesc_s, j > 0 ? 1u : 0u);
+            }
           }
+          if (!ok) break;
           mma_commit_(&sfull[s]);
         } else {
-          ok = mbar_wait(&xfull[s * AT_NG + 2], use & 1, abort_flag) && mbar_wait(&xfull[s * AT_NG + 3], use & 1, abort_flag) &&
-               mbar_wait(&xfull[s * AT_NG + 4], use & 1, abort_flag);
-          if (!ok) break;
           const uint32_t d = tmem + AT_SB_COL + 64 * s;
 #pragma unroll
-          for (int j = 0; j < 20; ++j) {
-            const int kb = j < 16 ? 4 + (j >> 2) : 8;
-            const uint64_t off = (uint64_t)((kb * AT_KBLK + 32 * (j & 3)) >> 4);
-            mma_bf16_(d, qd + off, xd + off, idesc_s, j > 0 ? 1u : 0u);
+          for (int g = 3; g < 5; ++g) {
+            if (!mbar_wait(&xfull[s * AT_NG + g], use & 1, abort_flag)) { ok = false; break; }
+            if (g < 4) {
+#pragma unroll
+              for (int jj = 0; jj < 8; ++jj) {
+                const int j = 8 * (g - 3) + jj;
+                const uint64_t off = (uint64_t)(((6 + (j >> 2)) * AT_KBLK + 32 * (j & 3)) >> 4);
+                mma_bf16_(d, qd + off, xd + off, idesc_s, j > 0 ? 1u : 0u);
+              }
+            } else {
+#pragma unroll
+              for (int j = 0; j < 4; ++j) {
+                const uint64_t off = (uint64_t)((8 * AT_KBLK + 32 * j) >> 4);
+                mma_bf16_(d, qd + off, xd + off, idesc_s, 1u);
+              }
+            }
           }
+          if (!ok) break;
           mma_commit_(&sfull[s]);
         }
         ++u;
@@ -528,7 +541,7 @@ __global__ void __launch_bounds__(AT_THREADS, 1) k_attn_tc(const __grid_constant
     }
   } else {
     // ------------------------------------------------------------------ softmax
-    // Two warps per TMEM lane quarter. Head hl = 16 q + (lane % 16); one tcgen05.ld 16x32bx2 per S half gives lanes
+    // Two warps per TMEM lane quarter. Head hl = 16 q + (lane % 16); one tcgen05.ld 16x32bx2 per S part gives lanes
     // 0..15 the head's rows 0..31 and lanes 16..31 its rows 32..63, so both warps of a quarter see the whole tile and
     // take its max alone. Of its 32 rows a lane writes P for 16: rows 32 hh + 16 rh .. + 15 (rh = 0 for warps 2..5,
     // 1 for warps 8..11). The rh = 0 warps publish the rescale factors and serve rescales.
@@ -638,7 +651,7 @@ __global__ void __launch_bounds__(AT_THREADS, 1) k_attn_tc(const __grid_constant
       if (u >= 2 && !check(u - 2)) { ok = false; break; }
       if (!warp_wait_(&sfull[s], use & 1, abort_flag, lane)) { ok = false; break; }
       tmem_fence_after();
-      // this warp's 16 rows per lane (sv) and the other row half's (ov), both S halves added: each warp of a quarter
+      // this warp's 16 rows per lane (sv) and the other row half's (ov), both S parts added: each warp of a quarter
       // takes the whole tile's max itself, so both reach the same running max without an exchange
       float sv[32];
       {
