@@ -343,11 +343,12 @@ cudaError_t launch_select_dense(int B, int H, int N, const float* scores, const 
 constexpr int THETA_R = 16;
 __global__ void __launch_bounds__(CAND_THREADS) k_theta(int ns, int ld, int off, int stride, int lo, int hi, int j,
                                                         const __nv_bfloat16* __restrict__ sample,
-                                                        float* __restrict__ theta) {
+                                                        float* __restrict__ theta, int* __restrict__ zero_cnt) {
   extern __shared__ __align__(16) unsigned char smem[];
   __shared__ unsigned int hist[256];
   __shared__ uint32_t scratch[64];
   const int64_t bh = blockIdx.x;
+  if (zero_cnt && threadIdx.x == 0) zero_cnt[bh] = 0;  // the candidate pass that follows counts from zero
   const __nv_bfloat16* a = sample + bh * (int64_t)ld;
   // sampled positions off + stride * i inside [lo, hi) are a contiguous index range [i0, i1)
   const int i0 = lo > off ? (lo - off + stride - 1) / stride : 0;
@@ -399,13 +400,13 @@ __global__ void __launch_bounds__(CAND_THREADS) k_theta(int ns, int ld, int off,
 }
 
 cudaError_t launch_theta(int B, int H, int ns, int ld, int off, int stride, int lo, int hi, int j, const void* sample,
-                         float* theta, cudaStream_t st) {
+                         float* theta, cudaStream_t st, int* zero_cnt) {
   // shared memory only when the samples outgrow the registers (na <= ns)
   const size_t smem = ns > THETA_R * CAND_THREADS ? (size_t)ns * 4 : 0;
   cudaError_t e = cudaFuncSetAttribute(k_theta, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
   k_theta<<<B * H, CAND_THREADS, smem, st>>>(ns, ld, off, stride, lo, hi, j,
-                                             static_cast<const __nv_bfloat16*>(sample), theta);
+                                             static_cast<const __nv_bfloat16*>(sample), theta, zero_cnt);
   count_launches(1);
   return cudaGetLastError();
 }

@@ -464,7 +464,7 @@ int vk_decode_step(const vk_view* view, const vk_params* params, const vk_index*
     float* theta = at<float>(ws, L.off_theta);
     int* ccnt = at<int>(ws, L.off_ccnt);
     int2* cand = at<int2>(ws, L.off_cand);
-    VK_CUDA(cudaMemsetAsync(ccnt, 0, sizeof(int) * B * H, st), "candidate counts");
+    if (k == 0) VK_CUDA(cudaMemsetAsync(ccnt, 0, sizeof(int) * B * H, st), "candidate counts");
     if (k > 0) {
       vk::ScoreTcArgs a{};
       a.mode = 0;
@@ -473,7 +473,8 @@ int vk_decode_step(const vk_view* view, const vk_params* params, const vk_index*
       a.scores_bf16 = 1;
       a.status = status;
       VK_CUDA(vk::launch_score_tc(v, r, digest, qhl, (int)L.soff, (int)L.ss, (int)L.ns, a, st), "sample scores");
-      VK_CUDA(vk::launch_theta(B, H, (int)L.ns, (int)L.sld, (int)L.soff, (int)L.ss, lo, hi, (int)L.j, sample, theta, st),
+      VK_CUDA(vk::launch_theta(B, H, (int)L.ns, (int)L.sld, (int)L.soff, (int)L.ss, lo, hi, (int)L.j, sample, theta, st,
+                               ccnt),   // also zeroes the candidate counts
               "theta");
       vk::ScoreTcArgs c{};
       c.mode = 1;

@@ -187,7 +187,8 @@ cudaError_t launch_sketch_basis(const void* queries, int dtype, int64_t n, int r
 // decreasing eigenvalue.
 cudaError_t launch_sym_eig64(const double* A, float* vec, float* eig, cudaStream_t st);
 cudaError_t launch_theta(int B, int H, int ns, int ld, int off, int stride, int lo, int hi, int j, const void* sample,
-                         float* theta, cudaStream_t st);
+                         float* theta, cudaStream_t st,
+                         int* zero_cnt = nullptr);
 cudaError_t launch_select_cand(int B, int H, int N, int lo, int hi, int64_t k, const int64_t* k_per_head,
                                const int* cand_cnt, const int2* cand, int capc, int force_fallback, const vk_view& v,
                                int r, const void* digest, const float* qt, int32_t* idx, int32_t* count, int cap,
