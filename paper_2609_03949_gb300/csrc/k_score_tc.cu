@@ -502,8 +502,13 @@ __global__ void __launch_bounds__(TcCfg<MH, NHG, TM_, G_, WPQ_, RW_, SK_, MODE>:
               }
             }
           } else if (MODE == 1) {
+            // v >= theta exactly when v - theta' has a clear sign bit, theta' = theta with +0 taken as -0 (so that
+            // v = -0 against theta = +0 gives +0, not -0): the sign bits are shifted in one instruction per row
+            const float tq = th[hg] == 0.f ? -0.f : th[hg];
+            uint32_t below = 0u;                         // bit 31 - k: row k is below theta
 #pragma unroll
-            for (int k = 0; k < 32; ++k) m |= (v[k] >= th[hg] ? 1u : 0u) << k;
+            for (int k = 0; k < 32; ++k) below = __funnelshift_l(__float_as_uint(v[k] - tq), below, 1);
+            m = ~__brev(below);
             m &= range_mask(rc, args.arch_lo, min(args.arch_hi, args.n_rows));
             if (!valid) m = 0u;
           } else {
