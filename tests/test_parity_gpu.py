@@ -183,6 +183,8 @@ EDGES = [
     dict(B=2, H=64, N=2048, rho=1.0, window=0),            # dense
     dict(B=2, H=64, N=3000, rho=1 / 8, window=64, dtype="f32"),
     dict(B=1, H=256, N=2048, rho=1 / 8, window=64),
+    dict(B=3, H=192, N=5000, rho=1 / 16, window=64),        # three head groups: ranges of (sequence, row tile) x 3
+    dict(B=5, H=128, N=700, rho=1 / 4, window=32),          # two groups, ranges that cross sequence boundaries
     dict(B=300, H=16, N=100, rho=1 / 4, window=8),         # attention CTAs that span several whole segments
     dict(B=1, H=16, N=300000, rho=1 / 64, window=256),      # bitmaps past the selection's shared-memory limit
 ]
