@@ -11,14 +11,17 @@
 //            MN-major straight from its TMA tile, B = the Phi^T chunk; M = 64, N = mp, K = 128 per chunk;
 //   phase 2  low [128 rows x 64 dims] = Phi_chunk C: A = the Phi chunk, B = C rounded to bf16 by the epilogue into
 //            shared memory; M = 128, N = 64, K = mp, into one of four tensor-memory buffers. The R chunk is loaded
-//            again (phase 1 read it just before, so it comes from L2) into a ring of its own, and the epilogue (one
-//            thread per row) takes the row's low part from tensor memory and the row from shared memory, and
-//            writes sigma.
+//            again (mostly from L2) into a ring of its own, and the epilogue (one thread per row) takes the row's low
+//            part from tensor memory and the row from shared memory, and writes sigma.
+// Phase 2 of an item needs the item's whole C, so the items are software-pipelined: in round r every role takes phase
+// 1 of the CTA's item r and phase 2 of item r - 1, chunk by chunk, and the R stream from HBM (phase 1, a ring of its
+// own) goes on while the item before takes its phase 2. C is double-buffered in shared memory (item r's is written
+// while item r - 1's phase 2 products may still read the other).
 // Roles: warp 0 TMA producer, warp 1 MMA issuer, warps 2..9 epilogue in two groups of four (one warp per
 // tensor-memory lane quarter each): group 0 writes C and takes the even phase 2 chunks, group 1 the odd ones.
 // Phi is built in the workspace in bf16 twice: Phi^T [mp][T] and Phi [T][mp] (mp = 32 for kappa <= 16, 64 for
 // kappa <= 32, else 128). At mp = 32 the phase 2 operands (the Phi chunk and C) have 64-byte rows and the 64-byte
-// swizzle, and the narrower stages let the ring hold six.
+// swizzle.
 // Rows past the last closed block (the open tail) get sigma = -1. Every wait is bounded.
 #include <cuda.h>
 #include <cudaTypedefs.h>
@@ -38,16 +41,17 @@ constexpr uint32_t SG_RBYTES = SG_CH * 128;  // one chunk of R: 128 rows x 64 bf
 
 template <int MP>
 struct SgCfg {
-  static constexpr uint32_t PHT = 2 * MP * 128;          // Phi^T chunk: two 64-row K blocks of MP x 128 B
-  static constexpr uint32_t STAGE = SG_RBYTES + PHT;     // phase 1 stage (phase 2 uses its first 128 x MP x 2 B)
-  static constexpr int STAGES = MP == 32 ? 6 : MP == 64 ? 4 : 3;
-  static constexpr int R2 = MP == 128 ? 3 : 4;           // phase 2 ring of R chunks for the epilogue
-  static constexpr uint32_t ROW2 = MP == 32 ? 64 : 128;  // phase 2 operand row bytes (Phi chunk and C)
+  static constexpr uint32_t PHT = 2 * MP * 128;          // Phi^T chunk: two 64-row boxes of MP x 128 B
+  static constexpr uint32_t STAGE1 = SG_RBYTES + PHT;    // a stage: an R chunk and its Phi^T chunk
+  static constexpr int S1 = MP == 32 ? 6 : MP == 64 ? 5 : 3;   // the stage ring (the HBM stream)
+  static constexpr int R2 = MP == 32 ? 4 : 3;                  // phase 2 ring of R chunks for the epilogue
+  static constexpr uint32_t ROW2 = MP == 32 ? 64 : 128;  // row bytes of C, the phase 2 B operand
   static constexpr int NL = 4;                           // tensor-memory buffers of the phase 2 product
-  static constexpr uint32_t cbuf = STAGES * STAGE;       // C as the phase 2 B operand: MP / 64 blocks of 64 x 128 B
-  static constexpr uint32_t r2 = cbuf + 64 * MP * 2;
+  static constexpr uint32_t CB = 64 * MP * 2;            // C as the phase 2 B operand: MP / 64 blocks of 64 x 128 B
+  static constexpr uint32_t cbuf = S1 * STAGE1;          // two C buffers: one block's C while the next is written
+  static constexpr uint32_t r2 = cbuf + 2 * CB;
   static constexpr uint32_t bars = r2 + R2 * SG_RBYTES;
-  static constexpr uint32_t total = bars + (2 * STAGES + 2 * R2 + 2 + 2 * NL) * 8 + 1024;
+  static constexpr uint32_t total = bars + (2 * S1 + 2 * R2 + 2 + 2 * NL) * 8 + 1024;
   static_assert(total <= 232448, "sigma shared memory exceeds the 227 KB opt-in limit");
 };
 
@@ -70,6 +74,11 @@ __device__ __forceinline__ void sg_tma_2d(void* dst, const CUtensorMap* map, int
 __device__ __forceinline__ uint64_t sg_desc(uint32_t saddr) {
   return (uint64_t)((saddr >> 4) & 0x3FFFu) | ((uint64_t)1u << 16) | ((uint64_t)(1024u >> 4) << 32) |
          ((uint64_t)1u << 46) | ((uint64_t)2u << 61);
+}
+// MN-major operand, 128-byte swizzle: 64-element atoms along M/N `lbo` bytes apart, 8-row K groups 1024 B apart.
+__device__ __forceinline__ uint64_t sg_desc_mn(uint32_t saddr, uint32_t lbo) {
+  return (uint64_t)((saddr >> 4) & 0x3FFFu) | ((uint64_t)((lbo >> 4) & 0x3FFFu) << 16) |
+         ((uint64_t)(1024u >> 4) << 32) | ((uint64_t)1u << 46) | ((uint64_t)2u << 61);
 }
 // K-major operand with 64-byte rows, 64-byte swizzle: 8-row groups 512 B apart.
 __device__ __forceinline__ uint64_t sg_desc64(uint32_t saddr) {
@@ -138,16 +147,15 @@ struct SigmaArgs {
 
 template <int MP>
 __global__ void __launch_bounds__(SG_THREADS, 1) k_sigma(const __grid_constant__ CUtensorMap rmap,
-                                                       const __grid_constant__ CUtensorMap ptmap,
-                                                       const __grid_constant__ CUtensorMap pmap, const SigmaArgs args) {
+                                                       const __grid_constant__ CUtensorMap ptmap, const SigmaArgs args) {
   using L = SgCfg<MP>;
   extern __shared__ __align__(1024) unsigned char smem_raw[];
   unsigned char* smem = reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   unsigned char* cb = smem + L::cbuf;
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + L::bars);
-  uint64_t* full = bars;                   // [STAGES]
-  uint64_t* empty = bars + L::STAGES;      // [STAGES]
-  uint64_t* c_full = empty + L::STAGES;    // phase 1 of an item is complete
+  uint64_t* full1 = bars;                  // [S1] a stage has landed
+  uint64_t* empty1 = full1 + L::S1;        // [S1] its products (both phases) are done
+  uint64_t* c_full = empty1 + L::S1;       // phase 1 of an item is complete
   uint64_t* c_ready = c_full + 1;          // the epilogue has written C (bf16) for phase 2
   uint64_t* l_full = c_ready + 1;          // [NL] a phase 2 chunk's low part is in tensor memory
   uint64_t* l_empty = l_full + L::NL;      // [NL] the epilogue has read it
@@ -164,7 +172,7 @@ __global__ void __launch_bounds__(SG_THREADS, 1) k_sigma(const __grid_constant__
 
   if (threadIdx.x == 0) {
     abort_flag = 0;
-    for (int s = 0; s < L::STAGES; ++s) { mbar_init(&full[s], 1); mbar_init(&empty[s], 1); }
+    for (int s = 0; s < L::S1; ++s) { mbar_init(&full1[s], 1); mbar_init(&empty1[s], 1); }
     mbar_init(c_full, 1);
     mbar_init(c_ready, 4);
     for (int i = 0; i < L::NL; ++i) { mbar_init(&l_full[i], 1); mbar_init(&l_empty[i], 4); }
@@ -179,37 +187,41 @@ __global__ void __launch_bounds__(SG_THREADS, 1) k_sigma(const __grid_constant__
 
   if (warp == 0) {
     // ------------------------------------------------------------------ producer
+    // Round r loads phase 1 of the CTA's item r and phase 2 of item r - 1, chunk by chunk, so that the phase 1 stream
+    // from HBM goes on while the item before takes its phase 2 (whose R chunks come again, mostly from L2).
     if (lane == 0) {
-      int n = 0, n2 = 0;                                  // loads issued into the ring and into the R ring
+      int n1 = 0, n2 = 0;                                 // phase 1 stages and phase 2 chunks issued
       bool ok = true;
-      for (long long it = i0; it < i1 && ok; ++it) {
-        const int b = (int)(it / args.nb), blk = (int)(it - (long long)b * args.nb);
-        for (int ph = 0; ph < 2 && ok; ++ph) {
-          for (int c = 0; c < nchunk; ++c, ++n) {
-            const int s = n % L::STAGES, use = n / L::STAGES;
-            if (use > 0 && !mbar_wait(&empty[s], (use - 1) & 1, &abort_flag)) { ok = false; break; }
-            unsigned char* st = smem + s * L::STAGE;
-            const int u0 = c * SG_CH;
-            if (ph == 0) {
-              mbar_arrive_expect_tx(&full[s], SG_RBYTES + L::PHT);
-              sg_tma_3d(st, &rmap, 0, blk * args.T + u0, b, &full[s]);
-              sg_tma_2d(st + SG_RBYTES, &ptmap, u0, 0, &full[s]);
-              sg_tma_2d(st + SG_RBYTES + MP * 128, &ptmap, u0 + 64, 0, &full[s]);
-            } else {
-              mbar_arrive_expect_tx(&full[s], (uint32_t)MP * 256u);
-              for (int kb = 0; kb < (MP + 63) / 64; ++kb) sg_tma_2d(st + kb * 16384, &pmap, 64 * kb, u0, &full[s]);
-              const int s2 = n2 % L::R2, use2 = n2 / L::R2;
-              if (use2 > 0 && !mbar_wait(&r_empty[s2], (use2 - 1) & 1, &abort_flag)) { ok = false; ++n; break; }
-              mbar_arrive_expect_tx(&r_full[s2], SG_RBYTES);
-              sg_tma_3d(rbuf + s2 * SG_RBYTES, &rmap, 0, blk * args.T + u0, b, &r_full[s2]);
-              ++n2;
-            }
+      const long long nitems = i1 - i0;
+      for (long long r = 0; r <= nitems && ok; ++r) {
+        const bool has1 = r < nitems, has2 = r >= 1;
+        const long long it1 = i0 + r, it2 = i0 + r - 1;
+        const int b1 = has1 ? (int)(it1 / args.nb) : 0, blk1 = has1 ? (int)(it1 - (long long)b1 * args.nb) : 0;
+        const int b2 = has2 ? (int)(it2 / args.nb) : 0, blk2 = has2 ? (int)(it2 - (long long)b2 * args.nb) : 0;
+        for (int c = 0; c < nchunk; ++c) {
+          const int u0 = c * SG_CH;
+          // the stage: chunk c of Phi^T (phase 1's B operand and phase 2's A operand: both phases of the round use
+          // the same rows of the basis) and, with a phase 1, item r's R chunk
+          const int s = n1 % L::S1, use = n1 / L::S1;
+          if (use > 0 && !mbar_wait(&empty1[s], (use - 1) & 1, &abort_flag)) { ok = false; break; }
+          unsigned char* st = smem + s * L::STAGE1;
+          mbar_arrive_expect_tx(&full1[s], L::PHT + (has1 ? SG_RBYTES : 0u));
+          if (has1) sg_tma_3d(st, &rmap, 0, blk1 * args.T + u0, b1, &full1[s]);
+          sg_tma_2d(st + SG_RBYTES, &ptmap, u0, 0, &full1[s]);
+          sg_tma_2d(st + SG_RBYTES + MP * 128, &ptmap, u0 + 64, 0, &full1[s]);
+          ++n1;
+          if (has2) {
+            const int s2 = n2 % L::R2, use2 = n2 / L::R2;
+            if (use2 > 0 && !mbar_wait(&r_empty[s2], (use2 - 1) & 1, &abort_flag)) { ok = false; break; }
+            mbar_arrive_expect_tx(&r_full[s2], SG_RBYTES);
+            sg_tma_3d(rbuf + s2 * SG_RBYTES, &rmap, 0, blk2 * args.T + u0, b2, &r_full[s2]);
+            ++n2;
           }
         }
       }
       if (!ok) abort_flag = 1;
       // drain: the last load of every stage has landed before the CTA may leave (already true unless it aborted)
-      for (int k = std::max(0, n - L::STAGES); k < n; ++k) mbar_wait(&full[k % L::STAGES], (k / L::STAGES) & 1, nullptr);
+      for (int k = std::max(0, n1 - L::S1); k < n1; ++k) mbar_wait(&full1[k % L::S1], (k / L::S1) & 1, nullptr);
       for (int k = std::max(0, n2 - L::R2); k < n2; ++k) mbar_wait(&r_full[k % L::R2], (k / L::R2) & 1, nullptr);
     }
   } else if (warp == 1) {
@@ -218,45 +230,56 @@ __global__ void __launch_bounds__(SG_THREADS, 1) k_sigma(const __grid_constant__
       // phase 1: D = C^T (M = 64 dims, N = MP), A = R^T MN-major (bit 15), B = Phi^T K-major
       constexpr uint32_t idesc1 = (1u << 4) | (1u << 7) | (1u << 10) | (1u << 15) | ((uint32_t)(MP >> 3) << 17) |
                                   ((uint32_t)(64 >> 4) << 24);
-      // phase 2: D = low (M = 128 rows, N = 64 dims), both K-major
-      constexpr uint32_t idesc2 = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(64 >> 3) << 17) |
+      // phase 2: D = low (M = 128 rows, N = 64 dims), A = Phi MN-major (bit 15: the Phi^T chunk), B = C K-major
+      constexpr uint32_t idesc2 = (1u << 4) | (1u << 7) | (1u << 10) | (1u << 15) | ((uint32_t)(64 >> 3) << 17) |
                                   ((uint32_t)(128 >> 4) << 24);
-      int n = 0, nit = 0, nl = 0;
+      // round r: phase 1 of item r (into C^T) and phase 2 of item r - 1 (from C in shared memory), chunk by chunk
+      int n1 = 0, n2 = 0, ncf = 0;                        // ncf: commits of c_full
       bool ok = true;
-      for (long long it = i0; it < i1 && ok; ++it, ++nit) {
-        for (int c = 0; c < nchunk; ++c, ++n) {
-          const int s = n % L::STAGES, use = n / L::STAGES;
-          if (!mbar_wait(&full[s], use & 1, &abort_flag)) { ok = false; break; }
+      const long long nitems = i1 - i0;
+      for (long long r = 0; r <= nitems && ok; ++r) {
+        const bool has1 = r < nitems, has2 = r >= 1;
+        if (has2) {
+          // item r - 1's C is in shared memory and its C^T has left tensor memory (item r may accumulate there)
+          if (!mbar_wait(c_ready, (uint32_t)((r - 1) & 1), &abort_flag)) { ok = false; break; }
           tmem_fence_after();
-          const uint32_t st = smem_addr(smem + s * L::STAGE);
-#pragma unroll
-          for (int j = 0; j < 8; ++j) {                   // 16 rows per instruction
-            const uint64_t ad = sg_desc(st + j * 2048);
-            const uint64_t bd = sg_desc(st + SG_RBYTES + (j >> 2) * (MP * 128) + (j & 3) * 32);
-            sg_mma(tmem + C_COL, ad, bd, idesc1, (c > 0 || j > 0) ? 1u : 0u);
-          }
-          sg_commit(&empty[s]);
         }
-        if (!ok) break;
-        sg_commit(c_full);
-        if (!mbar_wait(c_ready, nit & 1, &abort_flag)) { ok = false; break; }   // C in shared memory (bf16)
-        tmem_fence_after();
-        const uint32_t cba = smem_addr(cb);
-        for (int c = 0; c < nchunk; ++c, ++n, ++nl) {
-          const int s = n % L::STAGES, use = n / L::STAGES;
-          const int lb = nl % L::NL, luse = nl / L::NL;
-          if (!mbar_wait(&full[s], use & 1, &abort_flag)) { ok = false; break; }
-          if (luse > 0 && !mbar_wait(&l_empty[lb], (luse - 1) & 1, &abort_flag)) { ok = false; break; }
+        const uint32_t cba = smem_addr(cb + (uint32_t)((r - 1) & 1) * L::CB);
+        for (int c = 0; c < nchunk; ++c) {
+          const int s = n1 % L::S1, use = n1 / L::S1;
+          if (!mbar_wait(&full1[s], use & 1, &abort_flag)) { ok = false; break; }
+          const int lb = n2 % L::NL, luse = n2 / L::NL;
+          if (has2 && luse > 0 && !mbar_wait(&l_empty[lb], (luse - 1) & 1, &abort_flag)) { ok = false; break; }
           tmem_fence_after();
-          const uint32_t st = smem_addr(smem + s * L::STAGE);
+          const uint32_t st = smem_addr(smem + s * L::STAGE1);
+          if (has1) {
 #pragma unroll
-          for (int j = 0; j < MP / 16; ++j) {
-            const uint64_t ad = sg_desc2<MP>(st + (j >> 2) * 16384 + (j & 3) * 32);
-            const uint64_t bd = sg_desc2<MP>(cba + (j >> 2) * 8192 + (j & 3) * 32);
-            sg_mma(tmem + L_COL + 64 * lb, ad, bd, idesc2, j > 0 ? 1u : 0u);
+            for (int j = 0; j < 8; ++j) {                 // 16 rows per instruction
+              const uint64_t ad = sg_desc(st + j * 2048);
+              const uint64_t bd = sg_desc(st + SG_RBYTES + (j >> 2) * (MP * 128) + (j & 3) * 32);
+              sg_mma(tmem + C_COL, ad, bd, idesc1, (c > 0 || j > 0) ? 1u : 0u);
+            }
           }
-          sg_commit(&empty[s]);
-          sg_commit(&l_full[lb]);
+          if (has2) {
+            // A = the Phi^T chunk read MN-major (the chunk's 128 rows in two 64-row atoms MP x 128 B apart, 16 bins
+            // per instruction), B = item r - 1's C
+#pragma unroll
+            for (int j = 0; j < MP / 16; ++j) {
+              const uint64_t ad = sg_desc_mn(st + SG_RBYTES + j * 2048, MP * 128);
+              const uint64_t bd = sg_desc2<MP>(cba + (j >> 2) * 8192 + (j & 3) * 32);
+              sg_mma(tmem + L_COL + 64 * lb, ad, bd, idesc2, j > 0 ? 1u : 0u);
+            }
+          }
+          sg_commit(&empty1[s]);
+          ++n1;
+          if (has2) {
+            sg_commit(&l_full[lb]);
+            ++n2;
+          }
+        }
+        if (ok && has1) {
+          sg_commit(c_full);
+          ++ncf;
         }
       }
       if (!ok) {
@@ -265,19 +288,65 @@ __global__ void __launch_bounds__(SG_THREADS, 1) k_sigma(const __grid_constant__
       }
       // nothing this thread issued may outlive the CTA
       sg_commit(c_full);
-      mbar_wait(c_full, nit & 1, nullptr);
+      mbar_wait(c_full, ncf & 1, nullptr);
     }
   } else {
     // ------------------------------------------------------------------ epilogue
     const int q = warp & 3;                               // tensor-memory lane quarter
     const int eg = (warp - 2) >> 2;                       // epilogue group: 0 writes C, the groups split the chunks
     const uint32_t lq = (uint32_t)(32 * q) << 16;
-    int nit = 0;
+    // round r: phase 2 of item r - 1 (the groups take alternate chunks), then group 0 turns item r's C^T into C
     bool ok = true;
-    for (long long it = i0; it < i1 && ok; ++it, ++nit) {
-      const int b = (int)(it / args.nb), blk = (int)(it - (long long)b * args.nb);
-      if (eg == 0) {
-        if (!warp_wait_sg(c_full, nit & 1, &abort_flag, lane)) { ok = false; break; }
+    const long long nitems = i1 - i0;
+    for (long long r = 0; r <= nitems && ok; ++r) {
+      if (r >= 1) {
+        const long long it = i0 + r - 1;
+        const int b = (int)(it / args.nb), blk = (int)(it - (long long)b * args.nb);
+        // phase 2: one row per thread; the row from the R ring (128-byte swizzle: chunk k of row x sits at k ^ (x & 7));
+        // chunk c of this item is the ((r - 1) nchunk + c)-th phase 2 chunk of the CTA, taken by group c % 2
+        for (int c = eg; c < nchunk; c += 2) {
+          const int nl = (int)(r - 1) * nchunk + c;
+          const int lb = nl % L::NL, luse = nl / L::NL;
+          const int s2 = nl % L::R2, use2 = nl / L::R2;
+          if (!warp_wait_sg(&l_full[lb], luse & 1, &abort_flag, lane) ||
+              !warp_wait_sg(&r_full[s2], use2 & 1, &abort_flag, lane)) {
+            ok = false;
+            break;
+          }
+          tmem_fence_after();
+          float lo[64];
+          sg_ld32(tmem + lq + L_COL + 64 * lb, lo);
+          sg_ld32(tmem + lq + L_COL + 64 * lb + 32, lo + 32);
+          tmem_wait_ld();
+          tmem_fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(&l_empty[lb]);
+          const int x = 32 * q + lane;                      // row within the chunk
+          const int u = blk * args.T + c * SG_CH + x;
+          const unsigned char* rrow = rbuf + s2 * SG_RBYTES + x * 128;
+          uint4 rv[8];
+#pragma unroll
+          for (int k = 0; k < 8; ++k) rv[k] = *reinterpret_cast<const uint4*>(rrow + ((k ^ (x & 7)) * 16));
+          __syncwarp();
+          if (lane == 0) mbar_arrive(&r_empty[s2]);
+          float acc = 0.f;
+#pragma unroll
+          for (int k = 0; k < 8; ++k) {
+            const uint4 w = rv[k];
+            const uint32_t ww[4] = {w.x, w.y, w.z, w.w};
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+              const float d0 = bf_lo(ww[e]) - lo[8 * k + 2 * e], d1 = bf_hi(ww[e]) - lo[8 * k + 2 * e + 1];
+              acc = fmaf(d0, d0, acc);
+              acc = fmaf(d1, d1, acc);
+            }
+          }
+          args.sigma[(int64_t)b * args.N + u] = sqrtf(acc);
+        }
+        if (!ok) break;
+      }
+      if (r < nitems && eg == 0) {
+        if (!warp_wait_sg(c_full, (uint32_t)(r & 1), &abort_flag, lane)) { ok = false; break; }
         tmem_fence_after();
         {
           // C^T row d = 16 q + (lane % 16) (M = 64 layout), bins 32 (lane / 16) + 64 kb .. + 31 -> bf16 into the B
@@ -290,7 +359,7 @@ __global__ void __launch_bounds__(SG_THREADS, 1) k_sigma(const __grid_constant__
             sg_ld16x2(tmem + lq + C_COL + 64 * kb, v);
             tmem_wait_ld();
             if (MP == 32 && half) continue;               // columns past the 32 bins
-            unsigned char* row = cb + kb * 8192 + d * L::ROW2;
+            unsigned char* row = cb + (uint32_t)(r & 1) * L::CB + kb * 8192 + d * L::ROW2;
 #pragma unroll
             for (int k = 0; k < 4; ++k) {
               uint32_t w[4];
@@ -309,47 +378,6 @@ __global__ void __launch_bounds__(SG_THREADS, 1) k_sigma(const __grid_constant__
         __syncwarp();
         if (lane == 0) mbar_arrive(c_ready);
       }
-      // phase 2: one row per thread; the row from the R ring (128-byte swizzle: chunk k of row x sits at k ^ (x & 7));
-      // chunk c of this item is the (nit * nchunk + c)-th phase 2 chunk of the CTA, taken by group c % 2
-      for (int c = eg; c < nchunk; c += 2) {
-        const int nl = nit * nchunk + c;
-        const int lb = nl % L::NL, luse = nl / L::NL;
-        const int s2 = nl % L::R2, use2 = nl / L::R2;
-        if (!warp_wait_sg(&l_full[lb], luse & 1, &abort_flag, lane) ||
-            !warp_wait_sg(&r_full[s2], use2 & 1, &abort_flag, lane)) {
-          ok = false;
-          break;
-        }
-        tmem_fence_after();
-        float lo[64];
-        sg_ld32(tmem + lq + L_COL + 64 * lb, lo);
-        sg_ld32(tmem + lq + L_COL + 64 * lb + 32, lo + 32);
-        tmem_wait_ld();
-        tmem_fence_before();
-        __syncwarp();
-        if (lane == 0) mbar_arrive(&l_empty[lb]);
-        const int x = 32 * q + lane;                      // row within the chunk
-        const int u = blk * args.T + c * SG_CH + x;
-        const unsigned char* rrow = rbuf + s2 * SG_RBYTES + x * 128;
-        uint4 rv[8];
-#pragma unroll
-        for (int k = 0; k < 8; ++k) rv[k] = *reinterpret_cast<const uint4*>(rrow + ((k ^ (x & 7)) * 16));
-        __syncwarp();
-        if (lane == 0) mbar_arrive(&r_empty[s2]);
-        float acc = 0.f;
-#pragma unroll
-        for (int k = 0; k < 8; ++k) {
-          const uint4 w = rv[k];
-          const uint32_t ww[4] = {w.x, w.y, w.z, w.w};
-#pragma unroll
-          for (int e = 0; e < 4; ++e) {
-            const float d0 = bf_lo(ww[e]) - lo[8 * k + 2 * e], d1 = bf_hi(ww[e]) - lo[8 * k + 2 * e + 1];
-            acc = fmaf(d0, d0, acc);
-            acc = fmaf(d1, d1, acc);
-          }
-        }
-        args.sigma[(int64_t)b * args.N + u] = sqrtf(acc);
-      }
     }
     if (!ok && lane == 0) {
       abort_flag = 1;
@@ -364,28 +392,28 @@ __global__ void __launch_bounds__(SG_THREADS, 1) k_sigma(const __grid_constant__
   }
 }
 
-// The two bf16 copies of Phi (orthonormal low-pass basis, column n): 0 the constant 1/sqrt(T); 2 k - 1 and 2 k the
-// cosine and sine of bin k = 1 .. npair times sqrt(2/T); then the alternation (-1)^u / sqrt(T) when kappa > T/2;
-// zero up to mp. Angles are reduced exactly (k u mod T) before cospi / sinpi.
-__global__ void k_sigma_basis(int T, int kappa, int mp, __nv_bfloat16* phit, __nv_bfloat16* phi) {
+// Phi^T [mp][T] in bf16 (the orthonormal low-pass basis, column n of Phi = row n here): 0 the constant 1/sqrt(T);
+// 2 k - 1 and 2 k the cosine and sine of bin k = 1 .. npair times sqrt(2/T); then the alternation (-1)^u / sqrt(T)
+// when kappa > T/2; zero up to mp. The angle is reduced exactly (k u mod T, in integers) before cospif / sinpif: fp32
+// is ample for values rounded to bf16. Consecutive threads take consecutive positions u of one row.
+__global__ void k_sigma_basis(int T, int kappa, int mp, __nv_bfloat16* phit) {
   const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
   if (i >= (int64_t)T * mp) return;
-  const int u = (int)(i / mp), n = (int)(i - (int64_t)u * mp);
+  const int n = (int)(i / T), u = (int)(i - (int64_t)n * T);
   const int npair = max(0, min(kappa - 1, T / 2 - 1));     // bins 1 .. npair (T is even)
   const int m = 1 + 2 * npair + (kappa > T / 2 ? 1 : 0);
-  double v = 0.0;
+  const float inv_sqrt_t = rsqrtf((float)T);
+  float v = 0.f;
   if (n == 0) {
-    v = 1.0 / sqrt((double)T);
+    v = inv_sqrt_t;
   } else if (n < 1 + 2 * npair) {
     const int k = (n + 1) / 2;
-    const double x = 2.0 * (double)(((int64_t)k * u) % T) / (double)T;
-    v = sqrt(2.0 / (double)T) * ((n & 1) ? cospi(x) : sinpi(x));
+    const float x = 2.f * (float)(((int64_t)k * u) % T) / (float)T;
+    v = sqrtf(2.f) * inv_sqrt_t * ((n & 1) ? cospif(x) : sinpif(x));
   } else if (n < m) {
-    v = ((u & 1) ? -1.0 : 1.0) / sqrt((double)T);
+    v = ((u & 1) ? -1.f : 1.f) * inv_sqrt_t;
   }
-  const __nv_bfloat16 h = __double2bfloat16(v);
-  phi[(int64_t)u * mp + n] = h;
-  phit[(int64_t)n * T + u] = h;
+  phit[i] = __float2bfloat16_rn(v);
 }
 
 __global__ void k_sigma_tail(int N, int closed, float* sigma) {
@@ -411,9 +439,8 @@ cudaError_t launch_sigma_mp(const vk_view& v, int T, int kappa, float* sigma, vo
   auto encode = sg_encode();
   if (!encode) return cudaErrorNotSupported;
   __nv_bfloat16* phit = static_cast<__nv_bfloat16*>(ws);
-  __nv_bfloat16* phi = phit + (int64_t)MP * T;
   const int64_t ne = (int64_t)T * MP;
-  k_sigma_basis<<<(unsigned)((ne + 255) / 256), 256, 0, st>>>(T, kappa, MP, phit, phi);
+  k_sigma_basis<<<(unsigned)((ne + 255) / 256), 256, 0, st>>>(T, kappa, MP, phit);
   count_launches(1);
   const int nb = v.N / T, closed = nb * T;
   if (closed < v.N) {
@@ -422,7 +449,7 @@ cudaError_t launch_sigma_mp(const vk_view& v, int T, int kappa, float* sigma, vo
     count_launches(1);
   }
   if (nb == 0) return cudaGetLastError();
-  CUtensorMap rmap, ptmap, pmap;
+  CUtensorMap rmap, ptmap;
   {
     cuuint64_t dims[3] = {(cuuint64_t)D_ROPE, (cuuint64_t)v.N, (cuuint64_t)v.B};
     cuuint64_t str[2] = {(cuuint64_t)(v.rope_ld * 2), (cuuint64_t)(v.rope_bstride * 2)};
@@ -443,16 +470,6 @@ cudaError_t launch_sigma_mp(const vk_view& v, int T, int kappa, float* sigma, vo
                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
       return cudaErrorInvalidValue;
   }
-  {
-    cuuint64_t dims[2] = {(cuuint64_t)MP, (cuuint64_t)T};
-    cuuint64_t str[1] = {(cuuint64_t)MP * 2};
-    cuuint32_t box[2] = {(cuuint32_t)(MP < 64 ? MP : 64), (cuuint32_t)SG_CH};
-    cuuint32_t es[2] = {1, 1};
-    if (encode(&pmap, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, phi, dims, str, box, es, CU_TENSOR_MAP_INTERLEAVE_NONE,
-               MP == 32 ? CU_TENSOR_MAP_SWIZZLE_64B : CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
-               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
-      return cudaErrorInvalidValue;
-  }
   SigmaArgs a{};
   a.B = v.B;
   a.N = v.N;
@@ -468,7 +485,7 @@ cudaError_t launch_sigma_mp(const vk_view& v, int T, int kappa, float* sigma, vo
   const size_t smem = SgCfg<MP>::total;
   cudaError_t e = cudaFuncSetAttribute(k_sigma<MP>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
-  k_sigma<MP><<<grid, SG_THREADS, smem, st>>>(rmap, ptmap, pmap, a);
+  k_sigma<MP><<<grid, SG_THREADS, smem, st>>>(rmap, ptmap, a);
   count_launches(1);
   return cudaGetLastError();
 }
@@ -478,7 +495,7 @@ cudaError_t launch_sigma_mp(const vk_view& v, int T, int kappa, float* sigma, vo
 int sigma_basis_cols(int kappa) { return kappa <= 16 ? 32 : kappa <= 32 ? 64 : 128; }
 
 size_t sigma_workspace_bytes(int T, int kappa) {
-  return 256 + (size_t)2 * 2 * sigma_basis_cols(kappa) * (size_t)T;   // status word, Phi^T and Phi (bf16)
+  return 256 + (size_t)2 * sigma_basis_cols(kappa) * (size_t)T;   // status word, Phi^T (bf16)
 }
 
 cudaError_t launch_sigma(const vk_view& v, int T, int kappa, float* sigma, void* ws, cudaStream_t st) {
