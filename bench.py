@@ -346,6 +346,64 @@ def sigma_throughput(vk, view, B, N, stream, hbm_peak, T=4096, kappa=16, reps=5)
             "bound": "hbm (two bf16 contractions of 64 x 31 per row: 32 flop/B, below the tensor ridge)"}
 
 
+def offstep_throughput(vk, view, wl, w, B, N, H, dev, stream, hbm_peak, buf, reps=3):
+    """The parts of the method that run off the decode step, on the bench cache, each timed with CUDA events on the
+    launching stream (mean of `reps` calls after two warm-up calls), with the algorithmic bytes of its one pass over
+    the cache against the copy bandwidth: the PCA digest basis (the RoPE branch's second moment, then a 64 x 64
+    eigensolve), the rank-64 content sketch (its basis from the context's prefix queries, then every row's entry) and
+    the conformal calibration of z (every (b, h) of the step as a calibration query; its all-rows attention pass
+    reads every cached row once)."""
+    def timed(fn):
+        for _ in range(2):
+            fn()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        torch.cuda.synchronize()
+        e0.record(stream)
+        for _ in range(reps):
+            fn()
+        e1.record(stream)
+        torch.cuda.synchronize()
+        return e0.elapsed_time(e1) / reps
+
+    def roof(ms, byts):
+        gbs = byts / (ms * 1e-3) / 1e9
+        return {"algorithmic_bytes": byts, "achieved_gbs": gbs, "frac_of_peak": gbs / hbm_peak}
+
+    out = {}
+    rot = torch.empty(64, 64, device=dev)
+    eig = torch.empty(64, device=dev)
+    pws = vk.alloc_bytes(int(vk.lib().vk_pca_workspace_bytes()))
+    ms = timed(lambda: vk.vk_pca_basis(view, rot, eig, pws))
+    assert vk.vk_poll_status(pws) == vk.VK_OK
+    out["pca"] = {"kernels": "k_pca_moment + k_pca_jacobi", "rows": B * N, "ms": ms, **roof(ms, B * N * 128)}
+
+    q = datagen.prefix_queries(wl, N_PREFIX - 1).to(dev).contiguous()
+    basis = torch.empty(64, 512, device=dev)
+    sws = vk.vk_sketch_basis(q, 64, basis)
+    ms_b = timed(lambda: vk.vk_sketch_basis(q, 64, basis, ws=sws))
+    sketch = torch.empty(B, N, 64, dtype=torch.bfloat16, device=dev)
+    eta = torch.empty(B, N, device=dev)
+    ms_s = timed(lambda: vk.vk_build_sketch(view, 64, basis, sketch, eta))
+    out["sketch"] = {"r_sk": 64, "prefix_queries": int(q.shape[0]), "basis_ms": ms_b, "build_kernel": "k_sketch_rows",
+                     "build_ms": ms_s, **roof(ms_s, B * N * (1024 + 2 * 64 + 4))}
+    del sketch
+
+    params = vk.make_params(w.rho, r=64, window=w.window)
+    P = (N + 63) // 64
+    pres, pk, pe = (torch.empty(B, P, device=dev) for _ in range(3))
+    vk.vk_build_digest(view, params, wl.rot.contiguous(), None, eta, pres, pk, pe)
+    index = vk.make_index(None, eta, pres, None, pk, pe)
+    buf.run(view, params, index)
+    zq = torch.empty(B, H, device=dev)
+    z_out = torch.empty(3, device=dev)
+    cws = vk.vk_conformal_z(view, params, index, buf.idx, buf.count, zq, z_out)
+    ms_c = timed(lambda: vk.vk_conformal_z(view, params, index, buf.idx, buf.count, zq, z_out, ws=cws))
+    assert vk.vk_poll_status(cws) == vk.VK_OK
+    out["conformal"] = {"queries": B * H, "kernels": "k_attn_tc (all rows, argmax) + k_calib_zq + "
+                        "k_conformal_quantile", "ms": ms_c, **roof(ms_c, B * N * 1152)}
+    return out
+
+
 def run_native(args):
     rank, world, local = dist_env()
     if args.gpus != world and world > 1:
@@ -531,9 +589,10 @@ def run_native(args):
     assert all(torch.isfinite(t).all() for t in lseh)
     assert vk.vk_poll_status(bufs[1].ws) == vk.VK_OK
 
-    sigma = None
+    sigma = offstep = None
     if w.name == DEFAULT_CONFIG and w.dtype == "bf16":
         sigma = sigma_throughput(vk, view, B, N, stream, hbm_peak)
+        offstep = offstep_throughput(vk, view, wl, w, B, N, H, dev, stream, hbm_peak, buf)
 
     cpu = cpu1 = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
@@ -555,6 +614,7 @@ def run_native(args):
                  "fired_new_rows_per_seq": (U - U1) / B,
                  "stage_ms": {st: float(stage_ms[i]) for i, st in enumerate(STAGES)}},
         "sigma": sigma,
+        "offstep": offstep,
     }
     if rank == 0:
         print(json.dumps(line), flush=True)
