@@ -3,8 +3,8 @@
 // V (r_sk orthonormal directions of the 512-wide content space, the rows of basis [r_sk][512] fp32) splits the content
 // logit: qc . L = (V qc) . (V L) + delta with |delta| <= |(I - V^T V) qc| |(I - V^T V) L|.
 //   k_sketch_rows   index entry of every cached row: s_u = V L_u (bf16, round to nearest even) and eta_u =
-//                   |L_u - V^T s_u| (with the fp32 s_u). One warp per row, lane l holding dims l + 32 i; the basis
-//                   sits in shared memory.
+//                   |L_u - V^T s_u| (with the fp32 s_u). Four rows per warp, lane l holding dims l + 32 i of each;
+//                   the basis sits in shared memory, and each of its rows is read once for the four.
 //   k_sketch_query  per (b, h): p = V qc (fp32, and its bf16 high and low parts in the [B][2][H][r_sk] layout the
 //                   tensor-core trigger loads) and rho = |qc - V^T p|, the certificate's query norm.
 //   basis from the context's queries (V from the prefix queries): the second moment M = sum_i q_i q_i^T in fp32
@@ -19,6 +19,8 @@
 namespace vk {
 
 namespace {
+
+constexpr int SKR_RW = 4, SKR_NT = 256;             // rows per warp and threads per block of the index build
 
 __device__ __forceinline__ float warp_sum(float x) {
 #pragma unroll
@@ -50,26 +52,70 @@ __device__ __forceinline__ float project(const float* __restrict__ vb, int r_sk,
   return sqrtf(warp_sum(e));
 }
 
-template <typename T>
-__global__ void __launch_bounds__(256) k_sketch_rows(int64_t rows, int N, int r_sk, const T* __restrict__ latent,
-                                                     int64_t lld, int64_t lbs, const float* __restrict__ basis,
-                                                     __nv_bfloat16* __restrict__ sketch, float* __restrict__ eta) {
+// RW rows per warp: each basis row is loaded from shared memory once for all of them, and their warp sums run side by
+// side; every row takes the same operations in the same order as project() (the results do not depend on RW).
+template <typename T, int RW, int NT>
+__global__ void __launch_bounds__(NT) k_sketch_rows(int64_t rows, int N, int r_sk, const T* __restrict__ latent,
+                                                    int64_t lld, int64_t lbs, const float* __restrict__ basis,
+                                                    __nv_bfloat16* __restrict__ sketch, float* __restrict__ eta) {
   extern __shared__ float vb[];                       // [r_sk][512]
   for (int e = threadIdx.x; e < r_sk * D_LAT; e += blockDim.x) vb[e] = basis[e];
   __syncthreads();
   const int lane = threadIdx.x & 31, warps = blockDim.x >> 5;
-  for (int64_t row = (int64_t)blockIdx.x * warps + (threadIdx.x >> 5); row < rows; row += (int64_t)gridDim.x * warps) {
-    const int64_t b = row / N, u = row - b * N;
-    const T* L = latent + b * lbs + u * lld;
-    float x[16], sv[2];
+  const int64_t groups = (rows + RW - 1) / RW;
+  for (int64_t g = (int64_t)blockIdx.x * warps + (threadIdx.x >> 5); g < groups; g += (int64_t)gridDim.x * warps) {
+    float x[RW][16], res[RW][16], sv[RW][2];
 #pragma unroll
-    for (int i = 0; i < 16; ++i) x[i] = to_f(L[lane + 32 * i]);
-    const float e = project(vb, r_sk, x, sv, lane);
-    if (eta && lane == 0) eta[row] = e;
-    if (sketch) {
-      __nv_bfloat16* dst = sketch + row * r_sk;
-      if (lane < r_sk) dst[lane] = __float2bfloat16_rn(sv[0]);
-      if (lane + 32 < r_sk) dst[lane + 32] = __float2bfloat16_rn(sv[1]);
+    for (int q = 0; q < RW; ++q) {
+      const int64_t row = g * RW + q;
+      const int64_t rr = row < rows ? row : rows - 1;  // a short last group repeats a row and stores nothing for it
+      const int64_t b = rr / N, u = rr - b * N;
+      const T* L = latent + b * lbs + u * lld;
+#pragma unroll
+      for (int i = 0; i < 16; ++i) {
+        x[q][i] = to_f(L[lane + 32 * i]);
+        res[q][i] = x[q][i];
+      }
+      sv[q][0] = sv[q][1] = 0.f;
+    }
+    for (int j = 0; j < r_sk; ++j) {
+      const float* v = vb + j * D_LAT + lane;
+      float vv[16];
+#pragma unroll
+      for (int i = 0; i < 16; ++i) vv[i] = v[32 * i];
+      float acc[RW];
+#pragma unroll
+      for (int q = 0; q < RW; ++q) {
+        acc[q] = 0.f;
+#pragma unroll
+        for (int i = 0; i < 16; ++i) acc[q] = fmaf(vv[i], x[q][i], acc[q]);
+      }
+#pragma unroll
+      for (int o = 16; o; o >>= 1) {
+#pragma unroll
+        for (int q = 0; q < RW; ++q) acc[q] += __shfl_xor_sync(0xffffffffu, acc[q], o);
+      }
+#pragma unroll
+      for (int q = 0; q < RW; ++q) {
+        if ((j & 31) == lane) sv[q][j >> 5] = acc[q];
+#pragma unroll
+        for (int i = 0; i < 16; ++i) res[q][i] = fmaf(-acc[q], vv[i], res[q][i]);
+      }
+    }
+#pragma unroll
+    for (int q = 0; q < RW; ++q) {
+      const int64_t row = g * RW + q;
+      float e = 0.f;
+#pragma unroll
+      for (int i = 0; i < 16; ++i) e = fmaf(res[q][i], res[q][i], e);
+      e = sqrtf(warp_sum(e));
+      if (row >= rows) continue;
+      if (eta && lane == 0) eta[row] = e;
+      if (sketch) {
+        __nv_bfloat16* dst = sketch + row * r_sk;
+        if (lane < r_sk) dst[lane] = __float2bfloat16_rn(sv[q][0]);
+        if (lane + 32 < r_sk) dst[lane + 32] = __float2bfloat16_rn(sv[q][1]);
+      }
     }
   }
 }
@@ -302,17 +348,21 @@ cudaError_t launch_build_sketch(const vk_view& v, int r_sk, const float* basis, 
                                 cudaStream_t st) {
   const int64_t rows = (int64_t)v.B * v.N;
   const size_t smem = vb_smem(r_sk);
-  const int grid = (int)std::max<int64_t>(1, std::min<int64_t>((rows + 7) / 8, 2 * sm_count()));
+  constexpr int RW = SKR_RW, NT = SKR_NT;
+  const int64_t groups = (rows + RW - 1) / RW;
+  const int grid = (int)std::max<int64_t>(1, std::min<int64_t>((groups + NT / 32 - 1) / (NT / 32), sm_count()));
   auto* sk = static_cast<__nv_bfloat16*>(sketch);
   cudaError_t e;
   if (v.dtype == VK_BF16) {
-    if ((e = allow_smem(k_sketch_rows<__nv_bfloat16>, smem)) != cudaSuccess) return e;
-    k_sketch_rows<__nv_bfloat16><<<grid, 256, smem, st>>>(rows, v.N, r_sk, static_cast<const __nv_bfloat16*>(v.latent),
-                                                         v.latent_ld, v.latent_bstride, basis, sk, eta);
+    auto kern = k_sketch_rows<__nv_bfloat16, RW, NT>;
+    if ((e = allow_smem(kern, smem)) != cudaSuccess) return e;
+    kern<<<grid, NT, smem, st>>>(rows, v.N, r_sk, static_cast<const __nv_bfloat16*>(v.latent), v.latent_ld,
+                                 v.latent_bstride, basis, sk, eta);
   } else {
-    if ((e = allow_smem(k_sketch_rows<float>, smem)) != cudaSuccess) return e;
-    k_sketch_rows<float><<<grid, 256, smem, st>>>(rows, v.N, r_sk, static_cast<const float*>(v.latent), v.latent_ld,
-                                                 v.latent_bstride, basis, sk, eta);
+    auto kern = k_sketch_rows<float, RW, NT>;
+    if ((e = allow_smem(kern, smem)) != cudaSuccess) return e;
+    kern<<<grid, NT, smem, st>>>(rows, v.N, r_sk, static_cast<const float*>(v.latent), v.latent_ld, v.latent_bstride,
+                                 basis, sk, eta);
   }
   count_launches(1);
   return cudaGetLastError();
