@@ -204,6 +204,26 @@ __device__ void sk_mx(const float* __restrict__ M, const float* X, float* Y, int
   __syncthreads();
 }
 
+// The same product into X itself: each thread keeps its row of M X in registers until every thread is done reading X.
+__device__ void sk_mx_inplace(const float* __restrict__ M, float* X, int r) {
+  const int i = threadIdx.x;
+  float acc[SK_LD];
+#pragma unroll
+  for (int c = 0; c < SK_LD; ++c) acc[c] = 0.f;
+  const float* mi = M + (int64_t)i * D_LAT;
+  for (int k = 0; k < D_LAT; ++k) {
+    const float m = mi[k];
+    const float* xk = X + k * SK_LD;
+#pragma unroll
+    for (int c = 0; c < SK_LD; ++c) acc[c] = fmaf(m, xk[c], acc[c]);
+  }
+  __syncthreads();
+#pragma unroll
+  for (int c = 0; c < SK_LD; ++c)
+    if (c < r) X[i * SK_LD + c] = acc[c];
+  __syncthreads();
+}
+
 // One Cholesky-QR pass: C = S^T S, C = L L^T, X = S L^-T (S and X [512][64], only r columns; X may be S). Returns false
 // when a pivot is not positive (the columns are dependent).
 __device__ bool sk_cholqr(const float* S, float* X, float* C /* [64][65] */, int r, int* bad) {
@@ -274,8 +294,9 @@ __global__ void __launch_bounds__(SKI_THREADS, 1) k_sk_iterate(const float* __re
   __syncthreads();
   bool ok = true;
   for (int it = 0; it <= iters && ok; ++it) {
-    sk_mx(M, X, Y, r);
-    ok = sk_cholqr(Y, X, C, r, &bad) && sk_cholqr(X, X, C, r, &bad);
+    // the product stays in shared memory: both Cholesky-QR passes read their operand from there
+    sk_mx_inplace(M, X, r);
+    ok = sk_cholqr(X, X, C, r, &bad) && sk_cholqr(X, X, C, r, &bad);
   }
   if (!ok) {
     if (t == 0) raise_status(status, VK_ERR_INVALID_ARG);
