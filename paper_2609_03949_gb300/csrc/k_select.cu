@@ -335,17 +335,17 @@ cudaError_t launch_select_dense(int B, int H, int N, const float* scores, const 
 // Threshold from a strided sample of the archive: theta[b,h] = the j-th largest sampled score, so that about
 // j * stride archive rows score >= theta (chosen well above k). The candidate pass then emits only those rows.
 // sample[(b*H + h) * ns + i] is the score of position off + stride * i, in bf16 (theta only steers how many
-// candidates pass; the candidates themselves carry fp32 scores). Up to THETA_R x THETA_THREADS archive samples
-// are held in registers (THETA_R per thread, loaded together); more go through shared memory (ns x 4 bytes).
-// A block of four warps per head, about ten resident per SM: at B = 64, N = 65536, H = 64 the pass takes 21 us,
-// against 34 us with eight warps per head (eight blocks per SM; the blocks are latency-bound, so more of them in
-// flight pays). Measured slower: one warp per head with exact two-pass 8-bit histograms of the 16-bit bf16 keys
+// candidates pass; the candidates themselves carry fp32 scores). Up to THETA_R x NT archive samples are held in
+// registers (THETA_R per thread, loaded together); more go through shared memory (ns x 4 bytes). NT = 128 (four
+// warps per head, about ten blocks resident per SM) while the samples fit, else 256: at B = 64, N = 65536, H = 64
+// the pass takes 21 us with four warps per head against 34 us with eight (the blocks are latency-bound, so more of
+// them in flight pays). Measured slower: one warp per head with exact two-pass 8-bit histograms of the 16-bit bf16 keys
 // (43-47 us: a head's scores share a few exponents, so the first pass's shared-memory atomics pile onto a few
 // buckets), the same with the lanes of a bucket aggregated by match_any (102 us), match_any aggregation in the
 // eight-warp block (48 us), and a binary search over the keys with a block-wide count per step (45 us).
 constexpr int THETA_R = 16;
-constexpr int THETA_THREADS = 128;
-__global__ void __launch_bounds__(THETA_THREADS) k_theta(int ns, int ld, int off, int stride, int lo, int hi, int j,
+template <int NT>
+__global__ void __launch_bounds__(NT) k_theta(int ns, int ld, int off, int stride, int lo, int hi, int j,
                                                         const __nv_bfloat16* __restrict__ sample,
                                                         float* __restrict__ theta, int* __restrict__ zero_cnt) {
   extern __shared__ __align__(16) unsigned char smem[];
@@ -366,37 +366,37 @@ __global__ void __launch_bounds__(THETA_THREADS) k_theta(int ns, int ld, int off
   // two digits below the samples' first differing bit pin the j-th largest to a bucket of 2^-16 of their key
   // range; its lower bound is theta (a little below the exact order statistic: a few more candidates pass)
   uint32_t prefix;
-  if (na <= THETA_R * THETA_THREADS) {
+  if (na <= THETA_R * NT) {
     uint32_t kr[THETA_R];
 #pragma unroll
     for (int r = 0; r < THETA_R; ++r) {
-      const int e = threadIdx.x + r * THETA_THREADS;
+      const int e = threadIdx.x + r * NT;
       kr[r] = fkey(e < na ? __bfloat162float(a[i0 + e]) : 0.f);
     }
     auto each_key = [&](auto f) {
 #pragma unroll
       for (int r = 0; r < THETA_R; ++r)
-        if (threadIdx.x + r * THETA_THREADS < na) f(kr[r]);
+        if (threadIdx.x + r * NT < na) f(kr[r]);
     };
     prefix = radix_kth_desc(each_key, na, (unsigned int)j, hist, scratch, &need_eq, &ties, 2);
   } else {
     uint32_t* keys = reinterpret_cast<uint32_t*>(smem);         // the archive samples' keys
-    for (int i = threadIdx.x; i < na; i += 16 * THETA_THREADS) {
+    for (int i = threadIdx.x; i < na; i += 16 * NT) {
       float v[16];
 #pragma unroll
       for (int r = 0; r < 16; ++r) {
-        const int e = i + r * THETA_THREADS;
+        const int e = i + r * NT;
         v[r] = e < na ? __bfloat162float(a[i0 + e]) : 0.f;
       }
 #pragma unroll
       for (int r = 0; r < 16; ++r) {
-        const int e = i + r * THETA_THREADS;
+        const int e = i + r * NT;
         if (e < na) keys[e] = fkey(v[r]);
       }
     }
     __syncthreads();
     auto each_key = [&](auto f) {
-      for (int i = threadIdx.x; i < na; i += THETA_THREADS) f(keys[i]);
+      for (int i = threadIdx.x; i < na; i += NT) f(keys[i]);
     };
     prefix = radix_kth_desc(each_key, na, (unsigned int)j, hist, scratch, &need_eq, &ties, 2);
   }
@@ -405,12 +405,15 @@ __global__ void __launch_bounds__(THETA_THREADS) k_theta(int ns, int ld, int off
 
 cudaError_t launch_theta(int B, int H, int ns, int ld, int off, int stride, int lo, int hi, int j, const void* sample,
                          float* theta, cudaStream_t st, int* zero_cnt) {
-  // shared memory only when the samples outgrow the registers (na <= ns)
-  const size_t smem = ns > THETA_R * THETA_THREADS ? (size_t)ns * 4 : 0;
-  cudaError_t e = cudaFuncSetAttribute(k_theta, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  // four warps per head while the samples fit their registers (2048), else eight (4096); past that, shared memory
+  const bool small = ns <= THETA_R * 128;
+  const int nt = small ? 128 : 256;
+  const size_t smem = ns > THETA_R * nt ? (size_t)ns * 4 : 0;
+  auto kern = small ? k_theta<128> : k_theta<256>;
+  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
-  k_theta<<<B * H, THETA_THREADS, smem, st>>>(ns, ld, off, stride, lo, hi, j,
-                                             static_cast<const __nv_bfloat16*>(sample), theta, zero_cnt);
+  kern<<<B * H, nt, smem, st>>>(ns, ld, off, stride, lo, hi, j, static_cast<const __nv_bfloat16*>(sample), theta,
+                                zero_cnt);
   count_launches(1);
   return cudaGetLastError();
 }
