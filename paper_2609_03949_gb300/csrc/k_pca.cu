@@ -6,9 +6,9 @@
 //   k_pca_moment  one CTA per SM over a range of 128-row chunks: each chunk's 64 RoPE columns are TMA-loaded once
 //                 and serve as both operands of D += R^T R on tcgen05 (M = N = 64, K = 128 rows, both read
 //                 MN-major from the same tile); the CTA's fp32 sum is added into the fp64 moment at the end.
-//   k_pca_jacobi  one CTA: cyclic Jacobi in fp64 with the round-robin ordering (32 disjoint rotations at a time, 63
-//                 steps per sweep), then the eigenpairs sorted by decreasing eigenvalue, each eigenvector signed so
-//                 that its largest entry is positive.
+//   k_pca_jacobi  one CTA: cyclic Jacobi with the round-robin ordering (32 disjoint rotations at a time, 63 steps per
+//                 sweep), first in fp32, then re-orthonormalised and finished in fp64; then the eigenpairs sorted by
+//                 decreasing eigenvalue, each eigenvector signed so that its largest entry is positive.
 #include <cuda.h>
 #include <cudaTypedefs.h>
 
@@ -162,44 +162,44 @@ __global__ void __launch_bounds__(PC_THREADS, 1) k_pca_moment(const __grid_const
 
 // One CTA of 256 threads: the symmetric 64 x 64 eigenproblem by cyclic Jacobi, 32 disjoint rotations per step.
 constexpr int JC_THREADS = 256;
-__global__ void __launch_bounds__(JC_THREADS) k_pca_jacobi(const double* __restrict__ moment, float* __restrict__ rot,
-                                                         float* __restrict__ eig_out) {
-  extern __shared__ double jc_smem[];                 // A and V, 64 x 65 each (a padded column against bank conflicts)
-  double(*A)[65] = reinterpret_cast<double(*)[65]>(jc_smem);
-  double(*V)[65] = reinterpret_cast<double(*)[65]>(jc_smem + 64 * 65);
-  __shared__ double cs[32][2];
-  __shared__ int pr[32][2];
-  __shared__ double red[JC_THREADS];
-  __shared__ int ord[64];
+constexpr size_t JC_SMEM = 3 * 64 * 65 * sizeof(double) + 2 * 64 * 65 * sizeof(float);
+
+// Sum of x over the block (every thread gets it).
+__device__ __forceinline__ double jc_block_sum(double x, double* red) {
   const int t = threadIdx.x;
-  for (int i = t; i < 64 * 64; i += JC_THREADS) {
-    A[i / 64][i % 64] = moment[i];
-    V[i / 64][i % 64] = (i / 64 == i % 64) ? 1.0 : 0.0;
-  }
-  __syncthreads();
-  double total = 0.0;
-  for (int i = t; i < 64 * 64; i += JC_THREADS) total += A[i / 64][i % 64] * A[i / 64][i % 64];
-  red[t] = total;
+  red[t] = x;
   __syncthreads();
   for (int o = JC_THREADS / 2; o; o >>= 1) {
     if (t < o) red[t] += red[t + o];
     __syncthreads();
   }
-  total = red[0];
+  const double v = red[0];
   __syncthreads();
-  for (int sweep = 0; sweep < 40; ++sweep) {
+  return v;
+}
+
+// Cyclic Jacobi sweeps on A (V accumulates the rotations) in precision T, until the off-diagonal squared norm is at
+// most tol times the total squared norm, or it falls by less than 4x in a sweep once below stall times the total (the
+// rounding floor of precision T), or max_sweeps. Each rotation sets its a_pq, a_qp to zero and its a_pp, a_qq to
+// a_pp - t a_pq, a_qq + t a_pq (t = tan of the angle) instead of taking them from the update products, so that the
+// off-diagonal norm is not held up by their rounding.
+template <typename T>
+__device__ void jc_sweeps(T (*A)[65], T (*V)[65], double* red, double tol, double stall, int max_sweeps) {
+  __shared__ T cs[32][2];
+  __shared__ T dg[32][2];
+  __shared__ int pr[32][2];
+  const int t = threadIdx.x;
+  double total = 0.0;
+  for (int i = t; i < 64 * 64; i += JC_THREADS) total += (double)A[i / 64][i % 64] * (double)A[i / 64][i % 64];
+  total = jc_block_sum(total, red);
+  double prev = 0.0;
+  for (int sweep = 0; sweep < max_sweeps; ++sweep) {
     double off = 0.0;
     for (int i = t; i < 64 * 64; i += JC_THREADS)
-      if (i / 64 != i % 64) off += A[i / 64][i % 64] * A[i / 64][i % 64];
-    red[t] = off;
-    __syncthreads();
-    for (int o = JC_THREADS / 2; o; o >>= 1) {
-      if (t < o) red[t] += red[t + o];
-      __syncthreads();
-    }
-    const bool converged = red[0] <= 1e-30 * total;
-    __syncthreads();
-    if (converged) break;
+      if (i / 64 != i % 64) off += (double)A[i / 64][i % 64] * (double)A[i / 64][i % 64];
+    off = jc_block_sum(off, red);
+    if (off <= tol * total || (sweep > 0 && off <= stall * total && off > 0.25 * prev)) break;
+    prev = off;
     for (int step = 0; step < 63; ++step) {
       if (t < 32) {
         // round-robin: index 63 meets step; the others pair up symmetrically around it
@@ -207,43 +207,114 @@ __global__ void __launch_bounds__(JC_THREADS) k_pca_jacobi(const double* __restr
         if (p > q) { const int x = p; p = q; q = x; }
         pr[t][0] = p;
         pr[t][1] = q;
-        const double apq = A[p][q];
-        double c = 1.0, s = 0.0;
-        if (apq != 0.0) {
-          const double theta = (A[q][q] - A[p][p]) / (2.0 * apq);
-          const double tt = (theta >= 0.0 ? 1.0 : -1.0) / (fabs(theta) + sqrt(theta * theta + 1.0));
-          c = 1.0 / sqrt(tt * tt + 1.0);
-          s = tt * c;
+        const T apq = A[p][q], app = A[p][p], aqq = A[q][q];
+        T c = T(1), sn = T(0), tt = T(0);
+        if (apq != T(0)) {
+          const T theta = (aqq - app) / (T(2) * apq);
+          tt = (theta >= T(0) ? T(1) : T(-1)) / (fabs(theta) + sqrt(theta * theta + T(1)));
+          c = T(1) / sqrt(tt * tt + T(1));
+          sn = tt * c;
         }
         cs[t][0] = c;
-        cs[t][1] = s;
+        cs[t][1] = sn;
+        dg[t][0] = app - tt * apq;
+        dg[t][1] = aqq + tt * apq;
       }
       __syncthreads();
       // rows p, q of every pair: A <- J^T A
       for (int e = t; e < 32 * 64; e += JC_THREADS) {
         const int k = e & 63, w = e >> 6;
         const int p = pr[w][0], q = pr[w][1];
-        const double c = cs[w][0], s = cs[w][1];
-        const double apk = A[p][k], aqk = A[q][k];
-        A[p][k] = c * apk - s * aqk;
-        A[q][k] = s * apk + c * aqk;
+        const T c = cs[w][0], sn = cs[w][1];
+        const T apk = A[p][k], aqk = A[q][k];
+        A[p][k] = c * apk - sn * aqk;
+        A[q][k] = sn * apk + c * aqk;
       }
       __syncthreads();
       // columns p, q: A <- A J, V <- V J
       for (int e = t; e < 32 * 64; e += JC_THREADS) {
         const int k = e & 63, w = e >> 6;
         const int p = pr[w][0], q = pr[w][1];
-        const double c = cs[w][0], s = cs[w][1];
-        const double akp = A[k][p], akq = A[k][q];
-        A[k][p] = c * akp - s * akq;
-        A[k][q] = s * akp + c * akq;
-        const double vkp = V[k][p], vkq = V[k][q];
-        V[k][p] = c * vkp - s * vkq;
-        V[k][q] = s * vkp + c * vkq;
+        const T c = cs[w][0], sn = cs[w][1];
+        const T akp = A[k][p], akq = A[k][q];
+        T np = c * akp - sn * akq, nq = sn * akp + c * akq;
+        if (k == p) {
+          np = dg[w][0];
+          nq = T(0);
+        } else if (k == q) {
+          np = T(0);
+          nq = dg[w][1];
+        }
+        A[k][p] = np;
+        A[k][q] = nq;
+        const T vkp = V[k][p], vkq = V[k][q];
+        V[k][p] = c * vkp - sn * vkq;
+        V[k][q] = sn * vkp + c * vkq;
       }
       __syncthreads();
     }
   }
+}
+
+// The sweeps run first in fp32, many times faster than fp64 on this part, down to an off-diagonal norm at fp32's
+// level; the fp32 rotations are then re-orthonormalised in fp64 (classical Gram-Schmidt, twice), the moment is
+// projected on them in fp64, and fp64 sweeps finish from there to the threshold of a pure fp64 solve.
+__global__ void __launch_bounds__(JC_THREADS) k_pca_jacobi(const double* __restrict__ moment, float* __restrict__ rot,
+                                                         float* __restrict__ eig_out) {
+  extern __shared__ double jc_smem[];                 // padded 64 x 65 arrays against bank conflicts
+  double(*A)[65] = reinterpret_cast<double(*)[65]>(jc_smem);                // the moment, then V^T M V
+  double(*V)[65] = reinterpret_cast<double(*)[65]>(jc_smem + 64 * 65);      // the rotations
+  double(*W)[65] = reinterpret_cast<double(*)[65]>(jc_smem + 2 * 64 * 65);  // M V
+  float(*Af)[65] = reinterpret_cast<float(*)[65]>(jc_smem + 3 * 64 * 65);
+  float(*Vf)[65] = Af + 64;
+  __shared__ double red[JC_THREADS];
+  __shared__ double coef[64];
+  __shared__ int ord[64];
+  const int t = threadIdx.x;
+  for (int i = t; i < 64 * 64; i += JC_THREADS) {
+    const double m = moment[i];
+    A[i / 64][i % 64] = m;
+    Af[i / 64][i % 64] = (float)m;
+    Vf[i / 64][i % 64] = (i / 64 == i % 64) ? 1.f : 0.f;
+  }
+  __syncthreads();
+  jc_sweeps<float>(Af, Vf, red, 1e-12, 1e-7, 40);
+  for (int i = t; i < 64 * 64; i += JC_THREADS) V[i / 64][i % 64] = (double)Vf[i / 64][i % 64];
+  __syncthreads();
+  for (int c = 0; c < 64; ++c) {
+    for (int pass = 0; pass < 2; ++pass) {
+      if (t < c) {
+        double d = 0.0;
+        for (int k = 0; k < 64; ++k) d = fma(V[k][t], V[k][c], d);
+        coef[t] = d;
+      }
+      __syncthreads();
+      if (t < 64) {
+        double x = V[t][c];
+        for (int d = 0; d < c; ++d) x = fma(-coef[d], V[t][d], x);
+        V[t][c] = x;
+      }
+      __syncthreads();
+    }
+    const double nn = jc_block_sum(t < 64 ? V[t][c] * V[t][c] : 0.0, red);
+    if (t < 64) V[t][c] /= sqrt(nn);
+    __syncthreads();
+  }
+  for (int e = t; e < 64 * 64; e += JC_THREADS) {    // W = M V
+    const int i = e / 64, j = e % 64;
+    double x = 0.0;
+    for (int k = 0; k < 64; ++k) x = fma(A[i][k], V[k][j], x);
+    W[i][j] = x;
+  }
+  __syncthreads();
+  for (int e = t; e < 64 * 64; e += JC_THREADS) {    // A = V^T W
+    const int i = e / 64, j = e % 64;
+    double x = 0.0;
+    for (int k = 0; k < 64; ++k) x = fma(V[k][i], W[k][j], x);
+    A[i][j] = x;
+  }
+  __syncthreads();
+  jc_sweeps<double>(A, V, red, 1e-30, 1e-24, 40);
   if (t == 0) {
     for (int i = 0; i < 64; ++i) ord[i] = i;
     for (int i = 1; i < 64; ++i) {
@@ -309,7 +380,7 @@ cudaError_t launch_pca_basis(const vk_view& v, float* rot, float* eig, void* ws,
   e = cudaFuncSetAttribute(k_pca_moment, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
   k_pca_moment<<<grid, PC_THREADS, smem, st>>>(rmap, a);
-  const size_t jsmem = 2 * 64 * 65 * sizeof(double);
+  const size_t jsmem = JC_SMEM;
   e = cudaFuncSetAttribute(k_pca_jacobi, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)jsmem);
   if (e != cudaSuccess) return e;
   k_pca_jacobi<<<1, JC_THREADS, jsmem, st>>>(moment, rot, eig);
@@ -318,7 +389,7 @@ cudaError_t launch_pca_basis(const vk_view& v, float* rot, float* eig, void* ws,
 }
 
 cudaError_t launch_sym_eig64(const double* A, float* vec, float* eig, cudaStream_t st) {
-  const size_t jsmem = 2 * 64 * 65 * sizeof(double);
+  const size_t jsmem = JC_SMEM;
   cudaError_t e = cudaFuncSetAttribute(k_pca_jacobi, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)jsmem);
   if (e != cudaSuccess) return e;
   k_pca_jacobi<<<1, JC_THREADS, jsmem, st>>>(A, vec, eig);
