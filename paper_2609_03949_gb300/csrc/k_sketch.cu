@@ -182,92 +182,170 @@ __global__ void __launch_bounds__(256) k_sk_moment(int64_t n, const T* __restric
 }
 
 constexpr int SKI_THREADS = 512;                   // one row of X per thread
-constexpr int SK_LD = 64;                             // row stride of X and Y (r_sk <= 64)
+constexpr int SK_LD = 64;                             // row length of X and Y (r_sk <= 64)
+constexpr int SK_XLD = 68;                            // row stride of X and of L's rows in shared memory
 
-// Y[i][c] = sum_k M[i][k] X[k][c] for c < r (thread t: row t; the warp reads one X row at a time, a broadcast);
-// Y global.
+// X [512][64] sits in shared memory with rows 68 floats apart: chunk q (16 bytes) of row i is 16-byte unit 17 i + q,
+// so threads of a quarter-warp that read or write their own rows chunk by chunk meet distinct banks, and a warp
+// reading one row (a broadcast) reads 16 contiguous chunks. The rows of the Cholesky factor L use the same stride.
+__device__ __forceinline__ int sx_chunk(int i, int q) { return i * (SK_XLD / 4) + q; }
+__device__ __forceinline__ int sx(int i, int c) { return i * SK_XLD + c; }
+
+// acc[c] = sum_k M[i][k] X[k][c] for thread i's row, k ascending. M is symmetric (its tiles (a, b) and (b, a) sum the
+// same products in the same order), so column i is read: one coalesced load per k for the warp. The warp reads one
+// X row at a time, a broadcast.
+__device__ __forceinline__ void sk_mx_row(const float* __restrict__ M, const float* X, float (&acc)[SK_LD]) {
+  const int i = threadIdx.x;
+#pragma unroll
+  for (int c = 0; c < SK_LD; ++c) acc[c] = 0.f;
+  const float4* X4 = reinterpret_cast<const float4*>(X);
+  // M's entries are loaded four k ahead of their use (each k is a new line for the warp)
+  float m0 = M[i], m1 = M[D_LAT + i], m2 = M[2 * D_LAT + i], m3 = M[3 * D_LAT + i];
+#pragma unroll 1
+  for (int k = 0; k < D_LAT; ++k) {
+    const float m = m0;
+    m0 = m1;
+    m1 = m2;
+    m2 = m3;
+    m3 = k + 4 < D_LAT ? M[(int64_t)(k + 4) * D_LAT + i] : 0.f;
+    const float4* xk = X4 + sx_chunk(k, 0);
+#pragma unroll
+    for (int q = 0; q < SK_LD / 4; ++q) {
+      const float4 x = xk[q];
+      acc[4 * q + 0] = fmaf(m, x.x, acc[4 * q + 0]);
+      acc[4 * q + 1] = fmaf(m, x.y, acc[4 * q + 1]);
+      acc[4 * q + 2] = fmaf(m, x.z, acc[4 * q + 2]);
+      acc[4 * q + 3] = fmaf(m, x.w, acc[4 * q + 3]);
+    }
+  }
+}
+
+// Y = M X (columns c < r) into global memory, row-major [512][64].
 __device__ void sk_mx(const float* __restrict__ M, const float* X, float* Y, int r) {
   const int i = threadIdx.x;
   float acc[SK_LD];
-#pragma unroll
-  for (int c = 0; c < SK_LD; ++c) acc[c] = 0.f;
-  const float* mi = M + (int64_t)i * D_LAT;
-  for (int k = 0; k < D_LAT; ++k) {
-    const float m = mi[k];
-    const float* xk = X + k * SK_LD;
-#pragma unroll
-    for (int c = 0; c < SK_LD; ++c) acc[c] = fmaf(m, xk[c], acc[c]);
-  }
+  sk_mx_row(M, X, acc);
 #pragma unroll
   for (int c = 0; c < SK_LD; ++c)
     if (c < r) Y[i * SK_LD + c] = acc[c];
   __syncthreads();
 }
 
-// The same product into X itself: each thread keeps its row of M X in registers until every thread is done reading X.
+// The same product into X itself: each thread keeps its row of M X in registers until every thread is done reading X
+// (r is a multiple of 16, so whole chunks are written).
 __device__ void sk_mx_inplace(const float* __restrict__ M, float* X, int r) {
   const int i = threadIdx.x;
   float acc[SK_LD];
-#pragma unroll
-  for (int c = 0; c < SK_LD; ++c) acc[c] = 0.f;
-  const float* mi = M + (int64_t)i * D_LAT;
-  for (int k = 0; k < D_LAT; ++k) {
-    const float m = mi[k];
-    const float* xk = X + k * SK_LD;
-#pragma unroll
-    for (int c = 0; c < SK_LD; ++c) acc[c] = fmaf(m, xk[c], acc[c]);
-  }
+  sk_mx_row(M, X, acc);
   __syncthreads();
+  float4* X4 = reinterpret_cast<float4*>(X);
 #pragma unroll
-  for (int c = 0; c < SK_LD; ++c)
-    if (c < r) X[i * SK_LD + c] = acc[c];
+  for (int q = 0; q < SK_LD / 4; ++q)
+    if (4 * q < r) X4[sx_chunk(i, q)] = make_float4(acc[4 * q], acc[4 * q + 1], acc[4 * q + 2], acc[4 * q + 3]);
   __syncthreads();
 }
 
-// One Cholesky-QR pass: C = S^T S, C = L L^T, X = S L^-T (S and X [512][64], only r columns; X may be S). Returns false
-// when a pivot is not positive (the columns are dependent).
-__device__ bool sk_cholqr(const float* S, float* X, float* C /* [64][65] */, int r, int* bad) {
+// Shared scratch of a Cholesky-QR pass: the Gram matrix C [64][65] (lower triangle), the factor L twice (rows at the
+// stride of X for the substitution, columns contiguous for the trailing update) and its diagonal.
+struct SkChol {
+  float* C;
+  float* Lr;
+  float* Lc;
+  float* Dg;
+};
+
+// One Cholesky-QR pass on X in place, first r columns: C = X^T X, C = L L^T, X <- X L^-T. Returns false when a pivot
+// is not positive (the columns are dependent). Each entry of C sums over the rows in ascending order; column k of L
+// is C's column k over the square root of the pivot, and the trailing update subtracts l_ik l_jk; each row of
+// X L^-T is solved by forward substitution, k ascending.
+__device__ bool sk_cholqr(float* X, const SkChol& w, int r, int* bad) {
   const int t = threadIdx.x;
-  for (int e = t; e < r * r; e += SKI_THREADS) {
-    const int a = e / r, b = e - a * r;
-    if (b > a) continue;
-    float acc = 0.f;
-    for (int i = 0; i < D_LAT; ++i) acc = fmaf(S[i * SK_LD + a], S[i * SK_LD + b], acc);
-    C[a * 65 + b] = acc;
+  float* C = w.C;
+  // Gram matrix: thread t takes rows a0, a0 + 1 and columns b0 .. b0 + 3 of C, tiles wholly above the diagonal idle
+  {
+    const int a0 = (t >> 4) * 2, b0 = (t & 15) * 4;
+    if (b0 <= a0 + 1 && a0 < r && b0 < r) {
+      float acc[2][4];
+#pragma unroll
+      for (int u = 0; u < 2; ++u)
+#pragma unroll
+        for (int v = 0; v < 4; ++v) acc[u][v] = 0.f;
+      const float4* X4 = reinterpret_cast<const float4*>(X);
+#pragma unroll 4
+      for (int i = 0; i < D_LAT; ++i) {
+        const float4 xb = X4[sx_chunk(i, b0 >> 2)];
+        const float2 xa = *reinterpret_cast<const float2*>(X + sx(i, a0));
+        const float xav[2] = {xa.x, xa.y}, xbv[4] = {xb.x, xb.y, xb.z, xb.w};
+#pragma unroll
+        for (int u = 0; u < 2; ++u)
+#pragma unroll
+          for (int v = 0; v < 4; ++v) acc[u][v] = fmaf(xav[u], xbv[v], acc[u][v]);
+      }
+#pragma unroll
+      for (int u = 0; u < 2; ++u)
+#pragma unroll
+        for (int v = 0; v < 4; ++v)
+          if (b0 + v <= a0 + u) C[(a0 + u) * 65 + b0 + v] = acc[u][v];
+    }
   }
   if (t == 0) *bad = 0;
   __syncthreads();
+  // right-looking Cholesky, two barriers per column: thread t updates row t & 63, columns (t >> 6) + 8 m
+  const int ci = t & 63, cj0 = t >> 6;
   for (int k = 0; k < r; ++k) {
+    const float d = C[k * 65 + k];
+    const float dk = d > 0.f ? sqrtf(d) : 1.f;
     if (t == 0) {
-      const float d = C[k * 65 + k];
       if (!(d > 0.f)) *bad = 1;
-      C[k * 65 + k] = d > 0.f ? sqrtf(d) : 1.f;
+      w.Dg[k] = dk;
+    }
+    if (t > k && t < r) {
+      const float l = C[t * 65 + k] / dk;
+      w.Lc[k * 64 + t] = l;
+      w.Lr[sx(t, k)] = l;
     }
     __syncthreads();
-    const float dk = C[k * 65 + k];
-    for (int i = k + 1 + t; i < r; i += SKI_THREADS) C[i * 65 + k] /= dk;
-    __syncthreads();
-    const int m = r - k - 1;
-    for (int e = t; e < m * m; e += SKI_THREADS) {
-      const int i = k + 1 + e / m, j = k + 1 + e % m;
-      if (j <= i) C[i * 65 + j] = fmaf(-C[i * 65 + k], C[j * 65 + k], C[i * 65 + j]);
+    if (ci > k && ci < r) {
+      const float lik = w.Lc[k * 64 + ci];
+#pragma unroll
+      for (int m = 0; m < 8; ++m) {
+        const int j = cj0 + 8 * m;
+        if (j > k && j <= ci) C[ci * 65 + j] = fmaf(-lik, w.Lc[k * 64 + j], C[ci * 65 + j]);
+      }
     }
     __syncthreads();
   }
+  // row t: x L^T = s by forward substitution over the columns (x in registers: every index below is a constant)
   {
-    // row t: x L^T = s, forward substitution over the columns
+    float4* X4 = reinterpret_cast<float4*>(X);
+    const float4* L4 = reinterpret_cast<const float4*>(w.Lr);
     float x[SK_LD];
+#pragma unroll
+    for (int q = 0; q < SK_LD / 4; ++q) {
+      const float4 v = 4 * q < r ? X4[sx_chunk(t, q)] : make_float4(0.f, 0.f, 0.f, 0.f);
+      x[4 * q] = v.x;
+      x[4 * q + 1] = v.y;
+      x[4 * q + 2] = v.z;
+      x[4 * q + 3] = v.w;
+    }
 #pragma unroll
     for (int j = 0; j < SK_LD; ++j) {
       if (j < r) {
-        float acc = S[t * SK_LD + j];
-        for (int k = 0; k < j; ++k) acc = fmaf(-x[k], C[j * 65 + k], acc);
-        x[j] = acc / C[j * 65 + j];
+        float acc = x[j];
+#pragma unroll
+        for (int q = 0; q < (j + 3) / 4; ++q) {
+          const float4 l = L4[sx_chunk(j, q)];
+          const float lv[4] = {l.x, l.y, l.z, l.w};
+#pragma unroll
+          for (int u = 0; u < 4; ++u)
+            if (4 * q + u < j) acc = fmaf(-x[4 * q + u], lv[u], acc);
+        }
+        x[j] = acc / w.Dg[j];
       }
     }
 #pragma unroll
-    for (int j = 0; j < SK_LD; ++j)
-      if (j < r) X[t * SK_LD + j] = x[j];
+    for (int q = 0; q < SK_LD / 4; ++q)
+      if (4 * q < r) X4[sx_chunk(t, q)] = make_float4(x[4 * q], x[4 * q + 1], x[4 * q + 2], x[4 * q + 3]);
   }
   __syncthreads();
   return *bad == 0;
@@ -275,13 +353,17 @@ __device__ bool sk_cholqr(const float* S, float* X, float* C /* [64][65] */, int
 
 // Orthogonal iteration on one CTA: X0 = orth(M G) with G a fixed +-1 pattern, then iters steps X <- orth(M X)
 // (two Cholesky-QR passes each), then the Rayleigh-Ritz matrix R = X^T M X into Bout [64][64] fp64 (zero past r) and
-// X into Xout [512][64].
+// X into Xout [512][64] (row-major).
 __global__ void __launch_bounds__(SKI_THREADS, 1) k_sk_iterate(const float* __restrict__ M, int r, int iters,
                                                              float* __restrict__ Y, float* __restrict__ Xout,
                                                              double* __restrict__ Bout, int* __restrict__ status) {
-  extern __shared__ float smf[];
-  float* X = smf;                                     // [512][64]
-  float* C = X + D_LAT * SK_LD;                       // [64][65]
+  extern __shared__ __align__(16) float smf[];
+  float* X = smf;                                     // [512][64], rows SK_XLD apart
+  SkChol w;
+  w.C = X + D_LAT * SK_XLD;                           // [64][65]
+  w.Lr = w.C + 64 * 65;                               // [64][64], rows SK_XLD apart
+  w.Lc = w.Lr + 64 * SK_XLD;                          // [64][64], L^T row-major
+  w.Dg = w.Lc + 64 * 64;                              // [64]
   __shared__ int bad;
   const int t = threadIdx.x;
   for (int e = t; e < D_LAT * SK_LD; e += SKI_THREADS) {
@@ -289,14 +371,14 @@ __global__ void __launch_bounds__(SKI_THREADS, 1) k_sk_iterate(const float* __re
     h ^= h >> 15;
     h *= 2246822519u;
     h ^= h >> 13;
-    X[e] = (h & 1u) ? 1.f : -1.f;
+    X[sx(e >> 6, e & 63)] = (h & 1u) ? 1.f : -1.f;
   }
   __syncthreads();
   bool ok = true;
   for (int it = 0; it <= iters && ok; ++it) {
     // the product stays in shared memory: both Cholesky-QR passes read their operand from there
     sk_mx_inplace(M, X, r);
-    ok = sk_cholqr(X, X, C, r, &bad) && sk_cholqr(X, X, C, r, &bad);
+    ok = sk_cholqr(X, w, r, &bad) && sk_cholqr(X, w, r, &bad);
   }
   if (!ok) {
     if (t == 0) raise_status(status, VK_ERR_INVALID_ARG);
@@ -308,12 +390,12 @@ __global__ void __launch_bounds__(SKI_THREADS, 1) k_sk_iterate(const float* __re
     double v = 0.0;
     if (a < r && b < r) {
       float acc = 0.f;
-      for (int i = 0; i < D_LAT; ++i) acc = fmaf(X[i * SK_LD + a], Y[i * SK_LD + b], acc);
+      for (int i = 0; i < D_LAT; ++i) acc = fmaf(X[sx(i, a)], Y[i * SK_LD + b], acc);
       v = acc;
     }
     Bout[e] = v;
   }
-  for (int e = t; e < D_LAT * SK_LD; e += SKI_THREADS) Xout[e] = X[e];
+  for (int e = t; e < D_LAT * SK_LD; e += SKI_THREADS) Xout[e] = X[sx(e >> 6, e & 63)];
 }
 
 // basis row i = sum_j W[i][j] X[:, j] (W: the Ritz rotation's rows, by decreasing eigenvalue), signed so that its
@@ -445,7 +527,7 @@ cudaError_t launch_sketch_basis(const void* queries, int dtype, int64_t n, int r
     k_sk_moment<__nv_bfloat16><<<mg, 256, 0, st>>>(n, static_cast<const __nv_bfloat16*>(queries), M);
   else
     k_sk_moment<float><<<mg, 256, 0, st>>>(n, static_cast<const float*>(queries), M);
-  const size_t ismem = sizeof(float) * (D_LAT * SK_LD + 64 * 65);
+  const size_t ismem = sizeof(float) * (D_LAT * SK_XLD + 64 * 65 + 64 * SK_XLD + 64 * 64 + 64);
   if ((e = allow_smem(k_sk_iterate, ismem)) != cudaSuccess) return e;
   k_sk_iterate<<<1, SKI_THREADS, ismem, st>>>(M, r_sk, SK_ITERS, Y, X, Bm, status);
   if ((e = launch_sym_eig64(Bm, W, E, st)) != cudaSuccess) return e;
