@@ -239,7 +239,8 @@ int vk_conformal_z(const vk_view* view, const vk_params* params, const vk_index*
  * sequence of the view of K_u K_u^T, by decreasing eigenvalue, each signed so that its largest entry is positive;
  * usable as index->rot and as vk_build_digest's rot64, so that the width-r digest keeps the most branch energy.
  * eig [64] fp32 (device, may be NULL): the eigenvalues. M is accumulated on the tensor cores (bf16 rows, fp32 per
- * CTA, fp64 across CTAs); the 64 x 64 eigenproblem is solved by cyclic Jacobi in fp64. bf16 caches only. */
+ * CTA, fp64 across CTAs); the 64 x 64 eigenproblem is solved by cyclic Jacobi, sweeps in fp32 finished by sweeps in
+ * fp64 on the fp64 projection of M onto the re-orthonormalised fp32 eigenvectors. bf16 caches only. */
 size_t vk_pca_workspace_bytes(void);
 int vk_pca_basis(const vk_view* view, float* rot, float* eig, void* ws, size_t ws_bytes, void* stream);
 

@@ -9,7 +9,7 @@
 //                   tensor-core trigger loads) and rho = |qc - V^T p|, the certificate's query norm.
 //   basis from the context's queries (V from the prefix queries): the second moment M = sum_i q_i q_i^T in fp32
 //   (k_sk_moment), orthogonal iteration X <- orth(M X) on one CTA with two Cholesky-QR passes per step
-//   (k_sk_iterate), the Rayleigh-Ritz matrix X^T M X solved by the 64 x 64 fp64 Jacobi kernel of the PCA basis,
+//   (k_sk_iterate), the Rayleigh-Ritz matrix X^T M X solved by the 64 x 64 Jacobi kernel of the PCA basis (fp64 result),
 //   and the rotation of X into the Ritz vectors with the sign rule (entry of largest magnitude positive, ties the
 //   smaller index) in k_sk_finish.
 #include <algorithm>
