@@ -206,6 +206,18 @@ class ClockSampler:
                 "reasons": reasons, "samples": len(use), "in_timed_region": bool(inside)}
 
 
+def clocks_rejected(clk: dict) -> bool:
+    """True when a timed region's clock record rules its number out: a hardware or thermal slowdown was active, or
+    the SM clock sat well below its maximum with no reason given (a clock lock left by someone else). sw_power_cap
+    alone is kept: it is normal under a long dense load."""
+    bad = {"hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown"}
+    reasons = set(clk.get("reasons") or [])
+    if reasons & bad:
+        return True
+    mhz, top = clk.get("sm_mhz"), clk.get("sm_max_mhz")
+    return bool(mhz and top and mhz < 0.8 * top and not (reasons - {"nvidia-smi unavailable", "no samples"}))
+
+
 # ------------------------------------------------------------------------------------------------ bytes
 def union_rows(idx: torch.Tensor, count: torch.Tensor, n: int) -> int:
     """Distinct rows attended per sequence, summed over the batch (ids < 0 or past count are ignored)."""
@@ -462,35 +474,43 @@ def run_native(args):
     esz = 2 if w.dtype == "bf16" else 4
     # a cache that L2 could hold is evicted between steps by a 512 MB write outside the steps' events
     flush = torch.empty(512 << 20, dtype=torch.uint8, device=dev) if B * N * 576 * esz < 4 * 129e6 else None
-    clocks = ClockSampler(local)
-    clocks.start()
-    time.sleep(0.3)
     t_start = torch.cuda.Event(enable_timing=True)
     t_end = torch.cuda.Event(enable_timing=True)
-    if pg:
-        pg.barrier()
-    torch.cuda.synchronize()
-    # pass 1, the headline: the steps alone (no stage events), bracketed by events on the launching stream;
-    # with an L2 flush between steps, each step is bracketed by its own pair so that the flushes stay outside
-    launches0 = vk.vk_profile_launches()
-    clocks.mark(True)
-    t_start.record(stream)
-    for sb, se in step_brackets:
+
+    def headline_pass():
+        # the steps alone (no stage events), bracketed by events on the launching stream; with an L2 flush between
+        # steps, each step is bracketed by its own pair so that the flushes stay outside
+        clocks = ClockSampler(local)
+        clocks.start()
+        time.sleep(0.3)
+        if pg:
+            pg.barrier()
+        torch.cuda.synchronize()
+        launches0 = vk.vk_profile_launches()
+        clocks.mark(True)
+        t_start.record(stream)
+        for sb, se in step_brackets:
+            if flush is not None:
+                flush.fill_(1)
+                sb.record(stream)
+            buf.run(view, params, index)
+            if flush is not None:
+                se.record(stream)
+        t_end.record(stream)
+        torch.cuda.synchronize()
+        clocks.mark(False)
+        n_launch = vk.vk_profile_launches() - launches0
+        ms = t_start.elapsed_time(t_end)
         if flush is not None:
-            flush.fill_(1)
-            sb.record(stream)
-        buf.run(view, params, index)
-        if flush is not None:
-            se.record(stream)
-    t_end.record(stream)
-    torch.cuda.synchronize()
-    clocks.mark(False)
-    launches = vk.vk_profile_launches() - launches0
-    elapsed_ms = t_start.elapsed_time(t_end)
-    if flush is not None:
-        elapsed_ms = sum(sb.elapsed_time(se) for sb, se in step_brackets)
-    elapsed_ms = max_over_ranks(elapsed_ms, pg, dev)
-    clk = clocks.stop()
+            ms = sum(sb.elapsed_time(se) for sb, se in step_brackets)
+        return max_over_ranks(ms, pg, dev), n_launch, clocks.stop()
+
+    # pass 1, the headline; taken once more if any rank's clock record rules it out
+    elapsed_ms, launches, clk = headline_pass()
+    if max_over_ranks(1.0 if clocks_rejected(clk) else 0.0, pg, dev) > 0:
+        first = clk
+        elapsed_ms, launches, clk = headline_pass()
+        clk = dict(clk, remeasured_after=first)
     ms_step = elapsed_ms / args.steps
     assert vk.vk_poll_status(buf.ws) == vk.VK_OK
     # pass 2, the breakdown: the same steps again, each recording its stage boundaries into its own events
