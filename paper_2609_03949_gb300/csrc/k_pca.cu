@@ -178,6 +178,20 @@ __device__ __forceinline__ double jc_block_sum(double x, double* red) {
   return v;
 }
 
+// Largest x over the block (every thread gets it).
+__device__ __forceinline__ double jc_block_max(double x, double* red) {
+  const int t = threadIdx.x;
+  red[t] = x;
+  __syncthreads();
+  for (int o = JC_THREADS / 2; o; o >>= 1) {
+    if (t < o) red[t] = fmax(red[t], red[t + o]);
+    __syncthreads();
+  }
+  const double v = red[0];
+  __syncthreads();
+  return v;
+}
+
 // Cyclic Jacobi sweeps on A (V accumulates the rotations) in precision T, until the off-diagonal squared norm is at
 // most tol times the total squared norm, or it falls by less than 4x in a sweep once below stall times the total (the
 // rounding floor of precision T), or max_sweeps. Each rotation sets its a_pq, a_qp to zero and its a_pp, a_qq to
@@ -271,10 +285,16 @@ __global__ void __launch_bounds__(JC_THREADS) k_pca_jacobi(const double* __restr
   __shared__ double coef[64];
   __shared__ int ord[64];
   const int t = threadIdx.x;
+  // the fp32 copy is scaled by a power of two that brings the largest entry near 1, so that it neither overflows nor
+  // underflows whatever the data's scale; the scaling is exact and the rotations do not depend on it
+  double amax = 0.0;
+  for (int i = t; i < 64 * 64; i += JC_THREADS) amax = fmax(amax, fabs(moment[i]));
+  amax = jc_block_max(amax, red);
+  const double sc = amax > 0.0 && isfinite(amax) ? ldexp(1.0, -ilogb(amax)) : 1.0;
   for (int i = t; i < 64 * 64; i += JC_THREADS) {
     const double m = moment[i];
     A[i / 64][i % 64] = m;
-    Af[i / 64][i % 64] = (float)m;
+    Af[i / 64][i % 64] = (float)(m * sc);
     Vf[i / 64][i % 64] = (i / 64 == i % 64) ? 1.f : 0.f;
   }
   __syncthreads();
