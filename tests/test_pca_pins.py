@@ -80,7 +80,33 @@ def pin_pca_energy_optimal():
             assert e_pca >= float(((K @ O.T)[:, :r] ** 2).sum())
 
 
-PINS = [pin_sym_eig_matches_numpy, pin_second_moment_matmul, pin_pca_known_axes, pin_pca_energy_optimal]
+def pin_sym_eig_spread_repeated_zero():
+    # a spectrum over seven decades, a spectrum of three repeated values, and the zero matrix, each in a Haar frame:
+    # eigenvalues to the rounding of the largest; for a repeated value only its eigenspace is fixed, so the
+    # eigenvectors' projector is compared with the frame's
+    Q = datagen.haar_orthogonal(11)
+    spread = np.logspace(3, -4, 64)
+    eig, vec = oracle.sym_eig((Q.T * spread) @ Q)
+    np.testing.assert_allclose(eig, spread, rtol=1e-9, atol=1e-12 * spread[0])
+    np.testing.assert_allclose(vec @ vec.T, np.eye(64), atol=1e-12)
+    sep = np.abs(vec @ Q.T)                            # row i against the frame's row i: |cos| = 1 where separated
+    np.testing.assert_allclose(np.diag(sep)[:40], 1.0, atol=1e-9)
+    rep = np.repeat([5.0, 2.0, 1.0], [16, 16, 32])
+    eig, vec = oracle.sym_eig((Q.T * rep) @ Q)
+    np.testing.assert_allclose(eig, rep, rtol=1e-12)
+    for lo, hi_ in ((0, 16), (16, 32), (32, 64)):
+        P_got = vec[lo:hi_].T @ vec[lo:hi_]
+        P_want = Q[lo:hi_].T @ Q[lo:hi_]
+        np.testing.assert_allclose(P_got, P_want, atol=1e-10)
+    eig, vec = oracle.sym_eig(np.zeros((64, 64)))
+    assert np.all(eig == 0.0)
+    np.testing.assert_allclose(vec @ vec.T, np.eye(64), atol=1e-12)
+    big = np.abs(vec).argmax(axis=1)
+    assert np.all(vec[np.arange(64), big] > 0)
+
+
+PINS = [pin_sym_eig_matches_numpy, pin_sym_eig_spread_repeated_zero, pin_second_moment_matmul, pin_pca_known_axes,
+        pin_pca_energy_optimal]
 
 
 @pytest.mark.parametrize("pin", PINS, ids=lambda f: f.__name__)
