@@ -155,7 +155,11 @@ size_t vk_sketch_basis_workspace_bytes(int64_t n, int32_t r_sk);
  * its entry of largest magnitude is positive, as the rows of basis [r_sk, 512] fp32, and their eigenvalues in eig
  * [r_sk] fp32 (device; eig may be NULL). queries: [n, 512] contiguous, dtype a vk_dtype (device). r_sk in {16, 32,
  * 64}, n >= r_sk. The moment is accumulated in fp32 and its leading subspace found by orthogonal iteration with a
- * Rayleigh-Ritz step in fp64: directions whose eigenvalues are close are accurate as a subspace, not one by one. */
+ * Rayleigh-Ritz step in fp64: directions whose eigenvalues are close are accurate as a subspace, not one by one.
+ * Queries whose second moment has rank below r_sk (fewer than r_sk independent directions) leave the iteration's
+ * Cholesky factorisation with a pivot at the rounding level: the directions beyond the rank then come out as some
+ * orthonormal completion, or, where a pivot is not positive, the device status word of ws is set to
+ * VK_ERR_INVALID_ARG (read it with vk_poll_status) and basis is not valid. */
 int vk_sketch_basis(const void* queries, int32_t dtype, int64_t n, int32_t r_sk, float* basis, float* eig, void* ws,
                     size_t ws_bytes, void* stream);
 
